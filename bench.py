@@ -1,0 +1,352 @@
+"""Benchmark: ISM attention forward + backward on one packed batch of
+synthetic multi-turn dialogues (default: batch 2 x 8192 tokens, 32 query /
+8 KV heads, head_dim 128, bf16), reported as effective TFLOP/s counting only
+visible (unmasked) query-key pairs: 14 * D * N_vis per step (forward
+4 * D * N_vis, backward 10 * D * N_vis).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+For N > 1 launch one process per GPU with torch.distributed.run; every rank
+processes its own replica of the batch (weak scaling, no collective on the
+data path) and rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2408_00539_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "ISM attn fwd+bwd effective TFLOP/s and % of bf16 tensor peak at seq 8K, 1 GB300"
+L2_BYTES = 129 * 2 ** 20
+
+
+def n_visible(segs) -> int:
+    """Visible (row, key) pairs per head, from the segment lengths: a query
+    segment [s, e) contributes (e - s) * e pairs, an answer token j
+    contributes j + 1 (sequence-relative).  Counting only, no attention."""
+    total = 0
+    for b in range(segs.num_seqs):
+        _, _, se, st = segs.seq(b)
+        start = 0
+        for e, t in zip(se.tolist(), st.tolist()):
+            n = e - start
+            if t == wl.QUERY:
+                total += n * e
+            else:
+                total += (start + 1 + e) * n // 2
+            start = e
+    return total
+
+
+def read_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as fh:
+            d = json.load(fh)
+        return d, "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 200 ms."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (FileNotFoundError, OSError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[4:8]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup(args):
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(0)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------- oracle arm
+
+def oracle_sample(w, q, k, v, do, heads_per_sample: int):
+    """Bounded CPU sample: fwd+bwd of the oracle over the first sequence and
+    the first `heads_per_sample` query heads of one GQA group."""
+    from oracle import ism_oracle as orc
+    t0, L, se, st = w.segs.seq(0)
+    grp = w.num_heads_q // w.num_heads_kv
+    nh = min(heads_per_sample, grp)
+    sub = wl.pack([(se, st)])
+    qs = q[t0:t0 + L, :nh].contiguous()
+    dos = do[t0:t0 + L, :nh].contiguous()
+    ks = k[t0:t0 + L, :1].contiguous()
+    vs = v[t0:t0 + L, :1].contiguous()
+    n_vis = n_visible(sub) * nh
+    tic = time.perf_counter()
+    orc.attn_fwd(qs, ks, vs, sub, w.softmax_scale)
+    orc.attn_bwd(qs, ks, vs, dos, sub, w.softmax_scale)
+    dt = time.perf_counter() - tic
+    flops = 14 * w.head_dim * n_vis
+    return flops / dt / 1e12, dt, f"oracle fwd+bwd of sequence 0 ({L} tokens), {nh} query head(s) of KV head 0"
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+def run_reference(args, w):
+    world, rank, _ = dist_setup(args) if args.gpus > 1 else (1, 0, 0)
+    if rank != 0:
+        return
+    q, k, v, do = wl.attention_tensors(w)
+    vals, times = [], []
+    for i in range(args.warmup + args.steps):
+        val, dt, sample = oracle_sample(w, q, k, v, do, heads_per_sample=1)
+        if i >= args.warmup:
+            vals.append(val)
+            times.append(dt)
+    value = float(np.mean(vals))
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": float(np.mean(times)) * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------- CUDA arm
+
+def run_cuda(args, w):
+    import torch
+    from paper_2408_00539_gb300 import ism
+
+    world, rank, local = dist_setup(args)
+    dev = torch.device("cuda", local if world > 1 else 0)
+    ism.load()
+    peaks, peak_kind = read_peaks()
+
+    q, k, v, do = wl.attention_tensors(w)
+    segs = ism.Segments.from_workload(w.segs, dev)
+    qd, kd, vd, dod = (t.to(dev) for t in (q, k, v, do))
+    n_vis = n_visible(w.segs) * w.num_heads_q
+    D = w.head_dim
+    flops = 14 * D * n_vis
+    o, lse = ism.fwd(segs, qd, kd, vd, w.softmax_scale)
+    dq, dk, dv = ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale)
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+
+    def step():
+        ism.fwd(segs, qd, kd, vd, w.softmax_scale, out=o, lse=lse)
+        ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, dq=dq, dk=dk, dv=dv)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    ism.check_status(dev)
+
+    # per-kernel timers for the roofline (on the library's launch stream)
+    stream = torch.cuda.current_stream(dev)
+    kinds = {"fwd": ism.KERNEL_FWD, "bwd_dkdv": ism.KERNEL_BWD_DKDV, "bwd_dq": ism.KERNEL_BWD_DQ,
+             "bwd_pre": ism.KERNEL_BWD_PRE, "meta": ism.KERNEL_META}
+    ktimes = {n: [] for n in kinds}
+    step_ms = []
+    launches0 = ism.kernel_launches()
+    with ClockSampler(dev.index) as clocks:
+        barrier(world)
+        torch.cuda.synchronize()
+        for _ in range(args.steps):
+            flush.fill_(1)  # evict L2 between timed steps (outside the step's events)
+            ev = {n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for n in kinds}
+            for n, kid in kinds.items():
+                ism.set_kernel_timer(kid, *ev[n])
+            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            s0.record(stream)
+            step()
+            s1.record(stream)
+            s1.synchronize()
+            step_ms.append(s0.elapsed_time(s1))
+            for n in kinds:
+                ktimes[n].append(ev[n][0].elapsed_time(ev[n][1]))
+        torch.cuda.synchronize()
+        barrier(world)
+    for kid in kinds.values():
+        ism.set_kernel_timer(kid)
+    launches = ism.kernel_launches() - launches0
+    ism.check_status(dev)
+
+    total_ms = max_over_ranks(float(np.sum(step_ms)), world)
+    ms_per_step = total_ms / args.steps
+    value = flops * world * args.steps / (total_ms * 1e-3) / 1e12
+
+    # dominant kernel: largest share of the step
+    mean_k = {n: float(np.mean(t)) for n, t in ktimes.items()}
+    kflops = {"fwd": 4 * D * n_vis, "bwd_dkdv": 8 * D * n_vis, "bwd_dq": 6 * D * n_vis}
+    dom = max(kflops, key=lambda n: mean_k[n])
+    peak = peaks.get("bf16_tflops_sustained" if args.steps * ms_per_step > 2000 else "bf16_tflops")
+    achieved = kflops[dom] / (mean_k[dom] * 1e-3) / 1e12
+    roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
+                "flops_per_launch": kflops[dom], "ms_per_launch": mean_k[dom]}
+
+    # end to end through the public API with host buffers
+    pin = lambda t: t.pin_memory()  # noqa: E731
+    qh, kh, vh, doh = pin(q), pin(k), pin(v), pin(do)
+    dqh, dkh, dvh = (torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in (q, k, v))
+    h2d = sum(t.numel() * t.element_size() for t in (qh, kh, vh, doh))
+    d2h = sum(t.numel() * t.element_size() for t in (dqh, dkh, dvh))
+
+    def e2e_step():
+        qd.copy_(qh, non_blocking=True)
+        kd.copy_(kh, non_blocking=True)
+        vd.copy_(vh, non_blocking=True)
+        dod.copy_(doh, non_blocking=True)
+        step()
+        dqh.copy_(dq, non_blocking=True)
+        dkh.copy_(dk, non_blocking=True)
+        dvh.copy_(dv, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    e2e_ms = []
+    for _ in range(args.steps):
+        flush.fill_(1)
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        e2e_step()
+        a1.record(stream)
+        a1.synchronize()
+        e2e_ms.append(a0.elapsed_time(a1))
+    e2e_total = max_over_ranks(float(np.sum(e2e_ms)), world)
+    e2e_value = flops * world * args.steps / (e2e_total * 1e-3) / 1e12
+
+    if rank != 0:
+        return
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": w.name, "tokens": w.total_tokens, "n_vis_pairs": n_vis,
+                   "flops_per_step": flops, "flop_count": "14*D*N_vis (fwd 4, bwd 10)",
+                   "strict_tflops_12D": value * 12 / 14, "l2": "flushed between timed steps (258 MB write)",
+                   "pct_of_peak": value / peak * 100, "path": "tensor cores" if ism.has_tensor_cores()
+                   else "cuda cores", "parallelism": f"replicas x{world}"},
+        "kernel_ms": mean_k,
+        "roofline": roofline,
+        "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": e2e_total / args.steps},
+        "gpu_launches": int(launches),
+        "clocks": clocks.summary(),
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        val, dt, sample = oracle_sample(w, q, k, v, do, heads_per_sample=4)
+        line["cpu_baseline"] = {"value": val, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
+                                "sample": sample, "seconds": dt}
+    print(json.dumps(line), flush=True)
+
+
+WORKLOADS = {"gqa_8k": wl.gqa_8k, "mha_4k": wl.mha_4k, "packed_32k": wl.packed_32k}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="cuda", choices=["cuda", "reference"])
+    ap.add_argument("--workload", default="gqa_8k", choices=sorted(WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    w = WORKLOADS[args.workload]()
+    if args.impl == "reference":
+        run_reference(args, w)
+    else:
+        run_cuda(args, w)
+
+
+if __name__ == "__main__":
+    main()

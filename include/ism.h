@@ -1,0 +1,226 @@
+/*
+ * ism.h -- C ABI of libism: softmax attention under the Intermittent
+ * Semi-working Mask (ISM, arXiv 2408.00539) on NVIDIA GB300 (sm_103a).
+ *
+ * The mask (Section 2.1, Eq. e_ISM with the bound f(j) of Eq. fj): a
+ * dialogue [P, Q1, A1, ..., Q_{n-1}, A_{n-1}, Q_n] is cut into segments.
+ * A token of a query segment (the prompt P belongs to the first one) sees
+ * every key up to the end of its own query segment; a token of an answer
+ * segment sees keys up to and including itself; no token sees past the end
+ * of its own segment.  In 0-based indices row j of a sequence sees keys
+ * [0, kv_end[j]) with kv_end[j] = f(j+1).
+ *
+ * Conventions shared by every entry point
+ *  - Pointers without a `_host` suffix are DEVICE pointers; `_host` ones are
+ *    host mirrors of the same data, used for validation and sizing without a
+ *    device synchronisation.  Both must hold identical values.
+ *  - Tensors are dense, row-major and 16-byte aligned.  Q and O are
+ *    [tokens, Hq, D]; K and V are [tokens, Hkv, D]; LSE is [Hq, tokens] fp32
+ *    (natural log of the sum of exp(scale * q.k) over visible keys).
+ *  - Grouped-query attention: query head h uses KV head h / (Hq / Hkv).
+ *  - The caller owns and allocates every buffer, workspaces included.  The
+ *    library allocates no device memory and keeps no state between calls
+ *    except one device status word per device (see ism_check_status).
+ *  - Every call is asynchronous on `stream` (a cudaStream_t; NULL is the
+ *    legacy default stream).  Only ism_check_status synchronises.
+ *  - Arguments are validated on the host before anything is launched; on an
+ *    error nothing is launched, outputs are untouched, and ism_last_error()
+ *    describes the problem.
+ */
+#ifndef ISM_H_
+#define ISM_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* ism_stream_t; /* identical to cudaStream_t */
+
+typedef enum {
+  ISM_OK = 0,
+  ISM_ERR_INVALID_ARG = 1,  /* null/misaligned pointer, malformed segments, size overflow */
+  ISM_ERR_UNSUPPORTED = 2,  /* valid but not implemented (head_dim, dtype, tile size) */
+  ISM_ERR_CUDA = 3,         /* a CUDA runtime call or kernel launch failed */
+  ISM_ERR_TIMEOUT = 4,      /* a bounded device-side wait gave up (reported by ism_check_status) */
+  ISM_ERR_WORKSPACE = 5     /* workspace pointer null/misaligned or smaller than required */
+} ism_status_t;
+
+typedef enum { ISM_BF16 = 0, ISM_FP32 = 1 } ism_dtype_t;
+
+enum { ISM_SEG_QUERY = 0, ISM_SEG_ANSWER = 1 };
+enum { ISM_TILE_EMPTY = 0, ISM_TILE_FULL = 1, ISM_TILE_PARTIAL = 2 };
+
+/* Turn boundaries of a varlen batch (Section 2.1: the cumulative ends
+ * m_p, m_{q_k}, m_{a_k} of the dialogue's prompt, queries and answers).
+ *   cu_seqlens [num_seqs+1]  token offset of each packed sequence; cu_seqlens[0] = 0,
+ *                            non-decreasing.  Sequences never attend to each other.
+ *   cu_segs    [num_seqs+1]  segment offset of each sequence; cu_segs[0] = 0,
+ *                            cu_segs[num_seqs] = num_segs.
+ *   seg_end    [num_segs]    exclusive end of each segment relative to its
+ *                            sequence, non-decreasing within the sequence; the
+ *                            last one equals the sequence length.  Zero-length
+ *                            segments are allowed.
+ *   seg_type   [num_segs]    ISM_SEG_QUERY or ISM_SEG_ANSWER.  Consecutive query
+ *                            segments are separate bidirectional blocks.
+ * A sequence of length 0 has no segments or only zero-length ones. */
+typedef struct {
+  int32_t num_seqs;
+  int32_t num_segs;
+  const int32_t* cu_seqlens;
+  const int32_t* cu_seqlens_host;
+  const int32_t* cu_segs;
+  const int32_t* cu_segs_host;
+  const int32_t* seg_end;
+  const int32_t* seg_end_host;
+  const uint8_t* seg_type;
+  const uint8_t* seg_type_host;
+} ism_segments_t;
+
+/* Heads and element type.  Supported: head_dim 64 or 128; Hq % Hkv == 0;
+ * ISM_BF16 (fp32 accumulation, tensor cores) or ISM_FP32 (fp32 CUDA-core
+ * path).  softmax_scale multiplies q.k before the softmax (the paper omits
+ * the factor, Section 2.1; 1/sqrt(head_dim) is the usual choice). */
+typedef struct {
+  int32_t num_heads_q;
+  int32_t num_heads_kv;
+  int32_t head_dim;
+  int32_t dtype; /* ism_dtype_t */
+  float softmax_scale;
+} ism_attn_shape_t;
+
+/* ---------------------------------------------------------------------------
+ * Tile map.  Classifies each (q-tile, k-tile) rectangle of each sequence:
+ * rows [t*bm, t*bm+bm) and keys [c*bn, c*bn+bn) relative to the sequence.
+ * FULL: inside the sequence and every pair visible (run without a mask);
+ * EMPTY: no in-bounds pair visible (skipped); PARTIAL otherwise.  Because
+ * kv_end is non-decreasing (Eq. fj), each q-tile row of the map reads
+ * FULL* PARTIAL* EMPTY*.  No counterpart in the paper: it is a classification
+ * of the Eq. (fj) mask.
+ * ------------------------------------------------------------------------- */
+
+/* Sizes of the tile-map arrays: n_tiles = sum_b nqt_b*nkt_b, n_qtiles =
+ * sum_b ceil(L_b/bm), n_ktiles = sum_b ceil(L_b/bn).  bm, bn in {16,...,256}
+ * multiples of 16.  Host-only; reads the _host mirrors. */
+ism_status_t ism_tile_map_size(const ism_segments_t* segs, int32_t bm, int32_t bn,
+                               int64_t* n_tiles, int64_t* n_qtiles, int64_t* n_ktiles);
+
+/* Builds the tile map on the device (kernels on `stream`).  Outputs (device,
+ * any may be NULL to skip):
+ *   tile_class  [n_tiles]  uint8, per sequence a row-major [nqt_b, nkt_b] block
+ *   kt_full_end [n_qtiles] number of leading FULL k-tiles of each q-tile
+ *   kt_end      [n_qtiles] one past the last non-EMPTY k-tile
+ *   qt_begin    [n_ktiles] first non-EMPTY q-tile of each k-tile column
+ *   kv_end      [total_tokens] per-token exclusive key bound, sequence-relative
+ * Cited: Eq. (fj), Section 2.1. */
+ism_status_t ism_build_tile_map(const ism_segments_t* segs, int32_t bm, int32_t bn,
+                                uint8_t* tile_class, int32_t* kt_full_end, int32_t* kt_end,
+                                int32_t* qt_begin, int32_t* kv_end, ism_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * Forward over whole packed dialogues in one pass (Eq. e_ISM with softmax;
+ * Section 2.3 applies ISM by replacing the causal mask of a softmax LLM).
+ *   q [T, Hq, D], k/v [T, Hkv, D] (dtype), o [T, Hq, D] (dtype, written),
+ *   lse [Hq, T] fp32 (written; may be NULL only if no backward follows).
+ *   workspace: device scratch of at least ism_attn_fwd_workspace_size bytes,
+ *   256-byte aligned; its contents on entry do not matter.
+ * ------------------------------------------------------------------------- */
+ism_status_t ism_attn_fwd_workspace_size(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                                         size_t* bytes);
+ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                          const void* q, const void* k, const void* v, void* o, float* lse,
+                          void* workspace, size_t workspace_bytes, ism_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * Backward: gradients of sum(O * dO) with respect to Q, K, V, given the
+ * forward's O and LSE.  dq [T, Hq, D], dk/dv [T, Hkv, D] (dtype, written;
+ * dk/dv summed over the query heads that share a KV head).  Standard
+ * softmax-attention calculus over the Eq. (e_ISM) mask.
+ * ------------------------------------------------------------------------- */
+ism_status_t ism_attn_bwd_workspace_size(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                                         size_t* bytes);
+ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                          const void* q, const void* k, const void* v, const void* o,
+                          const float* lse, const void* dout,
+                          void* dq, void* dk, void* dv,
+                          void* workspace, size_t workspace_bytes, ism_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * Append-prefill of a new turn against a reused KV cache (Section 2.3: the
+ * history's keys/values C_h are reused, the new chunk's C_q are computed and
+ * [C_h; C_q] concatenated).  Valid because no token sees past the end of its
+ * own segment (prose after Eq. fj).  One call:
+ *   1. writes k_new/v_new into k_cache/v_cache at rows [cache_len[b], cache_len[b]+l_new);
+ *   2. computes, for every new token j of sequence b, attention over cache
+ *      keys [0, cache_len[b] + kv_end_new[j]) where kv_end_new is Eq. (fj)
+ *      applied to the chunk's own segments (all cached keys are visible);
+ *   3. advances the device cache_len[b] by l_new (the caller advances its
+ *      host mirror).
+ * A decode step is l_new = 1 with one ANSWER segment.
+ *   q_new [B, l_new, Hq, D], k_new/v_new [B, l_new, Hkv, D] (dtype)
+ *   new_seg_end_host/new_seg_type_host [n_new_segs]: chunk-relative segments,
+ *     the same for every sequence, last end == l_new, n_new_segs <= 256
+ *   k_cache/v_cache [B, cache_capacity, Hkv, D] (dtype, in/out)
+ *   cache_len [B] int32 device (in/out), cache_len_host [B] its host mirror;
+ *     cache_len_host[b] + l_new <= cache_capacity is required.
+ *   o_new [B, l_new, Hq, D] (dtype, written); lse_new [Hq, B, l_new] fp32 or NULL.
+ * If a cache ends inside a query segment its old rows would differ from a
+ * full pass once the segment grows; the new rows are still exact.
+ * ------------------------------------------------------------------------- */
+ism_status_t ism_attn_prefill_append_workspace_size(const ism_attn_shape_t* shape, int32_t batch,
+                                                    int32_t l_new, size_t* bytes);
+ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batch,
+                                     const void* q_new, const void* k_new, const void* v_new,
+                                     int32_t l_new, const int32_t* new_seg_end_host,
+                                     const uint8_t* new_seg_type_host, int32_t n_new_segs,
+                                     void* k_cache, void* v_cache, int64_t cache_capacity,
+                                     int32_t* cache_len, const int32_t* cache_len_host,
+                                     void* o_new, float* lse_new,
+                                     void* workspace, size_t workspace_bytes, ism_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * Status and diagnostics.
+ * ------------------------------------------------------------------------- */
+
+/* Synchronises `stream`, then reads and clears the current device's status
+ * word.  Returns ISM_ERR_TIMEOUT if any kernel gave up a bounded wait since
+ * the last check (the kernel exits early and its outputs are undefined),
+ * ISM_ERR_CUDA on a CUDA error, ISM_OK otherwise. */
+ism_status_t ism_check_status(ism_stream_t stream);
+
+/* Test hook for the bounded-wait machinery: launches one kernel that waits on
+ * a barrier nothing ever signals, with a spin limit of `spin_limit` polls,
+ * gives up, records ISM_ERR_TIMEOUT in the status word and returns.  Lets a
+ * test observe the timeout path without hanging a GPU. */
+ism_status_t ism_debug_timeout_probe(uint32_t spin_limit, ism_stream_t stream);
+
+/* Measurement hooks (no counterpart in the paper).
+ * ism_set_kernel_timer: while set, every launch of kernel kind `kernel_id`
+ * issued by this host thread is bracketed by cudaEventRecord(start_event)
+ * and cudaEventRecord(stop_event) on the launch's stream (the events are
+ * cudaEvent_t handles owned by the caller; NULL clears the timer).
+ * ism_kernel_launches: number of kernels this library has launched in the
+ * process so far (all threads). */
+enum {
+  ISM_KERNEL_FWD = 1,        /* one-pass forward (and append-prefill over a chunk) */
+  ISM_KERNEL_BWD_DKDV = 2,   /* backward dK/dV */
+  ISM_KERNEL_BWD_DQ = 3,     /* backward dQ */
+  ISM_KERNEL_BWD_PRE = 4,    /* backward preprocessing (Delta) */
+  ISM_KERNEL_DECODE = 5,     /* single-token append (split-KV + merge) */
+  ISM_KERNEL_META = 6        /* tile map / work lists */
+};
+ism_status_t ism_set_kernel_timer(int32_t kernel_id, void* start_event, void* stop_event);
+uint64_t ism_kernel_launches(void);
+
+const char* ism_status_string(ism_status_t status);
+/* Human-readable detail of the last failing call on this host thread. */
+const char* ism_last_error(void);
+/* 1 if the library was built with the sm_103a tensor-core kernels. */
+int32_t ism_has_tensor_cores(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ISM_H_ */

@@ -1,0 +1,565 @@
+// Host side of the C ABI: argument validation on the host mirrors, workspace
+// layout, kernel dispatch and the device status word.
+#include <cstdarg>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <atomic>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "ism_internal.cuh"
+
+namespace ism {
+namespace {
+
+thread_local std::string g_last_error;
+
+ism_status_t fail(ism_status_t st, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return st;
+}
+
+ism_status_t cuda_fail(cudaError_t e, const char* where) {
+  return fail(ISM_ERR_CUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+#define ISM_TRY_CUDA(expr, where)                 \
+  do {                                            \
+    cudaError_t e_ = (expr);                      \
+    if (e_ != cudaSuccess) return cuda_fail(e_, where); \
+  } while (0)
+
+// One status word per device; the library's only persistent device state.
+__device__ uint32_t g_status_word;
+
+std::mutex g_status_mu;
+std::vector<uint32_t*> g_status_ptr;
+
+ism_status_t status_ptr(uint32_t** out) {
+  int dev = 0;
+  ISM_TRY_CUDA(cudaGetDevice(&dev), "cudaGetDevice");
+  std::lock_guard<std::mutex> lk(g_status_mu);
+  if ((int)g_status_ptr.size() <= dev) g_status_ptr.resize(dev + 1, nullptr);
+  if (!g_status_ptr[dev]) {
+    void* p = nullptr;
+    ISM_TRY_CUDA(cudaGetSymbolAddress(&p, g_status_word), "cudaGetSymbolAddress(status)");
+    g_status_ptr[dev] = static_cast<uint32_t*>(p);
+  }
+  *out = g_status_ptr[dev];
+  return ISM_OK;
+}
+
+// ---------------------------------------------------------------- measurement
+
+constexpr int kTimerSlots = 8;
+thread_local cudaEvent_t g_timer_start[kTimerSlots];
+thread_local cudaEvent_t g_timer_stop[kTimerSlots];
+std::atomic<uint64_t> g_launches{0};
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+constexpr int kTile = 128;       // q/k tile rows of the attention kernels and their work lists
+constexpr int kMaxSplits = 64;   // split-KV chunks per (sequence, KV head) for decode
+
+struct SegInfo {
+  int64_t total_tokens = 0;
+  int64_t max_len = 0;
+};
+
+ism_status_t check_segments(const ism_segments_t* s, SegInfo* info) {
+  if (!s) return fail(ISM_ERR_INVALID_ARG, "segments is NULL");
+  if (s->num_seqs < 0 || s->num_segs < 0) return fail(ISM_ERR_INVALID_ARG, "negative counts");
+  if (s->num_seqs > kMaxSeqs) return fail(ISM_ERR_UNSUPPORTED, "num_seqs %d > %d", s->num_seqs, kMaxSeqs);
+  if (!s->cu_seqlens_host || !s->cu_segs_host || !s->cu_seqlens || !s->cu_segs)
+    return fail(ISM_ERR_INVALID_ARG, "cu_seqlens / cu_segs (device and host) must be non-NULL");
+  if (s->num_segs > 0 && (!s->seg_end || !s->seg_end_host || !s->seg_type || !s->seg_type_host))
+    return fail(ISM_ERR_INVALID_ARG, "seg_end / seg_type (device and host) must be non-NULL");
+  const int32_t* cs = s->cu_seqlens_host;
+  const int32_t* cg = s->cu_segs_host;
+  if (cs[0] != 0 || cg[0] != 0) return fail(ISM_ERR_INVALID_ARG, "cu_seqlens[0] and cu_segs[0] must be 0");
+  if (cg[s->num_seqs] != s->num_segs)
+    return fail(ISM_ERR_INVALID_ARG, "cu_segs[num_seqs]=%d != num_segs=%d", cg[s->num_seqs], s->num_segs);
+  int64_t max_len = 0;
+  for (int b = 0; b < s->num_seqs; ++b) {
+    int64_t L = (int64_t)cs[b + 1] - cs[b];
+    if (L < 0) return fail(ISM_ERR_INVALID_ARG, "cu_seqlens decreases at sequence %d", b);
+    if (cg[b + 1] < cg[b]) return fail(ISM_ERR_INVALID_ARG, "cu_segs decreases at sequence %d", b);
+    int32_t prev = 0;
+    for (int i = cg[b]; i < cg[b + 1]; ++i) {
+      int32_t e = s->seg_end_host[i];
+      if (e < prev) return fail(ISM_ERR_INVALID_ARG, "seq %d: seg_end not non-decreasing at segment %d", b, i);
+      if (s->seg_type_host[i] > 1) return fail(ISM_ERR_INVALID_ARG, "segment %d: type %d is not QUERY/ANSWER", i,
+                                               (int)s->seg_type_host[i]);
+      prev = e;
+    }
+    if (prev != L)
+      return fail(ISM_ERR_INVALID_ARG, "seq %d: segments end at %d but the sequence has %lld tokens", b, prev,
+                  (long long)L);
+    if (L > max_len) max_len = L;
+  }
+  info->total_tokens = cs[s->num_seqs];
+  info->max_len = max_len;
+  return ISM_OK;
+}
+
+ism_status_t check_shape(const ism_attn_shape_t* sh) {
+  if (!sh) return fail(ISM_ERR_INVALID_ARG, "shape is NULL");
+  if (sh->num_heads_q <= 0 || sh->num_heads_kv <= 0) return fail(ISM_ERR_INVALID_ARG, "head counts must be > 0");
+  if (sh->num_heads_q % sh->num_heads_kv)
+    return fail(ISM_ERR_INVALID_ARG, "num_heads_q (%d) is not a multiple of num_heads_kv (%d)", sh->num_heads_q,
+                sh->num_heads_kv);
+  if (sh->head_dim != 64 && sh->head_dim != 128)
+    return fail(ISM_ERR_UNSUPPORTED, "head_dim %d (supported: 64, 128)", sh->head_dim);
+  if (sh->dtype != ISM_BF16 && sh->dtype != ISM_FP32) return fail(ISM_ERR_UNSUPPORTED, "dtype %d", sh->dtype);
+  if (!(sh->softmax_scale > 0.f) || sh->softmax_scale != sh->softmax_scale)
+    return fail(ISM_ERR_INVALID_ARG, "softmax_scale must be a positive number");
+  return ISM_OK;
+}
+
+SegsDev dev_view(const ism_segments_t* s) {
+  SegsDev d;
+  d.num_seqs = s->num_seqs;
+  d.num_segs = s->num_segs;
+  d.cu_seqlens = s->cu_seqlens;
+  d.cu_segs = s->cu_segs;
+  d.seg_end = s->seg_end;
+  d.seg_type = s->seg_type;
+  return d;
+}
+
+// Bump allocator over a caller-provided workspace (256-byte aligned pieces).
+struct Carve {
+  uintptr_t base;
+  size_t off = 0;
+  explicit Carve(void* p) : base(reinterpret_cast<uintptr_t>(p)) {}
+  template <typename T>
+  T* take(int64_t n) {
+    off = (off + 255) & ~size_t(255);
+    T* p = reinterpret_cast<T*>(base + off);
+    off += sizeof(T) * (size_t)(n > 0 ? n : 0);
+    return p;
+  }
+};
+
+struct Counts {
+  int64_t nq = 0, nk = 0, ntiles = 0;
+  int max_cost = 0;
+};
+
+Counts count_tiles(const ism_segments_t* s, int bm, int bn) {
+  Counts c;
+  for (int b = 0; b < s->num_seqs; ++b) {
+    int64_t L = (int64_t)s->cu_seqlens_host[b + 1] - s->cu_seqlens_host[b];
+    int64_t nq = (L + bm - 1) / bm, nk = (L + bn - 1) / bn;
+    c.nq += nq;
+    c.nk += nk;
+    c.ntiles += nq * nk;
+    int mc = (int)(nq > nk ? nq : nk);
+    if (mc > c.max_cost) c.max_cost = mc;
+  }
+  return c;
+}
+
+// Workspace of the one-pass forward/backward.
+struct PassLayout {
+  int32_t* kv_end;
+  Tile *qtiles, *ktiles;
+  int32_t *q_order, *k_order;
+  float* delta;
+  size_t bytes;
+};
+
+PassLayout pass_layout(void* ws, const ism_segments_t* s, const Counts& c, int64_t T, int hq, bool bwd) {
+  Carve cv(ws);
+  PassLayout L;
+  L.kv_end = cv.take<int32_t>(T);
+  L.qtiles = cv.take<Tile>(c.nq);
+  L.q_order = cv.take<int32_t>(c.nq);
+  L.ktiles = bwd ? cv.take<Tile>(c.nk) : nullptr;
+  L.k_order = bwd ? cv.take<int32_t>(c.nk) : nullptr;
+  L.delta = bwd ? cv.take<float>((int64_t)hq * T) : nullptr;
+  L.bytes = ((cv.off + 255) & ~size_t(255)) + 256;
+  return L;
+}
+
+bool force_cuda_cores() {
+  const char* e = getenv("ISM_FORCE_CUDA_CORES");
+  return e && e[0] == '1';
+}
+
+bool use_tc(const ism_attn_shape_t* sh) {
+  return sh->dtype == ISM_BF16 && sh->head_dim == 128 && tc_available() && !force_cuda_cores();
+}
+
+ism_status_t check_ws(void* ws, size_t have, size_t need) {
+  if (have < need) return fail(ISM_ERR_WORKSPACE, "workspace of %zu bytes, %zu required", have, need);
+  if (need && !ws) return fail(ISM_ERR_WORKSPACE, "workspace is NULL");
+  if (reinterpret_cast<uintptr_t>(ws) & 255u) return fail(ISM_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+  return ISM_OK;
+}
+
+ism_status_t build_pass_meta(const ism_segments_t* s, const Counts& c, const PassLayout& L, bool bwd,
+                             cudaStream_t st) {
+  SegsDev d = dev_view(s);
+  timer_begin(ISM_KERNEL_META, st);
+  ISM_TRY_CUDA(launch_kv_end(d, L.kv_end, st), "kv_end launch");
+  ISM_TRY_CUDA(launch_tiles(d, kTile, kTile, L.kv_end, c.nq, bwd ? c.nk : 0, L.qtiles, L.ktiles, nullptr, nullptr,
+                            nullptr, nullptr, st),
+               "tiles launch");
+  ISM_TRY_CUDA(launch_order(L.qtiles, c.nq, L.ktiles, bwd ? c.nk : 0, c.max_cost, L.q_order, L.k_order, st),
+               "order launch");
+  timer_end(ISM_KERNEL_META, st);
+  count_launch(s->num_segs > 0 ? 3 : 2);
+  return ISM_OK;
+}
+
+}  // namespace
+
+void timer_begin(int id, cudaStream_t st) {
+  if (id > 0 && id < kTimerSlots && g_timer_start[id]) cudaEventRecord(g_timer_start[id], st);
+}
+void timer_end(int id, cudaStream_t st) {
+  if (id > 0 && id < kTimerSlots && g_timer_stop[id]) cudaEventRecord(g_timer_stop[id], st);
+}
+void count_launch(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+
+}  // namespace ism
+
+using namespace ism;
+
+extern "C" {
+
+const char* ism_status_string(ism_status_t s) {
+  switch (s) {
+    case ISM_OK: return "ISM_OK";
+    case ISM_ERR_INVALID_ARG: return "ISM_ERR_INVALID_ARG";
+    case ISM_ERR_UNSUPPORTED: return "ISM_ERR_UNSUPPORTED";
+    case ISM_ERR_CUDA: return "ISM_ERR_CUDA";
+    case ISM_ERR_TIMEOUT: return "ISM_ERR_TIMEOUT";
+    case ISM_ERR_WORKSPACE: return "ISM_ERR_WORKSPACE";
+  }
+  return "ISM_ERR_UNKNOWN";
+}
+
+const char* ism_last_error(void) { return g_last_error.c_str(); }
+
+int32_t ism_has_tensor_cores(void) { return tc_available() ? 1 : 0; }
+
+ism_status_t ism_set_kernel_timer(int32_t kernel_id, void* start_event, void* stop_event) {
+  if (kernel_id <= 0 || kernel_id >= kTimerSlots) return fail(ISM_ERR_INVALID_ARG, "kernel_id %d", kernel_id);
+  if ((start_event == nullptr) != (stop_event == nullptr))
+    return fail(ISM_ERR_INVALID_ARG, "give both events or neither");
+  g_timer_start[kernel_id] = static_cast<cudaEvent_t>(start_event);
+  g_timer_stop[kernel_id] = static_cast<cudaEvent_t>(stop_event);
+  return ISM_OK;
+}
+
+uint64_t ism_kernel_launches(void) { return g_launches.load(); }
+
+ism_status_t ism_tile_map_size(const ism_segments_t* segs, int32_t bm, int32_t bn, int64_t* n_tiles,
+                               int64_t* n_qtiles, int64_t* n_ktiles) {
+  SegInfo info;
+  ism_status_t r = check_segments(segs, &info);
+  if (r != ISM_OK) return r;
+  if (bm < 16 || bn < 16 || bm > 256 || bn > 256 || bm % 16 || bn % 16)
+    return fail(ISM_ERR_UNSUPPORTED, "tile sizes must be multiples of 16 in [16, 256]");
+  Counts c = count_tiles(segs, bm, bn);
+  if (n_tiles) *n_tiles = c.ntiles;
+  if (n_qtiles) *n_qtiles = c.nq;
+  if (n_ktiles) *n_ktiles = c.nk;
+  return ISM_OK;
+}
+
+ism_status_t ism_build_tile_map(const ism_segments_t* segs, int32_t bm, int32_t bn, uint8_t* tile_class,
+                                int32_t* kt_full_end, int32_t* kt_end, int32_t* qt_begin, int32_t* kv_end,
+                                ism_stream_t stream) {
+  int64_t nt, nq, nk;
+  ism_status_t r = ism_tile_map_size(segs, bm, bn, &nt, &nq, &nk);
+  if (r != ISM_OK) return r;
+  if (segs->cu_seqlens_host[segs->num_seqs] == 0) return ISM_OK;
+  if (!kv_end) return fail(ISM_ERR_INVALID_ARG, "kv_end output is required (the tile classes are derived from it)");
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  SegsDev d = dev_view(segs);
+  ISM_TRY_CUDA(launch_kv_end(d, kv_end, st), "kv_end launch");
+  if (tile_class || kt_full_end || kt_end || qt_begin)
+    ISM_TRY_CUDA(launch_tiles(d, bm, bn, kv_end, nq, qt_begin ? nk : 0, nullptr, nullptr, tile_class, kt_full_end,
+                              kt_end, qt_begin, st),
+                 "tiles launch");
+  return ISM_OK;
+}
+
+ism_status_t ism_attn_fwd_workspace_size(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                                         size_t* bytes) {
+  SegInfo info;
+  ism_status_t r = check_segments(segs, &info);
+  if (r != ISM_OK) return r;
+  if ((r = check_shape(shape)) != ISM_OK) return r;
+  if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
+  Counts c = count_tiles(segs, kTile, kTile);
+  *bytes = pass_layout(nullptr, segs, c, info.total_tokens, shape->num_heads_q, false).bytes;
+  return ISM_OK;
+}
+
+ism_status_t ism_attn_bwd_workspace_size(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                                         size_t* bytes) {
+  SegInfo info;
+  ism_status_t r = check_segments(segs, &info);
+  if (r != ISM_OK) return r;
+  if ((r = check_shape(shape)) != ISM_OK) return r;
+  if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
+  Counts c = count_tiles(segs, kTile, kTile);
+  *bytes = pass_layout(nullptr, segs, c, info.total_tokens, shape->num_heads_q, true).bytes;
+  return ISM_OK;
+}
+
+ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q,
+                          const void* k, const void* v, void* o, float* lse, void* workspace,
+                          size_t workspace_bytes, ism_stream_t stream) {
+  SegInfo info;
+  ism_status_t r = check_segments(segs, &info);
+  if (r != ISM_OK) return r;
+  if ((r = check_shape(shape)) != ISM_OK) return r;
+  if (info.total_tokens == 0) return ISM_OK;
+  if (!q || !k || !v || !o) return fail(ISM_ERR_INVALID_ARG, "q, k, v, o must be non-NULL");
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || (lse && !aligned16(lse)))
+    return fail(ISM_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  Counts c = count_tiles(segs, kTile, kTile);
+  PassLayout L = pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, false);
+  if ((r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
+  uint32_t* status;
+  if ((r = status_ptr(&status)) != ISM_OK) return r;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if ((r = build_pass_meta(segs, c, L, false, st)) != ISM_OK) return r;
+
+  AttnArgs a{};
+  a.q = q; a.k = k; a.v = v; a.out = o; a.lse = lse;
+  a.hq = shape->num_heads_q; a.hkv = shape->num_heads_kv; a.d = shape->head_dim; a.dtype = shape->dtype;
+  a.q_rows = info.total_tokens; a.scale = shape->softmax_scale;
+  a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order; a.nq = c.nq;
+  a.status = status;
+  timer_begin(ISM_KERNEL_FWD, st);
+  if (use_tc(shape)) {
+    ISM_TRY_CUDA(launch_tc_fwd(a, info.total_tokens, st), "tensor-core forward launch");
+  } else {
+    ISM_TRY_CUDA(launch_simt_fwd(a, st), "forward launch");
+  }
+  timer_end(ISM_KERNEL_FWD, st);
+  count_launch(1);
+  return ISM_OK;
+}
+
+ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q,
+                          const void* k, const void* v, const void* o, const float* lse, const void* dout,
+                          void* dq, void* dk, void* dv, void* workspace, size_t workspace_bytes,
+                          ism_stream_t stream) {
+  SegInfo info;
+  ism_status_t r = check_segments(segs, &info);
+  if (r != ISM_OK) return r;
+  if ((r = check_shape(shape)) != ISM_OK) return r;
+  if (info.total_tokens == 0) return ISM_OK;
+  if (!q || !k || !v || !o || !lse || !dout || !dq || !dk || !dv)
+    return fail(ISM_ERR_INVALID_ARG, "q, k, v, o, lse, dout, dq, dk, dv must be non-NULL");
+  const void* ptrs[] = {q, k, v, o, lse, dout, dq, dk, dv};
+  for (const void* p : ptrs)
+    if (!aligned16(p)) return fail(ISM_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  Counts c = count_tiles(segs, kTile, kTile);
+  PassLayout L = pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, true);
+  if ((r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
+  uint32_t* status;
+  if ((r = status_ptr(&status)) != ISM_OK) return r;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if ((r = build_pass_meta(segs, c, L, true, st)) != ISM_OK) return r;
+
+  AttnArgs a{};
+  a.q = q; a.k = k; a.v = v; a.o = o; a.dout = dout; a.lse_in = lse;
+  a.dq = dq; a.dk = dk; a.dv = dv; a.delta = L.delta;
+  a.hq = shape->num_heads_q; a.hkv = shape->num_heads_kv; a.d = shape->head_dim; a.dtype = shape->dtype;
+  a.q_rows = info.total_tokens; a.scale = shape->softmax_scale;
+  a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order; a.nq = c.nq;
+  a.ktiles = L.ktiles; a.k_order = L.k_order; a.nk = c.nk;
+  a.status = status;
+  if (use_tc(shape)) {
+    ISM_TRY_CUDA(launch_tc_bwd(a, info.total_tokens, st), "tensor-core backward launch");
+  } else {
+    ISM_TRY_CUDA(launch_simt_bwd(a, st), "backward launch");
+  }
+  return ISM_OK;
+}
+
+// ---------------------------------------------------------------- append
+
+namespace {
+
+struct AppendLayout {
+  int32_t* c_snap;
+  int32_t* kv_end;
+  Tile* qtiles;
+  int32_t* q_order;
+  float* part_o;
+  float* part_ml;
+  size_t bytes;
+};
+
+AppendLayout append_layout(void* ws, const ism_attn_shape_t* sh, int batch, int l_new) {
+  Carve cv(ws);
+  AppendLayout L;
+  int64_t nqt = (int64_t)batch * ((l_new + kTile - 1) / kTile);
+  L.c_snap = cv.take<int32_t>(batch);
+  L.kv_end = cv.take<int32_t>((int64_t)batch * l_new);
+  L.qtiles = cv.take<Tile>(nqt);
+  L.q_order = cv.take<int32_t>(nqt);
+  if (l_new == 1) {
+    L.part_o = cv.take<float>((int64_t)batch * sh->num_heads_q * kMaxSplits * sh->head_dim);
+    L.part_ml = cv.take<float>((int64_t)batch * sh->num_heads_q * kMaxSplits * 2);
+  } else {
+    L.part_o = L.part_ml = nullptr;
+  }
+  L.bytes = ((cv.off + 255) & ~size_t(255)) + 256;
+  return L;
+}
+
+}  // namespace
+
+ism_status_t ism_attn_prefill_append_workspace_size(const ism_attn_shape_t* shape, int32_t batch, int32_t l_new,
+                                                    size_t* bytes) {
+  ism_status_t r = check_shape(shape);
+  if (r != ISM_OK) return r;
+  if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
+  if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
+  *bytes = append_layout(nullptr, shape, batch, l_new).bytes;
+  return ISM_OK;
+}
+
+ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,
+                                     const void* k_new, const void* v_new, int32_t l_new,
+                                     const int32_t* new_seg_end_host, const uint8_t* new_seg_type_host,
+                                     int32_t n_new_segs, void* k_cache, void* v_cache, int64_t cache_capacity,
+                                     int32_t* cache_len, const int32_t* cache_len_host, void* o_new,
+                                     float* lse_new, void* workspace, size_t workspace_bytes,
+                                     ism_stream_t stream) {
+  ism_status_t r = check_shape(shape);
+  if (r != ISM_OK) return r;
+  if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
+  if (batch == 0 || l_new == 0) return ISM_OK;
+  if (!q_new || !k_new || !v_new || !k_cache || !v_cache || !cache_len || !cache_len_host || !o_new)
+    return fail(ISM_ERR_INVALID_ARG, "q_new, k_new, v_new, caches, cache_len (device+host), o_new must be non-NULL");
+  const void* ptrs[] = {q_new, k_new, v_new, k_cache, v_cache, o_new};
+  for (const void* p : ptrs)
+    if (!aligned16(p)) return fail(ISM_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  if (lse_new && !aligned16(lse_new)) return fail(ISM_ERR_INVALID_ARG, "lse_new must be 16-byte aligned");
+  if (!new_seg_end_host || !new_seg_type_host || n_new_segs <= 0 || n_new_segs > kMaxAppendSegs)
+    return fail(ISM_ERR_INVALID_ARG, "chunk needs 1..%d segments", kMaxAppendSegs);
+  AppendSegs sg;
+  memset(&sg, 0, sizeof(sg));
+  sg.n = n_new_segs;
+  sg.l_new = l_new;
+  int32_t prev = 0;
+  for (int i = 0; i < n_new_segs; ++i) {
+    if (new_seg_end_host[i] < prev) return fail(ISM_ERR_INVALID_ARG, "chunk seg_end not non-decreasing");
+    if (new_seg_type_host[i] > 1) return fail(ISM_ERR_INVALID_ARG, "chunk segment type %d", (int)new_seg_type_host[i]);
+    sg.end[i] = prev = new_seg_end_host[i];
+    sg.type[i] = new_seg_type_host[i];
+  }
+  if (prev != l_new) return fail(ISM_ERR_INVALID_ARG, "chunk segments end at %d, l_new is %d", prev, l_new);
+  if (cache_capacity <= 0 || (int64_t)batch * cache_capacity >= (int64_t(1) << 31))
+    return fail(ISM_ERR_INVALID_ARG, "batch * cache_capacity must be in (0, 2^31)");
+  if ((int64_t)batch * l_new >= (int64_t(1) << 31)) return fail(ISM_ERR_INVALID_ARG, "batch * l_new too large");
+  int32_t max_c = 0;
+  for (int b = 0; b < batch; ++b) {
+    int32_t c = cache_len_host[b];
+    if (c < 0 || (int64_t)c + l_new > cache_capacity)
+      return fail(ISM_ERR_INVALID_ARG, "sequence %d: cache_len %d + l_new %d exceeds capacity %lld", b, c, l_new,
+                  (long long)cache_capacity);
+    if (c > max_c) max_c = c;
+  }
+  AppendLayout L = append_layout(workspace, shape, batch, l_new);
+  if ((r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
+  uint32_t* status;
+  if ((r = status_ptr(&status)) != ISM_OK) return r;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const int hq = shape->num_heads_q, hkv = shape->num_heads_kv, d = shape->head_dim;
+
+  timer_begin(ISM_KERNEL_META, st);
+  ISM_TRY_CUDA(launch_append_plan(sg, batch, cache_capacity, kTile, kTile, cache_len, L.c_snap, L.kv_end, L.qtiles,
+                                  L.q_order, st),
+               "append plan launch");
+  ISM_TRY_CUDA(launch_cache_write(shape->dtype, batch, l_new, hkv, d, cache_capacity, L.c_snap, k_new, v_new,
+                                  k_cache, v_cache, st),
+               "cache write launch");
+  timer_end(ISM_KERNEL_META, st);
+  count_launch(2);
+  if (l_new == 1 && shape->dtype == ISM_BF16 && !force_cuda_cores()) {
+    DecodeArgs a{};
+    a.q = q_new; a.k_cache = k_cache; a.v_cache = v_cache; a.out = o_new; a.lse = lse_new; a.c_snap = L.c_snap;
+    a.batch = batch; a.hq = hq; a.hkv = hkv; a.d = d; a.dtype = shape->dtype; a.cap = cache_capacity;
+    a.scale = shape->softmax_scale;
+    // enough chunks to give every SM a few CTAs, each chunk a multiple of 64 keys
+    int64_t kv_max = (int64_t)max_c + 1;
+    int64_t pairs = (int64_t)batch * hkv;
+    int64_t want = (4 * 152 + pairs - 1) / pairs;
+    int64_t splits = want < 1 ? 1 : want > kMaxSplits ? kMaxSplits : want;
+    int64_t chunk = (kv_max + splits - 1) / splits;
+    chunk = (chunk + 63) / 64 * 64;
+    splits = (kv_max + chunk - 1) / chunk;
+    a.splits = (int32_t)splits;
+    a.chunk = (int32_t)chunk;
+    a.part_o = L.part_o; a.part_ml = L.part_ml;
+    timer_begin(ISM_KERNEL_DECODE, st);
+    ISM_TRY_CUDA(launch_decode(a, st), "decode launch");
+    timer_end(ISM_KERNEL_DECODE, st);
+    count_launch(2);
+    return ISM_OK;
+  }
+  AttnArgs a{};
+  a.q = q_new; a.k = k_cache; a.v = v_cache; a.out = o_new; a.lse = lse_new;
+  a.hq = hq; a.hkv = hkv; a.d = d; a.dtype = shape->dtype;
+  a.q_rows = (int64_t)batch * l_new; a.scale = shape->softmax_scale;
+  a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order;
+  a.nq = (int64_t)batch * ((l_new + kTile - 1) / kTile);
+  a.status = status;
+  timer_begin(ISM_KERNEL_FWD, st);
+  if (use_tc(shape)) {
+    ISM_TRY_CUDA(launch_tc_fwd(a, (int64_t)batch * cache_capacity, st), "tensor-core prefill launch");
+  } else {
+    ISM_TRY_CUDA(launch_simt_fwd(a, st), "prefill launch");
+  }
+  timer_end(ISM_KERNEL_FWD, st);
+  count_launch(1);
+  return ISM_OK;
+}
+
+// ---------------------------------------------------------------- status
+
+ism_status_t ism_check_status(ism_stream_t stream) {
+  uint32_t* status;
+  ism_status_t r = status_ptr(&status);
+  if (r != ISM_OK) return r;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  ISM_TRY_CUDA(cudaStreamSynchronize(st), "cudaStreamSynchronize");
+  uint32_t word = 0;
+  ISM_TRY_CUDA(cudaMemcpy(&word, status, sizeof(word), cudaMemcpyDeviceToHost), "status read");
+  if (word) {
+    uint32_t zero = 0;
+    ISM_TRY_CUDA(cudaMemcpy(status, &zero, sizeof(zero), cudaMemcpyHostToDevice), "status clear");
+  }
+  if (word & kStatusTimeout) return fail(ISM_ERR_TIMEOUT, "a device-side wait gave up (status word 0x%x)", word);
+  return ISM_OK;
+}
+
+ism_status_t ism_debug_timeout_probe(uint32_t spin_limit, ism_stream_t stream) {
+  uint32_t* status;
+  ism_status_t r = status_ptr(&status);
+  if (r != ISM_OK) return r;
+  if (spin_limit == 0 || spin_limit > (1u << 20)) return fail(ISM_ERR_INVALID_ARG, "spin_limit must be in [1, 2^20]");
+  ISM_TRY_CUDA(launch_timeout_probe(spin_limit, status, reinterpret_cast<cudaStream_t>(stream)), "probe launch");
+  return ISM_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,126 @@
+// Internal declarations shared by the libism translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/ism.h"
+
+namespace ism {
+
+// One tile of work for the attention kernels.  A "sequence" here is one
+// query stream attending to one key stream: a packed dialogue for the
+// one-pass forward/backward, or (new chunk of sequence b, its KV cache) for
+// append-prefill.  Key positions (and kv_end values) are relative to k_base.
+struct Tile {
+  int32_t q_base;   // global Q/O/dO row of query row 0 of the sequence
+  int32_t k_base;   // global K/V row of key 0 of the sequence
+  int32_t q_len;    // query rows of the sequence
+  int32_t k_len;    // keys of the sequence
+  int32_t tile;     // q-tile index t (or k-tile index c) within the sequence
+  int32_t a0;       // q-tile: number of leading FULL k-tiles; k-tile: first non-empty q-tile
+  int32_t a1;       // q-tile: one past the last non-empty k-tile; k-tile: number of q-tiles
+  int32_t kv_base;  // index of the sequence's query row 0 in the kv_end array
+};
+static_assert(sizeof(Tile) == 32, "Tile layout");
+
+// Device view of the segment arrays (device pointers only).
+struct SegsDev {
+  int32_t num_seqs;
+  int32_t num_segs;
+  const int32_t* cu_seqlens;
+  const int32_t* cu_segs;
+  const int32_t* seg_end;
+  const uint8_t* seg_type;
+};
+
+// Chunk segments of an append, passed to kernels by value.
+constexpr int kMaxAppendSegs = 256;
+struct AppendSegs {
+  int32_t n;
+  int32_t l_new;
+  int32_t end[kMaxAppendSegs];
+  uint8_t type[kMaxAppendSegs];
+};
+
+// Meta arrays carved out of a workspace.
+struct Meta {
+  int32_t* kv_end;      // [kv rows]
+  Tile* qtiles;         // [nq]
+  Tile* ktiles;         // [nk] (may be null)
+  int32_t* q_order;     // [nq] q-tile indices, most expensive first
+  int32_t* k_order;     // [nk]
+  int64_t nq, nk;
+};
+
+// Status word bits recorded by device code.
+enum : uint32_t { kStatusTimeout = 1u };
+
+// ---------------------------------------------------------------- launches
+// Each returns cudaSuccess or the launch error.
+
+// Tile-map kernels (ism_meta.cu).
+cudaError_t launch_kv_end(const SegsDev& s, int32_t* kv_end, cudaStream_t st);
+// At most kMaxSeqs sequences (per-sequence offsets are kept in shared memory).
+constexpr int kMaxSeqs = 8192;
+cudaError_t launch_tiles(const SegsDev& s, int bm, int bn, const int32_t* kv_end, int64_t nq, int64_t nk,
+                         Tile* qtiles, Tile* ktiles, uint8_t* tile_class, int32_t* kt_full_end,
+                         int32_t* kt_end, int32_t* qt_begin, cudaStream_t st);
+cudaError_t launch_order(const Tile* qtiles, int64_t nq, const Tile* ktiles, int64_t nk, int max_cost,
+                         int32_t* q_order, int32_t* k_order, cudaStream_t st);
+cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t cap, int bm, int bn,
+                               int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
+                               int32_t* q_order, cudaStream_t st);
+cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap,
+                               const int32_t* c_snap, const void* k_new, const void* v_new,
+                               void* k_cache, void* v_cache, cudaStream_t st);
+
+// CUDA-core attention (ism_simt.cu), fp32 or bf16 storage, fp32 math.
+struct AttnArgs {
+  const void* q; const void* k; const void* v; const void* o; const void* dout;
+  void* out; float* lse; const float* lse_in;
+  void* dq; void* dk; void* dv;
+  float* delta;
+  int32_t hq, hkv, d, dtype;
+  int64_t q_rows;      // rows of Q (LSE row stride)
+  float scale;
+  const int32_t* kv_end;
+  const Tile* qtiles; const int32_t* q_order; int64_t nq;
+  const Tile* ktiles; const int32_t* k_order; int64_t nk;
+  uint32_t* status;
+};
+cudaError_t launch_simt_fwd(const AttnArgs& a, cudaStream_t st);
+cudaError_t launch_simt_bwd(const AttnArgs& a, cudaStream_t st);
+
+// Split-KV decode for single-token appends (ism_decode.cu).
+struct DecodeArgs {
+  const void* q;         // [B, Hq, D]
+  const void* k_cache;   // [B, cap, Hkv, D]
+  const void* v_cache;
+  void* out;             // [B, Hq, D]
+  float* lse;            // [Hq, B] or null
+  const int32_t* c_snap; // cache length before the append, per sequence
+  int32_t batch, hq, hkv, d, dtype;
+  int64_t cap;
+  float scale;
+  int32_t splits, chunk;
+  float* part_o;         // [B, Hq, splits, D]
+  float* part_ml;        // [B, Hq, splits, 2]
+};
+cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st);
+
+// Tensor-core kernels (ism_fwd_tc.cu / ism_bwd_tc.cu), bf16 only.
+bool tc_available();
+cudaError_t launch_tc_fwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st);
+cudaError_t launch_tc_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st);
+
+cudaError_t launch_timeout_probe(uint32_t spin_limit, uint32_t* status, cudaStream_t st);
+
+// Measurement hooks (ism_api.cu): events recorded around launches of one
+// kernel kind on the calling host thread, and a count of every launch.
+void timer_begin(int kernel_id, cudaStream_t st);
+void timer_end(int kernel_id, cudaStream_t st);
+void count_launch(int n = 1);
+
+}  // namespace ism

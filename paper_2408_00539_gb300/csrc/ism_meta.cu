@@ -1,0 +1,294 @@
+// Segment metadata kernels: per-token key bound kv_end (Eq. fj, Section 2.1),
+// the (q-tile, k-tile) classification, work lists for the attention kernels
+// ordered most expensive first, and the append-prefill plan (Section 2.3).
+#include "ism_internal.cuh"
+
+namespace ism {
+namespace {
+
+__device__ __forceinline__ int upper_bound_i32(const int32_t* a, int n, int32_t x) {
+  // first index i in [0, n) with a[i] > x (n if none); a non-decreasing
+  int lo = 0, hi = n;
+  while (lo < hi) {
+    int mid = (lo + hi) >> 1;
+    if (a[mid] > x) hi = mid; else lo = mid + 1;
+  }
+  return lo;
+}
+
+// Per-sequence tile offsets computed by every block into shared memory:
+// qoff/koff [B+1] (q-tiles / k-tiles before sequence b) and toff [B+1]
+// (tile_class bytes before sequence b).  Block-wide scans over chunks of
+// blockDim.x sequences with a running carry.
+__device__ void seq_offsets_smem(const SegsDev& s, int bm, int bn, int32_t* qoff, int32_t* koff, int64_t* toff) {
+  __shared__ int32_t sq[256], sk[256];
+  __shared__ int64_t stl[256];
+  __shared__ int32_t cq, ck;
+  __shared__ int64_t ct;
+  if (threadIdx.x == 0) { cq = 0; ck = 0; ct = 0; qoff[0] = 0; koff[0] = 0; toff[0] = 0; }
+  __syncthreads();
+  for (int base = 0; base < s.num_seqs; base += blockDim.x) {
+    int b = base + threadIdx.x;
+    int32_t nq = 0, nk = 0;
+    if (b < s.num_seqs) {
+      int32_t L = s.cu_seqlens[b + 1] - s.cu_seqlens[b];
+      nq = (L + bm - 1) / bm;
+      nk = (L + bn - 1) / bn;
+    }
+    sq[threadIdx.x] = nq; sk[threadIdx.x] = nk; stl[threadIdx.x] = (int64_t)nq * nk;
+    __syncthreads();
+    for (int off = 1; off < blockDim.x; off <<= 1) {  // Hillis-Steele inclusive scan
+      int32_t a = 0, c = 0; int64_t t = 0;
+      if (threadIdx.x >= off) { a = sq[threadIdx.x - off]; c = sk[threadIdx.x - off]; t = stl[threadIdx.x - off]; }
+      __syncthreads();
+      sq[threadIdx.x] += a; sk[threadIdx.x] += c; stl[threadIdx.x] += t;
+      __syncthreads();
+    }
+    if (b < s.num_seqs) {
+      qoff[b + 1] = cq + sq[threadIdx.x];
+      koff[b + 1] = ck + sk[threadIdx.x];
+      toff[b + 1] = ct + stl[threadIdx.x];
+    }
+    __syncthreads();
+    if (threadIdx.x == blockDim.x - 1) { cq += sq[threadIdx.x]; ck += sk[threadIdx.x]; ct += stl[threadIdx.x]; }
+    __syncthreads();
+  }
+}
+
+// kv_end of every token (Eq. fj): a token of a query segment is bounded by
+// the end of its segment, a token of an answer segment by itself.  One block
+// per segment (grid-stride); threads over the segment's tokens.
+__global__ void kv_end_kernel(SegsDev s, int32_t* kv_end) {
+  for (int seg = blockIdx.x; seg < s.num_segs; seg += gridDim.x) {
+    int b = upper_bound_i32(s.cu_segs, s.num_seqs + 1, seg) - 1;
+    int32_t start = seg > s.cu_segs[b] ? s.seg_end[seg - 1] : 0;
+    int32_t end = s.seg_end[seg];
+    int32_t base = s.cu_seqlens[b];
+    bool query = s.seg_type[seg] == ISM_SEG_QUERY;
+    for (int32_t j = start + threadIdx.x; j < end; j += blockDim.x)
+      kv_end[base + j] = query ? end : j + 1;
+  }
+}
+
+// q-tile and k-tile descriptors plus the optional public tile-map arrays.
+// Since kv_end is non-decreasing within a sequence, q-tile t has
+// floor(kv_end[first row] / bn) leading FULL tiles when all of its rows lie
+// inside the sequence (0 otherwise), and ceil(kv_end[last row] / bn)
+// non-empty tiles; k-tile c is first reached by the q-tile holding the first
+// row whose kv_end exceeds c*bn.
+// Block size must be 256 (the offset scan's shared arrays).
+__global__ void __launch_bounds__(256) tiles_kernel(SegsDev s, int bm, int bn, const int32_t* __restrict__ kv_end,
+                             int64_t nq, int64_t nk, Tile* qtiles, Tile* ktiles, uint8_t* tile_class,
+                             int32_t* kt_full_end, int32_t* kt_end, int32_t* qt_begin) {
+  extern __shared__ __align__(16) unsigned char dyn[];
+  int64_t* toff = reinterpret_cast<int64_t*>(dyn);
+  int32_t* qoff = reinterpret_cast<int32_t*>(toff + s.num_seqs + 1);
+  int32_t* koff = qoff + s.num_seqs + 1;
+  seq_offsets_smem(s, bm, bn, qoff, koff, toff);
+  int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < nq; g += stride) {
+    int b = upper_bound_i32(qoff, s.num_seqs + 1, (int32_t)g) - 1;
+    int32_t t = (int32_t)g - qoff[b];
+    int32_t base = s.cu_seqlens[b];
+    int32_t L = s.cu_seqlens[b + 1] - base;
+    int32_t r0 = t * bm;
+    int32_t rl = min(L, r0 + bm) - 1;
+    int32_t full = (r0 + bm <= L) ? kv_end[base + r0] / bn : 0;
+    int32_t ne = (kv_end[base + rl] + bn - 1) / bn;
+    if (qtiles) {
+      Tile w;
+      w.q_base = base; w.k_base = base; w.q_len = L; w.k_len = L; w.tile = t;
+      w.a0 = full; w.a1 = ne; w.kv_base = base;
+      qtiles[g] = w;
+    }
+    if (kt_full_end) kt_full_end[g] = full;
+    if (kt_end) kt_end[g] = ne;
+    if (tile_class) {
+      int32_t nkt = (L + bn - 1) / bn;
+      uint8_t* row = tile_class + toff[b] + (int64_t)t * nkt;
+      for (int32_t c = 0; c < nkt; ++c)
+        row[c] = c < full ? (uint8_t)ISM_TILE_FULL : c < ne ? (uint8_t)ISM_TILE_PARTIAL : (uint8_t)ISM_TILE_EMPTY;
+    }
+  }
+  for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < nk; g += stride) {
+    int b = upper_bound_i32(koff, s.num_seqs + 1, (int32_t)g) - 1;
+    int32_t c = (int32_t)g - koff[b];
+    int32_t base = s.cu_seqlens[b];
+    int32_t L = s.cu_seqlens[b + 1] - base;
+    int32_t j = upper_bound_i32(kv_end + base, L, c * bn);  // first row that sees key c*bn
+    int32_t qb = j / bm;
+    if (qt_begin) qt_begin[g] = qb;
+    if (ktiles) {
+      Tile w;
+      w.q_base = base; w.k_base = base; w.q_len = L; w.k_len = L; w.tile = c;
+      w.a0 = qb; w.a1 = (L + bm - 1) / bm; w.kv_base = base;
+      ktiles[g] = w;
+    }
+  }
+}
+
+// Work lists ordered by decreasing cost (counting sort, one block).  Cost of
+// a q-tile = its non-empty k-tiles; of a k-tile = its non-empty q-tiles.
+// Items of equal cost come in arbitrary order; results do not depend on it.
+__global__ void order_kernel(const Tile* __restrict__ qtiles, int64_t nq, const Tile* __restrict__ ktiles,
+                             int64_t nk, int max_cost, int32_t* q_order, int32_t* k_order) {
+  extern __shared__ int32_t hist[];  // [max_cost + 1]
+  for (int pass = 0; pass < 2; ++pass) {
+    const Tile* items = pass == 0 ? qtiles : ktiles;
+    int64_t n = pass == 0 ? nq : nk;
+    int32_t* order = pass == 0 ? q_order : k_order;
+    if (items == nullptr || order == nullptr || n == 0) continue;
+    for (int i = threadIdx.x; i <= max_cost; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
+      Tile w = items[i];
+      int cost = pass == 0 ? w.a1 : w.a1 - w.a0;
+      cost = min(max(cost, 0), max_cost);
+      atomicAdd(&hist[cost], 1);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {  // exclusive scan from the highest cost down
+      int32_t run = 0;
+      for (int c = max_cost; c >= 0; --c) { int32_t h = hist[c]; hist[c] = run; run += h; }
+    }
+    __syncthreads();
+    for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
+      Tile w = items[i];
+      int cost = pass == 0 ? w.a1 : w.a1 - w.a0;
+      cost = min(max(cost, 0), max_cost);
+      order[atomicAdd(&hist[cost], 1)] = (int32_t)i;
+    }
+    __syncthreads();
+  }
+}
+
+__device__ __forceinline__ int32_t chunk_kv_end(const AppendSegs& sg, int32_t j) {
+  int32_t start = 0;
+  for (int i = 0; i < sg.n; ++i) {
+    int32_t e = sg.end[i];
+    if (j < e && j >= start) return sg.type[i] == ISM_SEG_QUERY ? e : j + 1;
+    start = e;
+  }
+  return j + 1;
+}
+
+// Append plan (one block): snapshot cache_len, advance it by l_new, write the
+// absolute key bound of every new row (all cached keys plus Eq. fj within
+// the chunk) and one q-tile descriptor per (sequence, chunk tile).
+__global__ void append_plan_kernel(AppendSegs sg, int batch, int64_t cap, int bm, int bn,
+                                   int32_t* cache_len, int32_t* c_snap, int32_t* kv_end,
+                                   Tile* qtiles, int32_t* q_order) {
+  __shared__ int32_t cs[1024];
+  const int32_t Ln = sg.l_new;
+  for (int base = 0; base < batch; base += 1024) {
+    // (batch > 1024 is handled in chunks; every thread sees its own chunk)
+    int b = base + threadIdx.x;
+    if (threadIdx.x < 1024 && b < batch) cs[threadIdx.x] = cache_len[b];
+    __syncthreads();
+    int nb = min(1024, batch - base);
+    for (int i = threadIdx.x; i < nb * Ln; i += blockDim.x) {
+      int bl = i / Ln, j = i % Ln;
+      kv_end[(int64_t)(base + bl) * Ln + j] = cs[bl] + chunk_kv_end(sg, j);
+    }
+    int nqt = (Ln + bm - 1) / bm;
+    for (int i = threadIdx.x; i < nb * nqt; i += blockDim.x) {
+      int bl = i / nqt, t = i % nqt;
+      int32_t c = cs[bl];
+      int32_t r0 = t * bm, rl = min(Ln, r0 + bm) - 1;
+      Tile w;
+      w.q_base = (base + bl) * Ln; w.k_base = (int32_t)((base + bl) * cap);
+      w.q_len = Ln; w.k_len = c + Ln; w.tile = t;
+      w.a0 = (r0 + bm <= Ln) ? (c + chunk_kv_end(sg, r0)) / bn : 0;
+      w.a1 = (c + chunk_kv_end(sg, rl) + bn - 1) / bn;
+      w.kv_base = (base + bl) * Ln;
+      int64_t g = (int64_t)(base + bl) * nqt + t;
+      qtiles[g] = w;
+      q_order[g] = (int32_t)g;
+    }
+    __syncthreads();
+    if (threadIdx.x < nb) {
+      c_snap[base + threadIdx.x] = cs[threadIdx.x];
+      cache_len[base + threadIdx.x] = cs[threadIdx.x] + Ln;
+    }
+    __syncthreads();
+  }
+}
+
+// K_new/V_new rows into the caches at [c_snap[b], c_snap[b] + l_new).
+__global__ void cache_write_kernel(int batch, int l_new, int row_bytes, int64_t cap,
+                                   const int32_t* __restrict__ c_snap, const uint4* __restrict__ k_new,
+                                   const uint4* __restrict__ v_new, uint4* k_cache, uint4* v_cache) {
+  const int vec_per_row = row_bytes / 16;
+  const int64_t total = (int64_t)batch * l_new * vec_per_row;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    int64_t row = i / vec_per_row;
+    int col = (int)(i % vec_per_row);
+    int b = (int)(row / l_new);
+    int j = (int)(row % l_new);
+    int64_t dst = ((int64_t)b * cap + c_snap[b] + j) * vec_per_row + col;
+    k_cache[dst] = k_new[i];
+    v_cache[dst] = v_new[i];
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_kv_end(const SegsDev& s, int32_t* kv_end, cudaStream_t st) {
+  if (s.num_segs == 0) return cudaSuccess;
+  int grid = s.num_segs < 4096 ? s.num_segs : 4096;
+  kv_end_kernel<<<grid, 256, 0, st>>>(s, kv_end);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tiles(const SegsDev& s, int bm, int bn, const int32_t* kv_end, int64_t nq, int64_t nk,
+                         Tile* qtiles, Tile* ktiles, uint8_t* tile_class, int32_t* kt_full_end,
+                         int32_t* kt_end, int32_t* qt_begin, cudaStream_t st) {
+  int64_t n = nq > nk ? nq : nk;
+  if (n == 0) return cudaSuccess;
+  int grid = (int)((n + 255) / 256);
+  if (grid > 608) grid = 608;
+  size_t smem = (size_t)(s.num_seqs + 1) * (sizeof(int64_t) + 2 * sizeof(int32_t));
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(tiles_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  tiles_kernel<<<grid, 256, smem, st>>>(s, bm, bn, kv_end, nq, nk, qtiles, ktiles, tile_class, kt_full_end,
+                                        kt_end, qt_begin);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_order(const Tile* qtiles, int64_t nq, const Tile* ktiles, int64_t nk, int max_cost,
+                         int32_t* q_order, int32_t* k_order, cudaStream_t st) {
+  size_t smem = sizeof(int32_t) * (size_t)(max_cost + 1);
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(order_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  order_kernel<<<1, 1024, smem, st>>>(qtiles, nq, ktiles, nk, max_cost, q_order, k_order);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t cap, int bm, int bn,
+                               int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
+                               int32_t* q_order, cudaStream_t st) {
+  append_plan_kernel<<<1, 1024, 0, st>>>(segs, batch, cap, bm, bn, cache_len, c_snap, kv_end, qtiles,
+                                         q_order);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap,
+                               const int32_t* c_snap, const void* k_new, const void* v_new,
+                               void* k_cache, void* v_cache, cudaStream_t st) {
+  int elem = dtype == ISM_BF16 ? 2 : 4;
+  int row_bytes = hkv * d * elem;
+  int64_t total = (int64_t)batch * l_new * (row_bytes / 16);
+  if (total == 0) return cudaSuccess;
+  int grid = (int)((total + 255) / 256);
+  if (grid > 152 * 16) grid = 152 * 16;
+  cache_write_kernel<<<grid, 256, 0, st>>>(batch, l_new, row_bytes, cap, c_snap, (const uint4*)k_new,
+                                           (const uint4*)v_new, (uint4*)k_cache, (uint4*)v_cache);
+  return cudaGetLastError();
+}
+
+}  // namespace ism

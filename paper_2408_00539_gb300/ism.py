@@ -1,0 +1,293 @@
+"""Python binding of libism (ctypes).  Argument marshalling only: every step
+of the attention path runs in the library's CUDA kernels.  PyTorch supplies
+device memory (outputs and workspaces) and the current CUDA stream.
+
+There is no fallback: if libism.so is missing or a call fails, an exception
+is raised.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+from dataclasses import dataclass
+from typing import Optional
+
+import numpy as np
+import torch
+
+from . import build as _build
+
+ISM_BF16, ISM_FP32 = 0, 1
+QUERY, ANSWER = 0, 1
+TILE_EMPTY, TILE_FULL, TILE_PARTIAL = 0, 1, 2
+
+_STATUS = {0: "ISM_OK", 1: "ISM_ERR_INVALID_ARG", 2: "ISM_ERR_UNSUPPORTED", 3: "ISM_ERR_CUDA",
+           4: "ISM_ERR_TIMEOUT", 5: "ISM_ERR_WORKSPACE"}
+
+
+class IsmError(RuntimeError):
+    def __init__(self, code: int, where: str, detail: str):
+        super().__init__(f"{where}: {_STATUS.get(code, code)}: {detail}")
+        self.code = code
+
+
+class _Segments(C.Structure):
+    _fields_ = [("num_seqs", C.c_int32), ("num_segs", C.c_int32),
+                ("cu_seqlens", C.c_void_p), ("cu_seqlens_host", C.c_void_p),
+                ("cu_segs", C.c_void_p), ("cu_segs_host", C.c_void_p),
+                ("seg_end", C.c_void_p), ("seg_end_host", C.c_void_p),
+                ("seg_type", C.c_void_p), ("seg_type_host", C.c_void_p)]
+
+
+class _Shape(C.Structure):
+    _fields_ = [("num_heads_q", C.c_int32), ("num_heads_kv", C.c_int32), ("head_dim", C.c_int32),
+                ("dtype", C.c_int32), ("softmax_scale", C.c_float)]
+
+
+EXPORTS = {
+    "ism_tile_map_size": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p]),
+    "ism_build_tile_map": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32] + [C.c_void_p] * 6),
+    "ism_attn_fwd_workspace_size": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "ism_attn_fwd": (C.c_int, [C.c_void_p] * 8 + [C.c_size_t, C.c_void_p]),
+    "ism_attn_bwd_workspace_size": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "ism_attn_bwd": (C.c_int, [C.c_void_p] * 12 + [C.c_size_t, C.c_void_p]),
+    "ism_attn_prefill_append_workspace_size": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_void_p]),
+    "ism_attn_prefill_append": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
+                                          C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_int64,
+                                          C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                          C.c_size_t, C.c_void_p]),
+    "ism_check_status": (C.c_int, [C.c_void_p]),
+    "ism_debug_timeout_probe": (C.c_int, [C.c_uint32, C.c_void_p]),
+    "ism_status_string": (C.c_char_p, [C.c_int]),
+    "ism_last_error": (C.c_char_p, []),
+    "ism_has_tensor_cores": (C.c_int32, []),
+    "ism_set_kernel_timer": (C.c_int, [C.c_int32, C.c_void_p, C.c_void_p]),
+    "ism_kernel_launches": (C.c_uint64, []),
+}
+
+KERNEL_FWD, KERNEL_BWD_DKDV, KERNEL_BWD_DQ, KERNEL_BWD_PRE, KERNEL_DECODE, KERNEL_META = 1, 2, 3, 4, 5, 6
+
+_lib = None
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = False):
+    """Load libism.so (building it first when asked)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB
+    if not os.path.exists(path):
+        if not build_if_missing:
+            raise RuntimeError(f"libism.so not built ({path}); run __graft_entry__.build()")
+        _build.build()
+    lib = C.CDLL(path)
+    for name, (res, args) in EXPORTS.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = lib
+    return lib
+
+
+def _check(code: int, where: str):
+    if code != 0:
+        raise IsmError(code, where, load().ism_last_error().decode())
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else C.c_void_p(t.data_ptr())
+
+
+def _stream(device=None):
+    return C.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return ISM_BF16
+    if t.dtype == torch.float32:
+        return ISM_FP32
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _workspace(nbytes: int, device) -> torch.Tensor:
+    ws = torch.empty(nbytes + 256, dtype=torch.uint8, device=device)
+    off = (-ws.data_ptr()) % 256
+    return ws[off:off + nbytes] if nbytes else ws[off:off]
+
+
+@dataclass
+class Segments:
+    """Varlen turn boundaries in both device and host form (the host mirrors
+    are used for validation and sizing without a device synchronisation)."""
+    cu_seqlens: torch.Tensor
+    cu_segs: torch.Tensor
+    seg_end: torch.Tensor
+    seg_type: torch.Tensor
+    cu_seqlens_host: np.ndarray
+    cu_segs_host: np.ndarray
+    seg_end_host: np.ndarray
+    seg_type_host: np.ndarray
+
+    @staticmethod
+    def from_numpy(cu_seqlens, cu_segs, seg_end, seg_type, device="cuda") -> "Segments":
+        h = [np.ascontiguousarray(cu_seqlens, dtype=np.int32), np.ascontiguousarray(cu_segs, dtype=np.int32),
+             np.ascontiguousarray(seg_end, dtype=np.int32), np.ascontiguousarray(seg_type, dtype=np.uint8)]
+        d = [torch.from_numpy(x.copy()).to(device) for x in h]
+        return Segments(*d, *h)
+
+    @staticmethod
+    def from_workload(segs, device="cuda") -> "Segments":
+        return Segments.from_numpy(segs.cu_seqlens, segs.cu_segs, segs.seg_end, segs.seg_type, device)
+
+    @property
+    def total_tokens(self) -> int:
+        return int(self.cu_seqlens_host[-1])
+
+    def struct(self) -> _Segments:
+        s = _Segments()
+        s.num_seqs = self.cu_seqlens_host.shape[0] - 1
+        s.num_segs = self.seg_end_host.shape[0]
+        s.cu_seqlens, s.cu_seqlens_host = self.cu_seqlens.data_ptr(), self.cu_seqlens_host.ctypes.data
+        s.cu_segs, s.cu_segs_host = self.cu_segs.data_ptr(), self.cu_segs_host.ctypes.data
+        s.seg_end, s.seg_end_host = self.seg_end.data_ptr(), self.seg_end_host.ctypes.data
+        s.seg_type, s.seg_type_host = self.seg_type.data_ptr(), self.seg_type_host.ctypes.data
+        return s
+
+
+def _shape(q: torch.Tensor, k: torch.Tensor, scale: float) -> _Shape:
+    sh = _Shape()
+    sh.num_heads_q, sh.head_dim = q.shape[-2], q.shape[-1]
+    sh.num_heads_kv = k.shape[-2]
+    sh.dtype = _dtype_code(q)
+    sh.softmax_scale = float(scale)
+    return sh
+
+
+def _contig(*ts):
+    for t in ts:
+        if t is not None and not t.is_contiguous():
+            raise ValueError("tensors must be contiguous")
+
+
+def tile_map(segs: Segments, bm: int = 128, bn: int = 128):
+    """Tile map of the segments (device tensors): tile_class, kt_full_end,
+    kt_end, qt_begin, kv_end."""
+    lib = load()
+    s = segs.struct()
+    nt, nq, nk = C.c_int64(), C.c_int64(), C.c_int64()
+    _check(lib.ism_tile_map_size(C.byref(s), bm, bn, C.byref(nt), C.byref(nq), C.byref(nk)), "ism_tile_map_size")
+    dev = segs.cu_seqlens.device
+    out = {
+        "tile_class": torch.empty(nt.value, dtype=torch.uint8, device=dev),
+        "kt_full_end": torch.empty(nq.value, dtype=torch.int32, device=dev),
+        "kt_end": torch.empty(nq.value, dtype=torch.int32, device=dev),
+        "qt_begin": torch.empty(nk.value, dtype=torch.int32, device=dev),
+        "kv_end": torch.empty(segs.total_tokens, dtype=torch.int32, device=dev),
+    }
+    _check(lib.ism_build_tile_map(C.byref(s), bm, bn, _ptr(out["tile_class"]), _ptr(out["kt_full_end"]),
+                                  _ptr(out["kt_end"]), _ptr(out["qt_begin"]), _ptr(out["kv_end"]), _stream(dev)),
+           "ism_build_tile_map")
+    return out
+
+
+def fwd(segs: Segments, q, k, v, softmax_scale: float, out=None, lse=None, workspace=None):
+    """Forward over packed dialogues.  q [T,Hq,D], k/v [T,Hkv,D] -> (o, lse [Hq,T])."""
+    lib = load()
+    _contig(q, k, v)
+    T, hq, D = q.shape
+    s, sh = segs.struct(), _shape(q, k, softmax_scale)
+    nbytes = C.c_size_t()
+    _check(lib.ism_attn_fwd_workspace_size(C.byref(s), C.byref(sh), C.byref(nbytes)), "ism_attn_fwd_workspace_size")
+    if out is None:
+        out = torch.empty_like(q)
+    if lse is None:
+        lse = torch.empty((hq, T), dtype=torch.float32, device=q.device)
+    if workspace is None or workspace.numel() < nbytes.value:
+        workspace = _workspace(nbytes.value, q.device)
+    _check(lib.ism_attn_fwd(C.byref(s), C.byref(sh), _ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(lse),
+                            _ptr(workspace), workspace.numel(), _stream(q.device)), "ism_attn_fwd")
+    return out, lse
+
+
+def bwd(segs: Segments, q, k, v, o, lse, dout, softmax_scale: float, dq=None, dk=None, dv=None, workspace=None):
+    """Backward: (dq, dk, dv) of sum(O * dout)."""
+    lib = load()
+    _contig(q, k, v, o, lse, dout)
+    s, sh = segs.struct(), _shape(q, k, softmax_scale)
+    nbytes = C.c_size_t()
+    _check(lib.ism_attn_bwd_workspace_size(C.byref(s), C.byref(sh), C.byref(nbytes)), "ism_attn_bwd_workspace_size")
+    dq = torch.empty_like(q) if dq is None else dq
+    dk = torch.empty_like(k) if dk is None else dk
+    dv = torch.empty_like(v) if dv is None else dv
+    if workspace is None or workspace.numel() < nbytes.value:
+        workspace = _workspace(nbytes.value, q.device)
+    _check(lib.ism_attn_bwd(C.byref(s), C.byref(sh), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), _ptr(dout),
+                            _ptr(dq), _ptr(dk), _ptr(dv), _ptr(workspace), workspace.numel(), _stream(q.device)),
+           "ism_attn_bwd")
+    return dq, dk, dv
+
+
+def prefill_append(q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_host, new_seg_end, new_seg_type,
+                   softmax_scale: float, out=None, lse=None, workspace=None):
+    """Append a new turn to the KV caches and attend (Section 2.3).
+    q_new [B,Ln,Hq,D], k_new/v_new [B,Ln,Hkv,D], caches [B,cap,Hkv,D],
+    cache_len int32 [B] on the device (advanced by Ln), cache_len_host its
+    host mirror (the caller advances it).  Returns (o_new, lse [Hq,B,Ln])."""
+    lib = load()
+    _contig(q_new, k_new, v_new, k_cache, v_cache, cache_len)
+    B, Ln, hq, D = q_new.shape
+    cap = k_cache.shape[1]
+    sh = _shape(q_new, k_new, softmax_scale)
+    se = np.ascontiguousarray(new_seg_end, dtype=np.int32)
+    st = np.ascontiguousarray(new_seg_type, dtype=np.uint8)
+    ch = np.ascontiguousarray(cache_len_host, dtype=np.int32)
+    nbytes = C.c_size_t()
+    _check(lib.ism_attn_prefill_append_workspace_size(C.byref(sh), B, Ln, C.byref(nbytes)),
+           "ism_attn_prefill_append_workspace_size")
+    if out is None:
+        out = torch.empty_like(q_new)
+    if lse is None:
+        lse = torch.empty((hq, B, Ln), dtype=torch.float32, device=q_new.device)
+    if workspace is None or workspace.numel() < nbytes.value:
+        workspace = _workspace(nbytes.value, q_new.device)
+    _check(lib.ism_attn_prefill_append(C.byref(sh), B, _ptr(q_new), _ptr(k_new), _ptr(v_new), Ln,
+                                       C.c_void_p(se.ctypes.data), C.c_void_p(st.ctypes.data), se.shape[0],
+                                       _ptr(k_cache), _ptr(v_cache), cap, _ptr(cache_len), C.c_void_p(ch.ctypes.data),
+                                       _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(),
+                                       _stream(q_new.device)),
+           "ism_attn_prefill_append")
+    return out, lse
+
+
+def check_status(device=None):
+    """Synchronise the current stream and raise if a kernel gave up a wait."""
+    _check(load().ism_check_status(_stream(device)), "ism_check_status")
+
+
+def debug_timeout_probe(spin_limit: int = 64, device=None) -> int:
+    """Run the bounded-wait probe; returns the status code ism_check_status
+    reports afterwards (expected ISM_ERR_TIMEOUT = 4)."""
+    lib = load()
+    _check(lib.ism_debug_timeout_probe(spin_limit, _stream(device)), "ism_debug_timeout_probe")
+    return lib.ism_check_status(_stream(device))
+
+
+def has_tensor_cores() -> bool:
+    return bool(load().ism_has_tensor_cores())
+
+
+def set_kernel_timer(kernel_id: int, start: "torch.cuda.Event" = None, stop: "torch.cuda.Event" = None):
+    """Bracket every launch of one kernel kind (on this thread) with the
+    given CUDA events; call with no events to clear."""
+    sp = None if start is None else C.c_void_p(start.cuda_event)
+    ep = None if stop is None else C.c_void_p(stop.cuda_event)
+    _check(load().ism_set_kernel_timer(kernel_id, sp, ep), "ism_set_kernel_timer")
+
+
+def kernel_launches() -> int:
+    return int(load().ism_kernel_launches())

@@ -1,0 +1,20 @@
+"""CPU checks of the benchmark's host logic."""
+import numpy as np
+
+import bench
+from oracle import ism_oracle as orc
+from paper_2408_00539_gb300 import workloads as wl
+
+
+def test_visible_pair_count_matches_mask():
+    rng = np.random.Generator(np.random.PCG64(5))
+    segs = wl.random_dialogue_set(rng, 20, 300)
+    assert bench.n_visible(segs) == int(orc.packed_mask(segs).sum())
+    tiny = wl.tiny_fp32().segs
+    assert bench.n_visible(tiny) == int(orc.packed_mask(tiny).sum())
+
+
+def test_headline_density_close_to_half():
+    w = wl.gqa_8k()
+    dens = bench.n_visible(w.segs) / sum(L * L for L in np.diff(w.segs.cu_seqlens))
+    assert 0.5 <= dens <= 0.56

@@ -1,0 +1,339 @@
+"""GPU parity tests: the CUDA path through the C ABI against the fp64 oracle
+on identical seeded inputs.
+
+Tolerances: tile maps bit-exact; bf16 inputs (fp32 accumulation) max-abs
+2e-2 and mean-abs 2e-3 on O, dQ, dK, dV; fp32 inputs max-abs 1e-4; LSE 1e-3
+(bf16) and 1e-5 (fp32) absolute.
+"""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import ism_oracle as orc
+from paper_2408_00539_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+BF16_MAX, BF16_MEAN, FP32_MAX = 2e-2, 2e-3, 1e-4
+
+
+@pytest.fixture(scope="module")
+def ism():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2408_00539_gb300 import ism as m
+    m.load(build_if_missing=True)
+    return m
+
+
+DEV = "cuda:0"
+
+
+def _np(t):
+    return t.detach().float().cpu().numpy().astype(np.float64) if t.dtype != torch.float64 else t.cpu().numpy()
+
+
+def _cmp(name, got, ref, dtype):
+    got = _np(got) if isinstance(got, torch.Tensor) else got
+    assert got.shape == ref.shape, (name, got.shape, ref.shape)
+    assert np.all(np.isfinite(got)), f"{name}: non-finite values"
+    err = np.abs(got - ref)
+    if dtype == "fp32":
+        assert err.max() <= FP32_MAX, f"{name}: max abs err {err.max():.3e}"
+    else:
+        assert err.max() <= BF16_MAX, f"{name}: max abs err {err.max():.3e}"
+        assert err.mean() <= BF16_MEAN, f"{name}: mean abs err {err.mean():.3e}"
+
+
+def _cmp_lse(name, got, ref, dtype):
+    got = _np(got)
+    err = np.abs(got - ref)
+    assert err.max() <= (1e-5 if dtype == "fp32" else 1e-3), f"{name}: max abs err {err.max():.3e}"
+
+
+def _run_pass(ism, w, seed_offset=0):
+    q, k, v, do = wl.attention_tensors(w, seed_offset=seed_offset)
+    segs = ism.Segments.from_workload(w.segs, DEV)
+    qd, kd, vd, dod = (t.to(DEV) for t in (q, k, v, do))
+    o, lse = ism.fwd(segs, qd, kd, vd, w.softmax_scale)
+    dq, dk, dv = ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale)
+    ism.check_status()
+    return (q, k, v, do), (o, lse, dq, dk, dv)
+
+
+# ---------------------------------------------------------------- tile map
+
+def _tile_cases():
+    rng = np.random.Generator(np.random.PCG64(101))
+    yield "random", wl.random_dialogue_set(rng, 40, 700)
+    yield "edges", wl.pack([([1], [1]), ([0, 0, 1], [0, 1, 0]), ([5, 5, 129], [0, 0, 1]),
+                            ([128, 256], [0, 1]), ([127, 128, 129], [1, 0, 0]), ([0, 0], [0, 1])])
+    yield "gqa_8k", wl.gqa_8k().segs
+    yield "packed_32k", wl.packed_32k().segs
+
+
+@pytest.mark.parametrize("bm,bn", [(128, 128), (128, 64), (64, 128), (64, 64)])
+def test_tile_map_bit_exact(ism, bm, bn):
+    for name, segs_np in _tile_cases():
+        segs = ism.Segments.from_workload(segs_np, DEV)
+        got = ism.tile_map(segs, bm, bn)
+        ref = orc.tile_map_packed(segs_np, bm, bn)
+        for key in ("tile_class", "kt_full_end", "kt_end", "qt_begin", "kv_end"):
+            g = got[key].cpu().numpy()
+            r = np.asarray(ref[key]).astype(g.dtype)
+            assert np.array_equal(g, r), f"{name} {key} bm={bm} bn={bn}"
+
+
+# ---------------------------------------------------------------- one pass
+
+def test_tiny_fp32_fwd_bwd(ism):
+    w = wl.tiny_fp32()
+    (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w)
+    o_ref, lse_ref = orc.attn_fwd(q, k, v, w.segs, w.softmax_scale)
+    dq_ref, dk_ref, dv_ref = orc.attn_bwd(q, k, v, do, w.segs, w.softmax_scale)
+    _cmp("o", o, o_ref, "fp32")
+    _cmp_lse("lse", lse, lse_ref, "fp32")
+    _cmp("dq", dq, dq_ref, "fp32")
+    _cmp("dk", dk, dk_ref, "fp32")
+    _cmp("dv", dv, dv_ref, "fp32")
+
+
+def _small_bf16(d, hq=8, hkv=2, seed=9):
+    segs = wl.pack([([70, 150, 170, 300], [0, 1, 0, 1]),      # ragged 300
+                    ([33, 90, 200, 517], [0, 1, 0, 1]),        # several tiles + tail
+                    ([129], [0]),                              # one query segment: full attention
+                    ([1], [1]),                                # single token
+                    ([0, 64, 64, 128, 256], [1, 0, 1, 0, 1]),  # tile-aligned, zero-length segment
+                    ([50, 51, 52, 383], [0, 0, 1, 0])])        # adjacent queries, long final query
+    return wl.Workload(f"small_d{d}", segs, hq, hkv, d, "bf16", d ** -0.5, 0.5, seed)
+
+
+@pytest.mark.parametrize("d", [128, 64])
+@pytest.mark.parametrize("path", ["default", "cuda_cores"])
+def test_small_bf16_fwd_bwd(ism, d, path, monkeypatch):
+    if path == "cuda_cores":
+        monkeypatch.setenv("ISM_FORCE_CUDA_CORES", "1")
+    w = _small_bf16(d)
+    (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w)
+    o_ref, lse_ref = orc.attn_fwd(q, k, v, w.segs, w.softmax_scale)
+    dq_ref, dk_ref, dv_ref = orc.attn_bwd(q, k, v, do, w.segs, w.softmax_scale)
+    _cmp("o", o, o_ref, "bf16")
+    _cmp_lse("lse", lse, lse_ref, "bf16")
+    _cmp("dq", dq, dq_ref, "bf16")
+    _cmp("dk", dk, dk_ref, "bf16")
+    _cmp("dv", dv, dv_ref, "bf16")
+
+
+def test_special_cases_match_causal_and_full(ism):
+    # every token its own answer -> causal; one query segment -> full attention
+    L = 300
+    segs_np = wl.pack([([L], [wl.ANSWER]), ([L], [wl.QUERY])])
+    w = wl.Workload("special", segs_np, 4, 4, 128, "bf16", 128 ** -0.5, 0.5, 13)
+    q, k, v, _ = wl.attention_tensors(w)
+    segs = ism.Segments.from_workload(segs_np, DEV)
+    o, _ = ism.fwd(segs, q.to(DEV), k.to(DEV), v.to(DEV), w.softmax_scale)
+    qf, kf, vf = (t.double().permute(1, 0, 2) for t in (q, k, v))
+    causal = torch.nn.functional.scaled_dot_product_attention(qf[:, :L], kf[:, :L], vf[:, :L], is_causal=True,
+                                                              scale=w.softmax_scale)
+    full = torch.nn.functional.scaled_dot_product_attention(qf[:, L:], kf[:, L:], vf[:, L:], scale=w.softmax_scale)
+    _cmp("causal", o[:L], causal.permute(1, 0, 2).numpy(), "bf16")
+    _cmp("full", o[L:], full.permute(1, 0, 2).numpy(), "bf16")
+
+
+def test_earlier_turn_rows_unchanged(ism):
+    # Section 2.3: appending turns leaves earlier rows unchanged; with the
+    # history ending on a 128-token tile boundary the GPU rows are identical.
+    full = wl.pack([([100, 256, 300, 512], [0, 1, 0, 1])])
+    pre = wl.pack([([100, 256], [0, 1])])
+    w = wl.Workload("inv", full, 4, 2, 128, "bf16", 128 ** -0.5, 0.5, 17)
+    q, k, v, _ = wl.attention_tensors(w)
+    o_full, l_full = ism.fwd(ism.Segments.from_workload(full, DEV), q.to(DEV), k.to(DEV), v.to(DEV), w.softmax_scale)
+    o_pre, l_pre = ism.fwd(ism.Segments.from_workload(pre, DEV), q[:256].contiguous().to(DEV),
+                           k[:256].contiguous().to(DEV), v[:256].contiguous().to(DEV), w.softmax_scale)
+    assert torch.equal(o_full[:256], o_pre)
+    assert torch.equal(l_full[:, :256], l_pre)
+
+
+def test_empty_batch_is_noop(ism):
+    segs = ism.Segments.from_numpy([0, 0], [0, 0], [], [], DEV)
+    q = torch.zeros((0, 4, 128), dtype=torch.bfloat16, device=DEV)
+    k = torch.zeros((0, 2, 128), dtype=torch.bfloat16, device=DEV)
+    o, lse = ism.fwd(segs, q, k, k, 0.1)
+    assert o.shape == (0, 4, 128)
+    ism.check_status()
+
+
+def test_bounded_wait_reports_timeout(ism):
+    assert ism.debug_timeout_probe(64) == 4          # ISM_ERR_TIMEOUT read back from the status word
+    ism.check_status()                               # cleared: the context is still usable
+    x = torch.ones(4, device=DEV)
+    assert float(x.sum()) == 4.0
+
+
+# ---------------------------------------------------------------- full sizes
+
+def _largest_seq(segs):
+    lens = np.diff(segs.cu_seqlens)
+    return int(np.argmax(lens))
+
+
+@pytest.mark.parametrize("make", [wl.mha_4k, wl.gqa_8k, wl.packed_32k], ids=["mha_4k", "gqa_8k", "packed_32k"])
+def test_full_size_parity_sampled_group(ism, make):
+    """Full-size launch (all sequences, all heads, as benchmarked); the oracle
+    recomputes one complete GQA group of one sequence (the longest)."""
+    w = make()
+    (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w)
+    b = _largest_seq(w.segs)
+    t0, L, se, st = w.segs.seq(b)
+    grp = w.num_heads_q // w.num_heads_kv
+    g = 1 if w.num_heads_kv > 1 else 0
+    hs = slice(g * grp, (g + 1) * grp)
+    sub = wl.pack([(se, st)])
+    sl = slice(t0, t0 + L)
+    qs, dos = q[sl][:, hs].contiguous(), do[sl][:, hs].contiguous()
+    ks, vs = k[sl][:, g:g + 1].contiguous(), v[sl][:, g:g + 1].contiguous()
+    o_ref, lse_ref = orc.attn_fwd(qs, ks, vs, sub, w.softmax_scale)
+    dq_ref, dk_ref, dv_ref = orc.attn_bwd(qs, ks, vs, dos, sub, w.softmax_scale)
+    _cmp("o", o[sl][:, hs], o_ref, "bf16")
+    _cmp_lse("lse", lse[hs][:, sl], lse_ref, "bf16")
+    _cmp("dq", dq[sl][:, hs], dq_ref, "bf16")
+    _cmp("dk", dk[sl][:, g:g + 1], dk_ref, "bf16")
+    _cmp("dv", dv[sl][:, g:g + 1], dv_ref, "bf16")
+
+
+# ---------------------------------------------------------------- KV cache
+
+def _append_inputs(B, cap, c_lens, l_new, hq, hkv, d, seed, std=0.5):
+    rng = np.random.Generator(np.random.PCG64(seed))
+    kc = wl.round_to(wl.normal(rng, (B, cap, hkv, d), std), "bf16")
+    vc = wl.round_to(wl.normal(rng, (B, cap, hkv, d), std), "bf16")
+    qn = wl.round_to(wl.normal(rng, (B, l_new, hq, d), std), "bf16")
+    kn = wl.round_to(wl.normal(rng, (B, l_new, hkv, d), std), "bf16")
+    vn = wl.round_to(wl.normal(rng, (B, l_new, hkv, d), std), "bf16")
+    return kc, vc, qn, kn, vn
+
+
+@pytest.mark.parametrize("l_new,segs", [(200, ([40, 41, 120, 200], [0, 1, 0, 1])), (128, ([128], [0])),
+                                        (1, ([1], [1])), (37, ([37], [0]))])
+def test_prefill_append_small(ism, l_new, segs):
+    B, hq, hkv, d = 3, 8, 2, 128
+    c_lens = np.array([0, 77, 300], dtype=np.int32)
+    cap = 300 + l_new + 5
+    kc, vc, qn, kn, vn = _append_inputs(B, cap, c_lens, l_new, hq, hkv, d, seed=l_new)
+    kcd, vcd = kc.to(DEV), vc.to(DEV)
+    cl = torch.from_numpy(c_lens.copy()).to(DEV)
+    scale = d ** -0.5
+    o, lse = ism.prefill_append(qn.to(DEV), kn.to(DEV), vn.to(DEV), kcd, vcd, cl, c_lens, segs[0], segs[1], scale)
+    ism.check_status()
+    assert cl.cpu().numpy().tolist() == (c_lens + l_new).tolist()
+    for b in range(B):
+        c = int(c_lens[b])
+        assert torch.equal(kcd[b, c:c + l_new].cpu(), kn[b]) and torch.equal(vcd[b, c:c + l_new].cpu(), vn[b])
+        assert torch.equal(kcd[b, :c].cpu(), kc[b, :c])
+    o_ref, lse_ref = orc.prefill_append(qn, kn, vn, kc, vc, c_lens, segs[0], segs[1], scale)
+    _cmp("o_new", o, o_ref, "bf16")
+    _cmp_lse("lse_new", lse, np.transpose(lse_ref, (1, 0, 2)), "bf16")
+
+
+def test_prefill_append_matches_one_pass_rows(ism):
+    # the appended turn's rows equal the rows of one pass over the whole dialogue
+    hist = ([100, 256], [0, 1])
+    new = ([60, 200], [0, 1])
+    c, Ln, hq, hkv, d = 256, 200, 8, 2, 128
+    full = wl.pack([(hist[0] + [c + e for e in new[0]], hist[1] + new[1])])
+    w = wl.Workload("app", full, hq, hkv, d, "bf16", d ** -0.5, 0.5, 23)
+    q, k, v, _ = wl.attention_tensors(w)
+    o_full, _ = ism.fwd(ism.Segments.from_workload(full, DEV), q.to(DEV), k.to(DEV), v.to(DEV), w.softmax_scale)
+    cap = c + Ln
+    kc = torch.zeros((1, cap, hkv, d), dtype=torch.bfloat16)
+    vc = torch.zeros((1, cap, hkv, d), dtype=torch.bfloat16)
+    kc[0, :c], vc[0, :c] = k[:c], v[:c]
+    cl = torch.tensor([c], dtype=torch.int32, device=DEV)
+    o_app, _ = ism.prefill_append(q[None, c:].contiguous().to(DEV), k[None, c:].contiguous().to(DEV),
+                                  v[None, c:].contiguous().to(DEV), kc.to(DEV), vc.to(DEV), cl, np.array([c]),
+                                  new[0], new[1], w.softmax_scale)
+    diff = (o_app[0].float() - o_full[c:].float()).abs().max().item()
+    assert diff <= 2e-2, diff
+
+
+def test_decode_steps_small(ism):
+    B, hq, hkv, d, c0, steps = 2, 8, 2, 128, 700, 6
+    cap = c0 + steps
+    kc, vc, qn, kn, vn = _append_inputs(B, cap, None, steps, hq, hkv, d, seed=31)
+    kcd, vcd = kc.clone().to(DEV), vc.clone().to(DEV)
+    c_start = np.array([c0, c0 - 123], dtype=np.int32)
+    c_host = c_start.copy()
+    cl = torch.from_numpy(c_host.copy()).to(DEV)
+    scale = d ** -0.5
+    for t in range(steps):
+        o, lse = ism.prefill_append(qn[:, t:t + 1].contiguous().to(DEV), kn[:, t:t + 1].contiguous().to(DEV),
+                                    vn[:, t:t + 1].contiguous().to(DEV), kcd, vcd, cl, c_host, [1], [1], scale)
+        # the cache the oracle sees: the initial one plus the tokens of the earlier steps
+        kc_now, vc_now = kc.clone(), vc.clone()
+        for b in range(B):
+            kc_now[b, c_start[b]:c_start[b] + t] = kn[b, :t]
+            vc_now[b, c_start[b]:c_start[b] + t] = vn[b, :t]
+        o_ref, lse_ref = orc.prefill_append(qn[:, t:t + 1], kn[:, t:t + 1], vn[:, t:t + 1], kc_now, vc_now,
+                                            c_host, [1], [1], scale)
+        _cmp(f"decode o step {t}", o, o_ref, "bf16")
+        _cmp_lse(f"decode lse step {t}", lse, np.transpose(lse_ref, (1, 0, 2)), "bf16")
+        c_host = c_host + 1
+    ism.check_status()
+    assert cl.cpu().numpy().tolist() == c_host.tolist()
+
+
+def test_append_16k_prefill_and_decode(ism):
+    """Cache of 16384 tokens (batch 8, 32/8 heads, d 128), a new 512-token
+    query segment, then 256 answer decode steps; the oracle checks one
+    (sequence, KV group) for the prefill and for a sample of decode steps."""
+    a = wl.append_16k()
+    B, cap, hq, hkv, d = a.batch, a.capacity, a.num_heads_q, a.num_heads_kv, a.head_dim
+    rng = np.random.Generator(np.random.PCG64(a.seed))
+    kcd = torch.empty((B, cap, hkv, d), dtype=torch.bfloat16, device=DEV)
+    vcd = torch.empty_like(kcd)
+    b, g = 5, 3
+    hs = list(range(g * hq // hkv, (g + 1) * hq // hkv))
+    for bb in range(B):  # generate per sequence to bound host memory
+        kh = wl.round_to(wl.normal(rng, (cap, hkv, d), a.value_std), "bf16")
+        vh = wl.round_to(wl.normal(rng, (cap, hkv, d), a.value_std), "bf16")
+        kcd[bb], vcd[bb] = kh.to(DEV), vh.to(DEV)
+        if bb == b:  # the oracle's own copy of the checked (sequence, KV head) cache
+            kb = kh[:, g:g + 1].clone()
+            vb = vh[:, g:g + 1].clone()
+    qn = wl.round_to(wl.normal(rng, (B, a.l_new, hq, d), a.value_std), "bf16")
+    kn = wl.round_to(wl.normal(rng, (B, a.l_new, hkv, d), a.value_std), "bf16")
+    vn = wl.round_to(wl.normal(rng, (B, a.l_new, hkv, d), a.value_std), "bf16")
+    c_host = a.cache_len.copy()
+    cl = torch.from_numpy(c_host.copy()).to(DEV)
+    o, lse = ism.prefill_append(qn.to(DEV), kn.to(DEV), vn.to(DEV), kcd, vcd, cl, c_host, a.new_seg_end,
+                                a.new_seg_type, a.softmax_scale)
+    ism.check_status()
+    o_ref, lse_ref = orc.prefill_append(qn[b:b + 1, :, hs], kn[b:b + 1, :, g:g + 1], vn[b:b + 1, :, g:g + 1],
+                                        kb[None], vb[None], c_host[b:b + 1], a.new_seg_end, a.new_seg_type,
+                                        a.softmax_scale)
+    c = int(c_host[b])
+    kb[c:c + a.l_new] = kn[b, :, g:g + 1]
+    vb[c:c + a.l_new] = vn[b, :, g:g + 1]
+    _cmp("prefill o", o[b:b + 1, :, hs], o_ref, "bf16")
+    _cmp_lse("prefill lse", lse[hs][:, b:b + 1], np.transpose(lse_ref, (1, 0, 2)), "bf16")
+    c_host = c_host + a.l_new
+    check = {0, 1, 127, a.decode_steps - 1}
+    for t in range(a.decode_steps):
+        qd = wl.round_to(wl.normal(rng, (B, 1, hq, d), a.value_std), "bf16")
+        kd = wl.round_to(wl.normal(rng, (B, 1, hkv, d), a.value_std), "bf16")
+        vd = wl.round_to(wl.normal(rng, (B, 1, hkv, d), a.value_std), "bf16")
+        o, lse = ism.prefill_append(qd.to(DEV), kd.to(DEV), vd.to(DEV), kcd, vcd, cl, c_host, [1], [1],
+                                    a.softmax_scale)
+        c = int(c_host[b])
+        if t in check:
+            o_ref, lse_ref = orc.prefill_append(qd[b:b + 1, :, hs], kd[b:b + 1, :, g:g + 1], vd[b:b + 1, :, g:g + 1],
+                                                kb[None], vb[None], np.array([c]), [1], [1], a.softmax_scale)
+            _cmp(f"decode o step {t}", o[b:b + 1, :, hs], o_ref, "bf16")
+            _cmp_lse(f"decode lse step {t}", lse[hs][:, b:b + 1], np.transpose(lse_ref, (1, 0, 2)), "bf16")
+        kb[c] = kd[b, 0, g:g + 1]
+        vb[c] = vd[b, 0, g:g + 1]
+        c_host = c_host + 1
+    ism.check_status()
+    assert cl.cpu().numpy().tolist() == c_host.tolist()
