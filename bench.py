@@ -241,6 +241,8 @@ def run_cuda(args, w):
             flush.fill_(1)  # evict L2 between timed steps (outside the step's events)
             ev = {n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for n in kinds}
             for n, kid in kinds.items():
+                for e in ev[n]:
+                    e.record(stream)  # creates the event; the library re-records it around its launch
                 ism.set_kernel_timer(kid, *ev[n])
             s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             s0.record(stream)

@@ -214,6 +214,14 @@ enum {
 ism_status_t ism_set_kernel_timer(int32_t kernel_id, void* start_event, void* stop_event);
 uint64_t ism_kernel_launches(void);
 
+/* Diagnostic of the tensor-core building blocks (no counterpart in the
+ * paper): one 128x128x128 bf16 tile product on tcgen05 with fp32 result.
+ *   a [128,128] bf16 row-major (M x K); c [128,128] fp32 row-major (written)
+ *   mode 0/2: b [128,128] is N x K and c = a * b^T
+ *   mode 1/3: b [128,128] is K x N and c = a * b
+ *   modes 0/1 stage the operands with plain stores, 2/3 with TMA. */
+ism_status_t ism_debug_mma_tile(const void* a, const void* b, float* c, int32_t mode, ism_stream_t stream);
+
 const char* ism_status_string(ism_status_t status);
 /* Human-readable detail of the last failing call on this host thread. */
 const char* ism_last_error(void);

@@ -197,6 +197,7 @@ bool force_cuda_cores() {
 bool use_tc(const ism_attn_shape_t* sh) {
   return sh->dtype == ISM_BF16 && sh->head_dim == 128 && tc_available() && !force_cuda_cores();
 }
+bool use_tc_bwd(const ism_attn_shape_t* sh) { return use_tc(sh) && tc_bwd_available(); }
 
 ism_status_t check_ws(void* ws, size_t have, size_t need) {
   if (have < need) return fail(ISM_ERR_WORKSPACE, "workspace of %zu bytes, %zu required", have, need);
@@ -385,7 +386,7 @@ ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order; a.nq = c.nq;
   a.ktiles = L.ktiles; a.k_order = L.k_order; a.nk = c.nk;
   a.status = status;
-  if (use_tc(shape)) {
+  if (use_tc_bwd(shape)) {
     ISM_TRY_CUDA(launch_tc_bwd(a, info.total_tokens, st), "tensor-core backward launch");
   } else {
     ISM_TRY_CUDA(launch_simt_bwd(a, st), "backward launch");
@@ -550,6 +551,17 @@ ism_status_t ism_check_status(ism_stream_t stream) {
     ISM_TRY_CUDA(cudaMemcpy(status, &zero, sizeof(zero), cudaMemcpyHostToDevice), "status clear");
   }
   if (word & kStatusTimeout) return fail(ISM_ERR_TIMEOUT, "a device-side wait gave up (status word 0x%x)", word);
+  return ISM_OK;
+}
+
+ism_status_t ism_debug_mma_tile(const void* a, const void* b, float* c, int32_t mode, ism_stream_t stream) {
+  if (!a || !b || !c || mode < 0 || mode > 3) return fail(ISM_ERR_INVALID_ARG, "a, b, c non-NULL and mode 0..3");
+  if (!tc_available()) return fail(ISM_ERR_UNSUPPORTED, "tensor-core kernels need an sm_103 device");
+  uint32_t* status;
+  ism_status_t r = status_ptr(&status);
+  if (r != ISM_OK) return r;
+  ISM_TRY_CUDA(launch_tc_mma_tile(a, b, c, mode, status, reinterpret_cast<cudaStream_t>(stream)), "mma tile launch");
+  count_launch(1);
   return ISM_OK;
 }
 

@@ -112,6 +112,8 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st);
 
 // Tensor-core kernels (ism_fwd_tc.cu / ism_bwd_tc.cu), bf16 only.
 bool tc_available();
+bool tc_bwd_available();
+cudaError_t launch_tc_mma_tile(const void* a, const void* b, float* c, int mode, uint32_t* status, cudaStream_t st);
 cudaError_t launch_tc_fwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st);
 cudaError_t launch_tc_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st);
 

@@ -1,0 +1,83 @@
+// Shared pieces of the sm_103a tensor-core kernels: tile geometry, TMA
+// tensor maps, bounded waits with a wall-clock limit, and the 128B-swizzled
+// shared-memory layout the TMA writes and tcgen05.mma reads.
+#pragma once
+
+#include <cuda.h>
+
+#include "ism_internal.cuh"
+#include "ptx.cuh"
+
+namespace ism {
+namespace tc {
+
+constexpr int kD = 128;                       // head dim handled by the tensor-core kernels
+constexpr int kRows = 128;                    // rows of a Q / K / V / P tile
+constexpr uint32_t kHalfBytes = 128u * 128u;  // one 64-column half of a tile: 128 rows x 128 B
+constexpr uint32_t kTileBytes = 2u * kHalfBytes;
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+// A device-side wait gives up after this long (ns of %globaltimer).
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Bounded mbarrier wait; on giving up records the timeout in the status word.
+__device__ __forceinline__ bool wait(uint64_t* bar, uint32_t parity, uint32_t* status) {
+  if (ptx::mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 64; ++i)
+      if (ptx::mbar_try_wait(bar, parity)) return true;
+    if (globaltimer() - t0 > kWaitLimitNs) {
+      atomicOr(status, kStatusTimeout);
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// Byte offset of element (r, c) of a [128 x 128] bf16 tile in the layout a
+// 128B-swizzled TMA box of 64 columns x 128 rows produces (two such boxes,
+// one per 64-column half): 16-byte chunk index XOR (row mod 8).
+__host__ __device__ __forceinline__ uint32_t swz_offset(uint32_t r, uint32_t c) {
+  return (c >> 6) * kHalfBytes + r * 128u + ((((c & 63u) >> 3) ^ (r & 7u)) << 4) + (c & 7u) * 2u;
+}
+
+// Descriptor of k-step kk (16 elements of K) of a K-major tile (rows = M or
+// N, 128 K columns in two 64-column swizzled halves).
+__device__ __forceinline__ uint64_t desc_kmajor(uint32_t tile_saddr, int kk) {
+  return ptx::smem_desc(tile_saddr + (uint32_t)(kk >> 2) * kHalfBytes + (uint32_t)(kk & 3) * 32u, 16u, 1024u,
+                        ptx::kSwizzle128B);
+}
+
+// Descriptor of k-step kk (16 rows of K) of an MN-major tile stored as
+// [128 K rows x 128 N columns] (two 64-column swizzled halves): 8-row groups
+// are 1024 B apart (stride offset), the halves 16 KB apart (leading offset).
+__device__ __forceinline__ uint64_t desc_mnmajor(uint32_t tile_saddr, int kk) {
+  return ptx::smem_desc(tile_saddr + (uint32_t)kk * 2048u, kHalfBytes, 1024u, ptx::kSwizzle128B);
+}
+
+// Host: 2D bf16 tensor map [rows, cols] with a 64 x 128 box, 128B swizzle.
+cudaError_t make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows);
+
+}  // namespace tc
+}  // namespace ism

@@ -63,6 +63,7 @@ EXPORTS = {
     "ism_has_tensor_cores": (C.c_int32, []),
     "ism_set_kernel_timer": (C.c_int, [C.c_int32, C.c_void_p, C.c_void_p]),
     "ism_kernel_launches": (C.c_uint64, []),
+    "ism_debug_mma_tile": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p]),
 }
 
 KERNEL_FWD, KERNEL_BWD_DKDV, KERNEL_BWD_DQ, KERNEL_BWD_PRE, KERNEL_DECODE, KERNEL_META = 1, 2, 3, 4, 5, 6
@@ -291,3 +292,11 @@ def set_kernel_timer(kernel_id: int, start: "torch.cuda.Event" = None, stop: "to
 
 def kernel_launches() -> int:
     return int(load().ism_kernel_launches())
+
+
+def debug_mma_tile(a: torch.Tensor, b: torch.Tensor, mode: int) -> torch.Tensor:
+    """One 128x128x128 tcgen05 tile product (diagnostic): mode 0/2 a @ b.T,
+    mode 1/3 a @ b; modes 2/3 stage operands with TMA."""
+    c = torch.empty((128, 128), dtype=torch.float32, device=a.device)
+    _check(load().ism_debug_mma_tile(_ptr(a), _ptr(b), _ptr(c), mode, _stream(a.device)), "ism_debug_mma_tile")
+    return c

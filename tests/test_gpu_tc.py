@@ -1,0 +1,30 @@
+"""Tensor-core building blocks on the GPU: one 128x128x128 tcgen05 tile
+product (shared-memory descriptors, instruction descriptor, TMEM loads, TMA
+swizzle) against a float64 product of the same bf16 values."""
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def ism():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2408_00539_gb300 import ism as m
+    m.load(build_if_missing=True)
+    if not m.has_tensor_cores():
+        pytest.skip("tensor-core kernels need sm_103")
+    return m
+
+
+@pytest.mark.parametrize("mode", [0, 1, 2, 3])
+def test_mma_tile(ism, mode):
+    g = torch.Generator().manual_seed(100 + mode)
+    a = torch.randn(128, 128, generator=g).to(torch.bfloat16)
+    b = torch.randn(128, 128, generator=g).to(torch.bfloat16)
+    c = ism.debug_mma_tile(a.cuda(), b.cuda(), mode)
+    ism.check_status()
+    ref = a.double() @ (b.double().T if mode in (0, 2) else b.double())
+    err = (c.double().cpu() - ref).abs().max().item()
+    assert err < 1e-3, f"mode {mode}: max abs err {err}"
