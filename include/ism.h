@@ -133,6 +133,28 @@ ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
                           const void* q, const void* k, const void* v, void* o, float* lse,
                           void* workspace, size_t workspace_bytes, ism_stream_t stream);
 
+/* Forward without a caller-provided workspace (the paper has no counterpart;
+ * this is a deployment convenience).  Some callers cannot allocate device
+ * memory at the point where they run attention: code recorded into a CUDA
+ * graph (allocation during capture is not allowed), servers that reserve all
+ * device memory once at start-up and never grow it, or plain C hosts with no
+ * device allocator of their own.  This variant takes the forward's scratch
+ * from a fixed array of ism_attn_fwd_noalloc_max_workspace() bytes (4 MiB)
+ * that the library keeps in device memory on every GPU that loads it, until
+ * the process exits.  It calls no allocator.
+ *  - Same arguments and results as ism_attn_fwd, minus the workspace.
+ *  - Batches whose forward workspace (ism_attn_fwd_workspace_size) exceeds
+ *    the array return ISM_ERR_WORKSPACE before anything is launched.
+ *  - The first call on a device looks the array's device address up
+ *    (cudaGetSymbolAddress) with that device current; make that first call
+ *    before any stream capture.
+ *  - All calls share the one array: calls whose kernels may overlap on the
+ *    GPU (different streams without ordering) race on it. */
+size_t ism_attn_fwd_noalloc_max_workspace(void);
+ism_status_t ism_attn_fwd_noalloc(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                                  const void* q, const void* k, const void* v, void* o, float* lse,
+                                  ism_stream_t stream);
+
 /* ---------------------------------------------------------------------------
  * Backward: gradients of sum(O * dO) with respect to Q, K, V, given the
  * forward's O and LSE.  dq [T, Hq, D], dk/dv [T, Hkv, D] (dtype, written;

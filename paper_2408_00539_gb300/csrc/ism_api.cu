@@ -230,6 +230,7 @@ void timer_end(int id, cudaStream_t st) {
   if (id > 0 && id < kTimerSlots && g_timer_stop[id]) cudaEventRecord(g_timer_stop[id], st);
 }
 void count_launch(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+void set_error(const char* msg) { g_last_error = msg; }
 
 }  // namespace ism
 

@@ -124,5 +124,7 @@ cudaError_t launch_timeout_probe(uint32_t spin_limit, uint32_t* status, cudaStre
 void timer_begin(int kernel_id, cudaStream_t st);
 void timer_end(int kernel_id, cudaStream_t st);
 void count_launch(int n = 1);
+// Sets the message returned by ism_last_error() on this host thread.
+void set_error(const char* msg);
 
 }  // namespace ism

@@ -64,6 +64,8 @@ EXPORTS = {
     "ism_set_kernel_timer": (C.c_int, [C.c_int32, C.c_void_p, C.c_void_p]),
     "ism_kernel_launches": (C.c_uint64, []),
     "ism_debug_mma_tile": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p]),
+    "ism_attn_fwd_noalloc_max_workspace": (C.c_size_t, []),
+    "ism_attn_fwd_noalloc": (C.c_int, [C.c_void_p] * 8),
 }
 
 KERNEL_FWD, KERNEL_BWD_DKDV, KERNEL_BWD_DQ, KERNEL_BWD_PRE, KERNEL_DECODE, KERNEL_META = 1, 2, 3, 4, 5, 6
