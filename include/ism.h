@@ -239,9 +239,10 @@ uint64_t ism_kernel_launches(void);
 /* Diagnostic of the tensor-core building blocks (no counterpart in the
  * paper): one 128x128x128 bf16 tile product on tcgen05 with fp32 result.
  *   a [128,128] bf16 row-major (M x K); c [128,128] fp32 row-major (written)
- *   mode 0/2: b [128,128] is N x K and c = a * b^T
- *   mode 1/3: b [128,128] is K x N and c = a * b
- *   modes 0/1 stage the operands with plain stores, 2/3 with TMA. */
+ *   mode 0/2/4: b [128,128] is N x K and c = a * b^T
+ *   mode 1/3/5: b [128,128] is K x N and c = a * b
+ *   modes 0/1 stage the operands with plain stores, 2/3 with TMA, 4/5 put
+ *   a in tensor memory (the A-from-TMEM form of the MMA). */
 ism_status_t ism_debug_mma_tile(const void* a, const void* b, float* c, int32_t mode, ism_stream_t stream);
 
 const char* ism_status_string(ism_status_t status);

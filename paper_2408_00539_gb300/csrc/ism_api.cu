@@ -552,11 +552,13 @@ ism_status_t ism_check_status(ism_stream_t stream) {
     ISM_TRY_CUDA(cudaMemcpy(status, &zero, sizeof(zero), cudaMemcpyHostToDevice), "status clear");
   }
   if (word & kStatusTimeout) return fail(ISM_ERR_TIMEOUT, "a device-side wait gave up (status word 0x%x)", word);
+  if (word & kStatusSmemAlign)
+    return fail(ISM_ERR_CUDA, "a kernel found its shared memory misaligned and skipped its work (0x%x)", word);
   return ISM_OK;
 }
 
 ism_status_t ism_debug_mma_tile(const void* a, const void* b, float* c, int32_t mode, ism_stream_t stream) {
-  if (!a || !b || !c || mode < 0 || mode > 3) return fail(ISM_ERR_INVALID_ARG, "a, b, c non-NULL and mode 0..3");
+  if (!a || !b || !c || mode < 0 || mode > 5) return fail(ISM_ERR_INVALID_ARG, "a, b, c non-NULL and mode 0..5");
   if (!tc_available()) return fail(ISM_ERR_UNSUPPORTED, "tensor-core kernels need an sm_103 device");
   uint32_t* status;
   ism_status_t r = status_ptr(&status);

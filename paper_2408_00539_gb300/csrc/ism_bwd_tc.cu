@@ -1,0 +1,643 @@
+// ISM attention backward on sm_103a tensor cores: the standard softmax
+// attention gradients over the Eq. (e_ISM) mask, with P recomputed from the
+// forward's log-sum-exp.
+//
+//   delta_kernel   Delta_j = sum_d dO_jd O_jd                      (HBM-bound)
+//   dq_kernel      per (query tile, query head), over the tile's non-empty
+//                  key blocks: S = Q K^T, dP = dO V^T (TMEM), dS = P (dP - Delta)
+//                  to shared memory, dQ += dS K (TMEM); dQ = scale * dQ.
+//   dkdv_kernel    per (key tile, KV head), over the query heads of the group
+//                  and the query tiles that see the key tile: S^T = K Q^T and
+//                  dP^T = V dO^T (TMEM), P^T back into TMEM (A operand of the
+//                  next MMA), dS^T to shared memory, dV += P^T dO, dK += dS^T Q
+//                  (TMEM accumulators); dK = scale * dK.
+// Warp roles in both MMA kernels: warps 0..7 compute (two warpgroups, each
+// owning 64 of the 128 columns of a tile; thread = TMEM lane = tile row),
+// warp 8 loads (TMA), warp 9 owns TMEM and issues the MMAs.
+#include "ism_tc_common.cuh"
+
+namespace ism {
+namespace tc {
+namespace {
+
+constexpr int kThreads = 320;
+constexpr int kComputeThreads = 256;
+constexpr uint32_t kTmemCols = 512;
+
+__device__ __forceinline__ bool aborted(const int32_t* f) { return *reinterpret_cast<const volatile int32_t*>(f) != 0; }
+__device__ __forceinline__ void set_abort(int32_t* f) { *reinterpret_cast<volatile int32_t*>(f) = 1; }
+
+__device__ __forceinline__ void ld64(uint32_t taddr, uint32_t (&a)[32], uint32_t (&b)[32]) {
+  ptx::tmem_ld32(taddr, a);
+  ptx::tmem_ld32(taddr + 32, b);
+}
+
+// Writes 64 bf16 values (32 packed words) as row r, half `half` of a
+// 128B-swizzled [128 x 128] tile.
+__device__ __forceinline__ void store_row_half(uint8_t* tile, int r, int half, const uint32_t (&pk)[32]) {
+  uint8_t* row = tile + half * kHalfBytes + r * 128;
+#pragma unroll
+  for (int c = 0; c < 8; ++c)
+    *reinterpret_cast<uint4*>(row + ((c ^ (r & 7)) << 4)) =
+        make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+}
+
+// ------------------------------------------------------------------ delta
+// One 16-lane group per (row, head): 8 bf16 per lane, D = 128.
+__global__ void delta_kernel(const __nv_bfloat16* __restrict__ O, const __nv_bfloat16* __restrict__ dO,
+                             float* __restrict__ delta, int64_t rows, int hq) {
+  const int64_t n = rows * hq;
+  const int sub = threadIdx.x & 15;
+  for (int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 4; i < n;
+       i += ((int64_t)gridDim.x * blockDim.x) >> 4) {
+    const uint4 a = reinterpret_cast<const uint4*>(O + i * kD)[sub];
+    const uint4 b = reinterpret_cast<const uint4*>(dO + i * kD)[sub];
+    const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&a);
+    const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&b);
+    float acc = 0.f;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 x = __bfloat1622float2(pa[k]), y = __bfloat1622float2(pb[k]);
+      acc = fmaf(x.x, y.x, fmaf(x.y, y.y, acc));
+    }
+#pragma unroll
+    for (int o = 8; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (sub == 0) {
+      const int64_t row = i / hq;
+      const int h = (int)(i % hq);
+      delta[(int64_t)h * rows + row] = acc;
+    }
+  }
+}
+
+// ------------------------------------------------------------------ dQ
+namespace dq {
+constexpr uint32_t OFF_Q = 0, OFF_DO = kTileBytes, OFF_K = 2 * kTileBytes, OFF_V = 4 * kTileBytes,
+                   OFF_DS = 6 * kTileBytes, OFF_BAR = 7 * kTileBytes;
+constexpr uint32_t kSmemBytes = OFF_BAR + 256 + 1024;
+constexpr uint32_t TM_S = 0, TM_DP = 128, TM_DQ = 256;
+
+struct Bars {
+  uint64_t qdo_full;
+  uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
+  uint64_t s_full, dp_full, sdp_free, p_full, dq_done, final_mma;
+  uint32_t tmem_base;
+  int32_t abort;
+};
+}  // namespace dq
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    dq_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmdO,
+              const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
+  using namespace dq;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  Bars* bar = reinterpret_cast<Bars*>(smem + OFF_BAR);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.x % a.hq;
+  const Tile w = a.qtiles[a.q_order[blockIdx.x / a.hq]];
+  const int g = h / (a.hq / a.hkv);
+  const int nkb = w.a1, kfull = w.a0;
+
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(&bar->qdo_full, 1);
+    for (int s = 0; s < 2; ++s) {
+      ptx::mbar_init(&bar->k_full[s], 1);
+      ptx::mbar_init(&bar->k_empty[s], 1);
+      ptx::mbar_init(&bar->v_full[s], 1);
+      ptx::mbar_init(&bar->v_empty[s], 1);
+    }
+    ptx::mbar_init(&bar->s_full, 1);
+    ptx::mbar_init(&bar->dp_full, 1);
+    ptx::mbar_init(&bar->sdp_free, kComputeThreads);
+    ptx::mbar_init(&bar->p_full, kComputeThreads);
+    ptx::mbar_init(&bar->dq_done, 1);
+    ptx::mbar_init(&bar->final_mma, 1);
+    bar->abort = 0;
+    ptx::fence_mbar_init();
+  }
+  if (warp == 9) {
+    ptx::tmem_alloc(&bar->tmem_base, kTmemCols);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = bar->tmem_base;
+
+  if (warp == 8) {
+    if (lane == 0 && nkb > 0) {
+      ptx::tma_prefetch_desc(&tmK);
+      ptx::tma_prefetch_desc(&tmV);
+      const int32_t qy = w.q_base + w.tile * kRows;
+      ptx::mbar_expect_tx(&bar->qdo_full, 2 * kTileBytes);
+      ptx::tma_load_2d(smem + OFF_Q, &tmQ, &bar->qdo_full, h * kD, qy);
+      ptx::tma_load_2d(smem + OFF_Q + kHalfBytes, &tmQ, &bar->qdo_full, h * kD + 64, qy);
+      ptx::tma_load_2d(smem + OFF_DO, &tmdO, &bar->qdo_full, h * kD, qy);
+      ptx::tma_load_2d(smem + OFF_DO + kHalfBytes, &tmdO, &bar->qdo_full, h * kD + 64, qy);
+      uint32_t nk[2] = {0, 0}, nv[2] = {0, 0};
+      for (int c = 0; c < nkb; ++c) {
+        const int s = c & 1;
+        const uint32_t n = (uint32_t)(c >> 1);
+        if (aborted(&bar->abort)) break;
+        const int32_t ky = w.k_base + c * kRows;
+        if (c >= 2 && !wait(&bar->k_empty[s], (n - 1) & 1, a.status)) { set_abort(&bar->abort); break; }
+        ptx::mbar_expect_tx(&bar->k_full[s], kTileBytes);
+        ptx::tma_load_2d(smem + OFF_K + s * kTileBytes, &tmK, &bar->k_full[s], g * kD, ky);
+        ptx::tma_load_2d(smem + OFF_K + s * kTileBytes + kHalfBytes, &tmK, &bar->k_full[s], g * kD + 64, ky);
+        ++nk[s];
+        if (c >= 2 && !wait(&bar->v_empty[s], (n - 1) & 1, a.status)) { set_abort(&bar->abort); break; }
+        ptx::mbar_expect_tx(&bar->v_full[s], kTileBytes);
+        ptx::tma_load_2d(smem + OFF_V + s * kTileBytes, &tmV, &bar->v_full[s], g * kD, ky);
+        ptx::tma_load_2d(smem + OFF_V + s * kTileBytes + kHalfBytes, &tmV, &bar->v_full[s], g * kD + 64, ky);
+        ++nv[s];
+      }
+      if (aborted(&bar->abort)) {
+        wait(&bar->qdo_full, 0, a.status);
+        for (int s = 0; s < 2; ++s) {
+          if (nk[s]) wait(&bar->k_full[s], (nk[s] - 1) & 1, a.status);
+          if (nv[s]) wait(&bar->v_full[s], (nv[s] - 1) & 1, a.status);
+        }
+      }
+    }
+  } else if (warp == 9) {
+    if (lane == 0 && nkb > 0) {
+      constexpr uint32_t idesc_nt = ptx::idesc_bf16_f32(128, 128, 0, 0);  // A K-major, B K-major
+      constexpr uint32_t idesc_nn = ptx::idesc_bf16_f32(128, 128, 0, 1);  // A K-major, B MN-major
+      const uint32_t sQ = ptx::smem_u32(smem + OFF_Q), sdO = ptx::smem_u32(smem + OFF_DO);
+      const uint32_t sdS = ptx::smem_u32(smem + OFF_DS);
+      bool ok = wait(&bar->qdo_full, 0, a.status);
+      auto issue_sdp = [&](int c) -> bool {
+        const int s = c & 1;
+        const uint32_t n = (uint32_t)(c >> 1);
+        if (!wait(&bar->k_full[s], n & 1, a.status)) return false;
+        ptx::tc_fence_after();
+        const uint32_t sK = ptx::smem_u32(smem + OFF_K + s * kTileBytes);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          ptx::mma_bf16_ss(tmem + TM_S, desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_nt, kk > 0 ? 1u : 0u);
+        ptx::mma_commit(&bar->s_full);
+        if (!wait(&bar->v_full[s], n & 1, a.status)) return false;
+        ptx::tc_fence_after();
+        const uint32_t sV = ptx::smem_u32(smem + OFF_V + s * kTileBytes);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          ptx::mma_bf16_ss(tmem + TM_DP, desc_kmajor(sdO, kk), desc_kmajor(sV, kk), idesc_nt, kk > 0 ? 1u : 0u);
+        ptx::mma_commit(&bar->dp_full);
+        ptx::mma_commit(&bar->v_empty[s]);
+        return true;
+      };
+      if (ok) ok = issue_sdp(0);
+      for (int c = 0; ok && c < nkb; ++c) {
+        if (aborted(&bar->abort)) { ok = false; break; }
+        if (c + 1 < nkb) {
+          if (!wait(&bar->sdp_free, (uint32_t)c & 1, a.status)) { ok = false; break; }
+          if (!issue_sdp(c + 1)) { ok = false; break; }
+        }
+        if (!wait(&bar->p_full, (uint32_t)c & 1, a.status)) { ok = false; break; }
+        ptx::tc_fence_after();
+        const uint32_t sK = ptx::smem_u32(smem + OFF_K + (c & 1) * kTileBytes);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          ptx::mma_bf16_ss(tmem + TM_DQ, desc_kmajor(sdS, kk), desc_mnmajor(sK, kk), idesc_nn,
+                           (c > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma_commit(&bar->dq_done);
+        ptx::mma_commit(&bar->k_empty[c & 1]);
+      }
+      if (!ok) set_abort(&bar->abort);
+      ptx::mma_commit(&bar->final_mma);
+      wait(&bar->final_mma, 0, a.status);
+    }
+    __syncwarp();
+  } else {
+    // compute: thread = query row r of the tile; warpgroup wg owns key columns [64 wg, 64 wg + 64)
+    const int wg = threadIdx.x >> 7, r = threadIdx.x & 127;
+    const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
+    const int row = w.tile * kRows + r;
+    const bool valid = row < w.q_len;
+    const int64_t grow = (int64_t)w.q_base + row;
+    const int ke = valid ? a.kv_end[w.kv_base + row] : 0;
+    const float lse2 = valid ? a.lse_in[(int64_t)h * a.q_rows + grow] * kLog2e : 0.f;
+    const float dl = valid ? a.delta[(int64_t)h * a.q_rows + grow] : 0.f;
+    const float sl2 = a.scale * kLog2e;
+    bool ok = nkb > 0;
+    for (int c = 0; ok && c < nkb; ++c) {
+      if (!wait(&bar->s_full, (uint32_t)c & 1, a.status) || !wait(&bar->dp_full, (uint32_t)c & 1, a.status)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+      uint32_t s0[32], s1[32], d0[32], d1[32];
+      ld64(tmem + lane_addr + TM_S + wg * 64, s0, s1);
+      ld64(tmem + lane_addr + TM_DP + wg * 64, d0, d1);
+      ptx::tmem_ld_wait();
+      ptx::reg_fence(s0);
+      ptx::reg_fence(s1);
+      ptx::reg_fence(d0);
+      ptx::reg_fence(d1);
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&bar->sdp_free);
+      const int lim = (c < kfull) ? 128 : ke - c * kRows - wg * 64;  // visible columns of this half
+      uint32_t pk[32];  // pk[k] holds columns 2k and 2k+1 of this half
+#pragma unroll
+      for (int k = 0; k < 32; ++k) {
+        float v[2];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int jj = 2 * k + e;
+          const float sv = __uint_as_float(jj < 32 ? s0[jj] : s1[jj - 32]);
+          const float dv = __uint_as_float(jj < 32 ? d0[jj] : d1[jj - 32]);
+          const float p = jj < lim ? ex2(sv * sl2 - lse2) : 0.f;
+          v[e] = p * (dv - dl);
+        }
+        pk[k] = pack_bf16(v[0], v[1]);
+      }
+      if (c >= 1 && !wait(&bar->dq_done, (uint32_t)(c - 1) & 1, a.status)) { ok = false; break; }
+      store_row_half(smem + OFF_DS, r, wg, pk);
+      ptx::fence_proxy_async_smem();
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&bar->p_full);
+    }
+    if (ok) ok = wait(&bar->dq_done, (uint32_t)(nkb - 1) & 1, a.status);
+    if (!ok) {
+      set_abort(&bar->abort);
+    } else {
+      ptx::tc_fence_after();
+      uint32_t q0[32], q1[32];
+      ld64(tmem + lane_addr + TM_DQ + wg * 64, q0, q1);
+      ptx::tmem_ld_wait();
+      ptx::reg_fence(q0);
+      ptx::reg_fence(q1);
+      if (valid) {
+        uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) + grow * a.hq * kD + h * kD +
+                                              wg * 64);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          uint4 v;
+          v.x = pack_bf16(__uint_as_float(q0[8 * i + 0]) * a.scale, __uint_as_float(q0[8 * i + 1]) * a.scale);
+          v.y = pack_bf16(__uint_as_float(q0[8 * i + 2]) * a.scale, __uint_as_float(q0[8 * i + 3]) * a.scale);
+          v.z = pack_bf16(__uint_as_float(q0[8 * i + 4]) * a.scale, __uint_as_float(q0[8 * i + 5]) * a.scale);
+          v.w = pack_bf16(__uint_as_float(q0[8 * i + 6]) * a.scale, __uint_as_float(q0[8 * i + 7]) * a.scale);
+          dst[i] = v;
+          v.x = pack_bf16(__uint_as_float(q1[8 * i + 0]) * a.scale, __uint_as_float(q1[8 * i + 1]) * a.scale);
+          v.y = pack_bf16(__uint_as_float(q1[8 * i + 2]) * a.scale, __uint_as_float(q1[8 * i + 3]) * a.scale);
+          v.z = pack_bf16(__uint_as_float(q1[8 * i + 4]) * a.scale, __uint_as_float(q1[8 * i + 5]) * a.scale);
+          v.w = pack_bf16(__uint_as_float(q1[8 * i + 6]) * a.scale, __uint_as_float(q1[8 * i + 7]) * a.scale);
+          dst[4 + i] = v;
+        }
+      }
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 9) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------ dK / dV
+namespace dkv {
+constexpr uint32_t OFF_K = 0, OFF_V = kTileBytes, OFF_Q = 2 * kTileBytes, OFF_DO = 4 * kTileBytes,
+                   OFF_DS = 6 * kTileBytes, OFF_META = 7 * kTileBytes;
+// per stage: lse2[128] f32, delta[128] f32, visible-key count[128] u8
+constexpr uint32_t kMetaStage = 128 * 4 + 128 * 4 + 128;
+constexpr uint32_t OFF_BAR = OFF_META + 2 * kMetaStage;
+constexpr uint32_t kSmemBytes = OFF_BAR + 256;  // needs a 1024-aligned dynamic shared base
+constexpr uint32_t TM_S = 0, TM_DP = 128, TM_DV = 256, TM_DK = 384;
+
+struct Bars {
+  uint64_t kv_full;
+  uint64_t q_full[2], q_empty[2], do_full[2], do_empty[2], meta_full[2], meta_empty[2];
+  uint64_t s_full, dp_full, s_free, p_full, dvk_done, final_mma;
+  uint32_t tmem_base;
+  int32_t abort;
+};
+}  // namespace dkv
+
+__global__ void __launch_bounds__(kThreads, 1)
+    dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmdO,
+                const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
+  using namespace dkv;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw;
+  Bars* bar = reinterpret_cast<Bars*>(smem + OFF_BAR);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (ptx::smem_u32(smem) & 1023u) {  // the swizzled tiles need 1024-byte alignment
+    if (threadIdx.x == 0) atomicOr(a.status, kStatusSmemAlign);
+    return;
+  }
+  const int g = blockIdx.x % a.hkv;
+  const Tile w = a.ktiles[a.k_order[blockIdx.x / a.hkv]];
+  const int group = a.hq / a.hkv;
+  const int qt0 = w.a0, nqt = w.a1;
+  const int per_head = nqt - qt0;
+  const int n_it = per_head > 0 ? per_head * group : 0;
+  const int c = w.tile;
+
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(&bar->kv_full, 1);
+    for (int s = 0; s < 2; ++s) {
+      ptx::mbar_init(&bar->q_full[s], 1);
+      ptx::mbar_init(&bar->q_empty[s], 1);
+      ptx::mbar_init(&bar->do_full[s], 1);
+      ptx::mbar_init(&bar->do_empty[s], 1);
+      ptx::mbar_init(&bar->meta_full[s], 32);
+      ptx::mbar_init(&bar->meta_empty[s], kComputeThreads);
+    }
+    ptx::mbar_init(&bar->s_full, 1);
+    ptx::mbar_init(&bar->dp_full, 1);
+    ptx::mbar_init(&bar->s_free, kComputeThreads);
+    ptx::mbar_init(&bar->p_full, kComputeThreads);
+    ptx::mbar_init(&bar->dvk_done, 1);
+    ptx::mbar_init(&bar->final_mma, 1);
+    bar->abort = 0;
+    ptx::fence_mbar_init();
+  }
+  if (warp == 9) {
+    ptx::tmem_alloc(&bar->tmem_base, kTmemCols);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = bar->tmem_base;
+
+  if (warp == 8) {
+    // ------------------------------------------------ loads (all 32 lanes fill the meta arrays)
+    uint32_t nq[2] = {0, 0}, ndo[2] = {0, 0};
+    const int32_t ky = w.k_base + c * kRows;
+    if (lane == 0 && n_it > 0) {
+      ptx::mbar_expect_tx(&bar->kv_full, 2 * kTileBytes);
+      ptx::tma_load_2d(smem + OFF_K, &tmK, &bar->kv_full, g * kD, ky);
+      ptx::tma_load_2d(smem + OFF_K + kHalfBytes, &tmK, &bar->kv_full, g * kD + 64, ky);
+      ptx::tma_load_2d(smem + OFF_V, &tmV, &bar->kv_full, g * kD, ky);
+      ptx::tma_load_2d(smem + OFF_V + kHalfBytes, &tmV, &bar->kv_full, g * kD + 64, ky);
+    }
+    for (int i = 0; i < n_it; ++i) {
+      const int s = i & 1;
+      const uint32_t n = (uint32_t)(i >> 1);
+      const int hh = i / per_head, t = qt0 + i % per_head;
+      const int h = g * group + hh;
+      const int32_t qy = w.q_base + t * kRows;
+      if (aborted(&bar->abort)) break;
+      if (lane == 0) {
+        bool ok = i < 2 || wait(&bar->q_empty[s], (n - 1) & 1, a.status);
+        if (ok) {
+          ptx::mbar_expect_tx(&bar->q_full[s], kTileBytes);
+          ptx::tma_load_2d(smem + OFF_Q + s * kTileBytes, &tmQ, &bar->q_full[s], h * kD, qy);
+          ptx::tma_load_2d(smem + OFF_Q + s * kTileBytes + kHalfBytes, &tmQ, &bar->q_full[s], h * kD + 64, qy);
+          ++nq[s];
+          ok = i < 2 || wait(&bar->do_empty[s], (n - 1) & 1, a.status);
+        }
+        if (ok) {
+          ptx::mbar_expect_tx(&bar->do_full[s], kTileBytes);
+          ptx::tma_load_2d(smem + OFF_DO + s * kTileBytes, &tmdO, &bar->do_full[s], h * kD, qy);
+          ptx::tma_load_2d(smem + OFF_DO + s * kTileBytes + kHalfBytes, &tmdO, &bar->do_full[s], h * kD + 64, qy);
+          ++ndo[s];
+        }
+        if (!ok) set_abort(&bar->abort);
+      }
+      __syncwarp();
+      if (aborted(&bar->abort)) break;
+      if (i >= 2 && !wait(&bar->meta_empty[s], (n - 1) & 1, a.status)) { set_abort(&bar->abort); break; }
+      uint8_t* meta = smem + OFF_META + s * kMetaStage;
+      float* mlse = reinterpret_cast<float*>(meta);
+      float* mdel = mlse + 128;
+      uint8_t* mlim = reinterpret_cast<uint8_t*>(mdel + 128);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int j = lane * 4 + e;
+        const int row = t * kRows + j;
+        const bool valid = row < w.q_len;
+        const int64_t grow = (int64_t)w.q_base + row;
+        mlse[j] = valid ? a.lse_in[(int64_t)h * a.q_rows + grow] * kLog2e : 0.f;
+        mdel[j] = valid ? a.delta[(int64_t)h * a.q_rows + grow] : 0.f;
+        const int vis = valid ? a.kv_end[w.kv_base + row] - c * kRows : 0;
+        mlim[j] = (uint8_t)(vis < 0 ? 0 : vis > 128 ? 128 : vis);
+      }
+      ptx::mbar_arrive(&bar->meta_full[s]);
+    }
+    if (lane == 0 && aborted(&bar->abort)) {
+      if (n_it > 0) wait(&bar->kv_full, 0, a.status);
+      for (int s = 0; s < 2; ++s) {
+        if (nq[s]) wait(&bar->q_full[s], (nq[s] - 1) & 1, a.status);
+        if (ndo[s]) wait(&bar->do_full[s], (ndo[s] - 1) & 1, a.status);
+      }
+    }
+  } else if (warp == 9) {
+    // ------------------------------------------------ MMA issue
+    if (lane == 0 && n_it > 0) {
+      constexpr uint32_t idesc_nt = ptx::idesc_bf16_f32(128, 128, 0, 0);
+      constexpr uint32_t idesc_nn = ptx::idesc_bf16_f32(128, 128, 0, 1);
+      const uint32_t sK = ptx::smem_u32(smem + OFF_K), sV = ptx::smem_u32(smem + OFF_V);
+      const uint32_t sdS = ptx::smem_u32(smem + OFF_DS);
+      bool ok = wait(&bar->kv_full, 0, a.status);
+      auto issue_s = [&](int i) -> bool {
+        const int s = i & 1;
+        if (!wait(&bar->q_full[s], (uint32_t)(i >> 1) & 1, a.status)) return false;
+        ptx::tc_fence_after();
+        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + s * kTileBytes);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          ptx::mma_bf16_ss(tmem + TM_S, desc_kmajor(sK, kk), desc_kmajor(sQ, kk), idesc_nt, kk > 0 ? 1u : 0u);
+        ptx::mma_commit(&bar->s_full);
+        return true;
+      };
+      auto issue_dp = [&](int i) -> bool {
+        const int s = i & 1;
+        if (!wait(&bar->do_full[s], (uint32_t)(i >> 1) & 1, a.status)) return false;
+        ptx::tc_fence_after();
+        const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + s * kTileBytes);
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          ptx::mma_bf16_ss(tmem + TM_DP, desc_kmajor(sV, kk), desc_kmajor(sdO, kk), idesc_nt, kk > 0 ? 1u : 0u);
+        ptx::mma_commit(&bar->dp_full);
+        return true;
+      };
+      if (ok) ok = issue_s(0) && issue_dp(0);
+      for (int i = 0; ok && i < n_it; ++i) {
+        const int s = i & 1;
+        if (aborted(&bar->abort)) { ok = false; break; }
+        if (i + 1 < n_it) {
+          if (!wait(&bar->s_free, (uint32_t)i & 1, a.status) || !issue_s(i + 1)) { ok = false; break; }
+        }
+        if (!wait(&bar->p_full, (uint32_t)i & 1, a.status)) { ok = false; break; }
+        ptx::tc_fence_after();
+        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + s * kTileBytes);
+        const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + s * kTileBytes);
+        // dV += P^T dO: P^T in TMEM, queries [0,64) at columns TM_DP + [0,32), [64,128) at TM_DP + 64 + [0,32)
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          ptx::mma_bf16_ts(tmem + TM_DV, tmem + TM_DP + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sdO, kk), idesc_nn,
+                           (i > 0 || kk > 0) ? 1u : 0u);
+        // dK += dS^T Q
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          ptx::mma_bf16_ss(tmem + TM_DK, desc_kmajor(sdS, kk), desc_mnmajor(sQ, kk), idesc_nn,
+                           (i > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma_commit(&bar->q_empty[s]);
+        ptx::mma_commit(&bar->do_empty[s]);
+        ptx::mma_commit(&bar->dvk_done);
+        if (i + 1 < n_it) {
+          // dP^T of the next tile overwrites the columns P^T was read from
+          if (!wait(&bar->dvk_done, (uint32_t)i & 1, a.status) || !issue_dp(i + 1)) { ok = false; break; }
+        }
+      }
+      if (!ok) set_abort(&bar->abort);
+      ptx::mma_commit(&bar->final_mma);
+      wait(&bar->final_mma, 0, a.status);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------ compute: thread = key row r, warpgroup wg owns queries [64 wg, 64 wg + 64)
+    const int wg = threadIdx.x >> 7, r = threadIdx.x & 127;
+    const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
+    const float sl2 = a.scale * kLog2e;
+    bool ok = true;
+    for (int i = 0; ok && i < n_it; ++i) {
+      const int s = i & 1;
+      if (!wait(&bar->meta_full[s], (uint32_t)(i >> 1) & 1, a.status) ||
+          !wait(&bar->s_full, (uint32_t)i & 1, a.status) || !wait(&bar->dp_full, (uint32_t)i & 1, a.status)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+      uint32_t s0[32], s1[32], d0[32], d1[32];
+      ld64(tmem + lane_addr + TM_S + wg * 64, s0, s1);
+      ld64(tmem + lane_addr + TM_DP + wg * 64, d0, d1);
+      ptx::tmem_ld_wait();
+      ptx::reg_fence(s0);
+      ptx::reg_fence(s1);
+      ptx::reg_fence(d0);
+      ptx::reg_fence(d1);
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&bar->s_free);
+      const uint8_t* meta = smem + OFF_META + s * kMetaStage;
+      const float* mlse = reinterpret_cast<const float*>(meta) + wg * 64;
+      const float* mdel = reinterpret_cast<const float*>(meta) + 128 + wg * 64;
+      const uint8_t* mlim = meta + 1024 + wg * 64;
+      uint32_t pp[32], pd[32];
+#pragma unroll
+      for (int k = 0; k < 32; ++k) {
+        float p[2], d[2];
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int jj = 2 * k + e;
+          const float sv = __uint_as_float(jj < 32 ? s0[jj] : s1[jj - 32]);
+          const float dv = __uint_as_float(jj < 32 ? d0[jj] : d1[jj - 32]);
+          p[e] = r < (int)mlim[jj] ? ex2(sv * sl2 - mlse[jj]) : 0.f;
+          d[e] = p[e] * (dv - mdel[jj]);
+        }
+        pp[k] = pack_bf16(p[0], p[1]);
+        pd[k] = pack_bf16(d[0], d[1]);
+      }
+      ptx::mbar_arrive(&bar->meta_empty[s]);
+      // P^T into the first half of this warpgroup's dP^T columns (already read)
+      ptx::tmem_st32(tmem + lane_addr + TM_DP + wg * 64, pp);
+      ptx::tmem_st_wait();
+      if (i >= 1 && !wait(&bar->dvk_done, (uint32_t)(i - 1) & 1, a.status)) { ok = false; break; }
+      store_row_half(smem + OFF_DS, r, wg, pd);
+      ptx::fence_proxy_async_smem();
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&bar->p_full);
+    }
+    if (ok && n_it > 0) ok = wait(&bar->dvk_done, (uint32_t)(n_it - 1) & 1, a.status);
+    if (!ok) {
+      set_abort(&bar->abort);
+    } else {
+      ptx::tc_fence_after();
+      const int key = c * kRows + r;
+      const bool kvalid = key < w.k_len;
+      const int64_t krow = (int64_t)w.k_base + key;
+      // warpgroup 0 writes dV, warpgroup 1 writes dK (scaled)
+      __nv_bfloat16* outp = reinterpret_cast<__nv_bfloat16*>(wg == 0 ? a.dv : a.dk) + krow * a.hkv * kD + g * kD;
+      const float f = wg == 0 ? 1.f : a.scale;
+      const uint32_t col = wg == 0 ? TM_DV : TM_DK;
+#pragma unroll 1
+      for (int q4 = 0; q4 < 4; ++q4) {
+        uint32_t v[32];
+        if (n_it > 0) {
+          ptx::tmem_ld32(tmem + lane_addr + col + q4 * 32, v);
+          ptx::tmem_ld_wait();
+          ptx::reg_fence(v);
+        } else {
+#pragma unroll
+          for (int k = 0; k < 32; ++k) v[k] = 0u;
+        }
+        if (kvalid) {
+          uint4* dst = reinterpret_cast<uint4*>(outp + q4 * 32);
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            uint4 o;
+            o.x = pack_bf16(__uint_as_float(v[8 * k + 0]) * f, __uint_as_float(v[8 * k + 1]) * f);
+            o.y = pack_bf16(__uint_as_float(v[8 * k + 2]) * f, __uint_as_float(v[8 * k + 3]) * f);
+            o.z = pack_bf16(__uint_as_float(v[8 * k + 4]) * f, __uint_as_float(v[8 * k + 5]) * f);
+            o.w = pack_bf16(__uint_as_float(v[8 * k + 6]) * f, __uint_as_float(v[8 * k + 7]) * f);
+            dst[k] = o;
+          }
+        }
+      }
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 9) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) {
+  cudaError_t e;
+  if (a.q_rows > 0) {
+    int64_t groups = a.q_rows * a.hq;
+    int grid = (int)((groups * 16 + 255) / 256);
+    if (grid > 152 * 16) grid = 152 * 16;
+    timer_begin(ISM_KERNEL_BWD_PRE, st);
+    delta_kernel<<<grid, 256, 0, st>>>((const __nv_bfloat16*)a.o, (const __nv_bfloat16*)a.dout, a.delta, a.q_rows,
+                                       a.hq);
+    timer_end(ISM_KERNEL_BWD_PRE, st);
+    count_launch();
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  CUtensorMap tq, tdo, tk, tv;
+  if ((e = make_tmap_bf16(&tq, a.q, (uint64_t)a.hq * kD, (uint64_t)a.q_rows)) != cudaSuccess) return e;
+  if ((e = make_tmap_bf16(&tdo, a.dout, (uint64_t)a.hq * kD, (uint64_t)a.q_rows)) != cudaSuccess) return e;
+  if ((e = make_tmap_bf16(&tk, a.k, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;
+  if ((e = make_tmap_bf16(&tv, a.v, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;
+  if (a.nq) {
+    if ((e = cudaFuncSetAttribute(dq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dq::kSmemBytes)) !=
+        cudaSuccess)
+      return e;
+    timer_begin(ISM_KERNEL_BWD_DQ, st);
+    dq_kernel<<<(unsigned)(a.nq * a.hq), kThreads, dq::kSmemBytes, st>>>(tq, tdo, tk, tv, a);
+    timer_end(ISM_KERNEL_BWD_DQ, st);
+    count_launch();
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  if (a.nk) {
+    if ((e = cudaFuncSetAttribute(dkdv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)dkv::kSmemBytes)) != cudaSuccess)
+      return e;
+    timer_begin(ISM_KERNEL_BWD_DKDV, st);
+    dkdv_kernel<<<(unsigned)(a.nk * a.hkv), kThreads, dkv::kSmemBytes, st>>>(tq, tdo, tk, tv, a);
+    timer_end(ISM_KERNEL_BWD_DKDV, st);
+    count_launch();
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace tc
+
+bool tc_bwd_available() { return tc::available(); }
+cudaError_t launch_tc_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) { return tc::launch_bwd(a, k_rows, st); }
+
+}  // namespace ism

@@ -309,7 +309,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ---------------------------------------------------------------- diagnostic
 // One 128x128x128 tile: C = A * B^T (B given as [N, K], K-major) or C = A * B
 // (B given as [K, N], MN-major).  Operands staged by plain stores in the
-// swizzled layout (modes 0/1) or by TMA (modes 2/3).
+// swizzled layout (modes 0/1), by TMA (modes 2/3), or A in tensor memory and
+// B by plain stores (modes 4/5).
 __global__ void __launch_bounds__(128, 1)
     mma_tile_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __nv_bfloat16* A, const __nv_bfloat16* B, float* C, int mode, uint32_t* status) {
@@ -321,16 +322,17 @@ __global__ void __launch_bounds__(128, 1)
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2);
   const int warp = threadIdx.x >> 5;
   const bool b_mn = (mode & 1) != 0;
+  const bool a_tmem = mode >= 4;
   if (threadIdx.x == 0) {
     ptx::mbar_init(&bars[0], 1);
     ptx::mbar_init(&bars[1], 1);
     ptx::fence_mbar_init();
   }
   if (warp == 0) {
-    ptx::tmem_alloc(tslot, 128);
+    ptx::tmem_alloc(tslot, 256);
     ptx::tmem_relinquish();
   }
-  if (mode < 2) {
+  if (mode < 2 || a_tmem) {
     for (int i = threadIdx.x; i < 128 * 128; i += blockDim.x) {
       const int r = i >> 7, c = i & 127;
       *reinterpret_cast<__nv_bfloat16*>(sa + swz_offset(r, c)) = A[i];
@@ -342,9 +344,26 @@ __global__ void __launch_bounds__(128, 1)
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem = *tslot;
+  const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
+  if (a_tmem) {
+    // row r of A into lane r, columns [128, 192): two bf16 of K per column
+    const int r = threadIdx.x;
+    for (int half = 0; half < 2; ++half) {
+      uint32_t v[32];
+      for (int i = 0; i < 32; ++i) {
+        const __nv_bfloat16 lo = A[r * 128 + half * 64 + 2 * i], hi = A[r * 128 + half * 64 + 2 * i + 1];
+        v[i] = (uint32_t)__bfloat16_as_ushort(lo) | ((uint32_t)__bfloat16_as_ushort(hi) << 16);
+      }
+      ptx::tmem_st32(tmem + lane_addr + 128 + half * 32, v);
+    }
+    ptx::tmem_st_wait();
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+  }
   bool ok = true;
   if (threadIdx.x == 0) {
-    if (mode >= 2) {
+    if (mode == 2 || mode == 3) {
       ptx::mbar_expect_tx(&bars[0], 2 * kTileBytes);
       ptx::tma_load_2d(sa, &tmA, &bars[0], 0, 0);
       ptx::tma_load_2d(sa + kHalfBytes, &tmA, &bars[0], 64, 0);
@@ -355,16 +374,19 @@ __global__ void __launch_bounds__(128, 1)
     if (ok) {
       const uint32_t idesc = ptx::idesc_bf16_f32(128, 128, 0, b_mn ? 1u : 0u);
       const uint32_t saa = ptx::smem_u32(sa), sbb = ptx::smem_u32(sb);
-      for (int kk = 0; kk < 8; ++kk)
-        ptx::mma_bf16_ss(tmem, desc_kmajor(saa, kk), b_mn ? desc_mnmajor(sbb, kk) : desc_kmajor(sbb, kk), idesc,
-                         kk > 0 ? 1u : 0u);
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint64_t bd = b_mn ? desc_mnmajor(sbb, kk) : desc_kmajor(sbb, kk);
+        if (a_tmem)
+          ptx::mma_bf16_ts(tmem, tmem + 128 + 8 * kk, bd, idesc, kk > 0 ? 1u : 0u);
+        else
+          ptx::mma_bf16_ss(tmem, desc_kmajor(saa, kk), bd, idesc, kk > 0 ? 1u : 0u);
+      }
     }
     ptx::mma_commit(&bars[1]);
     ok = wait(&bars[1], 0, status) && ok;
   }
   __syncthreads();
   ptx::tc_fence_after();
-  const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
   for (int c = 0; c < 4; ++c) {
     uint32_t v[32];
     ptx::tmem_ld32(tmem + lane_addr + c * 32, v);
@@ -376,7 +398,7 @@ __global__ void __launch_bounds__(128, 1)
   __syncthreads();
   if (warp == 0) {
     ptx::tc_fence_after();
-    ptx::tmem_dealloc(tmem, 128);
+    ptx::tmem_dealloc(tmem, 256);
   }
 }
 
@@ -432,7 +454,7 @@ cudaError_t launch_mma_tile(const void* A, const void* B, float* C, int mode, ui
   memset(&ta, 0, sizeof(ta));
   memset(&tb, 0, sizeof(tb));
   cudaError_t e;
-  if (mode >= 2) {
+  if (mode == 2 || mode == 3) {
     if ((e = make_tmap_bf16(&ta, A, 128, 128)) != cudaSuccess) return e;
     if ((e = make_tmap_bf16(&tb, B, 128, 128)) != cudaSuccess) return e;
   }

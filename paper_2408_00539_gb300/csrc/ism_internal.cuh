@@ -55,7 +55,7 @@ struct Meta {
 };
 
 // Status word bits recorded by device code.
-enum : uint32_t { kStatusTimeout = 1u };
+enum : uint32_t { kStatusTimeout = 1u, kStatusSmemAlign = 2u };
 
 // ---------------------------------------------------------------- launches
 // Each returns cudaSuccess or the launch error.
