@@ -50,6 +50,27 @@ def n_visible(segs) -> int:
     return total
 
 
+NCU_NAME = {"fwd": "fwd_kernel", "bwd_dkdv": "dkdv_kernel", "bwd_dq": "dq_kernel"}
+
+
+def kernel_traffic(kind: str, workload: str):
+    """DRAM bytes per launch from the committed ncu capture, or None when the
+    kernel's source changed since the counters were taken (or no capture of
+    this workload exists)."""
+    import hashlib
+    p = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as fh:
+        rec = json.load(fh).get(NCU_NAME.get(kind, ""))
+    if not rec or rec.get("workload") != workload:
+        return None
+    with open(os.path.join(ROOT, rec["source"]), "rb") as fh:
+        if hashlib.sha256(fh.read()).hexdigest() != rec["source_sha256"]:
+            return None
+    return rec["dram_bytes_per_launch"]
+
+
 def read_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -226,6 +247,12 @@ def run_cuda(args, w):
         step()
     torch.cuda.synchronize()
     ism.check_status(dev)
+    if args.profile_step:
+        # one more step for a profiler to capture, then stop (no timing, no JSON)
+        step()
+        torch.cuda.synchronize()
+        ism.check_status(dev)
+        return
 
     # per-kernel timers for the roofline (on the library's launch stream)
     stream = torch.cuda.current_stream(dev)
@@ -270,7 +297,7 @@ def run_cuda(args, w):
     peak = peaks.get("bf16_tflops_sustained" if args.steps * ms_per_step > 2000 else "bf16_tflops")
     achieved = kflops[dom] / (mean_k[dom] * 1e-3) / 1e12
     roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
+                "frac": achieved / peak, "traffic": kernel_traffic(dom, w.name), "peak_kind": peak_kind,
                 "flops_per_launch": kflops[dom], "ms_per_launch": mean_k[dom]}
 
     # end to end through the public API with host buffers
@@ -341,6 +368,8 @@ def main():
     ap.add_argument("--impl", default="cuda", choices=["cuda", "reference"])
     ap.add_argument("--workload", default="gqa_8k", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--profile-step", action="store_true",
+                    help="run the warm-up steps and one more step, print nothing (for ncu)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     w = WORKLOADS[args.workload]()
