@@ -1,0 +1,306 @@
+// ISM attention forward, two query heads per CTA (sm_103a tensor cores).
+//
+// When the query heads come in pairs that share a KV head (grouped-query
+// attention with an even group size), one CTA computes the same 128-row
+// query tile for both heads of a pair: every K/V block is loaded once and
+// used by both.  The two heads' softmax warpgroups alternate with the tensor
+// core (while one warpgroup turns S_A into P_A, the tensor core computes
+// S_B, and so on).  P is written back into tensor memory over the S it came
+// from and read there as the A operand of O += P V.
+//
+// Tensor memory (512 columns): S_A [0,128) O_A [128,256) S_B [256,384)
+// O_B [384,512).  Shared memory: Q_A, Q_B, and a 2-stage K / V ring.
+// Warps 0-3 softmax of head A, 4-7 of head B, 8 TMA producer, 9 MMA issuer.
+// The mask and the lazy-rescale online softmax are those of the one-head
+// kernel (Eq. e_ISM with the bound of Eq. fj; full tiles unmasked).
+#include "ism_tc_common.cuh"
+
+namespace ism {
+namespace tc {
+namespace {
+
+constexpr int kThreads = 320;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t OFF_QA = 0, OFF_QB = kTileBytes, OFF_K = 2 * kTileBytes, OFF_V = 4 * kTileBytes,
+                   OFF_BAR = 6 * kTileBytes;
+constexpr uint32_t kSmemBytes = OFF_BAR + 256 + 1024;
+
+struct Bars {
+  uint64_t q_full;
+  uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
+  uint64_t s_full[2], p_full[2], pv_done[2];  // per head of the pair
+  uint64_t final_mma;
+  uint32_t tmem_base;
+  int32_t abort;
+};
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+__device__ __forceinline__ bool aborted(const int32_t* f) { return *reinterpret_cast<const volatile int32_t*>(f) != 0; }
+__device__ __forceinline__ void set_abort(int32_t* f) { *reinterpret_cast<volatile int32_t*>(f) = 1; }
+
+__global__ void __launch_bounds__(kThreads, 1)
+    fwd_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                    const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  Bars* bar = reinterpret_cast<Bars*>(smem + OFF_BAR);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int npairs = a.hq >> 1;
+  const int hp = blockIdx.x % npairs;
+  const Tile w = a.qtiles[a.q_order[blockIdx.x / npairs]];
+  const int h0 = 2 * hp;
+  const int g = h0 / (a.hq / a.hkv);
+  const int nkb = w.a1, kfull = w.a0;
+
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(&bar->q_full, 1);
+    for (int s = 0; s < 2; ++s) {
+      ptx::mbar_init(&bar->k_full[s], 1);
+      ptx::mbar_init(&bar->k_empty[s], 1);
+      ptx::mbar_init(&bar->v_full[s], 1);
+      ptx::mbar_init(&bar->v_empty[s], 1);
+      ptx::mbar_init(&bar->s_full[s], 1);
+      ptx::mbar_init(&bar->p_full[s], 128);
+      ptx::mbar_init(&bar->pv_done[s], 1);
+    }
+    ptx::mbar_init(&bar->final_mma, 1);
+    bar->abort = 0;
+    ptx::fence_mbar_init();
+  }
+  if (warp == 9) {
+    ptx::tmem_alloc(&bar->tmem_base, kTmemCols);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = bar->tmem_base;
+
+  if (warp == 8) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0 && nkb > 0) {
+      ptx::tma_prefetch_desc(&tmK);
+      ptx::tma_prefetch_desc(&tmV);
+      const int32_t qy = w.q_base + w.tile * kRows;
+      ptx::mbar_expect_tx(&bar->q_full, 2 * kTileBytes);
+      ptx::tma_load_2d(smem + OFF_QA, &tmQ, &bar->q_full, h0 * kD, qy);
+      ptx::tma_load_2d(smem + OFF_QA + kHalfBytes, &tmQ, &bar->q_full, h0 * kD + 64, qy);
+      ptx::tma_load_2d(smem + OFF_QB, &tmQ, &bar->q_full, (h0 + 1) * kD, qy);
+      ptx::tma_load_2d(smem + OFF_QB + kHalfBytes, &tmQ, &bar->q_full, (h0 + 1) * kD + 64, qy);
+      uint32_t nk[2] = {0, 0}, nv[2] = {0, 0};
+      for (int j = 0; j < nkb; ++j) {
+        const int s = j & 1;
+        const uint32_t n = (uint32_t)(j >> 1);
+        if (aborted(&bar->abort)) break;
+        const int32_t ky = w.k_base + j * kRows;
+        if (j >= 2 && !wait(&bar->k_empty[s], (n - 1) & 1, a.status)) { set_abort(&bar->abort); break; }
+        ptx::mbar_expect_tx(&bar->k_full[s], kTileBytes);
+        ptx::tma_load_2d(smem + OFF_K + s * kTileBytes, &tmK, &bar->k_full[s], g * kD, ky);
+        ptx::tma_load_2d(smem + OFF_K + s * kTileBytes + kHalfBytes, &tmK, &bar->k_full[s], g * kD + 64, ky);
+        ++nk[s];
+        if (j >= 2 && !wait(&bar->v_empty[s], (n - 1) & 1, a.status)) { set_abort(&bar->abort); break; }
+        ptx::mbar_expect_tx(&bar->v_full[s], kTileBytes);
+        ptx::tma_load_2d(smem + OFF_V + s * kTileBytes, &tmV, &bar->v_full[s], g * kD, ky);
+        ptx::tma_load_2d(smem + OFF_V + s * kTileBytes + kHalfBytes, &tmV, &bar->v_full[s], g * kD + 64, ky);
+        ++nv[s];
+      }
+      if (aborted(&bar->abort)) {
+        wait(&bar->q_full, 0, a.status);
+        for (int s = 0; s < 2; ++s) {
+          if (nk[s]) wait(&bar->k_full[s], (nk[s] - 1) & 1, a.status);
+          if (nv[s]) wait(&bar->v_full[s], (nv[s] - 1) & 1, a.status);
+        }
+      }
+    }
+  } else if (warp == 9) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0 && nkb > 0) {
+      constexpr uint32_t idesc_qk = ptx::idesc_bf16_f32(128, 128, 0, 0);
+      constexpr uint32_t idesc_pv = ptx::idesc_bf16_f32(128, 128, 0, 1);
+      const uint32_t sQ0 = ptx::smem_u32(smem + OFF_QA);
+      // head x: Q at sQ0 + x * kTileBytes, S at tmem + 256 x, O at tmem + 128 + 256 x
+      auto issue_s = [&](int x, int j) {
+        const uint32_t sK = ptx::smem_u32(smem + OFF_K + (j & 1) * kTileBytes);
+        const uint32_t sQ = sQ0 + (uint32_t)x * kTileBytes, tS = tmem + 256u * (uint32_t)x;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          ptx::mma_bf16_ss(tS, desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_qk, kk > 0 ? 1u : 0u);
+        ptx::mma_commit(&bar->s_full[x]);
+      };
+      auto issue_pv = [&](int x, int j) {
+        const uint32_t sV = ptx::smem_u32(smem + OFF_V + (j & 1) * kTileBytes);
+        const uint32_t tS = tmem + 256u * (uint32_t)x, tO = tS + 128u;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          ptx::mma_bf16_ts(tO, tS + 8 * kk, desc_mnmajor(sV, kk), idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma_commit(&bar->pv_done[x]);
+      };
+      bool ok = wait(&bar->q_full, 0, a.status) && wait(&bar->k_full[0], 0, a.status);
+      if (ok) {
+        ptx::tc_fence_after();
+        issue_s(0, 0);
+        issue_s(1, 0);
+        ptx::mma_commit(&bar->k_empty[0]);
+      }
+      // Per block: PV_A(j), S_A(j+1), PV_B(j), S_B(j+1).  S_x(j+1) overwrites
+      // the P_x(j) that PV_x(j) reads, so it is issued once PV_x(j) is done;
+      // the other head's work keeps the tensor core busy meanwhile.
+      for (int j = 0; ok && j < nkb; ++j) {
+        const int s = j & 1, s1 = (j + 1) & 1;
+        const bool more = j + 1 < nkb;
+        if (aborted(&bar->abort)) { ok = false; break; }
+        if (!wait(&bar->v_full[s], (uint32_t)(j >> 1) & 1, a.status)) { ok = false; break; }
+        if (more && !wait(&bar->k_full[s1], (uint32_t)((j + 1) >> 1) & 1, a.status)) { ok = false; break; }
+        for (int x = 0; x < 2; ++x) {
+          if (!wait(&bar->p_full[x], (uint32_t)j & 1, a.status)) { ok = false; break; }
+          ptx::tc_fence_after();
+          issue_pv(x, j);
+          if (x == 1) ptx::mma_commit(&bar->v_empty[s]);
+          if (more) {
+            if (!wait(&bar->pv_done[x], (uint32_t)j & 1, a.status)) { ok = false; break; }
+            ptx::tc_fence_after();
+            issue_s(x, j + 1);
+            if (x == 1) ptx::mma_commit(&bar->k_empty[s1]);
+          }
+        }
+      }
+      if (!ok) set_abort(&bar->abort);
+      ptx::mma_commit(&bar->final_mma);
+      wait(&bar->final_mma, 0, a.status);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ softmax of head x
+    const int x = warp >> 2;
+    const int r = threadIdx.x & 127;
+    const int h = h0 + x;
+    const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
+    const uint32_t tS = tmem + lane_addr + (x ? 256u : 0u), tO = tmem + lane_addr + (x ? 384u : 128u);
+    const int row = w.tile * kRows + r;
+    const bool valid = row < w.q_len;
+    const int ke = a.kv_end[w.kv_base + (valid ? row : w.q_len - 1)];
+    const float sl2 = a.scale * kLog2e;
+    float m_use = -INFINITY, l = 0.f;
+    bool ok = nkb > 0;
+    for (int j = 0; ok && j < nkb; ++j) {
+      if (!wait(&bar->s_full[x], (uint32_t)j & 1, a.status)) { ok = false; break; }
+      ptx::tc_fence_after();
+      float xs[128];
+      {
+        uint32_t t[4][32];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) ptx::tmem_ld32(tS + c * 32, t[c]);
+        ptx::tmem_ld_wait();
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          ptx::reg_fence(t[c]);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) xs[c * 32 + i] = __uint_as_float(t[c][i]);
+        }
+      }
+      float mloc = -INFINITY;
+      if (j >= kfull) {
+        const int lim = ke - j * kRows;
+#pragma unroll
+        for (int c = 0; c < 128; ++c) {
+          xs[c] = c < lim ? xs[c] * sl2 : -INFINITY;
+          mloc = fmaxf(mloc, xs[c]);
+        }
+      } else {
+#pragma unroll
+        for (int c = 0; c < 128; ++c) {
+          xs[c] *= sl2;
+          mloc = fmaxf(mloc, xs[c]);
+        }
+      }
+      const float m_new = fmaxf(m_use, mloc);
+      if (j == 0) {
+        m_use = m_new;
+      } else if (m_new > m_use + 8.f) {
+        // bring O (complete through PV(j-1)) and l to the new max
+        if (!wait(&bar->pv_done[x], (uint32_t)(j - 1) & 1, a.status)) { ok = false; break; }
+        ptx::tc_fence_after();
+        const float f = ex2(m_use - m_new);
+        l *= f;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t o[32];
+          ptx::tmem_ld32(tO + c * 32, o);
+          ptx::tmem_ld_wait();
+          ptx::reg_fence(o);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * f);
+          ptx::tmem_st32(tO + c * 32, o);
+        }
+        m_use = m_new;
+      }
+      float rs = 0.f;
+      uint32_t pk[2][32];
+#pragma unroll
+      for (int c = 0; c < 64; ++c) {
+        const float p0 = ex2(xs[2 * c] - m_use);
+        const float p1 = ex2(xs[2 * c + 1] - m_use);
+        rs += p0 + p1;
+        pk[c >> 5][c & 31] = pack_bf16(p0, p1);
+      }
+      l += rs;
+      // P over the first 64 columns of S (already read)
+      ptx::tmem_st32(tS, pk[0]);
+      ptx::tmem_st32(tS + 32, pk[1]);
+      ptx::tmem_st_wait();
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&bar->p_full[x]);
+    }
+    if (ok) ok = wait(&bar->pv_done[x], (uint32_t)(nkb - 1) & 1, a.status);
+    if (!ok) {
+      set_abort(&bar->abort);
+    } else {
+      ptx::tc_fence_after();
+      const float inv = 1.f / l;
+      const int64_t orow = (int64_t)w.q_base + row;
+      uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.out) + orow * a.hq * kD + h * kD);
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        uint32_t o[32];
+        ptx::tmem_ld32(tO + c * 32, o);
+        ptx::tmem_ld_wait();
+        ptx::reg_fence(o);
+        if (valid) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            uint4 v4;
+            v4.x = pack_bf16(__uint_as_float(o[8 * i + 0]) * inv, __uint_as_float(o[8 * i + 1]) * inv);
+            v4.y = pack_bf16(__uint_as_float(o[8 * i + 2]) * inv, __uint_as_float(o[8 * i + 3]) * inv);
+            v4.z = pack_bf16(__uint_as_float(o[8 * i + 4]) * inv, __uint_as_float(o[8 * i + 5]) * inv);
+            v4.w = pack_bf16(__uint_as_float(o[8 * i + 6]) * inv, __uint_as_float(o[8 * i + 7]) * inv);
+            dst[c * 4 + i] = v4;
+          }
+        }
+      }
+      if (valid && a.lse) a.lse[(int64_t)h * a.q_rows + orow] = (m_use + log2f(l)) * kLn2;
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 9) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_fwd_pair(const AttnArgs& a, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                            cudaStream_t st) {
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(fwd_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
+      cudaSuccess)
+    return e;
+  fwd_pair_kernel<<<(unsigned)(a.nq * (a.hq / 2)), kThreads, kSmemBytes, st>>>(tq, tk, tv, a);
+  return cudaGetLastError();
+}
+
+}  // namespace tc
+}  // namespace ism

@@ -80,6 +80,9 @@ __device__ __forceinline__ uint64_t desc_mnmajor(uint32_t tile_saddr, int kk) {
 cudaError_t make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows);
 // Host: true on an sm_103 device with the tensor-map encoder available.
 bool available();
+// Host: forward with two query heads (sharing a KV head) per CTA.
+cudaError_t launch_fwd_pair(const AttnArgs& a, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                            cudaStream_t st);
 
 }  // namespace tc
 }  // namespace ism
