@@ -5,12 +5,12 @@
 //   delta_kernel   Delta_j = sum_d dO_jd O_jd                      (HBM-bound)
 //   dq_kernel      per (query tile, query head), over the tile's non-empty
 //                  key blocks: S = Q K^T, dP = dO V^T (TMEM), dS = P (dP - Delta)
-//                  to shared memory, dQ += dS K (TMEM); dQ = scale * dQ.
+//                  back into TMEM, dQ += dS K (TMEM); dQ = scale * dQ.
 //   dkdv_kernel    per (key tile, KV head), over the query heads of the group
 //                  and the query tiles that see the key tile: S^T = K Q^T and
-//                  dP^T = V dO^T (TMEM), P^T back into TMEM (A operand of the
-//                  next MMA), dS^T to shared memory, dV += P^T dO, dK += dS^T Q
-//                  (TMEM accumulators); dK = scale * dK.
+//                  dP^T = V dO^T (TMEM), P^T and dS^T back into TMEM (A operands
+//                  of the next MMAs), dV += P^T dO, dK += dS^T Q (TMEM
+//                  accumulators); dK = scale * dK.
 // Warp roles in both MMA kernels: warps 0..7 compute (two warpgroups, each
 // owning 64 of the 128 columns of a tile; thread = TMEM lane = tile row),
 // warp 8 loads (TMA), warp 9 owns TMEM and issues the MMAs.
@@ -30,16 +30,6 @@ __device__ __forceinline__ void set_abort(int32_t* f) { *reinterpret_cast<volati
 __device__ __forceinline__ void ld64(uint32_t taddr, uint32_t (&a)[32], uint32_t (&b)[32]) {
   ptx::tmem_ld32(taddr, a);
   ptx::tmem_ld32(taddr + 32, b);
-}
-
-// Writes 64 bf16 values (32 packed words) as row r, half `half` of a
-// 128B-swizzled [128 x 128] tile.
-__device__ __forceinline__ void store_row_half(uint8_t* tile, int r, int half, const uint32_t (&pk)[32]) {
-  uint8_t* row = tile + half * kHalfBytes + r * 128;
-#pragma unroll
-  for (int c = 0; c < 8; ++c)
-    *reinterpret_cast<uint4*>(row + ((c ^ (r & 7)) << 4)) =
-        make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
 }
 
 // ------------------------------------------------------------------ delta
@@ -71,19 +61,27 @@ __global__ void delta_kernel(const __nv_bfloat16* __restrict__ O, const __nv_bfl
 }
 
 // ------------------------------------------------------------------ dQ
+// dS goes back into tensor memory over the S it came from and is the A
+// operand of dQ += dS K, so shared memory holds Q, dO, a 3-stage K ring (K is
+// read by the first and the last MMA of a block) and a 2-stage V ring.  S is
+// double-buffered in tensor memory: S_{c+1} is computed while block c's
+// scores are turned into dS.
 namespace dq {
-constexpr uint32_t OFF_Q = 0, OFF_DO = kTileBytes, OFF_K = 2 * kTileBytes, OFF_V = 4 * kTileBytes,
-                   OFF_DS = 6 * kTileBytes, OFF_BAR = 7 * kTileBytes;
+constexpr int kKStages = 3;
+constexpr uint32_t OFF_Q = 0, OFF_DO = kTileBytes, OFF_K = 2 * kTileBytes, OFF_V = 5 * kTileBytes,
+                   OFF_BAR = 7 * kTileBytes;
 constexpr uint32_t kSmemBytes = OFF_BAR + 256 + 1024;
-constexpr uint32_t TM_S = 0, TM_DP = 128, TM_DQ = 256;
+constexpr uint32_t TM_S = 0, TM_DP = 256, TM_DQ = 384;  // S regions at 0 and 128
 
 struct Bars {
   uint64_t qdo_full;
-  uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
-  uint64_t s_full, dp_full, sdp_free, p_full, dq_done, final_mma;
+  uint64_t k_full[kKStages], k_empty[kKStages], v_full[2], v_empty[2];
+  uint64_t s_full[2], p_full[2];
+  uint64_t dp_full, dp_read, dq_done, final_mma;
   uint32_t tmem_base;
   int32_t abort;
 };
+static_assert(sizeof(Bars) <= 256, "barrier block");
 }  // namespace dq
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
@@ -105,16 +103,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     ptx::mbar_init(&bar->qdo_full, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kKStages; ++s) {
       ptx::mbar_init(&bar->k_full[s], 1);
       ptx::mbar_init(&bar->k_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
       ptx::mbar_init(&bar->v_full[s], 1);
       ptx::mbar_init(&bar->v_empty[s], 1);
+      ptx::mbar_init(&bar->s_full[s], 1);
+      ptx::mbar_init(&bar->p_full[s], kComputeThreads);
     }
-    ptx::mbar_init(&bar->s_full, 1);
     ptx::mbar_init(&bar->dp_full, 1);
-    ptx::mbar_init(&bar->sdp_free, kComputeThreads);
-    ptx::mbar_init(&bar->p_full, kComputeThreads);
+    ptx::mbar_init(&bar->dp_read, kComputeThreads);
     ptx::mbar_init(&bar->dq_done, 1);
     ptx::mbar_init(&bar->final_mma, 1);
     bar->abort = 0;
@@ -139,29 +139,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tma_load_2d(smem + OFF_Q + kHalfBytes, &tmQ, &bar->qdo_full, h * kD + 64, qy);
       ptx::tma_load_2d(smem + OFF_DO, &tmdO, &bar->qdo_full, h * kD, qy);
       ptx::tma_load_2d(smem + OFF_DO + kHalfBytes, &tmdO, &bar->qdo_full, h * kD + 64, qy);
-      uint32_t nk[2] = {0, 0}, nv[2] = {0, 0};
+      uint32_t nk[kKStages] = {0, 0, 0}, nv[2] = {0, 0};
       for (int c = 0; c < nkb; ++c) {
-        const int s = c & 1;
-        const uint32_t n = (uint32_t)(c >> 1);
+        const int sk = c % kKStages, sv = c & 1;
         if (aborted(&bar->abort)) break;
         const int32_t ky = w.k_base + c * kRows;
-        if (c >= 2 && !wait(&bar->k_empty[s], (n - 1) & 1, a.status)) { set_abort(&bar->abort); break; }
-        ptx::mbar_expect_tx(&bar->k_full[s], kTileBytes);
-        ptx::tma_load_2d(smem + OFF_K + s * kTileBytes, &tmK, &bar->k_full[s], g * kD, ky);
-        ptx::tma_load_2d(smem + OFF_K + s * kTileBytes + kHalfBytes, &tmK, &bar->k_full[s], g * kD + 64, ky);
-        ++nk[s];
-        if (c >= 2 && !wait(&bar->v_empty[s], (n - 1) & 1, a.status)) { set_abort(&bar->abort); break; }
-        ptx::mbar_expect_tx(&bar->v_full[s], kTileBytes);
-        ptx::tma_load_2d(smem + OFF_V + s * kTileBytes, &tmV, &bar->v_full[s], g * kD, ky);
-        ptx::tma_load_2d(smem + OFF_V + s * kTileBytes + kHalfBytes, &tmV, &bar->v_full[s], g * kD + 64, ky);
-        ++nv[s];
+        if (c >= kKStages && !wait(&bar->k_empty[sk], (uint32_t)(c / kKStages - 1) & 1, a.status)) {
+          set_abort(&bar->abort);
+          break;
+        }
+        ptx::mbar_expect_tx(&bar->k_full[sk], kTileBytes);
+        ptx::tma_load_2d(smem + OFF_K + sk * kTileBytes, &tmK, &bar->k_full[sk], g * kD, ky);
+        ptx::tma_load_2d(smem + OFF_K + sk * kTileBytes + kHalfBytes, &tmK, &bar->k_full[sk], g * kD + 64, ky);
+        ++nk[sk];
+        if (c >= 2 && !wait(&bar->v_empty[sv], (uint32_t)((c >> 1) - 1) & 1, a.status)) {
+          set_abort(&bar->abort);
+          break;
+        }
+        ptx::mbar_expect_tx(&bar->v_full[sv], kTileBytes);
+        ptx::tma_load_2d(smem + OFF_V + sv * kTileBytes, &tmV, &bar->v_full[sv], g * kD, ky);
+        ptx::tma_load_2d(smem + OFF_V + sv * kTileBytes + kHalfBytes, &tmV, &bar->v_full[sv], g * kD + 64, ky);
+        ++nv[sv];
       }
       if (aborted(&bar->abort)) {
         wait(&bar->qdo_full, 0, a.status);
-        for (int s = 0; s < 2; ++s) {
+        for (int s = 0; s < kKStages; ++s)
           if (nk[s]) wait(&bar->k_full[s], (nk[s] - 1) & 1, a.status);
+        for (int s = 0; s < 2; ++s)
           if (nv[s]) wait(&bar->v_full[s], (nv[s] - 1) & 1, a.status);
-        }
       }
     }
   } else if (warp == 9) {
@@ -169,44 +174,54 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idesc_nt = ptx::idesc_bf16_f32(128, 128, 0, 0);  // A K-major, B K-major
       constexpr uint32_t idesc_nn = ptx::idesc_bf16_f32(128, 128, 0, 1);  // A K-major, B MN-major
       const uint32_t sQ = ptx::smem_u32(smem + OFF_Q), sdO = ptx::smem_u32(smem + OFF_DO);
-      const uint32_t sdS = ptx::smem_u32(smem + OFF_DS);
-      bool ok = wait(&bar->qdo_full, 0, a.status);
-      auto issue_sdp = [&](int c) -> bool {
-        const int s = c & 1;
-        const uint32_t n = (uint32_t)(c >> 1);
-        if (!wait(&bar->k_full[s], n & 1, a.status)) return false;
+      auto issue_s = [&](int c) -> bool {
+        const int sk = c % kKStages;
+        if (!wait(&bar->k_full[sk], (uint32_t)(c / kKStages) & 1, a.status)) return false;
         ptx::tc_fence_after();
-        const uint32_t sK = ptx::smem_u32(smem + OFF_K + s * kTileBytes);
+        const uint32_t sK = ptx::smem_u32(smem + OFF_K + sk * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss(tmem + TM_S, desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_nt, kk > 0 ? 1u : 0u);
-        ptx::mma_commit(&bar->s_full);
-        if (!wait(&bar->v_full[s], n & 1, a.status)) return false;
+          ptx::mma_bf16_ss(tmem + TM_S + 128u * (c & 1), desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_nt,
+                           kk > 0 ? 1u : 0u);
+        ptx::mma_commit(&bar->s_full[c & 1]);
+        return true;
+      };
+      auto issue_dp = [&](int c) -> bool {
+        const int sv = c & 1;
+        if (!wait(&bar->v_full[sv], (uint32_t)(c >> 1) & 1, a.status)) return false;
         ptx::tc_fence_after();
-        const uint32_t sV = ptx::smem_u32(smem + OFF_V + s * kTileBytes);
+        const uint32_t sV = ptx::smem_u32(smem + OFF_V + sv * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
           ptx::mma_bf16_ss(tmem + TM_DP, desc_kmajor(sdO, kk), desc_kmajor(sV, kk), idesc_nt, kk > 0 ? 1u : 0u);
         ptx::mma_commit(&bar->dp_full);
-        ptx::mma_commit(&bar->v_empty[s]);
+        ptx::mma_commit(&bar->v_empty[sv]);
         return true;
       };
-      if (ok) ok = issue_sdp(0);
+      bool ok = wait(&bar->qdo_full, 0, a.status);
+      if (ok) ok = issue_s(0) && issue_dp(0);
+      if (ok && nkb > 1) ok = issue_s(1);
       for (int c = 0; ok && c < nkb; ++c) {
+        const int R = c & 1;
         if (aborted(&bar->abort)) { ok = false; break; }
         if (c + 1 < nkb) {
-          if (!wait(&bar->sdp_free, (uint32_t)c & 1, a.status)) { ok = false; break; }
-          if (!issue_sdp(c + 1)) { ok = false; break; }
+          if (!wait(&bar->dp_read, (uint32_t)c & 1, a.status) || !issue_dp(c + 1)) { ok = false; break; }
         }
-        if (!wait(&bar->p_full, (uint32_t)c & 1, a.status)) { ok = false; break; }
+        if (!wait(&bar->p_full[R], (uint32_t)(c >> 1) & 1, a.status)) { ok = false; break; }
         ptx::tc_fence_after();
-        const uint32_t sK = ptx::smem_u32(smem + OFF_K + (c & 1) * kTileBytes);
+        const uint32_t sK = ptx::smem_u32(smem + OFF_K + (c % kKStages) * kTileBytes);
+        // dQ += dS K_c: dS (bf16, keys packed two per column) in S region R, keys [0,64) at
+        // columns [0,32) and [64,128) at columns [64,96)
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss(tmem + TM_DQ, desc_kmajor(sdS, kk), desc_mnmajor(sK, kk), idesc_nn,
-                           (c > 0 || kk > 0) ? 1u : 0u);
+          ptx::mma_bf16_ts(tmem + TM_DQ, tmem + TM_S + 128u * R + 8 * kk + (kk >= 4 ? 32 : 0),
+                           desc_mnmajor(sK, kk), idesc_nn, (c > 0 || kk > 0) ? 1u : 0u);
         ptx::mma_commit(&bar->dq_done);
-        ptx::mma_commit(&bar->k_empty[c & 1]);
+        ptx::mma_commit(&bar->k_empty[c % kKStages]);
+        if (c + 2 < nkb) {
+          // S_{c+2} overwrites the dS that dQ_c reads: wait for dQ_c first
+          if (!wait(&bar->dq_done, (uint32_t)c & 1, a.status) || !issue_s(c + 2)) { ok = false; break; }
+        }
       }
       if (!ok) set_abort(&bar->abort);
       ptx::mma_commit(&bar->final_mma);
@@ -226,21 +241,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     const float sl2 = a.scale * kLog2e;
     bool ok = nkb > 0;
     for (int c = 0; ok && c < nkb; ++c) {
-      if (!wait(&bar->s_full, (uint32_t)c & 1, a.status) || !wait(&bar->dp_full, (uint32_t)c & 1, a.status)) {
+      const int R = c & 1;
+      const uint32_t tS = tmem + lane_addr + TM_S + 128u * R + 64u * wg;
+      if (!wait(&bar->s_full[R], (uint32_t)(c >> 1) & 1, a.status) || !wait(&bar->dp_full, (uint32_t)c & 1, a.status)) {
         ok = false;
         break;
       }
       ptx::tc_fence_after();
       uint32_t s0[32], s1[32], d0[32], d1[32];
-      ld64(tmem + lane_addr + TM_S + wg * 64, s0, s1);
-      ld64(tmem + lane_addr + TM_DP + wg * 64, d0, d1);
+      ld64(tS, s0, s1);
+      ld64(tmem + lane_addr + TM_DP + 64u * wg, d0, d1);
       ptx::tmem_ld_wait();
       ptx::reg_fence(s0);
       ptx::reg_fence(s1);
       ptx::reg_fence(d0);
       ptx::reg_fence(d1);
       ptx::tc_fence_before();
-      ptx::mbar_arrive(&bar->sdp_free);
+      ptx::mbar_arrive(&bar->dp_read);
       const int lim = (c < kfull) ? 128 : ke - c * kRows - wg * 64;  // visible columns of this half
       uint32_t pk[32];  // pk[k] holds columns 2k and 2k+1 of this half
 #pragma unroll
@@ -256,13 +273,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         pk[k] = pack_bf16(v[0], v[1]);
       }
-      if (c >= 1 && !wait(&bar->dq_done, (uint32_t)(c - 1) & 1, a.status)) { ok = false; break; }
-      store_row_half(smem + OFF_DS, r, wg, pk);
-      ptx::fence_proxy_async_smem();
+      // dS over the first 32 columns of this half of S (already read)
+      ptx::tmem_st32(tS, pk);
+      ptx::tmem_st_wait();
       ptx::tc_fence_before();
-      ptx::mbar_arrive(&bar->p_full);
+      ptx::mbar_arrive(&bar->p_full[R]);
     }
-    if (ok) ok = wait(&bar->dq_done, (uint32_t)(nkb - 1) & 1, a.status);
+    if (ok) ok = wait(&bar->final_mma, 0, a.status);
     if (!ok) {
       set_abort(&bar->abort);
     } else {
@@ -302,8 +319,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ------------------------------------------------------------------ dK / dV
 namespace dkv {
-constexpr uint32_t OFF_K = 0, OFF_V = kTileBytes, OFF_Q = 2 * kTileBytes, OFF_DO = 4 * kTileBytes,
-                   OFF_DS = 6 * kTileBytes, OFF_META = 7 * kTileBytes;
+// Q is read by the first (S^T) and the last (dK) MMA of an iteration, so it
+// gets a 3-stage ring; dO (dP^T early, dV late) 2 stages; P^T and dS^T live in
+// tensor memory over the dP^T they came from.
+constexpr int kQStages = 3;
+constexpr uint32_t OFF_K = 0, OFF_V = kTileBytes, OFF_Q = 2 * kTileBytes, OFF_DO = 5 * kTileBytes,
+                   OFF_META = 7 * kTileBytes;
 // per stage: lse2[128] f32, delta[128] f32, visible-key count[128] u8
 constexpr uint32_t kMetaStage = 128 * 4 + 128 * 4 + 128;
 constexpr uint32_t OFF_BAR = OFF_META + 2 * kMetaStage;
@@ -312,11 +333,12 @@ constexpr uint32_t TM_S = 0, TM_DP = 128, TM_DV = 256, TM_DK = 384;
 
 struct Bars {
   uint64_t kv_full;
-  uint64_t q_full[2], q_empty[2], do_full[2], do_empty[2], meta_full[2], meta_empty[2];
+  uint64_t q_full[kQStages], q_empty[kQStages], do_full[2], do_empty[2], meta_full[2], meta_empty[2];
   uint64_t s_full, dp_full, s_free, p_full, dvk_done, final_mma;
   uint32_t tmem_base;
   int32_t abort;
 };
+static_assert(sizeof(Bars) <= 256, "barrier block");
 }  // namespace dkv
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -341,9 +363,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     ptx::mbar_init(&bar->kv_full, 1);
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kQStages; ++s) {
       ptx::mbar_init(&bar->q_full[s], 1);
       ptx::mbar_init(&bar->q_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
       ptx::mbar_init(&bar->do_full[s], 1);
       ptx::mbar_init(&bar->do_empty[s], 1);
       ptx::mbar_init(&bar->meta_full[s], 32);
@@ -369,7 +393,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 8) {
     // ------------------------------------------------ loads (all 32 lanes fill the meta arrays)
-    uint32_t nq[2] = {0, 0}, ndo[2] = {0, 0};
+    uint32_t nq[kQStages] = {0, 0, 0}, ndo[2] = {0, 0};
     const int32_t ky = w.k_base + c * kRows;
     if (lane == 0 && n_it > 0) {
       ptx::mbar_expect_tx(&bar->kv_full, 2 * kTileBytes);
@@ -379,19 +403,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tma_load_2d(smem + OFF_V + kHalfBytes, &tmV, &bar->kv_full, g * kD + 64, ky);
     }
     for (int i = 0; i < n_it; ++i) {
-      const int s = i & 1;
+      const int sq = i % kQStages, s = i & 1;
       const uint32_t n = (uint32_t)(i >> 1);
       const int hh = i / per_head, t = qt0 + i % per_head;
       const int h = g * group + hh;
       const int32_t qy = w.q_base + t * kRows;
       if (aborted(&bar->abort)) break;
       if (lane == 0) {
-        bool ok = i < 2 || wait(&bar->q_empty[s], (n - 1) & 1, a.status);
+        bool ok = i < kQStages || wait(&bar->q_empty[sq], (uint32_t)(i / kQStages - 1) & 1, a.status);
         if (ok) {
-          ptx::mbar_expect_tx(&bar->q_full[s], kTileBytes);
-          ptx::tma_load_2d(smem + OFF_Q + s * kTileBytes, &tmQ, &bar->q_full[s], h * kD, qy);
-          ptx::tma_load_2d(smem + OFF_Q + s * kTileBytes + kHalfBytes, &tmQ, &bar->q_full[s], h * kD + 64, qy);
-          ++nq[s];
+          ptx::mbar_expect_tx(&bar->q_full[sq], kTileBytes);
+          ptx::tma_load_2d(smem + OFF_Q + sq * kTileBytes, &tmQ, &bar->q_full[sq], h * kD, qy);
+          ptx::tma_load_2d(smem + OFF_Q + sq * kTileBytes + kHalfBytes, &tmQ, &bar->q_full[sq], h * kD + 64, qy);
+          ++nq[sq];
           ok = i < 2 || wait(&bar->do_empty[s], (n - 1) & 1, a.status);
         }
         if (ok) {
@@ -424,10 +448,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     if (lane == 0 && aborted(&bar->abort)) {
       if (n_it > 0) wait(&bar->kv_full, 0, a.status);
-      for (int s = 0; s < 2; ++s) {
+      for (int s = 0; s < kQStages; ++s)
         if (nq[s]) wait(&bar->q_full[s], (nq[s] - 1) & 1, a.status);
+      for (int s = 0; s < 2; ++s)
         if (ndo[s]) wait(&bar->do_full[s], (ndo[s] - 1) & 1, a.status);
-      }
     }
   } else if (warp == 9) {
     // ------------------------------------------------ MMA issue
@@ -435,13 +459,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idesc_nt = ptx::idesc_bf16_f32(128, 128, 0, 0);
       constexpr uint32_t idesc_nn = ptx::idesc_bf16_f32(128, 128, 0, 1);
       const uint32_t sK = ptx::smem_u32(smem + OFF_K), sV = ptx::smem_u32(smem + OFF_V);
-      const uint32_t sdS = ptx::smem_u32(smem + OFF_DS);
       bool ok = wait(&bar->kv_full, 0, a.status);
       auto issue_s = [&](int i) -> bool {
-        const int s = i & 1;
-        if (!wait(&bar->q_full[s], (uint32_t)(i >> 1) & 1, a.status)) return false;
+        const int sq = i % kQStages;
+        if (!wait(&bar->q_full[sq], (uint32_t)(i / kQStages) & 1, a.status)) return false;
         ptx::tc_fence_after();
-        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + s * kTileBytes);
+        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + sq * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
           ptx::mma_bf16_ss(tmem + TM_S, desc_kmajor(sK, kk), desc_kmajor(sQ, kk), idesc_nt, kk > 0 ? 1u : 0u);
@@ -461,30 +484,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       if (ok) ok = issue_s(0) && issue_dp(0);
       for (int i = 0; ok && i < n_it; ++i) {
-        const int s = i & 1;
+        const int s = i & 1, sq = i % kQStages;
         if (aborted(&bar->abort)) { ok = false; break; }
         if (i + 1 < n_it) {
           if (!wait(&bar->s_free, (uint32_t)i & 1, a.status) || !issue_s(i + 1)) { ok = false; break; }
         }
         if (!wait(&bar->p_full, (uint32_t)i & 1, a.status)) { ok = false; break; }
         ptx::tc_fence_after();
-        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + s * kTileBytes);
+        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + sq * kTileBytes);
         const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + s * kTileBytes);
-        // dV += P^T dO: P^T in TMEM, queries [0,64) at columns TM_DP + [0,32), [64,128) at TM_DP + 64 + [0,32)
+        // P^T and dS^T (bf16, two queries per column) sit in the dP^T columns: warpgroup wg's
+        // queries [64 wg, 64 wg + 64) have P^T at TM_DP + 64 wg + [0,32) and dS^T at + [32,64)
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
           ptx::mma_bf16_ts(tmem + TM_DV, tmem + TM_DP + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sdO, kk), idesc_nn,
                            (i > 0 || kk > 0) ? 1u : 0u);
-        // dK += dS^T Q
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss(tmem + TM_DK, desc_kmajor(sdS, kk), desc_mnmajor(sQ, kk), idesc_nn,
-                           (i > 0 || kk > 0) ? 1u : 0u);
-        ptx::mma_commit(&bar->q_empty[s]);
+          ptx::mma_bf16_ts(tmem + TM_DK, tmem + TM_DP + 32 + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sQ, kk),
+                           idesc_nn, (i > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma_commit(&bar->q_empty[sq]);
         ptx::mma_commit(&bar->do_empty[s]);
         ptx::mma_commit(&bar->dvk_done);
         if (i + 1 < n_it) {
-          // dP^T of the next tile overwrites the columns P^T was read from
+          // dP^T of the next tile overwrites the P^T / dS^T just read: wait for dV, dK
           if (!wait(&bar->dvk_done, (uint32_t)i & 1, a.status) || !issue_dp(i + 1)) { ok = false; break; }
         }
       }
@@ -497,56 +520,77 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------ compute: thread = key row r, warpgroup wg owns queries [64 wg, 64 wg + 64)
     const int wg = threadIdx.x >> 7, r = threadIdx.x & 127;
     const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
+    const uint32_t tS = tmem + lane_addr + TM_S + 64u * wg, tP = tmem + lane_addr + TM_DP + 64u * wg;
     const float sl2 = a.scale * kLog2e;
     bool ok = true;
     for (int i = 0; ok && i < n_it; ++i) {
       const int s = i & 1;
-      if (!wait(&bar->meta_full[s], (uint32_t)(i >> 1) & 1, a.status) ||
-          !wait(&bar->s_full, (uint32_t)i & 1, a.status) || !wait(&bar->dp_full, (uint32_t)i & 1, a.status)) {
+      if (!wait(&bar->meta_full[s], (uint32_t)(i >> 1) & 1, a.status) || !wait(&bar->s_full, (uint32_t)i & 1, a.status)) {
         ok = false;
         break;
       }
       ptx::tc_fence_after();
-      uint32_t s0[32], s1[32], d0[32], d1[32];
-      ld64(tmem + lane_addr + TM_S + wg * 64, s0, s1);
-      ld64(tmem + lane_addr + TM_DP + wg * 64, d0, d1);
-      ptx::tmem_ld_wait();
-      ptx::reg_fence(s0);
-      ptx::reg_fence(s1);
-      ptx::reg_fence(d0);
-      ptx::reg_fence(d1);
-      ptx::tc_fence_before();
-      ptx::mbar_arrive(&bar->s_free);
       const uint8_t* meta = smem + OFF_META + s * kMetaStage;
-      const float* mlse = reinterpret_cast<const float*>(meta) + wg * 64;
-      const float* mdel = reinterpret_cast<const float*>(meta) + 128 + wg * 64;
-      const uint8_t* mlim = meta + 1024 + wg * 64;
-      uint32_t pp[32], pd[32];
+      const float4* mlse4 = reinterpret_cast<const float4*>(meta) + wg * 16;
+      const float4* mdel4 = reinterpret_cast<const float4*>(meta + 512) + wg * 16;
+      const uint32_t* mlim4 = reinterpret_cast<const uint32_t*>(meta + 1024) + wg * 16;
+      // phase 1: P from S^T (dP^T may still be in flight)
+      uint32_t pp[32];  // pp[k]: queries 64 wg + 2k, 64 wg + 2k + 1 (bf16)
+      {
+        uint32_t sv[2][32];
+        ld64(tS, sv[0], sv[1]);
+        ptx::tmem_ld_wait();
+        ptx::reg_fence(sv[0]);
+        ptx::reg_fence(sv[1]);
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(&bar->s_free);
 #pragma unroll
-      for (int k = 0; k < 32; ++k) {
-        float p[2], d[2];
+        for (int q4 = 0; q4 < 16; ++q4) {
+          const float4 l4 = mlse4[q4];
+          const uint32_t lim = mlim4[q4];
+          const float lv[4] = {l4.x, l4.y, l4.z, l4.w};
+          float p[4];
 #pragma unroll
-        for (int e = 0; e < 2; ++e) {
-          const int jj = 2 * k + e;
-          const float sv = __uint_as_float(jj < 32 ? s0[jj] : s1[jj - 32]);
-          const float dv = __uint_as_float(jj < 32 ? d0[jj] : d1[jj - 32]);
-          p[e] = r < (int)mlim[jj] ? ex2(sv * sl2 - mlse[jj]) : 0.f;
-          d[e] = p[e] * (dv - mdel[jj]);
+          for (int e = 0; e < 4; ++e) {
+            const int vis = (int)((lim >> (8 * e)) & 0xFFu);
+            p[e] = r < vis ? ex2(__uint_as_float(sv[q4 >> 3][(q4 & 7) * 4 + e]) * sl2 - lv[e]) : 0.f;
+          }
+          pp[q4 * 2] = pack_bf16(p[0], p[1]);
+          pp[q4 * 2 + 1] = pack_bf16(p[2], p[3]);
         }
-        pp[k] = pack_bf16(p[0], p[1]);
-        pd[k] = pack_bf16(d[0], d[1]);
+      }
+      // phase 2: dS from dP^T
+      if (!wait(&bar->dp_full, (uint32_t)i & 1, a.status)) { ok = false; break; }
+      ptx::tc_fence_after();
+      uint32_t pd[32];
+      {
+        uint32_t dv[2][32];
+        ld64(tP, dv[0], dv[1]);
+        ptx::tmem_ld_wait();
+        ptx::reg_fence(dv[0]);
+        ptx::reg_fence(dv[1]);
+#pragma unroll
+        for (int q4 = 0; q4 < 16; ++q4) {
+          const float4 d4 = mdel4[q4];
+          const uint32_t w0 = pp[q4 * 2], w1 = pp[q4 * 2 + 1];
+          const int b = (q4 & 7) * 4, hv = q4 >> 3;
+          const float v0 = __uint_as_float(w0 << 16) * (__uint_as_float(dv[hv][b + 0]) - d4.x);
+          const float v1 = __uint_as_float(w0 & 0xFFFF0000u) * (__uint_as_float(dv[hv][b + 1]) - d4.y);
+          const float v2 = __uint_as_float(w1 << 16) * (__uint_as_float(dv[hv][b + 2]) - d4.z);
+          const float v3 = __uint_as_float(w1 & 0xFFFF0000u) * (__uint_as_float(dv[hv][b + 3]) - d4.w);
+          pd[q4 * 2] = pack_bf16(v0, v1);
+          pd[q4 * 2 + 1] = pack_bf16(v2, v3);
+        }
       }
       ptx::mbar_arrive(&bar->meta_empty[s]);
-      // P^T into the first half of this warpgroup's dP^T columns (already read)
-      ptx::tmem_st32(tmem + lane_addr + TM_DP + wg * 64, pp);
+      // P^T and dS^T over this warpgroup's (already read) dP^T columns
+      ptx::tmem_st32(tP, pp);
+      ptx::tmem_st32(tP + 32, pd);
       ptx::tmem_st_wait();
-      if (i >= 1 && !wait(&bar->dvk_done, (uint32_t)(i - 1) & 1, a.status)) { ok = false; break; }
-      store_row_half(smem + OFF_DS, r, wg, pd);
-      ptx::fence_proxy_async_smem();
       ptx::tc_fence_before();
       ptx::mbar_arrive(&bar->p_full);
     }
-    if (ok && n_it > 0) ok = wait(&bar->dvk_done, (uint32_t)(n_it - 1) & 1, a.status);
+    if (ok && n_it > 0) ok = wait(&bar->final_mma, 0, a.status);
     if (!ok) {
       set_abort(&bar->abort);
     } else {
