@@ -76,8 +76,8 @@ constexpr uint32_t TM_S = 0, TM_DP = 256, TM_DQ = 384;  // S regions at 0 and 12
 struct Bars {
   uint64_t qdo_full;
   uint64_t k_full[kKStages], k_empty[kKStages], v_full[2], v_empty[2];
-  uint64_t s_full[2], p_full[2];
-  uint64_t dp_full, dp_read, dq_done, final_mma;
+  uint64_t s_full[2], p_full[2], dq_done[2];  // per S region
+  uint64_t dp_full, dp_read, final_mma;
   uint32_t tmem_base;
   int32_t abort;
 };
@@ -112,10 +112,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::mbar_init(&bar->v_empty[s], 1);
       ptx::mbar_init(&bar->s_full[s], 1);
       ptx::mbar_init(&bar->p_full[s], kComputeThreads);
+      ptx::mbar_init(&bar->dq_done[s], 1);
     }
     ptx::mbar_init(&bar->dp_full, 1);
     ptx::mbar_init(&bar->dp_read, kComputeThreads);
-    ptx::mbar_init(&bar->dq_done, 1);
     ptx::mbar_init(&bar->final_mma, 1);
     bar->abort = 0;
     ptx::fence_mbar_init();
@@ -174,41 +174,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idesc_nt = ptx::idesc_bf16_f32(128, 128, 0, 0);  // A K-major, B K-major
       constexpr uint32_t idesc_nn = ptx::idesc_bf16_f32(128, 128, 0, 1);  // A K-major, B MN-major
       const uint32_t sQ = ptx::smem_u32(smem + OFF_Q), sdO = ptx::smem_u32(smem + OFF_DO);
-      auto issue_s = [&](int c) -> bool {
-        const int sk = c % kKStages;
-        if (!wait(&bar->k_full[sk], (uint32_t)(c / kKStages) & 1, a.status)) return false;
-        ptx::tc_fence_after();
-        const uint32_t sK = ptx::smem_u32(smem + OFF_K + sk * kTileBytes);
+      auto issue_s = [&](int c) {
+        const uint32_t sK = ptx::smem_u32(smem + OFF_K + (c % kKStages) * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
           ptx::mma_bf16_ss(tmem + TM_S + 128u * (c & 1), desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_nt,
                            kk > 0 ? 1u : 0u);
         ptx::mma_commit(&bar->s_full[c & 1]);
-        return true;
       };
-      auto issue_dp = [&](int c) -> bool {
+      auto issue_dp = [&](int c) {
         const int sv = c & 1;
-        if (!wait(&bar->v_full[sv], (uint32_t)(c >> 1) & 1, a.status)) return false;
-        ptx::tc_fence_after();
         const uint32_t sV = ptx::smem_u32(smem + OFF_V + sv * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
           ptx::mma_bf16_ss(tmem + TM_DP, desc_kmajor(sdO, kk), desc_kmajor(sV, kk), idesc_nt, kk > 0 ? 1u : 0u);
         ptx::mma_commit(&bar->dp_full);
         ptx::mma_commit(&bar->v_empty[sv]);
-        return true;
       };
-      bool ok = wait(&bar->qdo_full, 0, a.status);
-      if (ok) ok = issue_s(0) && issue_dp(0);
-      if (ok && nkb > 1) ok = issue_s(1);
-      for (int c = 0; ok && c < nkb; ++c) {
+      auto issue_dq = [&](int c) {
         const int R = c & 1;
-        if (aborted(&bar->abort)) { ok = false; break; }
-        if (c + 1 < nkb) {
-          if (!wait(&bar->dp_read, (uint32_t)c & 1, a.status) || !issue_dp(c + 1)) { ok = false; break; }
-        }
-        if (!wait(&bar->p_full[R], (uint32_t)(c >> 1) & 1, a.status)) { ok = false; break; }
-        ptx::tc_fence_after();
         const uint32_t sK = ptx::smem_u32(smem + OFF_K + (c % kKStages) * kTileBytes);
         // dQ += dS K_c: dS (bf16, keys packed two per column) in S region R, keys [0,64) at
         // columns [0,32) and [64,128) at columns [64,96)
@@ -216,11 +200,54 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int kk = 0; kk < 8; ++kk)
           ptx::mma_bf16_ts(tmem + TM_DQ, tmem + TM_S + 128u * R + 8 * kk + (kk >= 4 ? 32 : 0),
                            desc_mnmajor(sK, kk), idesc_nn, (c > 0 || kk > 0) ? 1u : 0u);
-        ptx::mma_commit(&bar->dq_done);
+        ptx::mma_commit(&bar->dq_done[R]);
         ptx::mma_commit(&bar->k_empty[c % kKStages]);
-        if (c + 2 < nkb) {
-          // S_{c+2} overwrites the dS that dQ_c reads: wait for dQ_c first
-          if (!wait(&bar->dq_done, (uint32_t)c & 1, a.status) || !issue_s(c + 2)) { ok = false; break; }
+      };
+      // Event-driven issue: S_c, dP_c, dQ_c go out as soon as their inputs are
+      // ready, so no wait blocks an unrelated MMA.
+      //   S_c  needs K_c and dQ_{c-2} done (it overwrites the dS that dQ_{c-2} read)
+      //   dP_c needs V_c and dP_{c-1} read by the compute warps
+      //   dQ_c needs dS_c written
+      bool ok = wait(&bar->qdo_full, 0, a.status) && wait(&bar->k_full[0], 0, a.status) &&
+                wait(&bar->v_full[0], 0, a.status);
+      if (ok) {
+        ptx::tc_fence_after();
+        issue_s(0);
+        issue_dp(0);
+      }
+      int ns = 1, nd = 1, nq = 0;
+      uint64_t t_idle = 0;
+      while (ok && nq < nkb) {
+        bool progressed = false;
+        if (ns < nkb && (ns < 2 || nq > ns - 2) &&
+            (ns < 2 || ptx::mbar_test(&bar->dq_done[ns & 1], (uint32_t)((ns - 2) >> 1) & 1)) &&
+            ptx::mbar_test(&bar->k_full[ns % kKStages], (uint32_t)(ns / kKStages) & 1)) {
+          ptx::tc_fence_after();
+          issue_s(ns++);
+          progressed = true;
+        }
+        if (nd < nkb && ptx::mbar_test(&bar->dp_read, (uint32_t)(nd - 1) & 1) &&
+            ptx::mbar_test(&bar->v_full[nd & 1], (uint32_t)(nd >> 1) & 1)) {
+          ptx::tc_fence_after();
+          issue_dp(nd++);
+          progressed = true;
+        }
+        if (nq < ns && nq < nd && ptx::mbar_test(&bar->p_full[nq & 1], (uint32_t)(nq >> 1) & 1)) {
+          ptx::tc_fence_after();
+          issue_dq(nq++);
+          progressed = true;
+        }
+        if (progressed) {
+          t_idle = 0;
+        } else {
+          __nanosleep(16);
+          const uint64_t now = globaltimer();
+          if (t_idle == 0) {
+            t_idle = now;
+          } else if (now - t_idle > kWaitLimitNs || aborted(&bar->abort)) {
+            atomicOr(a.status, kStatusTimeout);
+            ok = false;
+          }
         }
       }
       if (!ok) set_abort(&bar->abort);
