@@ -194,6 +194,11 @@ bool force_cuda_cores() {
   return e && e[0] == '1';
 }
 
+uint32_t tc_flags() {
+  const char* e = getenv("ISM_DRAIN_TMEM_REUSE");
+  return (e && e[0] == '1') ? kFlagDrainTmemReuse : 0u;
+}
+
 bool use_tc(const ism_attn_shape_t* sh) {
   return sh->dtype == ISM_BF16 && sh->head_dim == 128 && tc_available() && !force_cuda_cores();
 }
@@ -346,6 +351,7 @@ ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   a.q_rows = info.total_tokens; a.scale = shape->softmax_scale;
   a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order; a.nq = c.nq;
   a.status = status;
+  a.flags = tc_flags();
   timer_begin(ISM_KERNEL_FWD, st);
   if (use_tc(shape)) {
     ISM_TRY_CUDA(launch_tc_fwd(a, info.total_tokens, st), "tensor-core forward launch");
@@ -387,6 +393,7 @@ ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order; a.nq = c.nq;
   a.ktiles = L.ktiles; a.k_order = L.k_order; a.nk = c.nk;
   a.status = status;
+  a.flags = tc_flags();
   if (use_tc_bwd(shape)) {
     ISM_TRY_CUDA(launch_tc_bwd(a, info.total_tokens, st), "tensor-core backward launch");
   } else {
@@ -526,6 +533,7 @@ ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batc
   a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order;
   a.nq = (int64_t)batch * ((l_new + kTile - 1) / kTile);
   a.status = status;
+  a.flags = tc_flags();
   timer_begin(ISM_KERNEL_FWD, st);
   if (use_tc(shape)) {
     ISM_TRY_CUDA(launch_tc_fwd(a, (int64_t)batch * cache_capacity, st), "tensor-core prefill launch");

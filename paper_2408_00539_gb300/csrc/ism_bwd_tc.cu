@@ -205,7 +205,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       // Event-driven issue: S_c, dP_c, dQ_c go out as soon as their inputs are
       // ready, so no wait blocks an unrelated MMA.
-      //   S_c  needs K_c and dQ_{c-2} done (it overwrites the dS that dQ_{c-2} read)
+      //   S_c  needs K_c and dQ_{c-2} issued (it overwrites the dS that dQ_{c-2}
+      //        reads; MMAs of this thread execute in order, or, with
+      //        kFlagDrainTmemReuse, dQ_{c-2} completed)
       //   dP_c needs V_c and dP_{c-1} read by the compute warps
       //   dQ_c needs dS_c written
       bool ok = wait(&bar->qdo_full, 0, a.status) && wait(&bar->k_full[0], 0, a.status) &&
@@ -220,7 +222,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       while (ok && nq < nkb) {
         bool progressed = false;
         if (ns < nkb && (ns < 2 || nq > ns - 2) &&
-            (ns < 2 || ptx::mbar_test(&bar->dq_done[ns & 1], (uint32_t)((ns - 2) >> 1) & 1)) &&
+            (ns < 2 || !(a.flags & kFlagDrainTmemReuse) ||
+             ptx::mbar_test(&bar->dq_done[ns & 1], (uint32_t)((ns - 2) >> 1) & 1)) &&
             ptx::mbar_test(&bar->k_full[ns % kKStages], (uint32_t)(ns / kKStages) & 1)) {
           ptx::tc_fence_after();
           issue_s(ns++);
@@ -534,8 +537,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::mma_commit(&bar->do_empty[s]);
         ptx::mma_commit(&bar->dvk_done);
         if (i + 1 < n_it) {
-          // dP^T of the next tile overwrites the P^T / dS^T just read: wait for dV, dK
-          if (!wait(&bar->dvk_done, (uint32_t)i & 1, a.status) || !issue_dp(i + 1)) { ok = false; break; }
+          // dP^T of the next tile overwrites the P^T / dS^T that dV, dK read (in
+          // issue order; kFlagDrainTmemReuse waits for dV, dK to complete)
+          if (((a.flags & kFlagDrainTmemReuse) && !wait(&bar->dvk_done, (uint32_t)i & 1, a.status)) ||
+              !issue_dp(i + 1)) {
+            ok = false;
+            break;
+          }
         }
       }
       if (!ok) set_abort(&bar->abort);

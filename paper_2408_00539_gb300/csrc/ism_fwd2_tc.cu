@@ -145,8 +145,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::mma_commit(&bar->k_empty[0]);
       }
       // Per block: PV_A(j), S_A(j+1), PV_B(j), S_B(j+1).  S_x(j+1) overwrites
-      // the P_x(j) that PV_x(j) reads, so it is issued once PV_x(j) is done;
-      // the other head's work keeps the tensor core busy meanwhile.
+      // the P_x(j) that PV_x(j) reads; MMAs issued by this thread execute in
+      // order, so S_x(j+1) follows PV_x(j) without a wait (kFlagDrainTmemReuse
+      // makes it wait for PV_x(j) to complete instead).
       for (int j = 0; ok && j < nkb; ++j) {
         const int s = j & 1, s1 = (j + 1) & 1;
         const bool more = j + 1 < nkb;
@@ -159,7 +160,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           issue_pv(x, j);
           if (x == 1) ptx::mma_commit(&bar->v_empty[s]);
           if (more) {
-            if (!wait(&bar->pv_done[x], (uint32_t)j & 1, a.status)) { ok = false; break; }
+            if ((a.flags & kFlagDrainTmemReuse) && !wait(&bar->pv_done[x], (uint32_t)j & 1, a.status)) {
+              ok = false;
+              break;
+            }
             ptx::tc_fence_after();
             issue_s(x, j + 1);
             if (x == 1) ptx::mma_commit(&bar->k_empty[s1]);

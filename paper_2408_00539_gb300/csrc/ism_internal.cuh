@@ -89,7 +89,12 @@ struct AttnArgs {
   const Tile* qtiles; const int32_t* q_order; int64_t nq;
   const Tile* ktiles; const int32_t* k_order; int64_t nk;
   uint32_t* status;
+  // Bit 0: before an MMA that overwrites tensor memory an earlier MMA reads
+  // as its A operand, wait for that earlier MMA to complete.  Clear: rely on
+  // MMAs issued by one thread executing in issue order.
+  uint32_t flags;
 };
+enum : uint32_t { kFlagDrainTmemReuse = 1u };
 cudaError_t launch_simt_fwd(const AttnArgs& a, cudaStream_t st);
 cudaError_t launch_simt_bwd(const AttnArgs& a, cudaStream_t st);
 

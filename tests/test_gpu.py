@@ -337,3 +337,28 @@ def test_append_16k_prefill_and_decode(ism):
         c_host = c_host + 1
     ism.check_status()
     assert cl.cpu().numpy().tolist() == c_host.tolist()
+
+
+def test_in_order_tmem_reuse_matches_drained_bit_exact(ism, monkeypatch):
+    """The tensor-core kernels issue an MMA that overwrites tensor memory
+    right after the MMA that reads it, relying on MMAs of one thread
+    executing in issue order.  The drained variant (each such MMA waits for
+    the reader to complete) computes the same arithmetic in the same order,
+    so the two must agree bit for bit, run after run."""
+    w = wl.gqa_8k()
+    q, k, v, do = (t.to(DEV) for t in wl.attention_tensors(w))
+    segs = ism.Segments.from_workload(w.segs, DEV)
+
+    def run():
+        o, lse = ism.fwd(segs, q, k, v, w.softmax_scale)
+        dq, dk, dv = ism.bwd(segs, q, k, v, o, lse, do, w.softmax_scale)
+        ism.check_status()
+        return o, lse, dq, dk, dv
+
+    monkeypatch.setenv("ISM_DRAIN_TMEM_REUSE", "1")
+    ref = run()
+    monkeypatch.setenv("ISM_DRAIN_TMEM_REUSE", "0")
+    for _ in range(8):
+        got = run()
+        for name, a_, b_ in zip(("o", "lse", "dq", "dk", "dv"), got, ref):
+            assert torch.equal(a_, b_), name
