@@ -204,22 +204,25 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int i = 0; i < 32; ++i) xs[c * 32 + i] = __uint_as_float(t[c][i]);
         }
       }
-      float mloc = -INFINITY;
+      // row max on the raw scores (the scale is positive), masked keys at -inf;
+      // eight independent partial maxima keep the dependency chain short
+      float mr[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) mr[k] = -INFINITY;
       if (j >= kfull) {
         const int lim = ke - j * kRows;
 #pragma unroll
         for (int c = 0; c < 128; ++c) {
-          xs[c] = c < lim ? xs[c] * sl2 : -INFINITY;
-          mloc = fmaxf(mloc, xs[c]);
+          xs[c] = c < lim ? xs[c] : -INFINITY;
+          mr[c & 7] = fmaxf(mr[c & 7], xs[c]);
         }
       } else {
 #pragma unroll
-        for (int c = 0; c < 128; ++c) {
-          xs[c] *= sl2;
-          mloc = fmaxf(mloc, xs[c]);
-        }
+        for (int c = 0; c < 128; ++c) mr[c & 7] = fmaxf(mr[c & 7], xs[c]);
       }
-      const float m_new = fmaxf(m_use, mloc);
+      const float mraw = fmaxf(fmaxf(fmaxf(mr[0], mr[1]), fmaxf(mr[2], mr[3])),
+                               fmaxf(fmaxf(mr[4], mr[5]), fmaxf(mr[6], mr[7])));
+      const float m_new = fmaxf(m_use, mraw * sl2);
       if (j == 0) {
         m_use = m_new;
       } else if (m_new > m_use + 8.f) {
@@ -240,19 +243,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         m_use = m_new;
       }
-      float rs = 0.f;
-      uint32_t pk[2][32];
+      // P over the first 64 columns of S (already read), 32 columns at a time
+      float rsv[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-      for (int c = 0; c < 64; ++c) {
-        const float p0 = ex2(xs[2 * c] - m_use);
-        const float p1 = ex2(xs[2 * c + 1] - m_use);
-        rs += p0 + p1;
-        pk[c >> 5][c & 31] = pack_bf16(p0, p1);
+      for (int hf = 0; hf < 2; ++hf) {
+        uint32_t pk[32];
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          const float p0 = ex2(fmaf(xs[64 * hf + 2 * c], sl2, -m_use));
+          const float p1 = ex2(fmaf(xs[64 * hf + 2 * c + 1], sl2, -m_use));
+          rsv[c & 3] += p0 + p1;
+          pk[c] = pack_bf16(p0, p1);
+        }
+        ptx::tmem_st32(tS + 32 * hf, pk);
       }
-      l += rs;
-      // P over the first 64 columns of S (already read)
-      ptx::tmem_st32(tS, pk[0]);
-      ptx::tmem_st32(tS + 32, pk[1]);
+      l += (rsv[0] + rsv[1]) + (rsv[2] + rsv[3]);
       ptx::tmem_st_wait();
       ptx::tc_fence_before();
       ptx::mbar_arrive(&bar->p_full[x]);

@@ -205,22 +205,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       ptx::tc_fence_before();
       ptx::mbar_arrive(&bar->s_free[s]);
-      float mloc = -INFINITY;
+      // row max on the raw scores (the scale is positive), masked keys at -inf;
+      // eight independent partial maxima keep the dependency chain short
+      float mr[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) mr[k] = -INFINITY;
       if (j >= kfull) {
         const int lim = ke - j * kRows;
 #pragma unroll
         for (int c = 0; c < 128; ++c) {
-          x[c] = c < lim ? x[c] * sl2 : -INFINITY;
-          mloc = fmaxf(mloc, x[c]);
+          x[c] = c < lim ? x[c] : -INFINITY;
+          mr[c & 7] = fmaxf(mr[c & 7], x[c]);
         }
       } else {
 #pragma unroll
-        for (int c = 0; c < 128; ++c) {
-          x[c] *= sl2;
-          mloc = fmaxf(mloc, x[c]);
-        }
+        for (int c = 0; c < 128; ++c) mr[c & 7] = fmaxf(mr[c & 7], x[c]);
       }
-      const float m_new = fmaxf(m_use, mloc);
+      const float mraw = fmaxf(fmaxf(fmaxf(mr[0], mr[1]), fmaxf(mr[2], mr[3])),
+                               fmaxf(fmaxf(mr[4], mr[5]), fmaxf(mr[6], mr[7])));
+      const float m_new = fmaxf(m_use, mraw * sl2);
       if (j == 0) {
         m_use = m_new;
       } else if (m_new > m_use + 8.f) {
@@ -243,16 +246,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tmem_st_wait();
         m_use = m_new;
       }
-      float rs = 0.f;
+      float rsv[4] = {0.f, 0.f, 0.f, 0.f};
       uint32_t pk[64];
 #pragma unroll
       for (int c = 0; c < 64; ++c) {
-        const float p0 = ex2(x[2 * c] - m_use);
-        const float p1 = ex2(x[2 * c + 1] - m_use);
-        rs += p0 + p1;
+        const float p0 = ex2(fmaf(x[2 * c], sl2, -m_use));
+        const float p1 = ex2(fmaf(x[2 * c + 1], sl2, -m_use));
+        rsv[c & 3] += p0 + p1;
         pk[c] = pack_bf16(p0, p1);
       }
-      l += rs;
+      l += (rsv[0] + rsv[1]) + (rsv[2] + rsv[3]);
       if (j >= 2 && !wait(&bar->p_free[s], (n - 1) & 1, a.status)) { ok = false; break; }
       uint8_t* prow = smem + OFF_P + s * kTileBytes + r * 128;
 #pragma unroll
