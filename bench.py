@@ -350,11 +350,83 @@ def run_cuda(args, w):
         "gpu_launches": int(launches),
         "clocks": clocks.summary(),
     }
+    if not args.no_append:
+        line["append"] = measure_append(dev, read_peaks()[0])
     if world == 1 and not args.no_cpu_baseline:
         val, dt, sample = oracle_sample(w, q, k, v, do, heads_per_sample=4)
         line["cpu_baseline"] = {"value": val, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
                                 "sample": sample, "seconds": dt}
     print(json.dumps(line), flush=True)
+
+
+def measure_append(dev, peaks):
+    """Append-prefill of a 512-token query turn against 8 x 16384 cached
+    tokens, then answer-token decode steps (reported beside the headline;
+    timed with CUDA events per call, caches larger than L2)."""
+    import torch
+    from paper_2408_00539_gb300 import ism
+    a = wl.append_16k()
+    B, cap, hq, hkv, d, ln = a.batch, a.capacity, a.num_heads_q, a.num_heads_kv, a.head_dim, a.l_new
+    g = torch.Generator(device=dev).manual_seed(a.seed)
+    kc = torch.randn((B, cap, hkv, d), generator=g, device=dev, dtype=torch.float32).mul_(a.value_std).bfloat16()
+    vc = torch.randn((B, cap, hkv, d), generator=g, device=dev, dtype=torch.float32).mul_(a.value_std).bfloat16()
+    qn = torch.randn((B, ln, hq, d), generator=g, device=dev).mul_(a.value_std).bfloat16()
+    kn = torch.randn((B, ln, hkv, d), generator=g, device=dev).mul_(a.value_std).bfloat16()
+    vn = torch.randn((B, ln, hkv, d), generator=g, device=dev).mul_(a.value_std).bfloat16()
+    qd = torch.randn((B, 1, hq, d), generator=g, device=dev).mul_(a.value_std).bfloat16()
+    kd = torch.randn((B, 1, hkv, d), generator=g, device=dev).mul_(a.value_std).bfloat16()
+    vd = torch.randn((B, 1, hkv, d), generator=g, device=dev).mul_(a.value_std).bfloat16()
+    c0 = a.cache_len.copy()
+    cl = torch.from_numpy(c0.copy()).to(dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+    # prefill: cache_len is reset before every call (outside the events)
+    pre_ms = []
+    for it in range(8):
+        cl.copy_(torch.from_numpy(c0))
+        flush.fill_(1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        ism.prefill_append(qn, kn, vn, kc, vc, cl, c0, a.new_seg_end, a.new_seg_type, a.softmax_scale)
+        e1.record(stream)
+        e1.synchronize()
+        if it >= 3:
+            pre_ms.append(e0.elapsed_time(e1))
+    ism.check_status(dev)
+    n_vis_pre = int(B * hq * ln * (int(c0[0]) + ln))  # every new row sees the cache and the whole new query
+    pre = float(np.median(pre_ms))
+    # decode steps after the prefill
+    c_host = c0 + ln
+    cl.copy_(torch.from_numpy(c_host))
+    dec_us, dec_kernel_us, dec_bytes = [], [], []
+    for t in range(a.decode_steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        k0, k1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        for e in (k0, k1):
+            e.record(stream)
+        ism.set_kernel_timer(ism.KERNEL_DECODE, k0, k1)
+        e0.record(stream)
+        ism.prefill_append(qd, kd, vd, kc, vc, cl, c_host, [1], [1], a.softmax_scale)
+        e1.record(stream)
+        e1.synchronize()
+        ism.set_kernel_timer(ism.KERNEL_DECODE)
+        dec_us.append(e0.elapsed_time(e1) * 1e3)
+        dec_kernel_us.append(k0.elapsed_time(k1) * 1e3)
+        dec_bytes.append(2 * B * (int(c_host[0]) + 1) * hkv * d * 2)
+        c_host = c_host + 1
+    ism.check_status(dev)
+    us = float(np.median(dec_us[3:]))
+    kus = float(np.median(dec_kernel_us[3:]))
+    gbs = float(np.median(np.array(dec_bytes[3:]) / (np.array(dec_kernel_us[3:]) * 1e-6) / 1e9))
+    return {"workload": a.name,
+            "prefill_ms": pre, "prefill_tflops": 4 * d * n_vis_pre / (pre * 1e-3) / 1e12,
+            "prefill_frac_of_bf16_peak": 4 * d * n_vis_pre / (pre * 1e-3) / 1e12 / peaks["bf16_tflops"],
+            "decode_us_per_call": us, "decode_kernel_us": kus,
+            "decode_hbm_gbs": gbs, "decode_frac_of_hbm": gbs / peaks["hbm_gbs"],
+            "decode_steps": a.decode_steps,
+            "note": "decode bytes = K and V cache read once: 2*B*(c+1)*Hkv*D*2 per step; GB/s over the "
+                    "split-KV + merge kernels (decode_kernel_us); decode_us_per_call adds the plan and "
+                    "cache-write kernels and host launch overhead"}
 
 
 WORKLOADS = {"gqa_8k": wl.gqa_8k, "mha_4k": wl.mha_4k, "packed_32k": wl.packed_32k}
@@ -368,6 +440,7 @@ def main():
     ap.add_argument("--impl", default="cuda", choices=["cuda", "reference"])
     ap.add_argument("--workload", default="gqa_8k", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-append", action="store_true", help="skip the append-prefill / decode measurement")
     ap.add_argument("--profile-step", action="store_true",
                     help="run the warm-up steps and one more step, print nothing (for ncu)")
     args = ap.parse_args()

@@ -509,10 +509,14 @@ ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batc
     a.q = q_new; a.k_cache = k_cache; a.v_cache = v_cache; a.out = o_new; a.lse = lse_new; a.c_snap = L.c_snap;
     a.batch = batch; a.hq = hq; a.hkv = hkv; a.d = d; a.dtype = shape->dtype; a.cap = cache_capacity;
     a.scale = shape->softmax_scale;
-    // enough chunks to give every SM a few CTAs, each chunk a multiple of 64 keys
+    // as many chunks as fill one wave of resident CTAs (4 per SM), each chunk a
+    // multiple of 64 keys
     int64_t kv_max = (int64_t)max_c + 1;
     int64_t pairs = (int64_t)batch * hkv;
-    int64_t want = (4 * 152 + pairs - 1) / pairs;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      sms = 152;
+    int64_t want = (4 * (int64_t)sms) / pairs;
     int64_t splits = want < 1 ? 1 : want > kMaxSplits ? kMaxSplits : want;
     int64_t chunk = (kv_max + splits - 1) / splits;
     chunk = (chunk + 63) / 64 * 64;

@@ -11,7 +11,6 @@ namespace ism {
 namespace {
 
 constexpr int kDecWarps = 4;
-constexpr int kKeysPerIter = 8;
 
 template <int N>
 struct BfVec;
@@ -21,8 +20,7 @@ template <>
 struct BfVec<2> { using T = uint32_t; };
 
 template <int DPL>
-__device__ __forceinline__ void load_bf16(const __nv_bfloat16* p, float (&x)[DPL]) {
-  typename BfVec<DPL>::T raw = *reinterpret_cast<const typename BfVec<DPL>::T*>(p);
+__device__ __forceinline__ void unpack_bf16(const typename BfVec<DPL>::T& raw, float (&x)[DPL]) {
   const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&raw);
 #pragma unroll
   for (int i = 0; i < DPL / 2; ++i) {
@@ -33,10 +31,16 @@ __device__ __forceinline__ void load_bf16(const __nv_bfloat16* p, float (&x)[DPL
 }
 
 // grid (splits, Hkv, B); block kDecWarps warps.  Lane l owns head dims
-// [l*DPL, l*DPL + DPL).
+// [l*DPL, l*DPL + DPL) for the dot products and the output accumulator.
+// A batch covers KPI = 32 / G keys, so the G x KPI partial dot products of a
+// lane are 32 values: a butterfly reduce-scatter (31 shuffles) leaves lane l
+// with the full score of (head l / KPI, key l % KPI); the softmax of a head
+// then runs across its KPI lanes, and the probabilities are broadcast back
+// for O += P V.
 template <int D, int G>
 __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs a) {
   constexpr int DPL = D / 32;
+  constexpr int KPI = 32 / G;  // keys per batch
   const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int hq = a.hq;
@@ -44,6 +48,7 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
   const int k0 = split * a.chunk;
   const int k1 = min(kv_len, k0 + a.chunk);
   const float qscale = a.scale * 1.4426950408889634f;
+  using Raw = typename BfVec<DPL>::T;
 
   const __nv_bfloat16* Q = (const __nv_bfloat16*)a.q;
   const __nv_bfloat16* Kc = (const __nv_bfloat16*)a.k_cache;
@@ -53,84 +58,94 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
   float q[G][DPL];
 #pragma unroll
   for (int h = 0; h < G; ++h) {
-    load_bf16<DPL>(Q + ((int64_t)b * hq + g * G + h) * D + lane * DPL, q[h]);
+    unpack_bf16<DPL>(*reinterpret_cast<const Raw*>(Q + ((int64_t)b * hq + g * G + h) * D + lane * DPL), q[h]);
 #pragma unroll
     for (int i = 0; i < DPL; ++i) q[h][i] *= qscale;
   }
-  float m[G], l[G], o[G][DPL];
+  // running max and sum of this lane's head (uniform across the head's KPI lanes)
+  const int my_h = lane / KPI, my_t = lane % KPI;
+  float m = -INFINITY, l = 0.f;
+  float o[G][DPL];
 #pragma unroll
-  for (int h = 0; h < G; ++h) {
-    m[h] = -INFINITY;
-    l[h] = 0.f;
+  for (int h = 0; h < G; ++h)
 #pragma unroll
     for (int i = 0; i < DPL; ++i) o[h][i] = 0.f;
-  }
 
   const __nv_bfloat16* kbase = Kc + (int64_t)b * a.cap * kstride + (int64_t)g * D + lane * DPL;
   const __nv_bfloat16* vbase = Vc + (int64_t)b * a.cap * kstride + (int64_t)g * D + lane * DPL;
-  for (int kb = k0 + warp * kKeysPerIter; kb < k1; kb += kDecWarps * kKeysPerIter) {
-    float s[G][kKeysPerIter];
+  for (int kb = k0 + warp * KPI; kb < k1; kb += kDecWarps * KPI) {
+    // every K and V row load of the batch is issued before any use; rows past
+    // the chunk re-read its last key and get probability 0
+    Raw kraw[KPI], vraw[KPI];
 #pragma unroll
-    for (int t = 0; t < kKeysPerIter; ++t) {
+    for (int t = 0; t < KPI; ++t) {
+      const int key = min(kb + t, k1 - 1);
+      kraw[t] = *reinterpret_cast<const Raw*>(kbase + (int64_t)key * kstride);
+      vraw[t] = *reinterpret_cast<const Raw*>(vbase + (int64_t)key * kstride);
+    }
+    float v[32];  // v[h * KPI + t]: this lane's partial dot product
+#pragma unroll
+    for (int t = 0; t < KPI; ++t) {
       float kx[DPL];
-      const int key = kb + t;
-      if (key < k1) {
-        load_bf16<DPL>(kbase + (int64_t)key * kstride, kx);
-      } else {
-#pragma unroll
-        for (int i = 0; i < DPL; ++i) kx[i] = 0.f;
-      }
+      unpack_bf16<DPL>(kraw[t], kx);
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         float acc = 0.f;
 #pragma unroll
         for (int i = 0; i < DPL; ++i) acc = fmaf(q[h][i], kx[i], acc);
-        s[h][t] = acc;
+        v[h * KPI + t] = acc;
       }
     }
+    // butterfly reduce-scatter: after the step with offset o a lane keeps the
+    // half of its values selected by lane bit o, plus the partner's partial sums
 #pragma unroll
-    for (int h = 0; h < G; ++h)
+    for (int o = 16; o >= 1; o >>= 1) {
+      const bool hi = (lane & o) != 0;
 #pragma unroll
-      for (int t = 0; t < kKeysPerIter; ++t) {
-        float x = s[h][t];
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) x += __shfl_xor_sync(0xffffffffu, x, off);
-        s[h][t] = (kb + t < k1) ? x : -INFINITY;
+      for (int i = 0; i < o; ++i) {
+        const float send = hi ? v[i] : v[o + i];
+        const float keep = hi ? v[o + i] : v[i];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
       }
-    float p[G][kKeysPerIter];
+    }
+    // lane holds the score of (my_h, my_t); softmax across the head's KPI lanes
+    const float sc = (kb + my_t < k1) ? v[0] : -INFINITY;
+    float mx = sc;
+#pragma unroll
+    for (int off = KPI / 2; off >= 1; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    const float m_new = fmaxf(m, mx);  // finite: key kb is inside the chunk
+    const float p = exp2f(sc - m_new);
+    float ps = p;
+#pragma unroll
+    for (int off = KPI / 2; off >= 1; off >>= 1) ps += __shfl_xor_sync(0xffffffffu, ps, off);
+    const float alpha = exp2f(m - m_new);  // 0 on the first batch (m = -inf)
+    l = l * alpha + ps;
+    m = m_new;
 #pragma unroll
     for (int h = 0; h < G; ++h) {
-      float mx = m[h];
+      const float ah = __shfl_sync(0xffffffffu, alpha, h * KPI);
 #pragma unroll
-      for (int t = 0; t < kKeysPerIter; ++t) mx = fmaxf(mx, s[h][t]);
-      const float alpha = exp2f(m[h] - mx);  // m = -inf on the first batch: alpha = 0
-      float sum = 0.f;
-#pragma unroll
-      for (int t = 0; t < kKeysPerIter; ++t) { p[h][t] = exp2f(s[h][t] - mx); sum += p[h][t]; }
-      l[h] = l[h] * alpha + sum;
-      m[h] = mx;
-#pragma unroll
-      for (int i = 0; i < DPL; ++i) o[h][i] *= alpha;
+      for (int i = 0; i < DPL; ++i) o[h][i] *= ah;
     }
 #pragma unroll
-    for (int t = 0; t < kKeysPerIter; ++t) {
-      const int key = kb + t;
-      if (key >= k1) break;
+    for (int t = 0; t < KPI; ++t) {
       float vx[DPL];
-      load_bf16<DPL>(vbase + (int64_t)key * kstride, vx);
+      unpack_bf16<DPL>(vraw[t], vx);
 #pragma unroll
-      for (int h = 0; h < G; ++h)
+      for (int h = 0; h < G; ++h) {
+        const float pht = __shfl_sync(0xffffffffu, p, h * KPI + t);
 #pragma unroll
-        for (int i = 0; i < DPL; ++i) o[h][i] = fmaf(p[h][t], vx[i], o[h][i]);
+        for (int i = 0; i < DPL; ++i) o[h][i] = fmaf(pht, vx[i], o[h][i]);
+      }
     }
   }
 
   // merge the warps of this CTA
   __shared__ float sm_m[kDecWarps][G], sm_l[kDecWarps][G];
   __shared__ float sm_o[kDecWarps][G][D];
-  if (lane == 0) {
-#pragma unroll
-    for (int h = 0; h < G; ++h) { sm_m[warp][h] = m[h]; sm_l[warp][h] = l[h]; }
+  if (my_t == 0) {
+    sm_m[warp][my_h] = m;
+    sm_l[warp][my_h] = l;
   }
 #pragma unroll
   for (int h = 0; h < G; ++h)
