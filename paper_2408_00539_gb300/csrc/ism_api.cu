@@ -509,14 +509,17 @@ ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batc
     a.q = q_new; a.k_cache = k_cache; a.v_cache = v_cache; a.out = o_new; a.lse = lse_new; a.c_snap = L.c_snap;
     a.batch = batch; a.hq = hq; a.hkv = hkv; a.d = d; a.dtype = shape->dtype; a.cap = cache_capacity;
     a.scale = shape->softmax_scale;
-    // as many chunks as fill one wave of resident CTAs (4 per SM), each chunk a
-    // multiple of 64 keys
+    // chunks of a multiple of 64 keys, as many as fill whole waves of resident
+    // CTAs: 4 per SM for the register kernel (one wave), 2 per SM for the TMA
+    // kernel (four waves, so each CTA's ring runs several tiles)
     int64_t kv_max = (int64_t)max_c + 1;
     int64_t pairs = (int64_t)batch * hkv;
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       sms = 152;
-    int64_t want = (4 * (int64_t)sms) / pairs;
+    const char* no_tma = getenv("ISM_DECODE_NO_TMA");
+    a.tma = (d == 128 && tc_available() && !(no_tma && no_tma[0] == '1')) ? 1 : 0;
+    int64_t want = (a.tma ? 8 * (int64_t)sms : 4 * (int64_t)sms) / pairs;
     int64_t splits = want < 1 ? 1 : want > kMaxSplits ? kMaxSplits : want;
     int64_t chunk = (kv_max + splits - 1) / splits;
     chunk = (chunk + 63) / 64 * 64;
@@ -524,6 +527,7 @@ ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batc
     a.splits = (int32_t)splits;
     a.chunk = (int32_t)chunk;
     a.part_o = L.part_o; a.part_ml = L.part_ml;
+    a.status = status;
     timer_begin(ISM_KERNEL_DECODE, st);
     ISM_TRY_CUDA(launch_decode(a, st), "decode launch");
     timer_end(ISM_KERNEL_DECODE, st);

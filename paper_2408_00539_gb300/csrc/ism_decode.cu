@@ -5,7 +5,10 @@
 // serves all query heads of that KV head's group; a second kernel merges the
 // per-chunk softmax partials.  Scores are kept in base 2 (q pre-scaled by
 // scale * log2 e).
+#include <cstdlib>
+
 #include "ism_internal.cuh"
+#include "ism_tc_common.cuh"
 
 namespace ism {
 namespace {
@@ -172,6 +175,175 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
   }
 }
 
+// TMA-pipelined variant for head_dim 128: warp 4 streams 64-key K and V tiles
+// of the chunk into a 3-stage shared-memory ring with TMA; warps 0-3 each take
+// 16 keys of a tile (batches of 32 / G keys, the same butterfly softmax as
+// above) reading the rows from shared memory.  Two CTAs fit on an SM, so
+// about six 32 KB tiles are in flight per SM.
+constexpr int kTmaTile = 64;
+constexpr int kTmaStages = 3;
+constexpr uint32_t kTmaHalf = kTmaTile * 128;       // 64 rows x 64 bf16
+constexpr uint32_t kTmaStageBytes = 4 * kTmaHalf;   // K and V, two halves each
+
+template <int G>
+__global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__ CUtensorMap tmK,
+                                                        const __grid_constant__ CUtensorMap tmV, DecodeArgs a) {
+  constexpr int D = 128, DPL = 4, KPI = 32 / G, NB = 16 / KPI;  // batches per warp per tile
+  extern __shared__ __align__(128) uint8_t dsm[];
+  uint64_t* full = reinterpret_cast<uint64_t*>(dsm + kTmaStages * kTmaStageBytes);
+  uint64_t* empty = full + kTmaStages;
+  float* sm_m = reinterpret_cast<float*>(empty + kTmaStages);  // [4][G]
+  float* sm_l = sm_m + 4 * G;                                   // [4][G]
+  float* sm_o = sm_l + 4 * G;                                   // [4][G][D]
+  const int split = blockIdx.x, g = blockIdx.y, b = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int kv_len = a.c_snap[b] + 1;
+  const int k0 = split * a.chunk;
+  const int k1 = min(kv_len, k0 + a.chunk);
+  const int ntiles = k1 > k0 ? (k1 - k0 + kTmaTile - 1) / kTmaTile : 0;
+  const int32_t row0 = (int32_t)((int64_t)b * a.cap + k0);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kTmaStages; ++s) {
+      ptx::mbar_init(&full[s], 1);
+      ptx::mbar_init(&empty[s], 4);
+    }
+    ptx::fence_mbar_init();
+  }
+  __syncthreads();
+  if (warp == 4) {
+    if (lane == 0) {
+      int issued = 0;
+      for (int t = 0; t < ntiles; ++t) {
+        const int s = t % kTmaStages;
+        if (t >= kTmaStages && !tc::wait(&empty[s], (uint32_t)(t / kTmaStages - 1) & 1, a.status)) break;
+        issued = t + 1;
+        uint8_t* st = dsm + s * kTmaStageBytes;
+        const int32_t y = row0 + t * kTmaTile;
+        ptx::mbar_expect_tx(&full[s], kTmaStageBytes);
+        ptx::tma_load_2d(st, &tmK, &full[s], g * D, y);
+        ptx::tma_load_2d(st + kTmaHalf, &tmK, &full[s], g * D + 64, y);
+        ptx::tma_load_2d(st + 2 * kTmaHalf, &tmV, &full[s], g * D, y);
+        ptx::tma_load_2d(st + 3 * kTmaHalf, &tmV, &full[s], g * D + 64, y);
+      }
+      // every issued copy completes before the CTA exits
+      for (int t = issued - kTmaStages > 0 ? issued - kTmaStages : 0; t < issued; ++t)
+        tc::wait(&full[t % kTmaStages], (uint32_t)(t / kTmaStages) & 1, a.status);
+    }
+  } else {
+    const float qscale = a.scale * 1.4426950408889634f;
+    const __nv_bfloat16* Q = (const __nv_bfloat16*)a.q;
+    float q[G][DPL];
+#pragma unroll
+    for (int h = 0; h < G; ++h) {
+      unpack_bf16<DPL>(*reinterpret_cast<const uint2*>(Q + ((int64_t)b * a.hq + g * G + h) * D + lane * DPL), q[h]);
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) q[h][i] *= qscale;
+    }
+    const int my_h = lane / KPI, my_t = lane % KPI;
+    float m = -INFINITY, l = 0.f;
+    float o[G][DPL];
+#pragma unroll
+    for (int h = 0; h < G; ++h)
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) o[h][i] = 0.f;
+    // lane's 8 bytes of a row: half lane/16, bytes (lane % 16) * 8
+    const uint32_t lane_off = (uint32_t)(lane >> 4) * kTmaHalf + (uint32_t)(lane & 15) * 8;
+    for (int t = 0; t < ntiles; ++t) {
+      const int s = t % kTmaStages;
+      if (!tc::wait(&full[s], (uint32_t)(t / kTmaStages) & 1, a.status)) break;
+      const uint8_t* st = dsm + s * kTmaStageBytes;
+#pragma unroll
+      for (int nb = 0; nb < NB; ++nb) {
+        const int r0 = warp * 16 + nb * KPI;           // first row of the batch in the tile
+        const int kb = k0 + t * kTmaTile + r0;         // its key index
+        float v[32];
+#pragma unroll
+        for (int tt = 0; tt < KPI; ++tt) {
+          float kx[DPL];
+          unpack_bf16<DPL>(*reinterpret_cast<const uint2*>(st + lane_off + (uint32_t)(r0 + tt) * 128), kx);
+#pragma unroll
+          for (int h = 0; h < G; ++h) {
+            float acc = 0.f;
+#pragma unroll
+            for (int i = 0; i < DPL; ++i) acc = fmaf(q[h][i], kx[i], acc);
+            v[h * KPI + tt] = acc;
+          }
+        }
+#pragma unroll
+        for (int o2 = 16; o2 >= 1; o2 >>= 1) {
+          const bool hi = (lane & o2) != 0;
+#pragma unroll
+          for (int i = 0; i < o2; ++i) {
+            const float send = hi ? v[i] : v[o2 + i];
+            const float keep = hi ? v[o2 + i] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o2);
+          }
+        }
+        const float sc = (kb + my_t < k1) ? v[0] : -INFINITY;
+        float mx = sc;
+#pragma unroll
+        for (int off = KPI / 2; off >= 1; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+        if (mx == -INFINITY) continue;  // the whole batch lies past the chunk (uniform per head group)
+        const float m_new = fmaxf(m, mx);
+        const float p = exp2f(sc - m_new);
+        float ps = p;
+#pragma unroll
+        for (int off = KPI / 2; off >= 1; off >>= 1) ps += __shfl_xor_sync(0xffffffffu, ps, off);
+        const float alpha = exp2f(m - m_new);
+        l = l * alpha + ps;
+        m = m_new;
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+          const float ah = __shfl_sync(0xffffffffu, alpha, h * KPI);
+#pragma unroll
+          for (int i = 0; i < DPL; ++i) o[h][i] *= ah;
+        }
+#pragma unroll
+        for (int tt = 0; tt < KPI; ++tt) {
+          float vx[DPL];
+          unpack_bf16<DPL>(*reinterpret_cast<const uint2*>(st + 2 * kTmaHalf + lane_off + (uint32_t)(r0 + tt) * 128),
+                           vx);
+#pragma unroll
+          for (int h = 0; h < G; ++h) {
+            const float pht = __shfl_sync(0xffffffffu, p, h * KPI + tt);
+#pragma unroll
+            for (int i = 0; i < DPL; ++i) o[h][i] = fmaf(pht, vx[i], o[h][i]);
+          }
+        }
+      }
+      __syncwarp();
+      if (lane == 0) ptx::mbar_arrive(&empty[s]);
+    }
+    if (my_t == 0) {
+      sm_m[warp * G + my_h] = m;
+      sm_l[warp * G + my_h] = l;
+    }
+#pragma unroll
+    for (int h = 0; h < G; ++h)
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) sm_o[(warp * G + h) * D + lane * DPL + i] = o[h][i];
+  }
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < G * D; idx += blockDim.x) {
+    const int h = idx / D, d = idx % D;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) M = fmaxf(M, sm_m[w * G + h]);
+    float acc = 0.f, lsum = 0.f;
+    if (M != -INFINITY) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w) {
+        const float f = exp2f(sm_m[w * G + h] - M);
+        acc = fmaf(sm_o[(w * G + h) * D + d], f, acc);
+        lsum = fmaf(sm_l[w * G + h], f, lsum);
+      }
+    }
+    const int64_t pidx = ((int64_t)b * a.hq + g * G + h) * a.splits + split;
+    a.part_o[pidx * D + d] = acc;
+    if (d == 0) { a.part_ml[pidx * 2] = M; a.part_ml[pidx * 2 + 1] = lsum; }
+  }
+}
+
 // grid B*Hq, block D threads.
 template <int D>
 __global__ void decode_combine_kernel(DecodeArgs a) {
@@ -198,8 +370,21 @@ __global__ void decode_combine_kernel(DecodeArgs a) {
 template <int D, int G>
 cudaError_t run(const DecodeArgs& a, cudaStream_t st) {
   dim3 grid(a.splits, a.hkv, a.batch);
-  decode_split_kernel<D, G><<<grid, kDecWarps * 32, 0, st>>>(a);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e;
+  if (a.tma) {
+    CUtensorMap tk, tv;
+    const uint64_t rows = (uint64_t)a.batch * a.cap;
+    if ((e = tc::make_tmap_bf16_plain(&tk, a.k_cache, (uint64_t)a.hkv * D, rows, kTmaTile)) != cudaSuccess) return e;
+    if ((e = tc::make_tmap_bf16_plain(&tv, a.v_cache, (uint64_t)a.hkv * D, rows, kTmaTile)) != cudaSuccess) return e;
+    const int smem = kTmaStages * kTmaStageBytes + 2 * kTmaStages * 8 + (8 * G + 4 * G * D) * 4;
+    if ((e = cudaFuncSetAttribute(decode_tma_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) !=
+        cudaSuccess)
+      return e;
+    decode_tma_kernel<G><<<grid, 160, smem, st>>>(tk, tv, a);
+  } else {
+    decode_split_kernel<D, G><<<grid, kDecWarps * 32, 0, st>>>(a);
+  }
+  e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   decode_combine_kernel<D><<<a.batch * a.hq, D, 0, st>>>(a);
   return cudaGetLastError();

@@ -112,6 +112,8 @@ struct DecodeArgs {
   int32_t splits, chunk;
   float* part_o;         // [B, Hq, splits, D]
   float* part_ml;        // [B, Hq, splits, 2]
+  int32_t tma;           // stream the cache with TMA (head_dim 128, sm_103)
+  uint32_t* status;      // device status word (bounded waits)
 };
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st);
 
