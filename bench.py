@@ -236,12 +236,16 @@ def run_cuda(args, w):
     D = w.head_dim
     flops = 14 * D * n_vis
     o, lse = ism.fwd(segs, qd, kd, vd, w.softmax_scale)
-    dq, dk, dv = ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale)
+    # backward workspace sized for the stored-dS schedule where it applies
+    ws_bytes = ism.bwd_workspace_size(segs, qd, kd, w.softmax_scale)
+    stored_ds = ws_bytes > ism.bwd_workspace_size(segs, qd, kd, w.softmax_scale, minimal=True)
+    ws_b = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    dq, dk, dv = ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, workspace=ws_b)
     flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
 
     def step():
         ism.fwd(segs, qd, kd, vd, w.softmax_scale, out=o, lse=lse)
-        ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, dq=dq, dk=dk, dv=dv)
+        ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws_b)
 
     for _ in range(args.warmup):
         step()
@@ -292,7 +296,8 @@ def run_cuda(args, w):
 
     # dominant kernel: largest share of the step
     mean_k = {n: float(np.mean(t)) for n, t in ktimes.items()}
-    kflops = {"fwd": 4 * D * n_vis, "bwd_dkdv": 8 * D * n_vis, "bwd_dq": 6 * D * n_vis}
+    # dQ recomputes S and dP (6 flops/D per pair) unless dS was stored (2)
+    kflops = {"fwd": 4 * D * n_vis, "bwd_dkdv": 8 * D * n_vis, "bwd_dq": (2 if stored_ds else 6) * D * n_vis}
     dom = max(kflops, key=lambda n: mean_k[n])
     peak = peaks.get("bf16_tflops_sustained" if args.steps * ms_per_step > 2000 else "bf16_tflops")
     achieved = kflops[dom] / (mean_k[dom] * 1e-3) / 1e12
@@ -320,7 +325,7 @@ def run_cuda(args, w):
             dod.copy_(doh, non_blocking=True)
         ism.fwd(segs, qd, kd, vd, w.softmax_scale, out=o, lse=lse)
         stream.wait_stream(copy_stream)
-        ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, dq=dq, dk=dk, dv=dv)
+        ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws_b)
         dqh.copy_(dq, non_blocking=True)
         dkh.copy_(dk, non_blocking=True)
         dvh.copy_(dv, non_blocking=True)
@@ -350,7 +355,8 @@ def run_cuda(args, w):
                    "flops_per_step": flops, "flop_count": "14*D*N_vis (fwd 4, bwd 10)",
                    "strict_tflops_12D": value * 12 / 14, "l2": "flushed between timed steps (258 MB write)",
                    "pct_of_peak": value / peak * 100, "path": "tensor cores" if ism.has_tensor_cores()
-                   else "cuda cores", "parallelism": f"replicas x{world}"},
+                   else "cuda cores", "bwd_schedule": "stored dS" if stored_ds else "recompute dQ",
+                   "bwd_workspace_bytes": ws_bytes, "parallelism": f"replicas x{world}"},
         "kernel_ms": mean_k,
         "roofline": roofline,
         "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,

@@ -160,9 +160,24 @@ ism_status_t ism_attn_fwd_noalloc(const ism_segments_t* segs, const ism_attn_sha
  * forward's O and LSE.  dq [T, Hq, D], dk/dv [T, Hkv, D] (dtype, written;
  * dk/dv summed over the query heads that share a KV head).  Standard
  * softmax-attention calculus over the Eq. (e_ISM) mask.
+ *
+ * Two schedules, chosen by the workspace the caller passes:
+ *  - stored-dS (bf16, head_dim 128, tensor cores): the dK/dV kernel also
+ *    keeps every visible 128x128 tile of dS^T (bf16) in the workspace and dQ
+ *    is a GEMM over those tiles; 32 KiB per visible (query tile, key tile,
+ *    query head) on top of the minimum.  Taken when workspace_bytes is at
+ *    least ism_attn_bwd_workspace_size; ISM_BWD_RECOMPUTE_DQ=1 in the
+ *    environment disables it.
+ *  - recompute: the dQ kernel recomputes S, P and dP; needs only
+ *    ism_attn_bwd_workspace_size_min bytes.
+ * ism_attn_bwd_workspace_size reports the stored-dS size where that schedule
+ * applies and the minimum otherwise.  Both schedules give dQ from the same
+ * bf16-rounded dS, so they differ only in fp32 summation order.
  * ------------------------------------------------------------------------- */
 ism_status_t ism_attn_bwd_workspace_size(const ism_segments_t* segs, const ism_attn_shape_t* shape,
                                          size_t* bytes);
+ism_status_t ism_attn_bwd_workspace_size_min(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                                             size_t* bytes);
 ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* shape,
                           const void* q, const void* k, const void* v, const void* o,
                           const float* lse, const void* dout,
@@ -242,7 +257,9 @@ uint64_t ism_kernel_launches(void);
  *   mode 0/2/4: b [128,128] is N x K and c = a * b^T
  *   mode 1/3/5: b [128,128] is K x N and c = a * b
  *   modes 0/1 stage the operands with plain stores, 2/3 with TMA, 4/5 put
- *   a in tensor memory (the A-from-TMEM form of the MMA). */
+ *   a in tensor memory (the A-from-TMEM form of the MMA)
+ *   mode 6: a [128,128] is K x M and b is K x N (both MN-major), c = a^T * b
+ *   mode 7: as mode 6, a staged in the 8-interleaved layout without swizzle. */
 ism_status_t ism_debug_mma_tile(const void* a, const void* b, float* c, int32_t mode, ism_stream_t stream);
 
 const char* ism_status_string(ism_status_t status);

@@ -167,16 +167,43 @@ Counts count_tiles(const ism_segments_t* s, int bm, int bn) {
   return c;
 }
 
-// Workspace of the one-pass forward/backward.
+// Visible (k-tile, q-tile) pairs over all sequences at kTile x kTile tiles:
+// k-tile c pairs with every q-tile from the one holding the first row whose
+// kv_end exceeds c*kTile to the last.  Under Eq. fj that row is the start of
+// the first segment ending after c*kTile when it is a query segment, else
+// max(segment start, c*kTile).  Host walk over segments and k-tiles.
+int64_t count_pairs(const ism_segments_t* s) {
+  int64_t pairs = 0;
+  for (int b = 0; b < s->num_seqs; ++b) {
+    const int32_t L = s->cu_seqlens_host[b + 1] - s->cu_seqlens_host[b];
+    const int32_t nt = (L + kTile - 1) / kTile;
+    int32_t seg = s->cu_segs_host[b], start = 0;
+    const int32_t seg1 = s->cu_segs_host[b + 1];
+    for (int32_t c = 0; c < nt; ++c) {
+      const int32_t x = c * kTile;
+      while (seg < seg1 && s->seg_end_host[seg] <= x) start = s->seg_end_host[seg++];
+      if (seg == seg1) break;
+      const int32_t j = s->seg_type_host[seg] == ISM_SEG_QUERY ? start : (x > start ? x : start);
+      pairs += nt - j / kTile;
+    }
+  }
+  return pairs;
+}
+
+// Workspace of the one-pass forward/backward.  ds_slots > 0 adds the
+// stored-dS backward's pair offsets and bf16 dS^T tiles (32 KiB a slot).
 struct PassLayout {
   int32_t* kv_end;
   Tile *qtiles, *ktiles;
   int32_t *q_order, *k_order;
   float* delta;
+  int32_t* kpair_off;
+  void* ds;
   size_t bytes;
 };
 
-PassLayout pass_layout(void* ws, const ism_segments_t* s, const Counts& c, int64_t T, int hq, bool bwd) {
+PassLayout pass_layout(void* ws, const ism_segments_t* s, const Counts& c, int64_t T, int hq, bool bwd,
+                       int64_t ds_slots = 0) {
   Carve cv(ws);
   PassLayout L;
   L.kv_end = cv.take<int32_t>(T);
@@ -185,6 +212,8 @@ PassLayout pass_layout(void* ws, const ism_segments_t* s, const Counts& c, int64
   L.ktiles = bwd ? cv.take<Tile>(c.nk) : nullptr;
   L.k_order = bwd ? cv.take<int32_t>(c.nk) : nullptr;
   L.delta = bwd ? cv.take<float>((int64_t)hq * T) : nullptr;
+  L.kpair_off = ds_slots > 0 ? cv.take<int32_t>(c.nk) : nullptr;
+  L.ds = ds_slots > 0 ? static_cast<void*>(cv.take<uint16_t>(ds_slots * kTile * kTile)) : nullptr;
   L.bytes = ((cv.off + 255) & ~size_t(255)) + 256;
   return L;
 }
@@ -204,6 +233,18 @@ bool use_tc(const ism_attn_shape_t* sh) {
 }
 bool use_tc_bwd(const ism_attn_shape_t* sh) { return use_tc(sh) && tc_bwd_available(); }
 
+// dS tile slots of the stored-dS backward (pairs x query heads), or 0 where
+// that path does not apply: CUDA-core backward, ISM_BWD_RECOMPUTE_DQ=1, or
+// more pairs than the 32-bit pair offsets hold.
+int64_t stored_ds_slots(const ism_segments_t* s, const ism_attn_shape_t* sh) {
+  if (!use_tc_bwd(sh)) return 0;
+  const char* e = getenv("ISM_BWD_RECOMPUTE_DQ");
+  if (e && e[0] == '1') return 0;
+  const int64_t pairs = count_pairs(s);
+  if (pairs >= (int64_t(1) << 31)) return 0;
+  return pairs * sh->num_heads_q;
+}
+
 ism_status_t check_ws(void* ws, size_t have, size_t need) {
   if (have < need) return fail(ISM_ERR_WORKSPACE, "workspace of %zu bytes, %zu required", have, need);
   if (need && !ws) return fail(ISM_ERR_WORKSPACE, "workspace is NULL");
@@ -221,8 +262,9 @@ ism_status_t build_pass_meta(const ism_segments_t* s, const Counts& c, const Pas
                "tiles launch");
   ISM_TRY_CUDA(launch_order(L.qtiles, c.nq, L.ktiles, bwd ? c.nk : 0, c.max_cost, L.q_order, L.k_order, st),
                "order launch");
+  if (L.kpair_off) ISM_TRY_CUDA(launch_pair_offsets(L.ktiles, c.nk, L.kpair_off, st), "pair offsets launch");
   timer_end(ISM_KERNEL_META, st);
-  count_launch(s->num_segs > 0 ? 3 : 2);
+  count_launch((s->num_segs > 0 ? 3 : 2) + (L.kpair_off && c.nk ? 1 : 0));
   return ISM_OK;
 }
 
@@ -322,6 +364,19 @@ ism_status_t ism_attn_bwd_workspace_size(const ism_segments_t* segs, const ism_a
   if ((r = check_shape(shape)) != ISM_OK) return r;
   if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
   Counts c = count_tiles(segs, kTile, kTile);
+  *bytes = pass_layout(nullptr, segs, c, info.total_tokens, shape->num_heads_q, true, stored_ds_slots(segs, shape))
+               .bytes;
+  return ISM_OK;
+}
+
+ism_status_t ism_attn_bwd_workspace_size_min(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                                             size_t* bytes) {
+  SegInfo info;
+  ism_status_t r = check_segments(segs, &info);
+  if (r != ISM_OK) return r;
+  if ((r = check_shape(shape)) != ISM_OK) return r;
+  if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
+  Counts c = count_tiles(segs, kTile, kTile);
   *bytes = pass_layout(nullptr, segs, c, info.total_tokens, shape->num_heads_q, true).bytes;
   return ISM_OK;
 }
@@ -378,7 +433,11 @@ ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   for (const void* p : ptrs)
     if (!aligned16(p)) return fail(ISM_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
   Counts c = count_tiles(segs, kTile, kTile);
-  PassLayout L = pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, true);
+  // the stored-dS path when the workspace holds its tiles, else recompute
+  const int64_t slots = stored_ds_slots(segs, shape);
+  PassLayout L = pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, true, slots);
+  if (slots > 0 && workspace_bytes < L.bytes)
+    L = pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, true);
   if ((r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
   uint32_t* status;
   if ((r = status_ptr(&status)) != ISM_OK) return r;
@@ -392,6 +451,7 @@ ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   a.q_rows = info.total_tokens; a.scale = shape->softmax_scale;
   a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order; a.nq = c.nq;
   a.ktiles = L.ktiles; a.k_order = L.k_order; a.nk = c.nk;
+  a.ds = L.ds; a.kpair_off = L.kpair_off; a.ds_slots = L.ds ? slots : 0;
   a.status = status;
   a.flags = tc_flags();
   if (use_tc_bwd(shape)) {
@@ -574,7 +634,7 @@ ism_status_t ism_check_status(ism_stream_t stream) {
 }
 
 ism_status_t ism_debug_mma_tile(const void* a, const void* b, float* c, int32_t mode, ism_stream_t stream) {
-  if (!a || !b || !c || mode < 0 || mode > 5) return fail(ISM_ERR_INVALID_ARG, "a, b, c non-NULL and mode 0..5");
+  if (!a || !b || !c || mode < 0 || mode > 7) return fail(ISM_ERR_INVALID_ARG, "a, b, c non-NULL and mode 0..7");
   if (!tc_available()) return fail(ISM_ERR_UNSUPPORTED, "tensor-core kernels need an sm_103 device");
   uint32_t* status;
   ism_status_t r = status_ptr(&status);

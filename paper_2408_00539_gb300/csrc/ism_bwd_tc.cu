@@ -384,7 +384,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     return;
   }
   const int g = blockIdx.x % a.hkv;
-  const Tile w = a.ktiles[a.k_order[blockIdx.x / a.hkv]];
+  const int gk = a.k_order[blockIdx.x / a.hkv];  // global k-tile index
+  const Tile w = a.ktiles[gk];
   const int group = a.hq / a.hkv;
   const int qt0 = w.a0, nqt = w.a1;
   const int per_head = nqt - qt0;
@@ -621,6 +622,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       // P^T and dS^T over this warpgroup's (already read) dP^T columns
       ptx::tmem_st32(tP, pp);
       ptx::tmem_st32(tP + 32, pd);
+      if (a.ds) {
+        // keep dS^T row r, queries [64 wg, 64 wg + 64), for the dQ GEMM, in
+        // the 8-interleaved layout (16-byte unit (query group, key)): the 32
+        // lanes of a warp store 512 contiguous bytes per instruction
+        const int hh = i / per_head, t = qt0 + i % per_head;
+        const int64_t slot = ((int64_t)a.kpair_off[gk] + (t - qt0)) * a.hq + (g * group + hh);
+        uint4* dst = reinterpret_cast<uint4*>(static_cast<uint8_t*>(a.ds) + slot * kTileBytes) + wg * 8 * kRows + r;
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          dst[k * kRows] = make_uint4(pd[4 * k], pd[4 * k + 1], pd[4 * k + 2], pd[4 * k + 3]);
+      }
       ptx::tmem_st_wait();
       ptx::tc_fence_before();
       ptx::mbar_arrive(&bar->p_full);
@@ -691,7 +703,9 @@ cudaError_t launch_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) {
   if ((e = make_tmap_bf16(&tdo, a.dout, (uint64_t)a.hq * kD, (uint64_t)a.q_rows)) != cudaSuccess) return e;
   if ((e = make_tmap_bf16(&tk, a.k, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;
   if ((e = make_tmap_bf16(&tv, a.v, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;
-  if (a.nq) {
+  // Recompute path: dQ recomputes S, P and dP itself and runs before dK/dV.
+  // Stored-dS path: dK/dV writes the dS^T tiles, then dQ is a GEMM over them.
+  if (a.nq && !a.ds) {
     if ((e = cudaFuncSetAttribute(dq_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dq::kSmemBytes)) !=
         cudaSuccess)
       return e;
@@ -710,6 +724,12 @@ cudaError_t launch_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) {
     timer_end(ISM_KERNEL_BWD_DKDV, st);
     count_launch();
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  if (a.nq && a.ds) {
+    timer_begin(ISM_KERNEL_BWD_DQ, st);
+    if ((e = launch_dq_gemm(a, tk, st)) != cudaSuccess) return e;
+    timer_end(ISM_KERNEL_BWD_DQ, st);
+    count_launch();
   }
   return cudaSuccess;
 }

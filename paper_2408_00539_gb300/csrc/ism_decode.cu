@@ -99,16 +99,16 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
         v[h * KPI + t] = acc;
       }
     }
-    // butterfly reduce-scatter: after the step with offset o a lane keeps the
-    // half of its values selected by lane bit o, plus the partner's partial sums
+    // butterfly reduce-scatter: after the step with offset sh a lane keeps the
+    // half of its values selected by lane bit sh, plus the partner's partial sums
 #pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) {
-      const bool hi = (lane & o) != 0;
+    for (int sh = 16; sh >= 1; sh >>= 1) {
+      const bool hi = (lane & sh) != 0;
 #pragma unroll
-      for (int i = 0; i < o; ++i) {
-        const float send = hi ? v[i] : v[o + i];
-        const float keep = hi ? v[o + i] : v[i];
-        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+      for (int i = 0; i < sh; ++i) {
+        const float send = hi ? v[i] : v[sh + i];
+        const float keep = hi ? v[sh + i] : v[i];
+        v[i] = keep + __shfl_xor_sync(0xffffffffu, send, sh);
       }
     }
     // lane holds the score of (my_h, my_t); softmax across the head's KPI lanes

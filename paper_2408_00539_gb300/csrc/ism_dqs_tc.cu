@@ -1,0 +1,171 @@
+// dQ of ISM attention as a GEMM over stored dS tiles (sm_103a).
+//
+// When the dK/dV kernel has kept every visible tile pair's dS (bf16, 128
+// queries x 128 keys, 32 KiB a tile) in the workspace, dQ_t = scale *
+// sum_c dS_tc K_c needs no recomputation of S, P or dP: one CTA per (query
+// tile, query head) streams the (dS, K) tile pairs of the tile's non-empty
+// key blocks through a 3-stage ring and accumulates dQ in tensor memory.
+// A dS tile is stored 8-interleaved (16-byte units of 8 consecutive queries
+// of one key, the 128 keys of a query group adjacent), which is the no-swizzle
+// MN-major operand layout: one contiguous bulk copy moves it into shared
+// memory as the A operand (M = queries).  K arrives by TMA in the 128-byte
+// swizzled layout as the MN-major B operand.
+// Warps 0-3 epilogue (thread = query row), warp 4 copy producer, warp 5 MMA.
+#include "ism_tc_common.cuh"
+
+namespace ism {
+namespace tc {
+namespace {
+
+constexpr int kThreads = 192;
+constexpr int kStages = 3;
+constexpr uint32_t kStageBytes = 2 * kTileBytes;  // dS^T tile + K tile
+constexpr uint32_t OFF_BAR = kStages * kStageBytes;
+constexpr uint32_t kSmemBytes = OFF_BAR + 128 + 1024;
+constexpr uint32_t kTmemCols = 128;
+
+struct Bars {
+  uint64_t full[kStages], empty[kStages], done;
+  uint32_t tmem_base;
+  int32_t abort;
+};
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+__device__ __forceinline__ bool aborted(const int32_t* f) { return *reinterpret_cast<const volatile int32_t*>(f) != 0; }
+__device__ __forceinline__ void set_abort(int32_t* f) { *reinterpret_cast<volatile int32_t*>(f) = 1; }
+
+__global__ void __launch_bounds__(kThreads, 1)
+    dq_gemm_kernel(const __grid_constant__ CUtensorMap tmK, const AttnArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  Bars* bar = reinterpret_cast<Bars*>(smem + OFF_BAR);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.x % a.hq;
+  const int gq = a.q_order[blockIdx.x / a.hq];
+  const Tile w = a.qtiles[gq];
+  const int g = h / (a.hq / a.hkv);
+  const int nkb = w.a1, t = w.tile;
+  const int gfirst = gq - t;  // q-tiles and k-tiles of a sequence are numbered alike
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      ptx::mbar_init(&bar->full[s], 1);
+      ptx::mbar_init(&bar->empty[s], 1);
+    }
+    ptx::mbar_init(&bar->done, 1);
+    bar->abort = 0;
+    ptx::fence_mbar_init();
+  }
+  if (warp == 5) {
+    ptx::tmem_alloc(&bar->tmem_base, kTmemCols);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = bar->tmem_base;
+
+  if (warp == 4) {
+    if (lane == 0 && nkb > 0) {
+      uint32_t nf[kStages] = {0, 0, 0};
+      for (int c = 0; c < nkb; ++c) {
+        const int s = c % kStages;
+        if (aborted(&bar->abort)) break;
+        if (c >= kStages && !wait(&bar->empty[s], (uint32_t)(c / kStages - 1) & 1, a.status)) {
+          set_abort(&bar->abort);
+          break;
+        }
+        const int gk = gfirst + c;
+        const int64_t slot = ((int64_t)a.kpair_off[gk] + (t - a.ktiles[gk].a0)) * a.hq + h;
+        const int32_t yk = w.k_base + c * kRows;
+        uint8_t* st = smem + s * kStageBytes;
+        ptx::mbar_expect_tx(&bar->full[s], kStageBytes);
+        ptx::bulk_load(st, static_cast<const uint8_t*>(a.ds) + slot * kTileBytes, kTileBytes, &bar->full[s]);
+        ptx::tma_load_2d(st + kTileBytes, &tmK, &bar->full[s], g * kD, yk);
+        ptx::tma_load_2d(st + kTileBytes + kHalfBytes, &tmK, &bar->full[s], g * kD + 64, yk);
+        ++nf[s];
+      }
+      if (aborted(&bar->abort))
+        for (int s = 0; s < kStages; ++s)
+          if (nf[s]) wait(&bar->full[s], (nf[s] - 1) & 1, a.status);
+    }
+  } else if (warp == 5) {
+    if (lane == 0 && nkb > 0) {
+      constexpr uint32_t idesc = ptx::idesc_bf16_f32(128, 128, 1, 1);  // A and B MN-major
+      bool ok = true;
+      for (int c = 0; c < nkb; ++c) {
+        const int s = c % kStages;
+        if (aborted(&bar->abort) || !wait(&bar->full[s], (uint32_t)(c / kStages) & 1, a.status)) {
+          ok = false;
+          break;
+        }
+        ptx::tc_fence_after();
+        const uint32_t sDS = ptx::smem_u32(smem + s * kStageBytes), sK = sDS + kTileBytes;
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          ptx::mma_bf16_ss(tmem, desc_ilv_mnmajor(sDS, kk), desc_mnmajor(sK, kk), idesc, (c > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma_commit(&bar->empty[s]);
+      }
+      if (!ok) set_abort(&bar->abort);
+      ptx::mma_commit(&bar->done);
+      wait(&bar->done, 0, a.status);
+    }
+    __syncwarp();
+  } else {
+    // epilogue: thread = query row
+    const int r = threadIdx.x;
+    const int row = t * kRows + r;
+    const bool valid = row < w.q_len;
+    const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
+    const bool ok = nkb > 0 && wait(&bar->done, 0, a.status) && !aborted(&bar->abort);
+    if (ok) ptx::tc_fence_after();
+    uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) +
+                                          ((int64_t)w.q_base + row) * a.hq * kD + h * kD);
+#pragma unroll 1
+    for (int q4 = 0; q4 < 4; ++q4) {
+      uint32_t v[32];
+      if (ok) {
+        ptx::tmem_ld32(tmem + lane_addr + 32 * q4, v);
+        ptx::tmem_ld_wait();
+        ptx::reg_fence(v);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 32; ++k) v[k] = 0u;
+      }
+      if (valid && (ok || nkb == 0)) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          uint4 o;
+          o.x = pack_bf16(__uint_as_float(v[8 * i + 0]) * a.scale, __uint_as_float(v[8 * i + 1]) * a.scale);
+          o.y = pack_bf16(__uint_as_float(v[8 * i + 2]) * a.scale, __uint_as_float(v[8 * i + 3]) * a.scale);
+          o.z = pack_bf16(__uint_as_float(v[8 * i + 4]) * a.scale, __uint_as_float(v[8 * i + 5]) * a.scale);
+          o.w = pack_bf16(__uint_as_float(v[8 * i + 6]) * a.scale, __uint_as_float(v[8 * i + 7]) * a.scale);
+          dst[4 * q4 + i] = o;
+        }
+      }
+    }
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == 5) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_dq_gemm(const AttnArgs& a, const CUtensorMap& tk, cudaStream_t st) {
+  cudaError_t e;
+  if ((reinterpret_cast<uintptr_t>(a.ds) & 15u) != 0) return cudaErrorMisalignedAddress;
+  if ((e = cudaFuncSetAttribute(dq_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
+      cudaSuccess)
+    return e;
+  dq_gemm_kernel<<<(unsigned)(a.nq * a.hq), kThreads, kSmemBytes, st>>>(tk, a);
+  return cudaGetLastError();
+}
+
+}  // namespace tc
+}  // namespace ism

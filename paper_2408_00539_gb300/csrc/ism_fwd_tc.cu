@@ -314,7 +314,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 // One 128x128x128 tile: C = A * B^T (B given as [N, K], K-major) or C = A * B
 // (B given as [K, N], MN-major).  Operands staged by plain stores in the
 // swizzled layout (modes 0/1), by TMA (modes 2/3), or A in tensor memory and
-// B by plain stores (modes 4/5).
+// B by plain stores (modes 4/5); mode 6: A given as [K, M] (MN-major) and B
+// as [K, N], C = A^T B; mode 7: as mode 6 with A in the 8-interleaved
+// MN-major layout without swizzle.
 __global__ void __launch_bounds__(128, 1)
     mma_tile_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __nv_bfloat16* A, const __nv_bfloat16* B, float* C, int mode, uint32_t* status) {
@@ -325,8 +327,10 @@ __global__ void __launch_bounds__(128, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 2 * kTileBytes);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2);
   const int warp = threadIdx.x >> 5;
-  const bool b_mn = (mode & 1) != 0;
-  const bool a_tmem = mode >= 4;
+  const bool a_mn = mode == 6 || mode == 7;
+  const bool a_ilv = mode == 7;
+  const bool b_mn = (mode & 1) != 0 || mode == 6;
+  const bool a_tmem = mode == 4 || mode == 5;
   if (threadIdx.x == 0) {
     ptx::mbar_init(&bars[0], 1);
     ptx::mbar_init(&bars[1], 1);
@@ -336,10 +340,10 @@ __global__ void __launch_bounds__(128, 1)
     ptx::tmem_alloc(tslot, 256);
     ptx::tmem_relinquish();
   }
-  if (mode < 2 || a_tmem) {
+  if (mode < 2 || a_tmem || a_mn) {
     for (int i = threadIdx.x; i < 128 * 128; i += blockDim.x) {
       const int r = i >> 7, c = i & 127;
-      *reinterpret_cast<__nv_bfloat16*>(sa + swz_offset(r, c)) = A[i];
+      *reinterpret_cast<__nv_bfloat16*>(sa + (a_ilv ? ilv_offset(c, r) : swz_offset(r, c))) = A[i];
       *reinterpret_cast<__nv_bfloat16*>(sb + swz_offset(r, c)) = B[i];
     }
     ptx::fence_proxy_async_smem();
@@ -376,14 +380,16 @@ __global__ void __launch_bounds__(128, 1)
       ok = wait(&bars[0], 0, status);
     }
     if (ok) {
-      const uint32_t idesc = ptx::idesc_bf16_f32(128, 128, 0, b_mn ? 1u : 0u);
+      const uint32_t idesc = ptx::idesc_bf16_f32(128, 128, a_mn ? 1u : 0u, b_mn ? 1u : 0u);
       const uint32_t saa = ptx::smem_u32(sa), sbb = ptx::smem_u32(sb);
       for (int kk = 0; kk < 8; ++kk) {
         const uint64_t bd = b_mn ? desc_mnmajor(sbb, kk) : desc_kmajor(sbb, kk);
         if (a_tmem)
           ptx::mma_bf16_ts(tmem, tmem + 128 + 8 * kk, bd, idesc, kk > 0 ? 1u : 0u);
         else
-          ptx::mma_bf16_ss(tmem, desc_kmajor(saa, kk), bd, idesc, kk > 0 ? 1u : 0u);
+          ptx::mma_bf16_ss(tmem,
+                           a_ilv ? desc_ilv_mnmajor(saa, kk) : a_mn ? desc_mnmajor(saa, kk) : desc_kmajor(saa, kk),
+                           bd, idesc, kk > 0 ? 1u : 0u);
       }
     }
     ptx::mma_commit(&bars[1]);

@@ -69,6 +69,7 @@ cudaError_t launch_tiles(const SegsDev& s, int bm, int bn, const int32_t* kv_end
                          int32_t* kt_end, int32_t* qt_begin, cudaStream_t st);
 cudaError_t launch_order(const Tile* qtiles, int64_t nq, const Tile* ktiles, int64_t nk, int max_cost,
                          int32_t* q_order, int32_t* k_order, cudaStream_t st);
+cudaError_t launch_pair_offsets(const Tile* ktiles, int64_t nk, int32_t* kpair_off, cudaStream_t st);
 cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t cap, int bm, int bn,
                                int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
                                int32_t* q_order, cudaStream_t st);
@@ -89,6 +90,13 @@ struct AttnArgs {
   const Tile* qtiles; const int32_t* q_order; int64_t nq;
   const Tile* ktiles; const int32_t* k_order; int64_t nk;
   uint32_t* status;
+  // Stored-dS backward: when ds is set, dK/dV also writes each bf16 dS tile
+  // (128 queries x 128 keys, 8-query-interleaved, 32 KiB) of (k-tile gk,
+  // q-tile t, head h) to slot (kpair_off[gk] + t - qt_begin(gk)) * hq + h,
+  // and dQ is a GEMM over them.
+  void* ds;
+  const int32_t* kpair_off;
+  int64_t ds_slots;
   // Bit 0: before an MMA that overwrites tensor memory an earlier MMA reads
   // as its A operand, wait for that earlier MMA to complete.  Clear: rely on
   // MMAs issued by one thread executing in issue order.

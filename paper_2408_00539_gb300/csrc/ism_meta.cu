@@ -162,6 +162,36 @@ __global__ void order_kernel(const Tile* __restrict__ qtiles, int64_t nq, const 
   }
 }
 
+// Exclusive prefix over k-tiles of their non-empty q-tile counts (a1 - a0):
+// the first (k-tile, q-tile) pair slot of each k-tile.  One block, chunks of
+// blockDim.x with a running carry.
+__global__ void pair_offsets_kernel(const Tile* __restrict__ ktiles, int64_t nk, int32_t* kpair_off) {
+  __shared__ int32_t buf[1024];
+  __shared__ int32_t carry;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int64_t base = 0; base < nk; base += blockDim.x) {
+    const int64_t i = base + threadIdx.x;
+    int32_t v = 0;
+    if (i < nk) {
+      const Tile w = ktiles[i];
+      v = w.a1 - w.a0 > 0 ? w.a1 - w.a0 : 0;
+    }
+    buf[threadIdx.x] = v;
+    __syncthreads();
+    for (int off = 1; off < blockDim.x; off <<= 1) {
+      const int32_t add = threadIdx.x >= off ? buf[threadIdx.x - off] : 0;
+      __syncthreads();
+      buf[threadIdx.x] += add;
+      __syncthreads();
+    }
+    if (i < nk) kpair_off[i] = carry + buf[threadIdx.x] - v;
+    __syncthreads();
+    if (threadIdx.x == blockDim.x - 1) carry += buf[threadIdx.x];
+    __syncthreads();
+  }
+}
+
 __device__ __forceinline__ int32_t chunk_kv_end(const AppendSegs& sg, int32_t j) {
   int32_t start = 0;
   for (int i = 0; i < sg.n; ++i) {
@@ -266,6 +296,12 @@ cudaError_t launch_order(const Tile* qtiles, int64_t nq, const Tile* ktiles, int
     if (e != cudaSuccess) return e;
   }
   order_kernel<<<1, 1024, smem, st>>>(qtiles, nq, ktiles, nk, max_cost, q_order, k_order);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pair_offsets(const Tile* ktiles, int64_t nk, int32_t* kpair_off, cudaStream_t st) {
+  if (nk == 0) return cudaSuccess;
+  pair_offsets_kernel<<<1, 1024, 0, st>>>(ktiles, nk, kpair_off);
   return cudaGetLastError();
 }
 

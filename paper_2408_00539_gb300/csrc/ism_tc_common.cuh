@@ -76,6 +76,20 @@ __device__ __forceinline__ uint64_t desc_mnmajor(uint32_t tile_saddr, int kk) {
   return ptx::smem_desc(tile_saddr + (uint32_t)kk * 2048u, kHalfBytes, 1024u, ptx::kSwizzle128B);
 }
 
+// 8-interleaved MN-major tile, no swizzle: element (mn, k) of a
+// [128 MN x 128 K] operand at byte ((mn / 8) * 128 + k) * 16 + (mn % 8) * 2,
+// i.e. 16-byte units of 8 consecutive MN elements, K-consecutive units
+// adjacent.  A core matrix (8 MN x 8 K) is 128 contiguous bytes; the next
+// 8 K rows are 128 bytes on (leading offset), the next 8 MN columns 2048
+// bytes on (stride offset).  k-step kk (16 K rows) starts 256 bytes on.
+constexpr uint32_t kIlvUnitRow = 128 * 16;  // bytes between MN groups of 8
+__host__ __device__ constexpr uint32_t ilv_offset(int mn, int k) {
+  return (uint32_t)(mn >> 3) * kIlvUnitRow + (uint32_t)k * 16u + (uint32_t)(mn & 7) * 2u;
+}
+__device__ __forceinline__ uint64_t desc_ilv_mnmajor(uint32_t tile_saddr, int kk) {
+  return ptx::smem_desc(tile_saddr + (uint32_t)kk * 256u, 128u, kIlvUnitRow, ptx::kSwizzleNone);
+}
+
 // Host: 2D bf16 tensor map [rows, cols] with a 64 x 128 box, 128B swizzle.
 cudaError_t make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows);
 // Host: 2D bf16 tensor map with a 64-column x box_rows box, no swizzle.
@@ -85,6 +99,8 @@ bool available();
 // Host: forward with two query heads (sharing a KV head) per CTA.
 cudaError_t launch_fwd_pair(const AttnArgs& a, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             cudaStream_t st);
+// Host: dQ as a GEMM over the dS^T tiles stored by the dK/dV kernel (a.ds).
+cudaError_t launch_dq_gemm(const AttnArgs& a, const CUtensorMap& tk, cudaStream_t st);
 
 }  // namespace tc
 }  // namespace ism

@@ -50,6 +50,7 @@ EXPORTS = {
     "ism_attn_fwd_workspace_size": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "ism_attn_fwd": (C.c_int, [C.c_void_p] * 8 + [C.c_size_t, C.c_void_p]),
     "ism_attn_bwd_workspace_size": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "ism_attn_bwd_workspace_size_min": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "ism_attn_bwd": (C.c_int, [C.c_void_p] * 12 + [C.c_size_t, C.c_void_p]),
     "ism_attn_prefill_append_workspace_size": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_void_p]),
     "ism_attn_prefill_append": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
@@ -217,13 +218,29 @@ def fwd(segs: Segments, q, k, v, softmax_scale: float, out=None, lse=None, works
     return out, lse
 
 
-def bwd(segs: Segments, q, k, v, o, lse, dout, softmax_scale: float, dq=None, dk=None, dv=None, workspace=None):
-    """Backward: (dq, dk, dv) of sum(O * dout)."""
+def bwd_workspace_size(segs: Segments, q, k, softmax_scale: float, minimal: bool = False) -> int:
+    """Workspace bytes of the backward: the stored-dS schedule's size where
+    it applies (else the minimum), or the minimum with minimal=True."""
+    lib = load()
+    s, sh = segs.struct(), _shape(q, k, softmax_scale)
+    nbytes = C.c_size_t()
+    fn = "ism_attn_bwd_workspace_size_min" if minimal else "ism_attn_bwd_workspace_size"
+    _check(getattr(lib, fn)(C.byref(s), C.byref(sh), C.byref(nbytes)), fn)
+    return nbytes.value
+
+
+def bwd(segs: Segments, q, k, v, o, lse, dout, softmax_scale: float, dq=None, dk=None, dv=None, workspace=None,
+        minimal_workspace: bool = False):
+    """Backward: (dq, dk, dv) of sum(O * dout).  The library takes the
+    stored-dS schedule when the workspace is large enough for it; with
+    minimal_workspace=True a fresh workspace gets only the minimum size (the
+    recompute schedule)."""
     lib = load()
     _contig(q, k, v, o, lse, dout)
     s, sh = segs.struct(), _shape(q, k, softmax_scale)
     nbytes = C.c_size_t()
-    _check(lib.ism_attn_bwd_workspace_size(C.byref(s), C.byref(sh), C.byref(nbytes)), "ism_attn_bwd_workspace_size")
+    fn = "ism_attn_bwd_workspace_size_min" if minimal_workspace else "ism_attn_bwd_workspace_size"
+    _check(getattr(lib, fn)(C.byref(s), C.byref(sh), C.byref(nbytes)), fn)
     dq = torch.empty_like(q) if dq is None else dq
     dk = torch.empty_like(k) if dk is None else dk
     dv = torch.empty_like(v) if dv is None else dv

@@ -53,12 +53,12 @@ def _cmp_lse(name, got, ref, dtype):
     assert err.max() <= (1e-5 if dtype == "fp32" else 1e-3), f"{name}: max abs err {err.max():.3e}"
 
 
-def _run_pass(ism, w, seed_offset=0):
+def _run_pass(ism, w, seed_offset=0, minimal_workspace=False):
     q, k, v, do = wl.attention_tensors(w, seed_offset=seed_offset)
     segs = ism.Segments.from_workload(w.segs, DEV)
     qd, kd, vd, dod = (t.to(DEV) for t in (q, k, v, do))
     o, lse = ism.fwd(segs, qd, kd, vd, w.softmax_scale)
-    dq, dk, dv = ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale)
+    dq, dk, dv = ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, minimal_workspace=minimal_workspace)
     ism.check_status()
     return (q, k, v, do), (o, lse, dq, dk, dv)
 
@@ -111,12 +111,12 @@ def _small_bf16(d, hq=8, hkv=2, seed=9):
 
 
 @pytest.mark.parametrize("d", [128, 64])
-@pytest.mark.parametrize("path", ["default", "cuda_cores"])
+@pytest.mark.parametrize("path", ["default", "recompute_dq", "cuda_cores"])
 def test_small_bf16_fwd_bwd(ism, d, path, monkeypatch):
     if path == "cuda_cores":
         monkeypatch.setenv("ISM_FORCE_CUDA_CORES", "1")
     w = _small_bf16(d)
-    (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w)
+    (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w, minimal_workspace=path == "recompute_dq")
     o_ref, lse_ref = orc.attn_fwd(q, k, v, w.segs, w.softmax_scale)
     dq_ref, dk_ref, dv_ref = orc.attn_bwd(q, k, v, do, w.segs, w.softmax_scale)
     _cmp("o", o, o_ref, "bf16")
@@ -362,3 +362,32 @@ def test_in_order_tmem_reuse_matches_drained_bit_exact(ism, monkeypatch):
         got = run()
         for name, a_, b_ in zip(("o", "lse", "dq", "dk", "dv"), got, ref):
             assert torch.equal(a_, b_), name
+
+
+def test_bwd_schedules_agree(ism):
+    """The stored-dS backward (dK/dV keeps every visible dS^T tile, dQ is a
+    GEMM over them) and the recompute backward run the same dK/dV arithmetic,
+    so dK and dV agree bit for bit; dQ is built from the same bf16-rounded
+    dS in another fp32 summation order.  The stored schedule's extra
+    workspace is 32 KiB per non-empty (q-tile, k-tile) pair and query head,
+    the pair count being the number of non-empty tiles of the tile map."""
+    w = wl.gqa_8k()
+    q, k, v, do = (t.to(DEV) for t in wl.attention_tensors(w))
+    segs = ism.Segments.from_workload(w.segs, DEV)
+    o, lse = ism.fwd(segs, q, k, v, w.softmax_scale)
+    full = ism.bwd_workspace_size(segs, q, k, w.softmax_scale)
+    low = ism.bwd_workspace_size(segs, q, k, w.softmax_scale, minimal=True)
+    if ism.has_tensor_cores():
+        pairs = int(orc.tile_map_packed(w.segs, 128, 128)["kt_end"].sum())
+        extra = pairs * w.num_heads_q * 128 * 128 * 2
+        nk = int(sum((n + 127) // 128 for n in np.diff(w.segs.cu_seqlens)))
+        assert extra <= full - low <= extra + 4 * nk + 1024
+    stored = ism.bwd(segs, q, k, v, o, lse, do, w.softmax_scale)
+    recomputed = ism.bwd(segs, q, k, v, o, lse, do, w.softmax_scale, minimal_workspace=True)
+    ism.check_status()
+    assert torch.equal(stored[1], recomputed[1]), "dk"
+    assert torch.equal(stored[2], recomputed[2]), "dv"
+    diff = (stored[0].float() - recomputed[0].float()).abs()
+    scale = recomputed[0].float().abs().max().item()
+    assert diff.max().item() <= 2e-2 * max(scale, 1.0), diff.max().item()
+    assert diff.mean().item() <= 1e-3, diff.mean().item()

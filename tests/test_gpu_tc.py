@@ -18,13 +18,16 @@ def ism():
     return m
 
 
-@pytest.mark.parametrize("mode", [0, 1, 2, 3, 4, 5])
+@pytest.mark.parametrize("mode", [0, 1, 2, 3, 4, 5, 6, 7])
 def test_mma_tile(ism, mode):
     g = torch.Generator().manual_seed(100 + mode)
     a = torch.randn(128, 128, generator=g).to(torch.bfloat16)
     b = torch.randn(128, 128, generator=g).to(torch.bfloat16)
     c = ism.debug_mma_tile(a.cuda(), b.cuda(), mode)
     ism.check_status()
-    ref = a.double() @ (b.double().T if mode % 2 == 0 else b.double())
+    if mode in (6, 7):
+        ref = a.double().T @ b.double()
+    else:
+        ref = a.double() @ (b.double().T if mode % 2 == 0 else b.double())
     err = (c.double().cpu() - ref).abs().max().item()
     assert err < 1e-3, f"mode {mode}: max abs err {err}"
