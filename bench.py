@@ -50,10 +50,26 @@ def n_visible(segs) -> int:
     return total
 
 
-NCU_NAME = {"fwd": "fwd_pair_kernel", "bwd_dkdv": "dkdv_kernel", "bwd_dq": "dq_kernel"}
+def n_tile_pairs(segs, tile: int = 128) -> int:
+    """Non-empty (q-tile, k-tile) pairs at tile x tile: q-tile t reaches
+    k-tiles [0, ceil(kv_end(last row) / tile)) (kv_end non-decreasing)."""
+    total = 0
+    for b in range(segs.num_seqs):
+        _, L, se, st = segs.seq(b)
+        for t in range((L + tile - 1) // tile):
+            last = min(L, (t + 1) * tile) - 1
+            i = int(np.searchsorted(se, last, side="right"))
+            kv = int(se[i]) if int(st[i]) == wl.QUERY else last + 1
+            total += (kv + tile - 1) // tile
+    return total
 
 
-def kernel_traffic(kind: str, workload: str):
+def ncu_name(kind: str, stored_ds: bool) -> str:
+    return {"fwd": "fwd_pair_kernel", "bwd_dkdv": "dkdv_kernel",
+            "bwd_dq": "dq_gemm_kernel" if stored_ds else "dq_kernel"}.get(kind, "")
+
+
+def kernel_traffic(kernel: str, workload: str):
     """DRAM bytes per launch from the committed ncu capture, or None when the
     kernel's source changed since the counters were taken (or no capture of
     this workload exists)."""
@@ -62,7 +78,7 @@ def kernel_traffic(kind: str, workload: str):
     if not os.path.exists(p):
         return None
     with open(p) as fh:
-        rec = json.load(fh).get(NCU_NAME.get(kind, ""))
+        rec = json.load(fh).get(kernel)
     if not rec or rec.get("workload") != workload:
         return None
     with open(os.path.join(ROOT, rec["source"]), "rb") as fh:
@@ -294,16 +310,32 @@ def run_cuda(args, w):
     ms_per_step = total_ms / args.steps
     value = flops * world * args.steps / (total_ms * 1e-3) / 1e12
 
-    # dominant kernel: largest share of the step
+    # roofline of each attention kernel; the dominant one (largest share of
+    # the step) is the line's "roofline"
     mean_k = {n: float(np.mean(t)) for n, t in ktimes.items()}
-    # dQ recomputes S and dP (6 flops/D per pair) unless dS was stored (2)
-    kflops = {"fwd": 4 * D * n_vis, "bwd_dkdv": 8 * D * n_vis, "bwd_dq": (2 if stored_ds else 6) * D * n_vis}
-    dom = max(kflops, key=lambda n: mean_k[n])
-    peak = peaks.get("bf16_tflops_sustained" if args.steps * ms_per_step > 2000 else "bf16_tflops")
-    achieved = kflops[dom] / (mean_k[dom] * 1e-3) / 1e12
-    roofline = {"bound": "tensor", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": achieved / peak, "traffic": kernel_traffic(dom, w.name), "peak_kind": peak_kind,
-                "flops_per_launch": kflops[dom], "ms_per_launch": mean_k[dom]}
+    peak_tc = peaks.get("bf16_tflops_sustained" if args.steps * ms_per_step > 2000 else "bf16_tflops")
+    T, Hq, Hkv = w.total_tokens, w.num_heads_q, w.num_heads_kv
+    ds_bytes = n_tile_pairs(w.segs) * Hq * 128 * 128 * 2 if stored_ds else 0
+    rooflines = {}
+    for kind, fl in (("fwd", 4), ("bwd_dkdv", 8), ("bwd_dq", 6)):
+        kname = ncu_name(kind, stored_ds)
+        ms = mean_k[kind]
+        if kind == "bwd_dq" and stored_ds:
+            # GEMM over the stored dS tiles: reads dS and K once, writes dQ
+            nbytes = ds_bytes + T * Hkv * D * 2 + T * Hq * D * 2
+            ach = nbytes / (ms * 1e-3) / 1e9
+            r = {"bound": "hbm", "achieved": ach, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                 "frac": ach / peaks["hbm_gbs"], "bytes_per_launch": nbytes}
+        else:
+            fpl = fl * D * n_vis
+            ach = fpl / (ms * 1e-3) / 1e12
+            r = {"bound": "tensor", "achieved": ach, "peak": peak_tc, "unit": "TFLOP/s", "frac": ach / peak_tc,
+                 "flops_per_launch": fpl}
+        r.update({"kernel": kname, "traffic": kernel_traffic(kname, w.name), "peak_kind": peak_kind,
+                  "ms_per_launch": ms})
+        rooflines[kind] = r
+    dom = max(rooflines, key=lambda n: mean_k[n])
+    roofline = dict(rooflines[dom])
 
     # end to end through the public API with host buffers
     pin = lambda t: t.pin_memory()  # noqa: E731
@@ -359,6 +391,7 @@ def run_cuda(args, w):
                    "bwd_workspace_bytes": ws_bytes, "parallelism": f"replicas x{world}"},
         "kernel_ms": mean_k,
         "roofline": roofline,
+        "kernel_rooflines": rooflines,
         "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_total / args.steps},
         "gpu_launches": int(launches),
@@ -443,7 +476,9 @@ def measure_append(dev, peaks):
                     "cache-write kernels and host launch overhead"}
 
 
-WORKLOADS = {"gqa_8k": wl.gqa_8k, "mha_4k": wl.mha_4k, "packed_32k": wl.packed_32k}
+WORKLOADS = {"gqa_8k": wl.gqa_8k, "mha_4k": wl.mha_4k, "packed_32k": wl.packed_32k,
+             # one 4K dialogue of the same recipe: small enough for full ncu captures
+             "gqa_4k_b1": lambda: wl.gqa_8k(batch=1, seqlen=4096)}
 
 
 def main():

@@ -18,3 +18,11 @@ def test_headline_density_close_to_half():
     w = wl.gqa_8k()
     dens = bench.n_visible(w.segs) / sum(L * L for L in np.diff(w.segs.cu_seqlens))
     assert 0.5 <= dens <= 0.56
+
+
+def test_tile_pair_count_matches_tile_map():
+    """The stored-dS traffic figure counts the non-empty 128 x 128 tiles."""
+    rng = np.random.Generator(np.random.PCG64(6))
+    for segs in (wl.random_dialogue_set(rng, 30, 700), wl.gqa_8k().segs, wl.tiny_fp32().segs):
+        ref = int(orc.tile_map_packed(segs, 128, 128)["kt_end"].sum())
+        assert bench.n_tile_pairs(segs) == ref
