@@ -386,7 +386,7 @@ def run_cuda(args, w):
         "config": {"workload": w.name, "tokens": w.total_tokens, "n_vis_pairs": n_vis,
                    "flops_per_step": flops, "flop_count": "14*D*N_vis (fwd 4, bwd 10)",
                    "strict_tflops_12D": value * 12 / 14, "l2": "flushed between timed steps (258 MB write)",
-                   "pct_of_peak": value / peak * 100, "path": "tensor cores" if ism.has_tensor_cores()
+                   "pct_of_peak": value / peak_tc * 100, "path": "tensor cores" if ism.has_tensor_cores()
                    else "cuda cores", "bwd_schedule": "stored dS" if stored_ds else "recompute dQ",
                    "bwd_workspace_bytes": ws_bytes, "parallelism": f"replicas x{world}"},
         "kernel_ms": mean_k,

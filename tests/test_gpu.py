@@ -391,3 +391,4 @@ def test_bwd_schedules_agree(ism):
     scale = recomputed[0].float().abs().max().item()
     assert diff.max().item() <= 2e-2 * max(scale, 1.0), diff.max().item()
     assert diff.mean().item() <= 1e-3, diff.mean().item()
+
