@@ -170,7 +170,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else if (warp == 9) {
-    if (lane == 0 && nkb > 0) {
+    // the whole warp runs the loop, one elected lane issues each instruction
+    if (nkb > 0) {
       constexpr uint32_t idesc_nt = ptx::idesc_bf16_f32(128, 128, 0, 0);  // A K-major, B K-major
       constexpr uint32_t idesc_nn = ptx::idesc_bf16_f32(128, 128, 0, 1);  // A K-major, B MN-major
       const uint32_t sQ = ptx::smem_u32(smem + OFF_Q), sdO = ptx::smem_u32(smem + OFF_DO);
@@ -178,18 +179,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t sK = ptx::smem_u32(smem + OFF_K + (c % kKStages) * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss(tmem + TM_S + 128u * (c & 1), desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_nt,
+          ptx::mma_bf16_ss_warp(tmem + TM_S + 128u * (c & 1), desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_nt,
                            kk > 0 ? 1u : 0u);
-        ptx::mma_commit(&bar->s_full[c & 1]);
+        ptx::mma_commit_warp(&bar->s_full[c & 1]);
       };
       auto issue_dp = [&](int c) {
         const int sv = c & 1;
         const uint32_t sV = ptx::smem_u32(smem + OFF_V + sv * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss(tmem + TM_DP, desc_kmajor(sdO, kk), desc_kmajor(sV, kk), idesc_nt, kk > 0 ? 1u : 0u);
-        ptx::mma_commit(&bar->dp_full);
-        ptx::mma_commit(&bar->v_empty[sv]);
+          ptx::mma_bf16_ss_warp(tmem + TM_DP, desc_kmajor(sdO, kk), desc_kmajor(sV, kk), idesc_nt, kk > 0 ? 1u : 0u);
+        ptx::mma_commit_warp(&bar->dp_full);
+        ptx::mma_commit_warp(&bar->v_empty[sv]);
       };
       auto issue_dq = [&](int c) {
         const int R = c & 1;
@@ -198,10 +199,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         // columns [0,32) and [64,128) at columns [64,96)
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ts(tmem + TM_DQ, tmem + TM_S + 128u * R + 8 * kk + (kk >= 4 ? 32 : 0),
+          ptx::mma_bf16_ts_warp(tmem + TM_DQ, tmem + TM_S + 128u * R + 8 * kk + (kk >= 4 ? 32 : 0),
                            desc_mnmajor(sK, kk), idesc_nn, (c > 0 || kk > 0) ? 1u : 0u);
-        ptx::mma_commit(&bar->dq_done[R]);
-        ptx::mma_commit(&bar->k_empty[c % kKStages]);
+        ptx::mma_commit_warp(&bar->dq_done[R]);
+        ptx::mma_commit_warp(&bar->k_empty[c % kKStages]);
       };
       // Event-driven issue: S_c, dP_c, dQ_c go out as soon as their inputs are
       // ready, so no wait blocks an unrelated MMA.
@@ -210,8 +211,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       //        kFlagDrainTmemReuse, dQ_{c-2} completed)
       //   dP_c needs V_c and dP_{c-1} read by the compute warps
       //   dQ_c needs dS_c written
-      bool ok = wait(&bar->qdo_full, 0, a.status) && wait(&bar->k_full[0], 0, a.status) &&
-                wait(&bar->v_full[0], 0, a.status);
+      bool ok = wait_warp(&bar->qdo_full, 0, a.status) && wait_warp(&bar->k_full[0], 0, a.status) &&
+                wait_warp(&bar->v_full[0], 0, a.status);
       if (ok) {
         ptx::tc_fence_after();
         issue_s(0);
@@ -223,19 +224,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool progressed = false;
         if (ns < nkb && (ns < 2 || nq > ns - 2) &&
             (ns < 2 || !(a.flags & kFlagDrainTmemReuse) ||
-             ptx::mbar_test(&bar->dq_done[ns & 1], (uint32_t)((ns - 2) >> 1) & 1)) &&
-            ptx::mbar_test(&bar->k_full[ns % kKStages], (uint32_t)(ns / kKStages) & 1)) {
+             ptx::mbar_test_warp(&bar->dq_done[ns & 1], (uint32_t)((ns - 2) >> 1) & 1)) &&
+            ptx::mbar_test_warp(&bar->k_full[ns % kKStages], (uint32_t)(ns / kKStages) & 1)) {
           ptx::tc_fence_after();
           issue_s(ns++);
           progressed = true;
         }
-        if (nd < nkb && ptx::mbar_test(&bar->dp_read, (uint32_t)(nd - 1) & 1) &&
-            ptx::mbar_test(&bar->v_full[nd & 1], (uint32_t)(nd >> 1) & 1)) {
+        if (nd < nkb && ptx::mbar_test_warp(&bar->dp_read, (uint32_t)(nd - 1) & 1) &&
+            ptx::mbar_test_warp(&bar->v_full[nd & 1], (uint32_t)(nd >> 1) & 1)) {
           ptx::tc_fence_after();
           issue_dp(nd++);
           progressed = true;
         }
-        if (nq < ns && nq < nd && ptx::mbar_test(&bar->p_full[nq & 1], (uint32_t)(nq >> 1) & 1)) {
+        if (nq < ns && nq < nd && ptx::mbar_test_warp(&bar->p_full[nq & 1], (uint32_t)(nq >> 1) & 1)) {
           ptx::tc_fence_after();
           issue_dq(nq++);
           progressed = true;
@@ -245,17 +246,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         } else {
           __nanosleep(16);
           const uint64_t now = globaltimer();
-          if (t_idle == 0) {
-            t_idle = now;
-          } else if (now - t_idle > kWaitLimitNs || aborted(&bar->abort)) {
-            atomicOr(a.status, kStatusTimeout);
+          if (t_idle == 0) t_idle = now;
+          const bool expired = __shfl_sync(0xffffffffu, (now - t_idle > kWaitLimitNs || aborted(&bar->abort)) ? 1 : 0, 0);
+          if (expired) {
+            if (lane == 0) atomicOr(a.status, kStatusTimeout);
             ok = false;
           }
         }
       }
-      if (!ok) set_abort(&bar->abort);
-      ptx::mma_commit(&bar->final_mma);
-      wait(&bar->final_mma, 0, a.status);
+      if (!ok && lane == 0) set_abort(&bar->abort);
+      __syncwarp();
+      ptx::mma_commit_warp(&bar->final_mma);
+      wait_warp(&bar->final_mma, 0, a.status);
     }
     __syncwarp();
   } else {
@@ -360,6 +362,9 @@ constexpr uint32_t kMetaStage = 128 * 4 + 128 * 4 + 128;
 constexpr uint32_t OFF_BAR = OFF_META + 2 * kMetaStage;
 constexpr uint32_t kSmemBytes = OFF_BAR + 256;  // needs a 1024-aligned dynamic shared base
 constexpr uint32_t TM_S = 0, TM_DP = 128, TM_DV = 256, TM_DK = 384;
+// warps 0-7 compute, 8 TMA loads, 9 TMEM + MMA issue, 10 per-query metadata
+constexpr int kLoadWarp = 8, kMmaWarp = 9, kMetaWarp = 10;
+constexpr int kThreads = 352;
 
 struct Bars {
   uint64_t kv_full;
@@ -371,7 +376,7 @@ struct Bars {
 static_assert(sizeof(Bars) <= 256, "barrier block");
 }  // namespace dkv
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(dkv::kThreads, 1)
     dkdv_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmdO,
                 const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
   using namespace dkv;
@@ -390,6 +395,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int qt0 = w.a0, nqt = w.a1;
   const int per_head = nqt - qt0;
   const int n_it = per_head > 0 ? per_head * group : 0;
+  // Iteration i visits query tile nqt - 1 - i / group of query head
+  // g * group + i % group: the key tiles of a sequence all start at its last
+  // query tile and move down together, so the CTAs running at the same time
+  // read the same Q / dO tiles and mostly hit L2.
   const int c = w.tile;
 
   if (threadIdx.x == 0) {
@@ -413,7 +422,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     bar->abort = 0;
     ptx::fence_mbar_init();
   }
-  if (warp == 9) {
+  if (warp == kMmaWarp) {
     ptx::tmem_alloc(&bar->tmem_base, kTmemCols);
     ptx::tmem_relinquish();
   }
@@ -422,8 +431,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   ptx::tc_fence_after();
   const uint32_t tmem = bar->tmem_base;
 
-  if (warp == 8) {
-    // ------------------------------------------------ loads (all 32 lanes fill the meta arrays)
+  if (warp == kLoadWarp) {
+    // ------------------------------------------------ TMA loads (lane 0)
     uint32_t nq[kQStages] = {0, 0, 0}, ndo[2] = {0, 0};
     const int32_t ky = w.k_base + c * kRows;
     if (lane == 0 && n_it > 0) {
@@ -432,15 +441,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tma_load_2d(smem + OFF_K + kHalfBytes, &tmK, &bar->kv_full, g * kD + 64, ky);
       ptx::tma_load_2d(smem + OFF_V, &tmV, &bar->kv_full, g * kD, ky);
       ptx::tma_load_2d(smem + OFF_V + kHalfBytes, &tmV, &bar->kv_full, g * kD + 64, ky);
-    }
-    for (int i = 0; i < n_it; ++i) {
-      const int sq = i % kQStages, s = i & 1;
-      const uint32_t n = (uint32_t)(i >> 1);
-      const int hh = i / per_head, t = qt0 + i % per_head;
-      const int h = g * group + hh;
-      const int32_t qy = w.q_base + t * kRows;
-      if (aborted(&bar->abort)) break;
-      if (lane == 0) {
+      for (int i = 0; i < n_it; ++i) {
+        const int sq = i % kQStages, s = i & 1;
+        const uint32_t n = (uint32_t)(i >> 1);
+        const int h = g * group + i % group;
+        const int32_t qy = w.q_base + (nqt - 1 - i / group) * kRows;
+        if (aborted(&bar->abort)) break;
         bool ok = i < kQStages || wait(&bar->q_empty[sq], (uint32_t)(i / kQStages - 1) & 1, a.status);
         if (ok) {
           ptx::mbar_expect_tx(&bar->q_full[sq], kTileBytes);
@@ -455,9 +461,27 @@ __global__ void __launch_bounds__(kThreads, 1)
           ptx::tma_load_2d(smem + OFF_DO + s * kTileBytes + kHalfBytes, &tmdO, &bar->do_full[s], h * kD + 64, qy);
           ++ndo[s];
         }
-        if (!ok) set_abort(&bar->abort);
+        if (!ok) {
+          set_abort(&bar->abort);
+          break;
+        }
       }
-      __syncwarp();
+      if (aborted(&bar->abort)) {
+        wait(&bar->kv_full, 0, a.status);
+        for (int s = 0; s < kQStages; ++s)
+          if (nq[s]) wait(&bar->q_full[s], (nq[s] - 1) & 1, a.status);
+        for (int s = 0; s < 2; ++s)
+          if (ndo[s]) wait(&bar->do_full[s], (ndo[s] - 1) & 1, a.status);
+      }
+    }
+    __syncwarp();
+  } else if (warp == kMetaWarp) {
+    // ------------------------------------------------ per-query metadata (all 32 lanes)
+    for (int i = 0; i < n_it; ++i) {
+      const int s = i & 1;
+      const uint32_t n = (uint32_t)(i >> 1);
+      const int hh = i % group, t = nqt - 1 - i / group;
+      const int h = g * group + hh;
       if (aborted(&bar->abort)) break;
       if (i >= 2 && !wait(&bar->meta_empty[s], (n - 1) & 1, a.status)) { set_abort(&bar->abort); break; }
       uint8_t* meta = smem + OFF_META + s * kMetaStage;
@@ -477,79 +501,92 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       ptx::mbar_arrive(&bar->meta_full[s]);
     }
-    if (lane == 0 && aborted(&bar->abort)) {
-      if (n_it > 0) wait(&bar->kv_full, 0, a.status);
-      for (int s = 0; s < kQStages; ++s)
-        if (nq[s]) wait(&bar->q_full[s], (nq[s] - 1) & 1, a.status);
-      for (int s = 0; s < 2; ++s)
-        if (ndo[s]) wait(&bar->do_full[s], (ndo[s] - 1) & 1, a.status);
-    }
-  } else if (warp == 9) {
-    // ------------------------------------------------ MMA issue
-    if (lane == 0 && n_it > 0) {
+  } else if (warp == kMmaWarp) {
+    // ------------------------------------------------ MMA issue (the whole warp runs the
+    // loop, one elected lane issues each instruction)
+    if (n_it > 0) {
       constexpr uint32_t idesc_nt = ptx::idesc_bf16_f32(128, 128, 0, 0);
       constexpr uint32_t idesc_nn = ptx::idesc_bf16_f32(128, 128, 0, 1);
       const uint32_t sK = ptx::smem_u32(smem + OFF_K), sV = ptx::smem_u32(smem + OFF_V);
-      bool ok = wait(&bar->kv_full, 0, a.status);
-      auto issue_s = [&](int i) -> bool {
-        const int sq = i % kQStages;
-        if (!wait(&bar->q_full[sq], (uint32_t)(i / kQStages) & 1, a.status)) return false;
-        ptx::tc_fence_after();
-        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + sq * kTileBytes);
+      auto issue_s = [&](int i) {
+        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + (i % kQStages) * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss(tmem + TM_S, desc_kmajor(sK, kk), desc_kmajor(sQ, kk), idesc_nt, kk > 0 ? 1u : 0u);
-        ptx::mma_commit(&bar->s_full);
-        return true;
+          ptx::mma_bf16_ss_warp(tmem + TM_S, desc_kmajor(sK, kk), desc_kmajor(sQ, kk), idesc_nt, kk > 0 ? 1u : 0u);
+        ptx::mma_commit_warp(&bar->s_full);
       };
-      auto issue_dp = [&](int i) -> bool {
-        const int s = i & 1;
-        if (!wait(&bar->do_full[s], (uint32_t)(i >> 1) & 1, a.status)) return false;
-        ptx::tc_fence_after();
-        const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + s * kTileBytes);
+      auto issue_dp = [&](int i) {
+        const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + (i & 1) * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss(tmem + TM_DP, desc_kmajor(sV, kk), desc_kmajor(sdO, kk), idesc_nt, kk > 0 ? 1u : 0u);
-        ptx::mma_commit(&bar->dp_full);
-        return true;
+          ptx::mma_bf16_ss_warp(tmem + TM_DP, desc_kmajor(sV, kk), desc_kmajor(sdO, kk), idesc_nt, kk > 0 ? 1u : 0u);
+        ptx::mma_commit_warp(&bar->dp_full);
       };
-      if (ok) ok = issue_s(0) && issue_dp(0);
-      for (int i = 0; ok && i < n_it; ++i) {
+      auto issue_dvk = [&](int i) {
         const int s = i & 1, sq = i % kQStages;
-        if (aborted(&bar->abort)) { ok = false; break; }
-        if (i + 1 < n_it) {
-          if (!wait(&bar->s_free, (uint32_t)i & 1, a.status) || !issue_s(i + 1)) { ok = false; break; }
-        }
-        if (!wait(&bar->p_full, (uint32_t)i & 1, a.status)) { ok = false; break; }
-        ptx::tc_fence_after();
         const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + sq * kTileBytes);
         const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + s * kTileBytes);
         // P^T and dS^T (bf16, two queries per column) sit in the dP^T columns: warpgroup wg's
         // queries [64 wg, 64 wg + 64) have P^T at TM_DP + 64 wg + [0,32) and dS^T at + [32,64)
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ts(tmem + TM_DV, tmem + TM_DP + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sdO, kk), idesc_nn,
-                           (i > 0 || kk > 0) ? 1u : 0u);
+          ptx::mma_bf16_ts_warp(tmem + TM_DV, tmem + TM_DP + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sdO, kk),
+                                idesc_nn, (i > 0 || kk > 0) ? 1u : 0u);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ts(tmem + TM_DK, tmem + TM_DP + 32 + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sQ, kk),
-                           idesc_nn, (i > 0 || kk > 0) ? 1u : 0u);
-        ptx::mma_commit(&bar->q_empty[sq]);
-        ptx::mma_commit(&bar->do_empty[s]);
-        ptx::mma_commit(&bar->dvk_done);
-        if (i + 1 < n_it) {
-          // dP^T of the next tile overwrites the P^T / dS^T that dV, dK read (in
-          // issue order; kFlagDrainTmemReuse waits for dV, dK to complete)
-          if (((a.flags & kFlagDrainTmemReuse) && !wait(&bar->dvk_done, (uint32_t)i & 1, a.status)) ||
-              !issue_dp(i + 1)) {
+          ptx::mma_bf16_ts_warp(tmem + TM_DK, tmem + TM_DP + 32 + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sQ, kk),
+                                idesc_nn, (i > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma_commit_warp(&bar->q_empty[sq]);
+        ptx::mma_commit_warp(&bar->do_empty[s]);
+        ptx::mma_commit_warp(&bar->dvk_done);
+      };
+      // Event-driven issue, in order of urgency (the tensor pipe runs MMAs in
+      // issue order, so whatever is issued first runs first):
+      //   dV_i, dK_i  need P^T_i and dS^T_i written (p_full)
+      //   dP_i        needs dO_i and dV_{i-1}, dK_{i-1} issued (it overwrites the
+      //               P^T / dS^T they read; MMAs of this thread execute in order,
+      //               or, with kFlagDrainTmemReuse, they completed)
+      //   S_i         needs Q_i and S_{i-1} read by the compute warps (s_free)
+      bool ok = wait_warp(&bar->kv_full, 0, a.status);
+      int ns = 0, np = 0, nv = 0;
+      uint64_t t_idle = 0;
+      while (ok && nv < n_it) {
+        bool progressed = false;
+        if (nv < np && ptx::mbar_test_warp(&bar->p_full, (uint32_t)nv & 1)) {
+          ptx::tc_fence_after();
+          issue_dvk(nv++);
+          progressed = true;
+        }
+        if (np < n_it && np <= nv && ptx::mbar_test_warp(&bar->do_full[np & 1], (uint32_t)(np >> 1) & 1) &&
+            (np == 0 || !(a.flags & kFlagDrainTmemReuse) ||
+             ptx::mbar_test_warp(&bar->dvk_done, (uint32_t)(np - 1) & 1))) {
+          ptx::tc_fence_after();
+          issue_dp(np++);
+          progressed = true;
+        }
+        if (ns < n_it && (ns == 0 || ptx::mbar_test_warp(&bar->s_free, (uint32_t)(ns - 1) & 1)) &&
+            ptx::mbar_test_warp(&bar->q_full[ns % kQStages], (uint32_t)(ns / kQStages) & 1)) {
+          ptx::tc_fence_after();
+          issue_s(ns++);
+          progressed = true;
+        }
+        if (progressed) {
+          t_idle = 0;
+        } else {
+          __nanosleep(16);
+          const uint64_t now = globaltimer();
+          if (t_idle == 0) t_idle = now;
+          const bool expired = __shfl_sync(0xffffffffu, (now - t_idle > kWaitLimitNs || aborted(&bar->abort)) ? 1 : 0, 0);
+          if (expired) {
+            if (lane == 0) atomicOr(a.status, kStatusTimeout);
             ok = false;
-            break;
           }
         }
       }
-      if (!ok) set_abort(&bar->abort);
-      ptx::mma_commit(&bar->final_mma);
-      wait(&bar->final_mma, 0, a.status);
+      if (!ok && lane == 0) set_abort(&bar->abort);
+      __syncwarp();
+      ptx::mma_commit_warp(&bar->final_mma);
+      wait_warp(&bar->final_mma, 0, a.status);
     }
     __syncwarp();
   } else {
@@ -622,20 +659,21 @@ __global__ void __launch_bounds__(kThreads, 1)
       // P^T and dS^T over this warpgroup's (already read) dP^T columns
       ptx::tmem_st32(tP, pp);
       ptx::tmem_st32(tP + 32, pd);
+      ptx::tmem_st_wait();
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&bar->p_full);
       if (a.ds) {
         // keep dS^T row r, queries [64 wg, 64 wg + 64), for the dQ GEMM, in
         // the 8-interleaved layout (16-byte unit (query group, key)): the 32
-        // lanes of a warp store 512 contiguous bytes per instruction
-        const int hh = i / per_head, t = qt0 + i % per_head;
+        // lanes of a warp store 512 contiguous bytes per instruction.  Issued
+        // after the hand-off so that the dV/dK MMAs do not wait for it.
+        const int hh = i % group, t = nqt - 1 - i / group;
         const int64_t slot = ((int64_t)a.kpair_off[gk] + (t - qt0)) * a.hq + (g * group + hh);
         uint4* dst = reinterpret_cast<uint4*>(static_cast<uint8_t*>(a.ds) + slot * kTileBytes) + wg * 8 * kRows + r;
 #pragma unroll
         for (int k = 0; k < 8; ++k)
           dst[k * kRows] = make_uint4(pd[4 * k], pd[4 * k + 1], pd[4 * k + 2], pd[4 * k + 3]);
       }
-      ptx::tmem_st_wait();
-      ptx::tc_fence_before();
-      ptx::mbar_arrive(&bar->p_full);
     }
     if (ok && n_it > 0) ok = wait(&bar->final_mma, 0, a.status);
     if (!ok) {
@@ -677,7 +715,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   ptx::tc_fence_before();
   __syncthreads();
-  if (warp == 9) {
+  if (warp == kMmaWarp) {
     ptx::tc_fence_after();
     ptx::tmem_dealloc(tmem, kTmemCols);
   }
@@ -720,7 +758,7 @@ cudaError_t launch_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) {
                                   (int)dkv::kSmemBytes)) != cudaSuccess)
       return e;
     timer_begin(ISM_KERNEL_BWD_DKDV, st);
-    dkdv_kernel<<<(unsigned)(a.nk * a.hkv), kThreads, dkv::kSmemBytes, st>>>(tq, tdo, tk, tv, a);
+    dkdv_kernel<<<(unsigned)(a.nk * a.hkv), dkv::kThreads, dkv::kSmemBytes, st>>>(tq, tdo, tk, tv, a);
     timer_end(ISM_KERNEL_BWD_DKDV, st);
     count_launch();
     if ((e = cudaGetLastError()) != cudaSuccess) return e;

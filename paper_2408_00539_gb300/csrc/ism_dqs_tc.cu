@@ -92,12 +92,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (nf[s]) wait(&bar->full[s], (nf[s] - 1) & 1, a.status);
     }
   } else if (warp == 5) {
-    if (lane == 0 && nkb > 0) {
+    // the whole warp runs the loop, one elected lane issues each instruction
+    if (nkb > 0) {
       constexpr uint32_t idesc = ptx::idesc_bf16_f32(128, 128, 1, 1);  // A and B MN-major
       bool ok = true;
       for (int c = 0; c < nkb; ++c) {
         const int s = c % kStages;
-        if (aborted(&bar->abort) || !wait(&bar->full[s], (uint32_t)(c / kStages) & 1, a.status)) {
+        if (__shfl_sync(0xffffffffu, aborted(&bar->abort) ? 1 : 0, 0) ||
+            !wait_warp(&bar->full[s], (uint32_t)(c / kStages) & 1, a.status)) {
           ok = false;
           break;
         }
@@ -105,12 +107,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t sDS = ptx::smem_u32(smem + s * kStageBytes), sK = sDS + kTileBytes;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss(tmem, desc_ilv_mnmajor(sDS, kk), desc_mnmajor(sK, kk), idesc, (c > 0 || kk > 0) ? 1u : 0u);
-        ptx::mma_commit(&bar->empty[s]);
+          ptx::mma_bf16_ss_warp(tmem, desc_ilv_mnmajor(sDS, kk), desc_mnmajor(sK, kk), idesc, (c > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma_commit_warp(&bar->empty[s]);
       }
-      if (!ok) set_abort(&bar->abort);
-      ptx::mma_commit(&bar->done);
-      wait(&bar->done, 0, a.status);
+      if (!ok && lane == 0) set_abort(&bar->abort);
+      __syncwarp();
+      ptx::mma_commit_warp(&bar->done);
+      wait_warp(&bar->done, 0, a.status);
     }
     __syncwarp();
   } else {

@@ -115,8 +115,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else if (warp == 9) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0 && nkb > 0) {
+    // ------------------------------------------------------------ MMA issuer (the whole
+    // warp runs the loop, one elected lane issues each instruction)
+    if (nkb > 0) {
       constexpr uint32_t idesc_qk = ptx::idesc_bf16_f32(128, 128, 0, 0);
       constexpr uint32_t idesc_pv = ptx::idesc_bf16_f32(128, 128, 0, 1);
       const uint32_t sQ0 = ptx::smem_u32(smem + OFF_QA);
@@ -126,23 +127,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t sQ = sQ0 + (uint32_t)x * kTileBytes, tS = tmem + 256u * (uint32_t)x;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss(tS, desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_qk, kk > 0 ? 1u : 0u);
-        ptx::mma_commit(&bar->s_full[x]);
+          ptx::mma_bf16_ss_warp(tS, desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_qk, kk > 0 ? 1u : 0u);
+        ptx::mma_commit_warp(&bar->s_full[x]);
       };
       auto issue_pv = [&](int x, int j) {
         const uint32_t sV = ptx::smem_u32(smem + OFF_V + (j & 1) * kTileBytes);
         const uint32_t tS = tmem + 256u * (uint32_t)x, tO = tS + 128u;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ts(tO, tS + 8 * kk, desc_mnmajor(sV, kk), idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
-        ptx::mma_commit(&bar->pv_done[x]);
+          ptx::mma_bf16_ts_warp(tO, tS + 8 * kk, desc_mnmajor(sV, kk), idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma_commit_warp(&bar->pv_done[x]);
       };
-      bool ok = wait(&bar->q_full, 0, a.status) && wait(&bar->k_full[0], 0, a.status);
+      bool ok = wait_warp(&bar->q_full, 0, a.status) && wait_warp(&bar->k_full[0], 0, a.status);
       if (ok) {
         ptx::tc_fence_after();
         issue_s(0, 0);
         issue_s(1, 0);
-        ptx::mma_commit(&bar->k_empty[0]);
+        ptx::mma_commit_warp(&bar->k_empty[0]);
       }
       // Per block: PV_A(j), S_A(j+1), PV_B(j), S_B(j+1).  S_x(j+1) overwrites
       // the P_x(j) that PV_x(j) reads; MMAs issued by this thread execute in
@@ -151,28 +152,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = 0; ok && j < nkb; ++j) {
         const int s = j & 1, s1 = (j + 1) & 1;
         const bool more = j + 1 < nkb;
-        if (aborted(&bar->abort)) { ok = false; break; }
-        if (!wait(&bar->v_full[s], (uint32_t)(j >> 1) & 1, a.status)) { ok = false; break; }
-        if (more && !wait(&bar->k_full[s1], (uint32_t)((j + 1) >> 1) & 1, a.status)) { ok = false; break; }
+        if (__shfl_sync(0xffffffffu, aborted(&bar->abort) ? 1 : 0, 0)) { ok = false; break; }
+        if (!wait_warp(&bar->v_full[s], (uint32_t)(j >> 1) & 1, a.status)) { ok = false; break; }
+        if (more && !wait_warp(&bar->k_full[s1], (uint32_t)((j + 1) >> 1) & 1, a.status)) { ok = false; break; }
         for (int x = 0; x < 2; ++x) {
-          if (!wait(&bar->p_full[x], (uint32_t)j & 1, a.status)) { ok = false; break; }
+          if (!wait_warp(&bar->p_full[x], (uint32_t)j & 1, a.status)) { ok = false; break; }
           ptx::tc_fence_after();
           issue_pv(x, j);
-          if (x == 1) ptx::mma_commit(&bar->v_empty[s]);
+          if (x == 1) ptx::mma_commit_warp(&bar->v_empty[s]);
           if (more) {
-            if ((a.flags & kFlagDrainTmemReuse) && !wait(&bar->pv_done[x], (uint32_t)j & 1, a.status)) {
+            if ((a.flags & kFlagDrainTmemReuse) && !wait_warp(&bar->pv_done[x], (uint32_t)j & 1, a.status)) {
               ok = false;
               break;
             }
             ptx::tc_fence_after();
             issue_s(x, j + 1);
-            if (x == 1) ptx::mma_commit(&bar->k_empty[s1]);
+            if (x == 1) ptx::mma_commit_warp(&bar->k_empty[s1]);
           }
         }
       }
-      if (!ok) set_abort(&bar->abort);
-      ptx::mma_commit(&bar->final_mma);
-      wait(&bar->final_mma, 0, a.status);
+      if (!ok && lane == 0) set_abort(&bar->abort);
+      __syncwarp();
+      ptx::mma_commit_warp(&bar->final_mma);
+      wait_warp(&bar->final_mma, 0, a.status);
     }
     __syncwarp();
   } else {

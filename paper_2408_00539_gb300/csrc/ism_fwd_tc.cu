@@ -131,48 +131,50 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   } else if (warp == 5) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0 && nkb > 0) {
+    // ------------------------------------------------------------ MMA issuer (the whole
+    // warp runs the loop, one elected lane issues each instruction)
+    if (nkb > 0) {
       constexpr uint32_t idesc_qk = ptx::idesc_bf16_f32(128, 128, 0, 0);
       constexpr uint32_t idesc_pv = ptx::idesc_bf16_f32(128, 128, 0, 1);
-      bool ok = wait(&bar->q_full, 0, a.status);
+      bool ok = wait_warp(&bar->q_full, 0, a.status);
       auto issue_pv = [&](int i) -> bool {
         const int s = i & 1;
         const uint32_t n = (uint32_t)(i >> 1);
-        if (!wait(&bar->p_full[s], n & 1, a.status)) return false;
-        if (!wait(&bar->v_full[s], n & 1, a.status)) return false;
+        if (!wait_warp(&bar->p_full[s], n & 1, a.status)) return false;
+        if (!wait_warp(&bar->v_full[s], n & 1, a.status)) return false;
         ptx::tc_fence_after();
         const uint32_t sP = ptx::smem_u32(smem + OFF_P + s * kTileBytes);
         const uint32_t sV = ptx::smem_u32(smem + OFF_V + s * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss(tmem + TM_O, desc_kmajor(sP, kk), desc_mnmajor(sV, kk), idesc_pv,
+          ptx::mma_bf16_ss_warp(tmem + TM_O, desc_kmajor(sP, kk), desc_mnmajor(sV, kk), idesc_pv,
                            (i > 0 || kk > 0) ? 1u : 0u);
-        ptx::mma_commit(&bar->p_free[s]);
-        ptx::mma_commit(&bar->v_empty[s]);
+        ptx::mma_commit_warp(&bar->p_free[s]);
+        ptx::mma_commit_warp(&bar->v_empty[s]);
         return true;
       };
       for (int j = 0; ok && j < nkb; ++j) {
         const int s = j & 1;
         const uint32_t n = (uint32_t)(j >> 1);
-        if (aborted(bar)) { ok = false; break; }
-        if (!wait(&bar->k_full[s], n & 1, a.status)) { ok = false; break; }
-        if (j >= 2 && !wait(&bar->s_free[s], (n - 1) & 1, a.status)) { ok = false; break; }
+        if (__shfl_sync(0xffffffffu, aborted(bar) ? 1 : 0, 0)) { ok = false; break; }
+        if (!wait_warp(&bar->k_full[s], n & 1, a.status)) { ok = false; break; }
+        if (j >= 2 && !wait_warp(&bar->s_free[s], (n - 1) & 1, a.status)) { ok = false; break; }
         ptx::tc_fence_after();
         const uint32_t sK = ptx::smem_u32(smem + OFF_K + s * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss(tmem + TM_S + s * 128, desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_qk,
+          ptx::mma_bf16_ss_warp(tmem + TM_S + s * 128, desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_qk,
                            kk > 0 ? 1u : 0u);
-        ptx::mma_commit(&bar->s_full[s]);
-        ptx::mma_commit(&bar->k_empty[s]);
+        ptx::mma_commit_warp(&bar->s_full[s]);
+        ptx::mma_commit_warp(&bar->k_empty[s]);
         if (j >= 1 && !issue_pv(j - 1)) { ok = false; break; }
       }
-      if (ok && !aborted(bar)) ok = issue_pv(nkb - 1);
-      if (!ok) set_abort(bar);
+      if (ok && !__shfl_sync(0xffffffffu, aborted(bar) ? 1 : 0, 0)) ok = issue_pv(nkb - 1);
+      if (!ok && lane == 0) set_abort(bar);
+      __syncwarp();
       // all MMAs of this thread complete before TMEM is released
-      ptx::mma_commit(&bar->final_mma);
-      wait(&bar->final_mma, 0, a.status);
+      ptx::mma_commit_warp(&bar->final_mma);
+      wait_warp(&bar->final_mma, 0, a.status);
     }
     __syncwarp();
   } else {

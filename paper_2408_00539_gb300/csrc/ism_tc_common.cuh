@@ -43,6 +43,23 @@ __device__ __forceinline__ bool wait(uint64_t* bar, uint32_t parity, uint32_t* s
   }
 }
 
+// Bounded wait of a whole (converged) warp: lane 0 polls the phase with the
+// non-blocking test and the warp stays converged.  (A blocking try_wait by
+// one lane while the other lanes wait at a warp barrier wakes up late.)
+__device__ __forceinline__ bool wait_warp(uint64_t* bar, uint32_t parity, uint32_t* status) {
+  if (ptx::mbar_test_warp(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  while (true) {
+#pragma unroll 1
+    for (int i = 0; i < 64; ++i)
+      if (ptx::mbar_test_warp(bar, parity)) return true;
+    if (__shfl_sync(0xffffffffu, (globaltimer() - t0 > kWaitLimitNs) ? 1 : 0, 0)) {
+      if ((threadIdx.x & 31) == 0) atomicOr(status, kStatusTimeout);
+      return false;
+    }
+  }
+}
+
 __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
