@@ -596,6 +596,10 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
     const uint32_t tS = tmem + lane_addr + TM_S + 64u * wg, tP = tmem + lane_addr + TM_DP + 64u * wg;
     const float sl2 = a.scale * kLog2e;
     bool ok = true;
+    // dS^T stores of the previous iteration left for after this iteration's P
+    // phase (half of them), where the compute warps wait for dP^T anyway
+    uint4* ds_dst = nullptr;
+    uint32_t ds_rest[16];
     for (int i = 0; ok && i < n_it; ++i) {
       const int s = i & 1;
       if (!wait(&bar->meta_full[s], (uint32_t)(i >> 1) & 1, a.status) || !wait(&bar->s_full, (uint32_t)i & 1, a.status)) {
@@ -631,6 +635,12 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
           pp[q4 * 2] = pack_bf16(p[0], p[1]);
           pp[q4 * 2 + 1] = pack_bf16(p[2], p[3]);
         }
+      }
+      if (ds_dst) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          ds_dst[(k + 4) * kRows] = make_uint4(ds_rest[4 * k], ds_rest[4 * k + 1], ds_rest[4 * k + 2], ds_rest[4 * k + 3]);
+        ds_dst = nullptr;
       }
       // phase 2: dS from dP^T
       if (!wait(&bar->dp_full, (uint32_t)i & 1, a.status)) { ok = false; break; }
@@ -671,9 +681,17 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
         const int64_t slot = ((int64_t)a.kpair_off[gk] + (t - qt0)) * a.hq + (g * group + hh);
         uint4* dst = reinterpret_cast<uint4*>(static_cast<uint8_t*>(a.ds) + slot * kTileBytes) + wg * 8 * kRows + r;
 #pragma unroll
-        for (int k = 0; k < 8; ++k)
+        for (int k = 0; k < 4; ++k)
           dst[k * kRows] = make_uint4(pd[4 * k], pd[4 * k + 1], pd[4 * k + 2], pd[4 * k + 3]);
+#pragma unroll
+        for (int k = 0; k < 16; ++k) ds_rest[k] = pd[16 + k];
+        ds_dst = dst;
       }
+    }
+    if (ds_dst) {
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        ds_dst[(k + 4) * kRows] = make_uint4(ds_rest[4 * k], ds_rest[4 * k + 1], ds_rest[4 * k + 2], ds_rest[4 * k + 3]);
     }
     if (ok && n_it > 0) ok = wait(&bar->final_mma, 0, a.status);
     if (!ok) {
