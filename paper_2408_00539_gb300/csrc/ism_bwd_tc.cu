@@ -372,6 +372,7 @@ struct Bars {
   uint64_t s_full, dp_full, s_free, p_full, dvk_done, final_mma;
   uint32_t tmem_base;
   int32_t abort;
+  uint32_t full[2][2];  // per meta stage and warpgroup: all 64 queries see all 128 keys
 };
 static_assert(sizeof(Bars) <= 256, "barrier block");
 }  // namespace dkv
@@ -488,6 +489,7 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
       float* mlse = reinterpret_cast<float*>(meta);
       float* mdel = mlse + 128;
       uint8_t* mlim = reinterpret_cast<uint8_t*>(mdel + 128);
+      bool all_full = true;
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int j = lane * 4 + e;
@@ -498,6 +500,13 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
         mdel[j] = valid ? a.delta[(int64_t)h * a.q_rows + grow] : 0.f;
         const int vis = valid ? a.kv_end[w.kv_base + row] - c * kRows : 0;
         mlim[j] = (uint8_t)(vis < 0 ? 0 : vis > 128 ? 128 : vis);
+        all_full = all_full && vis >= 128;
+      }
+      // lanes 0-15 hold the queries of warpgroup 0, lanes 16-31 those of warpgroup 1
+      const uint32_t fb = __ballot_sync(0xffffffffu, all_full);
+      if (lane == 0) {
+        bar->full[s][0] = (fb & 0xFFFFu) == 0xFFFFu;
+        bar->full[s][1] = (fb >> 16) == 0xFFFFu;
       }
       ptx::mbar_arrive(&bar->meta_full[s]);
     }
@@ -621,19 +630,31 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
         ptx::reg_fence(sv[1]);
         ptx::tc_fence_before();
         ptx::mbar_arrive(&bar->s_free);
+        if (bar->full[s][wg]) {
+          // every key of the tile is visible to every query of this warpgroup
 #pragma unroll
-        for (int q4 = 0; q4 < 16; ++q4) {
-          const float4 l4 = mlse4[q4];
-          const uint32_t lim = mlim4[q4];
-          const float lv[4] = {l4.x, l4.y, l4.z, l4.w};
-          float p[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int vis = (int)((lim >> (8 * e)) & 0xFFu);
-            p[e] = r < vis ? ex2(__uint_as_float(sv[q4 >> 3][(q4 & 7) * 4 + e]) * sl2 - lv[e]) : 0.f;
+          for (int q4 = 0; q4 < 16; ++q4) {
+            const float4 l4 = mlse4[q4];
+            const uint32_t* sq = &sv[q4 >> 3][(q4 & 7) * 4];
+            pp[q4 * 2] = pack_bf16(ex2(__uint_as_float(sq[0]) * sl2 - l4.x), ex2(__uint_as_float(sq[1]) * sl2 - l4.y));
+            pp[q4 * 2 + 1] =
+                pack_bf16(ex2(__uint_as_float(sq[2]) * sl2 - l4.z), ex2(__uint_as_float(sq[3]) * sl2 - l4.w));
           }
-          pp[q4 * 2] = pack_bf16(p[0], p[1]);
-          pp[q4 * 2 + 1] = pack_bf16(p[2], p[3]);
+        } else {
+#pragma unroll
+          for (int q4 = 0; q4 < 16; ++q4) {
+            const float4 l4 = mlse4[q4];
+            const uint32_t lim = mlim4[q4];
+            const float lv[4] = {l4.x, l4.y, l4.z, l4.w};
+            float p[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const int vis = (int)((lim >> (8 * e)) & 0xFFu);
+              p[e] = r < vis ? ex2(__uint_as_float(sv[q4 >> 3][(q4 & 7) * 4 + e]) * sl2 - lv[e]) : 0.f;
+            }
+            pp[q4 * 2] = pack_bf16(p[0], p[1]);
+            pp[q4 * 2 + 1] = pack_bf16(p[2], p[3]);
+          }
         }
       }
       if (ds_dst) {
