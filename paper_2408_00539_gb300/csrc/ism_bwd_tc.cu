@@ -633,12 +633,17 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
         if (bar->full[s][wg]) {
           // every key of the tile is visible to every query of this warpgroup
 #pragma unroll
+          const float2 sl2x2 = make_float2(sl2, sl2);
+#pragma unroll
           for (int q4 = 0; q4 < 16; ++q4) {
             const float4 l4 = mlse4[q4];
             const uint32_t* sq = &sv[q4 >> 3][(q4 & 7) * 4];
-            pp[q4 * 2] = pack_bf16(ex2(__uint_as_float(sq[0]) * sl2 - l4.x), ex2(__uint_as_float(sq[1]) * sl2 - l4.y));
-            pp[q4 * 2 + 1] =
-                pack_bf16(ex2(__uint_as_float(sq[2]) * sl2 - l4.z), ex2(__uint_as_float(sq[3]) * sl2 - l4.w));
+            const float2 a01 = fma2(make_float2(__uint_as_float(sq[0]), __uint_as_float(sq[1])), sl2x2,
+                                    make_float2(-l4.x, -l4.y));
+            const float2 a23 = fma2(make_float2(__uint_as_float(sq[2]), __uint_as_float(sq[3])), sl2x2,
+                                    make_float2(-l4.z, -l4.w));
+            pp[q4 * 2] = pack_bf16(ex2(a01.x), ex2(a01.y));
+            pp[q4 * 2 + 1] = pack_bf16(ex2(a23.x), ex2(a23.y));
           }
         } else {
 #pragma unroll
@@ -678,12 +683,14 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
           const float4 d4 = mdel4[q4];
           const uint32_t w0 = pp[q4 * 2], w1 = pp[q4 * 2 + 1];
           const int b = (q4 & 7) * 4, hv = q4 >> 3;
-          const float v0 = __uint_as_float(w0 << 16) * (__uint_as_float(dv[hv][b + 0]) - d4.x);
-          const float v1 = __uint_as_float(w0 & 0xFFFF0000u) * (__uint_as_float(dv[hv][b + 1]) - d4.y);
-          const float v2 = __uint_as_float(w1 << 16) * (__uint_as_float(dv[hv][b + 2]) - d4.z);
-          const float v3 = __uint_as_float(w1 & 0xFFFF0000u) * (__uint_as_float(dv[hv][b + 3]) - d4.w);
-          pd[q4 * 2] = pack_bf16(v0, v1);
-          pd[q4 * 2 + 1] = pack_bf16(v2, v3);
+          const float2 v01 = mul2(make_float2(__uint_as_float(w0 << 16), __uint_as_float(w0 & 0xFFFF0000u)),
+                                  add2(make_float2(__uint_as_float(dv[hv][b + 0]), __uint_as_float(dv[hv][b + 1])),
+                                       make_float2(-d4.x, -d4.y)));
+          const float2 v23 = mul2(make_float2(__uint_as_float(w1 << 16), __uint_as_float(w1 & 0xFFFF0000u)),
+                                  add2(make_float2(__uint_as_float(dv[hv][b + 2]), __uint_as_float(dv[hv][b + 3])),
+                                       make_float2(-d4.z, -d4.w)));
+          pd[q4 * 2] = pack_bf16(v01.x, v01.y);
+          pd[q4 * 2 + 1] = pack_bf16(v23.x, v23.y);
         }
       }
       ptx::mbar_arrive(&bar->meta_empty[s]);

@@ -246,20 +246,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         m_use = m_new;
       }
       // P over the first 64 columns of S (already read), 32 columns at a time
-      float rsv[4] = {0.f, 0.f, 0.f, 0.f};
+      float2 rsv[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+      const float2 sl2x2 = make_float2(sl2, sl2), negm = make_float2(-m_use, -m_use);
 #pragma unroll
       for (int hf = 0; hf < 2; ++hf) {
         uint32_t pk[32];
 #pragma unroll
         for (int c = 0; c < 32; ++c) {
-          const float p0 = ex2(fmaf(xs[64 * hf + 2 * c], sl2, -m_use));
-          const float p1 = ex2(fmaf(xs[64 * hf + 2 * c + 1], sl2, -m_use));
-          rsv[c & 3] += p0 + p1;
-          pk[c] = pack_bf16(p0, p1);
+          const float2 arg = fma2(make_float2(xs[64 * hf + 2 * c], xs[64 * hf + 2 * c + 1]), sl2x2, negm);
+          const float2 pr = make_float2(ex2(arg.x), ex2(arg.y));
+          rsv[c & 1] = add2(rsv[c & 1], pr);
+          pk[c] = pack_bf16(pr.x, pr.y);
         }
         ptx::tmem_st32(tS + 32 * hf, pk);
       }
-      l += (rsv[0] + rsv[1]) + (rsv[2] + rsv[3]);
+      l += (rsv[0].x + rsv[0].y) + (rsv[1].x + rsv[1].y);
       ptx::tmem_st_wait();
       ptx::tc_fence_before();
       ptx::mbar_arrive(&bar->p_full[x]);

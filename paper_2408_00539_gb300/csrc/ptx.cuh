@@ -170,11 +170,10 @@ __device__ __forceinline__ void mma_commit_warp(uint64_t* bar) {
       " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}" ::"r"(smem_u32(bar))
       : "memory");
 }
-// mbarrier phase test by lane 0, its answer broadcast (warp-uniform result).
+// mbarrier phase test by every lane of a converged warp, combined by a vote
+// (warp-uniform result).
 __device__ __forceinline__ bool mbar_test_warp(uint64_t* bar, uint32_t parity) {
-  uint32_t r = 0;
-  if ((threadIdx.x & 31) == 0) r = mbar_test(bar, parity) ? 1u : 0u;
-  return __shfl_sync(0xffffffffu, r, 0) != 0;
+  return __all_sync(0xffffffffu, mbar_test(bar, parity));
 }
 
 // Make `bar` track completion of all prior tcgen05.mma of this thread.
