@@ -130,43 +130,53 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = bar->tmem_base;
 
   if (warp == 8) {
-    if (lane == 0 && nkb > 0) {
-      ptx::tma_prefetch_desc(&tmK);
-      ptx::tma_prefetch_desc(&tmV);
-      const int32_t qy = w.q_base + w.tile * kRows;
-      ptx::mbar_expect_tx(&bar->qdo_full, 2 * kTileBytes);
-      ptx::tma_load_2d(smem + OFF_Q, &tmQ, &bar->qdo_full, h * kD, qy);
-      ptx::tma_load_2d(smem + OFF_Q + kHalfBytes, &tmQ, &bar->qdo_full, h * kD + 64, qy);
-      ptx::tma_load_2d(smem + OFF_DO, &tmdO, &bar->qdo_full, h * kD, qy);
-      ptx::tma_load_2d(smem + OFF_DO + kHalfBytes, &tmdO, &bar->qdo_full, h * kD + 64, qy);
+    // the warp waits converged, lane 0 issues the copies
+    if (nkb > 0) {
+      if (lane == 0) {
+        ptx::tma_prefetch_desc(&tmK);
+        ptx::tma_prefetch_desc(&tmV);
+        const int32_t qy = w.q_base + w.tile * kRows;
+        ptx::mbar_expect_tx(&bar->qdo_full, 2 * kTileBytes);
+        ptx::tma_load_2d(smem + OFF_Q, &tmQ, &bar->qdo_full, h * kD, qy);
+        ptx::tma_load_2d(smem + OFF_Q + kHalfBytes, &tmQ, &bar->qdo_full, h * kD + 64, qy);
+        ptx::tma_load_2d(smem + OFF_DO, &tmdO, &bar->qdo_full, h * kD, qy);
+        ptx::tma_load_2d(smem + OFF_DO + kHalfBytes, &tmdO, &bar->qdo_full, h * kD + 64, qy);
+      }
+      __syncwarp();
       uint32_t nk[kKStages] = {0, 0, 0}, nv[2] = {0, 0};
       for (int c = 0; c < nkb; ++c) {
         const int sk = c % kKStages, sv = c & 1;
-        if (aborted(&bar->abort)) break;
+        if (__any_sync(0xffffffffu, aborted(&bar->abort))) break;
         const int32_t ky = w.k_base + c * kRows;
-        if (c >= kKStages && !wait(&bar->k_empty[sk], (uint32_t)(c / kKStages - 1) & 1, a.status)) {
-          set_abort(&bar->abort);
+        if (c >= kKStages && !wait_warp(&bar->k_empty[sk], (uint32_t)(c / kKStages - 1) & 1, a.status)) {
+          if (lane == 0) set_abort(&bar->abort);
           break;
         }
-        ptx::mbar_expect_tx(&bar->k_full[sk], kTileBytes);
-        ptx::tma_load_2d(smem + OFF_K + sk * kTileBytes, &tmK, &bar->k_full[sk], g * kD, ky);
-        ptx::tma_load_2d(smem + OFF_K + sk * kTileBytes + kHalfBytes, &tmK, &bar->k_full[sk], g * kD + 64, ky);
+        if (lane == 0) {
+          ptx::mbar_expect_tx(&bar->k_full[sk], kTileBytes);
+          ptx::tma_load_2d(smem + OFF_K + sk * kTileBytes, &tmK, &bar->k_full[sk], g * kD, ky);
+          ptx::tma_load_2d(smem + OFF_K + sk * kTileBytes + kHalfBytes, &tmK, &bar->k_full[sk], g * kD + 64, ky);
+        }
+        __syncwarp();
         ++nk[sk];
-        if (c >= 2 && !wait(&bar->v_empty[sv], (uint32_t)((c >> 1) - 1) & 1, a.status)) {
-          set_abort(&bar->abort);
+        if (c >= 2 && !wait_warp(&bar->v_empty[sv], (uint32_t)((c >> 1) - 1) & 1, a.status)) {
+          if (lane == 0) set_abort(&bar->abort);
           break;
         }
-        ptx::mbar_expect_tx(&bar->v_full[sv], kTileBytes);
-        ptx::tma_load_2d(smem + OFF_V + sv * kTileBytes, &tmV, &bar->v_full[sv], g * kD, ky);
-        ptx::tma_load_2d(smem + OFF_V + sv * kTileBytes + kHalfBytes, &tmV, &bar->v_full[sv], g * kD + 64, ky);
+        if (lane == 0) {
+          ptx::mbar_expect_tx(&bar->v_full[sv], kTileBytes);
+          ptx::tma_load_2d(smem + OFF_V + sv * kTileBytes, &tmV, &bar->v_full[sv], g * kD, ky);
+          ptx::tma_load_2d(smem + OFF_V + sv * kTileBytes + kHalfBytes, &tmV, &bar->v_full[sv], g * kD + 64, ky);
+        }
+        __syncwarp();
         ++nv[sv];
       }
-      if (aborted(&bar->abort)) {
-        wait(&bar->qdo_full, 0, a.status);
+      if (__any_sync(0xffffffffu, aborted(&bar->abort))) {
+        wait_warp(&bar->qdo_full, 0, a.status);
         for (int s = 0; s < kKStages; ++s)
-          if (nk[s]) wait(&bar->k_full[s], (nk[s] - 1) & 1, a.status);
+          if (nk[s]) wait_warp(&bar->k_full[s], (nk[s] - 1) & 1, a.status);
         for (int s = 0; s < 2; ++s)
-          if (nv[s]) wait(&bar->v_full[s], (nv[s] - 1) & 1, a.status);
+          if (nv[s]) wait_warp(&bar->v_full[s], (nv[s] - 1) & 1, a.status);
       }
     }
   } else if (warp == 9) {
@@ -433,46 +443,56 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
   const uint32_t tmem = bar->tmem_base;
 
   if (warp == kLoadWarp) {
-    // ------------------------------------------------ TMA loads (lane 0)
+    // ------------------------------------------------ TMA loads (the warp waits converged,
+    // lane 0 issues the copies)
     uint32_t nq[kQStages] = {0, 0, 0}, ndo[2] = {0, 0};
     const int32_t ky = w.k_base + c * kRows;
-    if (lane == 0 && n_it > 0) {
-      ptx::mbar_expect_tx(&bar->kv_full, 2 * kTileBytes);
-      ptx::tma_load_2d(smem + OFF_K, &tmK, &bar->kv_full, g * kD, ky);
-      ptx::tma_load_2d(smem + OFF_K + kHalfBytes, &tmK, &bar->kv_full, g * kD + 64, ky);
-      ptx::tma_load_2d(smem + OFF_V, &tmV, &bar->kv_full, g * kD, ky);
-      ptx::tma_load_2d(smem + OFF_V + kHalfBytes, &tmV, &bar->kv_full, g * kD + 64, ky);
+    if (n_it > 0) {
+      if (lane == 0) {
+        ptx::mbar_expect_tx(&bar->kv_full, 2 * kTileBytes);
+        ptx::tma_load_2d(smem + OFF_K, &tmK, &bar->kv_full, g * kD, ky);
+        ptx::tma_load_2d(smem + OFF_K + kHalfBytes, &tmK, &bar->kv_full, g * kD + 64, ky);
+        ptx::tma_load_2d(smem + OFF_V, &tmV, &bar->kv_full, g * kD, ky);
+        ptx::tma_load_2d(smem + OFF_V + kHalfBytes, &tmV, &bar->kv_full, g * kD + 64, ky);
+      }
+      __syncwarp();
       for (int i = 0; i < n_it; ++i) {
         const int sq = i % kQStages, s = i & 1;
         const uint32_t n = (uint32_t)(i >> 1);
         const int h = g * group + i % group;
         const int32_t qy = w.q_base + (nqt - 1 - i / group) * kRows;
-        if (aborted(&bar->abort)) break;
-        bool ok = i < kQStages || wait(&bar->q_empty[sq], (uint32_t)(i / kQStages - 1) & 1, a.status);
+        if (__any_sync(0xffffffffu, aborted(&bar->abort))) break;
+        bool ok = i < kQStages || wait_warp(&bar->q_empty[sq], (uint32_t)(i / kQStages - 1) & 1, a.status);
         if (ok) {
-          ptx::mbar_expect_tx(&bar->q_full[sq], kTileBytes);
-          ptx::tma_load_2d(smem + OFF_Q + sq * kTileBytes, &tmQ, &bar->q_full[sq], h * kD, qy);
-          ptx::tma_load_2d(smem + OFF_Q + sq * kTileBytes + kHalfBytes, &tmQ, &bar->q_full[sq], h * kD + 64, qy);
+          if (lane == 0) {
+            ptx::mbar_expect_tx(&bar->q_full[sq], kTileBytes);
+            ptx::tma_load_2d(smem + OFF_Q + sq * kTileBytes, &tmQ, &bar->q_full[sq], h * kD, qy);
+            ptx::tma_load_2d(smem + OFF_Q + sq * kTileBytes + kHalfBytes, &tmQ, &bar->q_full[sq], h * kD + 64, qy);
+          }
+          __syncwarp();
           ++nq[sq];
-          ok = i < 2 || wait(&bar->do_empty[s], (n - 1) & 1, a.status);
+          ok = i < 2 || wait_warp(&bar->do_empty[s], (n - 1) & 1, a.status);
         }
         if (ok) {
-          ptx::mbar_expect_tx(&bar->do_full[s], kTileBytes);
-          ptx::tma_load_2d(smem + OFF_DO + s * kTileBytes, &tmdO, &bar->do_full[s], h * kD, qy);
-          ptx::tma_load_2d(smem + OFF_DO + s * kTileBytes + kHalfBytes, &tmdO, &bar->do_full[s], h * kD + 64, qy);
+          if (lane == 0) {
+            ptx::mbar_expect_tx(&bar->do_full[s], kTileBytes);
+            ptx::tma_load_2d(smem + OFF_DO + s * kTileBytes, &tmdO, &bar->do_full[s], h * kD, qy);
+            ptx::tma_load_2d(smem + OFF_DO + s * kTileBytes + kHalfBytes, &tmdO, &bar->do_full[s], h * kD + 64, qy);
+          }
+          __syncwarp();
           ++ndo[s];
         }
         if (!ok) {
-          set_abort(&bar->abort);
+          if (lane == 0) set_abort(&bar->abort);
           break;
         }
       }
-      if (aborted(&bar->abort)) {
-        wait(&bar->kv_full, 0, a.status);
+      if (__any_sync(0xffffffffu, aborted(&bar->abort))) {
+        wait_warp(&bar->kv_full, 0, a.status);
         for (int s = 0; s < kQStages; ++s)
-          if (nq[s]) wait(&bar->q_full[s], (nq[s] - 1) & 1, a.status);
+          if (nq[s]) wait_warp(&bar->q_full[s], (nq[s] - 1) & 1, a.status);
         for (int s = 0; s < 2; ++s)
-          if (ndo[s]) wait(&bar->do_full[s], (ndo[s] - 1) & 1, a.status);
+          if (ndo[s]) wait_warp(&bar->do_full[s], (ndo[s] - 1) & 1, a.status);
       }
     }
     __syncwarp();

@@ -68,28 +68,32 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = bar->tmem_base;
 
   if (warp == 4) {
-    if (lane == 0 && nkb > 0) {
+    // the warp waits converged, lane 0 issues the copies
+    if (nkb > 0) {
       uint32_t nf[kStages] = {0, 0, 0};
       for (int c = 0; c < nkb; ++c) {
         const int s = c % kStages;
-        if (aborted(&bar->abort)) break;
-        if (c >= kStages && !wait(&bar->empty[s], (uint32_t)(c / kStages - 1) & 1, a.status)) {
-          set_abort(&bar->abort);
+        if (__any_sync(0xffffffffu, aborted(&bar->abort))) break;
+        if (c >= kStages && !wait_warp(&bar->empty[s], (uint32_t)(c / kStages - 1) & 1, a.status)) {
+          if (lane == 0) set_abort(&bar->abort);
           break;
         }
-        const int gk = gfirst + c;
-        const int64_t slot = ((int64_t)a.kpair_off[gk] + (t - a.ktiles[gk].a0)) * a.hq + h;
-        const int32_t yk = w.k_base + c * kRows;
-        uint8_t* st = smem + s * kStageBytes;
-        ptx::mbar_expect_tx(&bar->full[s], kStageBytes);
-        ptx::bulk_load(st, static_cast<const uint8_t*>(a.ds) + slot * kTileBytes, kTileBytes, &bar->full[s]);
-        ptx::tma_load_2d(st + kTileBytes, &tmK, &bar->full[s], g * kD, yk);
-        ptx::tma_load_2d(st + kTileBytes + kHalfBytes, &tmK, &bar->full[s], g * kD + 64, yk);
+        if (lane == 0) {
+          const int gk = gfirst + c;
+          const int64_t slot = ((int64_t)a.kpair_off[gk] + (t - a.ktiles[gk].a0)) * a.hq + h;
+          const int32_t yk = w.k_base + c * kRows;
+          uint8_t* st = smem + s * kStageBytes;
+          ptx::mbar_expect_tx(&bar->full[s], kStageBytes);
+          ptx::bulk_load(st, static_cast<const uint8_t*>(a.ds) + slot * kTileBytes, kTileBytes, &bar->full[s]);
+          ptx::tma_load_2d(st + kTileBytes, &tmK, &bar->full[s], g * kD, yk);
+          ptx::tma_load_2d(st + kTileBytes + kHalfBytes, &tmK, &bar->full[s], g * kD + 64, yk);
+        }
+        __syncwarp();
         ++nf[s];
       }
-      if (aborted(&bar->abort))
+      if (__any_sync(0xffffffffu, aborted(&bar->abort)))
         for (int s = 0; s < kStages; ++s)
-          if (nf[s]) wait(&bar->full[s], (nf[s] - 1) & 1, a.status);
+          if (nf[s]) wait_warp(&bar->full[s], (nf[s] - 1) & 1, a.status);
     }
   } else if (warp == 5) {
     // the whole warp runs the loop, one elected lane issues each instruction

@@ -95,38 +95,54 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = bar->tmem_base;
 
   if (warp == 4) {
-    // ------------------------------------------------------------ producer
-    if (lane == 0 && nkb > 0) {
-      ptx::tma_prefetch_desc(&tmQ);
-      ptx::tma_prefetch_desc(&tmK);
-      ptx::tma_prefetch_desc(&tmV);
-      const int32_t qy = w.q_base + w.tile * kRows;
-      ptx::mbar_expect_tx(&bar->q_full, kTileBytes);
-      ptx::tma_load_2d(smem + OFF_Q, &tmQ, &bar->q_full, h * kD, qy);
-      ptx::tma_load_2d(smem + OFF_Q + kHalfBytes, &tmQ, &bar->q_full, h * kD + 64, qy);
+    // ------------------------------------------------------------ producer (the warp waits
+    // converged, lane 0 issues the copies)
+    if (nkb > 0) {
+      if (lane == 0) {
+        ptx::tma_prefetch_desc(&tmQ);
+        ptx::tma_prefetch_desc(&tmK);
+        ptx::tma_prefetch_desc(&tmV);
+        const int32_t qy = w.q_base + w.tile * kRows;
+        ptx::mbar_expect_tx(&bar->q_full, kTileBytes);
+        ptx::tma_load_2d(smem + OFF_Q, &tmQ, &bar->q_full, h * kD, qy);
+        ptx::tma_load_2d(smem + OFF_Q + kHalfBytes, &tmQ, &bar->q_full, h * kD + 64, qy);
+      }
+      __syncwarp();
       uint32_t nk[kStages] = {0, 0}, nv[kStages] = {0, 0};  // loads issued per stage barrier
       for (int j = 0; j < nkb; ++j) {
         const int s = j & 1;
         const uint32_t n = (uint32_t)(j >> 1);
-        if (aborted(bar)) break;
+        if (__any_sync(0xffffffffu, aborted(bar))) break;
         const int32_t ky = w.k_base + j * kRows;
-        if (j >= kStages && !wait(&bar->k_empty[s], (n - 1) & 1, a.status)) { set_abort(bar); break; }
-        ptx::mbar_expect_tx(&bar->k_full[s], kTileBytes);
-        ptx::tma_load_2d(smem + OFF_K + s * kTileBytes, &tmK, &bar->k_full[s], g * kD, ky);
-        ptx::tma_load_2d(smem + OFF_K + s * kTileBytes + kHalfBytes, &tmK, &bar->k_full[s], g * kD + 64, ky);
+        if (j >= kStages && !wait_warp(&bar->k_empty[s], (n - 1) & 1, a.status)) {
+          if (lane == 0) set_abort(bar);
+          break;
+        }
+        if (lane == 0) {
+          ptx::mbar_expect_tx(&bar->k_full[s], kTileBytes);
+          ptx::tma_load_2d(smem + OFF_K + s * kTileBytes, &tmK, &bar->k_full[s], g * kD, ky);
+          ptx::tma_load_2d(smem + OFF_K + s * kTileBytes + kHalfBytes, &tmK, &bar->k_full[s], g * kD + 64, ky);
+        }
+        __syncwarp();
         ++nk[s];
-        if (j >= kStages && !wait(&bar->v_empty[s], (n - 1) & 1, a.status)) { set_abort(bar); break; }
-        ptx::mbar_expect_tx(&bar->v_full[s], kTileBytes);
-        ptx::tma_load_2d(smem + OFF_V + s * kTileBytes, &tmV, &bar->v_full[s], g * kD, ky);
-        ptx::tma_load_2d(smem + OFF_V + s * kTileBytes + kHalfBytes, &tmV, &bar->v_full[s], g * kD + 64, ky);
+        if (j >= kStages && !wait_warp(&bar->v_empty[s], (n - 1) & 1, a.status)) {
+          if (lane == 0) set_abort(bar);
+          break;
+        }
+        if (lane == 0) {
+          ptx::mbar_expect_tx(&bar->v_full[s], kTileBytes);
+          ptx::tma_load_2d(smem + OFF_V + s * kTileBytes, &tmV, &bar->v_full[s], g * kD, ky);
+          ptx::tma_load_2d(smem + OFF_V + s * kTileBytes + kHalfBytes, &tmV, &bar->v_full[s], g * kD + 64, ky);
+        }
+        __syncwarp();
         ++nv[s];
       }
-      if (aborted(bar)) {
-        // wait (bounded) for this thread's own copies still in flight
-        wait(&bar->q_full, 0, a.status);
+      if (__any_sync(0xffffffffu, aborted(bar))) {
+        // wait (bounded) for this warp's own copies still in flight
+        wait_warp(&bar->q_full, 0, a.status);
         for (int s = 0; s < kStages; ++s) {
-          if (nk[s]) wait(&bar->k_full[s], (nk[s] - 1) & 1, a.status);
-          if (nv[s]) wait(&bar->v_full[s], (nv[s] - 1) & 1, a.status);
+          if (nk[s]) wait_warp(&bar->k_full[s], (nk[s] - 1) & 1, a.status);
+          if (nv[s]) wait_warp(&bar->v_full[s], (nv[s] - 1) & 1, a.status);
         }
       }
     }
