@@ -362,8 +362,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ------------------------------------------------------------------ dK / dV
 namespace dkv {
 // Q is read by the first (S^T) and the last (dK) MMA of an iteration, so it
-// gets a 3-stage ring; dO (dP^T early, dV late) 2 stages; P^T and dS^T live in
-// tensor memory over the dP^T they came from.
+// gets a 3-stage ring; dO (dP^T early, dV late) 2 stages.  P^T lives in tensor
+// memory over the S^T it came from and dS^T over the dP^T it came from, so dV
+// can start as soon as P is written and dP^T of the next tile only waits for dK.
 constexpr int kQStages = 3;
 constexpr uint32_t OFF_K = 0, OFF_V = kTileBytes, OFF_Q = 2 * kTileBytes, OFF_DO = 5 * kTileBytes,
                    OFF_META = 7 * kTileBytes;
@@ -379,7 +380,7 @@ constexpr int kThreads = 352;
 struct Bars {
   uint64_t kv_full;
   uint64_t q_full[kQStages], q_empty[kQStages], do_full[2], do_empty[2], meta_full[2], meta_empty[2];
-  uint64_t s_full, dp_full, s_free, p_full, dvk_done, final_mma;
+  uint64_t s_full, dp_full, pt_full, p_full, dv_done, dk_done, final_mma;
   uint32_t tmem_base;
   int32_t abort;
   uint32_t full[2][2];  // per meta stage and warpgroup: all 64 queries see all 128 keys
@@ -426,9 +427,10 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
     }
     ptx::mbar_init(&bar->s_full, 1);
     ptx::mbar_init(&bar->dp_full, 1);
-    ptx::mbar_init(&bar->s_free, kComputeThreads);
+    ptx::mbar_init(&bar->pt_full, kComputeThreads);
     ptx::mbar_init(&bar->p_full, kComputeThreads);
-    ptx::mbar_init(&bar->dvk_done, 1);
+    ptx::mbar_init(&bar->dv_done, 1);
+    ptx::mbar_init(&bar->dk_done, 1);
     ptx::mbar_init(&bar->final_mma, 1);
     bar->abort = 0;
     ptx::fence_mbar_init();
@@ -551,50 +553,62 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
           ptx::mma_bf16_ss_warp(tmem + TM_DP, desc_kmajor(sV, kk), desc_kmajor(sdO, kk), idesc_nt, kk > 0 ? 1u : 0u);
         ptx::mma_commit_warp(&bar->dp_full);
       };
-      auto issue_dvk = [&](int i) {
-        const int s = i & 1, sq = i % kQStages;
-        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + sq * kTileBytes);
+      // P^T (bf16, two queries per column) sits in the S^T columns and dS^T in the dP^T
+      // columns: warpgroup wg's queries [64 wg, 64 wg + 64) at column 64 wg + [0, 32)
+      auto issue_dv = [&](int i) {
+        const int s = i & 1;
         const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + s * kTileBytes);
-        // P^T and dS^T (bf16, two queries per column) sit in the dP^T columns: warpgroup wg's
-        // queries [64 wg, 64 wg + 64) have P^T at TM_DP + 64 wg + [0,32) and dS^T at + [32,64)
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ts_warp(tmem + TM_DV, tmem + TM_DP + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sdO, kk),
+          ptx::mma_bf16_ts_warp(tmem + TM_DV, tmem + TM_S + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sdO, kk),
                                 idesc_nn, (i > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma_commit_warp(&bar->do_empty[s]);
+        ptx::mma_commit_warp(&bar->dv_done);
+      };
+      auto issue_dk = [&](int i) {
+        const int sq = i % kQStages;
+        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + sq * kTileBytes);
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ts_warp(tmem + TM_DK, tmem + TM_DP + 32 + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sQ, kk),
+          ptx::mma_bf16_ts_warp(tmem + TM_DK, tmem + TM_DP + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sQ, kk),
                                 idesc_nn, (i > 0 || kk > 0) ? 1u : 0u);
         ptx::mma_commit_warp(&bar->q_empty[sq]);
-        ptx::mma_commit_warp(&bar->do_empty[s]);
-        ptx::mma_commit_warp(&bar->dvk_done);
+        ptx::mma_commit_warp(&bar->dk_done);
       };
       // Event-driven issue, in order of urgency (the tensor pipe runs MMAs in
       // issue order, so whatever is issued first runs first):
-      //   dV_i, dK_i  need P^T_i and dS^T_i written (p_full)
-      //   dP_i        needs dO_i and dV_{i-1}, dK_{i-1} issued (it overwrites the
-      //               P^T / dS^T they read; MMAs of this thread execute in order,
-      //               or, with kFlagDrainTmemReuse, they completed)
-      //   S_i         needs Q_i and S_{i-1} read by the compute warps (s_free)
+      //   dK_i  needs dS^T_i written (p_full)
+      //   dP_i  needs dO_i and dK_{i-1} issued (it overwrites the dS^T dK_{i-1}
+      //         reads; MMAs of this thread execute in order, or, with
+      //         kFlagDrainTmemReuse, dK_{i-1} completed)
+      //   dV_i  needs P^T_i written (pt_full) and dP_i issued (both read dO_i)
+      //   S_i   needs Q_i and dV_{i-1} issued (it overwrites the P^T dV_{i-1}
+      //         reads; in order, or with the flag, dV_{i-1} completed)
       bool ok = wait_warp(&bar->kv_full, 0, a.status);
-      int ns = 0, np = 0, nv = 0;
+      int ns = 0, np = 0, nv = 0, nk = 0;
       uint64_t t_idle = 0;
-      while (ok && nv < n_it) {
+      while (ok && nk < n_it) {
         bool progressed = false;
-        if (nv < np && ptx::mbar_test_warp(&bar->p_full, (uint32_t)nv & 1)) {
+        if (nk < nv && ptx::mbar_test_warp(&bar->p_full, (uint32_t)nk & 1)) {
           ptx::tc_fence_after();
-          issue_dvk(nv++);
+          issue_dk(nk++);
           progressed = true;
         }
-        if (np < n_it && np <= nv && ptx::mbar_test_warp(&bar->do_full[np & 1], (uint32_t)(np >> 1) & 1) &&
+        if (np < n_it && np <= nk && ptx::mbar_test_warp(&bar->do_full[np & 1], (uint32_t)(np >> 1) & 1) &&
             (np == 0 || !(a.flags & kFlagDrainTmemReuse) ||
-             ptx::mbar_test_warp(&bar->dvk_done, (uint32_t)(np - 1) & 1))) {
+             ptx::mbar_test_warp(&bar->dk_done, (uint32_t)(np - 1) & 1))) {
           ptx::tc_fence_after();
           issue_dp(np++);
           progressed = true;
         }
-        if (ns < n_it && (ns == 0 || ptx::mbar_test_warp(&bar->s_free, (uint32_t)(ns - 1) & 1)) &&
-            ptx::mbar_test_warp(&bar->q_full[ns % kQStages], (uint32_t)(ns / kQStages) & 1)) {
+        if (nv < np && ptx::mbar_test_warp(&bar->pt_full, (uint32_t)nv & 1)) {
+          ptx::tc_fence_after();
+          issue_dv(nv++);
+          progressed = true;
+        }
+        if (ns < n_it && ns <= nv && ptx::mbar_test_warp(&bar->q_full[ns % kQStages], (uint32_t)(ns / kQStages) & 1) &&
+            (ns == 0 || !(a.flags & kFlagDrainTmemReuse) ||
+             ptx::mbar_test_warp(&bar->dv_done, (uint32_t)(ns - 1) & 1))) {
           ptx::tc_fence_after();
           issue_s(ns++);
           progressed = true;
@@ -648,11 +662,8 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
         ptx::tmem_ld_wait();
         ptx::reg_fence(sv[0]);
         ptx::reg_fence(sv[1]);
-        ptx::tc_fence_before();
-        ptx::mbar_arrive(&bar->s_free);
         if (bar->full[s][wg]) {
           // every key of the tile is visible to every query of this warpgroup
-#pragma unroll
           const float2 sl2x2 = make_float2(sl2, sl2);
 #pragma unroll
           for (int q4 = 0; q4 < 16; ++q4) {
@@ -682,6 +693,11 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
           }
         }
       }
+      // P^T over this warpgroup's (already read) S^T columns; dV may start
+      ptx::tmem_st32(tS, pp);
+      ptx::tmem_st_wait();
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&bar->pt_full);
       if (ds_dst) {
 #pragma unroll
         for (int k = 0; k < 4; ++k)
@@ -714,9 +730,8 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
         }
       }
       ptx::mbar_arrive(&bar->meta_empty[s]);
-      // P^T and dS^T over this warpgroup's (already read) dP^T columns
-      ptx::tmem_st32(tP, pp);
-      ptx::tmem_st32(tP + 32, pd);
+      // dS^T over this warpgroup's (already read) dP^T columns
+      ptx::tmem_st32(tP, pd);
       ptx::tmem_st_wait();
       ptx::tc_fence_before();
       ptx::mbar_arrive(&bar->p_full);
