@@ -274,11 +274,8 @@ def run_cuda(args, w):
         ism.check_status(dev)
         return
 
-    # per-kernel timers for the roofline (on the library's launch stream)
+    # timed steps: CUDA events around each step only
     stream = torch.cuda.current_stream(dev)
-    kinds = {"fwd": ism.KERNEL_FWD, "bwd_dkdv": ism.KERNEL_BWD_DKDV, "bwd_dq": ism.KERNEL_BWD_DQ,
-             "bwd_pre": ism.KERNEL_BWD_PRE, "meta": ism.KERNEL_META}
-    ktimes = {n: [] for n in kinds}
     step_ms = []
     launches0 = ism.kernel_launches()
     with ClockSampler(dev.index) as clocks:
@@ -286,24 +283,35 @@ def run_cuda(args, w):
         torch.cuda.synchronize()
         for _ in range(args.steps):
             flush.fill_(1)  # evict L2 between timed steps (outside the step's events)
-            ev = {n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for n in kinds}
-            for n, kid in kinds.items():
-                for e in ev[n]:
-                    e.record(stream)  # creates the event; the library re-records it around its launch
-                ism.set_kernel_timer(kid, *ev[n])
             s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             s0.record(stream)
             step()
             s1.record(stream)
             s1.synchronize()
             step_ms.append(s0.elapsed_time(s1))
-            for n in kinds:
-                ktimes[n].append(ev[n][0].elapsed_time(ev[n][1]))
         torch.cuda.synchronize()
         barrier(world)
+    launches = ism.kernel_launches() - launches0
+    ism.check_status(dev)
+
+    # per-kernel times for the rooflines, from separate steps run with the
+    # library's kernel-timer hooks (events recorded on its launch stream)
+    kinds = {"fwd": ism.KERNEL_FWD, "bwd_dkdv": ism.KERNEL_BWD_DKDV, "bwd_dq": ism.KERNEL_BWD_DQ,
+             "bwd_pre": ism.KERNEL_BWD_PRE, "meta": ism.KERNEL_META}
+    ktimes = {n: [] for n in kinds}
+    for _ in range(max(3, min(args.steps, 10))):
+        flush.fill_(1)
+        ev = {n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for n in kinds}
+        for n, kid in kinds.items():
+            for e in ev[n]:
+                e.record(stream)  # creates the event; the library re-records it around its launch
+            ism.set_kernel_timer(kid, *ev[n])
+        step()
+        torch.cuda.synchronize()
+        for n in kinds:
+            ktimes[n].append(ev[n][0].elapsed_time(ev[n][1]))
     for kid in kinds.values():
         ism.set_kernel_timer(kid)
-    launches = ism.kernel_launches() - launches0
     ism.check_status(dev)
 
     total_ms = max_over_ranks(float(np.sum(step_ms)), world)
