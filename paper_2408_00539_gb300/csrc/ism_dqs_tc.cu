@@ -2,9 +2,12 @@
 //
 // When the dK/dV kernel has kept every visible tile pair's dS (bf16, 128
 // queries x 128 keys, 32 KiB a tile) in the workspace, dQ_t = scale *
-// sum_c dS_tc K_c needs no recomputation of S, P or dP: one CTA per (query
-// tile, query head) streams the (dS, K) tile pairs of the tile's non-empty
-// key blocks through a 3-stage ring and accumulates dQ in tensor memory.
+// sum_c dS_tc K_c needs no recomputation of S, P or dP.  A persistent CTA per
+// SM walks the (query tile, query head) items in cost order; for each it
+// streams the (dS, K) tile pairs of the tile's non-empty key blocks through a
+// 3-stage ring that runs on across items, and accumulates dQ in one of two
+// tensor-memory accumulators, so the epilogue of one item overlaps the MMAs
+// of the next.
 // A dS tile is stored 8-interleaved (16-byte units of 8 consecutive queries
 // of one key, the 128 keys of a query group adjacent), which is the no-swizzle
 // MN-major operand layout: one contiguous bulk copy moves it into shared
@@ -19,16 +22,17 @@ namespace {
 
 constexpr int kThreads = 192;
 constexpr int kStages = 3;
-constexpr uint32_t kStageBytes = 2 * kTileBytes;  // dS^T tile + K tile
+constexpr uint32_t kStageBytes = 2 * kTileBytes;  // dS tile + K tile
 constexpr uint32_t OFF_BAR = kStages * kStageBytes;
 constexpr uint32_t kSmemBytes = OFF_BAR + 128 + 1024;
-constexpr uint32_t kTmemCols = 128;
+constexpr uint32_t kTmemCols = 256;  // two 128-column dQ accumulators
 
 struct Bars {
-  uint64_t full[kStages], empty[kStages], done;
+  uint64_t full[kStages], empty[kStages], acc_full[2], acc_empty[2], final_mma;
   uint32_t tmem_base;
   int32_t abort;
 };
+static_assert(sizeof(Bars) <= 128, "barrier block");
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
@@ -36,25 +40,40 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 __device__ __forceinline__ bool aborted(const int32_t* f) { return *reinterpret_cast<const volatile int32_t*>(f) != 0; }
 __device__ __forceinline__ void set_abort(int32_t* f) { *reinterpret_cast<volatile int32_t*>(f) = 1; }
 
+// Work item `item` = (query tile q_order[item / hq], query head item % hq).
+struct Item {
+  int h, g, t, nkb, gfirst;
+  Tile w;
+};
+__device__ __forceinline__ Item decode(const AttnArgs& a, int64_t item) {
+  Item it;
+  it.h = (int)(item % a.hq);
+  const int gq = a.q_order[item / a.hq];
+  it.w = a.qtiles[gq];
+  it.g = it.h / (a.hq / a.hkv);
+  it.nkb = it.w.a1;
+  it.t = it.w.tile;
+  it.gfirst = gq - it.t;  // q-tiles and k-tiles of a sequence are numbered alike
+  return it;
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
-    dq_gemm_kernel(const __grid_constant__ CUtensorMap tmK, const AttnArgs a) {
+    dq_gemm_kernel(const __grid_constant__ CUtensorMap tmK, const AttnArgs a, int64_t n_items) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   Bars* bar = reinterpret_cast<Bars*>(smem + OFF_BAR);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = blockIdx.x % a.hq;
-  const int gq = a.q_order[blockIdx.x / a.hq];
-  const Tile w = a.qtiles[gq];
-  const int g = h / (a.hq / a.hkv);
-  const int nkb = w.a1, t = w.tile;
-  const int gfirst = gq - t;  // q-tiles and k-tiles of a sequence are numbered alike
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       ptx::mbar_init(&bar->full[s], 1);
       ptx::mbar_init(&bar->empty[s], 1);
     }
-    ptx::mbar_init(&bar->done, 1);
+    for (int b = 0; b < 2; ++b) {
+      ptx::mbar_init(&bar->acc_full[b], 1);
+      ptx::mbar_init(&bar->acc_empty[b], 128);
+    }
+    ptx::mbar_init(&bar->final_mma, 1);
     bar->abort = 0;
     ptx::fence_mbar_init();
   }
@@ -68,42 +87,53 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = bar->tmem_base;
 
   if (warp == 4) {
-    // the warp waits converged, lane 0 issues the copies
-    if (nkb > 0) {
-      uint32_t nf[kStages] = {0, 0, 0};
-      for (int c = 0; c < nkb; ++c) {
-        const int s = c % kStages;
-        if (__any_sync(0xffffffffu, aborted(&bar->abort))) break;
-        if (c >= kStages && !wait_warp(&bar->empty[s], (uint32_t)(c / kStages - 1) & 1, a.status)) {
+    // ------------------------------------------------ copies (the warp waits converged, lane 0 issues)
+    uint32_t it = 0;  // stage uses so far, across items
+    uint32_t nf[kStages] = {0, 0, 0};
+    bool ok = true;
+    for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
+      const Item x = decode(a, item);
+      for (int c = 0; c < x.nkb; ++c, ++it) {
+        const int s = (int)(it % kStages);
+        if (__any_sync(0xffffffffu, aborted(&bar->abort))) { ok = false; break; }
+        if (it >= kStages && !wait_warp(&bar->empty[s], (it / kStages - 1) & 1, a.status)) {
           if (lane == 0) set_abort(&bar->abort);
+          ok = false;
           break;
         }
         if (lane == 0) {
-          const int gk = gfirst + c;
-          const int64_t slot = ((int64_t)a.kpair_off[gk] + (t - a.ktiles[gk].a0)) * a.hq + h;
-          const int32_t yk = w.k_base + c * kRows;
+          const int gk = x.gfirst + c;
+          const int64_t slot = ((int64_t)a.kpair_off[gk] + (x.t - a.ktiles[gk].a0)) * a.hq + x.h;
+          const int32_t yk = x.w.k_base + c * kRows;
           uint8_t* st = smem + s * kStageBytes;
           ptx::mbar_expect_tx(&bar->full[s], kStageBytes);
           ptx::bulk_load(st, static_cast<const uint8_t*>(a.ds) + slot * kTileBytes, kTileBytes, &bar->full[s]);
-          ptx::tma_load_2d(st + kTileBytes, &tmK, &bar->full[s], g * kD, yk);
-          ptx::tma_load_2d(st + kTileBytes + kHalfBytes, &tmK, &bar->full[s], g * kD + 64, yk);
+          ptx::tma_load_2d(st + kTileBytes, &tmK, &bar->full[s], x.g * kD, yk);
+          ptx::tma_load_2d(st + kTileBytes + kHalfBytes, &tmK, &bar->full[s], x.g * kD + 64, yk);
         }
         __syncwarp();
         ++nf[s];
       }
-      if (__any_sync(0xffffffffu, aborted(&bar->abort)))
-        for (int s = 0; s < kStages; ++s)
-          if (nf[s]) wait_warp(&bar->full[s], (nf[s] - 1) & 1, a.status);
     }
+    if (!ok)
+      for (int s = 0; s < kStages; ++s)
+        if (nf[s]) wait_warp(&bar->full[s], (nf[s] - 1) & 1, a.status);
   } else if (warp == 5) {
-    // the whole warp runs the loop, one elected lane issues each instruction
-    if (nkb > 0) {
-      constexpr uint32_t idesc = ptx::idesc_bf16_f32(128, 128, 1, 1);  // A and B MN-major
-      bool ok = true;
-      for (int c = 0; c < nkb; ++c) {
-        const int s = c % kStages;
+    // ------------------------------------------------ MMA (the whole warp runs the loop,
+    // one elected lane issues each instruction)
+    constexpr uint32_t idesc = ptx::idesc_bf16_f32(128, 128, 1, 1);  // A and B MN-major
+    uint32_t it = 0, local = 0;
+    bool ok = true;
+    for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x, ++local) {
+      const Item x = decode(a, item);
+      const uint32_t b = local & 1, acc = tmem + 128u * b;
+      // the epilogue has read this accumulator's previous item
+      if (local >= 2 && !wait_warp(&bar->acc_empty[b], ((local >> 1) - 1) & 1, a.status)) { ok = false; break; }
+      ptx::tc_fence_after();
+      for (int c = 0; c < x.nkb; ++c, ++it) {
+        const int s = (int)(it % kStages);
         if (__shfl_sync(0xffffffffu, aborted(&bar->abort) ? 1 : 0, 0) ||
-            !wait_warp(&bar->full[s], (uint32_t)(c / kStages) & 1, a.status)) {
+            !wait_warp(&bar->full[s], (it / kStages) & 1, a.status)) {
           ok = false;
           break;
         }
@@ -111,47 +141,59 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t sDS = ptx::smem_u32(smem + s * kStageBytes), sK = sDS + kTileBytes;
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss_warp(tmem, desc_ilv_mnmajor(sDS, kk), desc_mnmajor(sK, kk), idesc, (c > 0 || kk > 0) ? 1u : 0u);
+          ptx::mma_bf16_ss_warp(acc, desc_ilv_mnmajor(sDS, kk), desc_mnmajor(sK, kk), idesc,
+                                (c > 0 || kk > 0) ? 1u : 0u);
         ptx::mma_commit_warp(&bar->empty[s]);
       }
-      if (!ok && lane == 0) set_abort(&bar->abort);
-      __syncwarp();
-      ptx::mma_commit_warp(&bar->done);
-      wait_warp(&bar->done, 0, a.status);
+      if (!ok) break;
+      ptx::mma_commit_warp(&bar->acc_full[b]);
     }
+    if (!ok && lane == 0) set_abort(&bar->abort);
     __syncwarp();
+    ptx::mma_commit_warp(&bar->final_mma);
+    wait_warp(&bar->final_mma, 0, a.status);
   } else {
-    // epilogue: thread = query row
+    // ------------------------------------------------ epilogue: thread = query row
     const int r = threadIdx.x;
-    const int row = t * kRows + r;
-    const bool valid = row < w.q_len;
     const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
-    const bool ok = nkb > 0 && wait(&bar->done, 0, a.status) && !aborted(&bar->abort);
-    if (ok) ptx::tc_fence_after();
-    uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) +
-                                          ((int64_t)w.q_base + row) * a.hq * kD + h * kD);
-#pragma unroll 1
-    for (int q4 = 0; q4 < 4; ++q4) {
-      uint32_t v[32];
-      if (ok) {
-        ptx::tmem_ld32(tmem + lane_addr + 32 * q4, v);
-        ptx::tmem_ld_wait();
-        ptx::reg_fence(v);
-      } else {
-#pragma unroll
-        for (int k = 0; k < 32; ++k) v[k] = 0u;
+    uint32_t local = 0;
+    for (int64_t item = blockIdx.x; item < n_items; item += gridDim.x, ++local) {
+      const Item x = decode(a, item);
+      const uint32_t b = local & 1, acc = tmem + lane_addr + 128u * b;
+      const int row = x.t * kRows + r;
+      const bool valid = row < x.w.q_len;
+      if (!wait(&bar->acc_full[b], (local >> 1) & 1, a.status) || aborted(&bar->abort)) {
+        set_abort(&bar->abort);
+        break;
       }
-      if (valid && (ok || nkb == 0)) {
+      ptx::tc_fence_after();
+      uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) +
+                                            ((int64_t)x.w.q_base + row) * a.hq * kD + x.h * kD);
+#pragma unroll 1
+      for (int q4 = 0; q4 < 4; ++q4) {
+        uint32_t v[32];
+        if (x.nkb > 0) {
+          ptx::tmem_ld32(acc + 32 * q4, v);
+          ptx::tmem_ld_wait();
+          ptx::reg_fence(v);
+        } else {
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          uint4 o;
-          o.x = pack_bf16(__uint_as_float(v[8 * i + 0]) * a.scale, __uint_as_float(v[8 * i + 1]) * a.scale);
-          o.y = pack_bf16(__uint_as_float(v[8 * i + 2]) * a.scale, __uint_as_float(v[8 * i + 3]) * a.scale);
-          o.z = pack_bf16(__uint_as_float(v[8 * i + 4]) * a.scale, __uint_as_float(v[8 * i + 5]) * a.scale);
-          o.w = pack_bf16(__uint_as_float(v[8 * i + 6]) * a.scale, __uint_as_float(v[8 * i + 7]) * a.scale);
-          dst[4 * q4 + i] = o;
+          for (int k = 0; k < 32; ++k) v[k] = 0u;
+        }
+        if (valid) {
+#pragma unroll
+          for (int i = 0; i < 4; ++i) {
+            uint4 o;
+            o.x = pack_bf16(__uint_as_float(v[8 * i + 0]) * a.scale, __uint_as_float(v[8 * i + 1]) * a.scale);
+            o.y = pack_bf16(__uint_as_float(v[8 * i + 2]) * a.scale, __uint_as_float(v[8 * i + 3]) * a.scale);
+            o.z = pack_bf16(__uint_as_float(v[8 * i + 4]) * a.scale, __uint_as_float(v[8 * i + 5]) * a.scale);
+            o.w = pack_bf16(__uint_as_float(v[8 * i + 6]) * a.scale, __uint_as_float(v[8 * i + 7]) * a.scale);
+            dst[4 * q4 + i] = o;
+          }
         }
       }
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&bar->acc_empty[b]);
     }
   }
   ptx::tc_fence_before();
@@ -170,7 +212,16 @@ cudaError_t launch_dq_gemm(const AttnArgs& a, const CUtensorMap& tk, cudaStream_
   if ((e = cudaFuncSetAttribute(dq_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
       cudaSuccess)
     return e;
-  dq_gemm_kernel<<<(unsigned)(a.nq * a.hq), kThreads, kSmemBytes, st>>>(tk, a);
+  int dev = 0, sms = 0;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  const int64_t n_items = a.nq * a.hq;
+  int grid = sms;
+  const char* ov = getenv("ISM_DQ_GRID");  // persistent grid size (default: one CTA per SM)
+  if (ov && atoi(ov) > 0) grid = atoi(ov);
+  if (grid > n_items) grid = (int)n_items;
+  if (grid <= 0) return cudaSuccess;
+  dq_gemm_kernel<<<(unsigned)grid, kThreads, kSmemBytes, st>>>(tk, a, n_items);
   return cudaGetLastError();
 }
 
