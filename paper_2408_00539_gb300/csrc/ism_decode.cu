@@ -175,20 +175,28 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
   }
 }
 
-// TMA-pipelined variant for head_dim 128: warp 4 streams 64-key K and V tiles
-// of the chunk into a 3-stage shared-memory ring with TMA; warps 0-3 each take
-// 16 keys of a tile (batches of 32 / G keys, the same butterfly softmax as
-// above) reading the rows from shared memory.  Two CTAs fit on an SM, so
-// about six 32 KB tiles are in flight per SM.
-constexpr int kTmaTile = 64;
-constexpr int kTmaStages = 3;
-constexpr uint32_t kTmaHalf = kTmaTile * 128;       // 64 rows x 64 bf16
-constexpr uint32_t kTmaStageBytes = 4 * kTmaHalf;   // K and V, two halves each
+// TMA-pipelined variant for head_dim 128 and at least two query heads per KV
+// head: warp 4 streams K and V tiles of the chunk into a shared-memory ring
+// with TMA; warps 0-3 each take a quarter of a tile (batches of 32 / G keys,
+// the same butterfly softmax as above) reading the rows from shared memory.
+// Tile rows and ring depth: a warp's share of a tile (kTile / 4 rows) must
+// hold whole batches of 32 / G keys.  A 2-stage ring of 64-key tiles (about
+// 70 KB of shared memory) lets three CTAs share an SM; measured on the 8 x 16K
+// cache it beats 3 or 4 stages and 32-key tiles.
+template <int G> struct TmaCfg {
+  static constexpr int kTile = 64;
+  static constexpr int kStages = 2;
+  static constexpr uint32_t kHalf = kTile * 128;      // kTile rows x 64 bf16
+  static constexpr uint32_t kStageBytes = 4 * kHalf;  // K and V, two halves each
+};
 
 template <int G>
 __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__ CUtensorMap tmK,
                                                         const __grid_constant__ CUtensorMap tmV, DecodeArgs a) {
-  constexpr int D = 128, DPL = 4, KPI = 32 / G, NB = 16 / KPI;  // batches per warp per tile
+  constexpr int kTmaTile = TmaCfg<G>::kTile, kTmaStages = TmaCfg<G>::kStages;
+  constexpr uint32_t kTmaHalf = TmaCfg<G>::kHalf, kTmaStageBytes = TmaCfg<G>::kStageBytes;
+  constexpr int D = 128, DPL = 4, KPI = 32 / G, RPW = kTmaTile / 4, NB = RPW / KPI;  // batches per warp per tile
+  static_assert(NB >= 1 && RPW % KPI == 0, "a warp's rows must hold whole batches");
   extern __shared__ __align__(128) uint8_t dsm[];
   uint64_t* full = reinterpret_cast<uint64_t*>(dsm + kTmaStages * kTmaStageBytes);
   uint64_t* empty = full + kTmaStages;
@@ -254,7 +262,7 @@ __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__
       const uint8_t* st = dsm + s * kTmaStageBytes;
 #pragma unroll
       for (int nb = 0; nb < NB; ++nb) {
-        const int r0 = warp * 16 + nb * KPI;           // first row of the batch in the tile
+        const int r0 = warp * RPW + nb * KPI;          // first row of the batch in the tile
         const int kb = k0 + t * kTmaTile + r0;         // its key index
         float v[32];
 #pragma unroll
@@ -371,16 +379,19 @@ template <int D, int G>
 cudaError_t run(const DecodeArgs& a, cudaStream_t st) {
   dim3 grid(a.splits, a.hkv, a.batch);
   cudaError_t e;
-  if (a.tma) {
+  // the TMA kernel needs at least two heads per KV head (batches of 32 / G keys)
+  if (a.tma && G >= 2) {
+    using Cfg = TmaCfg<G >= 2 ? G : 2>;
     CUtensorMap tk, tv;
     const uint64_t rows = (uint64_t)a.batch * a.cap;
-    if ((e = tc::make_tmap_bf16_plain(&tk, a.k_cache, (uint64_t)a.hkv * D, rows, kTmaTile)) != cudaSuccess) return e;
-    if ((e = tc::make_tmap_bf16_plain(&tv, a.v_cache, (uint64_t)a.hkv * D, rows, kTmaTile)) != cudaSuccess) return e;
-    const int smem = kTmaStages * kTmaStageBytes + 2 * kTmaStages * 8 + (8 * G + 4 * G * D) * 4;
-    if ((e = cudaFuncSetAttribute(decode_tma_kernel<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) !=
+    if ((e = tc::make_tmap_bf16_plain(&tk, a.k_cache, (uint64_t)a.hkv * D, rows, Cfg::kTile)) != cudaSuccess) return e;
+    if ((e = tc::make_tmap_bf16_plain(&tv, a.v_cache, (uint64_t)a.hkv * D, rows, Cfg::kTile)) != cudaSuccess) return e;
+    const int smem = Cfg::kStages * Cfg::kStageBytes + 2 * Cfg::kStages * 8 + (8 * G + 4 * G * D) * 4;
+    if ((e = cudaFuncSetAttribute(decode_tma_kernel<G >= 2 ? G : 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  smem)) !=
         cudaSuccess)
       return e;
-    decode_tma_kernel<G><<<grid, 160, smem, st>>>(tk, tv, a);
+    decode_tma_kernel<G >= 2 ? G : 2><<<grid, 160, smem, st>>>(tk, tv, a);
   } else {
     decode_split_kernel<D, G><<<grid, kDecWarps * 32, 0, st>>>(a);
   }

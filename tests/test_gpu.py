@@ -258,8 +258,9 @@ def test_prefill_append_matches_one_pass_rows(ism):
     assert diff <= 2e-2, diff
 
 
-def test_decode_steps_small(ism):
-    B, hq, hkv, d, c0, steps = 2, 8, 2, 128, 700, 6
+@pytest.mark.parametrize("hq,hkv", [(8, 2), (4, 4), (8, 1), (4, 2)])
+def test_decode_steps_small(ism, hq, hkv):
+    B, d, c0, steps = 2, 128, 700, 6
     cap = c0 + steps
     kc, vc, qn, kn, vn = _append_inputs(B, cap, None, steps, hq, hkv, d, seed=31)
     kcd, vcd = kc.clone().to(DEV), vc.clone().to(DEV)
