@@ -116,6 +116,16 @@ def test_small_bf16_fwd_bwd(ism, d, path, monkeypatch):
     if path == "cuda_cores":
         monkeypatch.setenv("ISM_FORCE_CUDA_CORES", "1")
     w = _small_bf16(d)
+    _check_small(ism, w, path)
+
+
+@pytest.mark.parametrize("hq,hkv", [(4, 4), (6, 2), (2, 1)])
+def test_small_bf16_group_sizes(ism, hq, hkv):
+    """Query heads per KV head 1 and 3 (one-head forward kernel) and 2."""
+    _check_small(ism, _small_bf16(128, hq=hq, hkv=hkv, seed=hq * 10 + hkv), "default")
+
+
+def _check_small(ism, w, path):
     (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w, minimal_workspace=path == "recompute_dq")
     o_ref, lse_ref = orc.attn_fwd(q, k, v, w.segs, w.softmax_scale)
     dq_ref, dk_ref, dv_ref = orc.attn_bwd(q, k, v, do, w.segs, w.softmax_scale)
@@ -215,10 +225,13 @@ def _append_inputs(B, cap, c_lens, l_new, hq, hkv, d, seed, std=0.5):
     return kc, vc, qn, kn, vn
 
 
-@pytest.mark.parametrize("l_new,segs", [(200, ([40, 41, 120, 200], [0, 1, 0, 1])), (128, ([128], [0])),
-                                        (1, ([1], [1])), (37, ([37], [0]))])
-def test_prefill_append_small(ism, l_new, segs):
-    B, hq, hkv, d = 3, 8, 2, 128
+@pytest.mark.parametrize("l_new,segs,hq,hkv", [(200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2),
+                                                (128, ([128], [0]), 8, 2), (1, ([1], [1]), 8, 2),
+                                                (37, ([37], [0]), 8, 2),
+                                                (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 3, 3),
+                                                (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 6, 2)])
+def test_prefill_append_small(ism, l_new, segs, hq, hkv):
+    B, d = 3, 128
     c_lens = np.array([0, 77, 300], dtype=np.int32)
     cap = 300 + l_new + 5
     kc, vc, qn, kn, vn = _append_inputs(B, cap, c_lens, l_new, hq, hkv, d, seed=l_new)
