@@ -150,6 +150,7 @@ struct Carve {
 
 struct Counts {
   int64_t nq = 0, nk = 0, ntiles = 0;
+  int64_t npairs = 0;  // q-tile pairs (neighbouring q-tiles of a sequence, the last one may be alone)
   int max_cost = 0;
 };
 
@@ -160,6 +161,7 @@ Counts count_tiles(const ism_segments_t* s, int bm, int bn) {
     int64_t nq = (L + bm - 1) / bm, nk = (L + bn - 1) / bn;
     c.nq += nq;
     c.nk += nk;
+    c.npairs += (nq + 1) / 2;
     c.ntiles += nq * nk;
     int mc = (int)(nq > nk ? nq : nk);
     if (mc > c.max_cost) c.max_cost = mc;
@@ -199,11 +201,12 @@ struct PassLayout {
   float* delta;
   int32_t* kpair_off;
   void* ds;
+  int32_t* pair_order;
   size_t bytes;
 };
 
 PassLayout pass_layout(void* ws, const ism_segments_t* s, const Counts& c, int64_t T, int hq, bool bwd,
-                       int64_t ds_slots = 0) {
+                       int64_t ds_slots = 0, bool tile_pairs = false) {
   Carve cv(ws);
   PassLayout L;
   L.kv_end = cv.take<int32_t>(T);
@@ -214,6 +217,7 @@ PassLayout pass_layout(void* ws, const ism_segments_t* s, const Counts& c, int64
   L.delta = bwd ? cv.take<float>((int64_t)hq * T) : nullptr;
   L.kpair_off = ds_slots > 0 ? cv.take<int32_t>(c.nk) : nullptr;
   L.ds = ds_slots > 0 ? static_cast<void*>(cv.take<uint16_t>(ds_slots * kTile * kTile)) : nullptr;
+  L.pair_order = tile_pairs ? cv.take<int32_t>(c.npairs) : nullptr;
   L.bytes = ((cv.off + 255) & ~size_t(255)) + 256;
   return L;
 }
@@ -232,6 +236,15 @@ bool use_tc(const ism_attn_shape_t* sh) {
   return sh->dtype == ISM_BF16 && sh->head_dim == 128 && tc_available() && !force_cuda_cores();
 }
 bool use_tc_bwd(const ism_attn_shape_t* sh) { return use_tc(sh) && tc_bwd_available(); }
+
+// The tensor-core forward pairs two query heads of a KV head per CTA; with an
+// odd number of query heads per KV head it pairs neighbouring query tiles of
+// one head instead, from a work list the metadata pass builds.
+bool fwd_tile_pairs(const ism_attn_shape_t* sh) {
+  if (!use_tc(sh) || (sh->num_heads_q / sh->num_heads_kv) % 2 == 0) return false;
+  const char* e = getenv("ISM_FWD_ONE_HEAD");
+  return !(e && e[0] == '1');
+}
 
 // dS tile slots of the stored-dS backward (pairs x query heads), or 0 where
 // that path does not apply: CUDA-core backward, ISM_BWD_RECOMPUTE_DQ=1, or
@@ -260,7 +273,8 @@ ism_status_t build_pass_meta(const ism_segments_t* s, const Counts& c, const Pas
   ISM_TRY_CUDA(launch_tiles(d, kTile, kTile, L.kv_end, c.nq, bwd ? c.nk : 0, L.qtiles, L.ktiles, nullptr, nullptr,
                             nullptr, nullptr, st),
                "tiles launch");
-  ISM_TRY_CUDA(launch_order(L.qtiles, c.nq, L.ktiles, bwd ? c.nk : 0, c.max_cost, L.q_order, L.k_order, st),
+  ISM_TRY_CUDA(launch_order(L.qtiles, c.nq, L.ktiles, bwd ? c.nk : 0, c.max_cost, L.q_order, L.k_order, st,
+                            L.pair_order),
                "order launch");
   if (L.kpair_off) ISM_TRY_CUDA(launch_pair_offsets(L.ktiles, c.nk, L.kpair_off, st), "pair offsets launch");
   timer_end(ISM_KERNEL_META, st);
@@ -352,7 +366,7 @@ ism_status_t ism_attn_fwd_workspace_size(const ism_segments_t* segs, const ism_a
   if ((r = check_shape(shape)) != ISM_OK) return r;
   if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
   Counts c = count_tiles(segs, kTile, kTile);
-  *bytes = pass_layout(nullptr, segs, c, info.total_tokens, shape->num_heads_q, false).bytes;
+  *bytes = pass_layout(nullptr, segs, c, info.total_tokens, shape->num_heads_q, false, 0, fwd_tile_pairs(shape)).bytes;
   return ISM_OK;
 }
 
@@ -393,7 +407,8 @@ ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || (lse && !aligned16(lse)))
     return fail(ISM_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
   Counts c = count_tiles(segs, kTile, kTile);
-  PassLayout L = pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, false);
+  PassLayout L =
+      pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, false, 0, fwd_tile_pairs(shape));
   if ((r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
   uint32_t* status;
   if ((r = status_ptr(&status)) != ISM_OK) return r;
@@ -405,6 +420,7 @@ ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   a.hq = shape->num_heads_q; a.hkv = shape->num_heads_kv; a.d = shape->head_dim; a.dtype = shape->dtype;
   a.q_rows = info.total_tokens; a.scale = shape->softmax_scale;
   a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order; a.nq = c.nq;
+  a.pair_order = L.pair_order; a.npairs = L.pair_order ? c.npairs : 0;
   a.status = status;
   a.flags = tc_flags();
   timer_begin(ISM_KERNEL_FWD, st);

@@ -1,9 +1,12 @@
-// ISM attention forward, two query heads per CTA (sm_103a tensor cores).
+// ISM attention forward, two (query head, query tile) units per CTA that
+// read the same K/V (sm_103a tensor cores).
 //
 // When the query heads come in pairs that share a KV head (grouped-query
 // attention with an even group size), one CTA computes the same 128-row
-// query tile for both heads of a pair: every K/V block is loaded once and
-// used by both.  The two heads' softmax warpgroups alternate with the tensor
+// query tile for both heads of a pair.  Otherwise (a.pair_order set) it
+// computes two neighbouring query tiles of one head; the second tile sees at
+// least the keys of the first, so it runs the same key blocks and possibly
+// more.  Either way every K/V block is loaded once and used by both units.  The two heads' softmax warpgroups alternate with the tensor
 // core (while one warpgroup turns S_A into P_A, the tensor core computes
 // S_B, and so on).  P is written back into tensor memory over the S it came
 // from and read there as the A operand of O += P V.
@@ -40,6 +43,7 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 __device__ __forceinline__ bool aborted(const int32_t* f) { return *reinterpret_cast<const volatile int32_t*>(f) != 0; }
 __device__ __forceinline__ void set_abort(int32_t* f) { *reinterpret_cast<volatile int32_t*>(f) = 1; }
 
+template <bool kTilePairs>
 __global__ void __launch_bounds__(kThreads, 1)
     fwd_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                     const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
@@ -47,12 +51,31 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = align1024(smem_raw);
   Bars* bar = reinterpret_cast<Bars*>(smem + OFF_BAR);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int npairs = a.hq >> 1;
-  const int hp = blockIdx.x % npairs;
-  const Tile w = a.qtiles[a.q_order[blockIdx.x / npairs]];
-  const int h0 = 2 * hp;
+  Tile w0, w1;
+  int h0, h1, nkb0, nkb1;
+  if constexpr (!kTilePairs) {
+    const int npairs = a.hq >> 1;
+    const int hp = blockIdx.x % npairs;
+    w0 = w1 = a.qtiles[a.q_order[blockIdx.x / npairs]];
+    h0 = 2 * hp;
+    h1 = h0 + 1;
+    nkb0 = nkb1 = w0.a1;
+  } else {
+    h0 = h1 = blockIdx.x % a.hq;
+    const int gq = a.pair_order[blockIdx.x / a.hq];
+    w0 = a.qtiles[gq];
+    bool second = false;
+    if (gq + 1 < a.nq) {
+      w1 = a.qtiles[gq + 1];
+      second = w1.q_base == w0.q_base && w1.tile == w0.tile + 1;
+    }
+    if (!second) w1 = w0;
+    nkb0 = w0.a1;
+    nkb1 = second ? w1.a1 : 0;
+  }
+  const Tile& w = w0;  // K/V rows (k_base) are those of the shared sequence
   const int g = h0 / (a.hq / a.hkv);
-  const int nkb = w.a1, kfull = w.a0;
+  const int nkb = nkb0 > nkb1 ? nkb0 : nkb1;
 
   if (threadIdx.x == 0) {
     ptx::mbar_init(&bar->q_full, 1);
@@ -85,12 +108,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) {
         ptx::tma_prefetch_desc(&tmK);
         ptx::tma_prefetch_desc(&tmV);
-        const int32_t qy = w.q_base + w.tile * kRows;
-        ptx::mbar_expect_tx(&bar->q_full, 2 * kTileBytes);
-        ptx::tma_load_2d(smem + OFF_QA, &tmQ, &bar->q_full, h0 * kD, qy);
-        ptx::tma_load_2d(smem + OFF_QA + kHalfBytes, &tmQ, &bar->q_full, h0 * kD + 64, qy);
-        ptx::tma_load_2d(smem + OFF_QB, &tmQ, &bar->q_full, (h0 + 1) * kD, qy);
-        ptx::tma_load_2d(smem + OFF_QB + kHalfBytes, &tmQ, &bar->q_full, (h0 + 1) * kD + 64, qy);
+        const int32_t qy0 = w0.q_base + w0.tile * kRows, qy1 = w1.q_base + w1.tile * kRows;
+        ptx::mbar_expect_tx(&bar->q_full, (nkb1 > 0 ? 2 : 1) * kTileBytes);
+        ptx::tma_load_2d(smem + OFF_QA, &tmQ, &bar->q_full, h0 * kD, qy0);
+        ptx::tma_load_2d(smem + OFF_QA + kHalfBytes, &tmQ, &bar->q_full, h0 * kD + 64, qy0);
+        if (nkb1 > 0) {
+          ptx::tma_load_2d(smem + OFF_QB, &tmQ, &bar->q_full, h1 * kD, qy1);
+          ptx::tma_load_2d(smem + OFF_QB + kHalfBytes, &tmQ, &bar->q_full, h1 * kD + 64, qy1);
+        }
       }
       __syncwarp();
       uint32_t nk[2] = {0, 0}, nv[2] = {0, 0};
@@ -155,10 +180,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::mma_commit_warp(&bar->pv_done[x]);
       };
       bool ok = wait_warp(&bar->q_full, 0, a.status) && wait_warp(&bar->k_full[0], 0, a.status);
+      // unit x runs key blocks [0, nkb_x); the last unit reading block j
+      // releases its K / V stages (unit 1 whenever it has the block: nkb1 is
+      // either equal to nkb0, at least nkb0, or 0)
+      auto last_user = [&](int j) { return j < nkb1 ? 1 : 0; };
       if (ok) {
         ptx::tc_fence_after();
-        issue_s(0, 0);
-        issue_s(1, 0);
+        if (nkb0 > 0) issue_s(0, 0);
+        if (nkb1 > 0) issue_s(1, 0);
         ptx::mma_commit_warp(&bar->k_empty[0]);
       }
       // Per block: PV_A(j), S_A(j+1), PV_B(j), S_B(j+1).  S_x(j+1) overwrites
@@ -172,18 +201,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!wait_warp(&bar->v_full[s], (uint32_t)(j >> 1) & 1, a.status)) { ok = false; break; }
         if (more && !wait_warp(&bar->k_full[s1], (uint32_t)((j + 1) >> 1) & 1, a.status)) { ok = false; break; }
         for (int x = 0; x < 2; ++x) {
+          const int nkbx = x ? nkb1 : nkb0;
+          if (j >= nkbx) continue;
           if (!wait_warp(&bar->p_full[x], (uint32_t)j & 1, a.status)) { ok = false; break; }
           ptx::tc_fence_after();
           issue_pv(x, j);
-          if (x == 1) ptx::mma_commit_warp(&bar->v_empty[s]);
-          if (more) {
+          if (x == last_user(j)) ptx::mma_commit_warp(&bar->v_empty[s]);
+          if (j + 1 < nkbx) {
             if ((a.flags & kFlagDrainTmemReuse) && !wait_warp(&bar->pv_done[x], (uint32_t)j & 1, a.status)) {
               ok = false;
               break;
             }
             ptx::tc_fence_after();
             issue_s(x, j + 1);
-            if (x == 1) ptx::mma_commit_warp(&bar->k_empty[s1]);
+            if (x == last_user(j + 1)) ptx::mma_commit_warp(&bar->k_empty[s1]);
           }
         }
       }
@@ -197,16 +228,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ softmax of head x
     const int x = warp >> 2;
     const int r = threadIdx.x & 127;
-    const int h = h0 + x;
+    const int h = x ? h1 : h0;
+    const Tile wm = x ? w1 : w0;
+    const int nkbm = x ? nkb1 : nkb0, kfull = wm.a0;
     const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
     const uint32_t tS = tmem + lane_addr + (x ? 256u : 0u), tO = tmem + lane_addr + (x ? 384u : 128u);
-    const int row = w.tile * kRows + r;
-    const bool valid = row < w.q_len;
-    const int ke = a.kv_end[w.kv_base + (valid ? row : w.q_len - 1)];
+    const int row = wm.tile * kRows + r;
+    const bool valid = row < wm.q_len;
+    const int ke = a.kv_end[wm.kv_base + (valid ? row : wm.q_len - 1)];
     const float sl2 = a.scale * kLog2e;
     float m_use = -INFINITY, l = 0.f;
-    bool ok = nkb > 0;
-    for (int j = 0; ok && j < nkb; ++j) {
+    bool ok = nkbm > 0;
+    for (int j = 0; ok && j < nkbm; ++j) {
       if (!wait(&bar->s_full[x], (uint32_t)j & 1, a.status)) { ok = false; break; }
       ptx::tc_fence_after();
       float xs[128];
@@ -281,13 +314,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tc_fence_before();
       ptx::mbar_arrive(&bar->p_full[x]);
     }
-    if (ok) ok = wait(&bar->pv_done[x], (uint32_t)(nkb - 1) & 1, a.status);
+    if (ok) ok = wait(&bar->pv_done[x], (uint32_t)(nkbm - 1) & 1, a.status);
     if (!ok) {
-      set_abort(&bar->abort);
+      if (nkbm > 0) set_abort(&bar->abort);  // a unit without key blocks has nothing to write
     } else {
       ptx::tc_fence_after();
       const float inv = 1.f / l;
-      const int64_t orow = (int64_t)w.q_base + row;
+      const int64_t orow = (int64_t)wm.q_base + row;
       uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.out) + orow * a.hq * kD + h * kD);
 #pragma unroll 1
       for (int c = 0; c < 4; ++c) {
@@ -323,10 +356,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 cudaError_t launch_fwd_pair(const AttnArgs& a, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             cudaStream_t st) {
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(fwd_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
-      cudaSuccess)
+  const bool tile_pairs = a.pair_order != nullptr;
+  auto kern = tile_pairs ? fwd_pair_kernel<true> : fwd_pair_kernel<false>;
+  if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) != cudaSuccess)
     return e;
-  fwd_pair_kernel<<<(unsigned)(a.nq * (a.hq / 2)), kThreads, kSmemBytes, st>>>(tq, tk, tv, a);
+  const int64_t grid = tile_pairs ? a.npairs * a.hq : a.nq * (a.hq / 2);
+  if (grid == 0) return cudaSuccess;
+  kern<<<(unsigned)grid, kThreads, kSmemBytes, st>>>(tq, tk, tv, a);
   return cudaGetLastError();
 }
 

@@ -484,7 +484,8 @@ cudaError_t launch_fwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) {
   if ((e = make_tmap_bf16(&tk, a.k, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;
   if ((e = make_tmap_bf16(&tv, a.v, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;
   const char* single = getenv("ISM_FWD_ONE_HEAD");
-  if ((a.hq / a.hkv) % 2 == 0 && !(single && single[0] == '1')) return launch_fwd_pair(a, tq, tk, tv, st);
+  if (((a.hq / a.hkv) % 2 == 0 || a.pair_order) && !(single && single[0] == '1'))
+    return launch_fwd_pair(a, tq, tk, tv, st);
   if ((e = cudaFuncSetAttribute(fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
       cudaSuccess)
     return e;

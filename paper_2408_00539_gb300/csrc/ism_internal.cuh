@@ -68,7 +68,7 @@ cudaError_t launch_tiles(const SegsDev& s, int bm, int bn, const int32_t* kv_end
                          Tile* qtiles, Tile* ktiles, uint8_t* tile_class, int32_t* kt_full_end,
                          int32_t* kt_end, int32_t* qt_begin, cudaStream_t st);
 cudaError_t launch_order(const Tile* qtiles, int64_t nq, const Tile* ktiles, int64_t nk, int max_cost,
-                         int32_t* q_order, int32_t* k_order, cudaStream_t st);
+                         int32_t* q_order, int32_t* k_order, cudaStream_t st, int32_t* pair_order = nullptr);
 cudaError_t launch_pair_offsets(const Tile* ktiles, int64_t nk, int32_t* kpair_off, cudaStream_t st);
 cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t cap, int bm, int bn,
                                int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
@@ -97,6 +97,11 @@ struct AttnArgs {
   void* ds;
   const int32_t* kpair_off;
   int64_t ds_slots;
+  // Query-tile pairs for the paired forward when the query heads of a KV head
+  // are odd in number: pair_order lists the even-indexed q-tiles (each with
+  // the next q-tile of its sequence, when there is one) in cost order.
+  const int32_t* pair_order;
+  int64_t npairs;
   // Bit 0: before an MMA that overwrites tensor memory an earlier MMA reads
   // as its A operand, wait for that earlier MMA to complete.  Clear: rely on
   // MMAs issued by one thread executing in issue order.

@@ -128,21 +128,41 @@ __global__ void __launch_bounds__(256) tiles_kernel(SegsDev s, int bm, int bn, c
 }
 
 // Work lists ordered by decreasing cost (counting sort, one block).  Cost of
-// a q-tile = its non-empty k-tiles; of a k-tile = its non-empty q-tiles.
+// a q-tile = its non-empty k-tiles; of a k-tile = its non-empty q-tiles.  The
+// optional third list holds the q-tiles with an even index in their sequence
+// (the first of each pair of neighbouring q-tiles), costed by the pair's
+// larger count (the second tile's, kv_end being non-decreasing).
 // Items of equal cost come in arbitrary order; results do not depend on it.
+__device__ __forceinline__ bool pair_head(const Tile* qtiles, int64_t nq, int64_t i, int* cost) {
+  const Tile w = qtiles[i];
+  if (w.tile & 1) return false;
+  int c = w.a1;
+  if (i + 1 < nq) {
+    const Tile n = qtiles[i + 1];
+    if (n.q_base == w.q_base && n.tile == w.tile + 1) c = max(c, n.a1);
+  }
+  *cost = c;
+  return true;
+}
+
 __global__ void order_kernel(const Tile* __restrict__ qtiles, int64_t nq, const Tile* __restrict__ ktiles,
-                             int64_t nk, int max_cost, int32_t* q_order, int32_t* k_order) {
+                             int64_t nk, int max_cost, int32_t* q_order, int32_t* k_order, int32_t* pair_order) {
   extern __shared__ int32_t hist[];  // [max_cost + 1]
-  for (int pass = 0; pass < 2; ++pass) {
-    const Tile* items = pass == 0 ? qtiles : ktiles;
-    int64_t n = pass == 0 ? nq : nk;
-    int32_t* order = pass == 0 ? q_order : k_order;
+  for (int pass = 0; pass < 3; ++pass) {
+    const Tile* items = pass == 1 ? ktiles : qtiles;
+    int64_t n = pass == 1 ? nk : nq;
+    int32_t* order = pass == 0 ? q_order : pass == 1 ? k_order : pair_order;
     if (items == nullptr || order == nullptr || n == 0) continue;
     for (int i = threadIdx.x; i <= max_cost; i += blockDim.x) hist[i] = 0;
     __syncthreads();
     for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
-      Tile w = items[i];
-      int cost = pass == 0 ? w.a1 : w.a1 - w.a0;
+      int cost;
+      if (pass == 2) {
+        if (!pair_head(items, n, i, &cost)) continue;
+      } else {
+        const Tile w = items[i];
+        cost = pass == 0 ? w.a1 : w.a1 - w.a0;
+      }
       cost = min(max(cost, 0), max_cost);
       atomicAdd(&hist[cost], 1);
     }
@@ -153,8 +173,13 @@ __global__ void order_kernel(const Tile* __restrict__ qtiles, int64_t nq, const 
     }
     __syncthreads();
     for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
-      Tile w = items[i];
-      int cost = pass == 0 ? w.a1 : w.a1 - w.a0;
+      int cost;
+      if (pass == 2) {
+        if (!pair_head(items, n, i, &cost)) continue;
+      } else {
+        const Tile w = items[i];
+        cost = pass == 0 ? w.a1 : w.a1 - w.a0;
+      }
       cost = min(max(cost, 0), max_cost);
       order[atomicAdd(&hist[cost], 1)] = (int32_t)i;
     }
@@ -289,13 +314,13 @@ cudaError_t launch_tiles(const SegsDev& s, int bm, int bn, const int32_t* kv_end
 }
 
 cudaError_t launch_order(const Tile* qtiles, int64_t nq, const Tile* ktiles, int64_t nk, int max_cost,
-                         int32_t* q_order, int32_t* k_order, cudaStream_t st) {
+                         int32_t* q_order, int32_t* k_order, cudaStream_t st, int32_t* pair_order) {
   size_t smem = sizeof(int32_t) * (size_t)(max_cost + 1);
   if (smem > 48 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(order_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }
-  order_kernel<<<1, 1024, smem, st>>>(qtiles, nq, ktiles, nk, max_cost, q_order, k_order);
+  order_kernel<<<1, 1024, smem, st>>>(qtiles, nq, ktiles, nk, max_cost, q_order, k_order, pair_order);
   return cudaGetLastError();
 }
 
