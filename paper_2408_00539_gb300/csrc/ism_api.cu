@@ -269,16 +269,11 @@ ism_status_t build_pass_meta(const ism_segments_t* s, const Counts& c, const Pas
                              cudaStream_t st) {
   SegsDev d = dev_view(s);
   timer_begin(ISM_KERNEL_META, st);
-  ISM_TRY_CUDA(launch_kv_end(d, L.kv_end, st), "kv_end launch");
-  ISM_TRY_CUDA(launch_tiles(d, kTile, kTile, L.kv_end, c.nq, bwd ? c.nk : 0, L.qtiles, L.ktiles, nullptr, nullptr,
-                            nullptr, nullptr, st),
-               "tiles launch");
-  ISM_TRY_CUDA(launch_order(L.qtiles, c.nq, L.ktiles, bwd ? c.nk : 0, c.max_cost, L.q_order, L.k_order, st,
-                            L.pair_order),
-               "order launch");
-  if (L.kpair_off) ISM_TRY_CUDA(launch_pair_offsets(L.ktiles, c.nk, L.kpair_off, st), "pair offsets launch");
+  ISM_TRY_CUDA(launch_pass_meta(d, L.kv_end, kTile, kTile, c.nq, bwd ? c.nk : 0, L.qtiles, bwd ? L.ktiles : nullptr,
+                                c.max_cost, L.q_order, bwd ? L.k_order : nullptr, L.pair_order, L.kpair_off, st),
+               "metadata launch");
   timer_end(ISM_KERNEL_META, st);
-  count_launch((s->num_segs > 0 ? 3 : 2) + (L.kpair_off && c.nk ? 1 : 0));
+  count_launch(1);
   return ISM_OK;
 }
 

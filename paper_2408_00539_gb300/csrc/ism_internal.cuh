@@ -70,6 +70,10 @@ cudaError_t launch_tiles(const SegsDev& s, int bm, int bn, const int32_t* kv_end
 cudaError_t launch_order(const Tile* qtiles, int64_t nq, const Tile* ktiles, int64_t nk, int max_cost,
                          int32_t* q_order, int32_t* k_order, cudaStream_t st, int32_t* pair_order = nullptr);
 cudaError_t launch_pair_offsets(const Tile* ktiles, int64_t nk, int32_t* kpair_off, cudaStream_t st);
+// kv_end, tiles, work lists (and pair offsets when kpair_off is set) in one launch.
+cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, int64_t nq, int64_t nk,
+                             Tile* qtiles, Tile* ktiles, int max_cost, int32_t* q_order, int32_t* k_order,
+                             int32_t* pair_order, int32_t* kpair_off, cudaStream_t st);
 cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t cap, int bm, int bn,
                                int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
                                int32_t* q_order, cudaStream_t st);

@@ -19,10 +19,10 @@ __device__ __forceinline__ int upper_bound_i32(const int32_t* a, int n, int32_t 
 // Per-sequence tile offsets computed by every block into shared memory:
 // qoff/koff [B+1] (q-tiles / k-tiles before sequence b) and toff [B+1]
 // (tile_class bytes before sequence b).  Block-wide scans over chunks of
-// blockDim.x sequences with a running carry.
+// blockDim.x (at most 1024) sequences with a running carry.
 __device__ void seq_offsets_smem(const SegsDev& s, int bm, int bn, int32_t* qoff, int32_t* koff, int64_t* toff) {
-  __shared__ int32_t sq[256], sk[256];
-  __shared__ int64_t stl[256];
+  __shared__ int32_t sq[1024], sk[1024];
+  __shared__ int64_t stl[1024];
   __shared__ int32_t cq, ck;
   __shared__ int64_t ct;
   if (threadIdx.x == 0) { cq = 0; ck = 0; ct = 0; qoff[0] = 0; koff[0] = 0; toff[0] = 0; }
@@ -76,11 +76,10 @@ __global__ void kv_end_kernel(SegsDev s, int32_t* kv_end) {
 // inside the sequence (0 otherwise), and ceil(kv_end[last row] / bn)
 // non-empty tiles; k-tile c is first reached by the q-tile holding the first
 // row whose kv_end exceeds c*bn.
-// Block size must be 256 (the offset scan's shared arrays).
-__global__ void __launch_bounds__(256) tiles_kernel(SegsDev s, int bm, int bn, const int32_t* __restrict__ kv_end,
-                             int64_t nq, int64_t nk, Tile* qtiles, Tile* ktiles, uint8_t* tile_class,
-                             int32_t* kt_full_end, int32_t* kt_end, int32_t* qt_begin) {
-  extern __shared__ __align__(16) unsigned char dyn[];
+// `dyn` holds the per-sequence offsets ((num_seqs + 1) * 16 bytes).
+__device__ void tiles_body(const SegsDev& s, int bm, int bn, const int32_t* __restrict__ kv_end, int64_t nq,
+                           int64_t nk, Tile* qtiles, Tile* ktiles, uint8_t* tile_class, int32_t* kt_full_end,
+                           int32_t* kt_end, int32_t* qt_begin, unsigned char* dyn) {
   int64_t* toff = reinterpret_cast<int64_t*>(dyn);
   int32_t* qoff = reinterpret_cast<int32_t*>(toff + s.num_seqs + 1);
   int32_t* koff = qoff + s.num_seqs + 1;
@@ -115,7 +114,14 @@ __global__ void __launch_bounds__(256) tiles_kernel(SegsDev s, int bm, int bn, c
     int32_t c = (int32_t)g - koff[b];
     int32_t base = s.cu_seqlens[b];
     int32_t L = s.cu_seqlens[b + 1] - base;
-    int32_t j = upper_bound_i32(kv_end + base, L, c * bn);  // first row that sees key c*bn
+    // first row that sees key x = c*bn: kv_end is non-decreasing, and under
+    // Eq. fj the first segment ending after x starts that row when it is a
+    // query segment, else the row is max(segment start, x)
+    const int32_t x = c * bn;
+    const int s0 = s.cu_segs[b], s1 = s.cu_segs[b + 1];
+    const int seg = s0 + upper_bound_i32(s.seg_end + s0, s1 - s0, x);
+    const int32_t start = seg > s0 ? s.seg_end[seg - 1] : 0;
+    int32_t j = s.seg_type[seg] == ISM_SEG_QUERY ? start : (x > start ? x : start);
     int32_t qb = j / bm;
     if (qt_begin) qt_begin[g] = qb;
     if (ktiles) {
@@ -125,6 +131,13 @@ __global__ void __launch_bounds__(256) tiles_kernel(SegsDev s, int bm, int bn, c
       ktiles[g] = w;
     }
   }
+}
+
+__global__ void __launch_bounds__(256) tiles_kernel(SegsDev s, int bm, int bn, const int32_t* __restrict__ kv_end,
+                             int64_t nq, int64_t nk, Tile* qtiles, Tile* ktiles, uint8_t* tile_class,
+                             int32_t* kt_full_end, int32_t* kt_end, int32_t* qt_begin) {
+  extern __shared__ __align__(16) unsigned char dyn[];
+  tiles_body(s, bm, bn, kv_end, nq, nk, qtiles, ktiles, tile_class, kt_full_end, kt_end, qt_begin, dyn);
 }
 
 // Work lists ordered by decreasing cost (counting sort, one block).  Cost of
@@ -145,9 +158,8 @@ __device__ __forceinline__ bool pair_head(const Tile* qtiles, int64_t nq, int64_
   return true;
 }
 
-__global__ void order_kernel(const Tile* __restrict__ qtiles, int64_t nq, const Tile* __restrict__ ktiles,
-                             int64_t nk, int max_cost, int32_t* q_order, int32_t* k_order, int32_t* pair_order) {
-  extern __shared__ int32_t hist[];  // [max_cost + 1]
+__device__ void order_body(const Tile* __restrict__ qtiles, int64_t nq, const Tile* __restrict__ ktiles, int64_t nk,
+                           int max_cost, int32_t* q_order, int32_t* k_order, int32_t* pair_order, int32_t* hist) {
   for (int pass = 0; pass < 3; ++pass) {
     const Tile* items = pass == 1 ? ktiles : qtiles;
     int64_t n = pass == 1 ? nk : nq;
@@ -187,10 +199,16 @@ __global__ void order_kernel(const Tile* __restrict__ qtiles, int64_t nq, const 
   }
 }
 
+__global__ void order_kernel(const Tile* __restrict__ qtiles, int64_t nq, const Tile* __restrict__ ktiles,
+                             int64_t nk, int max_cost, int32_t* q_order, int32_t* k_order, int32_t* pair_order) {
+  extern __shared__ int32_t hist[];  // [max_cost + 1]
+  order_body(qtiles, nq, ktiles, nk, max_cost, q_order, k_order, pair_order, hist);
+}
+
 // Exclusive prefix over k-tiles of their non-empty q-tile counts (a1 - a0):
 // the first (k-tile, q-tile) pair slot of each k-tile.  One block, chunks of
 // blockDim.x with a running carry.
-__global__ void pair_offsets_kernel(const Tile* __restrict__ ktiles, int64_t nk, int32_t* kpair_off) {
+__device__ void pair_offsets_body(const Tile* __restrict__ ktiles, int64_t nk, int32_t* kpair_off) {
   __shared__ int32_t buf[1024];
   __shared__ int32_t carry;
   if (threadIdx.x == 0) carry = 0;
@@ -215,6 +233,36 @@ __global__ void pair_offsets_kernel(const Tile* __restrict__ ktiles, int64_t nk,
     if (threadIdx.x == blockDim.x - 1) carry += buf[threadIdx.x];
     __syncthreads();
   }
+}
+
+__global__ void pair_offsets_kernel(const Tile* __restrict__ ktiles, int64_t nk, int32_t* kpair_off) {
+  pair_offsets_body(ktiles, nk, kpair_off);
+}
+
+// All metadata of one attention pass in a single block: kv_end per token
+// (Eq. fj, a warp per segment), the q-/k-tile descriptors, the cost-ordered work lists and, for
+// the stored-dS backward, the pair offsets.  Global writes of one phase are
+// visible to the block's threads after __syncthreads.
+__global__ void __launch_bounds__(1024)
+    pass_meta_kernel(SegsDev s, int32_t* kv_end, int bm, int bn, int64_t nq, int64_t nk, Tile* qtiles,
+                     Tile* ktiles, int max_cost, int32_t* q_order, int32_t* k_order, int32_t* pair_order,
+                     int32_t* kpair_off) {
+  extern __shared__ __align__(16) unsigned char dyn[];
+  // kv_end: one warp per segment, lanes over its tokens
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
+  for (int seg = warp; seg < s.num_segs; seg += nwarps) {
+    const int b = upper_bound_i32(s.cu_segs, s.num_seqs + 1, seg) - 1;
+    const int32_t start = seg > s.cu_segs[b] ? s.seg_end[seg - 1] : 0;
+    const int32_t end = s.seg_end[seg];
+    const int32_t base = s.cu_seqlens[b];
+    const bool query = s.seg_type[seg] == ISM_SEG_QUERY;
+    for (int32_t j = start + lane; j < end; j += 32) kv_end[base + j] = query ? end : j + 1;
+  }
+  __syncthreads();
+  tiles_body(s, bm, bn, kv_end, nq, nk, qtiles, ktiles, nullptr, nullptr, nullptr, nullptr, dyn);
+  __syncthreads();
+  order_body(qtiles, nq, ktiles, nk, max_cost, q_order, k_order, pair_order, reinterpret_cast<int32_t*>(dyn));
+  if (kpair_off) pair_offsets_body(ktiles, nk, kpair_off);
 }
 
 __device__ __forceinline__ int32_t chunk_kv_end(const AppendSegs& sg, int32_t j) {
@@ -321,6 +369,21 @@ cudaError_t launch_order(const Tile* qtiles, int64_t nq, const Tile* ktiles, int
     if (e != cudaSuccess) return e;
   }
   order_kernel<<<1, 1024, smem, st>>>(qtiles, nq, ktiles, nk, max_cost, q_order, k_order, pair_order);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, int64_t nq, int64_t nk,
+                             Tile* qtiles, Tile* ktiles, int max_cost, int32_t* q_order, int32_t* k_order,
+                             int32_t* pair_order, int32_t* kpair_off, cudaStream_t st) {
+  size_t a = (size_t)(s.num_seqs + 1) * (sizeof(int64_t) + 2 * sizeof(int32_t));
+  size_t b = sizeof(int32_t) * (size_t)(max_cost + 1);
+  size_t smem = a > b ? a : b;
+  if (smem > 48 * 1024) {
+    cudaError_t e = cudaFuncSetAttribute(pass_meta_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  pass_meta_kernel<<<1, 1024, smem, st>>>(s, kv_end, bm, bn, nq, nk, qtiles, ktiles, max_cost, q_order, k_order,
+                                          pair_order, kpair_off);
   return cudaGetLastError();
 }
 
