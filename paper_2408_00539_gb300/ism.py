@@ -232,20 +232,29 @@ def bwd_workspace_size(segs: Segments, q, k, softmax_scale: float, minimal: bool
 def bwd(segs: Segments, q, k, v, o, lse, dout, softmax_scale: float, dq=None, dk=None, dv=None, workspace=None,
         minimal_workspace: bool = False):
     """Backward: (dq, dk, dv) of sum(O * dout).  The library takes the
-    stored-dS schedule when the workspace is large enough for it; with
-    minimal_workspace=True a fresh workspace gets only the minimum size (the
-    recompute schedule)."""
+    stored-dS schedule when the workspace is large enough for it, else the
+    recompute schedule.  A given workspace is used as it is (it must hold at
+    least the minimum); without one, a workspace of the stored-dS size is
+    allocated (the minimum with minimal_workspace=True, or when the larger
+    one does not fit in device memory)."""
     lib = load()
     _contig(q, k, v, o, lse, dout)
     s, sh = segs.struct(), _shape(q, k, softmax_scale)
-    nbytes = C.c_size_t()
-    fn = "ism_attn_bwd_workspace_size_min" if minimal_workspace else "ism_attn_bwd_workspace_size"
-    _check(getattr(lib, fn)(C.byref(s), C.byref(sh), C.byref(nbytes)), fn)
+    full, low = C.c_size_t(), C.c_size_t()
+    _check(lib.ism_attn_bwd_workspace_size(C.byref(s), C.byref(sh), C.byref(full)), "ism_attn_bwd_workspace_size")
+    _check(lib.ism_attn_bwd_workspace_size_min(C.byref(s), C.byref(sh), C.byref(low)),
+           "ism_attn_bwd_workspace_size_min")
     dq = torch.empty_like(q) if dq is None else dq
     dk = torch.empty_like(k) if dk is None else dk
     dv = torch.empty_like(v) if dv is None else dv
-    if workspace is None or workspace.numel() < nbytes.value:
-        workspace = _workspace(nbytes.value, q.device)
+    if workspace is None or workspace.numel() < low.value:
+        if minimal_workspace:
+            workspace = _workspace(low.value, q.device)
+        else:
+            try:
+                workspace = _workspace(full.value, q.device)
+            except torch.cuda.OutOfMemoryError:
+                workspace = _workspace(low.value, q.device)
     _check(lib.ism_attn_bwd(C.byref(s), C.byref(sh), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), _ptr(dout),
                             _ptr(dq), _ptr(dk), _ptr(dv), _ptr(workspace), workspace.numel(), _stream(q.device)),
            "ism_attn_bwd")
