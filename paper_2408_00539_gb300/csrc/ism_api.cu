@@ -202,8 +202,10 @@ struct PassLayout {
   int32_t* kpair_off;
   void* ds;
   int32_t* pair_order;
+  int32_t* counters;  // work counters of the persistent backward kernels (backward only)
   size_t bytes;
 };
+constexpr int kPassCounters = 2;
 
 PassLayout pass_layout(void* ws, const ism_segments_t* s, const Counts& c, int64_t T, int hq, bool bwd,
                        int64_t ds_slots = 0, bool tile_pairs = false) {
@@ -218,6 +220,7 @@ PassLayout pass_layout(void* ws, const ism_segments_t* s, const Counts& c, int64
   L.kpair_off = ds_slots > 0 ? cv.take<int32_t>(c.nk) : nullptr;
   L.ds = ds_slots > 0 ? static_cast<void*>(cv.take<uint16_t>(ds_slots * kTile * kTile)) : nullptr;
   L.pair_order = tile_pairs ? cv.take<int32_t>(c.npairs) : nullptr;
+  L.counters = bwd ? cv.take<int32_t>(kPassCounters) : nullptr;
   L.bytes = ((cv.off + 255) & ~size_t(255)) + 256;
   return L;
 }
@@ -270,7 +273,8 @@ ism_status_t build_pass_meta(const ism_segments_t* s, const Counts& c, const Pas
   SegsDev d = dev_view(s);
   timer_begin(ISM_KERNEL_META, st);
   ISM_TRY_CUDA(launch_pass_meta(d, L.kv_end, kTile, kTile, c.nq, bwd ? c.nk : 0, L.qtiles, bwd ? L.ktiles : nullptr,
-                                c.max_cost, L.q_order, bwd ? L.k_order : nullptr, L.pair_order, L.kpair_off, st),
+                                c.max_cost, L.q_order, bwd ? L.k_order : nullptr, L.pair_order, L.kpair_off,
+                                L.counters, L.counters ? kPassCounters : 0, st),
                "metadata launch");
   timer_end(ISM_KERNEL_META, st);
   count_launch(1);
@@ -463,6 +467,7 @@ ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order; a.nq = c.nq;
   a.ktiles = L.ktiles; a.k_order = L.k_order; a.nk = c.nk;
   a.ds = L.ds; a.kpair_off = L.kpair_off; a.ds_slots = L.ds ? slots : 0;
+  a.work_counter = L.counters;
   a.status = status;
   a.flags = tc_flags();
   if (use_tc_bwd(shape)) {

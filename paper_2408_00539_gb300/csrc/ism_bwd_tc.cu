@@ -371,21 +371,25 @@ constexpr uint32_t OFF_K = 0, OFF_V = kTileBytes, OFF_Q = 2 * kTileBytes, OFF_DO
 // per stage: lse2[128] f32, delta[128] f32, visible-key count[128] u8
 constexpr uint32_t kMetaStage = 128 * 4 + 128 * 4 + 128;
 constexpr uint32_t OFF_BAR = OFF_META + 2 * kMetaStage;
-constexpr uint32_t kSmemBytes = OFF_BAR + 256;  // needs a 1024-aligned dynamic shared base
+constexpr uint32_t kSmemBytes = OFF_BAR + 512;  // needs a 1024-aligned dynamic shared base
 constexpr uint32_t TM_S = 0, TM_DP = 128, TM_DV = 256, TM_DK = 384;
-// warps 0-7 compute, 8 TMA loads, 9 TMEM + MMA issue, 10 per-query metadata
+// warps 0-7 compute, 8 work items + TMA loads, 9 TMEM + MMA issue, 10 per-query metadata
 constexpr int kLoadWarp = 8, kMmaWarp = 9, kMetaWarp = 10;
 constexpr int kThreads = 352;
+constexpr int kItemSlots = 4;  // work items published ahead of the roles that follow them
 
 struct Bars {
-  uint64_t kv_full;
+  uint64_t kv_full, kv_empty;
   uint64_t q_full[kQStages], q_empty[kQStages], do_full[2], do_empty[2], meta_full[2], meta_empty[2];
-  uint64_t s_full, dp_full, pt_full, p_full, dv_done, dk_done, final_mma;
+  uint64_t item_full[kItemSlots];
+  uint64_t s_full, dp_full, pt_full, p_full, dv_done, dk_done, acc_full, final_mma;
   uint32_t tmem_base;
   int32_t abort;
   uint32_t full[2][2];  // per meta stage and warpgroup: all 64 queries see all 128 keys
+  int32_t items[kItemSlots];
 };
-static_assert(sizeof(Bars) <= 256, "barrier block");
+static_assert(sizeof(Bars) <= 512, "barrier block");
+static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 }  // namespace dkv
 
 __global__ void __launch_bounds__(dkv::kThreads, 1)
@@ -400,21 +404,12 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
     if (threadIdx.x == 0) atomicOr(a.status, kStatusSmemAlign);
     return;
   }
-  const int g = blockIdx.x % a.hkv;
-  const int gk = a.k_order[blockIdx.x / a.hkv];  // global k-tile index
-  const Tile w = a.ktiles[gk];
   const int group = a.hq / a.hkv;
-  const int qt0 = w.a0, nqt = w.a1;
-  const int per_head = nqt - qt0;
-  const int n_it = per_head > 0 ? per_head * group : 0;
-  // Iteration i visits query tile nqt - 1 - i / group of query head
-  // g * group + i % group: the key tiles of a sequence all start at its last
-  // query tile and move down together, so the CTAs running at the same time
-  // read the same Q / dO tiles and mostly hit L2.
-  const int c = w.tile;
+  const int64_t n_items = a.nk * a.hkv;
 
   if (threadIdx.x == 0) {
     ptx::mbar_init(&bar->kv_full, 1);
+    ptx::mbar_init(&bar->kv_empty, 1);
     for (int s = 0; s < kQStages; ++s) {
       ptx::mbar_init(&bar->q_full[s], 1);
       ptx::mbar_init(&bar->q_empty[s], 1);
@@ -425,12 +420,14 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
       ptx::mbar_init(&bar->meta_full[s], 32);
       ptx::mbar_init(&bar->meta_empty[s], kComputeThreads);
     }
+    for (int s = 0; s < kItemSlots; ++s) ptx::mbar_init(&bar->item_full[s], 1);
     ptx::mbar_init(&bar->s_full, 1);
     ptx::mbar_init(&bar->dp_full, 1);
     ptx::mbar_init(&bar->pt_full, kComputeThreads);
     ptx::mbar_init(&bar->p_full, kComputeThreads);
     ptx::mbar_init(&bar->dv_done, 1);
     ptx::mbar_init(&bar->dk_done, 1);
+    ptx::mbar_init(&bar->acc_full, 1);
     ptx::mbar_init(&bar->final_mma, 1);
     bar->abort = 0;
     ptx::fence_mbar_init();
@@ -444,28 +441,101 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
   ptx::tc_fence_after();
   const uint32_t tmem = bar->tmem_base;
 
+  // Work items (k-tile k_order[item / hkv], KV head item % hkv) come from a
+  // global counter, most expensive first; the load warp takes them and
+  // publishes each in a small shared ring that the other roles follow, so
+  // every role of the CTA walks the same items.  A negative entry ends the walk.
+  struct Item {
+    int g, gk, c, qt0, nqt, n_it;
+    Tile w;
+  };
+  auto decode = [&](int item, Item& x) {
+    x.g = item % a.hkv;
+    x.gk = a.k_order[item / a.hkv];
+    x.w = a.ktiles[x.gk];
+    x.c = x.w.tile;
+    x.qt0 = x.w.a0;
+    x.nqt = x.w.a1;
+    x.n_it = x.nqt > x.qt0 ? (x.nqt - x.qt0) * group : 0;
+  };
+  // the item of slot u, waited for by every role but the load warp (false: stop)
+  auto next_item = [&](uint32_t u, Item& x) -> bool {
+    const int slot = (int)(u % kItemSlots);
+    if (!wait(&bar->item_full[slot], (u / kItemSlots) & 1, a.status)) return false;
+    const int item = *reinterpret_cast<volatile int32_t*>(&bar->items[slot]);
+    if (item < 0) return false;
+    decode(item, x);
+    return true;
+  };
+  // Iteration i of an item visits query tile nqt - 1 - i / group of query head
+  // g * group + i % group: the key tiles of a sequence all start at its last
+  // query tile and move down together, so the CTAs running at the same time
+  // read the same Q / dO tiles and mostly hit L2.  Barrier phases count
+  // iterations (I) and items (u) across the whole walk.
+
   if (warp == kLoadWarp) {
-    // ------------------------------------------------ TMA loads (the warp waits converged,
-    // lane 0 issues the copies)
-    uint32_t nq[kQStages] = {0, 0, 0}, ndo[2] = {0, 0};
-    const int32_t ky = w.k_base + c * kRows;
-    if (n_it > 0) {
+    // ------------------------------------------------ work items and TMA loads (the warp waits
+    // converged, lane 0 issues)
+    uint32_t I = 0, nq[kQStages] = {0, 0, 0}, ndo[2] = {0, 0}, nkv = 0;
+    bool ok = true;
+    for (uint32_t u = 0;;) {
+      int item = -1;
       if (lane == 0) {
-        ptx::mbar_expect_tx(&bar->kv_full, 2 * kTileBytes);
-        ptx::tma_load_2d(smem + OFF_K, &tmK, &bar->kv_full, g * kD, ky);
-        ptx::tma_load_2d(smem + OFF_K + kHalfBytes, &tmK, &bar->kv_full, g * kD + 64, ky);
-        ptx::tma_load_2d(smem + OFF_V, &tmV, &bar->kv_full, g * kD, ky);
-        ptx::tma_load_2d(smem + OFF_V + kHalfBytes, &tmV, &bar->kv_full, g * kD + 64, ky);
+        item = ok && !aborted(&bar->abort) ? atomicAdd(a.work_counter, 1) : -1;
+        if (item >= n_items) item = -1;
+      }
+      item = __shfl_sync(0xffffffffu, item, 0);
+      Item x;
+      if (item >= 0) {
+        decode(item, x);
+        if (x.n_it == 0) {
+          // no query sees these keys (with ISM segments every key sees at least
+          // itself, so this is only a guard): dK = dV = 0, and the item is not published
+          for (int rr = lane; rr < kRows; rr += 32) {
+            const int key = x.c * kRows + rr;
+            if (key >= x.w.k_len) break;
+            const int64_t off = ((int64_t)x.w.k_base + key) * a.hkv * kD + x.g * kD;
+            uint4* dk = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.dk) + off);
+            uint4* dv = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.dv) + off);
+            for (int k = 0; k < kD / 8; ++k) dk[k] = dv[k] = make_uint4(0u, 0u, 0u, 0u);
+          }
+          continue;
+        }
+      }
+      // Every published item has iterations, so the load warp cannot run more
+      // than one item ahead of the MMA warp (kv_empty) and a ring slot is never
+      // rewritten before every role has read it.
+      if (lane == 0) {
+        const int slot = (int)(u % kItemSlots);
+        bar->items[slot] = item;
+        ptx::mbar_arrive(&bar->item_full[slot]);  // release: the entry is visible to the waiters
       }
       __syncwarp();
-      for (int i = 0; i < n_it; ++i) {
-        const int sq = i % kQStages, s = i & 1;
-        const uint32_t n = (uint32_t)(i >> 1);
-        const int h = g * group + i % group;
-        const int32_t qy = w.q_base + (nqt - 1 - i / group) * kRows;
-        if (__any_sync(0xffffffffu, aborted(&bar->abort))) break;
-        bool ok = i < kQStages || wait_warp(&bar->q_empty[sq], (uint32_t)(i / kQStages - 1) & 1, a.status);
-        if (ok) {
+      ++u;
+      if (item < 0) break;
+      // K and V of this item once the previous item's S and dP MMAs are done with them
+      if (nkv > 0 && !wait_warp(&bar->kv_empty, (nkv - 1) & 1, a.status)) {
+        if (lane == 0) set_abort(&bar->abort);
+        ok = false;
+        continue;
+      }
+      const int32_t ky = x.w.k_base + x.c * kRows;
+      if (lane == 0) {
+        ptx::mbar_expect_tx(&bar->kv_full, 2 * kTileBytes);
+        ptx::tma_load_2d(smem + OFF_K, &tmK, &bar->kv_full, x.g * kD, ky);
+        ptx::tma_load_2d(smem + OFF_K + kHalfBytes, &tmK, &bar->kv_full, x.g * kD + 64, ky);
+        ptx::tma_load_2d(smem + OFF_V, &tmV, &bar->kv_full, x.g * kD, ky);
+        ptx::tma_load_2d(smem + OFF_V + kHalfBytes, &tmV, &bar->kv_full, x.g * kD + 64, ky);
+      }
+      __syncwarp();
+      ++nkv;
+      for (int i = 0; i < x.n_it; ++i, ++I) {
+        const int sq = (int)(I % kQStages), s = (int)(I & 1);
+        const int h = x.g * group + i % group;
+        const int32_t qy = x.w.q_base + (x.nqt - 1 - i / group) * kRows;
+        if (__any_sync(0xffffffffu, aborted(&bar->abort))) { ok = false; break; }
+        bool okq = I < kQStages || wait_warp(&bar->q_empty[sq], (I / kQStages - 1) & 1, a.status);
+        if (okq) {
           if (lane == 0) {
             ptx::mbar_expect_tx(&bar->q_full[sq], kTileBytes);
             ptx::tma_load_2d(smem + OFF_Q + sq * kTileBytes, &tmQ, &bar->q_full[sq], h * kD, qy);
@@ -473,9 +543,9 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
           }
           __syncwarp();
           ++nq[sq];
-          ok = i < 2 || wait_warp(&bar->do_empty[s], (n - 1) & 1, a.status);
+          okq = I < 2 || wait_warp(&bar->do_empty[s], ((I >> 1) - 1) & 1, a.status);
         }
-        if (ok) {
+        if (okq) {
           if (lane == 0) {
             ptx::mbar_expect_tx(&bar->do_full[s], kTileBytes);
             ptx::tma_load_2d(smem + OFF_DO + s * kTileBytes, &tmdO, &bar->do_full[s], h * kD, qy);
@@ -484,97 +554,100 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
           __syncwarp();
           ++ndo[s];
         }
-        if (!ok) {
+        if (!okq) {
           if (lane == 0) set_abort(&bar->abort);
+          ok = false;
           break;
         }
       }
-      if (__any_sync(0xffffffffu, aborted(&bar->abort))) {
-        wait_warp(&bar->kv_full, 0, a.status);
-        for (int s = 0; s < kQStages; ++s)
-          if (nq[s]) wait_warp(&bar->q_full[s], (nq[s] - 1) & 1, a.status);
-        for (int s = 0; s < 2; ++s)
-          if (ndo[s]) wait_warp(&bar->do_full[s], (ndo[s] - 1) & 1, a.status);
-      }
+    }
+    if (!ok) {
+      // every issued copy lands before the CTA exits
+      if (nkv) wait_warp(&bar->kv_full, (nkv - 1) & 1, a.status);
+      for (int s = 0; s < kQStages; ++s)
+        if (nq[s]) wait_warp(&bar->q_full[s], (nq[s] - 1) & 1, a.status);
+      for (int s = 0; s < 2; ++s)
+        if (ndo[s]) wait_warp(&bar->do_full[s], (ndo[s] - 1) & 1, a.status);
     }
     __syncwarp();
   } else if (warp == kMetaWarp) {
     // ------------------------------------------------ per-query metadata (all 32 lanes)
-    for (int i = 0; i < n_it; ++i) {
-      const int s = i & 1;
-      const uint32_t n = (uint32_t)(i >> 1);
-      const int hh = i % group, t = nqt - 1 - i / group;
-      const int h = g * group + hh;
-      if (aborted(&bar->abort)) break;
-      if (i >= 2 && !wait(&bar->meta_empty[s], (n - 1) & 1, a.status)) { set_abort(&bar->abort); break; }
-      uint8_t* meta = smem + OFF_META + s * kMetaStage;
-      float* mlse = reinterpret_cast<float*>(meta);
-      float* mdel = mlse + 128;
-      uint8_t* mlim = reinterpret_cast<uint8_t*>(mdel + 128);
-      bool all_full = true;
+    uint32_t I = 0;
+    Item x;
+    for (uint32_t u = 0; next_item(u, x); ++u) {
+      for (int i = 0; i < x.n_it; ++i, ++I) {
+        const int s = (int)(I & 1);
+        const int hh = i % group, t = x.nqt - 1 - i / group;
+        const int h = x.g * group + hh;
+        if (aborted(&bar->abort)) break;
+        if (I >= 2 && !wait(&bar->meta_empty[s], ((I >> 1) - 1) & 1, a.status)) { set_abort(&bar->abort); break; }
+        uint8_t* meta = smem + OFF_META + s * kMetaStage;
+        float* mlse = reinterpret_cast<float*>(meta);
+        float* mdel = mlse + 128;
+        uint8_t* mlim = reinterpret_cast<uint8_t*>(mdel + 128);
+        bool all_full = true;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int j = lane * 4 + e;
-        const int row = t * kRows + j;
-        const bool valid = row < w.q_len;
-        const int64_t grow = (int64_t)w.q_base + row;
-        mlse[j] = valid ? a.lse_in[(int64_t)h * a.q_rows + grow] * kLog2e : 0.f;
-        mdel[j] = valid ? a.delta[(int64_t)h * a.q_rows + grow] : 0.f;
-        const int vis = valid ? a.kv_end[w.kv_base + row] - c * kRows : 0;
-        mlim[j] = (uint8_t)(vis < 0 ? 0 : vis > 128 ? 128 : vis);
-        all_full = all_full && vis >= 128;
+        for (int e = 0; e < 4; ++e) {
+          const int j = lane * 4 + e;
+          const int row = t * kRows + j;
+          const bool valid = row < x.w.q_len;
+          const int64_t grow = (int64_t)x.w.q_base + row;
+          mlse[j] = valid ? a.lse_in[(int64_t)h * a.q_rows + grow] * kLog2e : 0.f;
+          mdel[j] = valid ? a.delta[(int64_t)h * a.q_rows + grow] : 0.f;
+          const int vis = valid ? a.kv_end[x.w.kv_base + row] - x.c * kRows : 0;
+          mlim[j] = (uint8_t)(vis < 0 ? 0 : vis > 128 ? 128 : vis);
+          all_full = all_full && vis >= 128;
+        }
+        // lanes 0-15 hold the queries of warpgroup 0, lanes 16-31 those of warpgroup 1
+        const uint32_t fb = __ballot_sync(0xffffffffu, all_full);
+        if (lane == 0) {
+          bar->full[s][0] = (fb & 0xFFFFu) == 0xFFFFu;
+          bar->full[s][1] = (fb >> 16) == 0xFFFFu;
+        }
+        ptx::mbar_arrive(&bar->meta_full[s]);
       }
-      // lanes 0-15 hold the queries of warpgroup 0, lanes 16-31 those of warpgroup 1
-      const uint32_t fb = __ballot_sync(0xffffffffu, all_full);
-      if (lane == 0) {
-        bar->full[s][0] = (fb & 0xFFFFu) == 0xFFFFu;
-        bar->full[s][1] = (fb >> 16) == 0xFFFFu;
-      }
-      ptx::mbar_arrive(&bar->meta_full[s]);
+      if (aborted(&bar->abort)) break;
     }
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------ MMA issue (the whole warp runs the
     // loop, one elected lane issues each instruction)
-    if (n_it > 0) {
-      constexpr uint32_t idesc_nt = ptx::idesc_bf16_f32(128, 128, 0, 0);
-      constexpr uint32_t idesc_nn = ptx::idesc_bf16_f32(128, 128, 0, 1);
-      const uint32_t sK = ptx::smem_u32(smem + OFF_K), sV = ptx::smem_u32(smem + OFF_V);
-      auto issue_s = [&](int i) {
-        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + (i % kQStages) * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss_warp(tmem + TM_S, desc_kmajor(sK, kk), desc_kmajor(sQ, kk), idesc_nt, kk > 0 ? 1u : 0u);
-        ptx::mma_commit_warp(&bar->s_full);
-      };
-      auto issue_dp = [&](int i) {
-        const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + (i & 1) * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss_warp(tmem + TM_DP, desc_kmajor(sV, kk), desc_kmajor(sdO, kk), idesc_nt, kk > 0 ? 1u : 0u);
-        ptx::mma_commit_warp(&bar->dp_full);
-      };
-      // P^T (bf16, two queries per column) sits in the S^T columns and dS^T in the dP^T
-      // columns: warpgroup wg's queries [64 wg, 64 wg + 64) at column 64 wg + [0, 32)
-      auto issue_dv = [&](int i) {
-        const int s = i & 1;
-        const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + s * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ts_warp(tmem + TM_DV, tmem + TM_S + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sdO, kk),
-                                idesc_nn, (i > 0 || kk > 0) ? 1u : 0u);
-        ptx::mma_commit_warp(&bar->do_empty[s]);
-        ptx::mma_commit_warp(&bar->dv_done);
-      };
-      auto issue_dk = [&](int i) {
-        const int sq = i % kQStages;
-        const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + sq * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ts_warp(tmem + TM_DK, tmem + TM_DP + 8 * kk + (kk >= 4 ? 32 : 0), desc_mnmajor(sQ, kk),
-                                idesc_nn, (i > 0 || kk > 0) ? 1u : 0u);
-        ptx::mma_commit_warp(&bar->q_empty[sq]);
-        ptx::mma_commit_warp(&bar->dk_done);
-      };
+    constexpr uint32_t idesc_nt = ptx::idesc_bf16_f32(128, 128, 0, 0);
+    constexpr uint32_t idesc_nn = ptx::idesc_bf16_f32(128, 128, 0, 1);
+    const uint32_t sK = ptx::smem_u32(smem + OFF_K), sV = ptx::smem_u32(smem + OFF_V);
+    uint32_t I0 = 0, nkv = 0;  // iterations of earlier items; items with K / V loaded
+    bool ok = true;
+    auto issue_s = [&](uint32_t gi) {
+      const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + (gi % kQStages) * kTileBytes);
+      ptx::mma8_bf16_ss_kmajor_warp(tmem + TM_S, desc_kmajor(sK, 0), desc_kmajor(sQ, 0), idesc_nt, 0u);
+      ptx::mma_commit_warp(&bar->s_full);
+    };
+    auto issue_dp = [&](uint32_t gi) {
+      const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + (gi & 1) * kTileBytes);
+      ptx::mma8_bf16_ss_kmajor_warp(tmem + TM_DP, desc_kmajor(sV, 0), desc_kmajor(sdO, 0), idesc_nt, 0u);
+      ptx::mma_commit_warp(&bar->dp_full);
+    };
+    // P^T (bf16, two queries per column) sits in the S^T columns and dS^T in the dP^T
+    // columns: warpgroup wg's queries [64 wg, 64 wg + 64) at column 64 wg + [0, 32)
+    auto issue_dv = [&](uint32_t gi, bool first) {
+      const uint32_t s = gi & 1;
+      const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + s * kTileBytes);
+      ptx::mma8_bf16_ts_mnmajor_warp(tmem + TM_DV, tmem + TM_S, desc_mnmajor(sdO, 0), idesc_nn, first ? 0u : 1u);
+      ptx::mma_commit_warp(&bar->do_empty[s]);
+      ptx::mma_commit_warp(&bar->dv_done);
+    };
+    auto issue_dk = [&](uint32_t gi, bool first) {
+      const uint32_t sq = gi % kQStages;
+      const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + sq * kTileBytes);
+      ptx::mma8_bf16_ts_mnmajor_warp(tmem + TM_DK, tmem + TM_DP, desc_mnmajor(sQ, 0), idesc_nn, first ? 0u : 1u);
+      ptx::mma_commit_warp(&bar->q_empty[sq]);
+      ptx::mma_commit_warp(&bar->dk_done);
+    };
+    Item x;
+    for (uint32_t u = 0; ok; ++u) {
+      if (!__all_sync(0xffffffffu, next_item(u, x))) break;
+      const int n_it = x.n_it;
+      if (!wait_warp(&bar->kv_full, nkv & 1, a.status)) { ok = false; break; }
+      ++nkv;
       // Event-driven issue, in order of urgency (the tensor pipe runs MMAs in
       // issue order, so whatever is issued first runs first):
       //   dK_i  needs dS^T_i written (p_full)
@@ -584,34 +657,45 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
       //   dV_i  needs P^T_i written (pt_full) and dP_i issued (both read dO_i)
       //   S_i   needs Q_i and dV_{i-1} issued (it overwrites the P^T dV_{i-1}
       //         reads; in order, or with the flag, dV_{i-1} completed)
-      bool ok = wait_warp(&bar->kv_full, 0, a.status);
-      int ns = 0, np = 0, nv = 0, nk = 0;
+      // The first dV / dK of an item restart the accumulators, which the
+      // compute warps have read out (their epilogue of the previous item comes
+      // before the P^T / dS^T writes these MMAs wait for).
+      // counters of issued S, dP, dV, dK over the whole walk; this item ends at `end`
+      const uint32_t end = I0 + (uint32_t)n_it;
+      uint32_t ns = I0, np = I0, nv = I0, nk = I0;
+      uint32_t qs = I0 % kQStages, qph = (I0 / kQStages) & 1;  // Q stage and phase of S_ns
       uint64_t t_idle = 0;
-      while (ok && nk < n_it) {
+      while (ok && nk < end) {
         bool progressed = false;
-        if (nk < nv && ptx::mbar_test_warp(&bar->p_full, (uint32_t)nk & 1)) {
+        if (nk < nv && ptx::mbar_test_warp(&bar->p_full, nk & 1)) {
           ptx::tc_fence_after();
-          issue_dk(nk++);
+          issue_dk(nk, nk == I0);
+          ++nk;
           progressed = true;
         }
-        if (np < n_it && np <= nk && ptx::mbar_test_warp(&bar->do_full[np & 1], (uint32_t)(np >> 1) & 1) &&
-            (np == 0 || !(a.flags & kFlagDrainTmemReuse) ||
-             ptx::mbar_test_warp(&bar->dk_done, (uint32_t)(np - 1) & 1))) {
+        if (np < end && np <= nk && ptx::mbar_test_warp(&bar->do_full[np & 1], (np >> 1) & 1) &&
+            (np == 0 || !(a.flags & kFlagDrainTmemReuse) || ptx::mbar_test_warp(&bar->dk_done, (np - 1) & 1))) {
           ptx::tc_fence_after();
-          issue_dp(np++);
+          issue_dp(np);
+          ++np;
+          progressed = true;
+          // the last MMAs reading this item's K and V are issued: the next K / V may load
+          if (np == end && ns == end) ptx::mma_commit_warp(&bar->kv_empty);
+        }
+        if (nv < np && ptx::mbar_test_warp(&bar->pt_full, nv & 1)) {
+          ptx::tc_fence_after();
+          issue_dv(nv, nv == I0);
+          ++nv;
           progressed = true;
         }
-        if (nv < np && ptx::mbar_test_warp(&bar->pt_full, (uint32_t)nv & 1)) {
+        if (ns < end && ns <= nv && ptx::mbar_test_warp(&bar->q_full[qs], qph) &&
+            (ns == 0 || !(a.flags & kFlagDrainTmemReuse) || ptx::mbar_test_warp(&bar->dv_done, (ns - 1) & 1))) {
           ptx::tc_fence_after();
-          issue_dv(nv++);
+          issue_s(ns);
+          ++ns;
+          if (++qs == kQStages) { qs = 0; qph ^= 1; }
           progressed = true;
-        }
-        if (ns < n_it && ns <= nv && ptx::mbar_test_warp(&bar->q_full[ns % kQStages], (uint32_t)(ns / kQStages) & 1) &&
-            (ns == 0 || !(a.flags & kFlagDrainTmemReuse) ||
-             ptx::mbar_test_warp(&bar->dv_done, (uint32_t)(ns - 1) & 1))) {
-          ptx::tc_fence_after();
-          issue_s(ns++);
-          progressed = true;
+          if (np == end && ns == end) ptx::mma_commit_warp(&bar->kv_empty);
         }
         if (progressed) {
           t_idle = 0;
@@ -626,11 +710,14 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
           }
         }
       }
-      if (!ok && lane == 0) set_abort(&bar->abort);
-      __syncwarp();
-      ptx::mma_commit_warp(&bar->final_mma);
-      wait_warp(&bar->final_mma, 0, a.status);
+      if (!ok) break;
+      ptx::mma_commit_warp(&bar->acc_full);  // dV, dK of this item complete
+      I0 = end;
     }
+    if (!ok && lane == 0) set_abort(&bar->abort);
+    __syncwarp();
+    ptx::mma_commit_warp(&bar->final_mma);
+    wait_warp(&bar->final_mma, 0, a.status);
     __syncwarp();
   } else {
     // ------------------------------------------------ compute: thread = key row r, warpgroup wg owns queries [64 wg, 64 wg + 64)
@@ -639,146 +726,146 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
     const uint32_t tS = tmem + lane_addr + TM_S + 64u * wg, tP = tmem + lane_addr + TM_DP + 64u * wg;
     const float sl2 = a.scale * kLog2e;
     bool ok = true;
-    // dS^T stores of the previous iteration left for after this iteration's P
-    // phase (half of them), where the compute warps wait for dP^T anyway
-    uint4* ds_dst = nullptr;
-    uint32_t ds_rest[16];
-    for (int i = 0; ok && i < n_it; ++i) {
-      const int s = i & 1;
-      if (!wait(&bar->meta_full[s], (uint32_t)(i >> 1) & 1, a.status) || !wait(&bar->s_full, (uint32_t)i & 1, a.status)) {
-        ok = false;
-        break;
-      }
-      ptx::tc_fence_after();
-      const uint8_t* meta = smem + OFF_META + s * kMetaStage;
-      const float4* mlse4 = reinterpret_cast<const float4*>(meta) + wg * 16;
-      const float4* mdel4 = reinterpret_cast<const float4*>(meta + 512) + wg * 16;
-      const uint32_t* mlim4 = reinterpret_cast<const uint32_t*>(meta + 1024) + wg * 16;
-      // phase 1: P from S^T (dP^T may still be in flight)
-      uint32_t pp[32];  // pp[k]: queries 64 wg + 2k, 64 wg + 2k + 1 (bf16)
-      {
-        uint32_t sv[2][32];
-        ld64(tS, sv[0], sv[1]);
-        ptx::tmem_ld_wait();
-        ptx::reg_fence(sv[0]);
-        ptx::reg_fence(sv[1]);
-        if (bar->full[s][wg]) {
-          // every key of the tile is visible to every query of this warpgroup
-          const float2 sl2x2 = make_float2(sl2, sl2);
+    uint32_t I = 0, nacc = 0;
+    Item x;
+    for (uint32_t u = 0; ok && next_item(u, x); ++u) {
+      const int n_it = x.n_it;
+      // dS^T stores of the previous iteration left for after this iteration's P
+      // phase (half of them), where the compute warps wait for dP^T anyway
+      uint4* ds_dst = nullptr;
+      uint32_t ds_rest[16];
+      for (int i = 0; ok && i < n_it; ++i, ++I) {
+        const int s = (int)(I & 1);
+        if (!wait(&bar->meta_full[s], (I >> 1) & 1, a.status) || !wait(&bar->s_full, I & 1, a.status)) {
+          ok = false;
+          break;
+        }
+        ptx::tc_fence_after();
+        const uint8_t* meta = smem + OFF_META + s * kMetaStage;
+        const float4* mlse4 = reinterpret_cast<const float4*>(meta) + wg * 16;
+        const float4* mdel4 = reinterpret_cast<const float4*>(meta + 512) + wg * 16;
+        const uint32_t* mlim4 = reinterpret_cast<const uint32_t*>(meta + 1024) + wg * 16;
+        // phase 1: P from S^T (dP^T may still be in flight)
+        uint32_t pp[32];  // pp[k]: queries 64 wg + 2k, 64 wg + 2k + 1 (bf16)
+        {
+          uint32_t sv[2][32];
+          ld64(tS, sv[0], sv[1]);
+          ptx::tmem_ld_wait();
+          ptx::reg_fence(sv[0]);
+          ptx::reg_fence(sv[1]);
+          if (bar->full[s][wg]) {
+            // every key of the tile is visible to every query of this warpgroup
+            const float2 sl2x2 = make_float2(sl2, sl2);
 #pragma unroll
-          for (int q4 = 0; q4 < 16; ++q4) {
-            const float4 l4 = mlse4[q4];
-            const uint32_t* sq = &sv[q4 >> 3][(q4 & 7) * 4];
-            const float2 a01 = fma2(make_float2(__uint_as_float(sq[0]), __uint_as_float(sq[1])), sl2x2,
-                                    make_float2(-l4.x, -l4.y));
-            const float2 a23 = fma2(make_float2(__uint_as_float(sq[2]), __uint_as_float(sq[3])), sl2x2,
-                                    make_float2(-l4.z, -l4.w));
-            pp[q4 * 2] = pack_bf16(ex2(a01.x), ex2(a01.y));
-            pp[q4 * 2 + 1] = pack_bf16(ex2(a23.x), ex2(a23.y));
-          }
-        } else {
-#pragma unroll
-          for (int q4 = 0; q4 < 16; ++q4) {
-            const float4 l4 = mlse4[q4];
-            const uint32_t lim = mlim4[q4];
-            const float lv[4] = {l4.x, l4.y, l4.z, l4.w};
-            float p[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const int vis = (int)((lim >> (8 * e)) & 0xFFu);
-              p[e] = r < vis ? ex2(__uint_as_float(sv[q4 >> 3][(q4 & 7) * 4 + e]) * sl2 - lv[e]) : 0.f;
+            for (int q4 = 0; q4 < 16; ++q4) {
+              const float4 l4 = mlse4[q4];
+              const uint32_t* sq = &sv[q4 >> 3][(q4 & 7) * 4];
+              const float2 a01 = fma2(make_float2(__uint_as_float(sq[0]), __uint_as_float(sq[1])), sl2x2,
+                                      make_float2(-l4.x, -l4.y));
+              const float2 a23 = fma2(make_float2(__uint_as_float(sq[2]), __uint_as_float(sq[3])), sl2x2,
+                                      make_float2(-l4.z, -l4.w));
+              pp[q4 * 2] = pack_bf16(ex2(a01.x), ex2(a01.y));
+              pp[q4 * 2 + 1] = pack_bf16(ex2(a23.x), ex2(a23.y));
             }
-            pp[q4 * 2] = pack_bf16(p[0], p[1]);
-            pp[q4 * 2 + 1] = pack_bf16(p[2], p[3]);
+          } else {
+#pragma unroll
+            for (int q4 = 0; q4 < 16; ++q4) {
+              const float4 l4 = mlse4[q4];
+              const uint32_t lim = mlim4[q4];
+              const float lv[4] = {l4.x, l4.y, l4.z, l4.w};
+              float p[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int vis = (int)((lim >> (8 * e)) & 0xFFu);
+                p[e] = r < vis ? ex2(__uint_as_float(sv[q4 >> 3][(q4 & 7) * 4 + e]) * sl2 - lv[e]) : 0.f;
+              }
+              pp[q4 * 2] = pack_bf16(p[0], p[1]);
+              pp[q4 * 2 + 1] = pack_bf16(p[2], p[3]);
+            }
           }
         }
+        // P^T over this warpgroup's (already read) S^T columns; dV may start
+        ptx::tmem_st32(tS, pp);
+        ptx::tmem_st_wait();
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(&bar->pt_full);
+        if (ds_dst) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            ds_dst[(k + 4) * kRows] =
+                make_uint4(ds_rest[4 * k], ds_rest[4 * k + 1], ds_rest[4 * k + 2], ds_rest[4 * k + 3]);
+          ds_dst = nullptr;
+        }
+        // phase 2: dS from dP^T
+        if (!wait(&bar->dp_full, I & 1, a.status)) { ok = false; break; }
+        ptx::tc_fence_after();
+        uint32_t pd[32];
+        {
+          uint32_t dv[2][32];
+          ld64(tP, dv[0], dv[1]);
+          ptx::tmem_ld_wait();
+          ptx::reg_fence(dv[0]);
+          ptx::reg_fence(dv[1]);
+#pragma unroll
+          for (int q4 = 0; q4 < 16; ++q4) {
+            const float4 d4 = mdel4[q4];
+            const uint32_t w0 = pp[q4 * 2], w1 = pp[q4 * 2 + 1];
+            const int b = (q4 & 7) * 4, hv = q4 >> 3;
+            const float2 v01 = mul2(make_float2(__uint_as_float(w0 << 16), __uint_as_float(w0 & 0xFFFF0000u)),
+                                    add2(make_float2(__uint_as_float(dv[hv][b + 0]), __uint_as_float(dv[hv][b + 1])),
+                                         make_float2(-d4.x, -d4.y)));
+            const float2 v23 = mul2(make_float2(__uint_as_float(w1 << 16), __uint_as_float(w1 & 0xFFFF0000u)),
+                                    add2(make_float2(__uint_as_float(dv[hv][b + 2]), __uint_as_float(dv[hv][b + 3])),
+                                         make_float2(-d4.z, -d4.w)));
+            pd[q4 * 2] = pack_bf16(v01.x, v01.y);
+            pd[q4 * 2 + 1] = pack_bf16(v23.x, v23.y);
+          }
+        }
+        ptx::mbar_arrive(&bar->meta_empty[s]);
+        // dS^T over this warpgroup's (already read) dP^T columns
+        ptx::tmem_st32(tP, pd);
+        ptx::tmem_st_wait();
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(&bar->p_full);
+        if (a.ds) {
+          // keep dS^T row r, queries [64 wg, 64 wg + 64), for the dQ GEMM, in
+          // the 8-interleaved layout (16-byte unit (query group, key)): the 32
+          // lanes of a warp store 512 contiguous bytes per instruction.  Issued
+          // after the hand-off so that the dV/dK MMAs do not wait for it.
+          const int hh = i % group, t = x.nqt - 1 - i / group;
+          const int64_t slot = ((int64_t)a.kpair_off[x.gk] + (t - x.qt0)) * a.hq + (x.g * group + hh);
+          uint4* dst = reinterpret_cast<uint4*>(static_cast<uint8_t*>(a.ds) + slot * kTileBytes) + wg * 8 * kRows + r;
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            dst[k * kRows] = make_uint4(pd[4 * k], pd[4 * k + 1], pd[4 * k + 2], pd[4 * k + 3]);
+#pragma unroll
+          for (int k = 0; k < 16; ++k) ds_rest[k] = pd[16 + k];
+          ds_dst = dst;
+        }
       }
-      // P^T over this warpgroup's (already read) S^T columns; dV may start
-      ptx::tmem_st32(tS, pp);
-      ptx::tmem_st_wait();
-      ptx::tc_fence_before();
-      ptx::mbar_arrive(&bar->pt_full);
       if (ds_dst) {
 #pragma unroll
         for (int k = 0; k < 4; ++k)
           ds_dst[(k + 4) * kRows] = make_uint4(ds_rest[4 * k], ds_rest[4 * k + 1], ds_rest[4 * k + 2], ds_rest[4 * k + 3]);
-        ds_dst = nullptr;
       }
-      // phase 2: dS from dP^T
-      if (!wait(&bar->dp_full, (uint32_t)i & 1, a.status)) { ok = false; break; }
+      if (!ok) break;
+      // epilogue of the item: dV, dK from tensor memory
+      if (!wait(&bar->acc_full, nacc & 1, a.status)) { ok = false; break; }
+      ++nacc;
       ptx::tc_fence_after();
-      uint32_t pd[32];
-      {
-        uint32_t dv[2][32];
-        ld64(tP, dv[0], dv[1]);
-        ptx::tmem_ld_wait();
-        ptx::reg_fence(dv[0]);
-        ptx::reg_fence(dv[1]);
-#pragma unroll
-        for (int q4 = 0; q4 < 16; ++q4) {
-          const float4 d4 = mdel4[q4];
-          const uint32_t w0 = pp[q4 * 2], w1 = pp[q4 * 2 + 1];
-          const int b = (q4 & 7) * 4, hv = q4 >> 3;
-          const float2 v01 = mul2(make_float2(__uint_as_float(w0 << 16), __uint_as_float(w0 & 0xFFFF0000u)),
-                                  add2(make_float2(__uint_as_float(dv[hv][b + 0]), __uint_as_float(dv[hv][b + 1])),
-                                       make_float2(-d4.x, -d4.y)));
-          const float2 v23 = mul2(make_float2(__uint_as_float(w1 << 16), __uint_as_float(w1 & 0xFFFF0000u)),
-                                  add2(make_float2(__uint_as_float(dv[hv][b + 2]), __uint_as_float(dv[hv][b + 3])),
-                                       make_float2(-d4.z, -d4.w)));
-          pd[q4 * 2] = pack_bf16(v01.x, v01.y);
-          pd[q4 * 2 + 1] = pack_bf16(v23.x, v23.y);
-        }
-      }
-      ptx::mbar_arrive(&bar->meta_empty[s]);
-      // dS^T over this warpgroup's (already read) dP^T columns
-      ptx::tmem_st32(tP, pd);
-      ptx::tmem_st_wait();
-      ptx::tc_fence_before();
-      ptx::mbar_arrive(&bar->p_full);
-      if (a.ds) {
-        // keep dS^T row r, queries [64 wg, 64 wg + 64), for the dQ GEMM, in
-        // the 8-interleaved layout (16-byte unit (query group, key)): the 32
-        // lanes of a warp store 512 contiguous bytes per instruction.  Issued
-        // after the hand-off so that the dV/dK MMAs do not wait for it.
-        const int hh = i % group, t = nqt - 1 - i / group;
-        const int64_t slot = ((int64_t)a.kpair_off[gk] + (t - qt0)) * a.hq + (g * group + hh);
-        uint4* dst = reinterpret_cast<uint4*>(static_cast<uint8_t*>(a.ds) + slot * kTileBytes) + wg * 8 * kRows + r;
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-          dst[k * kRows] = make_uint4(pd[4 * k], pd[4 * k + 1], pd[4 * k + 2], pd[4 * k + 3]);
-#pragma unroll
-        for (int k = 0; k < 16; ++k) ds_rest[k] = pd[16 + k];
-        ds_dst = dst;
-      }
-    }
-    if (ds_dst) {
-#pragma unroll
-      for (int k = 0; k < 4; ++k)
-        ds_dst[(k + 4) * kRows] = make_uint4(ds_rest[4 * k], ds_rest[4 * k + 1], ds_rest[4 * k + 2], ds_rest[4 * k + 3]);
-    }
-    if (ok && n_it > 0) ok = wait(&bar->final_mma, 0, a.status);
-    if (!ok) {
-      set_abort(&bar->abort);
-    } else {
-      ptx::tc_fence_after();
-      const int key = c * kRows + r;
-      const bool kvalid = key < w.k_len;
-      const int64_t krow = (int64_t)w.k_base + key;
+      const int key = x.c * kRows + r;
+      const bool kvalid = key < x.w.k_len;
+      const int64_t krow = (int64_t)x.w.k_base + key;
       // warpgroup 0 writes dV, warpgroup 1 writes dK (scaled)
-      __nv_bfloat16* outp = reinterpret_cast<__nv_bfloat16*>(wg == 0 ? a.dv : a.dk) + krow * a.hkv * kD + g * kD;
+      __nv_bfloat16* outp = reinterpret_cast<__nv_bfloat16*>(wg == 0 ? a.dv : a.dk) + krow * a.hkv * kD + x.g * kD;
       const float f = wg == 0 ? 1.f : a.scale;
       const uint32_t col = wg == 0 ? TM_DV : TM_DK;
 #pragma unroll 1
       for (int q4 = 0; q4 < 4; ++q4) {
         uint32_t v[32];
-        if (n_it > 0) {
-          ptx::tmem_ld32(tmem + lane_addr + col + q4 * 32, v);
-          ptx::tmem_ld_wait();
-          ptx::reg_fence(v);
-        } else {
-#pragma unroll
-          for (int k = 0; k < 32; ++k) v[k] = 0u;
-        }
+        ptx::tmem_ld32(tmem + lane_addr + col + q4 * 32, v);
+        ptx::tmem_ld_wait();
+        ptx::reg_fence(v);
         if (kvalid) {
           uint4* dst = reinterpret_cast<uint4*>(outp + q4 * 32);
 #pragma unroll
@@ -792,7 +879,9 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
           }
         }
       }
+      ptx::tc_fence_before();
     }
+    if (!ok) set_abort(&bar->abort);
   }
   ptx::tc_fence_before();
   __syncthreads();
@@ -838,8 +927,17 @@ cudaError_t launch_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) {
     if ((e = cudaFuncSetAttribute(dkdv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)dkv::kSmemBytes)) != cudaSuccess)
       return e;
+    // persistent: one CTA per SM takes (k-tile, KV head) items from the work counter
+    int dev = 0, sms = 0;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+    int64_t grid = sms;
+    const char* ov = getenv("ISM_DKDV_GRID");  // persistent grid size (default: one CTA per SM)
+    if (ov && atoi(ov) > 0) grid = atoi(ov);
+    if (grid > a.nk * a.hkv) grid = a.nk * a.hkv;
+    if (!a.work_counter) return cudaErrorInvalidValue;
     timer_begin(ISM_KERNEL_BWD_DKDV, st);
-    dkdv_kernel<<<(unsigned)(a.nk * a.hkv), dkv::kThreads, dkv::kSmemBytes, st>>>(tq, tdo, tk, tv, a);
+    dkdv_kernel<<<(unsigned)grid, dkv::kThreads, dkv::kSmemBytes, st>>>(tq, tdo, tk, tv, a);
     timer_end(ISM_KERNEL_BWD_DKDV, st);
     count_launch();
     if ((e = cudaGetLastError()) != cudaSuccess) return e;

@@ -73,7 +73,8 @@ cudaError_t launch_pair_offsets(const Tile* ktiles, int64_t nk, int32_t* kpair_o
 // kv_end, tiles, work lists (and pair offsets when kpair_off is set) in one launch.
 cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, int64_t nq, int64_t nk,
                              Tile* qtiles, Tile* ktiles, int max_cost, int32_t* q_order, int32_t* k_order,
-                             int32_t* pair_order, int32_t* kpair_off, cudaStream_t st);
+                             int32_t* pair_order, int32_t* kpair_off, int32_t* counters, int n_counters,
+                             cudaStream_t st);
 cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t cap, int bm, int bn,
                                int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
                                int32_t* q_order, cudaStream_t st);
@@ -106,6 +107,8 @@ struct AttnArgs {
   // the next q-tile of its sequence, when there is one) in cost order.
   const int32_t* pair_order;
   int64_t npairs;
+  // Work counter of the persistent dK/dV kernel (zeroed by the metadata pass).
+  int32_t* work_counter;
   // Bit 0: before an MMA that overwrites tensor memory an earlier MMA reads
   // as its A operand, wait for that earlier MMA to complete.  Clear: rely on
   // MMAs issued by one thread executing in issue order.

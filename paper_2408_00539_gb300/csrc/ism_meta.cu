@@ -246,8 +246,9 @@ __global__ void pair_offsets_kernel(const Tile* __restrict__ ktiles, int64_t nk,
 __global__ void __launch_bounds__(1024)
     pass_meta_kernel(SegsDev s, int32_t* kv_end, int bm, int bn, int64_t nq, int64_t nk, Tile* qtiles,
                      Tile* ktiles, int max_cost, int32_t* q_order, int32_t* k_order, int32_t* pair_order,
-                     int32_t* kpair_off) {
+                     int32_t* kpair_off, int32_t* counters, int n_counters) {
   extern __shared__ __align__(16) unsigned char dyn[];
+  if ((int)threadIdx.x < n_counters) counters[threadIdx.x] = 0;  // work counters of the kernels that follow
   // kv_end: one warp per segment, lanes over its tokens
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
   for (int seg = warp; seg < s.num_segs; seg += nwarps) {
@@ -374,7 +375,8 @@ cudaError_t launch_order(const Tile* qtiles, int64_t nq, const Tile* ktiles, int
 
 cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, int64_t nq, int64_t nk,
                              Tile* qtiles, Tile* ktiles, int max_cost, int32_t* q_order, int32_t* k_order,
-                             int32_t* pair_order, int32_t* kpair_off, cudaStream_t st) {
+                             int32_t* pair_order, int32_t* kpair_off, int32_t* counters, int n_counters,
+                             cudaStream_t st) {
   size_t a = (size_t)(s.num_seqs + 1) * (sizeof(int64_t) + 2 * sizeof(int32_t));
   size_t b = sizeof(int32_t) * (size_t)(max_cost + 1);
   size_t smem = a > b ? a : b;
@@ -383,7 +385,7 @@ cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, 
     if (e != cudaSuccess) return e;
   }
   pass_meta_kernel<<<1, 1024, smem, st>>>(s, kv_end, bm, bn, nq, nk, qtiles, ktiles, max_cost, q_order, k_order,
-                                          pair_order, kpair_off);
+                                          pair_order, kpair_off, counters, n_counters);
   return cudaGetLastError();
 }
 

@@ -164,6 +164,62 @@ __device__ __forceinline__ void mma_bf16_ts_warp(uint32_t d_tmem, uint32_t a_tme
       "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// The eight k-steps (K = 128 in steps of 16) of one 128 x N contraction,
+// issued by one elected lane of a converged warp: the other lanes branch past
+// the block, so the whole sequence costs one election, and the descriptors of
+// k-step kk are formed inside the block as the first ones plus a fixed offset
+// (in descriptor units of 16 bytes; the address field is the low 14 bits and
+// every tile lies inside the 256 KB it spans, so the sum never carries out).
+//   ss_kmajor: A and B K-major, 128-byte swizzled, two 64-column halves
+//              16 KB apart: offset(kk) = (kk / 4) * 1024 + (kk % 4) * 2
+//   ts_mnmajor: A from tensor memory at column a + {0, 8, 16, 24, 64, 72, 80, 88}[kk]
+//              (bf16 pairs), B MN-major swizzled: offset(kk) = kk * 128
+// k-step 0 accumulates when acc != 0, the others always.
+__device__ __forceinline__ void mma8_bf16_ss_kmajor_warp(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                                         uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred e, p, t;\n .reg .b64 a1, a2, a3, a4, a5, a6, a7, b1, b2, b3, b4, b5, b6, b7;\n"
+      " elect.sync _|e, 0xffffffff;\n @!e bra MMA8_SS_DONE;\n"
+      " setp.ne.b32 p, %4, 0;\n setp.eq.u32 t, 0, 0;\n"
+      " add.s64 a1, %1, 2; add.s64 a2, %1, 4; add.s64 a3, %1, 6; add.s64 a4, %1, 1024;\n"
+      " add.s64 a5, %1, 1026; add.s64 a6, %1, 1028; add.s64 a7, %1, 1030;\n"
+      " add.s64 b1, %2, 2; add.s64 b2, %2, 4; add.s64 b3, %2, 6; add.s64 b4, %2, 1024;\n"
+      " add.s64 b5, %2, 1026; add.s64 b6, %2, 1028; add.s64 b7, %2, 1030;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], a1, b1, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], a2, b2, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], a3, b3, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], a4, b4, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], a5, b5, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], a6, b6, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], a7, b7, %3, t;\n"
+      " MMA8_SS_DONE:\n}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(acc)
+      : "memory");
+}
+__device__ __forceinline__ void mma8_bf16_ts_mnmajor_warp(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                                          uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred e, p, t;\n .reg .b32 a1, a2, a3, a4, a5, a6, a7;\n"
+      " .reg .b64 b1, b2, b3, b4, b5, b6, b7;\n"
+      " elect.sync _|e, 0xffffffff;\n @!e bra MMA8_TS_DONE;\n"
+      " setp.ne.b32 p, %4, 0;\n setp.eq.u32 t, 0, 0;\n"
+      " add.u32 a1, %1, 8; add.u32 a2, %1, 16; add.u32 a3, %1, 24; add.u32 a4, %1, 64;\n"
+      " add.u32 a5, %1, 72; add.u32 a6, %1, 80; add.u32 a7, %1, 88;\n"
+      " add.s64 b1, %2, 128; add.s64 b2, %2, 256; add.s64 b3, %2, 384; add.s64 b4, %2, 512;\n"
+      " add.s64 b5, %2, 640; add.s64 b6, %2, 768; add.s64 b7, %2, 896;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [a1], b1, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [a2], b2, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [a3], b3, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [a4], b4, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [a5], b5, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [a6], b6, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [a7], b7, %3, t;\n"
+      " MMA8_TS_DONE:\n}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(acc)
+      : "memory");
+}
 __device__ __forceinline__ void mma_commit_warp(uint64_t* bar) {
   asm volatile(
       "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
