@@ -259,7 +259,10 @@ uint64_t ism_kernel_launches(void);
  *   modes 0/1 stage the operands with plain stores, 2/3 with TMA, 4/5 put
  *   a in tensor memory (the A-from-TMEM form of the MMA)
  *   mode 6: a [128,128] is K x M and b is K x N (both MN-major), c = a^T * b
- *   mode 7: as mode 6, a staged in the 8-interleaved layout without swizzle. */
+ *   mode 7: as mode 6, a staged in the 8-interleaved layout without swizzle.
+ *   mode 8 + m: as mode m with the eight k-steps issued by one warp through
+ *   the batched form the attention kernels use (one election, descriptors
+ *   advanced by fixed offsets). */
 ism_status_t ism_debug_mma_tile(const void* a, const void* b, float* c, int32_t mode, ism_stream_t stream);
 
 const char* ism_status_string(ism_status_t status);

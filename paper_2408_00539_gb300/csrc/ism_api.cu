@@ -650,7 +650,7 @@ ism_status_t ism_check_status(ism_stream_t stream) {
 }
 
 ism_status_t ism_debug_mma_tile(const void* a, const void* b, float* c, int32_t mode, ism_stream_t stream) {
-  if (!a || !b || !c || mode < 0 || mode > 7) return fail(ISM_ERR_INVALID_ARG, "a, b, c non-NULL and mode 0..7");
+  if (!a || !b || !c || mode < 0 || mode > 15) return fail(ISM_ERR_INVALID_ARG, "a, b, c non-NULL and mode 0..15");
   if (!tc_available()) return fail(ISM_ERR_UNSUPPORTED, "tensor-core kernels need an sm_103 device");
   uint32_t* status;
   ism_status_t r = status_ptr(&status);

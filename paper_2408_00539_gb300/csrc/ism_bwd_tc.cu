@@ -187,18 +187,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t sQ = ptx::smem_u32(smem + OFF_Q), sdO = ptx::smem_u32(smem + OFF_DO);
       auto issue_s = [&](int c) {
         const uint32_t sK = ptx::smem_u32(smem + OFF_K + (c % kKStages) * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss_warp(tmem + TM_S + 128u * (c & 1), desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_nt,
-                           kk > 0 ? 1u : 0u);
+        ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128>(tmem + TM_S + 128u * (c & 1), desc_kmajor(sQ, 0),
+                                                                  desc_kmajor(sK, 0), idesc_nt, 0u);
         ptx::mma_commit_warp(&bar->s_full[c & 1]);
       };
       auto issue_dp = [&](int c) {
         const int sv = c & 1;
         const uint32_t sV = ptx::smem_u32(smem + OFF_V + sv * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss_warp(tmem + TM_DP, desc_kmajor(sdO, kk), desc_kmajor(sV, kk), idesc_nt, kk > 0 ? 1u : 0u);
+        ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128>(tmem + TM_DP, desc_kmajor(sdO, 0), desc_kmajor(sV, 0),
+                                                                  idesc_nt, 0u);
         ptx::mma_commit_warp(&bar->dp_full);
         ptx::mma_commit_warp(&bar->v_empty[sv]);
       };
@@ -207,10 +204,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t sK = ptx::smem_u32(smem + OFF_K + (c % kKStages) * kTileBytes);
         // dQ += dS K_c: dS (bf16, keys packed two per column) in S region R, keys [0,64) at
         // columns [0,32) and [64,128) at columns [64,96)
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ts_warp(tmem + TM_DQ, tmem + TM_S + 128u * R + 8 * kk + (kk >= 4 ? 32 : 0),
-                           desc_mnmajor(sK, kk), idesc_nn, (c > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma8_bf16_ts_warp<ptx::TmemPairsGap32, ptx::MnMajorSw128>(tmem + TM_DQ, tmem + TM_S + 128u * R,
+                                                                      desc_mnmajor(sK, 0), idesc_nn, c > 0 ? 1u : 0u);
         ptx::mma_commit_warp(&bar->dq_done[R]);
         ptx::mma_commit_warp(&bar->k_empty[c % kKStages]);
       };
@@ -618,12 +613,12 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
     bool ok = true;
     auto issue_s = [&](uint32_t gi) {
       const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + (gi % kQStages) * kTileBytes);
-      ptx::mma8_bf16_ss_kmajor_warp(tmem + TM_S, desc_kmajor(sK, 0), desc_kmajor(sQ, 0), idesc_nt, 0u);
+      ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128>(tmem + TM_S, desc_kmajor(sK, 0), desc_kmajor(sQ, 0), idesc_nt, 0u);
       ptx::mma_commit_warp(&bar->s_full);
     };
     auto issue_dp = [&](uint32_t gi) {
       const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + (gi & 1) * kTileBytes);
-      ptx::mma8_bf16_ss_kmajor_warp(tmem + TM_DP, desc_kmajor(sV, 0), desc_kmajor(sdO, 0), idesc_nt, 0u);
+      ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128>(tmem + TM_DP, desc_kmajor(sV, 0), desc_kmajor(sdO, 0), idesc_nt, 0u);
       ptx::mma_commit_warp(&bar->dp_full);
     };
     // P^T (bf16, two queries per column) sits in the S^T columns and dS^T in the dP^T
@@ -631,14 +626,14 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
     auto issue_dv = [&](uint32_t gi, bool first) {
       const uint32_t s = gi & 1;
       const uint32_t sdO = ptx::smem_u32(smem + OFF_DO + s * kTileBytes);
-      ptx::mma8_bf16_ts_mnmajor_warp(tmem + TM_DV, tmem + TM_S, desc_mnmajor(sdO, 0), idesc_nn, first ? 0u : 1u);
+      ptx::mma8_bf16_ts_warp<ptx::TmemPairsGap32, ptx::MnMajorSw128>(tmem + TM_DV, tmem + TM_S, desc_mnmajor(sdO, 0), idesc_nn, first ? 0u : 1u);
       ptx::mma_commit_warp(&bar->do_empty[s]);
       ptx::mma_commit_warp(&bar->dv_done);
     };
     auto issue_dk = [&](uint32_t gi, bool first) {
       const uint32_t sq = gi % kQStages;
       const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + sq * kTileBytes);
-      ptx::mma8_bf16_ts_mnmajor_warp(tmem + TM_DK, tmem + TM_DP, desc_mnmajor(sQ, 0), idesc_nn, first ? 0u : 1u);
+      ptx::mma8_bf16_ts_warp<ptx::TmemPairsGap32, ptx::MnMajorSw128>(tmem + TM_DK, tmem + TM_DP, desc_mnmajor(sQ, 0), idesc_nn, first ? 0u : 1u);
       ptx::mma_commit_warp(&bar->q_empty[sq]);
       ptx::mma_commit_warp(&bar->dk_done);
     };

@@ -139,10 +139,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         ptx::tc_fence_after();
         const uint32_t sDS = ptx::smem_u32(smem + s * kStageBytes), sK = sDS + kTileBytes;
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss_warp(acc, desc_ilv_mnmajor(sDS, kk), desc_mnmajor(sK, kk), idesc,
-                                (c > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma8_bf16_ss_warp<ptx::MnMajorIlv8, ptx::MnMajorSw128>(acc, desc_ilv_mnmajor(sDS, 0), desc_mnmajor(sK, 0),
+                                                                   idesc, c > 0 ? 1u : 0u);
         ptx::mma_commit_warp(&bar->empty[s]);
       }
       if (!ok) break;

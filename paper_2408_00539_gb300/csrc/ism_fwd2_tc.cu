@@ -166,17 +166,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       auto issue_s = [&](int x, int j) {
         const uint32_t sK = ptx::smem_u32(smem + OFF_K + (j & 1) * kTileBytes);
         const uint32_t sQ = sQ0 + (uint32_t)x * kTileBytes, tS = tmem + 256u * (uint32_t)x;
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss_warp(tS, desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_qk, kk > 0 ? 1u : 0u);
+        ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128>(tS, desc_kmajor(sQ, 0), desc_kmajor(sK, 0), idesc_qk,
+                                                                  0u);
         ptx::mma_commit_warp(&bar->s_full[x]);
       };
       auto issue_pv = [&](int x, int j) {
         const uint32_t sV = ptx::smem_u32(smem + OFF_V + (j & 1) * kTileBytes);
         const uint32_t tS = tmem + 256u * (uint32_t)x, tO = tS + 128u;
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ts_warp(tO, tS + 8 * kk, desc_mnmajor(sV, kk), idesc_pv, (j > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma8_bf16_ts_warp<ptx::TmemPairs, ptx::MnMajorSw128>(tO, tS, desc_mnmajor(sV, 0), idesc_pv, j > 0 ? 1u : 0u);
         ptx::mma_commit_warp(&bar->pv_done[x]);
       };
       bool ok = wait_warp(&bar->q_full, 0, a.status) && wait_warp(&bar->k_full[0], 0, a.status);

@@ -161,10 +161,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tc_fence_after();
         const uint32_t sP = ptx::smem_u32(smem + OFF_P + s * kTileBytes);
         const uint32_t sV = ptx::smem_u32(smem + OFF_V + s * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss_warp(tmem + TM_O, desc_kmajor(sP, kk), desc_mnmajor(sV, kk), idesc_pv,
-                           (i > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::MnMajorSw128>(tmem + TM_O, desc_kmajor(sP, 0), desc_mnmajor(sV, 0),
+                                                                   idesc_pv, i > 0 ? 1u : 0u);
         ptx::mma_commit_warp(&bar->p_free[s]);
         ptx::mma_commit_warp(&bar->v_empty[s]);
         return true;
@@ -177,10 +175,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (j >= 2 && !wait_warp(&bar->s_free[s], (n - 1) & 1, a.status)) { ok = false; break; }
         ptx::tc_fence_after();
         const uint32_t sK = ptx::smem_u32(smem + OFF_K + s * kTileBytes);
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          ptx::mma_bf16_ss_warp(tmem + TM_S + s * 128, desc_kmajor(sQ, kk), desc_kmajor(sK, kk), idesc_qk,
-                           kk > 0 ? 1u : 0u);
+        ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128>(tmem + TM_S + s * 128, desc_kmajor(sQ, 0),
+                                                                  desc_kmajor(sK, 0), idesc_qk, 0u);
         ptx::mma_commit_warp(&bar->s_full[s]);
         ptx::mma_commit_warp(&bar->k_empty[s]);
         if (j >= 1 && !issue_pv(j - 1)) { ok = false; break; }
@@ -334,7 +330,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 // swizzled layout (modes 0/1), by TMA (modes 2/3), or A in tensor memory and
 // B by plain stores (modes 4/5); mode 6: A given as [K, M] (MN-major) and B
 // as [K, N], C = A^T B; mode 7: as mode 6 with A in the 8-interleaved
-// MN-major layout without swizzle.
+// MN-major layout without swizzle.  Bit 3 of the mode: the same with the eight
+// k-steps issued by warp 0 through the batched (one election) form.
 __global__ void __launch_bounds__(128, 1)
     mma_tile_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __nv_bfloat16* A, const __nv_bfloat16* B, float* C, int mode, uint32_t* status) {
@@ -345,6 +342,8 @@ __global__ void __launch_bounds__(128, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 2 * kTileBytes);
   uint32_t* tslot = reinterpret_cast<uint32_t*>(bars + 2);
   const int warp = threadIdx.x >> 5;
+  const bool batched = (mode & 8) != 0;
+  mode &= 7;
   const bool a_mn = mode == 6 || mode == 7;
   const bool a_ilv = mode == 7;
   const bool b_mn = (mode & 1) != 0 || mode == 6;
@@ -388,18 +387,40 @@ __global__ void __launch_bounds__(128, 1)
     ptx::tc_fence_after();
   }
   bool ok = true;
-  if (threadIdx.x == 0) {
+  if (batched ? warp == 0 : threadIdx.x == 0) {
     if (mode == 2 || mode == 3) {
-      ptx::mbar_expect_tx(&bars[0], 2 * kTileBytes);
-      ptx::tma_load_2d(sa, &tmA, &bars[0], 0, 0);
-      ptx::tma_load_2d(sa + kHalfBytes, &tmA, &bars[0], 64, 0);
-      ptx::tma_load_2d(sb, &tmB, &bars[0], 0, 0);
-      ptx::tma_load_2d(sb + kHalfBytes, &tmB, &bars[0], 64, 0);
+      if (threadIdx.x == 0) {
+        ptx::mbar_expect_tx(&bars[0], 2 * kTileBytes);
+        ptx::tma_load_2d(sa, &tmA, &bars[0], 0, 0);
+        ptx::tma_load_2d(sa + kHalfBytes, &tmA, &bars[0], 64, 0);
+        ptx::tma_load_2d(sb, &tmB, &bars[0], 0, 0);
+        ptx::tma_load_2d(sb + kHalfBytes, &tmB, &bars[0], 64, 0);
+      }
       ok = wait(&bars[0], 0, status);
     }
-    if (ok) {
-      const uint32_t idesc = ptx::idesc_bf16_f32(128, 128, a_mn ? 1u : 0u, b_mn ? 1u : 0u);
-      const uint32_t saa = ptx::smem_u32(sa), sbb = ptx::smem_u32(sb);
+    const uint32_t idesc = ptx::idesc_bf16_f32(128, 128, a_mn ? 1u : 0u, b_mn ? 1u : 0u);
+    const uint32_t saa = ptx::smem_u32(sa), sbb = ptx::smem_u32(sb);
+    if (batched) {
+      // the whole warp, converged; one elected lane issues and commits
+      ok = __all_sync(0xffffffffu, ok);
+      if (ok) {
+        using namespace ptx;
+        const uint64_t bd = b_mn ? desc_mnmajor(sbb, 0) : desc_kmajor(sbb, 0);
+        if (a_tmem && b_mn)
+          mma8_bf16_ts_warp<TmemPairs, MnMajorSw128>(tmem, tmem + 128, bd, idesc, 0u);
+        else if (a_tmem)
+          mma8_bf16_ts_warp<TmemPairs, KMajorSw128>(tmem, tmem + 128, bd, idesc, 0u);
+        else if (a_ilv)
+          mma8_bf16_ss_warp<MnMajorIlv8, MnMajorSw128>(tmem, desc_ilv_mnmajor(saa, 0), bd, idesc, 0u);
+        else if (a_mn)
+          mma8_bf16_ss_warp<MnMajorSw128, MnMajorSw128>(tmem, desc_mnmajor(saa, 0), bd, idesc, 0u);
+        else if (b_mn)
+          mma8_bf16_ss_warp<KMajorSw128, MnMajorSw128>(tmem, desc_kmajor(saa, 0), bd, idesc, 0u);
+        else
+          mma8_bf16_ss_warp<KMajorSw128, KMajorSw128>(tmem, desc_kmajor(saa, 0), bd, idesc, 0u);
+      }
+      ptx::mma_commit_warp(&bars[1]);
+    } else if (ok) {
       for (int kk = 0; kk < 8; ++kk) {
         const uint64_t bd = b_mn ? desc_mnmajor(sbb, kk) : desc_kmajor(sbb, kk);
         if (a_tmem)
@@ -410,7 +431,7 @@ __global__ void __launch_bounds__(128, 1)
                            bd, idesc, kk > 0 ? 1u : 0u);
       }
     }
-    ptx::mma_commit(&bars[1]);
+    if (!batched) ptx::mma_commit(&bars[1]);
     ok = wait(&bars[1], 0, status) && ok;
   }
   __syncthreads();
@@ -498,7 +519,7 @@ cudaError_t launch_mma_tile(const void* A, const void* B, float* C, int mode, ui
   memset(&ta, 0, sizeof(ta));
   memset(&tb, 0, sizeof(tb));
   cudaError_t e;
-  if (mode == 2 || mode == 3) {
+  if ((mode & 7) == 2 || (mode & 7) == 3) {
     if ((e = make_tmap_bf16(&ta, A, 128, 128)) != cudaSuccess) return e;
     if ((e = make_tmap_bf16(&tb, B, 128, 128)) != cudaSuccess) return e;
   }

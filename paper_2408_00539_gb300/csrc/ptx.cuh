@@ -166,25 +166,35 @@ __device__ __forceinline__ void mma_bf16_ts_warp(uint32_t d_tmem, uint32_t a_tme
 }
 // The eight k-steps (K = 128 in steps of 16) of one 128 x N contraction,
 // issued by one elected lane of a converged warp: the other lanes branch past
-// the block, so the whole sequence costs one election, and the descriptors of
+// the block, so the whole sequence costs one election, and the operands of
 // k-step kk are formed inside the block as the first ones plus a fixed offset
-// (in descriptor units of 16 bytes; the address field is the low 14 bits and
-// every tile lies inside the 256 KB it spans, so the sum never carries out).
-//   ss_kmajor: A and B K-major, 128-byte swizzled, two 64-column halves
-//              16 KB apart: offset(kk) = (kk / 4) * 1024 + (kk % 4) * 2
-//   ts_mnmajor: A from tensor memory at column a + {0, 8, 16, 24, 64, 72, 80, 88}[kk]
-//              (bf16 pairs), B MN-major swizzled: offset(kk) = kk * 128
+//   offset(kk) = (kk % 4) * kStep + (kk / 4) * kHalf
+// (descriptors in units of 16 bytes: the address field is the low 14 bits and
+// every tile lies inside the 256 KB it spans, so the sum never carries out;
+// tensor-memory A operands in columns).  Layouts used:
+//   KMajorSw128    K-major, 128-byte swizzled, two 64-column halves 16 KB apart
+//   MnMajorSw128   MN-major, 128-byte swizzled, 2 KB a k-step
+//   MnMajorIlv8    8-interleaved MN-major, 256 bytes a k-step
+//   TmemPairs      bf16 pairs in tensor memory, 8 columns a k-step
+//   TmemPairsGap32 the same with a 32-column gap after k-step 3
 // k-step 0 accumulates when acc != 0, the others always.
-__device__ __forceinline__ void mma8_bf16_ss_kmajor_warp(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                                         uint32_t idesc, uint32_t acc) {
+struct KMajorSw128 { static constexpr uint32_t step = 2, half = 1024; };
+struct MnMajorSw128 { static constexpr uint32_t step = 128, half = 512; };
+struct MnMajorIlv8 { static constexpr uint32_t step = 16, half = 64; };
+struct TmemPairs { static constexpr uint32_t step = 8, half = 32; };
+struct TmemPairsGap32 { static constexpr uint32_t step = 8, half = 64; };
+template <class LA, class LB, uint32_t kAStep = LA::step, uint32_t kAHalf = LA::half, uint32_t kBStep = LB::step,
+          uint32_t kBHalf = LB::half>
+__device__ __forceinline__ void mma8_bf16_ss_warp(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                                  uint32_t acc) {
   asm volatile(
       "{\n .reg .pred e, p, t;\n .reg .b64 a1, a2, a3, a4, a5, a6, a7, b1, b2, b3, b4, b5, b6, b7;\n"
       " elect.sync _|e, 0xffffffff;\n @!e bra MMA8_SS_DONE;\n"
       " setp.ne.b32 p, %4, 0;\n setp.eq.u32 t, 0, 0;\n"
-      " add.s64 a1, %1, 2; add.s64 a2, %1, 4; add.s64 a3, %1, 6; add.s64 a4, %1, 1024;\n"
-      " add.s64 a5, %1, 1026; add.s64 a6, %1, 1028; add.s64 a7, %1, 1030;\n"
-      " add.s64 b1, %2, 2; add.s64 b2, %2, 4; add.s64 b3, %2, 6; add.s64 b4, %2, 1024;\n"
-      " add.s64 b5, %2, 1026; add.s64 b6, %2, 1028; add.s64 b7, %2, 1030;\n"
+      " add.s64 a1, %1, %5; add.s64 a2, %1, %6; add.s64 a3, %1, %7; add.s64 a4, %1, %8;\n"
+      " add.s64 a5, %1, %9; add.s64 a6, %1, %10; add.s64 a7, %1, %11;\n"
+      " add.s64 b1, %2, %12; add.s64 b2, %2, %13; add.s64 b3, %2, %14; add.s64 b4, %2, %15;\n"
+      " add.s64 b5, %2, %16; add.s64 b6, %2, %17; add.s64 b7, %2, %18;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], a1, b1, %3, t;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], a2, b2, %3, t;\n"
@@ -194,20 +204,24 @@ __device__ __forceinline__ void mma8_bf16_ss_kmajor_warp(uint32_t d_tmem, uint64
       " tcgen05.mma.cta_group::1.kind::f16 [%0], a6, b6, %3, t;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], a7, b7, %3, t;\n"
       " MMA8_SS_DONE:\n}" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(acc)
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(acc), "n"(kAStep), "n"(2 * kAStep), "n"(3 * kAStep), "n"(kAHalf),
+      "n"(kAHalf + kAStep), "n"(kAHalf + 2 * kAStep), "n"(kAHalf + 3 * kAStep), "n"(kBStep), "n"(2 * kBStep),
+      "n"(3 * kBStep), "n"(kBHalf), "n"(kBHalf + kBStep), "n"(kBHalf + 2 * kBStep), "n"(kBHalf + 3 * kBStep)
       : "memory");
 }
-__device__ __forceinline__ void mma8_bf16_ts_mnmajor_warp(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
-                                                          uint32_t idesc, uint32_t acc) {
+template <class LA, class LB, uint32_t kAStep = LA::step, uint32_t kAHalf = LA::half, uint32_t kBStep = LB::step,
+          uint32_t kBHalf = LB::half>
+__device__ __forceinline__ void mma8_bf16_ts_warp(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                                  uint32_t acc) {
   asm volatile(
       "{\n .reg .pred e, p, t;\n .reg .b32 a1, a2, a3, a4, a5, a6, a7;\n"
       " .reg .b64 b1, b2, b3, b4, b5, b6, b7;\n"
       " elect.sync _|e, 0xffffffff;\n @!e bra MMA8_TS_DONE;\n"
       " setp.ne.b32 p, %4, 0;\n setp.eq.u32 t, 0, 0;\n"
-      " add.u32 a1, %1, 8; add.u32 a2, %1, 16; add.u32 a3, %1, 24; add.u32 a4, %1, 64;\n"
-      " add.u32 a5, %1, 72; add.u32 a6, %1, 80; add.u32 a7, %1, 88;\n"
-      " add.s64 b1, %2, 128; add.s64 b2, %2, 256; add.s64 b3, %2, 384; add.s64 b4, %2, 512;\n"
-      " add.s64 b5, %2, 640; add.s64 b6, %2, 768; add.s64 b7, %2, 896;\n"
+      " add.u32 a1, %1, %5; add.u32 a2, %1, %6; add.u32 a3, %1, %7; add.u32 a4, %1, %8;\n"
+      " add.u32 a5, %1, %9; add.u32 a6, %1, %10; add.u32 a7, %1, %11;\n"
+      " add.s64 b1, %2, %12; add.s64 b2, %2, %13; add.s64 b3, %2, %14; add.s64 b4, %2, %15;\n"
+      " add.s64 b5, %2, %16; add.s64 b6, %2, %17; add.s64 b7, %2, %18;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], [a1], b1, %3, t;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], [a2], b2, %3, t;\n"
@@ -217,7 +231,9 @@ __device__ __forceinline__ void mma8_bf16_ts_mnmajor_warp(uint32_t d_tmem, uint3
       " tcgen05.mma.cta_group::1.kind::f16 [%0], [a6], b6, %3, t;\n"
       " tcgen05.mma.cta_group::1.kind::f16 [%0], [a7], b7, %3, t;\n"
       " MMA8_TS_DONE:\n}" ::"r"(d_tmem),
-      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(acc)
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(acc), "n"(kAStep), "n"(2 * kAStep), "n"(3 * kAStep), "n"(kAHalf),
+      "n"(kAHalf + kAStep), "n"(kAHalf + 2 * kAStep), "n"(kAHalf + 3 * kAStep), "n"(kBStep), "n"(2 * kBStep),
+      "n"(3 * kBStep), "n"(kBHalf), "n"(kBHalf + kBStep), "n"(kBHalf + 2 * kBStep), "n"(kBHalf + 3 * kBStep)
       : "memory");
 }
 __device__ __forceinline__ void mma_commit_warp(uint64_t* bar) {

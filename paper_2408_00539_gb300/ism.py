@@ -323,8 +323,10 @@ def kernel_launches() -> int:
 
 
 def debug_mma_tile(a: torch.Tensor, b: torch.Tensor, mode: int) -> torch.Tensor:
-    """One 128x128x128 tcgen05 tile product (diagnostic): mode 0/2 a @ b.T,
-    mode 1/3 a @ b; modes 2/3 stage operands with TMA."""
+    """One 128x128x128 tcgen05 tile product (diagnostic): mode 0/2/4 a @ b.T,
+    mode 1/3/5 a @ b, mode 6/7 a.T @ b; modes 2/3 stage operands with TMA,
+    4/5 put a in tensor memory, 7 stages a 8-interleaved; mode + 8 issues the
+    k-steps through the batched one-election form."""
     c = torch.empty((128, 128), dtype=torch.float32, device=a.device)
     _check(load().ism_debug_mma_tile(_ptr(a), _ptr(b), _ptr(c), mode, _stream(a.device)), "ism_debug_mma_tile")
     return c

@@ -18,14 +18,16 @@ def ism():
     return m
 
 
-@pytest.mark.parametrize("mode", [0, 1, 2, 3, 4, 5, 6, 7])
+@pytest.mark.parametrize("mode", list(range(16)))
 def test_mma_tile(ism, mode):
-    g = torch.Generator().manual_seed(100 + mode)
+    """Each operand layout, with the k-steps issued one by one (modes 0-7) and
+    through the batched eight-step form (modes 8-15)."""
+    g = torch.Generator().manual_seed(100 + mode % 8)
     a = torch.randn(128, 128, generator=g).to(torch.bfloat16)
     b = torch.randn(128, 128, generator=g).to(torch.bfloat16)
     c = ism.debug_mma_tile(a.cuda(), b.cuda(), mode)
     ism.check_status()
-    if mode in (6, 7):
+    if mode % 8 in (6, 7):
         ref = a.double().T @ b.double()
     else:
         ref = a.double() @ (b.double().T if mode % 2 == 0 else b.double())
