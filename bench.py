@@ -469,6 +469,7 @@ def run_cuda(args, w):
     }
     if not args.no_append:
         line["append"] = measure_append(dev, read_peaks()[0])
+        line["session"] = measure_session(dev)
     if world == 1 and not args.no_cpu_baseline:
         val, dt, sample = oracle_sample(w, q, k, v, do, heads_per_sample=4)
         line["cpu_baseline"] = {"value": val, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
@@ -544,6 +545,76 @@ def measure_append(dev, peaks):
             "note": "decode bytes = K and V cache read once: 2*B*(c+1)*Hkv*D*2 per step; GB/s over the "
                     "split-KV + merge kernels (decode_kernel_us); decode_us_per_call adds the plan and "
                     "cache-write kernels and host launch overhead"}
+
+
+def measure_session(dev):
+    """A serving session in the shape of the paper's latency experiment
+    (Section 3.6): per turn, the query is appended in one prefill call (the
+    attention share of time to first token) and the answer generated by
+    single-token decode calls (time per output token), the KV cache growing
+    to the whole dialogue.  Each call is timed alone with CUDA events and a
+    synchronise after it, as a generation loop must wait for its token.  The
+    query turns run twice: under ISM (bidirectional query segment) and as a
+    causal chunk, the comparison the paper makes between the ISM and the
+    causal fine-tuned models."""
+    import torch
+    from paper_2408_00539_gb300 import ism
+    s = wl.latency_session()
+    B, hq, hkv, d, cap = s.batch, s.num_heads_q, s.num_heads_kv, s.head_dim, s.capacity
+    g = torch.Generator(device=dev).manual_seed(s.seed)
+
+    def rnd(*shape):
+        return torch.randn(shape, generator=g, device=dev).mul_(s.value_std).bfloat16()
+
+    kc, vc = rnd(B, cap, hkv, d), rnd(B, cap, hkv, d)
+    qn, kn, vn = rnd(B, s.q_len, hq, d), rnd(B, s.q_len, hkv, d), rnd(B, s.q_len, hkv, d)
+    qd, kd, vd = rnd(B, 1, hq, d), rnd(B, 1, hkv, d), rnd(B, 1, hkv, d)
+    ws = torch.empty(max(ism.append_workspace_size(qn, kn, s.softmax_scale),
+                         ism.append_workspace_size(qd, kd, s.softmax_scale)), dtype=torch.uint8, device=dev)
+    o_pre, o_dec = torch.empty_like(qn), torch.empty_like(qd)
+    l_pre = torch.empty((hq, B, s.q_len), dtype=torch.float32, device=dev)
+    l_dec = torch.empty((hq, B, 1), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def timed(fn):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        fn()
+        e1.record(stream)
+        e1.synchronize()
+        return e0.elapsed_time(e1)
+
+    result = {}
+    for mode, qtype in (("ism", wl.QUERY), ("causal", wl.ANSWER)):
+        cl = torch.zeros((B,), dtype=torch.int32, device=dev)
+        c_host = np.zeros((B,), dtype=np.int32)
+        ttft, tpot = [], []
+        for t in range(s.turns):
+            ttft.append(timed(lambda: ism.prefill_append(qn, kn, vn, kc, vc, cl, c_host, [s.q_len], [qtype],
+                                                         s.softmax_scale, out=o_pre, lse=l_pre, workspace=ws)))
+            c_host = c_host + s.q_len
+            if mode == "ism":
+                turn = []
+                for _ in range(s.a_len):
+                    turn.append(timed(lambda: ism.prefill_append(qd, kd, vd, kc, vc, cl, c_host, [1], [wl.ANSWER],
+                                                                 s.softmax_scale, out=o_dec, lse=l_dec, workspace=ws)))
+                    c_host = c_host + 1
+                tpot.append(float(np.mean(turn)) * 1e3)
+            else:  # the answer tokens' K / V are already in the cache from the first pass
+                c_host = c_host + s.a_len
+                cl.fill_(int(c_host[0]))
+        ism.check_status(dev)
+        result[mode] = (ttft, tpot)
+    ttft_i, tpot = result["ism"]
+    ttft_c, _ = result["causal"]
+    return {"workload": s.name, "heads": f"{hq}/{hkv}", "head_dim": d,
+            "context_tokens": s.capacity,
+            "ttft_ms_ism": float(np.mean(ttft_i)), "ttft_ms_causal": float(np.mean(ttft_c)),
+            "ttft_ism_over_causal": float(np.mean(ttft_i) / np.mean(ttft_c)),
+            "ttft_ms_first_last_turn": [float(ttft_i[0]), float(ttft_i[-1])],
+            "tpot_us": float(np.mean(tpot)), "tpot_us_first_last_turn": [tpot[0], tpot[-1]],
+            "note": "one attention layer per call (append plan, cache write, attention); the first turn's "
+                    "calls include warm-up"}
 
 
 WORKLOADS = {"gqa_8k": wl.gqa_8k, "mha_4k": wl.mha_4k, "packed_32k": wl.packed_32k,

@@ -261,6 +261,17 @@ def bwd(segs: Segments, q, k, v, o, lse, dout, softmax_scale: float, dq=None, dk
     return dq, dk, dv
 
 
+def append_workspace_size(q_new, k_new, softmax_scale: float) -> int:
+    """Workspace bytes ``prefill_append`` needs for this batch and chunk length."""
+    lib = load()
+    B, Ln = q_new.shape[0], q_new.shape[1]
+    sh = _shape(q_new, k_new, softmax_scale)
+    nbytes = C.c_size_t()
+    _check(lib.ism_attn_prefill_append_workspace_size(C.byref(sh), B, Ln, C.byref(nbytes)),
+           "ism_attn_prefill_append_workspace_size")
+    return nbytes.value
+
+
 def prefill_append(q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_host, new_seg_end, new_seg_type,
                    softmax_scale: float, out=None, lse=None, workspace=None):
     """Append a new turn to the KV caches and attend (Section 2.3).

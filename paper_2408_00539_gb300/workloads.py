@@ -207,6 +207,48 @@ def append_16k(seed: int = 5, batch: int = 8, cache_len: int = 16384, l_new: int
                           decode_steps, 32, 8, 128, 1.0 / np.sqrt(128.0), 0.5, seed)
 
 
+@dataclass
+class SessionWorkload:
+    """A serving session: every dialogue of the batch alternates a query turn,
+    appended in one prefill call, and an answer generated one token at a time
+    (decode calls), against a KV cache that keeps the whole dialogue."""
+    name: str
+    batch: int
+    turns: int
+    q_len: int
+    a_len: int
+    num_heads_q: int
+    num_heads_kv: int
+    head_dim: int
+    softmax_scale: float
+    value_std: float
+    seed: int
+
+    @property
+    def capacity(self) -> int:
+        return self.turns * (self.q_len + self.a_len)
+
+    def dialogue(self):
+        """(seg_end, seg_type) of one whole dialogue."""
+        ends, types, pos = [], [], 0
+        for _ in range(self.turns):
+            pos += self.q_len
+            ends.append(pos)
+            types.append(QUERY)
+            pos += self.a_len
+            ends.append(pos)
+            types.append(ANSWER)
+        return ends, types
+
+
+def latency_session(seed: int = 6, batch: int = 40, turns: int = 20, q_len: int = 40, a_len: int = 160) -> SessionWorkload:
+    """The shape of the paper's latency experiment (Section 3.6): 40 dialogues of
+    20 turns, 40 query and 160 answer tokens a turn (context up to 4000 tokens),
+    here for one attention layer of 32 query / 8 KV heads, head_dim 128, bf16."""
+    return SessionWorkload(f"session_b{batch}_t{turns}_q{q_len}_a{a_len}", batch, turns, q_len, a_len, 32, 8, 128,
+                           1.0 / np.sqrt(128.0), 0.5, seed)
+
+
 def normal(rng: np.random.Generator, shape, std: float) -> np.ndarray:
     return (rng.standard_normal(size=shape, dtype=np.float32) * np.float32(std)).astype(np.float32)
 

@@ -26,3 +26,11 @@ def test_tile_pair_count_matches_tile_map():
     for segs in (wl.random_dialogue_set(rng, 30, 700), wl.gqa_8k().segs, wl.tiny_fp32().segs):
         ref = int(orc.tile_map_packed(segs, 128, 128)["kt_end"].sum())
         assert bench.n_tile_pairs(segs) == ref
+
+
+def test_session_workload_shape():
+    s = wl.latency_session()
+    ends, types = s.dialogue()
+    assert s.capacity == 4000 and ends[-1] == s.capacity and len(ends) == 2 * s.turns
+    assert types == [wl.QUERY, wl.ANSWER] * s.turns
+    assert all(b - a in (s.q_len, s.a_len) for a, b in zip([0] + ends[:-1], ends))

@@ -406,3 +406,43 @@ def test_bwd_schedules_agree(ism):
     assert diff.max().item() <= 2e-2 * max(scale, 1.0), diff.max().item()
     assert diff.mean().item() <= 1e-3, diff.mean().item()
 
+
+
+def test_session_turn_by_turn_matches_one_pass(ism):
+    """A dialogue served turn by turn (each query appended in one call, each
+    answer token decoded alone against the growing cache) gives the rows of
+    one ISM pass over the whole dialogue (Section 2.3: the KV cache of earlier
+    turns is reused unchanged)."""
+    s = wl.SessionWorkload("session_test", 2, 3, 24, 6, 8, 2, 128, 128 ** -0.5, 0.5, 41)
+    B, T, hq, hkv, d = s.batch, s.capacity, s.num_heads_q, s.num_heads_kv, s.head_dim
+    rng = np.random.Generator(np.random.PCG64(s.seed))
+    q = wl.round_to(wl.normal(rng, (B, T, hq, d), s.value_std), "bf16")
+    k = wl.round_to(wl.normal(rng, (B, T, hkv, d), s.value_std), "bf16")
+    v = wl.round_to(wl.normal(rng, (B, T, hkv, d), s.value_std), "bf16")
+    kc = torch.zeros((B, T, hkv, d), dtype=torch.bfloat16, device=DEV)
+    vc = torch.zeros_like(kc)
+    cl = torch.zeros((B,), dtype=torch.int32, device=DEV)
+    c_host = np.zeros((B,), dtype=np.int32)
+    o = torch.full((B, T, hq, d), float("nan"), dtype=torch.bfloat16, device=DEV)
+    pos = 0
+    for _ in range(s.turns):
+        sl = slice(pos, pos + s.q_len)
+        o[:, sl], _ = ism.prefill_append(q[:, sl].contiguous().to(DEV), k[:, sl].contiguous().to(DEV),
+                                         v[:, sl].contiguous().to(DEV), kc, vc, cl, c_host, [s.q_len], [wl.QUERY],
+                                         s.softmax_scale)
+        pos += s.q_len
+        c_host = c_host + s.q_len
+        for _ in range(s.a_len):
+            sl = slice(pos, pos + 1)
+            o[:, sl], _ = ism.prefill_append(q[:, sl].contiguous().to(DEV), k[:, sl].contiguous().to(DEV),
+                                             v[:, sl].contiguous().to(DEV), kc, vc, cl, c_host, [1], [wl.ANSWER],
+                                             s.softmax_scale)
+            pos += 1
+            c_host = c_host + 1
+    ism.check_status()
+    assert cl.cpu().numpy().tolist() == [T] * B
+    assert torch.equal(kc.cpu(), k) and torch.equal(vc.cpu(), v)
+    segs = wl.pack([s.dialogue()])
+    for b in range(B):
+        o_ref, _ = orc.attn_fwd(q[b], k[b], v[b], segs, s.softmax_scale)
+        _cmp(f"session dialogue {b}", o[b], o_ref, "bf16")
