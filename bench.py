@@ -536,15 +536,68 @@ def measure_append(dev, peaks):
     us = float(np.median(dec_us[3:]))
     kus = float(np.median(dec_kernel_us[3:]))
     gbs = float(np.median(np.array(dec_bytes[3:]) / (np.array(dec_kernel_us[3:]) * 1e-6) / 1e9))
+    paged = measure_append_paged(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush)
     return {"workload": a.name,
             "prefill_ms": pre, "prefill_tflops": 4 * d * n_vis_pre / (pre * 1e-3) / 1e12,
             "prefill_frac_of_bf16_peak": 4 * d * n_vis_pre / (pre * 1e-3) / 1e12 / peaks["bf16_tflops"],
             "decode_us_per_call": us, "decode_kernel_us": kus,
             "decode_hbm_gbs": gbs, "decode_frac_of_hbm": gbs / peaks["hbm_gbs"],
             "decode_steps": a.decode_steps,
+            "paged": paged,
             "note": "decode bytes = K and V cache read once: 2*B*(c+1)*Hkv*D*2 per step; GB/s over the "
                     "split-KV + merge kernels (decode_kernel_us); decode_us_per_call adds the plan and "
                     "cache-write kernels and host launch overhead"}
+
+
+def measure_append_paged(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, page_size=256, decode_steps=64):
+    """The append-prefill and decode of ``measure_append`` against the same
+    cache held in shuffled pages of one pool (block table per sequence)."""
+    import torch
+    from paper_2408_00539_gb300 import ism
+    B, cap = kc.shape[0], kc.shape[1]
+    max_pages = (cap + page_size - 1) // page_size
+    rng = np.random.Generator(np.random.PCG64(a.seed))
+    table = rng.permutation(B * max_pages).reshape(B, max_pages).astype(np.int32)
+    rows = (torch.from_numpy(table).to(dev).long()[:, :, None] * page_size +
+            torch.arange(page_size, device=dev)[None, None, :]).reshape(B, -1)[:, :cap]
+    kp = torch.empty((B * max_pages * page_size,) + tuple(kc.shape[2:]), dtype=kc.dtype, device=dev)
+    vp = torch.empty_like(kp)
+    kp[rows.reshape(-1)] = kc.reshape((-1,) + tuple(kc.shape[2:]))
+    vp[rows.reshape(-1)] = vc.reshape((-1,) + tuple(vc.shape[2:]))
+    del rows
+    td = torch.from_numpy(table).to(dev)
+    c0 = a.cache_len.copy()
+    cl = torch.from_numpy(c0.copy()).to(dev)
+    stream = torch.cuda.current_stream(dev)
+    pre_ms = []
+    for it in range(8):
+        cl.copy_(torch.from_numpy(c0))
+        flush.fill_(1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        ism.prefill_append_paged(qn, kn, vn, kp, vp, page_size, td, table, cl, c0, a.new_seg_end, a.new_seg_type,
+                                 a.softmax_scale)
+        e1.record(stream)
+        e1.synchronize()
+        if it >= 3:
+            pre_ms.append(e0.elapsed_time(e1))
+    c_host = c0 + a.l_new
+    cl.copy_(torch.from_numpy(c_host))
+    dec_kernel_us = []
+    for t in range(decode_steps):
+        k0, k1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        for e in (k0, k1):
+            e.record(stream)
+        ism.set_kernel_timer(ism.KERNEL_DECODE, k0, k1)
+        ism.prefill_append_paged(qd, kd, vd, kp, vp, page_size, td, table, cl, c_host, [1], [1], a.softmax_scale)
+        k1.synchronize()
+        ism.set_kernel_timer(ism.KERNEL_DECODE)
+        dec_kernel_us.append(k0.elapsed_time(k1) * 1e3)
+        c_host = c_host + 1
+    ism.check_status(dev)
+    del kp, vp
+    return {"page_size": page_size, "prefill_ms": float(np.median(pre_ms)),
+            "decode_kernel_us": float(np.median(dec_kernel_us[3:])), "decode_steps": decode_steps}
 
 
 def measure_session(dev):

@@ -218,6 +218,37 @@ ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batc
                                      void* workspace, size_t workspace_bytes, ism_stream_t stream);
 
 /* ---------------------------------------------------------------------------
+ * Append-prefill and decode against a paged KV cache: the same operation as
+ * ism_attn_prefill_append (Section 2.3, Eq. fj on the new chunk, every cached
+ * key visible), with the keys and values of sequence b kept in fixed-size
+ * pages of a shared pool instead of one contiguous row range.  Key position p
+ * of sequence b lives in row  block_table[b * max_pages + p / page_size] *
+ * page_size + p % page_size  of the pools.
+ *   k_pool/v_pool [num_pages * page_size, Hkv, D] (dtype, in/out)
+ *   page_size: a multiple of 128 (a 128-key tile never spans two pages)
+ *   block_table [B, max_pages] int32 device, block_table_host its host mirror:
+ *     the pages of sequence b, in key order; entries that cover keys
+ *     [0, cache_len[b] + l_new) must lie in [0, num_pages), the rest are not read.
+ *     Two sequences may share a page only where both only read it.
+ *   cache_len / cache_len_host as for ism_attn_prefill_append;
+ *     cache_len_host[b] + l_new <= max_pages * page_size is required.
+ * The other arguments, the outputs and the workspace
+ * (ism_attn_prefill_append_workspace_size) are those of ism_attn_prefill_append.
+ * Results equal those of ism_attn_prefill_append on the gathered cache.
+ * Errors: ISM_ERR_INVALID_ARG for a page_size that is not a positive multiple
+ * of 128, a block-table entry outside the pool, or too few pages.
+ * ------------------------------------------------------------------------- */
+ism_status_t ism_attn_prefill_append_paged(const ism_attn_shape_t* shape, int32_t batch,
+                                           const void* q_new, const void* k_new, const void* v_new,
+                                           int32_t l_new, const int32_t* new_seg_end_host,
+                                           const uint8_t* new_seg_type_host, int32_t n_new_segs,
+                                           void* k_pool, void* v_pool, int32_t num_pages, int32_t page_size,
+                                           const int32_t* block_table, const int32_t* block_table_host,
+                                           int32_t max_pages, int32_t* cache_len, const int32_t* cache_len_host,
+                                           void* o_new, float* lse_new,
+                                           void* workspace, size_t workspace_bytes, ism_stream_t stream);
+
+/* ---------------------------------------------------------------------------
  * Status and diagnostics.
  * ------------------------------------------------------------------------- */
 

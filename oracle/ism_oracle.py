@@ -350,3 +350,28 @@ def prefill_append(q_new, k_new, v_new, k_cache, v_cache, cache_len, new_seg_end
             o[b, want, h] = ob
             lse[b, h, want] = lb
     return o, lse
+
+
+def gather_pages(pool, block_table, page_size: int, n_keys: int):
+    """Keys [0, n_keys) of one sequence of a paged cache, in order: key p is
+    row block_table[p // page_size] * page_size + p % page_size of the pool."""
+    pool = np.asarray(pool) if not hasattr(pool, "numpy") else pool
+    rows = [int(block_table[p // page_size]) * page_size + p % page_size for p in range(n_keys)]
+    return pool[rows]
+
+
+def prefill_append_paged(q_new, k_new, v_new, k_pool, v_pool, page_size: int, block_table, cache_len,
+                         new_seg_end, new_seg_type, scale: float):
+    """Append-prefill against a paged cache: the same operation as
+    ``prefill_append`` on the cache each sequence's block table gathers.
+    block_table [B, max_pages].  Returns (O_new, LSE_new) as float64."""
+    B = q_new.shape[0]
+    cap = max(int(c) for c in cache_len) if B else 0
+    kc = np.zeros((B, cap) + tuple(k_new.shape[2:]))
+    vc = np.zeros((B, cap) + tuple(v_new.shape[2:]))
+    for b in range(B):
+        c = int(cache_len[b])
+        kc[b, :c] = _f64(gather_pages(k_pool, block_table[b], page_size, c))
+        vc[b, :c] = _f64(gather_pages(v_pool, block_table[b], page_size, c))
+    return prefill_append(q_new, k_new, v_new, kc, vc, cache_len, new_seg_end, new_seg_type, scale)
+

@@ -522,17 +522,24 @@ ism_status_t ism_attn_prefill_append_workspace_size(const ism_attn_shape_t* shap
   return ISM_OK;
 }
 
-ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,
-                                     const void* k_new, const void* v_new, int32_t l_new,
-                                     const int32_t* new_seg_end_host, const uint8_t* new_seg_type_host,
-                                     int32_t n_new_segs, void* k_cache, void* v_cache, int64_t cache_capacity,
-                                     int32_t* cache_len, const int32_t* cache_len_host, void* o_new,
-                                     float* lse_new, void* workspace, size_t workspace_bytes,
-                                     ism_stream_t stream) {
-  ism_status_t r = check_shape(shape);
-  if (r != ISM_OK) return r;
-  if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
-  if (batch == 0 || l_new == 0) return ISM_OK;
+}  // extern "C"
+
+namespace {
+
+// Cache geometry of one append call: contiguous [B, cap] caches, or pages.
+struct CacheGeom {
+  int64_t cap;       // contiguous: rows per sequence
+  int64_t kv_rows;   // rows of the K / V tensors (tensor-map extent)
+  int64_t max_keys;  // keys a sequence can hold
+  KvPages pages;     // table == nullptr: contiguous
+};
+
+ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const void* q_new, const void* k_new,
+                         const void* v_new, int32_t l_new, const int32_t* new_seg_end_host,
+                         const uint8_t* new_seg_type_host, int32_t n_new_segs, void* k_cache, void* v_cache,
+                         const CacheGeom& cg, int32_t* cache_len, const int32_t* cache_len_host, void* o_new,
+                         float* lse_new, void* workspace, size_t workspace_bytes, cudaStream_t st) {
+  ism_status_t r;
   if (!q_new || !k_new || !v_new || !k_cache || !v_cache || !cache_len || !cache_len_host || !o_new)
     return fail(ISM_ERR_INVALID_ARG, "q_new, k_new, v_new, caches, cache_len (device+host), o_new must be non-NULL");
   const void* ptrs[] = {q_new, k_new, v_new, k_cache, v_cache, o_new};
@@ -553,37 +560,37 @@ ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batc
     sg.type[i] = new_seg_type_host[i];
   }
   if (prev != l_new) return fail(ISM_ERR_INVALID_ARG, "chunk segments end at %d, l_new is %d", prev, l_new);
-  if (cache_capacity <= 0 || (int64_t)batch * cache_capacity >= (int64_t(1) << 31))
-    return fail(ISM_ERR_INVALID_ARG, "batch * cache_capacity must be in (0, 2^31)");
   if ((int64_t)batch * l_new >= (int64_t(1) << 31)) return fail(ISM_ERR_INVALID_ARG, "batch * l_new too large");
   int32_t max_c = 0;
   for (int b = 0; b < batch; ++b) {
     int32_t c = cache_len_host[b];
-    if (c < 0 || (int64_t)c + l_new > cache_capacity)
+    if (c < 0 || (int64_t)c + l_new > cg.max_keys)
       return fail(ISM_ERR_INVALID_ARG, "sequence %d: cache_len %d + l_new %d exceeds capacity %lld", b, c, l_new,
-                  (long long)cache_capacity);
+                  (long long)cg.max_keys);
     if (c > max_c) max_c = c;
   }
   AppendLayout L = append_layout(workspace, shape, batch, l_new);
   if ((r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
   uint32_t* status;
   if ((r = status_ptr(&status)) != ISM_OK) return r;
-  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   const int hq = shape->num_heads_q, hkv = shape->num_heads_kv, d = shape->head_dim;
+  const bool paged = cg.pages.table != nullptr;
 
   timer_begin(ISM_KERNEL_META, st);
-  ISM_TRY_CUDA(launch_append_plan(sg, batch, cache_capacity, kTile, kTile, cache_len, L.c_snap, L.kv_end, L.qtiles,
+  ISM_TRY_CUDA(launch_append_plan(sg, batch, paged ? 1 : cg.cap, kTile, kTile, cache_len, L.c_snap, L.kv_end, L.qtiles,
                                   L.q_order, st),
                "append plan launch");
-  ISM_TRY_CUDA(launch_cache_write(shape->dtype, batch, l_new, hkv, d, cache_capacity, L.c_snap, k_new, v_new,
+  ISM_TRY_CUDA(launch_cache_write(shape->dtype, batch, l_new, hkv, d, cg.cap, cg.pages, L.c_snap, k_new, v_new,
                                   k_cache, v_cache, st),
                "cache write launch");
   timer_end(ISM_KERNEL_META, st);
   count_launch(2);
   if (l_new == 1 && shape->dtype == ISM_BF16 && !force_cuda_cores()) {
     DecodeArgs a{};
-    a.q = q_new; a.k_cache = k_cache; a.v_cache = v_cache; a.out = o_new; a.lse = lse_new; a.c_snap = L.c_snap;
-    a.batch = batch; a.hq = hq; a.hkv = hkv; a.d = d; a.dtype = shape->dtype; a.cap = cache_capacity;
+    a.q = q_new; a.k_cache = k_cache; a.v_cache = v_cache; a.pages = cg.pages; a.out = o_new; a.lse = lse_new;
+    a.c_snap = L.c_snap;
+    a.batch = batch; a.hq = hq; a.hkv = hkv; a.d = d; a.dtype = shape->dtype; a.cap = cg.cap;
+    a.kv_rows = cg.kv_rows;
     a.scale = shape->softmax_scale;
     // chunks of a multiple of 64 keys, as many as fill whole waves of resident
     // CTAs: 4 per SM for the register kernel (one wave), 2 per SM for the TMA
@@ -616,17 +623,86 @@ ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batc
   a.q_rows = (int64_t)batch * l_new; a.scale = shape->softmax_scale;
   a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order;
   a.nq = (int64_t)batch * ((l_new + kTile - 1) / kTile);
+  a.pages = cg.pages;
   a.status = status;
   a.flags = tc_flags();
   timer_begin(ISM_KERNEL_FWD, st);
   if (use_tc(shape)) {
-    ISM_TRY_CUDA(launch_tc_fwd(a, (int64_t)batch * cache_capacity, st), "tensor-core prefill launch");
+    ISM_TRY_CUDA(launch_tc_fwd(a, cg.kv_rows, st), "tensor-core prefill launch");
   } else {
     ISM_TRY_CUDA(launch_simt_fwd(a, st), "prefill launch");
   }
   timer_end(ISM_KERNEL_FWD, st);
   count_launch(1);
   return ISM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,
+                                     const void* k_new, const void* v_new, int32_t l_new,
+                                     const int32_t* new_seg_end_host, const uint8_t* new_seg_type_host,
+                                     int32_t n_new_segs, void* k_cache, void* v_cache, int64_t cache_capacity,
+                                     int32_t* cache_len, const int32_t* cache_len_host, void* o_new,
+                                     float* lse_new, void* workspace, size_t workspace_bytes,
+                                     ism_stream_t stream) {
+  ism_status_t r = check_shape(shape);
+  if (r != ISM_OK) return r;
+  if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
+  if (batch == 0 || l_new == 0) return ISM_OK;
+  if (cache_capacity <= 0 || (int64_t)batch * cache_capacity >= (int64_t(1) << 31))
+    return fail(ISM_ERR_INVALID_ARG, "batch * cache_capacity must be in (0, 2^31)");
+  CacheGeom cg;
+  cg.cap = cache_capacity;
+  cg.kv_rows = (int64_t)batch * cache_capacity;
+  cg.max_keys = cache_capacity;
+  cg.pages = KvPages{nullptr, 0, 0};
+  return append_impl(shape, batch, q_new, k_new, v_new, l_new, new_seg_end_host, new_seg_type_host, n_new_segs,
+                     k_cache, v_cache, cg, cache_len, cache_len_host, o_new, lse_new, workspace, workspace_bytes,
+                     reinterpret_cast<cudaStream_t>(stream));
+}
+
+ism_status_t ism_attn_prefill_append_paged(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,
+                                           const void* k_new, const void* v_new, int32_t l_new,
+                                           const int32_t* new_seg_end_host, const uint8_t* new_seg_type_host,
+                                           int32_t n_new_segs, void* k_pool, void* v_pool, int32_t num_pages,
+                                           int32_t page_size, const int32_t* block_table,
+                                           const int32_t* block_table_host, int32_t max_pages, int32_t* cache_len,
+                                           const int32_t* cache_len_host, void* o_new, float* lse_new,
+                                           void* workspace, size_t workspace_bytes, ism_stream_t stream) {
+  ism_status_t r = check_shape(shape);
+  if (r != ISM_OK) return r;
+  if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
+  if (batch == 0 || l_new == 0) return ISM_OK;
+  if (page_size <= 0 || page_size % kTile != 0)
+    return fail(ISM_ERR_INVALID_ARG, "page_size %d must be a positive multiple of %d", page_size, kTile);
+  if (num_pages <= 0 || (int64_t)num_pages * page_size >= (int64_t(1) << 31))
+    return fail(ISM_ERR_INVALID_ARG, "num_pages * page_size must be in (0, 2^31)");
+  if (max_pages <= 0 || !block_table || !block_table_host || !cache_len_host)
+    return fail(ISM_ERR_INVALID_ARG, "block_table (device+host), cache_len_host and max_pages > 0 are required");
+  // every page a sequence reads or writes in this call lies in the pool
+  for (int b = 0; b < batch; ++b) {
+    const int64_t keys = (int64_t)cache_len_host[b] + l_new;
+    if (cache_len_host[b] < 0 || keys > (int64_t)max_pages * page_size)
+      return fail(ISM_ERR_INVALID_ARG, "sequence %d: cache_len %d + l_new %d exceeds its %d pages", b, cache_len_host[b],
+                  l_new, max_pages);
+    for (int64_t i = 0; i < (keys + page_size - 1) / page_size; ++i) {
+      const int32_t pg = block_table_host[(int64_t)b * max_pages + i];
+      if (pg < 0 || pg >= num_pages)
+        return fail(ISM_ERR_INVALID_ARG, "sequence %d: page %lld of the block table is %d, outside [0, %d)", b,
+                    (long long)i, pg, num_pages);
+    }
+  }
+  CacheGeom cg;
+  cg.cap = 0;
+  cg.kv_rows = (int64_t)num_pages * page_size;
+  cg.max_keys = (int64_t)max_pages * page_size;
+  cg.pages = KvPages{block_table, page_size, max_pages};
+  return append_impl(shape, batch, q_new, k_new, v_new, l_new, new_seg_end_host, new_seg_type_host, n_new_segs,
+                     k_pool, v_pool, cg, cache_len, cache_len_host, o_new, lse_new, workspace, workspace_bytes,
+                     reinterpret_cast<cudaStream_t>(stream));
 }
 
 // ---------------------------------------------------------------- status

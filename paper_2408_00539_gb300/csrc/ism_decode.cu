@@ -74,8 +74,8 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
 #pragma unroll
     for (int i = 0; i < DPL; ++i) o[h][i] = 0.f;
 
-  const __nv_bfloat16* kbase = Kc + (int64_t)b * a.cap * kstride + (int64_t)g * D + lane * DPL;
-  const __nv_bfloat16* vbase = Vc + (int64_t)b * a.cap * kstride + (int64_t)g * D + lane * DPL;
+  const __nv_bfloat16* kbase = Kc + (int64_t)g * D + lane * DPL;
+  const __nv_bfloat16* vbase = Vc + (int64_t)g * D + lane * DPL;
   for (int kb = k0 + warp * KPI; kb < k1; kb += kDecWarps * KPI) {
     // every K and V row load of the batch is issued before any use; rows past
     // the chunk re-read its last key and get probability 0
@@ -83,8 +83,9 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
 #pragma unroll
     for (int t = 0; t < KPI; ++t) {
       const int key = min(kb + t, k1 - 1);
-      kraw[t] = *reinterpret_cast<const Raw*>(kbase + (int64_t)key * kstride);
-      vraw[t] = *reinterpret_cast<const Raw*>(vbase + (int64_t)key * kstride);
+      const int64_t row = a.pages.table ? paged_row(a.pages, b, key) : (int64_t)b * a.cap + key;
+      kraw[t] = *reinterpret_cast<const Raw*>(kbase + row * kstride);
+      vraw[t] = *reinterpret_cast<const Raw*>(vbase + row * kstride);
     }
     float v[32];  // v[h * KPI + t]: this lane's partial dot product
 #pragma unroll
@@ -226,7 +227,9 @@ __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__
         if (t >= kTmaStages && !tc::wait(&empty[s], (uint32_t)(t / kTmaStages - 1) & 1, a.status)) break;
         issued = t + 1;
         uint8_t* st = dsm + s * kTmaStageBytes;
-        const int32_t y = row0 + t * kTmaTile;
+        // a page holds whole tiles: page_size is a multiple of 128, tiles start at multiples of 64
+        const int32_t y = a.pages.table ? (int32_t)paged_row(a.pages, b, (int64_t)k0 + t * kTmaTile)
+                                        : row0 + t * kTmaTile;
         ptx::mbar_expect_tx(&full[s], kTmaStageBytes);
         ptx::tma_load_2d(st, &tmK, &full[s], g * D, y);
         ptx::tma_load_2d(st + kTmaHalf, &tmK, &full[s], g * D + 64, y);
@@ -383,7 +386,7 @@ cudaError_t run(const DecodeArgs& a, cudaStream_t st) {
   if (a.tma && G >= 2) {
     using Cfg = TmaCfg<G >= 2 ? G : 2>;
     CUtensorMap tk, tv;
-    const uint64_t rows = (uint64_t)a.batch * a.cap;
+    const uint64_t rows = (uint64_t)a.kv_rows;
     if ((e = tc::make_tmap_bf16_plain(&tk, a.k_cache, (uint64_t)a.hkv * D, rows, Cfg::kTile)) != cudaSuccess) return e;
     if ((e = tc::make_tmap_bf16_plain(&tv, a.v_cache, (uint64_t)a.hkv * D, rows, Cfg::kTile)) != cudaSuccess) return e;
     const int smem = Cfg::kStages * Cfg::kStageBytes + 2 * Cfg::kStages * 8 + (8 * G + 4 * G * D) * 4;

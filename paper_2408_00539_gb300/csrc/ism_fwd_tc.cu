@@ -113,7 +113,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int s = j & 1;
         const uint32_t n = (uint32_t)(j >> 1);
         if (__any_sync(0xffffffffu, aborted(bar))) break;
-        const int32_t ky = w.k_base + j * kRows;
+        const int32_t ky = a.pages.table ? (int32_t)paged_row(a.pages, w.k_base, (int64_t)j * kRows)
+                                         : w.k_base + j * kRows;
         if (j >= kStages && !wait_warp(&bar->k_empty[s], (n - 1) & 1, a.status)) {
           if (lane == 0) set_abort(bar);
           break;

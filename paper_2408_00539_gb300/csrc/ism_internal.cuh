@@ -25,6 +25,18 @@ struct Tile {
 };
 static_assert(sizeof(Tile) == 32, "Tile layout");
 
+// Paged K/V cache (append-prefill and decode): key p of sequence b sits in
+// row table[b * max_pages + p / page_size] * page_size + p % page_size of the
+// pools.  With table == nullptr the cache is contiguous: the rows of sequence
+// b start at b * cap (append kernels) or at Tile::k_base (attention kernels).
+struct KvPages {
+  const int32_t* table;
+  int32_t page_size, max_pages;
+};
+__device__ __forceinline__ int64_t paged_row(const KvPages& pg, int b, int64_t p) {
+  return (int64_t)__ldg(pg.table + (int64_t)b * pg.max_pages + p / pg.page_size) * pg.page_size + p % pg.page_size;
+}
+
 // Device view of the segment arrays (device pointers only).
 struct SegsDev {
   int32_t num_seqs;
@@ -75,10 +87,11 @@ cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, 
                              Tile* qtiles, Tile* ktiles, int max_cost, int32_t* q_order, int32_t* k_order,
                              int32_t* pair_order, int32_t* kpair_off, int32_t* counters, int n_counters,
                              cudaStream_t st);
-cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t cap, int bm, int bn,
+// k_base of sequence b's tiles = b * kbase_stride (the cache capacity, or 1 for a paged cache)
+cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t kbase_stride, int bm, int bn,
                                int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
                                int32_t* q_order, cudaStream_t st);
-cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap,
+cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap, const KvPages& pages,
                                const int32_t* c_snap, const void* k_new, const void* v_new,
                                void* k_cache, void* v_cache, cudaStream_t st);
 
@@ -109,6 +122,9 @@ struct AttnArgs {
   int64_t npairs;
   // Work counter of the persistent dK/dV kernel (zeroed by the metadata pass).
   int32_t* work_counter;
+  // Paged K/V (forward over an appended chunk only): Tile::k_base holds the
+  // sequence index and key p's row is paged_row(pages, k_base, p).
+  KvPages pages;
   // Bit 0: before an MMA that overwrites tensor memory an earlier MMA reads
   // as its A operand, wait for that earlier MMA to complete.  Clear: rely on
   // MMAs issued by one thread executing in issue order.
@@ -121,13 +137,15 @@ cudaError_t launch_simt_bwd(const AttnArgs& a, cudaStream_t st);
 // Split-KV decode for single-token appends (ism_decode.cu).
 struct DecodeArgs {
   const void* q;         // [B, Hq, D]
-  const void* k_cache;   // [B, cap, Hkv, D]
+  const void* k_cache;   // [B, cap, Hkv, D], or the page pools [pages * page_size, Hkv, D]
   const void* v_cache;
+  KvPages pages;         // table == nullptr: contiguous caches
   void* out;             // [B, Hq, D]
   float* lse;            // [Hq, B] or null
   const int32_t* c_snap; // cache length before the append, per sequence
   int32_t batch, hq, hkv, d, dtype;
   int64_t cap;
+  int64_t kv_rows;       // rows of the K / V tensors: batch * cap, or pages * page_size
   float scale;
   int32_t splits, chunk;
   float* part_o;         // [B, Hq, splits, D]

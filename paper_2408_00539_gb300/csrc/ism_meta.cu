@@ -279,7 +279,7 @@ __device__ __forceinline__ int32_t chunk_kv_end(const AppendSegs& sg, int32_t j)
 // Append plan (one block): snapshot cache_len, advance it by l_new, write the
 // absolute key bound of every new row (all cached keys plus Eq. fj within
 // the chunk) and one q-tile descriptor per (sequence, chunk tile).
-__global__ void append_plan_kernel(AppendSegs sg, int batch, int64_t cap, int bm, int bn,
+__global__ void append_plan_kernel(AppendSegs sg, int batch, int64_t kbase_stride, int bm, int bn,
                                    int32_t* cache_len, int32_t* c_snap, int32_t* kv_end,
                                    Tile* qtiles, int32_t* q_order) {
   __shared__ int32_t cs[1024];
@@ -300,7 +300,7 @@ __global__ void append_plan_kernel(AppendSegs sg, int batch, int64_t cap, int bm
       int32_t c = cs[bl];
       int32_t r0 = t * bm, rl = min(Ln, r0 + bm) - 1;
       Tile w;
-      w.q_base = (base + bl) * Ln; w.k_base = (int32_t)((base + bl) * cap);
+      w.q_base = (base + bl) * Ln; w.k_base = (int32_t)((base + bl) * kbase_stride);
       w.q_len = Ln; w.k_len = c + Ln; w.tile = t;
       w.a0 = (r0 + bm <= Ln) ? (c + chunk_kv_end(sg, r0)) / bn : 0;
       w.a1 = (c + chunk_kv_end(sg, rl) + bn - 1) / bn;
@@ -318,8 +318,9 @@ __global__ void append_plan_kernel(AppendSegs sg, int batch, int64_t cap, int bm
   }
 }
 
-// K_new/V_new rows into the caches at [c_snap[b], c_snap[b] + l_new).
-__global__ void cache_write_kernel(int batch, int l_new, int row_bytes, int64_t cap,
+// K_new/V_new rows into the caches at [c_snap[b], c_snap[b] + l_new) (rows of
+// sequence b from b * cap, or through the page table).
+__global__ void cache_write_kernel(int batch, int l_new, int row_bytes, int64_t cap, KvPages pages,
                                    const int32_t* __restrict__ c_snap, const uint4* __restrict__ k_new,
                                    const uint4* __restrict__ v_new, uint4* k_cache, uint4* v_cache) {
   const int vec_per_row = row_bytes / 16;
@@ -330,7 +331,8 @@ __global__ void cache_write_kernel(int batch, int l_new, int row_bytes, int64_t 
     int col = (int)(i % vec_per_row);
     int b = (int)(row / l_new);
     int j = (int)(row % l_new);
-    int64_t dst = ((int64_t)b * cap + c_snap[b] + j) * vec_per_row + col;
+    const int64_t p = (int64_t)c_snap[b] + j;
+    int64_t dst = (pages.table ? paged_row(pages, b, p) : (int64_t)b * cap + p) * vec_per_row + col;
     k_cache[dst] = k_new[i];
     v_cache[dst] = v_new[i];
   }
@@ -395,15 +397,15 @@ cudaError_t launch_pair_offsets(const Tile* ktiles, int64_t nk, int32_t* kpair_o
   return cudaGetLastError();
 }
 
-cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t cap, int bm, int bn,
+cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t kbase_stride, int bm, int bn,
                                int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
                                int32_t* q_order, cudaStream_t st) {
-  append_plan_kernel<<<1, 1024, 0, st>>>(segs, batch, cap, bm, bn, cache_len, c_snap, kv_end, qtiles,
+  append_plan_kernel<<<1, 1024, 0, st>>>(segs, batch, kbase_stride, bm, bn, cache_len, c_snap, kv_end, qtiles,
                                          q_order);
   return cudaGetLastError();
 }
 
-cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap,
+cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap, const KvPages& pages,
                                const int32_t* c_snap, const void* k_new, const void* v_new,
                                void* k_cache, void* v_cache, cudaStream_t st) {
   int elem = dtype == ISM_BF16 ? 2 : 4;
@@ -412,7 +414,7 @@ cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, 
   if (total == 0) return cudaSuccess;
   int grid = (int)((total + 255) / 256);
   if (grid > 152 * 16) grid = 152 * 16;
-  cache_write_kernel<<<grid, 256, 0, st>>>(batch, l_new, row_bytes, cap, c_snap, (const uint4*)k_new,
+  cache_write_kernel<<<grid, 256, 0, st>>>(batch, l_new, row_bytes, cap, pages, c_snap, (const uint4*)k_new,
                                            (const uint4*)v_new, (uint4*)k_cache, (uint4*)v_cache);
   return cudaGetLastError();
 }

@@ -61,6 +61,10 @@ __global__ void __launch_bounds__(kWarps * 32) simt_fwd_kernel(AttnArgs a) {
     for (int d = lane; d < D; d += 32) qs[warp][d] = ld(Q + qrow * qstride + (int64_t)h * D + d);
     __syncwarp();
     const int ke = a.kv_end[w.kv_base + row];
+    // K / V row of key p (through the page table for a paged cache)
+    auto kvrow = [&](int p) -> int64_t {
+      return a.pages.table ? paged_row(a.pages, w.k_base, p) : (int64_t)w.k_base + p;
+    };
     float m = -INFINITY, l = 0.f;
     float acc[D / 32];
 #pragma unroll
@@ -68,7 +72,7 @@ __global__ void __launch_bounds__(kWarps * 32) simt_fwd_kernel(AttnArgs a) {
     for (int kb = 0; kb < ke; kb += 32) {
       const int key = kb + lane;
       float s = -INFINITY;
-      if (key < ke) s = a.scale * dot_row<T, D>(qs[warp], K + ((int64_t)w.k_base + key) * kstride + (int64_t)g * D);
+      if (key < ke) s = a.scale * dot_row<T, D>(qs[warp], K + kvrow(key) * kstride + (int64_t)g * D);
       const float mc = warp_max(s);
       const float mn = fmaxf(m, mc);
       const float alpha = (m == -INFINITY) ? 0.f : expf(m - mn);
@@ -79,7 +83,7 @@ __global__ void __launch_bounds__(kWarps * 32) simt_fwd_kernel(AttnArgs a) {
       const int nk = min(32, ke - kb);
       for (int t = 0; t < nk; ++t) {
         const float pt = __shfl_sync(0xffffffffu, p, t);
-        const T* vrow = V + ((int64_t)w.k_base + kb + t) * kstride + (int64_t)g * D;
+        const T* vrow = V + kvrow(kb + t) * kstride + (int64_t)g * D;
 #pragma unroll
         for (int i = 0; i < D / 32; ++i) acc[i] = fmaf(pt, ld(vrow + lane + 32 * i), acc[i]);
       }

@@ -57,6 +57,11 @@ EXPORTS = {
                                           C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_int64,
                                           C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                           C.c_size_t, C.c_void_p]),
+    "ism_attn_prefill_append_paged": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
+                                                C.c_int32, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p,
+                                                C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p,
+                                                C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
+                                                C.c_void_p]),
     "ism_check_status": (C.c_int, [C.c_void_p]),
     "ism_debug_timeout_probe": (C.c_int, [C.c_uint32, C.c_void_p]),
     "ism_status_string": (C.c_char_p, [C.c_int]),
@@ -301,6 +306,41 @@ def prefill_append(q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_h
                                        _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(),
                                        _stream(q_new.device)),
            "ism_attn_prefill_append")
+    return out, lse
+
+
+def prefill_append_paged(q_new, k_new, v_new, k_pool, v_pool, page_size: int, block_table, block_table_host,
+                         cache_len, cache_len_host, new_seg_end, new_seg_type, softmax_scale: float, out=None,
+                         lse=None, workspace=None):
+    """``prefill_append`` against a paged cache (Section 2.3): k_pool/v_pool
+    [num_pages * page_size, Hkv, D]; key p of sequence b is pool row
+    block_table[b, p // page_size] * page_size + p % page_size.  block_table
+    int32 [B, max_pages] on the device, block_table_host its host mirror
+    (numpy); cache_len / cache_len_host as for ``prefill_append``."""
+    lib = load()
+    _contig(q_new, k_new, v_new, k_pool, v_pool, cache_len, block_table)
+    B, Ln, hq, D = q_new.shape
+    rows = k_pool.shape[0]
+    if rows % page_size:
+        raise ValueError("pool rows must be a whole number of pages")
+    sh = _shape(q_new, k_new, softmax_scale)
+    se = np.ascontiguousarray(new_seg_end, dtype=np.int32)
+    st = np.ascontiguousarray(new_seg_type, dtype=np.uint8)
+    ch = np.ascontiguousarray(cache_len_host, dtype=np.int32)
+    bt = np.ascontiguousarray(block_table_host, dtype=np.int32)
+    if out is None:
+        out = torch.empty_like(q_new)
+    if lse is None:
+        lse = torch.empty((hq, B, Ln), dtype=torch.float32, device=q_new.device)
+    if workspace is None:
+        workspace = _workspace(append_workspace_size(q_new, k_new, softmax_scale), q_new.device)
+    _check(lib.ism_attn_prefill_append_paged(C.byref(sh), B, _ptr(q_new), _ptr(k_new), _ptr(v_new), Ln,
+                                             C.c_void_p(se.ctypes.data), C.c_void_p(st.ctypes.data), se.shape[0],
+                                             _ptr(k_pool), _ptr(v_pool), rows // page_size, page_size,
+                                             _ptr(block_table), C.c_void_p(bt.ctypes.data), block_table.shape[1],
+                                             _ptr(cache_len), C.c_void_p(ch.ctypes.data), _ptr(out), _ptr(lse),
+                                             _ptr(workspace), workspace.numel(), _stream(q_new.device)),
+           "ism_attn_prefill_append_paged")
     return out, lse
 
 

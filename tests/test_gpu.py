@@ -446,3 +446,74 @@ def test_session_turn_by_turn_matches_one_pass(ism):
     for b in range(B):
         o_ref, _ = orc.attn_fwd(q[b], k[b], v[b], segs, s.softmax_scale)
         _cmp(f"session dialogue {b}", o[b], o_ref, "bf16")
+
+
+def _to_pages(kc, vc, page_size, rng, spare=3):
+    """Scatter contiguous caches [B, cap, Hkv, D] into shuffled pages of one pool
+    (plus a few unused pages): returns (k_pool, v_pool, block_table [B, max_pages])."""
+    B, cap = kc.shape[:2]
+    max_pages = (cap + page_size - 1) // page_size
+    n_pages = B * max_pages + spare
+    table = rng.permutation(n_pages)[:B * max_pages].reshape(B, max_pages).astype(np.int32)
+    kp = torch.zeros((n_pages * page_size,) + tuple(kc.shape[2:]), dtype=kc.dtype)
+    vp = torch.zeros_like(kp)
+    for b in range(B):
+        for i in range(max_pages):
+            n = min(page_size, cap - i * page_size)
+            r = int(table[b, i]) * page_size
+            kp[r:r + n] = kc[b, i * page_size:i * page_size + n]
+            vp[r:r + n] = vc[b, i * page_size:i * page_size + n]
+    return kp, vp, table
+
+
+@pytest.mark.parametrize("l_new,segs,hq,hkv,d", [(200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2, 128),
+                                                  (128, ([128], [0]), 8, 2, 128), (1, ([1], [1]), 8, 2, 128),
+                                                  (1, ([1], [1]), 8, 1, 128), (37, ([37], [0]), 3, 3, 128),
+                                                  (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2, 64)])
+def test_prefill_append_paged_matches_contiguous(ism, l_new, segs, hq, hkv, d):
+    """The paged cache gives bit for bit the contiguous result (same kernels,
+    rows through the block table) and the oracle's result on the gathered cache."""
+    B, ps = 3, 128
+    c_lens = np.array([0, 77, 300], dtype=np.int32)
+    cap = int(c_lens.max()) + l_new
+    kc, vc, qn, kn, vn = _append_inputs(B, cap, c_lens, l_new, hq, hkv, d, seed=100 + l_new + d)
+    rng = np.random.Generator(np.random.PCG64(7 + l_new))
+    kp, vp, table = _to_pages(kc, vc, ps, rng)
+    scale = d ** -0.5
+    kcd, vcd = kc.to(DEV), vc.to(DEV)
+    cl = torch.from_numpy(c_lens.copy()).to(DEV)
+    o_c, l_c = ism.prefill_append(qn.to(DEV), kn.to(DEV), vn.to(DEV), kcd, vcd, cl, c_lens, segs[0], segs[1], scale)
+    kpd, vpd = kp.to(DEV), vp.to(DEV)
+    clp = torch.from_numpy(c_lens.copy()).to(DEV)
+    o_p, l_p = ism.prefill_append_paged(qn.to(DEV), kn.to(DEV), vn.to(DEV), kpd, vpd, ps,
+                                        torch.from_numpy(table).to(DEV), table, clp, c_lens, segs[0], segs[1], scale)
+    ism.check_status()
+    assert torch.equal(o_p, o_c) and torch.equal(l_p, l_c)
+    assert clp.cpu().numpy().tolist() == (c_lens + l_new).tolist()
+    # the new keys / values sit in the sequences' pages
+    kpc = kpd.cpu()
+    for b in range(B):
+        for j in range(l_new):
+            p = int(c_lens[b]) + j
+            r = int(table[b, p // ps]) * ps + p % ps
+            assert torch.equal(kpc[r], kn[b, j])
+    o_ref, lse_ref = orc.prefill_append_paged(qn, kn, vn, kp, vp, ps, table, c_lens, segs[0], segs[1], scale)
+    _cmp("paged o_new", o_p, o_ref, "bf16")
+    _cmp_lse("paged lse_new", l_p, np.transpose(lse_ref, (1, 0, 2)), "bf16")
+
+
+def test_paged_append_rejects_bad_tables(ism):
+    B, ps, hq, hkv, d = 2, 128, 8, 2, 128
+    c_lens = np.array([100, 200], dtype=np.int32)
+    kc, vc, qn, kn, vn = _append_inputs(B, 256, c_lens, 8, hq, hkv, d, seed=5)
+    kp, vp, table = _to_pages(kc, vc, ps, np.random.Generator(np.random.PCG64(1)))
+    cl = torch.from_numpy(c_lens.copy()).to(DEV)
+    args = (qn.to(DEV), kn.to(DEV), vn.to(DEV), kp.to(DEV), vp.to(DEV))
+    bad = table.copy()
+    bad[1, 1] = kp.shape[0] // ps  # one past the pool
+    with pytest.raises(ism.IsmError):
+        ism.prefill_append_paged(*args, ps, torch.from_numpy(bad).to(DEV), bad, cl, c_lens, [8], [0], d ** -0.5)
+    with pytest.raises(ism.IsmError):  # a page size that splits a 128-key tile
+        ism.prefill_append_paged(*args, 64, torch.from_numpy(table).to(DEV), table, cl, c_lens, [8], [0], d ** -0.5)
+    ism.check_status()
+    assert cl.cpu().numpy().tolist() == c_lens.tolist()  # nothing ran

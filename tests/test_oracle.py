@@ -376,6 +376,32 @@ def test_decode_is_causal_step_over_whole_cache():
             np.testing.assert_allclose(o[b, 0, h], (p / p.sum()) @ vals, rtol=1e-12, atol=1e-13)
 
 
+def test_paged_append_equals_contiguous_append():
+    # a paged cache holding the same keys (pages scattered over a shared pool,
+    # written here key by key) gives exactly the contiguous result
+    rng = np.random.Generator(np.random.PCG64(43))
+    B, Ln, hq, hkv, D, ps = 3, 7, 4, 2, 6, 4
+    c_lens = np.array([0, 5, 13])
+    cap = int(c_lens.max()) + Ln
+    kc, vc = _rand(rng, B, cap, hkv, D), _rand(rng, B, cap, hkv, D)
+    qn, kn, vn = _rand(rng, B, Ln, hq, D), _rand(rng, B, Ln, hkv, D), _rand(rng, B, Ln, hkv, D)
+    max_pages = (cap + ps - 1) // ps
+    perm = rng.permutation(B * max_pages)
+    table = perm.reshape(B, max_pages)
+    kpool = np.full((B * max_pages * ps, hkv, D), np.nan)
+    vpool = np.full((B * max_pages * ps, hkv, D), np.nan)
+    for b in range(B):
+        for p in range(int(c_lens[b])):
+            page, off = divmod(p, ps)
+            kpool[table[b, page] * ps + off] = kc[b, p]
+            vpool[table[b, page] * ps + off] = vc[b, p]
+    new_e, new_t = [3, 7], [0, 1]
+    o_ref, l_ref = orc.prefill_append(qn, kn, vn, kc, vc, c_lens, new_e, new_t, 0.5)
+    o, l = orc.prefill_append_paged(qn, kn, vn, kpool, vpool, ps, table, c_lens, new_e, new_t, 0.5)
+    np.testing.assert_array_equal(o, o_ref)
+    np.testing.assert_array_equal(l, l_ref)
+
+
 def test_workload_generator_shapes():
     for w in (wl.tiny_fp32(), wl.mha_4k(), wl.gqa_8k(), wl.packed_32k()):
         s = w.segs
