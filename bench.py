@@ -470,6 +470,7 @@ def run_cuda(args, w):
     if not args.no_append:
         line["append"] = measure_append(dev, read_peaks()[0])
         line["session"] = measure_session(dev)
+        line["training_cost"] = measure_training_cost(dev, w)
     if world == 1 and not args.no_cpu_baseline:
         val, dt, sample = oracle_sample(w, q, k, v, do, heads_per_sample=4)
         line["cpu_baseline"] = {"value": val, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
@@ -598,6 +599,44 @@ def measure_append_paged(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, page_siz
     del kp, vp
     return {"page_size": page_size, "prefill_ms": float(np.median(pre_ms)),
             "decode_kernel_us": float(np.median(dec_kernel_us[3:])), "decode_steps": decode_steps}
+
+
+def measure_training_cost(dev, w, reps=3):
+    """What one ISM pass saves in training against a prefix-LM, which needs
+    one sample per answer turn (history and query as a bidirectional prefix,
+    then the answer): tokens, visible pairs and the measured fwd+bwd time of
+    the same kernels on both batches (random values, same heads)."""
+    import torch
+    from paper_2408_00539_gb300 import ism
+    out = {}
+    for name, segs_np in (("ism_one_pass", w.segs), ("prefix_lm_triplets", wl.triplet_expansion(w.segs))):
+        T = segs_np.total_tokens
+        g = torch.Generator(device=dev).manual_seed(w.seed)
+        q = torch.randn((T, w.num_heads_q, w.head_dim), generator=g, device=dev).mul_(w.value_std).bfloat16()
+        k = torch.randn((T, w.num_heads_kv, w.head_dim), generator=g, device=dev).mul_(w.value_std).bfloat16()
+        v = torch.randn((T, w.num_heads_kv, w.head_dim), generator=g, device=dev).mul_(w.value_std).bfloat16()
+        do = torch.randn((T, w.num_heads_q, w.head_dim), generator=g, device=dev).bfloat16()
+        segs = ism.Segments.from_workload(segs_np, dev)
+        ms = []
+        for it in range(reps + 1):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            o, lse = ism.fwd(segs, q, k, v, w.softmax_scale)
+            ism.bwd(segs, q, k, v, o, lse, do, w.softmax_scale)
+            e1.record()
+            e1.synchronize()
+            if it:
+                ms.append(e0.elapsed_time(e1))
+        ism.check_status(dev)
+        out[name] = {"samples": segs_np.num_seqs, "tokens": T, "n_vis_pairs": n_visible(segs_np) * w.num_heads_q,
+                     "fwd_bwd_ms": float(np.median(ms))}
+        del q, k, v, do, o, lse
+        torch.cuda.empty_cache()
+    a, b = out["ism_one_pass"], out["prefix_lm_triplets"]
+    out["tokens_ratio"] = b["tokens"] / a["tokens"]
+    out["flops_ratio"] = b["n_vis_pairs"] / a["n_vis_pairs"]
+    out["time_ratio"] = b["fwd_bwd_ms"] / a["fwd_bwd_ms"]
+    return out
 
 
 def measure_session(dev):

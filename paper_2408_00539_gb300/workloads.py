@@ -207,6 +207,22 @@ def append_16k(seed: int = 5, batch: int = 8, cache_len: int = 16384, l_new: int
                           decode_steps, 32, 8, 128, 1.0 / np.sqrt(128.0), 0.5, seed)
 
 
+def triplet_expansion(segs: Segments) -> Segments:
+    """The training samples a prefix-LM needs for the same dialogues: one per
+    answer segment, holding everything before the answer as one bidirectional
+    prefix (a QUERY segment) followed by the answer (causal).  Each sample
+    re-reads the whole history that the one-pass ISM sequence shares."""
+    samples = []
+    for b in range(segs.num_seqs):
+        _, _, se, st = segs.seq(b)
+        start = 0
+        for e, t in zip(se.tolist(), st.tolist()):
+            if t == ANSWER and e > start:
+                samples.append(([start, e], [QUERY, ANSWER]) if start > 0 else ([e], [ANSWER]))
+            start = e
+    return pack(samples)
+
+
 @dataclass
 class SessionWorkload:
     """A serving session: every dialogue of the batch alternates a query turn,

@@ -34,3 +34,17 @@ def test_session_workload_shape():
     assert s.capacity == 4000 and ends[-1] == s.capacity and len(ends) == 2 * s.turns
     assert types == [wl.QUERY, wl.ANSWER] * s.turns
     assert all(b - a in (s.q_len, s.a_len) for a, b in zip([0] + ends[:-1], ends))
+
+
+def test_triplet_expansion_samples_and_counts():
+    # one sample per non-empty answer: everything before it as one bidirectional
+    # prefix, then the answer; pair counts agree with the materialised masks
+    segs = wl.pack([([5, 12, 20, 33], [wl.QUERY, wl.ANSWER, wl.QUERY, wl.ANSWER]),
+                    ([4, 9, 9], [wl.ANSWER, wl.QUERY, wl.ANSWER])])
+    tri = wl.triplet_expansion(segs)
+    got = [(tri.seq(b)[2].tolist(), tri.seq(b)[3].tolist()) for b in range(tri.num_seqs)]
+    assert got == [([5, 12], [0, 1]), ([20, 33], [0, 1]), ([4], [1])]
+    brute = sum(int(orc.mask_eq_fj(se, st).sum()) for _, _, se, st in (tri.seq(b) for b in range(tri.num_seqs)))
+    assert bench.n_visible(tri) == brute
+    # the one pass over each dialogue sees fewer pairs than its samples together
+    assert bench.n_visible(segs) < bench.n_visible(tri)
