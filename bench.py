@@ -471,6 +471,7 @@ def run_cuda(args, w):
         line["append"] = measure_append(dev, read_peaks()[0])
         line["session"] = measure_session(dev)
         line["training_cost"] = measure_training_cost(dev, w)
+        line["fwd_e4m3"] = measure_fwd_e4m3(dev, w, read_peaks()[0])
     if world == 1 and not args.no_cpu_baseline:
         val, dt, sample = oracle_sample(w, q, k, v, do, heads_per_sample=4)
         line["cpu_baseline"] = {"value": val, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
@@ -637,6 +638,43 @@ def measure_training_cost(dev, w, reps=3):
     out["flops_ratio"] = b["n_vis_pairs"] / a["n_vis_pairs"]
     out["time_ratio"] = b["fwd_bwd_ms"] / a["fwd_bwd_ms"]
     return out
+
+
+def measure_fwd_e4m3(dev, w, peaks, reps=10):
+    """The forward on e4m3 copies of the workload's Q, K, V (per-tensor scales,
+    fp8 tensor cores), against the bf16 forward of the same inputs; L2 flushed
+    between calls, CUDA events around each."""
+    import torch
+    from paper_2408_00539_gb300 import ism
+    q, k, v, _ = wl.attention_tensors(w)
+    segs = ism.Segments.from_workload(w.segs, dev)
+    qb, kb, vb = (t.to(dev) for t in (q, k, v))
+    q8, k8, v8 = (wl.quantize_e4m3(t) for t in (qb, kb, vb))
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def timed(fn):
+        ms = []
+        for it in range(reps + 2):
+            flush.fill_(1)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            e1.synchronize()
+            if it >= 2:
+                ms.append(e0.elapsed_time(e1))
+        return float(np.median(ms))
+
+    ms8 = timed(lambda: ism.fwd_e4m3(segs, q8[0], k8[0], v8[0], q8[1], k8[1], v8[1], w.softmax_scale))
+    ms16 = timed(lambda: ism.fwd(segs, qb, kb, vb, w.softmax_scale))
+    ism.check_status(dev)
+    flops = 4 * w.head_dim * n_visible(w.segs) * w.num_heads_q
+    peak8 = 2 * peaks["bf16_tflops"]  # e4m3 dense rate = 2x bf16 (nominal 4.5 vs 2.25 PFLOP/s)
+    return {"workload": w.name, "ms": ms8, "tflops": flops / (ms8 * 1e-3) / 1e12,
+            "frac_of_e4m3_peak": flops / (ms8 * 1e-3) / 1e12 / peak8, "e4m3_peak_tflops": peak8,
+            "bf16_fwd_ms": ms16, "speedup_over_bf16": ms16 / ms8,
+            "note": "fwd call incl. metadata pass; peak = measured bf16 x 2 (nominal fp8/bf16 ratio)"}
 
 
 def measure_session(dev):

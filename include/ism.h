@@ -48,7 +48,7 @@ typedef enum {
   ISM_ERR_WORKSPACE = 5     /* workspace pointer null/misaligned or smaller than required */
 } ism_status_t;
 
-typedef enum { ISM_BF16 = 0, ISM_FP32 = 1 } ism_dtype_t;
+typedef enum { ISM_BF16 = 0, ISM_FP32 = 1, ISM_E4M3 = 2 } ism_dtype_t;
 
 enum { ISM_SEG_QUERY = 0, ISM_SEG_ANSWER = 1 };
 enum { ISM_TILE_EMPTY = 0, ISM_TILE_FULL = 1, ISM_TILE_PARTIAL = 2 };
@@ -81,7 +81,8 @@ typedef struct {
 
 /* Heads and element type.  Supported: head_dim 64 or 128; Hq % Hkv == 0;
  * ISM_BF16 (fp32 accumulation, tensor cores) or ISM_FP32 (fp32 CUDA-core
- * path).  softmax_scale multiplies q.k before the softmax (the paper omits
+ * path); ISM_E4M3 (fp8 inputs, head_dim 128) only for ism_attn_fwd_e4m3 and
+ * its workspace query.  softmax_scale multiplies q.k before the softmax (the paper omits
  * the factor, Section 2.1; 1/sqrt(head_dim) is the usual choice). */
 typedef struct {
   int32_t num_heads_q;
@@ -132,6 +133,25 @@ ism_status_t ism_attn_fwd_workspace_size(const ism_segments_t* segs, const ism_a
 ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* shape,
                           const void* q, const void* k, const void* v, void* o, float* lse,
                           void* workspace, size_t workspace_bytes, ism_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * Forward with e4m3 (fp8) Q, K, V: the operation of ism_attn_fwd (Eq. e_ISM,
+ * the bound of Eq. fj) on the dequantised inputs q * q_descale, k * k_descale,
+ * v * v_descale (one factor per tensor).  shape->dtype must be ISM_E4M3 and
+ * head_dim 128; q [T, Hq, 128], k/v [T, Hkv, 128] e4m3 (OCP fp8 E4M3FN);
+ * o [T, Hq, 128] bf16 (written); lse [Hq, T] fp32 or NULL.  The score
+ * contraction and O += P V run on the fp8 tensor cores (kind::f8f6f4) with
+ * fp32 accumulation; P is rounded to e4m3 (round to nearest) for P V, the
+ * softmax statistics stay fp32.  Workspace: ism_attn_fwd_workspace_size with
+ * the same shape.  Errors as ism_attn_fwd, plus ISM_ERR_UNSUPPORTED without
+ * the sm_103 tensor cores and ISM_ERR_INVALID_ARG for a descale that is not
+ * a positive finite number.
+ * ------------------------------------------------------------------------- */
+ism_status_t ism_attn_fwd_e4m3(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                               const void* q, const void* k, const void* v,
+                               float q_descale, float k_descale, float v_descale,
+                               void* o, float* lse, void* workspace, size_t workspace_bytes,
+                               ism_stream_t stream);
 
 /* Forward without a caller-provided workspace (the paper has no counterpart;
  * this is a deployment convenience).  Some callers cannot allocate device
@@ -295,6 +315,12 @@ uint64_t ism_kernel_launches(void);
  *   the batched form the attention kernels use (one election, descriptors
  *   advanced by fixed offsets). */
 ism_status_t ism_debug_mma_tile(const void* a, const void* b, float* c, int32_t mode, ism_stream_t stream);
+/* The same for e4m3 operands (kind::f8f6f4, K = 32 a step), the layouts of
+ * the e4m3 forward: a [128,128] e4m3 row-major (M x K), c fp32 [128,128].
+ *   mode 0: b [128,128] is N x K, c = a * b^T (both K-major in shared memory)
+ *   mode 1: b is K x N (MN-major), c = a * b
+ *   mode 2: as mode 1 with a in tensor memory (four e4m3 a column). */
+ism_status_t ism_debug_mma_tile_e4m3(const void* a, const void* b, float* c, int32_t mode, ism_stream_t stream);
 
 const char* ism_status_string(ism_status_t status);
 /* Human-readable detail of the last failing call on this host thread. */

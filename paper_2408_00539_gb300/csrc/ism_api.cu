@@ -109,7 +109,7 @@ ism_status_t check_segments(const ism_segments_t* s, SegInfo* info) {
   return ISM_OK;
 }
 
-ism_status_t check_shape(const ism_attn_shape_t* sh) {
+ism_status_t check_shape(const ism_attn_shape_t* sh, bool allow_e4m3 = false) {
   if (!sh) return fail(ISM_ERR_INVALID_ARG, "shape is NULL");
   if (sh->num_heads_q <= 0 || sh->num_heads_kv <= 0) return fail(ISM_ERR_INVALID_ARG, "head counts must be > 0");
   if (sh->num_heads_q % sh->num_heads_kv)
@@ -117,7 +117,12 @@ ism_status_t check_shape(const ism_attn_shape_t* sh) {
                 sh->num_heads_kv);
   if (sh->head_dim != 64 && sh->head_dim != 128)
     return fail(ISM_ERR_UNSUPPORTED, "head_dim %d (supported: 64, 128)", sh->head_dim);
-  if (sh->dtype != ISM_BF16 && sh->dtype != ISM_FP32) return fail(ISM_ERR_UNSUPPORTED, "dtype %d", sh->dtype);
+  if (sh->dtype == ISM_E4M3) {
+    if (!allow_e4m3) return fail(ISM_ERR_UNSUPPORTED, "e4m3 inputs only in ism_attn_fwd_e4m3");
+    if (sh->head_dim != 128) return fail(ISM_ERR_UNSUPPORTED, "e4m3 needs head_dim 128");
+  } else if (sh->dtype != ISM_BF16 && sh->dtype != ISM_FP32) {
+    return fail(ISM_ERR_UNSUPPORTED, "dtype %d", sh->dtype);
+  }
   if (!(sh->softmax_scale > 0.f) || sh->softmax_scale != sh->softmax_scale)
     return fail(ISM_ERR_INVALID_ARG, "softmax_scale must be a positive number");
   return ISM_OK;
@@ -244,7 +249,9 @@ bool use_tc_bwd(const ism_attn_shape_t* sh) { return use_tc(sh) && tc_bwd_availa
 // odd number of query heads per KV head it pairs neighbouring query tiles of
 // one head instead, from a work list the metadata pass builds.
 bool fwd_tile_pairs(const ism_attn_shape_t* sh) {
-  if (!use_tc(sh) || (sh->num_heads_q / sh->num_heads_kv) % 2 == 0) return false;
+  if ((sh->num_heads_q / sh->num_heads_kv) % 2 == 0) return false;
+  if (sh->dtype == ISM_E4M3) return true;  // the e4m3 forward runs only the paired kernel
+  if (!use_tc(sh)) return false;
   const char* e = getenv("ISM_FWD_ONE_HEAD");
   return !(e && e[0] == '1');
 }
@@ -362,7 +369,7 @@ ism_status_t ism_attn_fwd_workspace_size(const ism_segments_t* segs, const ism_a
   SegInfo info;
   ism_status_t r = check_segments(segs, &info);
   if (r != ISM_OK) return r;
-  if ((r = check_shape(shape)) != ISM_OK) return r;
+  if ((r = check_shape(shape, true)) != ISM_OK) return r;
   if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
   Counts c = count_tiles(segs, kTile, kTile);
   *bytes = pass_layout(nullptr, segs, c, info.total_tokens, shape->num_heads_q, false, 0, fwd_tile_pairs(shape)).bytes;
@@ -428,6 +435,47 @@ ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   } else {
     ISM_TRY_CUDA(launch_simt_fwd(a, st), "forward launch");
   }
+  timer_end(ISM_KERNEL_FWD, st);
+  count_launch(1);
+  return ISM_OK;
+}
+
+ism_status_t ism_attn_fwd_e4m3(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q,
+                               const void* k, const void* v, float q_descale, float k_descale, float v_descale,
+                               void* o, float* lse, void* workspace, size_t workspace_bytes, ism_stream_t stream) {
+  SegInfo info;
+  ism_status_t r = check_segments(segs, &info);
+  if (r != ISM_OK) return r;
+  if ((r = check_shape(shape, true)) != ISM_OK) return r;
+  if (shape->dtype != ISM_E4M3) return fail(ISM_ERR_INVALID_ARG, "ism_attn_fwd_e4m3 needs shape->dtype ISM_E4M3");
+  const float ds[3] = {q_descale, k_descale, v_descale};
+  for (float x : ds)
+    if (!(x > 0.f) || x > 3.0e38f) return fail(ISM_ERR_INVALID_ARG, "descales must be positive finite numbers");
+  if (!tc_available()) return fail(ISM_ERR_UNSUPPORTED, "e4m3 forward needs the sm_103 tensor cores");
+  if (info.total_tokens == 0) return ISM_OK;
+  if (!q || !k || !v || !o) return fail(ISM_ERR_INVALID_ARG, "q, k, v, o must be non-NULL");
+  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || (lse && !aligned16(lse)))
+    return fail(ISM_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  Counts c = count_tiles(segs, kTile, kTile);
+  PassLayout L =
+      pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, false, 0, fwd_tile_pairs(shape));
+  if ((r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
+  uint32_t* status;
+  if ((r = status_ptr(&status)) != ISM_OK) return r;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if ((r = build_pass_meta(segs, c, L, false, st)) != ISM_OK) return r;
+
+  AttnArgs a{};
+  a.q = q; a.k = k; a.v = v; a.out = o; a.lse = lse;
+  a.hq = shape->num_heads_q; a.hkv = shape->num_heads_kv; a.d = shape->head_dim; a.dtype = ISM_E4M3;
+  a.q_rows = info.total_tokens; a.scale = shape->softmax_scale;
+  a.qk_descale = q_descale * k_descale; a.v_descale = v_descale;
+  a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order; a.nq = c.nq;
+  a.pair_order = L.pair_order; a.npairs = L.pair_order ? c.npairs : 0;
+  a.status = status;
+  a.flags = tc_flags();
+  timer_begin(ISM_KERNEL_FWD, st);
+  ISM_TRY_CUDA(launch_tc_fwd(a, info.total_tokens, st), "e4m3 forward launch");
   timer_end(ISM_KERNEL_FWD, st);
   count_launch(1);
   return ISM_OK;
@@ -732,6 +780,18 @@ ism_status_t ism_debug_mma_tile(const void* a, const void* b, float* c, int32_t 
   ism_status_t r = status_ptr(&status);
   if (r != ISM_OK) return r;
   ISM_TRY_CUDA(launch_tc_mma_tile(a, b, c, mode, status, reinterpret_cast<cudaStream_t>(stream)), "mma tile launch");
+  count_launch(1);
+  return ISM_OK;
+}
+
+ism_status_t ism_debug_mma_tile_e4m3(const void* a, const void* b, float* c, int32_t mode, ism_stream_t stream) {
+  if (!a || !b || !c || mode < 0 || mode > 2) return fail(ISM_ERR_INVALID_ARG, "a, b, c non-NULL and mode 0..2");
+  if (!tc_available()) return fail(ISM_ERR_UNSUPPORTED, "tensor-core kernels need an sm_103 device");
+  uint32_t* status;
+  ism_status_t r = status_ptr(&status);
+  if (r != ISM_OK) return r;
+  ISM_TRY_CUDA(tc::launch_mma_tile_e4m3(a, b, c, mode, status, reinterpret_cast<cudaStream_t>(stream)),
+               "e4m3 mma tile launch");
   count_launch(1);
   return ISM_OK;
 }

@@ -24,9 +24,14 @@ namespace {
 
 constexpr int kThreads = 320;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t OFF_QA = 0, OFF_QB = kTileBytes, OFF_K = 2 * kTileBytes, OFF_V = 4 * kTileBytes,
-                   OFF_BAR = 6 * kTileBytes;
-constexpr uint32_t kSmemBytes = OFF_BAR + 256 + 1024;
+// Shared memory: Q_A, Q_B, K ring (2), V ring (2), barriers.  A 128 x 128 tile
+// is 32 KB in bf16 (two 64-column swizzled halves) and 16 KB in e4m3 (one).
+template <bool kE4M3>
+struct PairLayout {
+  static constexpr uint32_t TB = kE4M3 ? 16384u : kTileBytes;
+  static constexpr uint32_t QA = 0, QB = TB, K = 2 * TB, V = 4 * TB, BAR = 6 * TB;
+  static constexpr uint32_t SMEM = BAR + 256 + 1024;
+};
 
 struct Bars {
   uint64_t q_full;
@@ -43,13 +48,18 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 __device__ __forceinline__ bool aborted(const int32_t* f) { return *reinterpret_cast<const volatile int32_t*>(f) != 0; }
 __device__ __forceinline__ void set_abort(int32_t* f) { *reinterpret_cast<volatile int32_t*>(f) = 1; }
 
-template <bool kTilePairs>
+// kE4M3: Q, K, V in e4m3 (kind::f8f6f4 MMAs, K = 32 a step); the scores are
+// scaled by qk_descale, P is rounded to e4m3 for O += P V and O is scaled by
+// v_descale (per-tensor dequantisation factors of the inputs).
+template <bool kTilePairs, bool kE4M3>
 __global__ void __launch_bounds__(kThreads, 1)
     fwd_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                     const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
+  using L = PairLayout<kE4M3>;
+  constexpr uint32_t kTB = L::TB;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  Bars* bar = reinterpret_cast<Bars*>(smem + OFF_BAR);
+  Bars* bar = reinterpret_cast<Bars*>(smem + L::BAR);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   Tile w0, w1;
   int h0, h1, nkb0, nkb1;
@@ -105,17 +115,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ producer (the warp waits
     // converged, lane 0 issues the copies)
     if (nkb > 0) {
+      // one 128 x 128 tile: two 64-column boxes in bf16, one 128-column box in e4m3
+      auto load_tile = [&](uint8_t* dst, const CUtensorMap* map, uint64_t* b, int32_t x, int32_t y) {
+        ptx::tma_load_2d(dst, map, b, x, y);
+        if (!kE4M3) ptx::tma_load_2d(dst + kHalfBytes, map, b, x + 64, y);
+      };
       if (lane == 0) {
         ptx::tma_prefetch_desc(&tmK);
         ptx::tma_prefetch_desc(&tmV);
         const int32_t qy0 = w0.q_base + w0.tile * kRows, qy1 = w1.q_base + w1.tile * kRows;
-        ptx::mbar_expect_tx(&bar->q_full, (nkb1 > 0 ? 2 : 1) * kTileBytes);
-        ptx::tma_load_2d(smem + OFF_QA, &tmQ, &bar->q_full, h0 * kD, qy0);
-        ptx::tma_load_2d(smem + OFF_QA + kHalfBytes, &tmQ, &bar->q_full, h0 * kD + 64, qy0);
-        if (nkb1 > 0) {
-          ptx::tma_load_2d(smem + OFF_QB, &tmQ, &bar->q_full, h1 * kD, qy1);
-          ptx::tma_load_2d(smem + OFF_QB + kHalfBytes, &tmQ, &bar->q_full, h1 * kD + 64, qy1);
-        }
+        ptx::mbar_expect_tx(&bar->q_full, (nkb1 > 0 ? 2 : 1) * kTB);
+        load_tile(smem + L::QA, &tmQ, &bar->q_full, h0 * kD, qy0);
+        if (nkb1 > 0) load_tile(smem + L::QB, &tmQ, &bar->q_full, h1 * kD, qy1);
       }
       __syncwarp();
       uint32_t nk[2] = {0, 0}, nv[2] = {0, 0};
@@ -130,9 +141,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         if (lane == 0) {
-          ptx::mbar_expect_tx(&bar->k_full[s], kTileBytes);
-          ptx::tma_load_2d(smem + OFF_K + s * kTileBytes, &tmK, &bar->k_full[s], g * kD, ky);
-          ptx::tma_load_2d(smem + OFF_K + s * kTileBytes + kHalfBytes, &tmK, &bar->k_full[s], g * kD + 64, ky);
+          ptx::mbar_expect_tx(&bar->k_full[s], kTB);
+          load_tile(smem + L::K + s * kTB, &tmK, &bar->k_full[s], g * kD, ky);
         }
         __syncwarp();
         ++nk[s];
@@ -141,9 +151,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         if (lane == 0) {
-          ptx::mbar_expect_tx(&bar->v_full[s], kTileBytes);
-          ptx::tma_load_2d(smem + OFF_V + s * kTileBytes, &tmV, &bar->v_full[s], g * kD, ky);
-          ptx::tma_load_2d(smem + OFF_V + s * kTileBytes + kHalfBytes, &tmV, &bar->v_full[s], g * kD + 64, ky);
+          ptx::mbar_expect_tx(&bar->v_full[s], kTB);
+          load_tile(smem + L::V + s * kTB, &tmV, &bar->v_full[s], g * kD, ky);
         }
         __syncwarp();
         ++nv[s];
@@ -160,21 +169,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ MMA issuer (the whole
     // warp runs the loop, one elected lane issues each instruction)
     if (nkb > 0) {
-      constexpr uint32_t idesc_qk = ptx::idesc_bf16_f32(128, 128, 0, 0);
-      constexpr uint32_t idesc_pv = ptx::idesc_bf16_f32(128, 128, 0, 1);
-      const uint32_t sQ0 = ptx::smem_u32(smem + OFF_QA);
-      // head x: Q at sQ0 + x * kTileBytes, S at tmem + 256 x, O at tmem + 128 + 256 x
+      constexpr uint32_t idesc_qk = kE4M3 ? ptx::idesc_e4m3_f32(128, 128, 0, 0) : ptx::idesc_bf16_f32(128, 128, 0, 0);
+      constexpr uint32_t idesc_pv = kE4M3 ? ptx::idesc_e4m3_f32(128, 128, 0, 1) : ptx::idesc_bf16_f32(128, 128, 0, 1);
+      const uint32_t sQ0 = ptx::smem_u32(smem + L::QA);
+      // head x: Q at sQ0 + x * kTB, S at tmem + 256 x, O at tmem + 128 + 256 x
       auto issue_s = [&](int x, int j) {
-        const uint32_t sK = ptx::smem_u32(smem + OFF_K + (j & 1) * kTileBytes);
-        const uint32_t sQ = sQ0 + (uint32_t)x * kTileBytes, tS = tmem + 256u * (uint32_t)x;
-        ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128>(tS, desc_kmajor(sQ, 0), desc_kmajor(sK, 0), idesc_qk,
-                                                                  0u);
+        const uint32_t sK = ptx::smem_u32(smem + L::K + (j & 1) * kTB);
+        const uint32_t sQ = sQ0 + (uint32_t)x * kTB, tS = tmem + 256u * (uint32_t)x;
+        if constexpr (kE4M3)  // 128-byte rows: k-steps of 32 bytes
+          ptx::mma4_e4m3_ss_warp<2, 2>(tS, desc_kmajor(sQ, 0), desc_kmajor(sK, 0), idesc_qk, 0u);
+        else
+          ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128>(tS, desc_kmajor(sQ, 0), desc_kmajor(sK, 0),
+                                                                    idesc_qk, 0u);
         ptx::mma_commit_warp(&bar->s_full[x]);
       };
       auto issue_pv = [&](int x, int j) {
-        const uint32_t sV = ptx::smem_u32(smem + OFF_V + (j & 1) * kTileBytes);
+        const uint32_t sV = ptx::smem_u32(smem + L::V + (j & 1) * kTB);
         const uint32_t tS = tmem + 256u * (uint32_t)x, tO = tS + 128u;
-        ptx::mma8_bf16_ts_warp<ptx::TmemPairs, ptx::MnMajorSw128>(tO, tS, desc_mnmajor(sV, 0), idesc_pv, j > 0 ? 1u : 0u);
+        if constexpr (kE4M3)  // P: four e4m3 a column; V MN-major, 32 rows of 128 bytes a k-step
+          ptx::mma4_e4m3_ts_warp<8, 256>(tO, tS, desc_kmajor(sV, 0), idesc_pv, j > 0 ? 1u : 0u);
+        else
+          ptx::mma8_bf16_ts_warp<ptx::TmemPairs, ptx::MnMajorSw128>(tO, tS, desc_mnmajor(sV, 0), idesc_pv,
+                                                                   j > 0 ? 1u : 0u);
         ptx::mma_commit_warp(&bar->pv_done[x]);
       };
       bool ok = wait_warp(&bar->q_full, 0, a.status) && wait_warp(&bar->k_full[0], 0, a.status);
@@ -234,7 +250,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row = wm.tile * kRows + r;
     const bool valid = row < wm.q_len;
     const int ke = a.kv_end[wm.kv_base + (valid ? row : wm.q_len - 1)];
-    const float sl2 = a.scale * kLog2e;
+    const float sl2 = a.scale * kLog2e * (kE4M3 ? a.qk_descale : 1.f);
     float m_use = -INFINITY, l = 0.f;
     bool ok = nkbm > 0;
     for (int j = 0; ok && j < nkbm; ++j) {
@@ -295,17 +311,32 @@ __global__ void __launch_bounds__(kThreads, 1)
       // P over the first 64 columns of S (already read), 32 columns at a time
       float2 rsv[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
       const float2 sl2x2 = make_float2(sl2, sl2), negm = make_float2(-m_use, -m_use);
-#pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {
+      if constexpr (kE4M3) {
+        // P as e4m3 over the first 32 columns of S: column c holds keys 4c .. 4c + 3
         uint32_t pk[32];
 #pragma unroll
         for (int c = 0; c < 32; ++c) {
-          const float2 arg = fma2(make_float2(xs[64 * hf + 2 * c], xs[64 * hf + 2 * c + 1]), sl2x2, negm);
-          const float2 pr = make_float2(ex2(arg.x), ex2(arg.y));
-          rsv[c & 1] = add2(rsv[c & 1], pr);
-          pk[c] = pack_bf16(pr.x, pr.y);
+          const float2 a01 = fma2(make_float2(xs[4 * c], xs[4 * c + 1]), sl2x2, negm);
+          const float2 a23 = fma2(make_float2(xs[4 * c + 2], xs[4 * c + 3]), sl2x2, negm);
+          const float2 p01 = make_float2(ex2(a01.x), ex2(a01.y)), p23 = make_float2(ex2(a23.x), ex2(a23.y));
+          rsv[0] = add2(rsv[0], p01);
+          rsv[1] = add2(rsv[1], p23);
+          pk[c] = pack_e4m3x4(p01.x, p01.y, p23.x, p23.y);
         }
-        ptx::tmem_st32(tS + 32 * hf, pk);
+        ptx::tmem_st32(tS, pk);
+      } else {
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {
+          uint32_t pk[32];
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            const float2 arg = fma2(make_float2(xs[64 * hf + 2 * c], xs[64 * hf + 2 * c + 1]), sl2x2, negm);
+            const float2 pr = make_float2(ex2(arg.x), ex2(arg.y));
+            rsv[c & 1] = add2(rsv[c & 1], pr);
+            pk[c] = pack_bf16(pr.x, pr.y);
+          }
+          ptx::tmem_st32(tS + 32 * hf, pk);
+        }
       }
       l += (rsv[0].x + rsv[0].y) + (rsv[1].x + rsv[1].y);
       ptx::tmem_st_wait();
@@ -317,7 +348,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (nkbm > 0) set_abort(&bar->abort);  // a unit without key blocks has nothing to write
     } else {
       ptx::tc_fence_after();
-      const float inv = 1.f / l;
+      const float inv = (kE4M3 ? a.v_descale : 1.f) / l;
       const int64_t orow = (int64_t)wm.q_base + row;
       uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.out) + orow * a.hq * kD + h * kD);
 #pragma unroll 1
@@ -349,19 +380,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+template <bool kE4M3>
+cudaError_t launch_fwd_pair_t(const AttnArgs& a, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
+                              cudaStream_t st) {
+  cudaError_t e;
+  const bool tile_pairs = a.pair_order != nullptr;
+  auto kern = tile_pairs ? fwd_pair_kernel<true, kE4M3> : fwd_pair_kernel<false, kE4M3>;
+  constexpr uint32_t smem = PairLayout<kE4M3>::SMEM;
+  if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
+    return e;
+  const int64_t grid = tile_pairs ? a.npairs * a.hq : a.nq * (a.hq / 2);
+  if (grid == 0) return cudaSuccess;
+  kern<<<(unsigned)grid, kThreads, smem, st>>>(tq, tk, tv, a);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_fwd_pair(const AttnArgs& a, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             cudaStream_t st) {
-  cudaError_t e;
-  const bool tile_pairs = a.pair_order != nullptr;
-  auto kern = tile_pairs ? fwd_pair_kernel<true> : fwd_pair_kernel<false>;
-  if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) != cudaSuccess)
-    return e;
-  const int64_t grid = tile_pairs ? a.npairs * a.hq : a.nq * (a.hq / 2);
-  if (grid == 0) return cudaSuccess;
-  kern<<<(unsigned)grid, kThreads, kSmemBytes, st>>>(tq, tk, tv, a);
-  return cudaGetLastError();
+  return a.dtype == ISM_E4M3 ? launch_fwd_pair_t<true>(a, tq, tk, tv, st) : launch_fwd_pair_t<false>(a, tq, tk, tv, st);
 }
 
 }  // namespace tc

@@ -498,10 +498,30 @@ cudaError_t make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t cols, uint
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
+// 2D e4m3 tensor map [rows, cols] with a 128 x 128 box (128-byte rows), 128B swizzle.
+cudaError_t make_tmap_e4m3(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return cudaErrorNotSupported;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols};
+  cuuint32_t box[2] = {128, 128};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box, es,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 cudaError_t launch_fwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) {
   if (a.nq == 0) return cudaSuccess;
   CUtensorMap tq, tk, tv;
   cudaError_t e;
+  if (a.dtype == ISM_E4M3) {  // only the paired kernel has the e4m3 form
+    if ((e = make_tmap_e4m3(&tq, a.q, (uint64_t)a.hq * kD, (uint64_t)a.q_rows)) != cudaSuccess) return e;
+    if ((e = make_tmap_e4m3(&tk, a.k, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;
+    if ((e = make_tmap_e4m3(&tv, a.v, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;
+    return launch_fwd_pair(a, tq, tk, tv, st);
+  }
   if ((e = make_tmap_bf16(&tq, a.q, (uint64_t)a.hq * kD, (uint64_t)a.q_rows)) != cudaSuccess) return e;
   if ((e = make_tmap_bf16(&tk, a.k, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;
   if ((e = make_tmap_bf16(&tv, a.v, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;

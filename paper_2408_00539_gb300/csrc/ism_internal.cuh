@@ -125,6 +125,9 @@ struct AttnArgs {
   // Paged K/V (forward over an appended chunk only): Tile::k_base holds the
   // sequence index and key p's row is paged_row(pages, k_base, p).
   KvPages pages;
+  // e4m3 forward: per-tensor dequantisation factors (scores scaled by
+  // q_descale * k_descale, the output by v_descale).
+  float qk_descale, v_descale;
   // Bit 0: before an MMA that overwrites tensor memory an earlier MMA reads
   // as its A operand, wait for that earlier MMA to complete.  Clear: rely on
   // MMAs issued by one thread executing in issue order.
@@ -159,6 +162,9 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st);
 bool tc_available();
 bool tc_bwd_available();
 cudaError_t launch_tc_mma_tile(const void* a, const void* b, float* c, int mode, uint32_t* status, cudaStream_t st);
+namespace tc {
+cudaError_t launch_mma_tile_e4m3(const void* a, const void* b, float* c, int mode, uint32_t* status, cudaStream_t st);
+}
 cudaError_t launch_tc_fwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st);
 cudaError_t launch_tc_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st);
 

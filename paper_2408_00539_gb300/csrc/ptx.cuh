@@ -315,5 +315,59 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t m, uint32_t n, ui
          | ((m >> 4) << 24);  // M / 16
 }
 
+// Instruction descriptor for kind::f8f6f4 with e4m3 A/B and fp32 D (K = 32 a step).
+__host__ __device__ constexpr uint32_t idesc_e4m3_f32(uint32_t m, uint32_t n, uint32_t a_mn, uint32_t b_mn) {
+  return (1u << 4)            // D format: f32
+         | (0u << 7)          // A format: e4m3
+         | (0u << 10)         // B format: e4m3
+         | (a_mn << 15)       // A major
+         | (b_mn << 16)       // B major
+         | ((n >> 3) << 17)   // N / 8
+         | ((m >> 4) << 24);  // M / 16
+}
+
+// The four k-steps (K = 128 in steps of 32) of one 128 x N e4m3 contraction
+// (kind::f8f6f4), issued like mma8_bf16_*_warp: one elected lane, k-step kk
+// at the first operands plus kk * kStep.  Layouts (kStep):
+//   K-major, 128-byte swizzled, 128-byte rows:  2 (32 bytes)
+//   MN-major, 128-byte swizzled, 128-byte rows: 256 (32 rows of 128 bytes)
+//   e4m3 quads in tensor memory:                8 columns
+template <uint32_t kAStep, uint32_t kBStep>
+__device__ __forceinline__ void mma4_e4m3_ss_warp(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                                  uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred e, p, t;\n .reg .b64 a1, a2, a3, b1, b2, b3;\n"
+      " elect.sync _|e, 0xffffffff;\n @!e bra MMA4_SS_DONE;\n"
+      " setp.ne.b32 p, %4, 0;\n setp.eq.u32 t, 0, 0;\n"
+      " add.s64 a1, %1, %5; add.s64 a2, %1, %6; add.s64 a3, %1, %7;\n"
+      " add.s64 b1, %2, %8; add.s64 b2, %2, %9; add.s64 b3, %2, %10;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %1, %2, %3, p;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], a1, b1, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], a2, b2, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], a3, b3, %3, t;\n"
+      " MMA4_SS_DONE:\n}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(acc), "n"(kAStep), "n"(2 * kAStep), "n"(3 * kAStep), "n"(kBStep),
+      "n"(2 * kBStep), "n"(3 * kBStep)
+      : "memory");
+}
+template <uint32_t kAStep, uint32_t kBStep>
+__device__ __forceinline__ void mma4_e4m3_ts_warp(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                                  uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred e, p, t;\n .reg .b32 a1, a2, a3;\n .reg .b64 b1, b2, b3;\n"
+      " elect.sync _|e, 0xffffffff;\n @!e bra MMA4_TS_DONE;\n"
+      " setp.ne.b32 p, %4, 0;\n setp.eq.u32 t, 0, 0;\n"
+      " add.u32 a1, %1, %5; add.u32 a2, %1, %6; add.u32 a3, %1, %7;\n"
+      " add.s64 b1, %2, %8; add.s64 b2, %2, %9; add.s64 b3, %2, %10;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [%1], %2, %3, p;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [a1], b1, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [a2], b2, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], [a3], b3, %3, t;\n"
+      " MMA4_TS_DONE:\n}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(acc), "n"(kAStep), "n"(2 * kAStep), "n"(3 * kAStep), "n"(kBStep),
+      "n"(2 * kBStep), "n"(3 * kBStep)
+      : "memory");
+}
+
 }  // namespace ptx
 }  // namespace ism

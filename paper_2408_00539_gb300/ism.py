@@ -17,7 +17,7 @@ import torch
 
 from . import build as _build
 
-ISM_BF16, ISM_FP32 = 0, 1
+ISM_BF16, ISM_FP32, ISM_E4M3 = 0, 1, 2
 QUERY, ANSWER = 0, 1
 TILE_EMPTY, TILE_FULL, TILE_PARTIAL = 0, 1, 2
 
@@ -49,6 +49,7 @@ EXPORTS = {
     "ism_build_tile_map": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32] + [C.c_void_p] * 6),
     "ism_attn_fwd_workspace_size": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "ism_attn_fwd": (C.c_int, [C.c_void_p] * 8 + [C.c_size_t, C.c_void_p]),
+    "ism_attn_fwd_e4m3": (C.c_int, [C.c_void_p] * 5 + [C.c_float] * 3 + [C.c_void_p] * 3 + [C.c_size_t, C.c_void_p]),
     "ism_attn_bwd_workspace_size": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "ism_attn_bwd_workspace_size_min": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "ism_attn_bwd": (C.c_int, [C.c_void_p] * 12 + [C.c_size_t, C.c_void_p]),
@@ -70,6 +71,7 @@ EXPORTS = {
     "ism_set_kernel_timer": (C.c_int, [C.c_int32, C.c_void_p, C.c_void_p]),
     "ism_kernel_launches": (C.c_uint64, []),
     "ism_debug_mma_tile": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p]),
+    "ism_debug_mma_tile_e4m3": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p]),
     "ism_attn_fwd_noalloc_max_workspace": (C.c_size_t, []),
     "ism_attn_fwd_noalloc": (C.c_int, [C.c_void_p] * 8),
 }
@@ -120,6 +122,8 @@ def _dtype_code(t: torch.Tensor) -> int:
         return ISM_BF16
     if t.dtype == torch.float32:
         return ISM_FP32
+    if t.dtype == torch.float8_e4m3fn:
+        return ISM_E4M3
     raise TypeError(f"unsupported dtype {t.dtype}")
 
 
@@ -220,6 +224,29 @@ def fwd(segs: Segments, q, k, v, softmax_scale: float, out=None, lse=None, works
         workspace = _workspace(nbytes.value, q.device)
     _check(lib.ism_attn_fwd(C.byref(s), C.byref(sh), _ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(lse),
                             _ptr(workspace), workspace.numel(), _stream(q.device)), "ism_attn_fwd")
+    return out, lse
+
+
+def fwd_e4m3(segs: Segments, q, k, v, q_descale: float, k_descale: float, v_descale: float, softmax_scale: float,
+             out=None, lse=None, workspace=None):
+    """Forward with e4m3 inputs (torch.float8_e4m3fn; head_dim 128): the
+    attention of q * q_descale, k * k_descale, v * v_descale.  Returns
+    (o bf16 [T,Hq,D], lse [Hq,T])."""
+    lib = load()
+    _contig(q, k, v)
+    T, hq, D = q.shape
+    s, sh = segs.struct(), _shape(q, k, softmax_scale)
+    nbytes = C.c_size_t()
+    _check(lib.ism_attn_fwd_workspace_size(C.byref(s), C.byref(sh), C.byref(nbytes)), "ism_attn_fwd_workspace_size")
+    if out is None:
+        out = torch.empty(q.shape, dtype=torch.bfloat16, device=q.device)
+    if lse is None:
+        lse = torch.empty((hq, T), dtype=torch.float32, device=q.device)
+    if workspace is None or workspace.numel() < nbytes.value:
+        workspace = _workspace(nbytes.value, q.device)
+    _check(lib.ism_attn_fwd_e4m3(C.byref(s), C.byref(sh), _ptr(q), _ptr(k), _ptr(v), q_descale, k_descale, v_descale,
+                                 _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(), _stream(q.device)),
+           "ism_attn_fwd_e4m3")
     return out, lse
 
 
@@ -342,6 +369,15 @@ def prefill_append_paged(q_new, k_new, v_new, k_pool, v_pool, page_size: int, bl
                                              _ptr(workspace), workspace.numel(), _stream(q_new.device)),
            "ism_attn_prefill_append_paged")
     return out, lse
+
+
+def debug_mma_tile_e4m3(a: torch.Tensor, b: torch.Tensor, mode: int) -> torch.Tensor:
+    """One 128x128x128 e4m3 tcgen05 tile product (diagnostic): mode 0 a @ b.T,
+    mode 1 a @ b, mode 2 a @ b with a in tensor memory; a, b float8_e4m3fn."""
+    c = torch.empty((128, 128), dtype=torch.float32, device=a.device)
+    _check(load().ism_debug_mma_tile_e4m3(_ptr(a), _ptr(b), _ptr(c), mode, _stream(a.device)),
+           "ism_debug_mma_tile_e4m3")
+    return c
 
 
 def check_status(device=None):

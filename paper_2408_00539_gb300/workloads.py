@@ -290,6 +290,17 @@ def attention_tensors(w: Workload, with_dout: bool = True, seed_offset: int = 0)
     return tuple(out)
 
 
+def quantize_e4m3(x):
+    """Per-tensor e4m3 (float8_e4m3fn) copy of a torch tensor: the values are
+    scaled so that the largest magnitude maps to 448, the format's largest
+    finite value, and rounded to nearest.  Returns (x8, descale) with
+    x ~= x8.float() * descale."""
+    import torch
+    amax = float(x.float().abs().max())
+    descale = amax / 448.0 if amax > 0 else 1.0
+    return (x.float() / descale).to(torch.float8_e4m3fn), descale
+
+
 def random_dialogue_set(rng: np.random.Generator, n_seqs: int, max_len: int,
                         zero_len: bool = True, min_len: int = 1) -> Segments:
     """Small random segmentations for tests: any mix of QUERY/ANSWER

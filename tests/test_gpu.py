@@ -517,3 +517,67 @@ def test_paged_append_rejects_bad_tables(ism):
         ism.prefill_append_paged(*args, 64, torch.from_numpy(table).to(DEV), table, cl, c_lens, [8], [0], d ** -0.5)
     ism.check_status()
     assert cl.cpu().numpy().tolist() == c_lens.tolist()  # nothing ran
+
+
+# ---------------------------------------------------------------- e4m3 forward
+
+def _e4m3_pass(ism, w):
+    """e4m3 copies of the workload's Q, K, V (per-tensor scales), the GPU
+    forward on them, and their exact dequantised values for the oracle."""
+    q, k, v, _ = wl.attention_tensors(w)
+    (q8, qs), (k8, ks), (v8, vs) = (wl.quantize_e4m3(t) for t in (q, k, v))
+    segs = ism.Segments.from_workload(w.segs, DEV)
+    o, lse = ism.fwd_e4m3(segs, q8.to(DEV), k8.to(DEV), v8.to(DEV), qs, ks, vs, w.softmax_scale)
+    ism.check_status()
+    deq = [t.double() * s for t, s in ((q8, qs), (k8, ks), (v8, vs))]
+    return deq, o, lse
+
+
+def _cmp_e4m3(name, got, ref, vmax):
+    """P is rounded to e4m3 for O = P V / l (relative error at most 2^-4 per
+    term), O to bf16 (2^-9): |O - O_ref| <= (2^-4 + 2^-9) max|V| bounds every
+    element; the errors are independent across keys, so their mean is far
+    smaller (mean-abs 4e-3, twice the bf16 bound)."""
+    got = _np(got)
+    assert np.all(np.isfinite(got)), f"{name}: non-finite values"
+    err = np.abs(got - ref)
+    assert err.max() <= (2 ** -4 + 2 ** -9) * vmax, f"{name}: max abs err {err.max():.3e} (max|V| {vmax:.3f})"
+    assert err.mean() <= 4e-3, f"{name}: mean abs err {err.mean():.3e}"
+
+
+@pytest.mark.parametrize("hq,hkv", [(8, 2), (3, 3), (6, 2)])
+def test_small_e4m3_fwd(ism, hq, hkv):
+    """Paired heads (even group) and paired query tiles (odd group sizes)."""
+    w = _small_bf16(128, hq=hq, hkv=hkv, seed=50 + hq)
+    (q, k, v), o, lse = _e4m3_pass(ism, w)
+    o_ref, lse_ref = orc.attn_fwd(q, k, v, w.segs, w.softmax_scale)
+    _cmp_e4m3("o", o, o_ref, float(v.abs().max()))
+    _cmp_lse("lse", lse, lse_ref, "bf16")
+
+
+@pytest.mark.parametrize("make", [wl.gqa_8k, wl.mha_4k], ids=["gqa_8k", "mha_4k"])
+def test_full_size_e4m3_fwd_sampled_group(ism, make):
+    w = make()
+    (q, k, v), o, lse = _e4m3_pass(ism, w)
+    b = _largest_seq(w.segs)
+    t0, L, se, st = w.segs.seq(b)
+    grp = w.num_heads_q // w.num_heads_kv
+    g = 1 if w.num_heads_kv > 1 else 0
+    hs = slice(g * grp, (g + 1) * grp)
+    sl = slice(t0, t0 + L)
+    o_ref, lse_ref = orc.attn_fwd(q[sl][:, hs], k[sl][:, g:g + 1], v[sl][:, g:g + 1], wl.pack([(se, st)]),
+                                  w.softmax_scale)
+    _cmp_e4m3("o", o[sl][:, hs], o_ref, float(v.abs().max()))
+    _cmp_lse("lse", lse[hs][:, sl], lse_ref, "bf16")
+
+
+def test_e4m3_rejects_other_entry_points(ism):
+    w = _small_bf16(128)
+    q, k, v, _ = wl.attention_tensors(w)
+    q8, k8, v8 = (wl.quantize_e4m3(t)[0].to(DEV) for t in (q, k, v))
+    segs = ism.Segments.from_workload(w.segs, DEV)
+    with pytest.raises(ism.IsmError):  # e4m3 only through ism_attn_fwd_e4m3
+        ism.fwd(segs, q8, k8, v8, w.softmax_scale)
+    with pytest.raises(ism.IsmError):  # descales must be positive
+        ism.fwd_e4m3(segs, q8, k8, v8, 0.0, 1.0, 1.0, w.softmax_scale)
+    ism.check_status()

@@ -33,3 +33,17 @@ def test_mma_tile(ism, mode):
         ref = a.double() @ (b.double().T if mode % 2 == 0 else b.double())
     err = (c.double().cpu() - ref).abs().max().item()
     assert err < 1e-3, f"mode {mode}: max abs err {err}"
+
+
+@pytest.mark.parametrize("mode", [0, 1, 2])
+def test_mma_tile_e4m3(ism, mode):
+    """The e4m3 operand layouts (kind::f8f6f4): K-major A and B, MN-major B, A in
+    tensor memory; e4m3 products are exact in the fp32 accumulator."""
+    g = torch.Generator().manual_seed(200 + mode)
+    a = (torch.randn(128, 128, generator=g) * 2).to(torch.float8_e4m3fn)
+    b = (torch.randn(128, 128, generator=g) * 2).to(torch.float8_e4m3fn)
+    c = ism.debug_mma_tile_e4m3(a.cuda(), b.cuda(), mode)
+    ism.check_status()
+    ref = a.double() @ (b.double().T if mode == 0 else b.double())
+    err = (c.double().cpu() - ref).abs().max().item()
+    assert err < 1e-4 * ref.abs().max().item(), f"mode {mode}: max abs err {err}"
