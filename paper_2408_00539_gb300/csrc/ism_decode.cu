@@ -58,10 +58,17 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
   const __nv_bfloat16* Vc = (const __nv_bfloat16*)a.v_cache;
   const int64_t kstride = (int64_t)a.hkv * D;
 
+  // G is the group size padded to a power of two: heads h >= grp are zero and not written
+  const int grp = a.group;
   float q[G][DPL];
 #pragma unroll
   for (int h = 0; h < G; ++h) {
-    unpack_bf16<DPL>(*reinterpret_cast<const Raw*>(Q + ((int64_t)b * hq + g * G + h) * D + lane * DPL), q[h]);
+    if (h < grp) {
+      unpack_bf16<DPL>(*reinterpret_cast<const Raw*>(Q + ((int64_t)b * hq + g * grp + h) * D + lane * DPL), q[h]);
+    } else {
+#pragma unroll
+      for (int i = 0; i < DPL; ++i) q[h][i] = 0.f;
+    }
 #pragma unroll
     for (int i = 0; i < DPL; ++i) q[h][i] *= qscale;
   }
@@ -156,7 +163,7 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
 #pragma unroll
     for (int i = 0; i < DPL; ++i) sm_o[warp][h][lane * DPL + i] = o[h][i];
   __syncthreads();
-  for (int idx = threadIdx.x; idx < G * D; idx += blockDim.x) {
+  for (int idx = threadIdx.x; idx < grp * D; idx += blockDim.x) {
     const int h = idx / D, d = idx % D;
     float M = -INFINITY;
 #pragma unroll
@@ -170,7 +177,7 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
         lsum = fmaf(sm_l[w][h], f, lsum);
       }
     }
-    const int64_t pidx = ((int64_t)b * hq + g * G + h) * a.splits + split;
+    const int64_t pidx = ((int64_t)b * hq + g * grp + h) * a.splits + split;
     a.part_o[pidx * D + d] = acc;
     if (d == 0) { a.part_ml[pidx * 2] = M; a.part_ml[pidx * 2 + 1] = lsum; }
   }
@@ -246,7 +253,13 @@ __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__
     float q[G][DPL];
 #pragma unroll
     for (int h = 0; h < G; ++h) {
-      unpack_bf16<DPL>(*reinterpret_cast<const uint2*>(Q + ((int64_t)b * a.hq + g * G + h) * D + lane * DPL), q[h]);
+      if (h < a.group) {
+        unpack_bf16<DPL>(*reinterpret_cast<const uint2*>(Q + ((int64_t)b * a.hq + g * a.group + h) * D + lane * DPL),
+                         q[h]);
+      } else {
+#pragma unroll
+        for (int i = 0; i < DPL; ++i) q[h][i] = 0.f;
+      }
 #pragma unroll
       for (int i = 0; i < DPL; ++i) q[h][i] *= qscale;
     }
@@ -335,7 +348,7 @@ __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__
       for (int i = 0; i < DPL; ++i) sm_o[(warp * G + h) * D + lane * DPL + i] = o[h][i];
   }
   __syncthreads();
-  for (int idx = threadIdx.x; idx < G * D; idx += blockDim.x) {
+  for (int idx = threadIdx.x; idx < a.group * D; idx += blockDim.x) {
     const int h = idx / D, d = idx % D;
     float M = -INFINITY;
 #pragma unroll
@@ -349,7 +362,7 @@ __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__
         lsum = fmaf(sm_l[w * G + h], f, lsum);
       }
     }
-    const int64_t pidx = ((int64_t)b * a.hq + g * G + h) * a.splits + split;
+    const int64_t pidx = ((int64_t)b * a.hq + g * a.group + h) * a.splits + split;
     a.part_o[pidx * D + d] = acc;
     if (d == 0) { a.part_ml[pidx * 2] = M; a.part_ml[pidx * 2 + 1] = lsum; }
   }
@@ -404,15 +417,16 @@ cudaError_t run(const DecodeArgs& a, cudaStream_t st) {
   return cudaGetLastError();
 }
 
+// the kernels take the group size padded to a power of two (a batch of 32 / G keys)
 template <int D>
 cudaError_t run_d(const DecodeArgs& a, cudaStream_t st) {
-  switch (a.hq / a.hkv) {
-    case 1: return run<D, 1>(a, st);
-    case 2: return run<D, 2>(a, st);
-    case 4: return run<D, 4>(a, st);
-    case 8: return run<D, 8>(a, st);
-    default: return cudaErrorInvalidValue;
-  }
+  const int grp = a.group;
+  if (grp <= 1) return run<D, 1>(a, st);
+  if (grp <= 2) return run<D, 2>(a, st);
+  if (grp <= 4) return run<D, 4>(a, st);
+  if (grp <= 8) return run<D, 8>(a, st);
+  if (grp <= 16) return run<D, 16>(a, st);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace

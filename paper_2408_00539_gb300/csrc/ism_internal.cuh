@@ -147,6 +147,7 @@ struct DecodeArgs {
   float* lse;            // [Hq, B] or null
   const int32_t* c_snap; // cache length before the append, per sequence
   int32_t batch, hq, hkv, d, dtype;
+  int32_t group;         // query heads per KV head (the kernels pad it to a power of two)
   int64_t cap;
   int64_t kv_rows;       // rows of the K / V tensors: batch * cap, or pages * page_size
   float scale;
