@@ -238,6 +238,27 @@ ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batc
                                      void* workspace, size_t workspace_bytes, ism_stream_t stream);
 
 /* ---------------------------------------------------------------------------
+ * Append-prefill and decode with e4m3 (fp8) queries and KV caches: the
+ * operation of ism_attn_prefill_append on q * q_descale, k * k_descale,
+ * v * v_descale, where k_descale / v_descale are the factors of the whole
+ * cache (the caller quantises k_new / v_new with them).  shape->dtype must be
+ * ISM_E4M3, head_dim 128.  q_new, k_new, v_new and the caches are e4m3;
+ * o_new is bf16 [B, l_new, Hq, 128]; lse_new [Hq, B, l_new] fp32 or NULL.
+ * The attention runs on the fp8 tensor cores (the kernel of
+ * ism_attn_fwd_e4m3; P rounded to e4m3), including single-token steps.
+ * Workspace: ism_attn_prefill_append_workspace_size with the same shape.
+ * ------------------------------------------------------------------------- */
+ism_status_t ism_attn_prefill_append_e4m3(const ism_attn_shape_t* shape, int32_t batch,
+                                          const void* q_new, const void* k_new, const void* v_new,
+                                          int32_t l_new, const int32_t* new_seg_end_host,
+                                          const uint8_t* new_seg_type_host, int32_t n_new_segs,
+                                          void* k_cache, void* v_cache, int64_t cache_capacity,
+                                          int32_t* cache_len, const int32_t* cache_len_host,
+                                          float q_descale, float k_descale, float v_descale,
+                                          void* o_new, float* lse_new,
+                                          void* workspace, size_t workspace_bytes, ism_stream_t stream);
+
+/* ---------------------------------------------------------------------------
  * Append-prefill and decode against a paged KV cache: the same operation as
  * ism_attn_prefill_append (Section 2.3, Eq. fj on the new chunk, every cached
  * key visible), with the keys and values of sequence b kept in fixed-size

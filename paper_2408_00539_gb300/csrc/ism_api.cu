@@ -535,6 +535,8 @@ struct AppendLayout {
   int32_t* kv_end;
   Tile* qtiles;
   int32_t* q_order;
+  int32_t* pair_order;  // neighbouring q-tiles of a chunk, for the paired forward
+  int64_t npairs;
   float* part_o;
   float* part_ml;
   size_t bytes;
@@ -543,11 +545,14 @@ struct AppendLayout {
 AppendLayout append_layout(void* ws, const ism_attn_shape_t* sh, int batch, int l_new) {
   Carve cv(ws);
   AppendLayout L;
-  int64_t nqt = (int64_t)batch * ((l_new + kTile - 1) / kTile);
+  const int64_t nqt_seq = (l_new + kTile - 1) / kTile;
+  int64_t nqt = (int64_t)batch * nqt_seq;
   L.c_snap = cv.take<int32_t>(batch);
   L.kv_end = cv.take<int32_t>((int64_t)batch * l_new);
   L.qtiles = cv.take<Tile>(nqt);
   L.q_order = cv.take<int32_t>(nqt);
+  L.npairs = (int64_t)batch * ((nqt_seq + 1) / 2);
+  L.pair_order = cv.take<int32_t>(L.npairs);
   if (l_new == 1) {
     L.part_o = cv.take<float>((int64_t)batch * sh->num_heads_q * kMaxSplits * sh->head_dim);
     L.part_ml = cv.take<float>((int64_t)batch * sh->num_heads_q * kMaxSplits * 2);
@@ -562,11 +567,11 @@ AppendLayout append_layout(void* ws, const ism_attn_shape_t* sh, int batch, int 
 
 ism_status_t ism_attn_prefill_append_workspace_size(const ism_attn_shape_t* shape, int32_t batch, int32_t l_new,
                                                     size_t* bytes) {
-  ism_status_t r = check_shape(shape);
+  ism_status_t r = check_shape(shape, true);
   if (r != ISM_OK) return r;
   if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
   if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
-  *bytes = append_layout(nullptr, shape, batch, l_new).bytes;
+  *bytes = append_layout(nullptr, shape, batch, l_new).bytes;  // (e4m3 shapes included)
   return ISM_OK;
 }
 
@@ -588,7 +593,8 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
                          const void* v_new, int32_t l_new, const int32_t* new_seg_end_host,
                          const uint8_t* new_seg_type_host, int32_t n_new_segs, void* k_cache, void* v_cache,
                          const CacheGeom& cg, int32_t* cache_len, const int32_t* cache_len_host, void* o_new,
-                         float* lse_new, void* workspace, size_t workspace_bytes, cudaStream_t st) {
+                         float* lse_new, void* workspace, size_t workspace_bytes, cudaStream_t st,
+                         float qk_descale = 1.f, float v_descale = 1.f) {
   ism_status_t r;
   if (!q_new || !k_new || !v_new || !k_cache || !v_cache || !cache_len || !cache_len_host || !o_new)
     return fail(ISM_ERR_INVALID_ARG, "q_new, k_new, v_new, caches, cache_len (device+host), o_new must be non-NULL");
@@ -628,7 +634,7 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
 
   timer_begin(ISM_KERNEL_META, st);
   ISM_TRY_CUDA(launch_append_plan(sg, batch, paged ? 1 : cg.cap, kTile, kTile, cache_len, L.c_snap, L.kv_end, L.qtiles,
-                                  L.q_order, st),
+                                  L.q_order, L.pair_order, st),
                "append plan launch");
   ISM_TRY_CUDA(launch_cache_write(shape->dtype, batch, l_new, hkv, d, cg.cap, cg.pages, L.c_snap, k_new, v_new,
                                   k_cache, v_cache, st),
@@ -677,10 +683,19 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
   a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order;
   a.nq = (int64_t)batch * ((l_new + kTile - 1) / kTile);
   a.pages = cg.pages;
+  if (shape->dtype == ISM_E4M3) {
+    // the e4m3 forward is the paired kernel: neighbouring q-tiles for an odd group
+    a.qk_descale = qk_descale;
+    a.v_descale = v_descale;
+    if ((hq / hkv) % 2) {
+      a.pair_order = L.pair_order;
+      a.npairs = L.npairs;
+    }
+  }
   a.status = status;
   a.flags = tc_flags();
   timer_begin(ISM_KERNEL_FWD, st);
-  if (use_tc(shape)) {
+  if (use_tc(shape) || shape->dtype == ISM_E4M3) {
     ISM_TRY_CUDA(launch_tc_fwd(a, cg.kv_rows, st), "tensor-core prefill launch");
   } else {
     ISM_TRY_CUDA(launch_simt_fwd(a, st), "prefill launch");
@@ -715,6 +730,34 @@ ism_status_t ism_attn_prefill_append(const ism_attn_shape_t* shape, int32_t batc
   return append_impl(shape, batch, q_new, k_new, v_new, l_new, new_seg_end_host, new_seg_type_host, n_new_segs,
                      k_cache, v_cache, cg, cache_len, cache_len_host, o_new, lse_new, workspace, workspace_bytes,
                      reinterpret_cast<cudaStream_t>(stream));
+}
+
+ism_status_t ism_attn_prefill_append_e4m3(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,
+                                          const void* k_new, const void* v_new, int32_t l_new,
+                                          const int32_t* new_seg_end_host, const uint8_t* new_seg_type_host,
+                                          int32_t n_new_segs, void* k_cache, void* v_cache, int64_t cache_capacity,
+                                          int32_t* cache_len, const int32_t* cache_len_host, float q_descale,
+                                          float k_descale, float v_descale, void* o_new, float* lse_new,
+                                          void* workspace, size_t workspace_bytes, ism_stream_t stream) {
+  ism_status_t r = check_shape(shape, true);
+  if (r != ISM_OK) return r;
+  if (shape->dtype != ISM_E4M3) return fail(ISM_ERR_INVALID_ARG, "ism_attn_prefill_append_e4m3 needs ISM_E4M3");
+  const float ds[3] = {q_descale, k_descale, v_descale};
+  for (float x : ds)
+    if (!(x > 0.f) || x > 3.0e38f) return fail(ISM_ERR_INVALID_ARG, "descales must be positive finite numbers");
+  if (!tc_available()) return fail(ISM_ERR_UNSUPPORTED, "e4m3 attention needs the sm_103 tensor cores");
+  if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
+  if (batch == 0 || l_new == 0) return ISM_OK;
+  if (cache_capacity <= 0 || (int64_t)batch * cache_capacity >= (int64_t(1) << 31))
+    return fail(ISM_ERR_INVALID_ARG, "batch * cache_capacity must be in (0, 2^31)");
+  CacheGeom cg;
+  cg.cap = cache_capacity;
+  cg.kv_rows = (int64_t)batch * cache_capacity;
+  cg.max_keys = cache_capacity;
+  cg.pages = KvPages{nullptr, 0, 0};
+  return append_impl(shape, batch, q_new, k_new, v_new, l_new, new_seg_end_host, new_seg_type_host, n_new_segs,
+                     k_cache, v_cache, cg, cache_len, cache_len_host, o_new, lse_new, workspace, workspace_bytes,
+                     reinterpret_cast<cudaStream_t>(stream), q_descale * k_descale, v_descale);
 }
 
 ism_status_t ism_attn_prefill_append_paged(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,

@@ -90,7 +90,7 @@ cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, 
 // k_base of sequence b's tiles = b * kbase_stride (the cache capacity, or 1 for a paged cache)
 cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t kbase_stride, int bm, int bn,
                                int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
-                               int32_t* q_order, cudaStream_t st);
+                               int32_t* q_order, int32_t* pair_order, cudaStream_t st);
 cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap, const KvPages& pages,
                                const int32_t* c_snap, const void* k_new, const void* v_new,
                                void* k_cache, void* v_cache, cudaStream_t st);

@@ -281,7 +281,7 @@ __device__ __forceinline__ int32_t chunk_kv_end(const AppendSegs& sg, int32_t j)
 // the chunk) and one q-tile descriptor per (sequence, chunk tile).
 __global__ void append_plan_kernel(AppendSegs sg, int batch, int64_t kbase_stride, int bm, int bn,
                                    int32_t* cache_len, int32_t* c_snap, int32_t* kv_end,
-                                   Tile* qtiles, int32_t* q_order) {
+                                   Tile* qtiles, int32_t* q_order, int32_t* pair_order) {
   __shared__ int32_t cs[1024];
   const int32_t Ln = sg.l_new;
   for (int base = 0; base < batch; base += 1024) {
@@ -309,6 +309,13 @@ __global__ void append_plan_kernel(AppendSegs sg, int batch, int64_t kbase_strid
       qtiles[g] = w;
       q_order[g] = (int32_t)g;
     }
+    // q-tile pairs (2i, 2i + 1) of each sequence's chunk for the paired forward
+    const int npt = (nqt + 1) / 2;
+    if (pair_order)
+      for (int i = threadIdx.x; i < nb * npt; i += blockDim.x) {
+        const int bl = i / npt, p = i % npt;
+        pair_order[(int64_t)(base + bl) * npt + p] = (int32_t)((int64_t)(base + bl) * nqt + 2 * p);
+      }
     __syncthreads();
     if (threadIdx.x < nb) {
       c_snap[base + threadIdx.x] = cs[threadIdx.x];
@@ -399,16 +406,16 @@ cudaError_t launch_pair_offsets(const Tile* ktiles, int64_t nk, int32_t* kpair_o
 
 cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t kbase_stride, int bm, int bn,
                                int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
-                               int32_t* q_order, cudaStream_t st) {
+                               int32_t* q_order, int32_t* pair_order, cudaStream_t st) {
   append_plan_kernel<<<1, 1024, 0, st>>>(segs, batch, kbase_stride, bm, bn, cache_len, c_snap, kv_end, qtiles,
-                                         q_order);
+                                         q_order, pair_order);
   return cudaGetLastError();
 }
 
 cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap, const KvPages& pages,
                                const int32_t* c_snap, const void* k_new, const void* v_new,
                                void* k_cache, void* v_cache, cudaStream_t st) {
-  int elem = dtype == ISM_BF16 ? 2 : 4;
+  int elem = dtype == ISM_BF16 ? 2 : dtype == ISM_E4M3 ? 1 : 4;
   int row_bytes = hkv * d * elem;
   int64_t total = (int64_t)batch * l_new * (row_bytes / 16);
   if (total == 0) return cudaSuccess;

@@ -58,6 +58,10 @@ EXPORTS = {
                                           C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_int64,
                                           C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                           C.c_size_t, C.c_void_p]),
+    "ism_attn_prefill_append_e4m3": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
+                                               C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_int64,
+                                               C.c_void_p, C.c_void_p, C.c_float, C.c_float, C.c_float, C.c_void_p,
+                                               C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]),
     "ism_attn_prefill_append_paged": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
                                                 C.c_int32, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p,
                                                 C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p,
@@ -333,6 +337,34 @@ def prefill_append(q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_h
                                        _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(),
                                        _stream(q_new.device)),
            "ism_attn_prefill_append")
+    return out, lse
+
+
+def prefill_append_e4m3(q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_host, new_seg_end, new_seg_type,
+                        q_descale: float, k_descale: float, v_descale: float, softmax_scale: float, out=None, lse=None,
+                        workspace=None):
+    """``prefill_append`` with e4m3 (torch.float8_e4m3fn) q_new, k_new, v_new and
+    caches, dequantised by the per-tensor factors; returns (o bf16, lse)."""
+    lib = load()
+    _contig(q_new, k_new, v_new, k_cache, v_cache, cache_len)
+    B, Ln, hq, D = q_new.shape
+    cap = k_cache.shape[1]
+    sh = _shape(q_new, k_new, softmax_scale)
+    se = np.ascontiguousarray(new_seg_end, dtype=np.int32)
+    st = np.ascontiguousarray(new_seg_type, dtype=np.uint8)
+    ch = np.ascontiguousarray(cache_len_host, dtype=np.int32)
+    if out is None:
+        out = torch.empty(q_new.shape, dtype=torch.bfloat16, device=q_new.device)
+    if lse is None:
+        lse = torch.empty((hq, B, Ln), dtype=torch.float32, device=q_new.device)
+    if workspace is None:
+        workspace = _workspace(append_workspace_size(q_new, k_new, softmax_scale), q_new.device)
+    _check(lib.ism_attn_prefill_append_e4m3(C.byref(sh), B, _ptr(q_new), _ptr(k_new), _ptr(v_new), Ln,
+                                            C.c_void_p(se.ctypes.data), C.c_void_p(st.ctypes.data), se.shape[0],
+                                            _ptr(k_cache), _ptr(v_cache), cap, _ptr(cache_len),
+                                            C.c_void_p(ch.ctypes.data), q_descale, k_descale, v_descale, _ptr(out),
+                                            _ptr(lse), _ptr(workspace), workspace.numel(), _stream(q_new.device)),
+           "ism_attn_prefill_append_e4m3")
     return out, lse
 
 

@@ -583,3 +583,35 @@ def test_e4m3_rejects_other_entry_points(ism):
     with pytest.raises(ism.IsmError):  # descales must be positive
         ism.fwd_e4m3(segs, q8, k8, v8, 0.0, 1.0, 1.0, w.softmax_scale)
     ism.check_status()
+
+
+@pytest.mark.parametrize("l_new,segs,hq,hkv", [(200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2),
+                                                (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 3, 3),
+                                                (1, ([1], [1]), 8, 2), (1, ([1], [1]), 6, 2)])
+def test_prefill_append_e4m3(ism, l_new, segs, hq, hkv):
+    """e4m3 queries and caches (cache factors shared by the new keys / values)
+    against the oracle on the dequantised values."""
+    B, d = 3, 128
+    c_lens = np.array([0, 77, 300], dtype=np.int32)
+    cap = 300 + l_new + 5
+    kc, vc, qn, kn, vn = _append_inputs(B, cap, c_lens, l_new, hq, hkv, d, seed=60 + l_new + hq)
+    _, ks = wl.quantize_e4m3(torch.cat([kc.reshape(-1), kn.reshape(-1)]))
+    _, vs = wl.quantize_e4m3(torch.cat([vc.reshape(-1), vn.reshape(-1)]))
+    q8, qs = wl.quantize_e4m3(qn)
+    k8c, k8n = ((t.float() / ks).to(torch.float8_e4m3fn) for t in (kc, kn))
+    v8c, v8n = ((t.float() / vs).to(torch.float8_e4m3fn) for t in (vc, vn))
+    kcd, vcd = k8c.to(DEV), v8c.to(DEV)
+    cl = torch.from_numpy(c_lens.copy()).to(DEV)
+    o, lse = ism.prefill_append_e4m3(q8.to(DEV), k8n.to(DEV), v8n.to(DEV), kcd, vcd, cl, c_lens, segs[0], segs[1],
+                                     qs, ks, vs, d ** -0.5)
+    ism.check_status()
+    assert cl.cpu().numpy().tolist() == (c_lens + l_new).tolist()
+    for b in range(B):
+        c = int(c_lens[b])
+        assert torch.equal(kcd[b, c:c + l_new].cpu().view(torch.uint8), k8n[b].view(torch.uint8))
+    deq = lambda t, s: t.double() * s  # noqa: E731
+    o_ref, lse_ref = orc.prefill_append(deq(q8, qs), deq(k8n, ks), deq(v8n, vs), deq(k8c, ks), deq(v8c, vs), c_lens,
+                                        segs[0], segs[1], d ** -0.5)
+    vmax = max(float(deq(v8c, vs).abs().max()), float(deq(v8n, vs).abs().max()))
+    _cmp_e4m3("o_new", o, o_ref, vmax)
+    _cmp_lse("lse_new", lse, np.transpose(lse_ref, (1, 0, 2)), "bf16")
