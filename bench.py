@@ -539,6 +539,7 @@ def measure_append(dev, peaks):
     kus = float(np.median(dec_kernel_us[3:]))
     gbs = float(np.median(np.array(dec_bytes[3:]) / (np.array(dec_kernel_us[3:]) * 1e-6) / 1e9))
     paged = measure_append_paged(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush)
+    e4m3 = measure_append_e4m3(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, peaks)
     return {"workload": a.name,
             "prefill_ms": pre, "prefill_tflops": 4 * d * n_vis_pre / (pre * 1e-3) / 1e12,
             "prefill_frac_of_bf16_peak": 4 * d * n_vis_pre / (pre * 1e-3) / 1e12 / peaks["bf16_tflops"],
@@ -546,6 +547,7 @@ def measure_append(dev, peaks):
             "decode_hbm_gbs": gbs, "decode_frac_of_hbm": gbs / peaks["hbm_gbs"],
             "decode_steps": a.decode_steps,
             "paged": paged,
+            "e4m3": e4m3,
             "note": "decode bytes = K and V cache read once: 2*B*(c+1)*Hkv*D*2 per step; GB/s over the "
                     "split-KV + merge kernels (decode_kernel_us); decode_us_per_call adds the plan and "
                     "cache-write kernels and host launch overhead"}
@@ -675,6 +677,57 @@ def measure_fwd_e4m3(dev, w, peaks, reps=10):
             "frac_of_e4m3_peak": flops / (ms8 * 1e-3) / 1e12 / peak8, "e4m3_peak_tflops": peak8,
             "bf16_fwd_ms": ms16, "speedup_over_bf16": ms16 / ms8,
             "note": "fwd call incl. metadata pass; peak = measured bf16 x 2 (nominal fp8/bf16 ratio)"}
+
+
+def measure_append_e4m3(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, peaks, decode_steps=64):
+    """The append-prefill and decode of ``measure_append`` with e4m3 queries
+    and caches (per-tensor factors): fp8 tensor cores for the prefill, half
+    the cache bytes for the decode."""
+    import torch
+    from paper_2408_00539_gb300 import ism
+    _, ks = wl.quantize_e4m3(kc)
+    _, vs = wl.quantize_e4m3(vc)
+    k8, v8 = (kc.float() / ks).to(torch.float8_e4m3fn), (vc.float() / vs).to(torch.float8_e4m3fn)
+    q8, qs = wl.quantize_e4m3(qn)
+    kn8, vn8 = (kn.float() / ks).to(torch.float8_e4m3fn), (vn.float() / vs).to(torch.float8_e4m3fn)
+    qd8, qds = wl.quantize_e4m3(qd)
+    kd8, vd8 = (kd.float() / ks).to(torch.float8_e4m3fn), (vd.float() / vs).to(torch.float8_e4m3fn)
+    B, hkv, d = kc.shape[0], kc.shape[2], kc.shape[3]
+    c0 = a.cache_len.copy()
+    cl = torch.from_numpy(c0.copy()).to(dev)
+    stream = torch.cuda.current_stream(dev)
+    pre_ms = []
+    for it in range(8):
+        cl.copy_(torch.from_numpy(c0))
+        flush.fill_(1)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        ism.prefill_append_e4m3(q8, kn8, vn8, k8, v8, cl, c0, a.new_seg_end, a.new_seg_type, qs, ks, vs,
+                                a.softmax_scale)
+        e1.record(stream)
+        e1.synchronize()
+        if it >= 3:
+            pre_ms.append(e0.elapsed_time(e1))
+    c_host = c0 + a.l_new
+    cl.copy_(torch.from_numpy(c_host))
+    dec_kernel_us, dec_bytes = [], []
+    for t in range(decode_steps):
+        k0, k1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        for e in (k0, k1):
+            e.record(stream)
+        ism.set_kernel_timer(ism.KERNEL_DECODE, k0, k1)
+        ism.prefill_append_e4m3(qd8, kd8, vd8, k8, v8, cl, c_host, [1], [1], qds, ks, vs, a.softmax_scale)
+        k1.synchronize()
+        ism.set_kernel_timer(ism.KERNEL_DECODE)
+        dec_kernel_us.append(k0.elapsed_time(k1) * 1e3)
+        dec_bytes.append(2 * B * (int(c_host[0]) + 1) * hkv * d)
+        c_host = c_host + 1
+    ism.check_status(dev)
+    kus = float(np.median(dec_kernel_us[3:]))
+    gbs = float(np.median(np.array(dec_bytes[3:]) / (np.array(dec_kernel_us[3:]) * 1e-6) / 1e9))
+    return {"prefill_ms": float(np.median(pre_ms)), "decode_kernel_us": kus, "decode_hbm_gbs": gbs,
+            "decode_frac_of_hbm": gbs / peaks["hbm_gbs"], "decode_steps": decode_steps,
+            "note": "decode bytes = e4m3 K and V cache read once: 2*B*(c+1)*Hkv*D per step"}
 
 
 def measure_session(dev):

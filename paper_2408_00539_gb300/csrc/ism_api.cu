@@ -643,12 +643,14 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
   count_launch(2);
   // decode kernels serve up to kMaxDecodeGroup query heads per KV head; larger
   // groups take the forward kernels (one query row per tile)
-  if (l_new == 1 && shape->dtype == ISM_BF16 && !force_cuda_cores() && hq / hkv <= kMaxDecodeGroup) {
+  if (l_new == 1 && (shape->dtype == ISM_BF16 || shape->dtype == ISM_E4M3) && !force_cuda_cores() &&
+      hq / hkv <= kMaxDecodeGroup) {
     DecodeArgs a{};
     a.q = q_new; a.k_cache = k_cache; a.v_cache = v_cache; a.pages = cg.pages; a.out = o_new; a.lse = lse_new;
     a.c_snap = L.c_snap;
     a.batch = batch; a.hq = hq; a.hkv = hkv; a.d = d; a.dtype = shape->dtype; a.cap = cg.cap;
     a.group = hq / hkv;
+    a.qk_descale = qk_descale; a.v_descale = v_descale;
     a.kv_rows = cg.kv_rows;
     a.scale = shape->softmax_scale;
     // chunks of a multiple of 64 keys, as many as fill whole waves of resident

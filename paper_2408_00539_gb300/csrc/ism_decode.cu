@@ -6,6 +6,9 @@
 // per-chunk softmax partials.  Scores are kept in base 2 (q pre-scaled by
 // scale * log2 e).
 #include <cstdlib>
+#include <type_traits>
+
+#include <cuda_fp16.h>
 
 #include "ism_internal.cuh"
 #include "ism_tc_common.cuh"
@@ -21,6 +24,27 @@ template <>
 struct BfVec<4> { using T = uint2; };
 template <>
 struct BfVec<2> { using T = uint32_t; };
+
+// e4m3 elements: DPL bytes a lane
+template <int N>
+struct F8Vec;
+template <>
+struct F8Vec<4> { using T = uint32_t; };
+template <>
+struct F8Vec<2> { using T = uint16_t; };
+
+template <int DPL>
+__device__ __forceinline__ void unpack_e4m3(const typename F8Vec<DPL>::T& raw, float (&x)[DPL]) {
+  const uint16_t* pairs = reinterpret_cast<const uint16_t*>(&raw);
+#pragma unroll
+  for (int i = 0; i < DPL / 2; ++i) {
+    uint32_t h2;  // two halves, the lower from the lower byte
+    asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h2) : "h"(pairs[i]));
+    const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&h2));
+    x[2 * i] = f.x;
+    x[2 * i + 1] = f.y;
+  }
+}
 
 template <int DPL>
 __device__ __forceinline__ void unpack_bf16(const typename BfVec<DPL>::T& raw, float (&x)[DPL]) {
@@ -40,7 +64,9 @@ __device__ __forceinline__ void unpack_bf16(const typename BfVec<DPL>::T& raw, f
 // with the full score of (head l / KPI, key l % KPI); the softmax of a head
 // then runs across its KPI lanes, and the probabilities are broadcast back
 // for O += P V.
-template <int D, int G>
+// kE4M3: e4m3 query and caches (one byte an element), dequantised by
+// qk_descale in the scores and v_descale in the output.
+template <int D, int G, bool kE4M3 = false>
 __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs a) {
   constexpr int DPL = D / 32;
   constexpr int KPI = 32 / G;  // keys per batch
@@ -50,12 +76,19 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
   const int kv_len = a.c_snap[b] + 1;
   const int k0 = split * a.chunk;
   const int k1 = min(kv_len, k0 + a.chunk);
-  const float qscale = a.scale * 1.4426950408889634f;
-  using Raw = typename BfVec<DPL>::T;
+  const float qscale = a.scale * 1.4426950408889634f * (kE4M3 ? a.qk_descale : 1.f);
+  using Raw = typename std::conditional<kE4M3, typename F8Vec<DPL>::T, typename BfVec<DPL>::T>::type;
+  using Elem = typename std::conditional<kE4M3, uint8_t, __nv_bfloat16>::type;
+  auto unpack = [](const Raw& raw, float (&x)[DPL]) {
+    if constexpr (kE4M3)
+      unpack_e4m3<DPL>(raw, x);
+    else
+      unpack_bf16<DPL>(raw, x);
+  };
 
-  const __nv_bfloat16* Q = (const __nv_bfloat16*)a.q;
-  const __nv_bfloat16* Kc = (const __nv_bfloat16*)a.k_cache;
-  const __nv_bfloat16* Vc = (const __nv_bfloat16*)a.v_cache;
+  const Elem* Q = (const Elem*)a.q;
+  const Elem* Kc = (const Elem*)a.k_cache;
+  const Elem* Vc = (const Elem*)a.v_cache;
   const int64_t kstride = (int64_t)a.hkv * D;
 
   // G is the group size padded to a power of two: heads h >= grp are zero and not written
@@ -64,7 +97,7 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
 #pragma unroll
   for (int h = 0; h < G; ++h) {
     if (h < grp) {
-      unpack_bf16<DPL>(*reinterpret_cast<const Raw*>(Q + ((int64_t)b * hq + g * grp + h) * D + lane * DPL), q[h]);
+      unpack(*reinterpret_cast<const Raw*>(Q + ((int64_t)b * hq + g * grp + h) * D + lane * DPL), q[h]);
     } else {
 #pragma unroll
       for (int i = 0; i < DPL; ++i) q[h][i] = 0.f;
@@ -81,8 +114,8 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
 #pragma unroll
     for (int i = 0; i < DPL; ++i) o[h][i] = 0.f;
 
-  const __nv_bfloat16* kbase = Kc + (int64_t)g * D + lane * DPL;
-  const __nv_bfloat16* vbase = Vc + (int64_t)g * D + lane * DPL;
+  const Elem* kbase = Kc + (int64_t)g * D + lane * DPL;
+  const Elem* vbase = Vc + (int64_t)g * D + lane * DPL;
   for (int kb = k0 + warp * KPI; kb < k1; kb += kDecWarps * KPI) {
     // every K and V row load of the batch is issued before any use; rows past
     // the chunk re-read its last key and get probability 0
@@ -98,7 +131,7 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
 #pragma unroll
     for (int t = 0; t < KPI; ++t) {
       float kx[DPL];
-      unpack_bf16<DPL>(kraw[t], kx);
+      unpack(kraw[t], kx);
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         float acc = 0.f;
@@ -141,7 +174,7 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
 #pragma unroll
     for (int t = 0; t < KPI; ++t) {
       float vx[DPL];
-      unpack_bf16<DPL>(vraw[t], vx);
+      unpack(vraw[t], vx);
 #pragma unroll
       for (int h = 0; h < G; ++h) {
         const float pht = __shfl_sync(0xffffffffu, p, h * KPI + t);
@@ -178,7 +211,7 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
       }
     }
     const int64_t pidx = ((int64_t)b * hq + g * grp + h) * a.splits + split;
-    a.part_o[pidx * D + d] = acc;
+    a.part_o[pidx * D + d] = kE4M3 ? acc * a.v_descale : acc;
     if (d == 0) { a.part_ml[pidx * 2] = M; a.part_ml[pidx * 2 + 1] = lsum; }
   }
 }
@@ -191,18 +224,22 @@ __global__ void __launch_bounds__(kDecWarps * 32) decode_split_kernel(DecodeArgs
 // hold whole batches of 32 / G keys.  A 2-stage ring of 64-key tiles (about
 // 70 KB of shared memory) lets three CTAs share an SM; measured on the 8 x 16K
 // cache it beats 3 or 4 stages and 32-key tiles.
-template <int G> struct TmaCfg {
+// With e4m3 caches a row is 128 bytes (one box of 128 columns), a K or V
+// tile half the bf16 size.
+template <int G, bool kE4M3 = false> struct TmaCfg {
   static constexpr int kTile = 64;
   static constexpr int kStages = 2;
-  static constexpr uint32_t kHalf = kTile * 128;      // kTile rows x 64 bf16
-  static constexpr uint32_t kStageBytes = 4 * kHalf;  // K and V, two halves each
+  static constexpr uint32_t kHalf = kTile * 128;                    // kTile rows x 128 bytes
+  static constexpr uint32_t kKV = (kE4M3 ? 1 : 2) * kHalf;          // one K (or V) tile
+  static constexpr uint32_t kStageBytes = 2 * kKV;                  // K and V
 };
 
-template <int G>
+template <int G, bool kE4M3 = false>
 __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__ CUtensorMap tmK,
                                                         const __grid_constant__ CUtensorMap tmV, DecodeArgs a) {
-  constexpr int kTmaTile = TmaCfg<G>::kTile, kTmaStages = TmaCfg<G>::kStages;
-  constexpr uint32_t kTmaHalf = TmaCfg<G>::kHalf, kTmaStageBytes = TmaCfg<G>::kStageBytes;
+  using Cfg = TmaCfg<G, kE4M3>;
+  constexpr int kTmaTile = Cfg::kTile, kTmaStages = Cfg::kStages;
+  constexpr uint32_t kTmaHalf = Cfg::kHalf, kTmaKV = Cfg::kKV, kTmaStageBytes = Cfg::kStageBytes;
   constexpr int D = 128, DPL = 4, KPI = 32 / G, RPW = kTmaTile / 4, NB = RPW / KPI;  // batches per warp per tile
   static_assert(NB >= 1 && RPW % KPI == 0, "a warp's rows must hold whole batches");
   extern __shared__ __align__(128) uint8_t dsm[];
@@ -239,23 +276,36 @@ __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__
                                         : row0 + t * kTmaTile;
         ptx::mbar_expect_tx(&full[s], kTmaStageBytes);
         ptx::tma_load_2d(st, &tmK, &full[s], g * D, y);
-        ptx::tma_load_2d(st + kTmaHalf, &tmK, &full[s], g * D + 64, y);
-        ptx::tma_load_2d(st + 2 * kTmaHalf, &tmV, &full[s], g * D, y);
-        ptx::tma_load_2d(st + 3 * kTmaHalf, &tmV, &full[s], g * D + 64, y);
+        ptx::tma_load_2d(st + kTmaKV, &tmV, &full[s], g * D, y);
+        if (!kE4M3) {  // bf16 rows: the second 64 columns
+          ptx::tma_load_2d(st + kTmaHalf, &tmK, &full[s], g * D + 64, y);
+          ptx::tma_load_2d(st + kTmaKV + kTmaHalf, &tmV, &full[s], g * D + 64, y);
+        }
       }
       // every issued copy completes before the CTA exits
       for (int t = issued - kTmaStages > 0 ? issued - kTmaStages : 0; t < issued; ++t)
         tc::wait(&full[t % kTmaStages], (uint32_t)(t / kTmaStages) & 1, a.status);
     }
   } else {
-    const float qscale = a.scale * 1.4426950408889634f;
-    const __nv_bfloat16* Q = (const __nv_bfloat16*)a.q;
+    const float qscale = a.scale * 1.4426950408889634f * (kE4M3 ? a.qk_descale : 1.f);
+    // this lane's DPL elements of a row (bf16: 8 bytes in half lane / 16; e4m3: 4 bytes)
+    auto row_at = [&](const uint8_t* base, float (&x)[DPL]) {
+      if constexpr (kE4M3)
+        unpack_e4m3<DPL>(*reinterpret_cast<const uint32_t*>(base + lane * 4), x);
+      else
+        unpack_bf16<DPL>(*reinterpret_cast<const uint2*>(base + (lane >> 4) * kTmaHalf + (lane & 15) * 8), x);
+    };
+    const uint8_t* Q = static_cast<const uint8_t*>(a.q);
+    const int64_t qrow_bytes = (int64_t)D * (kE4M3 ? 1 : 2);
     float q[G][DPL];
 #pragma unroll
     for (int h = 0; h < G; ++h) {
       if (h < a.group) {
-        unpack_bf16<DPL>(*reinterpret_cast<const uint2*>(Q + ((int64_t)b * a.hq + g * a.group + h) * D + lane * DPL),
-                         q[h]);
+        const uint8_t* qr = Q + ((int64_t)b * a.hq + g * a.group + h) * qrow_bytes + lane * DPL * (kE4M3 ? 1 : 2);
+        if constexpr (kE4M3)
+          unpack_e4m3<DPL>(*reinterpret_cast<const uint32_t*>(qr), q[h]);
+        else
+          unpack_bf16<DPL>(*reinterpret_cast<const uint2*>(qr), q[h]);
       } else {
 #pragma unroll
         for (int i = 0; i < DPL; ++i) q[h][i] = 0.f;
@@ -270,8 +320,6 @@ __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__
     for (int h = 0; h < G; ++h)
 #pragma unroll
       for (int i = 0; i < DPL; ++i) o[h][i] = 0.f;
-    // lane's 8 bytes of a row: half lane/16, bytes (lane % 16) * 8
-    const uint32_t lane_off = (uint32_t)(lane >> 4) * kTmaHalf + (uint32_t)(lane & 15) * 8;
     for (int t = 0; t < ntiles; ++t) {
       const int s = t % kTmaStages;
       if (!tc::wait(&full[s], (uint32_t)(t / kTmaStages) & 1, a.status)) break;
@@ -284,7 +332,7 @@ __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__
 #pragma unroll
         for (int tt = 0; tt < KPI; ++tt) {
           float kx[DPL];
-          unpack_bf16<DPL>(*reinterpret_cast<const uint2*>(st + lane_off + (uint32_t)(r0 + tt) * 128), kx);
+          row_at(st + (uint32_t)(r0 + tt) * 128, kx);
 #pragma unroll
           for (int h = 0; h < G; ++h) {
             float acc = 0.f;
@@ -325,8 +373,7 @@ __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__
 #pragma unroll
         for (int tt = 0; tt < KPI; ++tt) {
           float vx[DPL];
-          unpack_bf16<DPL>(*reinterpret_cast<const uint2*>(st + 2 * kTmaHalf + lane_off + (uint32_t)(r0 + tt) * 128),
-                           vx);
+          row_at(st + kTmaKV + (uint32_t)(r0 + tt) * 128, vx);
 #pragma unroll
           for (int h = 0; h < G; ++h) {
             const float pht = __shfl_sync(0xffffffffu, p, h * KPI + tt);
@@ -363,7 +410,7 @@ __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__
       }
     }
     const int64_t pidx = ((int64_t)b * a.hq + g * a.group + h) * a.splits + split;
-    a.part_o[pidx * D + d] = acc;
+    a.part_o[pidx * D + d] = kE4M3 ? acc * a.v_descale : acc;
     if (d == 0) { a.part_ml[pidx * 2] = M; a.part_ml[pidx * 2 + 1] = lsum; }
   }
 }
@@ -396,7 +443,21 @@ cudaError_t run(const DecodeArgs& a, cudaStream_t st) {
   dim3 grid(a.splits, a.hkv, a.batch);
   cudaError_t e;
   // the TMA kernel needs at least two heads per KV head (batches of 32 / G keys)
-  if (a.tma && G >= 2) {
+  if (a.dtype == ISM_E4M3 && !(a.tma && G >= 2)) {
+    if (D != 128) return cudaErrorInvalidValue;
+    decode_split_kernel<D, G, true><<<grid, kDecWarps * 32, 0, st>>>(a);
+  } else if (a.dtype == ISM_E4M3) {
+    using Cfg = TmaCfg<G >= 2 ? G : 2, true>;
+    CUtensorMap tk, tv;
+    const uint64_t rows = (uint64_t)a.kv_rows;
+    if ((e = tc::make_tmap_e4m3_plain(&tk, a.k_cache, (uint64_t)a.hkv * D, rows, Cfg::kTile)) != cudaSuccess) return e;
+    if ((e = tc::make_tmap_e4m3_plain(&tv, a.v_cache, (uint64_t)a.hkv * D, rows, Cfg::kTile)) != cudaSuccess) return e;
+    const int smem = Cfg::kStages * Cfg::kStageBytes + 2 * Cfg::kStages * 8 + (8 * G + 4 * G * D) * 4;
+    if ((e = cudaFuncSetAttribute(decode_tma_kernel<G >= 2 ? G : 2, true>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
+      return e;
+    decode_tma_kernel<G >= 2 ? G : 2, true><<<grid, 160, smem, st>>>(tk, tv, a);
+  } else if (a.tma && G >= 2) {
     using Cfg = TmaCfg<G >= 2 ? G : 2>;
     CUtensorMap tk, tv;
     const uint64_t rows = (uint64_t)a.kv_rows;

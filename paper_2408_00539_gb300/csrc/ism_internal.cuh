@@ -148,6 +148,7 @@ struct DecodeArgs {
   const int32_t* c_snap; // cache length before the append, per sequence
   int32_t batch, hq, hkv, d, dtype;
   int32_t group;         // query heads per KV head (the kernels pad it to a power of two)
+  float qk_descale, v_descale;  // e4m3: dequantisation of the scores and of the output
   int64_t cap;
   int64_t kv_rows;       // rows of the K / V tensors: batch * cap, or pages * page_size
   float scale;

@@ -147,6 +147,8 @@ __device__ __forceinline__ uint64_t desc_ilv_mnmajor(uint32_t tile_saddr, int kk
 cudaError_t make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows);
 // Host: 2D bf16 tensor map with a 64-column x box_rows box, no swizzle.
 cudaError_t make_tmap_bf16_plain(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows);
+// 1-byte elements, box of 128 columns x box_rows, no swizzle
+cudaError_t make_tmap_e4m3_plain(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows);
 // Host: true on an sm_103 device with the tensor-map encoder available.
 bool available();
 // Host: forward with two query heads (sharing a KV head) per CTA.
