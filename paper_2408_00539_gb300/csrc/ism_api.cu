@@ -401,13 +401,21 @@ ism_status_t ism_attn_bwd_workspace_size_min(const ism_segments_t* segs, const i
   return ISM_OK;
 }
 
-ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q,
-                          const void* k, const void* v, void* o, float* lse, void* workspace,
-                          size_t workspace_bytes, ism_stream_t stream) {
+}  // extern "C"
+
+namespace {
+
+// The one-pass forward for bf16 / fp32 (ism_attn_fwd) and e4m3 inputs
+// (ism_attn_fwd_e4m3; qk_descale = q_descale * k_descale).
+ism_status_t fwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q, const void* k,
+                      const void* v, void* o, float* lse, void* workspace, size_t workspace_bytes, ism_stream_t stream,
+                      float qk_descale, float v_descale) {
   SegInfo info;
   ism_status_t r = check_segments(segs, &info);
   if (r != ISM_OK) return r;
-  if ((r = check_shape(shape)) != ISM_OK) return r;
+  const bool e4m3 = shape && shape->dtype == ISM_E4M3;
+  if ((r = check_shape(shape, e4m3)) != ISM_OK) return r;
+  if (e4m3 && !tc_available()) return fail(ISM_ERR_UNSUPPORTED, "e4m3 forward needs the sm_103 tensor cores");
   if (info.total_tokens == 0) return ISM_OK;
   if (!q || !k || !v || !o) return fail(ISM_ERR_INVALID_ARG, "q, k, v, o must be non-NULL");
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || (lse && !aligned16(lse)))
@@ -425,12 +433,13 @@ ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   a.q = q; a.k = k; a.v = v; a.out = o; a.lse = lse;
   a.hq = shape->num_heads_q; a.hkv = shape->num_heads_kv; a.d = shape->head_dim; a.dtype = shape->dtype;
   a.q_rows = info.total_tokens; a.scale = shape->softmax_scale;
+  a.qk_descale = qk_descale; a.v_descale = v_descale;
   a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order; a.nq = c.nq;
   a.pair_order = L.pair_order; a.npairs = L.pair_order ? c.npairs : 0;
   a.status = status;
   a.flags = tc_flags();
   timer_begin(ISM_KERNEL_FWD, st);
-  if (use_tc(shape)) {
+  if (use_tc(shape) || e4m3) {
     ISM_TRY_CUDA(launch_tc_fwd(a, info.total_tokens, st), "tensor-core forward launch");
   } else {
     ISM_TRY_CUDA(launch_simt_fwd(a, st), "forward launch");
@@ -440,45 +449,33 @@ ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   return ISM_OK;
 }
 
+bool valid_descales(float q_descale, float k_descale, float v_descale) {
+  const float ds[3] = {q_descale, k_descale, v_descale};
+  for (float x : ds)
+    if (!(x > 0.f) || x > 3.0e38f) return false;
+  return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+ism_status_t ism_attn_fwd(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q,
+                          const void* k, const void* v, void* o, float* lse, void* workspace,
+                          size_t workspace_bytes, ism_stream_t stream) {
+  if (shape && shape->dtype == ISM_E4M3)
+    return fail(ISM_ERR_UNSUPPORTED, "e4m3 inputs only in ism_attn_fwd_e4m3");
+  return fwd_impl(segs, shape, q, k, v, o, lse, workspace, workspace_bytes, stream, 1.f, 1.f);
+}
+
 ism_status_t ism_attn_fwd_e4m3(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q,
                                const void* k, const void* v, float q_descale, float k_descale, float v_descale,
                                void* o, float* lse, void* workspace, size_t workspace_bytes, ism_stream_t stream) {
-  SegInfo info;
-  ism_status_t r = check_segments(segs, &info);
-  if (r != ISM_OK) return r;
-  if ((r = check_shape(shape, true)) != ISM_OK) return r;
-  if (shape->dtype != ISM_E4M3) return fail(ISM_ERR_INVALID_ARG, "ism_attn_fwd_e4m3 needs shape->dtype ISM_E4M3");
-  const float ds[3] = {q_descale, k_descale, v_descale};
-  for (float x : ds)
-    if (!(x > 0.f) || x > 3.0e38f) return fail(ISM_ERR_INVALID_ARG, "descales must be positive finite numbers");
-  if (!tc_available()) return fail(ISM_ERR_UNSUPPORTED, "e4m3 forward needs the sm_103 tensor cores");
-  if (info.total_tokens == 0) return ISM_OK;
-  if (!q || !k || !v || !o) return fail(ISM_ERR_INVALID_ARG, "q, k, v, o must be non-NULL");
-  if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || (lse && !aligned16(lse)))
-    return fail(ISM_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
-  Counts c = count_tiles(segs, kTile, kTile);
-  PassLayout L =
-      pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, false, 0, fwd_tile_pairs(shape));
-  if ((r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
-  uint32_t* status;
-  if ((r = status_ptr(&status)) != ISM_OK) return r;
-  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if ((r = build_pass_meta(segs, c, L, false, st)) != ISM_OK) return r;
-
-  AttnArgs a{};
-  a.q = q; a.k = k; a.v = v; a.out = o; a.lse = lse;
-  a.hq = shape->num_heads_q; a.hkv = shape->num_heads_kv; a.d = shape->head_dim; a.dtype = ISM_E4M3;
-  a.q_rows = info.total_tokens; a.scale = shape->softmax_scale;
-  a.qk_descale = q_descale * k_descale; a.v_descale = v_descale;
-  a.kv_end = L.kv_end; a.qtiles = L.qtiles; a.q_order = L.q_order; a.nq = c.nq;
-  a.pair_order = L.pair_order; a.npairs = L.pair_order ? c.npairs : 0;
-  a.status = status;
-  a.flags = tc_flags();
-  timer_begin(ISM_KERNEL_FWD, st);
-  ISM_TRY_CUDA(launch_tc_fwd(a, info.total_tokens, st), "e4m3 forward launch");
-  timer_end(ISM_KERNEL_FWD, st);
-  count_launch(1);
-  return ISM_OK;
+  if (!shape || shape->dtype != ISM_E4M3)
+    return fail(ISM_ERR_INVALID_ARG, "ism_attn_fwd_e4m3 needs shape->dtype ISM_E4M3");
+  if (!valid_descales(q_descale, k_descale, v_descale))
+    return fail(ISM_ERR_INVALID_ARG, "descales must be positive finite numbers");
+  return fwd_impl(segs, shape, q, k, v, o, lse, workspace, workspace_bytes, stream, q_descale * k_descale, v_descale);
 }
 
 ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q,
@@ -744,9 +741,8 @@ ism_status_t ism_attn_prefill_append_e4m3(const ism_attn_shape_t* shape, int32_t
   ism_status_t r = check_shape(shape, true);
   if (r != ISM_OK) return r;
   if (shape->dtype != ISM_E4M3) return fail(ISM_ERR_INVALID_ARG, "ism_attn_prefill_append_e4m3 needs ISM_E4M3");
-  const float ds[3] = {q_descale, k_descale, v_descale};
-  for (float x : ds)
-    if (!(x > 0.f) || x > 3.0e38f) return fail(ISM_ERR_INVALID_ARG, "descales must be positive finite numbers");
+  if (!valid_descales(q_descale, k_descale, v_descale))
+    return fail(ISM_ERR_INVALID_ARG, "descales must be positive finite numbers");
   if (!tc_available()) return fail(ISM_ERR_UNSUPPORTED, "e4m3 attention needs the sm_103 tensor cores");
   if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
   if (batch == 0 || l_new == 0) return ISM_OK;
