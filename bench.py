@@ -770,21 +770,23 @@ def measure_session(dev):
     result = {}
     for mode, qtype in (("ism", wl.QUERY), ("causal", wl.ANSWER)):
         cl = torch.zeros((B,), dtype=torch.int32, device=dev)
-        c_host = np.zeros((B,), dtype=np.int32)
+        c_host = np.zeros((B,), dtype=np.int32)  # advanced in place: the prepared calls hold it
+        prefill = ism.AppendStep(qn, kn, vn, kc, vc, cl, c_host, [s.q_len], [qtype], s.softmax_scale,
+                                 out=o_pre, lse=l_pre, workspace=ws)
+        decode = ism.AppendStep(qd, kd, vd, kc, vc, cl, c_host, [1], [wl.ANSWER], s.softmax_scale,
+                                out=o_dec, lse=l_dec, workspace=ws)
         ttft, tpot = [], []
         for t in range(s.turns):
-            ttft.append(timed(lambda: ism.prefill_append(qn, kn, vn, kc, vc, cl, c_host, [s.q_len], [qtype],
-                                                         s.softmax_scale, out=o_pre, lse=l_pre, workspace=ws)))
-            c_host = c_host + s.q_len
+            ttft.append(timed(prefill))
+            c_host += s.q_len
             if mode == "ism":
                 turn = []
                 for _ in range(s.a_len):
-                    turn.append(timed(lambda: ism.prefill_append(qd, kd, vd, kc, vc, cl, c_host, [1], [wl.ANSWER],
-                                                                 s.softmax_scale, out=o_dec, lse=l_dec, workspace=ws)))
-                    c_host = c_host + 1
+                    turn.append(timed(decode))
+                    c_host += 1
                 tpot.append(float(np.mean(turn)) * 1e3)
             else:  # the answer tokens' K / V are already in the cache from the first pass
-                c_host = c_host + s.a_len
+                c_host += s.a_len
                 cl.fill_(int(c_host[0]))
         ism.check_status(dev)
         result[mode] = (ttft, tpot)
@@ -796,8 +798,8 @@ def measure_session(dev):
             "ttft_ism_over_causal": float(np.mean(ttft_i) / np.mean(ttft_c)),
             "ttft_ms_first_last_turn": [float(ttft_i[0]), float(ttft_i[-1])],
             "tpot_us": float(np.mean(tpot)), "tpot_us_first_last_turn": [tpot[0], tpot[-1]],
-            "note": "one attention layer per call (append plan, cache write, attention); the first turn's "
-                    "calls include warm-up"}
+            "note": "one attention layer per call (append plan, cache write, attention) through a prepared "
+                    "ism.AppendStep (one C call a step); the first turn's calls include warm-up"}
 
 
 WORKLOADS = {"gqa_8k": wl.gqa_8k, "mha_4k": wl.mha_4k, "packed_32k": wl.packed_32k,

@@ -340,6 +340,42 @@ def prefill_append(q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_h
     return out, lse
 
 
+class AppendStep:
+    """A prepared ``prefill_append`` call for a generation loop: the arguments
+    are marshalled once, so each step is one C call.  The caller keeps the new
+    token buffers (q_new, k_new, v_new) and the int32 numpy ``cache_len_host``
+    array, refills the buffers before each call and advances the host array in
+    place after it (the device ``cache_len`` advances itself)."""
+
+    def __init__(self, q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_host: np.ndarray, new_seg_end,
+                 new_seg_type, softmax_scale: float, out=None, lse=None, workspace=None):
+        lib = load()
+        _contig(q_new, k_new, v_new, k_cache, v_cache, cache_len)
+        if not (isinstance(cache_len_host, np.ndarray) and cache_len_host.dtype == np.int32 and
+                cache_len_host.flags["C_CONTIGUOUS"]):
+            raise TypeError("cache_len_host must be a contiguous int32 numpy array (advanced in place)")
+        B, Ln, hq, D = q_new.shape
+        self._sh = _shape(q_new, k_new, softmax_scale)
+        self._se = np.ascontiguousarray(new_seg_end, dtype=np.int32)
+        self._st = np.ascontiguousarray(new_seg_type, dtype=np.uint8)
+        self._host = cache_len_host
+        self.out = torch.empty_like(q_new) if out is None else out
+        self.lse = torch.empty((hq, B, Ln), dtype=torch.float32, device=q_new.device) if lse is None else lse
+        if workspace is None:
+            workspace = _workspace(append_workspace_size(q_new, k_new, softmax_scale), q_new.device)
+        self._keep = (q_new, k_new, v_new, k_cache, v_cache, cache_len, workspace)
+        self._fn = lib.ism_attn_prefill_append
+        self._args = (C.byref(self._sh), B, _ptr(q_new), _ptr(k_new), _ptr(v_new), Ln,
+                      C.c_void_p(self._se.ctypes.data), C.c_void_p(self._st.ctypes.data), self._se.shape[0],
+                      _ptr(k_cache), _ptr(v_cache), k_cache.shape[1], _ptr(cache_len),
+                      C.c_void_p(cache_len_host.ctypes.data), _ptr(self.out), _ptr(self.lse), _ptr(workspace),
+                      workspace.numel(), _stream(q_new.device))
+
+    def __call__(self):
+        _check(self._fn(*self._args), "ism_attn_prefill_append")
+        return self.out, self.lse
+
+
 def prefill_append_e4m3(q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_host, new_seg_end, new_seg_type,
                         q_descale: float, k_descale: float, v_descale: float, softmax_scale: float, out=None, lse=None,
                         workspace=None):

@@ -615,3 +615,30 @@ def test_prefill_append_e4m3(ism, l_new, segs, hq, hkv):
     vmax = max(float(deq(v8c, vs).abs().max()), float(deq(v8n, vs).abs().max()))
     _cmp_e4m3("o_new", o, o_ref, vmax)
     _cmp_lse("lse_new", lse, np.transpose(lse_ref, (1, 0, 2)), "bf16")
+
+
+def test_append_step_matches_prefill_append(ism):
+    """The prepared call (arguments marshalled once, host lengths advanced in
+    place) gives the results of prefill_append step by step."""
+    B, d, c0, steps, hq, hkv = 2, 128, 300, 4, 8, 2
+    cap = c0 + steps
+    kc, vc, qn, kn, vn = _append_inputs(B, cap, None, steps, hq, hkv, d, seed=77)
+    outs = []
+    for prepared in (False, True):
+        kcd, vcd = kc.clone().to(DEV), vc.clone().to(DEV)
+        c_host = np.array([c0, c0 - 50], dtype=np.int32)
+        cl = torch.from_numpy(c_host.copy()).to(DEV)
+        qb, kb, vb = (torch.empty((B, 1) + tuple(t.shape[2:]), dtype=t.dtype, device=DEV) for t in (qn, kn, vn))
+        step = ism.AppendStep(qb, kb, vb, kcd, vcd, cl, c_host, [1], [1], d ** -0.5) if prepared else None
+        got = []
+        for t in range(steps):
+            qb.copy_(qn[:, t:t + 1]); kb.copy_(kn[:, t:t + 1]); vb.copy_(vn[:, t:t + 1])
+            if prepared:
+                o, _ = step()
+            else:
+                o, _ = ism.prefill_append(qb, kb, vb, kcd, vcd, cl, c_host, [1], [1], d ** -0.5)
+            got.append(o.clone())
+            c_host += 1
+        ism.check_status()
+        outs.append(torch.stack(got))
+    assert torch.equal(outs[0], outs[1])
