@@ -1,4 +1,6 @@
-// e4m3 (fp8) tensor-core building blocks and forward (sm_103a, kind::f8f6f4).
+// e4m3 (fp8) tensor-core building block check (sm_103a, kind::f8f6f4): one
+// tile product in each operand layout the e4m3 forward (fwd_pair_kernel with
+// e4m3 operands, ism_fwd2_tc.cu) uses.
 #include "ism_tc_common.cuh"
 
 namespace ism {

@@ -141,3 +141,40 @@ def test_append_errors(lib):
     assert call(seg_type=np.array([0, 2], np.uint8)) == 1
     assert call(nseg=0) == 1
     assert call(cache_host=np.array([-1, 0], np.int32)) == 1
+
+
+def test_paged_append_errors(lib):
+    sh = _shape()
+    se = np.array([4, 8], np.int32)
+    st = np.array([0, 1], np.uint8)
+    ch = np.array([10, 20], np.int32)
+    bt = np.array([[0, 1], [2, 3]], np.int32)
+
+    def call(page_size=128, num_pages=4, table=bt, max_pages=2, cache_host=ch):
+        return lib.ism_attn_prefill_append_paged(C.byref(sh), 2, FAKE, FAKE, FAKE, 8, se.ctypes.data, st.ctypes.data,
+                                                 2, FAKE, FAKE, num_pages, page_size, FAKE, table.ctypes.data,
+                                                 max_pages, FAKE, cache_host.ctypes.data, FAKE, None, FAKE, 1 << 30,
+                                                 None)
+    assert call(page_size=64) == 1 and "page_size" in lib.ism_last_error().decode()
+    bad = bt.copy()
+    bad[1, 0] = 4                                                 # one past the pool
+    assert call(table=bad) == 1 and "outside" in lib.ism_last_error().decode()
+    assert call(cache_host=np.array([10, 250], np.int32)) == 1   # 250 + 8 keys > 2 pages of 128
+    assert call(max_pages=0) == 1
+    assert call(num_pages=0) == 1
+
+
+def test_e4m3_entry_errors(lib):
+    keep = _Keep()
+    s = _segs([0, 10], [0, 2], [4, 10], [0, 1], keep)
+    assert _fwd(lib, s, _shape(dtype=2)) == 2                    # e4m3 only through ism_attn_fwd_e4m3
+
+    def fwd8(sh, qd=1.0, kd=1.0, vd=1.0):
+        return lib.ism_attn_fwd_e4m3(C.byref(s), C.byref(sh), FAKE, FAKE, FAKE, qd, kd, vd, FAKE, FAKE, FAKE, 1 << 30,
+                                     None)
+    assert fwd8(_shape(dtype=0)) == 1                            # shape must say ISM_E4M3
+    assert fwd8(_shape(dtype=2), qd=0.0) == 1                    # descales positive
+    assert fwd8(_shape(dtype=2), vd=float("inf")) == 1
+    need = C.c_size_t()
+    assert lib.ism_attn_fwd_workspace_size(C.byref(s), C.byref(_shape(dtype=2)), C.byref(need)) == 0
+    assert lib.ism_attn_fwd_workspace_size(C.byref(s), C.byref(_shape(dtype=2, d=64)), C.byref(need)) == 2
