@@ -151,15 +151,20 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def dist_setup(args):
+def dist_setup(args, backend: str = "nccl"):
+    """One process per GPU (torchrun's RANK / LOCAL_RANK / WORLD_SIZE /
+    MASTER_*); backend "gloo" runs the same bookkeeping on CPU processes."""
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+            dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        else:
+            dist.init_process_group(backend)
     elif torch.cuda.is_available():
         torch.cuda.set_device(0)
     return world, rank, local
@@ -172,13 +177,21 @@ def barrier(world):
 
 
 def max_over_ranks(x: float, world: int) -> float:
+    """The slowest rank's time: the whole job's wall time for replicas."""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_throughput(units_per_rank: float, world: int, steps: int, total_ms: float) -> float:
+    """Whole-job rate of N replicas: every rank processes units_per_rank a
+    step, over the slowest rank's time."""
+    return units_per_rank * world * steps / (total_ms * 1e-3)
 
 
 # ---------------------------------------------------------------- oracle arm
@@ -316,7 +329,7 @@ def run_cuda(args, w):
 
     total_ms = max_over_ranks(float(np.sum(step_ms)), world)
     ms_per_step = total_ms / args.steps
-    value = flops * world * args.steps / (total_ms * 1e-3) / 1e12
+    value = job_throughput(flops, world, args.steps, total_ms) / 1e12
 
     # roofline of each attention kernel; the dominant one (largest share of
     # the step) is the line's "roofline"
@@ -439,7 +452,7 @@ def run_cuda(args, w):
     torch.cuda.synchronize()
     barrier(world)
     e2e_total = max_over_ranks(run_pipelined(args.steps), world)
-    e2e_value = flops * world * args.steps / (e2e_total * 1e-3) / 1e12
+    e2e_value = job_throughput(flops, world, args.steps, e2e_total) / 1e12
 
     if rank != 0:
         return
@@ -461,7 +474,7 @@ def run_cuda(args, w):
                 "how": "K steps back to back through ism.fwd/ism.bwd; step i+1's Q, K, V, dO uploads (pinned host, "
                        "copy stream) and step i's dQ, dK, dV read-backs (second copy stream) overlap the kernels; "
                        "double-buffered device tensors; inputs (335 MB) exceed L2, no flush",
-                "serial": {"value": flops * world * args.steps / (serial_total * 1e-3) / 1e12,
+                "serial": {"value": job_throughput(flops, world, args.steps, serial_total) / 1e12,
                            "ms_per_step": serial_total / args.steps,
                            "how": "each step alone: upload, fwd+bwd, read-back, L2 flushed between steps"}},
         "gpu_launches": int(launches),
