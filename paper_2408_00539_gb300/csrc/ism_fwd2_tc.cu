@@ -36,7 +36,7 @@ struct PairLayout {
 struct Bars {
   uint64_t q_full;
   uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2];
-  uint64_t s_full[2], p_full[2], pv_done[2];  // per head of the pair
+  uint64_t s_full[2], p_half[2], p_full[2], pv_done[2];  // per head of the pair
   uint64_t final_mma;
   uint32_t tmem_base;
   int32_t abort;
@@ -95,6 +95,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::mbar_init(&bar->v_full[s], 1);
       ptx::mbar_init(&bar->v_empty[s], 1);
       ptx::mbar_init(&bar->s_full[s], 1);
+      ptx::mbar_init(&bar->p_half[s], 128);
       ptx::mbar_init(&bar->p_full[s], 128);
       ptx::mbar_init(&bar->pv_done[s], 1);
     }
@@ -183,15 +184,23 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                                     idesc_qk, 0u);
         ptx::mma_commit_warp(&bar->s_full[x]);
       };
-      auto issue_pv = [&](int x, int j) {
+      // P V in two halves of 64 keys for bf16: the first as soon as the softmax
+      // warps have written P of keys [0, 64) (p_half), the second after p_full
+      auto issue_pv = [&](int x, int j) -> bool {
         const uint32_t sV = ptx::smem_u32(smem + L::V + (j & 1) * kTB);
         const uint32_t tS = tmem + 256u * (uint32_t)x, tO = tS + 128u;
+        if (!wait_warp(&bar->p_half[x], (uint32_t)j & 1, a.status)) return false;
+        ptx::tc_fence_after();
+        if constexpr (!kE4M3)
+          ptx::mma4_bf16_ts_warp<8, 128>(tO, tS, desc_mnmajor(sV, 0), idesc_pv, j > 0 ? 1u : 0u);
+        if (!wait_warp(&bar->p_full[x], (uint32_t)j & 1, a.status)) return false;
+        ptx::tc_fence_after();
         if constexpr (kE4M3)  // P: four e4m3 a column; V MN-major, 32 rows of 128 bytes a k-step
           ptx::mma4_e4m3_ts_warp<8, 256>(tO, tS, desc_kmajor(sV, 0), idesc_pv, j > 0 ? 1u : 0u);
-        else
-          ptx::mma8_bf16_ts_warp<ptx::TmemPairs, ptx::MnMajorSw128>(tO, tS, desc_mnmajor(sV, 0), idesc_pv,
-                                                                   j > 0 ? 1u : 0u);
+        else  // keys [64, 128): P columns 32 + 8 kk, V rows 64 + 16 kk
+          ptx::mma4_bf16_ts_warp<8, 128>(tO, tS + 32, desc_mnmajor(sV, 4), idesc_pv, 1u);
         ptx::mma_commit_warp(&bar->pv_done[x]);
+        return true;
       };
       bool ok = wait_warp(&bar->q_full, 0, a.status) && wait_warp(&bar->k_full[0], 0, a.status);
       // unit x runs key blocks [0, nkb_x); the last unit reading block j
@@ -217,9 +226,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int x = 0; x < 2; ++x) {
           const int nkbx = x ? nkb1 : nkb0;
           if (j >= nkbx) continue;
-          if (!wait_warp(&bar->p_full[x], (uint32_t)j & 1, a.status)) { ok = false; break; }
-          ptx::tc_fence_after();
-          issue_pv(x, j);
+          if (!issue_pv(x, j)) { ok = false; break; }
           if (x == last_user(j)) ptx::mma_commit_warp(&bar->v_empty[s]);
           if (j + 1 < nkbx) {
             if ((a.flags & kFlagDrainTmemReuse) && !wait_warp(&bar->pv_done[x], (uint32_t)j & 1, a.status)) {
@@ -324,6 +331,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           pk[c] = pack_e4m3x4(p01.x, p01.y, p23.x, p23.y);
         }
         ptx::tmem_st32(tS, pk);
+        ptx::tmem_st_wait();
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(&bar->p_half[x]);
       } else {
 #pragma unroll
         for (int hf = 0; hf < 2; ++hf) {
@@ -336,6 +346,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             pk[c] = pack_bf16(pr.x, pr.y);
           }
           ptx::tmem_st32(tS + 32 * hf, pk);
+          if (hf == 0) {  // keys [0, 64): the first half of P V may start
+            ptx::tmem_st_wait();
+            ptx::tc_fence_before();
+            ptx::mbar_arrive(&bar->p_half[x]);
+          }
         }
       }
       l += (rsv[0].x + rsv[0].y) + (rsv[1].x + rsv[1].y);

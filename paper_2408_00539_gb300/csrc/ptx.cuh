@@ -315,6 +315,26 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t m, uint32_t n, ui
          | ((m >> 4) << 24);  // M / 16
 }
 
+// Four k-steps (K = 64) of a bf16 TS contraction, issued like mma8_bf16_ts_warp.
+template <uint32_t kAStep, uint32_t kBStep>
+__device__ __forceinline__ void mma4_bf16_ts_warp(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                                  uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred e, p, t;\n .reg .b32 a1, a2, a3;\n .reg .b64 b1, b2, b3;\n"
+      " elect.sync _|e, 0xffffffff;\n @!e bra MMA4_BF_DONE;\n"
+      " setp.ne.b32 p, %4, 0;\n setp.eq.u32 t, 0, 0;\n"
+      " add.u32 a1, %1, %5; add.u32 a2, %1, %6; add.u32 a3, %1, %7;\n"
+      " add.s64 b1, %2, %8; add.s64 b2, %2, %9; add.s64 b3, %2, %10;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [a1], b1, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [a2], b2, %3, t;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [a3], b3, %3, t;\n"
+      " MMA4_BF_DONE:\n}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(acc), "n"(kAStep), "n"(2 * kAStep), "n"(3 * kAStep), "n"(kBStep),
+      "n"(2 * kBStep), "n"(3 * kBStep)
+      : "memory");
+}
+
 // Instruction descriptor for kind::f8f6f4 with e4m3 A/B and fp32 D (K = 32 a step).
 __host__ __device__ constexpr uint32_t idesc_e4m3_f32(uint32_t m, uint32_t n, uint32_t a_mn, uint32_t b_mn) {
   return (1u << 4)            // D format: f32
