@@ -97,8 +97,12 @@ def read_peaks():
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons, sampled every 200 ms."""
-    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+    """nvidia-smi clocks and throttle reasons, sampled every 50 ms from before
+    the warm-up on; ``summary`` keeps the samples taken inside the timed
+    window (``mark_start`` / ``mark_end``), or, when the window is shorter
+    than one sampling interval, the first sample after its start (the GPU is
+    still running the same steps then)."""
+    Q = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
          "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
          "clocks_event_reasons.sw_power_cap")
 
@@ -106,11 +110,12 @@ class ClockSampler:
         self.gpu = gpu_index
         self.proc = None
         self.lines = []
+        self.t0 = self.t1 = None
 
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
@@ -120,7 +125,13 @@ class ClockSampler:
 
     def _read(self):
         for line in self.proc.stdout:
-            self.lines.append(line.strip())
+            self.lines.append((time.time(), line.strip()))
+
+    def mark_start(self):
+        self.t0 = time.time()
+
+    def mark_end(self):
+        self.t1 = time.time()
 
     def __exit__(self, *exc):
         if self.proc is not None:
@@ -131,24 +142,27 @@ class ClockSampler:
                 self.proc.kill()
 
     def summary(self):
-        sm, mx, reasons = [], [], set()
+        rows = []
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in self.lines:
+        for t, line in self.lines:
             parts = [p.strip() for p in line.split(",")]
-            if len(parts) < 8:
+            if len(parts) < 9:
                 continue
             try:
-                sm.append(float(parts[1]))
-                mx.append(float(parts[2]))
+                rows.append((t, float(parts[2]), float(parts[3]), parts[5:9]))
             except ValueError:
                 continue
-            for name, val in zip(names, parts[4:8]):
-                if val.lower() == "active":
-                    reasons.add(name)
-        if not sm:
+        t0 = self.t0 if self.t0 is not None else -np.inf
+        t1 = self.t1 if self.t1 is not None else np.inf
+        inside = [r for r in rows if t0 <= r[0] <= t1]
+        if not inside:
+            inside = [r for r in rows if r[0] >= t0][:1]
+        if not inside:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
-        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+        reasons = sorted({n for r in inside for n, v in zip(names, r[3]) if v.lower() == "active"})
+        return {"sm_mhz": float(np.median([r[1] for r in inside])), "sm_max_mhz": max(r[2] for r in inside),
+                "reasons": reasons, "samples": len(inside),
+                "window_ms": None if self.t1 is None or self.t0 is None else (self.t1 - self.t0) * 1e3}
 
 
 def dist_setup(args, backend: str = "nccl"):
@@ -276,6 +290,10 @@ def run_cuda(args, w):
         ism.fwd(segs, qd, kd, vd, w.softmax_scale, out=o, lse=lse)
         ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws_b)
 
+    # clocks are sampled from the warm-up on (nvidia-smi needs a moment to start)
+    clocks = ClockSampler(dev.index) if not args.profile_step else None
+    if clocks is not None:
+        clocks.__enter__()
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
@@ -291,20 +309,27 @@ def run_cuda(args, w):
     stream = torch.cuda.current_stream(dev)
     step_ms = []
     launches0 = ism.kernel_launches()
-    with ClockSampler(dev.index) as clocks:
-        barrier(world)
-        torch.cuda.synchronize()
-        for _ in range(args.steps):
-            flush.fill_(1)  # evict L2 between timed steps (outside the step's events)
-            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            s0.record(stream)
-            step()
-            s1.record(stream)
-            s1.synchronize()
-            step_ms.append(s0.elapsed_time(s1))
-        torch.cuda.synchronize()
-        barrier(world)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.mark_start()
+    for _ in range(args.steps):
+        flush.fill_(1)  # evict L2 between timed steps (outside the step's events)
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        step()
+        s1.record(stream)
+        s1.synchronize()
+        step_ms.append(s0.elapsed_time(s1))
+    torch.cuda.synchronize()
+    clocks.mark_end()
+    barrier(world)
     launches = ism.kernel_launches() - launches0
+    # keep the GPU busy with the same steps a little longer, so that a timed
+    # region shorter than the sampling interval still gets a sample
+    for _ in range(3):
+        step()
+    torch.cuda.synchronize()
+    clocks.__exit__(None, None, None)
     ism.check_status(dev)
 
     # per-kernel times for the rooflines, from separate steps run with the
