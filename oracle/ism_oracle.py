@@ -375,3 +375,50 @@ def prefill_append_paged(q_new, k_new, v_new, k_pool, v_pool, page_size: int, bl
         vc[b, :c] = _f64(gather_pages(v_pool, block_table[b], page_size, c))
     return prefill_append(q_new, k_new, v_new, kc, vc, cache_len, new_seg_end, new_seg_type, scale)
 
+
+
+# --------------------------------------------------------------------------
+# Rotary position encoding of appended tokens.  Positional encoding is outside
+# the paper's operation (Section 2.1 omits it; Section 2.3 applies ISM to
+# models that bring their own); serving stacks rotate the new queries and
+# keys by their absolute positions before the keys enter the cache.  The
+# rotation is the rotary encoding of Su et al. (RoFormer) in its rotate-half
+# form: coordinate k is paired with coordinate k + D/2.
+# --------------------------------------------------------------------------
+
+def rope_rotate(x, positions, cos_table, sin_table):
+    """Rotate x [N, H, D] (row n at position positions[n]) pair by pair: for
+    k < D/2 the pair (x_k, x_{k+D/2}) is turned by the angle whose cosine and
+    sine are cos_table[p, k] and sin_table[p, k]:
+
+        y_k       = x_k cos - x_{k+D/2} sin
+        y_{k+D/2} = x_{k+D/2} cos + x_k sin
+
+    The tables are taken as given (exact fp32 values upcast).  Returns float64."""
+    x = _f64(x)
+    c = _f64(cos_table)[np.asarray(positions)][:, None, :]   # [N, 1, D/2]
+    s = _f64(sin_table)[np.asarray(positions)][:, None, :]
+    half = x.shape[-1] // 2
+    lo, hi = x[..., :half], x[..., half:]
+    return np.concatenate([lo * c - hi * s, hi * c + lo * s], axis=-1)
+
+
+def prefill_append_rope(q_new, k_new, v_new, k_cache, v_cache, cache_len, new_seg_end, new_seg_type,
+                        cos_table, sin_table, scale: float, key_round=None):
+    """Append-prefill with rotary encoding applied to the new tokens: token j
+    of sequence b sits at position cache_len[b] + j; its query and key are
+    rotated there (``rope_rotate``), the rotated keys are appended to the
+    cache (already holding rotated keys of the history), values unchanged,
+    and the new rows attend as in ``prefill_append``.  ``key_round`` maps the
+    rotated keys to the values the cache stores (the cache's element type);
+    None keeps them exact.  Returns (O_new, LSE_new, K_rot [B, Ln, Hkv, D])."""
+    B, Ln = q_new.shape[0], q_new.shape[1]
+    q_rot = np.zeros(tuple(q_new.shape))
+    k_rot = np.zeros(tuple(k_new.shape))
+    for b in range(B):
+        pos = int(cache_len[b]) + np.arange(Ln)
+        q_rot[b] = rope_rotate(q_new[b], pos, cos_table, sin_table)
+        k_rot[b] = rope_rotate(k_new[b], pos, cos_table, sin_table)
+    k_used = k_rot if key_round is None else _f64(key_round(k_rot))
+    o, lse = prefill_append(q_rot, k_used, v_new, k_cache, v_cache, cache_len, new_seg_end, new_seg_type, scale)
+    return o, lse, k_rot

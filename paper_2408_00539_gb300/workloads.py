@@ -301,6 +301,17 @@ def quantize_e4m3(x):
     return (x.float() / descale).to(torch.float8_e4m3fn), descale
 
 
+def rope_tables(rows: int, head_dim: int, base: float = 10000.0):
+    """Rotary-encoding tables, an input of the RoPE append: position p and
+    pair k < head_dim/2 get the angle p * base**(-2k/head_dim) (the usual
+    frequency schedule); returns (cos, sin) as float32 numpy arrays
+    [rows, head_dim/2].  Any table of cosines and sines is a valid input."""
+    half = head_dim // 2
+    inv_freq = base ** (-2.0 * np.arange(half, dtype=np.float64) / head_dim)
+    ang = np.arange(rows, dtype=np.float64)[:, None] * inv_freq[None, :]
+    return np.cos(ang).astype(np.float32), np.sin(ang).astype(np.float32)
+
+
 def random_dialogue_set(rng: np.random.Generator, n_seqs: int, max_len: int,
                         zero_len: bool = True, min_len: int = 1) -> Segments:
     """Small random segmentations for tests: any mix of QUERY/ANSWER

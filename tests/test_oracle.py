@@ -402,6 +402,75 @@ def test_paged_append_equals_contiguous_append():
     np.testing.assert_array_equal(l, l_ref)
 
 
+# ---------------------------------------------------------------- rotary encoding
+
+def _complex_rotate(x, angles):
+    # the rotary encoding as a complex product (RoFormer): coordinates k and
+    # k + D/2 are the real and imaginary parts of z_k, turned by e^{i angle}
+    half = x.shape[-1] // 2
+    z = (x[..., :half] + 1j * x[..., half:]) * np.exp(1j * angles)
+    return np.concatenate([z.real, z.imag], axis=-1)
+
+
+def test_rope_rotate_is_complex_multiplication():
+    rng = np.random.Generator(np.random.PCG64(51))
+    N, H, D, rows = 7, 3, 10, 40
+    ang = rng.uniform(-7.0, 7.0, size=(rows, D // 2))
+    cos_t, sin_t = np.cos(ang), np.sin(ang)
+    pos = rng.integers(0, rows, size=N)
+    x = rng.standard_normal((N, H, D))
+    y = orc.rope_rotate(x, pos, cos_t, sin_t)
+    np.testing.assert_allclose(y, _complex_rotate(x, ang[pos][:, None, :]), rtol=1e-13, atol=1e-13)
+    # position 0 of the usual schedule is the identity; rotations keep norms
+    c32, s32 = wl.rope_tables(rows, D)
+    np.testing.assert_array_equal(orc.rope_rotate(x, np.zeros(N, dtype=int), c32, s32), x)
+    yn = orc.rope_rotate(x, pos, c32, s32)
+    np.testing.assert_allclose(np.linalg.norm(yn, axis=-1), np.linalg.norm(x, axis=-1), rtol=1e-6)
+
+
+def test_rope_scores_depend_on_relative_position_only():
+    # <R(p) q, R(p') k> is a function of p - p' (the property rotary encoding
+    # is built for); the fp32 tables hold it to about 1e-6
+    rng = np.random.Generator(np.random.PCG64(52))
+    D, rows = 16, 600
+    cos_t, sin_t = wl.rope_tables(rows, D)
+    q, k = rng.standard_normal((1, 1, D)), rng.standard_normal((1, 1, D))
+    for p, pk, shift in [(5, 2, 100), (37, 37, 400), (3, 90, 250)]:
+        a = orc.rope_rotate(q, [p], cos_t, sin_t)[0, 0] @ orc.rope_rotate(k, [pk], cos_t, sin_t)[0, 0]
+        b = orc.rope_rotate(q, [p + shift], cos_t, sin_t)[0, 0] @ orc.rope_rotate(k, [pk + shift], cos_t, sin_t)[0, 0]
+        assert abs(a - b) < 1e-4 * (np.linalg.norm(q) * np.linalg.norm(k))
+
+
+def test_rope_appends_equal_one_pass_over_rotated_dialogue():
+    # two turns appended one after the other (keys rotated at their absolute
+    # positions, stored, reused) give the rows of one forward pass over the
+    # whole dialogue with every query and key rotated at its position
+    rng = np.random.Generator(np.random.PCG64(53))
+    hq, hkv, D = 4, 2, 8
+    t1_e, t1_t = [4, 11], [0, 1]
+    t2_e, t2_t = [3, 8], [0, 1]
+    L1, L2 = t1_e[-1], t2_e[-1]
+    L = L1 + L2
+    ang = rng.uniform(-3.0, 3.0, size=(L + 5, D // 2))
+    cos_t, sin_t = np.cos(ang), np.sin(ang)
+    q, k, v = _rand(rng, L, hq, D), _rand(rng, L, hkv, D), _rand(rng, L, hkv, D)
+    cap = L + 2
+    kc, vc = np.zeros((1, cap, hkv, D)), np.zeros((1, cap, hkv, D))
+    o1, l1, kr1 = orc.prefill_append_rope(q[None, :L1], k[None, :L1], v[None, :L1], kc, vc, [0], t1_e, t1_t,
+                                          cos_t, sin_t, 0.4)
+    kc[0, :L1], vc[0, :L1] = kr1[0], v[:L1]
+    o2, l2, _ = orc.prefill_append_rope(q[None, L1:], k[None, L1:], v[None, L1:], kc, vc, [L1], t2_e, t2_t,
+                                        cos_t, sin_t, 0.4)
+    pos = np.arange(L)
+    qr = _complex_rotate(q, ang[pos][:, None, :])
+    kr = _complex_rotate(k, ang[pos][:, None, :])
+    segs = wl.pack([(t1_e + [L1 + e for e in t2_e], t1_t + t2_t)])
+    of, lf = orc.attn_fwd(qr, kr, v, segs, 0.4)
+    np.testing.assert_allclose(o1[0], of[:L1], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(o2[0], of[L1:], rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(l2[0], lf[:, L1:], rtol=1e-12, atol=1e-12)
+
+
 def test_workload_generator_shapes():
     for w in (wl.tiny_fp32(), wl.mha_4k(), wl.gqa_8k(), wl.packed_32k()):
         s = w.segs
