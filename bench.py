@@ -578,6 +578,7 @@ def measure_append(dev, peaks):
     gbs = float(np.median(np.array(dec_bytes[3:]) / (np.array(dec_kernel_us[3:]) * 1e-6) / 1e9))
     paged = measure_append_paged(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush)
     e4m3 = measure_append_e4m3(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, peaks)
+    rope = measure_append_rope(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush)
     return {"workload": a.name,
             "prefill_ms": pre, "prefill_tflops": 4 * d * n_vis_pre / (pre * 1e-3) / 1e12,
             "prefill_frac_of_bf16_peak": 4 * d * n_vis_pre / (pre * 1e-3) / 1e12 / peaks["bf16_tflops"],
@@ -586,6 +587,7 @@ def measure_append(dev, peaks):
             "decode_steps": a.decode_steps,
             "paged": paged,
             "e4m3": e4m3,
+            "rope": rope,
             "note": "decode bytes = K and V cache read once: 2*B*(c+1)*Hkv*D*2 per step; GB/s over the "
                     "split-KV + merge kernels (decode_kernel_us); decode_us_per_call adds the plan and "
                     "cache-write kernels and host launch overhead"}
@@ -640,6 +642,61 @@ def measure_append_paged(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, page_siz
     del kp, vp
     return {"page_size": page_size, "prefill_ms": float(np.median(pre_ms)),
             "decode_kernel_us": float(np.median(dec_kernel_us[3:])), "decode_steps": decode_steps}
+
+
+def measure_append_rope(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, decode_steps=64):
+    """The append-prefill and decode of ``measure_append`` with rotary
+    encoding of the new queries and keys fused into the cache-write pass,
+    against the same calls without it; the metadata timer gives the plan +
+    cache-write kernels alone (L2 flushed before each prefill)."""
+    import torch
+    from paper_2408_00539_gb300 import ism
+    cap, d = kc.shape[1], kc.shape[3]
+    cos_np, sin_np = wl.rope_tables(cap, d)
+    cos_t, sin_t = torch.from_numpy(cos_np).to(dev), torch.from_numpy(sin_np).to(dev)
+    c0 = a.cache_len.copy()
+    cl = torch.from_numpy(c0.copy()).to(dev)
+    stream = torch.cuda.current_stream(dev)
+    out = {}
+    for name, call in (("plain", lambda q, k, v, ch, se, st: ism.prefill_append(q, k, v, kc, vc, cl, ch, se, st,
+                                                                                  a.softmax_scale)),
+                       ("rope", lambda q, k, v, ch, se, st: ism.prefill_append_rope(q, k, v, kc, vc, cl, ch, se, st,
+                                                                                     cos_t, sin_t, a.softmax_scale))):
+        pre_ms, meta_us = [], []
+        for it in range(8):
+            cl.copy_(torch.from_numpy(c0))
+            flush.fill_(1)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            m0, m1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            for e in (m0, m1):
+                e.record(stream)
+            ism.set_kernel_timer(ism.KERNEL_META, m0, m1)
+            e0.record(stream)
+            call(qn, kn, vn, c0, a.new_seg_end, a.new_seg_type)
+            e1.record(stream)
+            e1.synchronize()
+            ism.set_kernel_timer(ism.KERNEL_META)
+            if it >= 3:
+                pre_ms.append(e0.elapsed_time(e1))
+                meta_us.append(m0.elapsed_time(m1) * 1e3)
+        c_host = c0 + a.l_new
+        cl.copy_(torch.from_numpy(c_host))
+        dec_us = []
+        for t in range(decode_steps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            call(qd, kd, vd, c_host, [1], [1])
+            e1.record(stream)
+            e1.synchronize()
+            dec_us.append(e0.elapsed_time(e1) * 1e3)
+            c_host = c_host + 1
+        ism.check_status(dev)
+        out[name] = {"prefill_ms": float(np.median(pre_ms)), "prefill_plan_and_cache_write_us": float(np.median(meta_us)),
+                     "decode_us_per_call": float(np.median(dec_us[3:]))}
+    out["decode_steps"] = decode_steps
+    out["note"] = ("rope: new queries and keys rotated at positions cache_len + j (tables [cap, D/2] fp32) inside "
+                   "the cache-write kernel; the attention kernels are the same")
+    return out
 
 
 def measure_training_cost(dev, w, reps=3):

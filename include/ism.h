@@ -290,6 +290,47 @@ ism_status_t ism_attn_prefill_append_paged(const ism_attn_shape_t* shape, int32_
                                            void* workspace, size_t workspace_bytes, ism_stream_t stream);
 
 /* ---------------------------------------------------------------------------
+ * Append-prefill and decode with rotary position encoding applied on the way
+ * into the cache.  Positional encoding is outside the operation of Section 2.1
+ * (which leaves it out); models that take up ISM (Section 2.3) rotate queries
+ * and keys by their absolute positions before attention.  Token j of
+ * sequence b sits at position p = cache_len[b] + j; for k < D/2 the pair
+ * (x_k, x_{k+D/2}) of its query and of its key is turned by the angle whose
+ * cosine and sine are rope->cos[p * D/2 + k] and rope->sin[p * D/2 + k]:
+ *     y_k = x_k cos - x_{k+D/2} sin,     y_{k+D/2} = x_{k+D/2} cos + x_k sin
+ * (the rotary encoding of RoFormer in its rotate-half form), in fp32 and
+ * rounded once to bf16.  The rotated keys are what the cache stores, values
+ * are stored unchanged, and the new rows attend exactly as in
+ * ism_attn_prefill_append, with the rotated queries.  The rotation runs inside
+ * the pass that writes the cache (no extra launch); the rotated queries go to
+ * the workspace.
+ *   rope->cos / rope->sin: fp32 device tables [rope->rows, D/2], 16-byte
+ *     aligned, read only; cache_len_host[b] + l_new <= rope->rows is required.
+ *   shape->dtype must be ISM_BF16; head_dim 64 or 128.
+ *   q_new / k_new are the unrotated values; every other argument is that of
+ *   ism_attn_prefill_append (contiguous caches).
+ * Workspace: ism_attn_prefill_append_rope_workspace_size (the append's
+ * workspace plus B * l_new * Hq * D bf16 for the rotated queries).
+ * Errors: ISM_ERR_INVALID_ARG for a missing or misaligned table, rows too few
+ * for the positions written, or a dtype other than ISM_BF16.
+ * ------------------------------------------------------------------------- */
+typedef struct {
+  const float* cos;
+  const float* sin;
+  int32_t rows;
+} ism_rope_t;
+ism_status_t ism_attn_prefill_append_rope_workspace_size(const ism_attn_shape_t* shape, int32_t batch,
+                                                         int32_t l_new, size_t* bytes);
+ism_status_t ism_attn_prefill_append_rope(const ism_attn_shape_t* shape, int32_t batch,
+                                          const void* q_new, const void* k_new, const void* v_new,
+                                          int32_t l_new, const int32_t* new_seg_end_host,
+                                          const uint8_t* new_seg_type_host, int32_t n_new_segs,
+                                          void* k_cache, void* v_cache, int64_t cache_capacity,
+                                          int32_t* cache_len, const int32_t* cache_len_host,
+                                          const ism_rope_t* rope, void* o_new, float* lse_new,
+                                          void* workspace, size_t workspace_bytes, ism_stream_t stream);
+
+/* ---------------------------------------------------------------------------
  * Status and diagnostics.
  * ------------------------------------------------------------------------- */
 

@@ -536,10 +536,11 @@ struct AppendLayout {
   int64_t npairs;
   float* part_o;
   float* part_ml;
+  void* q_rot;  // rotated queries of a RoPE append (bf16 [batch * l_new, Hq, D]), else null
   size_t bytes;
 };
 
-AppendLayout append_layout(void* ws, const ism_attn_shape_t* sh, int batch, int l_new) {
+AppendLayout append_layout(void* ws, const ism_attn_shape_t* sh, int batch, int l_new, bool rope = false) {
   Carve cv(ws);
   AppendLayout L;
   const int64_t nqt_seq = (l_new + kTile - 1) / kTile;
@@ -556,6 +557,7 @@ AppendLayout append_layout(void* ws, const ism_attn_shape_t* sh, int batch, int 
   } else {
     L.part_o = L.part_ml = nullptr;
   }
+  L.q_rot = rope ? (void*)cv.take<__nv_bfloat16>((int64_t)batch * l_new * sh->num_heads_q * sh->head_dim) : nullptr;
   L.bytes = ((cv.off + 255) & ~size_t(255)) + 256;
   return L;
 }
@@ -569,6 +571,16 @@ ism_status_t ism_attn_prefill_append_workspace_size(const ism_attn_shape_t* shap
   if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
   if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
   *bytes = append_layout(nullptr, shape, batch, l_new).bytes;  // (e4m3 shapes included)
+  return ISM_OK;
+}
+
+ism_status_t ism_attn_prefill_append_rope_workspace_size(const ism_attn_shape_t* shape, int32_t batch,
+                                                         int32_t l_new, size_t* bytes) {
+  ism_status_t r = check_shape(shape);
+  if (r != ISM_OK) return r;
+  if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
+  if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
+  *bytes = append_layout(nullptr, shape, batch, l_new, true).bytes;
   return ISM_OK;
 }
 
@@ -591,7 +603,7 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
                          const uint8_t* new_seg_type_host, int32_t n_new_segs, void* k_cache, void* v_cache,
                          const CacheGeom& cg, int32_t* cache_len, const int32_t* cache_len_host, void* o_new,
                          float* lse_new, void* workspace, size_t workspace_bytes, cudaStream_t st,
-                         float qk_descale = 1.f, float v_descale = 1.f) {
+                         float qk_descale = 1.f, float v_descale = 1.f, const ism_rope_t* rope = nullptr) {
   ism_status_t r;
   if (!q_new || !k_new || !v_new || !k_cache || !v_cache || !cache_len || !cache_len_host || !o_new)
     return fail(ISM_ERR_INVALID_ARG, "q_new, k_new, v_new, caches, cache_len (device+host), o_new must be non-NULL");
@@ -622,7 +634,14 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
                   (long long)cg.max_keys);
     if (c > max_c) max_c = c;
   }
-  AppendLayout L = append_layout(workspace, shape, batch, l_new);
+  if (rope) {
+    if (!rope->cos || !rope->sin || !aligned16(rope->cos) || !aligned16(rope->sin))
+      return fail(ISM_ERR_INVALID_ARG, "rope tables must be non-NULL and 16-byte aligned");
+    if ((int64_t)max_c + l_new > rope->rows)
+      return fail(ISM_ERR_INVALID_ARG, "rope tables cover %d positions, the append writes up to %lld", rope->rows,
+                  (long long)max_c + l_new);
+  }
+  AppendLayout L = append_layout(workspace, shape, batch, l_new, rope != nullptr);
   if ((r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
   uint32_t* status;
   if ((r = status_ptr(&status)) != ISM_OK) return r;
@@ -633,9 +652,16 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
   ISM_TRY_CUDA(launch_append_plan(sg, batch, paged ? 1 : cg.cap, kTile, kTile, cache_len, L.c_snap, L.kv_end, L.qtiles,
                                   L.q_order, L.pair_order, st),
                "append plan launch");
-  ISM_TRY_CUDA(launch_cache_write(shape->dtype, batch, l_new, hkv, d, cg.cap, cg.pages, L.c_snap, k_new, v_new,
-                                  k_cache, v_cache, st),
-               "cache write launch");
+  if (rope) {
+    ISM_TRY_CUDA(launch_rope_cache_write(batch, l_new, hq, hkv, d, cg.cap, cg.pages, L.c_snap, q_new, k_new, v_new,
+                                         rope->cos, rope->sin, L.q_rot, k_cache, v_cache, st),
+                 "rope cache write launch");
+    q_new = L.q_rot;  // the attention below reads the rotated queries
+  } else {
+    ISM_TRY_CUDA(launch_cache_write(shape->dtype, batch, l_new, hkv, d, cg.cap, cg.pages, L.c_snap, k_new, v_new,
+                                    k_cache, v_cache, st),
+                 "cache write launch");
+  }
   timer_end(ISM_KERNEL_META, st);
   count_launch(2);
   // decode kernels serve up to kMaxDecodeGroup query heads per KV head; larger
@@ -756,6 +782,31 @@ ism_status_t ism_attn_prefill_append_e4m3(const ism_attn_shape_t* shape, int32_t
   return append_impl(shape, batch, q_new, k_new, v_new, l_new, new_seg_end_host, new_seg_type_host, n_new_segs,
                      k_cache, v_cache, cg, cache_len, cache_len_host, o_new, lse_new, workspace, workspace_bytes,
                      reinterpret_cast<cudaStream_t>(stream), q_descale * k_descale, v_descale);
+}
+
+ism_status_t ism_attn_prefill_append_rope(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,
+                                          const void* k_new, const void* v_new, int32_t l_new,
+                                          const int32_t* new_seg_end_host, const uint8_t* new_seg_type_host,
+                                          int32_t n_new_segs, void* k_cache, void* v_cache, int64_t cache_capacity,
+                                          int32_t* cache_len, const int32_t* cache_len_host, const ism_rope_t* rope,
+                                          void* o_new, float* lse_new, void* workspace, size_t workspace_bytes,
+                                          ism_stream_t stream) {
+  ism_status_t r = check_shape(shape);
+  if (r != ISM_OK) return r;
+  if (shape->dtype != ISM_BF16) return fail(ISM_ERR_INVALID_ARG, "ism_attn_prefill_append_rope needs ISM_BF16");
+  if (!rope) return fail(ISM_ERR_INVALID_ARG, "rope is NULL");
+  if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
+  if (batch == 0 || l_new == 0) return ISM_OK;
+  if (cache_capacity <= 0 || (int64_t)batch * cache_capacity >= (int64_t(1) << 31))
+    return fail(ISM_ERR_INVALID_ARG, "batch * cache_capacity must be in (0, 2^31)");
+  CacheGeom cg;
+  cg.cap = cache_capacity;
+  cg.kv_rows = (int64_t)batch * cache_capacity;
+  cg.max_keys = cache_capacity;
+  cg.pages = KvPages{nullptr, 0, 0};
+  return append_impl(shape, batch, q_new, k_new, v_new, l_new, new_seg_end_host, new_seg_type_host, n_new_segs,
+                     k_cache, v_cache, cg, cache_len, cache_len_host, o_new, lse_new, workspace, workspace_bytes,
+                     reinterpret_cast<cudaStream_t>(stream), 1.f, 1.f, rope);
 }
 
 ism_status_t ism_attn_prefill_append_paged(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,

@@ -94,6 +94,13 @@ cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t kbase_
 cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap, const KvPages& pages,
                                const int32_t* c_snap, const void* k_new, const void* v_new,
                                void* k_cache, void* v_cache, cudaStream_t st);
+// Cache write with the rotary encoding of the new queries and keys (bf16,
+// head_dim a multiple of 16): rotated keys and plain values into the cache,
+// rotated queries into q_rot [batch * l_new, hq, d].
+cudaError_t launch_rope_cache_write(int batch, int l_new, int hq, int hkv, int d, int64_t cap,
+                                   const KvPages& pages, const int32_t* c_snap, const void* q_new,
+                                   const void* k_new, const void* v_new, const float* cos_t, const float* sin_t,
+                                   void* q_rot, void* k_cache, void* v_cache, cudaStream_t st);
 
 // CUDA-core attention (ism_simt.cu), fp32 or bf16 storage, fp32 math.
 struct AttnArgs {

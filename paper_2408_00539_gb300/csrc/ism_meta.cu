@@ -345,6 +345,75 @@ __global__ void cache_write_kernel(int batch, int l_new, int row_bytes, int64_t 
   }
 }
 
+// Rotary encoding fused with the cache write.  One thread takes eight
+// consecutive coordinates k0..k0+7 of the first half of one head row and
+// their partners k0+D/2.. (a query head, a key head, or a value head, which
+// is copied as is).  Position of new token j of sequence b: c_snap[b] + j.
+__device__ __forceinline__ void rotate8(const uint4& lo, const uint4& hi, const float* c, const float* s,
+                                        uint4& out_lo, uint4& out_hi) {
+  const __nv_bfloat162* l2 = reinterpret_cast<const __nv_bfloat162*>(&lo);
+  const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&hi);
+  __nv_bfloat162* ol = reinterpret_cast<__nv_bfloat162*>(&out_lo);
+  __nv_bfloat162* oh = reinterpret_cast<__nv_bfloat162*>(&out_hi);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float2 x = __bfloat1622float2(l2[e]);
+    const float2 y = __bfloat1622float2(h2[e]);
+    const float c0 = c[2 * e], c1 = c[2 * e + 1], s0 = s[2 * e], s1 = s[2 * e + 1];
+    ol[e] = __floats2bfloat162_rn(x.x * c0 - y.x * s0, x.y * c1 - y.y * s1);
+    oh[e] = __floats2bfloat162_rn(y.x * c0 + x.x * s0, y.y * c1 + x.y * s1);
+  }
+}
+
+__global__ void rope_cache_write_kernel(int batch, int l_new, int hq, int hkv, int d, int64_t cap, KvPages pages,
+                                        const int32_t* __restrict__ c_snap, const __nv_bfloat16* __restrict__ q_new,
+                                        const __nv_bfloat16* __restrict__ k_new,
+                                        const __nv_bfloat16* __restrict__ v_new, const float* __restrict__ cos_t,
+                                        const float* __restrict__ sin_t, __nv_bfloat16* q_rot,
+                                        __nv_bfloat16* k_cache, __nv_bfloat16* v_cache) {
+  const int half = d / 2;
+  const int units = half / 8;  // 8-coordinate units in one half of a head row
+  const int per_row = (hq + 2 * hkv) * units;
+  const int64_t total = (int64_t)batch * l_new * per_row;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t row = i / per_row;  // b * l_new + j
+    const int r = (int)(i % per_row);
+    const int head = r / units;
+    const int k0 = (r % units) * 8;
+    const int b = (int)(row / l_new);
+    const int64_t p = (int64_t)c_snap[b] + row % l_new;
+    const int64_t dst_row = pages.table ? paged_row(pages, b, p) : (int64_t)b * cap + p;
+    const __nv_bfloat16* src;
+    __nv_bfloat16* dst;
+    if (head < hq) {
+      src = q_new + (row * hq + head) * d;
+      dst = q_rot + (row * hq + head) * d;
+    } else if (head < hq + hkv) {
+      src = k_new + (row * hkv + (head - hq)) * d;
+      dst = k_cache + (dst_row * hkv + (head - hq)) * d;
+    } else {
+      src = v_new + (row * hkv + (head - hq - hkv)) * d;
+      dst = v_cache + (dst_row * hkv + (head - hq - hkv)) * d;
+      *reinterpret_cast<uint4*>(dst + k0) = *reinterpret_cast<const uint4*>(src + k0);
+      *reinterpret_cast<uint4*>(dst + half + k0) = *reinterpret_cast<const uint4*>(src + half + k0);
+      continue;
+    }
+    const uint4 lo = *reinterpret_cast<const uint4*>(src + k0);
+    const uint4 hi = *reinterpret_cast<const uint4*>(src + half + k0);
+    float c[8], s[8];
+    const float4* cp = reinterpret_cast<const float4*>(cos_t + p * half + k0);
+    const float4* sp = reinterpret_cast<const float4*>(sin_t + p * half + k0);
+    const float4 c0 = __ldg(cp), c1 = __ldg(cp + 1), s0 = __ldg(sp), s1 = __ldg(sp + 1);
+    c[0] = c0.x; c[1] = c0.y; c[2] = c0.z; c[3] = c0.w; c[4] = c1.x; c[5] = c1.y; c[6] = c1.z; c[7] = c1.w;
+    s[0] = s0.x; s[1] = s0.y; s[2] = s0.z; s[3] = s0.w; s[4] = s1.x; s[5] = s1.y; s[6] = s1.z; s[7] = s1.w;
+    uint4 out_lo, out_hi;
+    rotate8(lo, hi, c, s, out_lo, out_hi);
+    *reinterpret_cast<uint4*>(dst + k0) = out_lo;
+    *reinterpret_cast<uint4*>(dst + half + k0) = out_hi;
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_kv_end(const SegsDev& s, int32_t* kv_end, cudaStream_t st) {
@@ -423,6 +492,21 @@ cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, 
   if (grid > 152 * 16) grid = 152 * 16;
   cache_write_kernel<<<grid, 256, 0, st>>>(batch, l_new, row_bytes, cap, pages, c_snap, (const uint4*)k_new,
                                            (const uint4*)v_new, (uint4*)k_cache, (uint4*)v_cache);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rope_cache_write(int batch, int l_new, int hq, int hkv, int d, int64_t cap,
+                                   const KvPages& pages, const int32_t* c_snap, const void* q_new,
+                                   const void* k_new, const void* v_new, const float* cos_t, const float* sin_t,
+                                   void* q_rot, void* k_cache, void* v_cache, cudaStream_t st) {
+  const int64_t total = (int64_t)batch * l_new * (hq + 2 * hkv) * (d / 16);
+  if (total == 0) return cudaSuccess;
+  int grid = (int)((total + 255) / 256);
+  if (grid > 152 * 16) grid = 152 * 16;
+  rope_cache_write_kernel<<<grid, 256, 0, st>>>(
+      batch, l_new, hq, hkv, d, cap, pages, c_snap, (const __nv_bfloat16*)q_new, (const __nv_bfloat16*)k_new,
+      (const __nv_bfloat16*)v_new, cos_t, sin_t, (__nv_bfloat16*)q_rot, (__nv_bfloat16*)k_cache,
+      (__nv_bfloat16*)v_cache);
   return cudaGetLastError();
 }
 

@@ -39,6 +39,10 @@ class _Segments(C.Structure):
                 ("seg_type", C.c_void_p), ("seg_type_host", C.c_void_p)]
 
 
+class _Rope(C.Structure):
+    _fields_ = [("cos", C.c_void_p), ("sin", C.c_void_p), ("rows", C.c_int32)]
+
+
 class _Shape(C.Structure):
     _fields_ = [("num_heads_q", C.c_int32), ("num_heads_kv", C.c_int32), ("head_dim", C.c_int32),
                 ("dtype", C.c_int32), ("softmax_scale", C.c_float)]
@@ -67,6 +71,11 @@ EXPORTS = {
                                                 C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p,
                                                 C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t,
                                                 C.c_void_p]),
+    "ism_attn_prefill_append_rope_workspace_size": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_void_p]),
+    "ism_attn_prefill_append_rope": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
+                                               C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_int64,
+                                               C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                               C.c_void_p, C.c_size_t, C.c_void_p]),
     "ism_check_status": (C.c_int, [C.c_void_p]),
     "ism_debug_timeout_probe": (C.c_int, [C.c_uint32, C.c_void_p]),
     "ism_status_string": (C.c_char_p, [C.c_int]),
@@ -297,15 +306,53 @@ def bwd(segs: Segments, q, k, v, o, lse, dout, softmax_scale: float, dq=None, dk
     return dq, dk, dv
 
 
-def append_workspace_size(q_new, k_new, softmax_scale: float) -> int:
-    """Workspace bytes ``prefill_append`` needs for this batch and chunk length."""
+def append_workspace_size(q_new, k_new, softmax_scale: float, rope: bool = False) -> int:
+    """Workspace bytes ``prefill_append`` (``prefill_append_rope`` when rope is
+    set) needs for this batch and chunk length."""
     lib = load()
     B, Ln = q_new.shape[0], q_new.shape[1]
     sh = _shape(q_new, k_new, softmax_scale)
     nbytes = C.c_size_t()
-    _check(lib.ism_attn_prefill_append_workspace_size(C.byref(sh), B, Ln, C.byref(nbytes)),
-           "ism_attn_prefill_append_workspace_size")
+    name = "ism_attn_prefill_append_rope_workspace_size" if rope else "ism_attn_prefill_append_workspace_size"
+    _check(getattr(lib, name)(C.byref(sh), B, Ln, C.byref(nbytes)), name)
     return nbytes.value
+
+
+def _rope_struct(cos, sin) -> _Rope:
+    _contig(cos, sin)
+    if cos.dtype != torch.float32 or sin.dtype != torch.float32 or cos.shape != sin.shape or cos.dim() != 2:
+        raise ValueError("rope tables must be float32 [rows, head_dim/2] tensors of one shape")
+    return _Rope(_ptr(cos), _ptr(sin), cos.shape[0])
+
+
+def prefill_append_rope(q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_host, new_seg_end, new_seg_type,
+                        rope_cos, rope_sin, softmax_scale: float, out=None, lse=None, workspace=None):
+    """``prefill_append`` with rotary encoding of the new queries and keys at
+    positions cache_len[b] + j (rotate-half pairs, angles given by the fp32
+    tables rope_cos / rope_sin [rows, D/2]); the caches receive the rotated
+    keys.  Returns (o_new, lse [Hq,B,Ln])."""
+    lib = load()
+    _contig(q_new, k_new, v_new, k_cache, v_cache, cache_len)
+    B, Ln, hq, D = q_new.shape
+    sh = _shape(q_new, k_new, softmax_scale)
+    se = np.ascontiguousarray(new_seg_end, dtype=np.int32)
+    st = np.ascontiguousarray(new_seg_type, dtype=np.uint8)
+    ch = np.ascontiguousarray(cache_len_host, dtype=np.int32)
+    rope = _rope_struct(rope_cos, rope_sin)
+    nbytes = append_workspace_size(q_new, k_new, softmax_scale, rope=True)
+    if out is None:
+        out = torch.empty_like(q_new)
+    if lse is None:
+        lse = torch.empty((hq, B, Ln), dtype=torch.float32, device=q_new.device)
+    if workspace is None or workspace.numel() < nbytes:
+        workspace = _workspace(nbytes, q_new.device)
+    _check(lib.ism_attn_prefill_append_rope(C.byref(sh), B, _ptr(q_new), _ptr(k_new), _ptr(v_new), Ln,
+                                            C.c_void_p(se.ctypes.data), C.c_void_p(st.ctypes.data), se.shape[0],
+                                            _ptr(k_cache), _ptr(v_cache), k_cache.shape[1], _ptr(cache_len),
+                                            C.c_void_p(ch.ctypes.data), C.byref(rope), _ptr(out), _ptr(lse),
+                                            _ptr(workspace), workspace.numel(), _stream(q_new.device)),
+           "ism_attn_prefill_append_rope")
+    return out, lse
 
 
 def prefill_append(q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_host, new_seg_end, new_seg_type,
@@ -348,7 +395,7 @@ class AppendStep:
     place after it (the device ``cache_len`` advances itself)."""
 
     def __init__(self, q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_host: np.ndarray, new_seg_end,
-                 new_seg_type, softmax_scale: float, out=None, lse=None, workspace=None):
+                 new_seg_type, softmax_scale: float, out=None, lse=None, workspace=None, rope=None):
         lib = load()
         _contig(q_new, k_new, v_new, k_cache, v_cache, cache_len)
         if not (isinstance(cache_len_host, np.ndarray) and cache_len_host.dtype == np.int32 and
@@ -362,17 +409,25 @@ class AppendStep:
         self.out = torch.empty_like(q_new) if out is None else out
         self.lse = torch.empty((hq, B, Ln), dtype=torch.float32, device=q_new.device) if lse is None else lse
         if workspace is None:
-            workspace = _workspace(append_workspace_size(q_new, k_new, softmax_scale), q_new.device)
-        self._keep = (q_new, k_new, v_new, k_cache, v_cache, cache_len, workspace)
-        self._fn = lib.ism_attn_prefill_append
-        self._args = (C.byref(self._sh), B, _ptr(q_new), _ptr(k_new), _ptr(v_new), Ln,
-                      C.c_void_p(self._se.ctypes.data), C.c_void_p(self._st.ctypes.data), self._se.shape[0],
-                      _ptr(k_cache), _ptr(v_cache), k_cache.shape[1], _ptr(cache_len),
-                      C.c_void_p(cache_len_host.ctypes.data), _ptr(self.out), _ptr(self.lse), _ptr(workspace),
-                      workspace.numel(), _stream(q_new.device))
+            workspace = _workspace(append_workspace_size(q_new, k_new, softmax_scale, rope=rope is not None),
+                                   q_new.device)
+        self._keep = (q_new, k_new, v_new, k_cache, v_cache, cache_len, workspace, rope)
+        head = (C.byref(self._sh), B, _ptr(q_new), _ptr(k_new), _ptr(v_new), Ln,
+                C.c_void_p(self._se.ctypes.data), C.c_void_p(self._st.ctypes.data), self._se.shape[0],
+                _ptr(k_cache), _ptr(v_cache), k_cache.shape[1], _ptr(cache_len),
+                C.c_void_p(cache_len_host.ctypes.data))
+        tail = (_ptr(self.out), _ptr(self.lse), _ptr(workspace), workspace.numel(), _stream(q_new.device))
+        if rope is None:
+            self._name = "ism_attn_prefill_append"
+            self._args = head + tail
+        else:
+            self._rope = _rope_struct(*rope)
+            self._name = "ism_attn_prefill_append_rope"
+            self._args = head + (C.byref(self._rope),) + tail
+        self._fn = getattr(lib, self._name)
 
     def __call__(self):
-        _check(self._fn(*self._args), "ism_attn_prefill_append")
+        _check(self._fn(*self._args), self._name)
         return self.out, self.lse
 
 

@@ -164,6 +164,33 @@ def test_paged_append_errors(lib):
     assert call(num_pages=0) == 1
 
 
+class _Rope(C.Structure):
+    _fields_ = [("cos", C.c_void_p), ("sin", C.c_void_p), ("rows", C.c_int32)]
+
+
+def test_rope_append_errors(lib):
+    se = np.array([4, 8], np.int32)
+    st = np.array([0, 1], np.uint8)
+    ch = np.array([10, 20], np.int32)
+
+    def call(rope, sh=None):
+        sh = _shape() if sh is None else sh
+        return lib.ism_attn_prefill_append_rope(C.byref(sh), 2, FAKE, FAKE, FAKE, 8, se.ctypes.data, st.ctypes.data,
+                                                2, FAKE, FAKE, 64, FAKE, ch.ctypes.data,
+                                                None if rope is None else C.byref(rope), FAKE, None, FAKE, 1 << 30,
+                                                None)
+    assert call(None) == 1 and "rope is NULL" in lib.ism_last_error().decode()
+    assert call(_Rope(FAKE, FAKE, 28), sh=_shape(dtype=1)) == 1          # bf16 only
+    assert call(_Rope(FAKE + 4, FAKE, 28)) == 1                          # misaligned table
+    assert call(_Rope(None, FAKE, 28)) == 1
+    assert call(_Rope(FAKE, FAKE, 27)) == 1                              # positions up to 20 + 8
+    assert "rope tables cover 27" in lib.ism_last_error().decode()
+    need, base = C.c_size_t(), C.c_size_t()
+    assert lib.ism_attn_prefill_append_rope_workspace_size(C.byref(_shape()), 2, 8, C.byref(need)) == 0
+    assert lib.ism_attn_prefill_append_workspace_size(C.byref(_shape()), 2, 8, C.byref(base)) == 0
+    assert need.value >= base.value + 2 * 8 * 4 * 128 * 2                # plus the rotated queries
+
+
 def test_e4m3_entry_errors(lib):
     keep = _Keep()
     s = _segs([0, 10], [0, 2], [4, 10], [0, 1], keep)

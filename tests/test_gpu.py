@@ -642,3 +642,132 @@ def test_append_step_matches_prefill_append(ism):
         ism.check_status()
         outs.append(torch.stack(got))
     assert torch.equal(outs[0], outs[1])
+
+
+# ---------------------------------------------------------------- rotary encoding on append
+
+def _bf16_round(x):
+    return torch.from_numpy(np.ascontiguousarray(x)).to(torch.bfloat16).to(torch.float64).numpy()
+
+
+def _rope_tables(rows, d, kind, seed):
+    if kind == "schedule":
+        c, s = wl.rope_tables(rows, d)
+    else:  # any angles: the kernel reads the tables, it assumes no schedule
+        rng = np.random.Generator(np.random.PCG64(seed))
+        ang = rng.uniform(-np.pi, np.pi, size=(rows, d // 2))
+        c, s = np.cos(ang).astype(np.float32), np.sin(ang).astype(np.float32)
+    return torch.from_numpy(c), torch.from_numpy(s)
+
+
+def _check_rotated_keys(name, got, ref):
+    # the kernel rotates in fp32 and rounds once to bf16; the oracle rotates in
+    # fp64, so the two differ by at most half a bf16 ulp of the result (2^-8
+    # relative) plus the fp32 rotation error
+    got = _np(got)
+    err = np.abs(got - ref)
+    bound = 2.0 ** -8 * np.abs(ref) + 2e-6
+    assert np.all(err <= bound), f"{name}: worst excess {np.max(err - bound):.3e}"
+
+
+@pytest.mark.parametrize("l_new,segs,hq,hkv,d,kind", [
+    (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2, 128, "schedule"),
+    (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2, 128, "random"),
+    (37, ([37], [0]), 6, 2, 128, "random"),
+    (150, ([50, 150], [0, 1]), 4, 2, 64, "random"),
+    (1, ([1], [1]), 8, 2, 128, "schedule"),
+    (1, ([1], [1]), 32, 8, 64, "random")])
+def test_prefill_append_rope(ism, l_new, segs, hq, hkv, d, kind):
+    B = 3
+    c_lens = np.array([0, 77, 300], dtype=np.int32)
+    cap = 300 + l_new + 5
+    kc, vc, qn, kn, vn = _append_inputs(B, cap, c_lens, l_new, hq, hkv, d, seed=l_new + 100)
+    cos_t, sin_t = _rope_tables(300 + l_new, d, kind, seed=l_new + d)   # exactly the positions written
+    kcd, vcd = kc.to(DEV), vc.to(DEV)
+    cl = torch.from_numpy(c_lens.copy()).to(DEV)
+    scale = d ** -0.5
+    o, lse = ism.prefill_append_rope(qn.to(DEV), kn.to(DEV), vn.to(DEV), kcd, vcd, cl, c_lens, segs[0], segs[1],
+                                     cos_t.to(DEV), sin_t.to(DEV), scale)
+    ism.check_status()
+    assert cl.cpu().numpy().tolist() == (c_lens + l_new).tolist()
+    o_ref, lse_ref, k_rot = orc.prefill_append_rope(qn, kn, vn, kc, vc, c_lens, segs[0], segs[1], cos_t.numpy(),
+                                                    sin_t.numpy(), scale, key_round=_bf16_round)
+    for b in range(B):
+        c = int(c_lens[b])
+        _check_rotated_keys(f"cached keys of sequence {b}", kcd[b, c:c + l_new], k_rot[b])
+        assert torch.equal(vcd[b, c:c + l_new].cpu(), vn[b])
+        assert torch.equal(kcd[b, :c].cpu(), kc[b, :c]) and torch.equal(kcd[b, c + l_new:].cpu(), kc[b, c + l_new:])
+    _cmp("o_new", o, o_ref, "bf16")
+    _cmp_lse("lse_new", lse, np.transpose(lse_ref, (1, 0, 2)), "bf16")
+
+
+def test_rope_turns_equal_one_pass_over_rotated_dialogue(ism):
+    # a prefill of the first turn and then single-token decode steps, all with
+    # rotary encoding, give the rows the one-pass forward computes on the
+    # dialogue whose queries and keys the oracle rotated at their positions
+    hq, hkv, d = 8, 2, 128
+    t1 = ([70, 300], [0, 1])
+    steps = 5
+    L = t1[0][-1] + steps
+    full = wl.pack([(t1[0] + [L], t1[1] + [1])])
+    w = wl.Workload("rope", full, hq, hkv, d, "bf16", d ** -0.5, 0.5, 29)
+    q, k, v, _ = wl.attention_tensors(w)
+    cos_t, sin_t = _rope_tables(L, d, "schedule", 0)
+    pos = np.arange(L)
+    qr = torch.from_numpy(_bf16_round(orc.rope_rotate(q, pos, cos_t.numpy(), sin_t.numpy()))).to(torch.bfloat16)
+    kr = torch.from_numpy(_bf16_round(orc.rope_rotate(k, pos, cos_t.numpy(), sin_t.numpy()))).to(torch.bfloat16)
+    o_full, _ = ism.fwd(ism.Segments.from_workload(full, DEV), qr.to(DEV), kr.to(DEV), v.to(DEV), w.softmax_scale)
+    kcd = torch.zeros((1, L, hkv, d), dtype=torch.bfloat16, device=DEV)
+    vcd = torch.zeros_like(kcd)
+    c_host = np.zeros(1, dtype=np.int32)
+    cl = torch.zeros(1, dtype=torch.int32, device=DEV)
+    cd, sd = cos_t.to(DEV), sin_t.to(DEV)
+    chunks = [(0, t1[0][-1], t1)] + [(t1[0][-1] + i, 1, ([1], [1])) for i in range(steps)]
+    for s0, n, sg in chunks:
+        o, _ = ism.prefill_append_rope(q[None, s0:s0 + n].contiguous().to(DEV), k[None, s0:s0 + n].contiguous().to(DEV),
+                                       v[None, s0:s0 + n].contiguous().to(DEV), kcd, vcd, cl, c_host, sg[0], sg[1],
+                                       cd, sd, w.softmax_scale)
+        diff = (o[0].float() - o_full[s0:s0 + n].float()).abs().max().item()
+        assert diff <= 2e-2, (s0, diff)
+        c_host = c_host + n
+    ism.check_status()
+    assert (kcd[0].float() - kr.to(DEV).float()).abs().max().item() <= 2.0 ** -6   # at most one bf16 ulp at |x| < 4
+
+
+def test_append_16k_rope_prefill_sampled(ism):
+    """The 8 x 16K cache with a 512-token query appended under rotary
+    encoding: every stored key against the oracle's rotation, and the
+    attention rows of one (sequence, KV group)."""
+    a = wl.append_16k()
+    B, cap, hq, hkv, d = a.batch, a.capacity, a.num_heads_q, a.num_heads_kv, a.head_dim
+    rng = np.random.Generator(np.random.PCG64(a.seed + 50))
+    kcd = torch.empty((B, cap, hkv, d), dtype=torch.bfloat16, device=DEV)
+    vcd = torch.empty_like(kcd)
+    b, g = 6, 5
+    hs = list(range(g * hq // hkv, (g + 1) * hq // hkv))
+    for bb in range(B):
+        kh = wl.round_to(wl.normal(rng, (cap, hkv, d), a.value_std), "bf16")
+        vh = wl.round_to(wl.normal(rng, (cap, hkv, d), a.value_std), "bf16")
+        kcd[bb], vcd[bb] = kh.to(DEV), vh.to(DEV)
+        if bb == b:
+            kb = kh[:, g:g + 1].clone()
+            vb = vh[:, g:g + 1].clone()
+    qn = wl.round_to(wl.normal(rng, (B, a.l_new, hq, d), a.value_std), "bf16")
+    kn = wl.round_to(wl.normal(rng, (B, a.l_new, hkv, d), a.value_std), "bf16")
+    vn = wl.round_to(wl.normal(rng, (B, a.l_new, hkv, d), a.value_std), "bf16")
+    cos_t, sin_t = _rope_tables(cap, d, "schedule", 0)
+    c_host = a.cache_len.copy()
+    cl = torch.from_numpy(c_host.copy()).to(DEV)
+    o, lse = ism.prefill_append_rope(qn.to(DEV), kn.to(DEV), vn.to(DEV), kcd, vcd, cl, c_host, a.new_seg_end,
+                                     a.new_seg_type, cos_t.to(DEV), sin_t.to(DEV), a.softmax_scale)
+    ism.check_status()
+    c = int(c_host[0])
+    pos = c + np.arange(a.l_new)
+    for bb in range(B):
+        _check_rotated_keys(f"stored keys of sequence {bb}", kcd[bb, c:c + a.l_new],
+                            orc.rope_rotate(kn[bb], pos, cos_t.numpy(), sin_t.numpy()))
+    o_ref, lse_ref, _ = orc.prefill_append_rope(qn[b:b + 1, :, hs], kn[b:b + 1, :, g:g + 1], vn[b:b + 1, :, g:g + 1],
+                                                kb[None], vb[None], c_host[b:b + 1], a.new_seg_end, a.new_seg_type,
+                                                cos_t.numpy(), sin_t.numpy(), a.softmax_scale, key_round=_bf16_round)
+    _cmp("prefill o", o[b:b + 1, :, hs], o_ref, "bf16")
+    _cmp_lse("prefill lse", lse[hs][:, b:b + 1], np.transpose(lse_ref, (1, 0, 2)), "bf16")
