@@ -91,6 +91,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t it = 0;  // stage uses so far, across items
     uint32_t nf[kStages] = {0, 0, 0};
     bool ok = true;
+    // each dS tile is read once; K tiles are read by every query tile and head
+    // of their sequence, so keep them in L2 ahead of the dS stream
+    const uint64_t pol_ds = ptx::l2_policy_evict_first(), pol_k = ptx::l2_policy_evict_last();
     for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
       const Item x = decode(a, item);
       for (int c = 0; c < x.nkb; ++c, ++it) {
@@ -107,9 +110,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int32_t yk = x.w.k_base + c * kRows;
           uint8_t* st = smem + s * kStageBytes;
           ptx::mbar_expect_tx(&bar->full[s], kStageBytes);
-          ptx::bulk_load(st, static_cast<const uint8_t*>(a.ds) + slot * kTileBytes, kTileBytes, &bar->full[s]);
-          ptx::tma_load_2d(st + kTileBytes, &tmK, &bar->full[s], x.g * kD, yk);
-          ptx::tma_load_2d(st + kTileBytes + kHalfBytes, &tmK, &bar->full[s], x.g * kD + 64, yk);
+          ptx::bulk_load_hint(st, static_cast<const uint8_t*>(a.ds) + slot * kTileBytes, kTileBytes, &bar->full[s],
+                              pol_ds);
+          ptx::tma_load_2d_hint(st + kTileBytes, &tmK, &bar->full[s], x.g * kD, yk, pol_k);
+          ptx::tma_load_2d_hint(st + kTileBytes + kHalfBytes, &tmK, &bar->full[s], x.g * kD + 64, yk, pol_k);
         }
         __syncwarp();
         ++nf[s];
