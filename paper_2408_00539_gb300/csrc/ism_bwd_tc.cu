@@ -720,6 +720,9 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
     const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
     const uint32_t tS = tmem + lane_addr + TM_S + 64u * wg, tP = tmem + lane_addr + TM_DP + 64u * wg;
     const float sl2 = a.scale * kLog2e;
+    // the stored dS is read back only by the dQ GEMM, after this kernel: its
+    // lines go first when L2 needs room, ahead of the Q / dO tiles other CTAs reuse
+    const uint64_t pol_ds = ptx::l2_policy_evict_first();
     bool ok = true;
     uint32_t I = 0, nacc = 0;
     Item x;
@@ -787,8 +790,9 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
         if (ds_dst) {
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            ds_dst[(k + 4) * kRows] =
-                make_uint4(ds_rest[4 * k], ds_rest[4 * k + 1], ds_rest[4 * k + 2], ds_rest[4 * k + 3]);
+            ptx::st_global_v4_hint(ds_dst + (k + 4) * kRows,
+                                   make_uint4(ds_rest[4 * k], ds_rest[4 * k + 1], ds_rest[4 * k + 2], ds_rest[4 * k + 3]),
+                                   pol_ds);
           ds_dst = nullptr;
         }
         // phase 2: dS from dP^T
@@ -832,7 +836,8 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
           uint4* dst = reinterpret_cast<uint4*>(static_cast<uint8_t*>(a.ds) + slot * kTileBytes) + wg * 8 * kRows + r;
 #pragma unroll
           for (int k = 0; k < 4; ++k)
-            dst[k * kRows] = make_uint4(pd[4 * k], pd[4 * k + 1], pd[4 * k + 2], pd[4 * k + 3]);
+            ptx::st_global_v4_hint(dst + k * kRows, make_uint4(pd[4 * k], pd[4 * k + 1], pd[4 * k + 2], pd[4 * k + 3]),
+                                   pol_ds);
 #pragma unroll
           for (int k = 0; k < 16; ++k) ds_rest[k] = pd[16 + k];
           ds_dst = dst;
@@ -841,7 +846,9 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
       if (ds_dst) {
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          ds_dst[(k + 4) * kRows] = make_uint4(ds_rest[4 * k], ds_rest[4 * k + 1], ds_rest[4 * k + 2], ds_rest[4 * k + 3]);
+          ptx::st_global_v4_hint(ds_dst + (k + 4) * kRows,
+                                 make_uint4(ds_rest[4 * k], ds_rest[4 * k + 1], ds_rest[4 * k + 2], ds_rest[4 * k + 3]),
+                                 pol_ds);
       }
       if (!ok) break;
       // epilogue of the item: dV, dK from tensor memory
