@@ -225,6 +225,12 @@ ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
  *   o_new [B, l_new, Hq, D] (dtype, written); lse_new [Hq, B, l_new] fp32 or NULL.
  * If a cache ends inside a query segment its old rows would differ from a
  * full pass once the segment grows; the new rows are still exact.
+ * The attention reads the cache in tiles of 128 keys from key 0; so that rows
+ * past the new end never reach the P V contraction with NaN or Inf bit
+ * patterns, the call also sets v_cache rows [cache_len[b] + l_new,
+ * round_up(cache_len[b] + l_new, 128)) to zero (within the capacity; the same
+ * holds for the paged, e4m3 and RoPE appends).  Nothing else past the new end
+ * is read or written.
  * ------------------------------------------------------------------------- */
 ism_status_t ism_attn_prefill_append_workspace_size(const ism_attn_shape_t* shape, int32_t batch,
                                                     int32_t l_new, size_t* bytes);

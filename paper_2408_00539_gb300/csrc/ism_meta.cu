@@ -327,6 +327,33 @@ __global__ void append_plan_kernel(AppendSegs sg, int batch, int64_t kbase_strid
 
 // K_new/V_new rows into the caches at [c_snap[b], c_snap[b] + l_new) (rows of
 // sequence b from b * cap, or through the page table).
+// The attention kernels read keys in tiles of 128 from key 0, so the last
+// tile of a sequence runs past its last key.  Masked keys get P = 0, but the
+// P V contraction still multiplies those rows of V, and unwritten cache
+// memory may hold NaN or Inf bit patterns (0 * NaN = NaN).  Value rows
+// [c + l_new, round_up(c + l_new, 128)) are therefore set to zero by every
+// cache write (clipped to the capacity of a contiguous cache; a paged tile
+// lies within one page).  Keys need no such care: masked scores are replaced,
+// not multiplied.
+__device__ __forceinline__ void zero_value_tail(int batch, int l_new, int vec_per_row, int64_t cap,
+                                                const KvPages& pages, const int32_t* __restrict__ c_snap,
+                                                uint4* v_cache) {
+  const int64_t total = (int64_t)batch * 128 * vec_per_row;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t row = i / vec_per_row;
+    const int col = (int)(i % vec_per_row);
+    const int b = (int)(row / 128);
+    const int64_t end = (int64_t)c_snap[b] + l_new;
+    const int64_t p = end + row % 128;
+    int64_t stop = (end + 127) / 128 * 128;
+    if (!pages.table && stop > cap) stop = cap;
+    if (p >= stop) continue;
+    const int64_t dst = (pages.table ? paged_row(pages, b, p) : (int64_t)b * cap + p) * vec_per_row + col;
+    v_cache[dst] = make_uint4(0u, 0u, 0u, 0u);
+  }
+}
+
 __global__ void cache_write_kernel(int batch, int l_new, int row_bytes, int64_t cap, KvPages pages,
                                    const int32_t* __restrict__ c_snap, const uint4* __restrict__ k_new,
                                    const uint4* __restrict__ v_new, uint4* k_cache, uint4* v_cache) {
@@ -343,6 +370,7 @@ __global__ void cache_write_kernel(int batch, int l_new, int row_bytes, int64_t 
     k_cache[dst] = k_new[i];
     v_cache[dst] = v_new[i];
   }
+  zero_value_tail(batch, l_new, vec_per_row, cap, pages, c_snap, v_cache);
 }
 
 // Rotary encoding fused with the cache write.  One thread takes eight
@@ -412,6 +440,7 @@ __global__ void rope_cache_write_kernel(int batch, int l_new, int hq, int hkv, i
     *reinterpret_cast<uint4*>(dst + k0) = out_lo;
     *reinterpret_cast<uint4*>(dst + half + k0) = out_hi;
   }
+  zero_value_tail(batch, l_new, hkv * d / 8, cap, pages, c_snap, reinterpret_cast<uint4*>(v_cache));
 }
 
 }  // namespace
@@ -488,6 +517,8 @@ cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, 
   int row_bytes = hkv * d * elem;
   int64_t total = (int64_t)batch * l_new * (row_bytes / 16);
   if (total == 0) return cudaSuccess;
+  const int64_t tail = (int64_t)batch * 128 * (row_bytes / 16);  // value rows zeroed past the new end
+  if (tail > total) total = tail;
   int grid = (int)((total + 255) / 256);
   if (grid > 152 * 16) grid = 152 * 16;
   cache_write_kernel<<<grid, 256, 0, st>>>(batch, l_new, row_bytes, cap, pages, c_snap, (const uint4*)k_new,
@@ -499,8 +530,10 @@ cudaError_t launch_rope_cache_write(int batch, int l_new, int hq, int hkv, int d
                                    const KvPages& pages, const int32_t* c_snap, const void* q_new,
                                    const void* k_new, const void* v_new, const float* cos_t, const float* sin_t,
                                    void* q_rot, void* k_cache, void* v_cache, cudaStream_t st) {
-  const int64_t total = (int64_t)batch * l_new * (hq + 2 * hkv) * (d / 16);
+  int64_t total = (int64_t)batch * l_new * (hq + 2 * hkv) * (d / 16);
   if (total == 0) return cudaSuccess;
+  const int64_t tail = (int64_t)batch * 128 * (hkv * d / 8);  // value rows zeroed past the new end
+  if (tail > total) total = tail;
   int grid = (int)((total + 255) / 256);
   if (grid > 152 * 16) grid = 152 * 16;
   rope_cache_write_kernel<<<grid, 256, 0, st>>>(

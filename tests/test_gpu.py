@@ -771,3 +771,90 @@ def test_append_16k_rope_prefill_sampled(ism):
                                                 cos_t.numpy(), sin_t.numpy(), a.softmax_scale, key_round=_bf16_round)
     _cmp("prefill o", o[b:b + 1, :, hs], o_ref, "bf16")
     _cmp_lse("prefill lse", lse[hs][:, b:b + 1], np.transpose(lse_ref, (1, 0, 2)), "bf16")
+
+
+# ---------------------------------------------------------------- garbage past the cached keys
+
+def _poison_past(cache, c_lens, extra_cols=0):
+    # NaN and Inf bit patterns in every row at or past cache_len[b] (unwritten
+    # cache memory may hold anything)
+    bad = torch.tensor([float("nan"), float("inf"), float("-inf")], dtype=cache.dtype)
+    for b in range(cache.shape[0]):
+        c = int(c_lens[b])
+        n = cache.shape[1] - c
+        if n > 0:
+            idx = torch.arange(n * int(np.prod(cache.shape[2:]))) % 3
+            cache[b, c:] = bad[idx].reshape((n,) + tuple(cache.shape[2:]))
+    return cache
+
+
+@pytest.mark.parametrize("l_new,segs,hq,hkv,d,cap_extra", [
+    (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2, 128, 5),     # capacity not a multiple of 128
+    (64, ([64], [0]), 4, 4, 128, 100),
+    (1, ([1], [1]), 8, 2, 128, 3),
+    (1, ([1], [1]), 4, 4, 128, 60),                                # one query head per KV head
+    (1, ([1], [1]), 40, 2, 128, 7),                                # forward kernels for the step
+    (150, ([50, 150], [0, 1]), 4, 2, 64, 9)])
+def test_append_ignores_garbage_past_cache_len(ism, l_new, segs, hq, hkv, d, cap_extra):
+    B = 3
+    c_lens = np.array([0, 77, 300], dtype=np.int32)
+    cap = 300 + l_new + cap_extra
+    kc, vc, qn, kn, vn = _append_inputs(B, cap, c_lens, l_new, hq, hkv, d, seed=l_new + 7)
+    kc, vc = _poison_past(kc.clone(), c_lens), _poison_past(vc.clone(), c_lens)
+    kcd, vcd = kc.to(DEV), vc.to(DEV)
+    cl = torch.from_numpy(c_lens.copy()).to(DEV)
+    scale = d ** -0.5
+    o, lse = ism.prefill_append(qn.to(DEV), kn.to(DEV), vn.to(DEV), kcd, vcd, cl, c_lens, segs[0], segs[1], scale)
+    ism.check_status()
+    o_ref, lse_ref = orc.prefill_append(qn, kn, vn, kc, vc, c_lens, segs[0], segs[1], scale)
+    _cmp("o_new", o, o_ref, "bf16")
+    _cmp_lse("lse_new", lse, np.transpose(lse_ref, (1, 0, 2)), "bf16")
+    # the documented side effect: value rows up to the next 128-key boundary
+    # are zeroed, every other row past the new end is left as it was
+    for b in range(B):
+        e = int(c_lens[b]) + l_new
+        stop = min((e + 127) // 128 * 128, cap)
+        assert bool((vcd[b, e:stop] == 0).all())
+        assert torch.equal(vcd[b, stop:].cpu().view(torch.int16), vc[b, stop:].view(torch.int16))
+        assert torch.equal(kcd[b, e:].cpu().view(torch.int16), kc[b, e:].view(torch.int16))
+
+
+def test_paged_and_e4m3_appends_ignore_garbage(ism):
+    B, hq, hkv, d, l_new, ps = 2, 8, 2, 128, 90, 256
+    c_lens = np.array([30, 300], dtype=np.int32)
+    cap = 512
+    kc, vc, qn, kn, vn = _append_inputs(B, cap, c_lens, l_new, hq, hkv, d, seed=77)
+    segs = ([20, 90], [0, 1])
+    scale = d ** -0.5
+    o_ref, _ = orc.prefill_append(qn, kn, vn, kc, vc, c_lens, segs[0], segs[1], scale)
+    # paged: pages of the two sequences interleaved in one pool, garbage past each length
+    kcp, vcp = _poison_past(kc.clone(), c_lens), _poison_past(vc.clone(), c_lens)
+    table = np.array([[3, 0], [1, 2]], dtype=np.int32)
+    kp = torch.empty((4 * ps, hkv, d), dtype=torch.bfloat16)
+    vp = torch.empty_like(kp)
+    for b in range(B):
+        for pg in range(2):
+            kp[table[b, pg] * ps:(table[b, pg] + 1) * ps] = kcp[b, pg * ps:(pg + 1) * ps]
+            vp[table[b, pg] * ps:(table[b, pg] + 1) * ps] = vcp[b, pg * ps:(pg + 1) * ps]
+    cl = torch.from_numpy(c_lens.copy()).to(DEV)
+    o, _ = ism.prefill_append_paged(qn.to(DEV), kn.to(DEV), vn.to(DEV), kp.to(DEV), vp.to(DEV), ps,
+                                    torch.from_numpy(table).to(DEV), table, cl, c_lens, segs[0], segs[1], scale)
+    ism.check_status()
+    _cmp("paged o_new", o, o_ref, "bf16")
+    # e4m3 caches: the e4m3 NaN pattern (0x7f) past each length
+    k8, kd_ = wl.quantize_e4m3(torch.cat([kc, kn], 1))
+    v8, vd_ = wl.quantize_e4m3(torch.cat([vc, vn], 1))
+    q8, qd_ = wl.quantize_e4m3(qn)
+    kc8, kn8 = k8[:, :cap].contiguous(), k8[:, cap:].contiguous()
+    vc8, vn8 = v8[:, :cap].contiguous(), v8[:, cap:].contiguous()
+    for b in range(B):
+        kc8.view(torch.uint8)[b, c_lens[b]:] = 0x7F
+        vc8.view(torch.uint8)[b, c_lens[b]:] = 0x7F
+    deq = lambda t, s: t.float() * s
+    o8_ref, _ = orc.prefill_append(deq(q8, qd_), deq(kn8, kd_), deq(vn8, vd_), deq(kc8, kd_), deq(vc8, vd_), c_lens,
+                                   segs[0], segs[1], scale)
+    cl = torch.from_numpy(c_lens.copy()).to(DEV)
+    o8, _ = ism.prefill_append_e4m3(q8.to(DEV), kn8.to(DEV), vn8.to(DEV), kc8.to(DEV), vc8.to(DEV), cl, c_lens,
+                                    segs[0], segs[1], qd_, kd_, vd_, scale)
+    ism.check_status()
+    _cmp_e4m3("e4m3 o_new", o8, o8_ref, float(torch.cat([vc, vn], 1).float().abs().max()))
