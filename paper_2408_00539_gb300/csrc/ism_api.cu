@@ -685,12 +685,38 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
     if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
       sms = 152;
     const char* no_tma = getenv("ISM_DECODE_NO_TMA");
+    const char* no_tc = getenv("ISM_DECODE_NO_TC");
     a.tma = (d == 128 && tc_available() && !(no_tma && no_tma[0] == '1')) ? 1 : 0;
-    int64_t want = (a.tma ? 8 * (int64_t)sms : 4 * (int64_t)sms) / pairs;
-    int64_t splits = want < 1 ? 1 : want > kMaxSplits ? kMaxSplits : want;
-    int64_t chunk = (kv_max + splits - 1) / splits;
-    chunk = (chunk + 63) / 64 * 64;
-    splits = (kv_max + chunk - 1) / chunk;
+    a.tc = (a.tma && shape->dtype == ISM_BF16 && !(no_tc && no_tc[0] == '1') &&
+            kv_max <= (int64_t)kMaxSplits * kDecTcMaxKeys)
+               ? 1
+               : 0;
+    int64_t splits, chunk;
+    if (a.tc) {
+      // persistent tensor-core kernel: the split count that minimises the
+      // busiest CTA's work, (items per CTA) x (128-key tiles per item + 1 for
+      // the item's hand-offs), over chunks of whole tiles up to kDecTcMaxKeys
+      int64_t best = -1;
+      splits = chunk = 0;
+      for (int64_t sp = 1; sp <= kMaxSplits; ++sp) {
+        const int64_t ch = ((kv_max + sp - 1) / sp + 127) / 128 * 128;
+        if (ch > kDecTcMaxKeys) continue;
+        const int64_t used = (kv_max + ch - 1) / ch;
+        const int64_t per_cta = (pairs * used + sms - 1) / sms;
+        const int64_t cost = per_cta * (ch / 128 + 1);
+        if (best < 0 || cost < best) {
+          best = cost;
+          splits = used;
+          chunk = ch;
+        }
+      }
+    } else {
+      int64_t want = (a.tma ? 8 * (int64_t)sms : 4 * (int64_t)sms) / pairs;
+      splits = want < 1 ? 1 : want > kMaxSplits ? kMaxSplits : want;
+      chunk = (kv_max + splits - 1) / splits;
+      chunk = (chunk + 63) / 64 * 64;
+      splits = (kv_max + chunk - 1) / chunk;
+    }
     a.splits = (int32_t)splits;
     a.chunk = (int32_t)chunk;
     a.part_o = L.part_o; a.part_ml = L.part_ml;

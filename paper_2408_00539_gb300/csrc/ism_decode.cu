@@ -494,6 +494,12 @@ cudaError_t run_d(const DecodeArgs& a, cudaStream_t st) {
 
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st) {
   if (a.batch == 0) return cudaSuccess;
+  if (a.tc) {
+    cudaError_t e = tc::launch_decode_tc(a, st);
+    if (e != cudaSuccess) return e;
+    decode_combine_kernel<128><<<a.batch * a.hq, 128, 0, st>>>(a);
+    return cudaGetLastError();
+  }
   return a.d == 64 ? run_d<64>(a, st) : run_d<128>(a, st);
 }
 

@@ -1,0 +1,419 @@
+// Single-token decode on the tensor cores (sm_103a), bf16 caches, head_dim 128.
+//
+// A decode step (Section 2.3: the new answer token attends to the whole reused
+// cache plus itself) reads every cached key and value of a (sequence, KV head)
+// once, so it is bound by HBM.  The CUDA-core decode spends most of its issue
+// slots on dot products and the reductions that assemble them; here both
+// contractions run on the tensor cores and the threads only do the softmax.
+//
+// Work item: (sequence b, KV head g, split) = keys [k0, k1) of the cache, in
+// tiles of 128 keys.  A persistent CTA per SM walks the items; per item
+//   pass 1: S^T_t = K_t Q^T for every tile t (M = 128 keys, N = 16 query
+//           heads of the group, zero or foreign rows past the group), all
+//           tiles kept in tensor memory (16 columns each);
+//   the exact maximum per head over the item's keys;
+//   pass 2: P_t = exp2(S_t * scale * log2 e - m) as bf16 into a 128-byte
+//           swizzled K-major operand in shared memory (rows = heads), then
+//           O += P_t V_t (M = 128 with the group in rows 0-15, N = 128
+//           dimensions, K = 128 keys; V MN-major as it arrives).
+// With the exact maximum known before any P, no rescaling of O is needed.
+// The item's (max, sum, unnormalised O) per head go to the split partials,
+// which decode_combine_kernel merges as for the CUDA-core kernels.
+// Warps 0-3: softmax and epilogue (thread = key of a tile, TMEM lane);
+// warp 4: TMA loads (Q of the item, then its K tiles, then its V tiles,
+// through one 4-stage ring); warp 5: MMA issue.
+#include "ism_tc_common.cuh"
+
+namespace ism {
+namespace tc {
+namespace {
+
+constexpr int kStages = 4;
+constexpr int kHeadsPad = 16;  // N of S^T = K Q^T
+constexpr int kMaxTiles = kDecTcMaxKeys / 128;
+constexpr uint32_t kQHalf = kHeadsPad * 128;  // one 64-column half of the Q tile: 16 rows x 128 B
+constexpr uint32_t kQBytes = 2 * kQHalf;
+constexpr uint32_t OFF_RING = 0, OFF_P = kStages * kTileBytes, OFF_Q = OFF_P + 2 * kTileBytes,
+                   OFF_BAR = OFF_Q + 2 * kQBytes;
+constexpr uint32_t kSmemBytes = OFF_BAR + 1024 + 1024;  // barrier block + 1024-byte alignment slack
+constexpr int kThreads = 192;
+constexpr int kLoadWarp = 4, kMmaWarp = 5;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t TM_O = 0, TM_S = 128;
+static_assert(TM_S + kHeadsPad * kMaxTiles <= kTmemCols, "S tiles fit in tensor memory");
+static_assert(kSmemBytes <= 232448, "shared memory per CTA");
+
+struct Bars {
+  uint64_t full[kStages], empty[kStages];
+  uint64_t q_full[2], q_empty[2];
+  uint64_t s_full, s_free, p_ready[2], p_free[2], o_full, o_free, final_mma;
+  uint64_t red_m_full, red_l_full;  // the four softmax warps' partial maxima / sums are written
+  uint32_t tmem_base;
+  int32_t abort;
+  float red_m[4][kHeadsPad], red_l[4][kHeadsPad];
+};
+static_assert(sizeof(Bars) <= 1024, "barrier block");
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+__device__ __forceinline__ bool aborted(const int32_t* f) { return *reinterpret_cast<const volatile int32_t*>(f) != 0; }
+__device__ __forceinline__ void set_abort(int32_t* f) { *reinterpret_cast<volatile int32_t*>(f) = 1; }
+
+struct DecItem {
+  int b, g, split, k0, k1, nt;
+};
+// item = (split * hkv + g) * batch + b: consecutive CTAs take the same split
+// of different sequences
+__device__ __forceinline__ DecItem dec_item(const DecodeArgs& a, int64_t item) {
+  DecItem x;
+  x.b = (int)(item % a.batch);
+  const int64_t rest = item / a.batch;
+  x.g = (int)(rest % a.hkv);
+  x.split = (int)(rest / a.hkv);
+  const int kv_len = a.c_snap[x.b] + 1;
+  x.k0 = x.split * a.chunk;
+  x.k1 = min(kv_len, x.k0 + a.chunk);
+  x.nt = x.k1 > x.k0 ? (x.k1 - x.k0 + 127) / 128 : 0;
+  return x;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    decode_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                     const __grid_constant__ CUtensorMap tmV, const DecodeArgs a, int64_t n_items) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = align1024(smem_raw);
+  Bars* bar = reinterpret_cast<Bars*>(smem + OFF_BAR);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      ptx::mbar_init(&bar->full[s], 1);
+      ptx::mbar_init(&bar->empty[s], 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      ptx::mbar_init(&bar->q_full[i], 1);
+      ptx::mbar_init(&bar->q_empty[i], 1);
+      ptx::mbar_init(&bar->p_ready[i], 128);
+      ptx::mbar_init(&bar->p_free[i], 1);
+    }
+    ptx::mbar_init(&bar->s_full, 1);
+    ptx::mbar_init(&bar->s_free, 128);
+    ptx::mbar_init(&bar->o_full, 1);
+    ptx::mbar_init(&bar->o_free, 32);
+    ptx::mbar_init(&bar->final_mma, 1);
+    ptx::mbar_init(&bar->red_m_full, 128);
+    ptx::mbar_init(&bar->red_l_full, 128);
+    bar->abort = 0;
+    ptx::fence_mbar_init();
+  }
+  if (warp == kMmaWarp) {
+    ptx::tmem_alloc(&bar->tmem_base, kTmemCols);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem = bar->tmem_base;
+
+  if (warp == kLoadWarp) {
+    // ------------------------------------------------ TMA loads (the warp waits converged, lane 0 issues)
+    uint32_t nl = 0, nu = 0;  // ring tiles issued; non-empty items
+    uint32_t nf[kStages] = {0, 0, 0, 0}, nq[2] = {0, 0};
+    bool ok = true;
+    const uint64_t pol = ptx::l2_policy_evict_first();  // the cache is streamed once per step
+    if (lane == 0) {
+      ptx::tma_prefetch_desc(&tmK);
+      ptx::tma_prefetch_desc(&tmV);
+    }
+    for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
+      const DecItem x = dec_item(a, item);
+      if (x.nt == 0) continue;
+      const uint32_t qb = nu & 1;
+      if (__any_sync(0xffffffffu, aborted(&bar->abort)) ||
+          (nu >= 2 && !wait_warp(&bar->q_empty[qb], ((nu >> 1) - 1) & 1, a.status))) {
+        ok = false;
+        break;
+      }
+      if (lane == 0) {
+        // the 16 query rows from the group's first head (rows past the group
+        // are other heads' queries or zero fill; their outputs are not used)
+        const int32_t qy = x.b * a.hq + x.g * a.group;
+        uint8_t* dq = smem + OFF_Q + qb * kQBytes;
+        ptx::mbar_expect_tx(&bar->q_full[qb], kQBytes);
+        ptx::tma_load_2d(dq, &tmQ, &bar->q_full[qb], 0, qy);
+        ptx::tma_load_2d(dq + kQHalf, &tmQ, &bar->q_full[qb], 64, qy);
+      }
+      __syncwarp();
+      ++nq[qb];
+      ++nu;
+      for (int pass = 0; ok && pass < 2; ++pass) {
+        const CUtensorMap* map = pass ? &tmV : &tmK;
+        for (int t = 0; t < x.nt; ++t, ++nl) {
+          const uint32_t s = nl % kStages;
+          if (__any_sync(0xffffffffu, aborted(&bar->abort)) ||
+              (nl >= kStages && !wait_warp(&bar->empty[s], ((nl / kStages) - 1) & 1, a.status))) {
+            ok = false;
+            break;
+          }
+          if (lane == 0) {
+            // a tile starts at a multiple of 128 keys and lies in one page
+            const int64_t p = (int64_t)x.k0 + (int64_t)t * 128;
+            const int32_t y = a.pages.table ? (int32_t)paged_row(a.pages, x.b, p) : (int32_t)((int64_t)x.b * a.cap + p);
+            uint8_t* dst = smem + OFF_RING + s * kTileBytes;
+            ptx::mbar_expect_tx(&bar->full[s], kTileBytes);
+            ptx::tma_load_2d_hint(dst, map, &bar->full[s], x.g * kD, y, pol);
+            ptx::tma_load_2d_hint(dst + kHalfBytes, map, &bar->full[s], x.g * kD + 64, y, pol);
+          }
+          __syncwarp();
+          ++nf[s];
+        }
+      }
+    }
+    if (!ok) {
+      if (lane == 0) set_abort(&bar->abort);
+      // every issued copy lands before the CTA exits
+      for (int s = 0; s < kStages; ++s)
+        if (nf[s]) wait_warp(&bar->full[s], (nf[s] - 1) & 1, a.status);
+      for (int i = 0; i < 2; ++i)
+        if (nq[i]) wait_warp(&bar->q_full[i], (nq[i] - 1) & 1, a.status);
+    }
+    __syncwarp();
+  } else if (warp == kMmaWarp) {
+    // ------------------------------------------------ MMA issue (the whole warp runs the loop,
+    // one elected lane issues each instruction)
+    constexpr uint32_t idesc_s = ptx::idesc_bf16_f32(128, kHeadsPad, 0, 0);
+    constexpr uint32_t idesc_pv = ptx::idesc_bf16_f32(128, 128, 0, 1);
+    uint32_t nl = 0, nu = 0, T = 0;  // ring tiles consumed; non-empty items; P tiles
+    bool ok = true;
+    for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
+      const DecItem x = dec_item(a, item);
+      if (x.nt == 0) continue;
+      const uint32_t qb = nu & 1;
+      // Q landed; the softmax warps have read the previous item's S
+      if (!wait_warp(&bar->q_full[qb], (nu >> 1) & 1, a.status) ||
+          (nu >= 1 && !wait_warp(&bar->s_free, (nu - 1) & 1, a.status))) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+      const uint32_t sQ = ptx::smem_u32(smem + OFF_Q + qb * kQBytes);
+      for (int t = 0; t < x.nt; ++t, ++nl) {
+        const uint32_t s = nl % kStages;
+        if (__shfl_sync(0xffffffffu, aborted(&bar->abort) ? 1 : 0, 0) ||
+            !wait_warp(&bar->full[s], (nl / kStages) & 1, a.status)) {
+          ok = false;
+          break;
+        }
+        ptx::tc_fence_after();
+        const uint32_t sK = ptx::smem_u32(smem + OFF_RING + s * kTileBytes);
+        ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128Rows16>(
+            tmem + TM_S + kHeadsPad * (uint32_t)t, desc_kmajor(sK, 0), desc_kmajor(sQ, 0), idesc_s, 0u);
+        ptx::mma_commit_warp(&bar->empty[s]);
+      }
+      if (!ok) break;
+      ptx::mma_commit_warp(&bar->s_full);
+      ptx::mma_commit_warp(&bar->q_empty[qb]);
+      // the epilogue has read the previous item's O
+      if (nu >= 1 && !wait_warp(&bar->o_free, (nu - 1) & 1, a.status)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+      for (int t = 0; t < x.nt; ++t, ++nl, ++T) {
+        const uint32_t s = nl % kStages, pb = T & 1;
+        if (__shfl_sync(0xffffffffu, aborted(&bar->abort) ? 1 : 0, 0) ||
+            !wait_warp(&bar->p_ready[pb], (T >> 1) & 1, a.status) ||
+            !wait_warp(&bar->full[s], (nl / kStages) & 1, a.status)) {
+          ok = false;
+          break;
+        }
+        ptx::tc_fence_after();
+        const uint32_t sP = ptx::smem_u32(smem + OFF_P + pb * kTileBytes);
+        const uint32_t sV = ptx::smem_u32(smem + OFF_RING + s * kTileBytes);
+        ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::MnMajorSw128>(tmem + TM_O, desc_kmajor(sP, 0),
+                                                                   desc_mnmajor(sV, 0), idesc_pv, t > 0 ? 1u : 0u);
+        ptx::mma_commit_warp(&bar->empty[s]);
+        ptx::mma_commit_warp(&bar->p_free[pb]);
+      }
+      if (!ok) break;
+      ptx::mma_commit_warp(&bar->o_full);
+      ++nu;
+    }
+    if (!ok && lane == 0) set_abort(&bar->abort);
+    __syncwarp();
+    ptx::mma_commit_warp(&bar->final_mma);
+    wait_warp(&bar->final_mma, 0, a.status);
+    __syncwarp();
+  } else {
+    // ------------------------------------------------ softmax and epilogue: thread r = key r of a tile
+    const int r = threadIdx.x;
+    const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
+    const float c2 = a.scale * kLog2e;
+    const int group = a.group;
+    uint32_t nu = 0, T = 0;
+    bool ok = true;
+    for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
+      const DecItem x = dec_item(a, item);
+      const int64_t pbase = ((int64_t)x.b * a.hq + (int64_t)x.g * group) * a.splits + x.split;
+      if (x.nt == 0) {
+        // a split past the sequence's keys: a partial the combine skips
+        if (warp == 0 && lane < group) {
+          a.part_ml[(pbase + (int64_t)lane * a.splits) * 2] = -INFINITY;
+          a.part_ml[(pbase + (int64_t)lane * a.splits) * 2 + 1] = 0.f;
+        }
+        continue;
+      }
+      if (!wait(&bar->s_full, nu & 1, a.status)) {
+        ok = false;
+        break;
+      }
+      ptx::tc_fence_after();
+      // pass 1: maximum of the scaled scores per head over the item's keys
+      float mx[kHeadsPad];
+#pragma unroll
+      for (int h = 0; h < kHeadsPad; ++h) mx[h] = -INFINITY;
+      for (int t = 0; t < x.nt; ++t) {
+        uint32_t v[kHeadsPad];
+        ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)t, v);
+        ptx::tmem_ld_wait();
+        ptx::reg_fence(v);
+        if (x.k0 + t * 128 + r < x.k1) {
+#pragma unroll
+          for (int h = 0; h < kHeadsPad; ++h) mx[h] = fmaxf(mx[h], __uint_as_float(v[h]));
+        }
+      }
+#pragma unroll
+      for (int h = 0; h < kHeadsPad; ++h) {
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], o));
+      }
+      if (lane == 0) {
+#pragma unroll
+        for (int h = 0; h < kHeadsPad; ++h) bar->red_m[warp][h] = mx[h];
+      }
+      ptx::mbar_arrive(&bar->red_m_full);
+      if (!wait(&bar->red_m_full, nu & 1, a.status)) {
+        ok = false;
+        break;
+      }
+      float m2[kHeadsPad];  // max of scale * log2(e) * S per head (finite: every item has a key)
+#pragma unroll
+      for (int h = 0; h < kHeadsPad; ++h)
+        m2[h] = fmaxf(fmaxf(bar->red_m[0][h], bar->red_m[1][h]), fmaxf(bar->red_m[2][h], bar->red_m[3][h])) * c2;
+      // pass 2: P as bf16 into the A operand of O += P V (rows = heads, columns = keys)
+      float l[kHeadsPad];
+#pragma unroll
+      for (int h = 0; h < kHeadsPad; ++h) l[h] = 0.f;
+      for (int t = 0; t < x.nt; ++t, ++T) {
+        uint32_t v[kHeadsPad];
+        ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)t, v);
+        ptx::tmem_ld_wait();
+        ptx::reg_fence(v);
+        const bool valid = x.k0 + t * 128 + r < x.k1;
+        const uint32_t pb = T & 1;
+        if (T >= 2 && !wait(&bar->p_free[pb], ((T >> 1) - 1) & 1, a.status)) {
+          ok = false;
+          break;
+        }
+        uint8_t* P = smem + OFF_P + pb * kTileBytes;
+#pragma unroll
+        for (int h = 0; h < kHeadsPad; ++h) {
+          const float p = (valid && h < group) ? ex2(__uint_as_float(v[h]) * c2 - m2[h]) : 0.f;
+          const __nv_bfloat16 pr = __float2bfloat16_rn(p);
+          l[h] += __bfloat162float(pr);  // the sum of the P that enters P V
+          *reinterpret_cast<__nv_bfloat16*>(P + swz_offset((uint32_t)h, (uint32_t)r)) = pr;
+        }
+        ptx::fence_proxy_async_smem();
+        ptx::mbar_arrive(&bar->p_ready[pb]);
+      }
+      if (!ok) break;
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&bar->s_free);
+#pragma unroll
+      for (int h = 0; h < kHeadsPad; ++h) {
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) l[h] += __shfl_xor_sync(0xffffffffu, l[h], o);
+      }
+      if (lane == 0) {
+#pragma unroll
+        for (int h = 0; h < kHeadsPad; ++h) bar->red_l[warp][h] = l[h];
+      }
+      ptx::mbar_arrive(&bar->red_l_full);
+      if (!wait(&bar->red_l_full, nu & 1, a.status)) {
+        ok = false;
+        break;
+      }
+      if (warp == 0) {
+        // epilogue: lane h holds row h of O = the unnormalised output of head h
+        if (!wait(&bar->o_full, nu & 1, a.status)) {
+          ok = false;
+          break;
+        }
+        ptx::tc_fence_after();
+        const bool mine = lane < group;
+        float* dst = a.part_o + (pbase + (int64_t)(mine ? lane : 0) * a.splits) * kD;
+#pragma unroll 1
+        for (int q4 = 0; q4 < 4; ++q4) {
+          uint32_t o[32];
+          ptx::tmem_ld32(tmem + TM_O + 32u * q4, o);
+          ptx::tmem_ld_wait();
+          ptx::reg_fence(o);
+          if (mine) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+              reinterpret_cast<float4*>(dst + 32 * q4)[i] =
+                  make_float4(__uint_as_float(o[4 * i]), __uint_as_float(o[4 * i + 1]), __uint_as_float(o[4 * i + 2]),
+                              __uint_as_float(o[4 * i + 3]));
+          }
+        }
+        if (mine) {
+          float mh = -INFINITY, lh = 0.f;
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            mh = fmaxf(mh, bar->red_m[w][lane]);
+            lh += bar->red_l[w][lane];
+          }
+          a.part_ml[(pbase + (int64_t)lane * a.splits) * 2] = mh * c2;
+          a.part_ml[(pbase + (int64_t)lane * a.splits) * 2 + 1] = lh;
+        }
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(&bar->o_free);
+      }
+      ++nu;
+    }
+    if (!ok) set_abort(&bar->abort);
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (warp == kMmaWarp) {
+    ptx::tc_fence_after();
+    ptx::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t st) {
+  if (a.d != kD || a.dtype != ISM_BF16 || a.group > kHeadsPad || a.chunk % 128 != 0 || a.chunk > kDecTcMaxKeys)
+    return cudaErrorInvalidValue;
+  CUtensorMap tq, tk, tv;
+  cudaError_t e;
+  if ((e = make_tmap_bf16_box(&tq, a.q, (uint64_t)kD, (uint64_t)a.batch * a.hq, kHeadsPad)) != cudaSuccess) return e;
+  if ((e = make_tmap_bf16(&tk, a.k_cache, (uint64_t)a.hkv * kD, (uint64_t)a.kv_rows)) != cudaSuccess) return e;
+  if ((e = make_tmap_bf16(&tv, a.v_cache, (uint64_t)a.hkv * kD, (uint64_t)a.kv_rows)) != cudaSuccess) return e;
+  if ((e = cudaFuncSetAttribute(decode_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
+      cudaSuccess)
+    return e;
+  int dev = 0, sms = 0;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  const int64_t n_items = (int64_t)a.batch * a.hkv * a.splits;
+  int64_t grid = sms < n_items ? sms : n_items;
+  if (grid <= 0) return cudaSuccess;
+  decode_tc_kernel<<<(unsigned)grid, kThreads, kSmemBytes, st>>>(tq, tk, tv, a, n_items);
+  return cudaGetLastError();
+}
+
+}  // namespace tc
+}  // namespace ism

@@ -163,8 +163,12 @@ struct DecodeArgs {
   float* part_o;         // [B, Hq, splits, D]
   float* part_ml;        // [B, Hq, splits, 2]
   int32_t tma;           // stream the cache with TMA (head_dim 128, sm_103)
+  int32_t tc;            // tensor-core kernel (bf16, head_dim 128, group <= 16; chunk a multiple of 128)
   uint32_t* status;      // device status word (bounded waits)
 };
+// Keys one work item of the tensor-core decode covers at most (its scores of
+// 24 tiles of 128 keys stay in tensor memory).
+constexpr int kDecTcMaxKeys = 24 * 128;
 cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st);
 
 // Tensor-core kernels (ism_fwd_tc.cu / ism_bwd_tc.cu), bf16 only.

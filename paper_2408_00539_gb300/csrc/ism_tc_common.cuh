@@ -145,6 +145,8 @@ __device__ __forceinline__ uint64_t desc_ilv_mnmajor(uint32_t tile_saddr, int kk
 
 // Host: 2D bf16 tensor map [rows, cols] with a 64 x 128 box, 128B swizzle.
 cudaError_t make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows);
+// Host: the same with a 64-column x box_rows box (box_rows <= 256).
+cudaError_t make_tmap_bf16_box(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows);
 // Host: 2D bf16 tensor map with a 64-column x box_rows box, no swizzle.
 cudaError_t make_tmap_bf16_plain(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows);
 // 1-byte elements, box of 128 columns x box_rows, no swizzle
@@ -154,6 +156,10 @@ bool available();
 // Host: forward with two query heads (sharing a KV head) per CTA.
 cudaError_t launch_fwd_pair(const AttnArgs& a, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                             cudaStream_t st);
+// Host: single-token decode on the tensor cores (bf16 caches, head_dim 128,
+// at most 16 query heads per KV head; a.chunk a multiple of 128, at most
+// kDecTcMaxKeys): partials for decode_combine_kernel.
+cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t st);
 // Host: dQ as a GEMM over the dS^T tiles stored by the dK/dV kernel (a.ds).
 cudaError_t launch_dq_gemm(const AttnArgs& a, const CUtensorMap& tk, cudaStream_t st);
 

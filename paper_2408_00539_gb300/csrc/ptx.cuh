@@ -212,12 +212,15 @@ __device__ __forceinline__ void mma_bf16_ts_warp(uint32_t d_tmem, uint32_t a_tme
 //   MnMajorIlv8    8-interleaved MN-major, 256 bytes a k-step
 //   TmemPairs      bf16 pairs in tensor memory, 8 columns a k-step
 //   TmemPairsGap32 the same with a 32-column gap after k-step 3
+//   KMajorSw128Rows16  K-major, 128-byte swizzled, 16-row operand (halves 2 KB apart)
 // k-step 0 accumulates when acc != 0, the others always.
 struct KMajorSw128 { static constexpr uint32_t step = 2, half = 1024; };
 struct MnMajorSw128 { static constexpr uint32_t step = 128, half = 512; };
 struct MnMajorIlv8 { static constexpr uint32_t step = 16, half = 64; };
 struct TmemPairs { static constexpr uint32_t step = 8, half = 32; };
 struct TmemPairsGap32 { static constexpr uint32_t step = 8, half = 64; };
+// K-major, 128-byte swizzled, 16 rows: two 64-column halves 2 KB apart
+struct KMajorSw128Rows16 { static constexpr uint32_t step = 2, half = 128; };
 template <class LA, class LB, uint32_t kAStep = LA::step, uint32_t kAHalf = LA::half, uint32_t kBStep = LB::step,
           uint32_t kBHalf = LB::half>
 __device__ __forceinline__ void mma8_bf16_ss_warp(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
@@ -303,6 +306,15 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
       : "r"(taddr));
 }
 
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
   asm volatile(
       "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
@@ -321,6 +333,10 @@ __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.
 __device__ __forceinline__ void reg_fence(uint32_t (&r)[32]) {
 #pragma unroll
   for (int i = 0; i < 32; ++i) asm volatile("" : "+r"(r[i]));
+}
+__device__ __forceinline__ void reg_fence(uint32_t (&r)[16]) {
+#pragma unroll
+  for (int i = 0; i < 16; ++i) asm volatile("" : "+r"(r[i]));
 }
 __device__ __forceinline__ void tmem_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 

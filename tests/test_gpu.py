@@ -271,10 +271,13 @@ def test_prefill_append_matches_one_pass_rows(ism):
     assert diff <= 2e-2, diff
 
 
+@pytest.mark.parametrize("path", ["tensor_cores", "cuda_cores"])
 @pytest.mark.parametrize("hq,hkv", [(8, 2), (4, 4), (8, 1), (4, 2), (6, 2), (10, 2), (7, 1), (16, 1), (40, 2)])
-def test_decode_steps_small(ism, hq, hkv):
-    """Group sizes 1-16 run the decode kernels (padded to a power of two), 20
-    the forward kernels."""
+def test_decode_steps_small(ism, hq, hkv, path, monkeypatch):
+    """Group sizes 1-16 run the decode kernels (the tensor-core kernel, or the
+    CUDA-core ones padded to a power of two), 20 the forward kernels."""
+    if path == "cuda_cores":
+        monkeypatch.setenv("ISM_DECODE_NO_TC", "1")
     B, d, c0, steps = 2, 128, 700, 6
     cap = c0 + steps
     kc, vc, qn, kn, vn = _append_inputs(B, cap, None, steps, hq, hkv, d, seed=31)
