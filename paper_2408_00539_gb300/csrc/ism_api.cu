@@ -648,27 +648,34 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
   const int hq = shape->num_heads_q, hkv = shape->num_heads_kv, d = shape->head_dim;
   const bool paged = cg.pages.table != nullptr;
 
+  // decode kernels serve up to kMaxDecodeGroup query heads per KV head; larger
+  // groups take the forward kernels (one query row per tile)
+  const bool decode = l_new == 1 && (shape->dtype == ISM_BF16 || shape->dtype == ISM_E4M3) && !force_cuda_cores() &&
+                      hq / hkv <= kMaxDecodeGroup;
+  // A single-token step needs no tile plan: the cache write reads the cache
+  // lengths and snapshots them, and the decode's combine kernel advances them.
   timer_begin(ISM_KERNEL_META, st);
-  ISM_TRY_CUDA(launch_append_plan(sg, batch, paged ? 1 : cg.cap, kTile, kTile, cache_len, L.c_snap, L.kv_end, L.qtiles,
-                                  L.q_order, L.pair_order, st),
-               "append plan launch");
+  if (!decode)
+    ISM_TRY_CUDA(launch_append_plan(sg, batch, paged ? 1 : cg.cap, kTile, kTile, cache_len, L.c_snap, L.kv_end,
+                                    L.qtiles, L.q_order, L.pair_order, st),
+                 "append plan launch");
+  const int32_t* c_src = decode ? cache_len : L.c_snap;
+  int32_t* snap_out = decode ? L.c_snap : nullptr;
   if (rope) {
-    ISM_TRY_CUDA(launch_rope_cache_write(batch, l_new, hq, hkv, d, cg.cap, cg.pages, L.c_snap, q_new, k_new, v_new,
-                                         rope->cos, rope->sin, L.q_rot, k_cache, v_cache, st),
+    ISM_TRY_CUDA(launch_rope_cache_write(batch, l_new, hq, hkv, d, cg.cap, cg.pages, c_src, q_new, k_new, v_new,
+                                         rope->cos, rope->sin, L.q_rot, k_cache, v_cache, st, snap_out),
                  "rope cache write launch");
     q_new = L.q_rot;  // the attention below reads the rotated queries
   } else {
-    ISM_TRY_CUDA(launch_cache_write(shape->dtype, batch, l_new, hkv, d, cg.cap, cg.pages, L.c_snap, k_new, v_new,
-                                    k_cache, v_cache, st),
+    ISM_TRY_CUDA(launch_cache_write(shape->dtype, batch, l_new, hkv, d, cg.cap, cg.pages, c_src, k_new, v_new,
+                                    k_cache, v_cache, st, snap_out),
                  "cache write launch");
   }
   timer_end(ISM_KERNEL_META, st);
-  count_launch(2);
-  // decode kernels serve up to kMaxDecodeGroup query heads per KV head; larger
-  // groups take the forward kernels (one query row per tile)
-  if (l_new == 1 && (shape->dtype == ISM_BF16 || shape->dtype == ISM_E4M3) && !force_cuda_cores() &&
-      hq / hkv <= kMaxDecodeGroup) {
+  count_launch(decode ? 1 : 2);
+  if (decode) {
     DecodeArgs a{};
+    a.cache_len = cache_len;
     a.q = q_new; a.k_cache = k_cache; a.v_cache = v_cache; a.pages = cg.pages; a.out = o_new; a.lse = lse_new;
     a.c_snap = L.c_snap;
     a.batch = batch; a.hq = hq; a.hkv = hkv; a.d = d; a.dtype = shape->dtype; a.cap = cg.cap;

@@ -415,9 +415,12 @@ __global__ void __launch_bounds__(160) decode_tma_kernel(const __grid_constant__
   }
 }
 
-// grid B*Hq, block D threads.
+// grid B*Hq, block D threads.  Launched as a programmatic dependent of the
+// split kernel: it may start while that kernel runs and waits for it (and
+// its memory) before reading the partials.
 template <int D>
 __global__ void decode_combine_kernel(DecodeArgs a) {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int bh = blockIdx.x;
   const int d = threadIdx.x;
   const float* pml = a.part_ml + (int64_t)bh * a.splits * 2;
@@ -426,16 +429,31 @@ __global__ void decode_combine_kernel(DecodeArgs a) {
   float acc = 0.f, L = 0.f;
   for (int s = 0; s < a.splits; ++s) {
     const float ms = pml[2 * s];
-    if (ms == -INFINITY) continue;
+    if (ms == -INFINITY) continue;  // a split without keys (its partial O is not written)
     const float f = exp2f(ms - M);
     acc = fmaf(a.part_o[((int64_t)bh * a.splits + s) * D + d], f, acc);
     L = fmaf(pml[2 * s + 1], f, L);
   }
   ((__nv_bfloat16*)a.out)[(int64_t)bh * D + d] = __float2bfloat16_rn(acc / L);
-  if (a.lse && d == 0) {
-    const int b = bh / a.hq, h = bh % a.hq;
-    a.lse[(int64_t)h * a.batch + b] = (M + log2f(L)) * 0.6931471805599453f;
-  }
+  const int b = bh / a.hq, h = bh % a.hq;
+  if (a.lse && d == 0) a.lse[(int64_t)h * a.batch + b] = (M + log2f(L)) * 0.6931471805599453f;
+  // the attention of this step has read the cache lengths: advance them
+  if (a.cache_len && h == 0 && d == 0) a.cache_len[b] = a.c_snap[b] + 1;
+}
+
+// The combine as a programmatic dependent launch of the kernel before it.
+template <int D>
+cudaError_t launch_combine(const DecodeArgs& a, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(a.batch * a.hq));
+  cfg.blockDim = dim3(D);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, decode_combine_kernel<D>, a);
 }
 
 template <int D, int G>
@@ -474,8 +492,7 @@ cudaError_t run(const DecodeArgs& a, cudaStream_t st) {
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  decode_combine_kernel<D><<<a.batch * a.hq, D, 0, st>>>(a);
-  return cudaGetLastError();
+  return launch_combine<D>(a, st);
 }
 
 // the kernels take the group size padded to a power of two (a batch of 32 / G keys)
@@ -497,8 +514,7 @@ cudaError_t launch_decode(const DecodeArgs& a, cudaStream_t st) {
   if (a.tc) {
     cudaError_t e = tc::launch_decode_tc(a, st);
     if (e != cudaSuccess) return e;
-    decode_combine_kernel<128><<<a.batch * a.hq, 128, 0, st>>>(a);
-    return cudaGetLastError();
+    return launch_combine<128>(a, st);
   }
   return a.d == 64 ? run_d<64>(a, st) : run_d<128>(a, st);
 }

@@ -115,6 +115,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem = bar->tmem_base;
+  // launched as a programmatic dependent of the cache write: the set-up above
+  // overlaps it; the cache lengths and the new rows are read only after it
+  // has completed.  The combine kernel after this one may start early and
+  // waits for this grid in turn.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == kLoadWarp) {
     // ------------------------------------------------ TMA loads (the warp waits converged, lane 0 issues)
@@ -411,8 +417,17 @@ cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t st) {
   const int64_t n_items = (int64_t)a.batch * a.hkv * a.splits;
   int64_t grid = sms < n_items ? sms : n_items;
   if (grid <= 0) return cudaSuccess;
-  decode_tc_kernel<<<(unsigned)grid, kThreads, kSmemBytes, st>>>(tq, tk, tv, a, n_items);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, decode_tc_kernel, tq, tk, tv, a, n_items);
 }
 
 }  // namespace tc

@@ -91,16 +91,19 @@ cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, 
 cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t kbase_stride, int bm, int bn,
                                int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
                                int32_t* q_order, int32_t* pair_order, cudaStream_t st);
+// c_snap: cache lengths before the append.  snap_out (nullable): receives a
+// copy of them (single-token steps pass cache_len itself as c_snap).
 cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap, const KvPages& pages,
                                const int32_t* c_snap, const void* k_new, const void* v_new,
-                               void* k_cache, void* v_cache, cudaStream_t st);
+                               void* k_cache, void* v_cache, cudaStream_t st, int32_t* snap_out = nullptr);
 // Cache write with the rotary encoding of the new queries and keys (bf16,
 // head_dim a multiple of 16): rotated keys and plain values into the cache,
 // rotated queries into q_rot [batch * l_new, hq, d].
 cudaError_t launch_rope_cache_write(int batch, int l_new, int hq, int hkv, int d, int64_t cap,
                                    const KvPages& pages, const int32_t* c_snap, const void* q_new,
                                    const void* k_new, const void* v_new, const float* cos_t, const float* sin_t,
-                                   void* q_rot, void* k_cache, void* v_cache, cudaStream_t st);
+                                   void* q_rot, void* k_cache, void* v_cache, cudaStream_t st,
+                                   int32_t* snap_out = nullptr);
 
 // CUDA-core attention (ism_simt.cu), fp32 or bf16 storage, fp32 math.
 struct AttnArgs {
@@ -165,6 +168,7 @@ struct DecodeArgs {
   int32_t tma;           // stream the cache with TMA (head_dim 128, sm_103)
   int32_t tc;            // tensor-core kernel (bf16, head_dim 128, group <= 16; chunk a multiple of 128)
   uint32_t* status;      // device status word (bounded waits)
+  int32_t* cache_len;    // nullable: the combine kernel advances it by one (single-token steps)
 };
 // Keys one work item of the tensor-core decode covers at most (its scores of
 // 24 tiles of 128 keys stay in tensor memory).

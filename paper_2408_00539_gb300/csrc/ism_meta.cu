@@ -335,6 +335,15 @@ __global__ void append_plan_kernel(AppendSegs sg, int batch, int64_t kbase_strid
 // cache write (clipped to the capacity of a contiguous cache; a paged tile
 // lies within one page).  Keys need no such care: masked scores are replaced,
 // not multiplied.
+// Single-token steps run without the plan kernel: the cache write reads the
+// cache lengths itself (c_snap = cache_len, unchanged until the decode's
+// combine kernel advances it) and records them in snap_out for the decode.
+__device__ __forceinline__ void copy_snapshot(int batch, const int32_t* __restrict__ c_snap, int32_t* snap_out) {
+  if (!snap_out) return;
+  for (int64_t b = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; b < batch; b += (int64_t)gridDim.x * blockDim.x)
+    snap_out[b] = c_snap[b];
+}
+
 __device__ __forceinline__ void zero_value_tail(int batch, int l_new, int vec_per_row, int64_t cap,
                                                 const KvPages& pages, const int32_t* __restrict__ c_snap,
                                                 uint4* v_cache) {
@@ -356,8 +365,12 @@ __device__ __forceinline__ void zero_value_tail(int batch, int l_new, int vec_pe
 
 __global__ void cache_write_kernel(int batch, int l_new, int row_bytes, int64_t cap, KvPages pages,
                                    const int32_t* __restrict__ c_snap, const uint4* __restrict__ k_new,
-                                   const uint4* __restrict__ v_new, uint4* k_cache, uint4* v_cache) {
+                                   const uint4* __restrict__ v_new, uint4* k_cache, uint4* v_cache,
+                                   int32_t* snap_out) {
+  // a decode kernel launched as a programmatic dependent may start its set-up now
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int vec_per_row = row_bytes / 16;
+  copy_snapshot(batch, c_snap, snap_out);
   const int64_t total = (int64_t)batch * l_new * vec_per_row;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
        i += (int64_t)gridDim.x * blockDim.x) {
@@ -398,7 +411,9 @@ __global__ void rope_cache_write_kernel(int batch, int l_new, int hq, int hkv, i
                                         const __nv_bfloat16* __restrict__ k_new,
                                         const __nv_bfloat16* __restrict__ v_new, const float* __restrict__ cos_t,
                                         const float* __restrict__ sin_t, __nv_bfloat16* q_rot,
-                                        __nv_bfloat16* k_cache, __nv_bfloat16* v_cache) {
+                                        __nv_bfloat16* k_cache, __nv_bfloat16* v_cache, int32_t* snap_out) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  copy_snapshot(batch, c_snap, snap_out);
   const int half = d / 2;
   const int units = half / 8;  // 8-coordinate units in one half of a head row
   const int per_row = (hq + 2 * hkv) * units;
@@ -512,7 +527,7 @@ cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t kbase_
 
 cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap, const KvPages& pages,
                                const int32_t* c_snap, const void* k_new, const void* v_new,
-                               void* k_cache, void* v_cache, cudaStream_t st) {
+                               void* k_cache, void* v_cache, cudaStream_t st, int32_t* snap_out) {
   int elem = dtype == ISM_BF16 ? 2 : dtype == ISM_E4M3 ? 1 : 4;
   int row_bytes = hkv * d * elem;
   int64_t total = (int64_t)batch * l_new * (row_bytes / 16);
@@ -522,14 +537,15 @@ cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, 
   int grid = (int)((total + 255) / 256);
   if (grid > 152 * 16) grid = 152 * 16;
   cache_write_kernel<<<grid, 256, 0, st>>>(batch, l_new, row_bytes, cap, pages, c_snap, (const uint4*)k_new,
-                                           (const uint4*)v_new, (uint4*)k_cache, (uint4*)v_cache);
+                                           (const uint4*)v_new, (uint4*)k_cache, (uint4*)v_cache, snap_out);
   return cudaGetLastError();
 }
 
 cudaError_t launch_rope_cache_write(int batch, int l_new, int hq, int hkv, int d, int64_t cap,
                                    const KvPages& pages, const int32_t* c_snap, const void* q_new,
                                    const void* k_new, const void* v_new, const float* cos_t, const float* sin_t,
-                                   void* q_rot, void* k_cache, void* v_cache, cudaStream_t st) {
+                                   void* q_rot, void* k_cache, void* v_cache, cudaStream_t st,
+                                   int32_t* snap_out) {
   int64_t total = (int64_t)batch * l_new * (hq + 2 * hkv) * (d / 16);
   if (total == 0) return cudaSuccess;
   const int64_t tail = (int64_t)batch * 128 * (hkv * d / 8);  // value rows zeroed past the new end
@@ -539,7 +555,7 @@ cudaError_t launch_rope_cache_write(int batch, int l_new, int hq, int hkv, int d
   rope_cache_write_kernel<<<grid, 256, 0, st>>>(
       batch, l_new, hq, hkv, d, cap, pages, c_snap, (const __nv_bfloat16*)q_new, (const __nv_bfloat16*)k_new,
       (const __nv_bfloat16*)v_new, cos_t, sin_t, (__nv_bfloat16*)q_rot, (__nv_bfloat16*)k_cache,
-      (__nv_bfloat16*)v_cache);
+      (__nv_bfloat16*)v_cache, snap_out);
   return cudaGetLastError();
 }
 
