@@ -694,7 +694,7 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
     const char* no_tma = getenv("ISM_DECODE_NO_TMA");
     const char* no_tc = getenv("ISM_DECODE_NO_TC");
     a.tma = (d == 128 && tc_available() && !(no_tma && no_tma[0] == '1')) ? 1 : 0;
-    a.tc = (a.tma && shape->dtype == ISM_BF16 && !(no_tc && no_tc[0] == '1') &&
+    a.tc = (a.tma && !(no_tc && no_tc[0] == '1') &&
             kv_max <= (int64_t)kMaxSplits * kDecTcMaxKeys)
                ? 1
                : 0;

@@ -21,30 +21,41 @@
 // which decode_combine_kernel merges as for the CUDA-core kernels.
 // Warps 0-3: softmax and epilogue (thread = key of a tile, TMEM lane);
 // warp 4: TMA loads (Q of the item, then its K tiles, then its V tiles,
-// through one 4-stage ring); warp 5: MMA issue.
+// through one ring); warp 5: MMA issue.
+// e4m3 caches (kE4M3): Q, K, V, P in e4m3 (kind::f8f6f4 MMAs, K = 32 a step,
+// 128-byte rows: one swizzled box a tile), scores scaled by qk_descale, O by
+// v_descale; tiles are half the size, so the ring has twice the stages.
 #include "ism_tc_common.cuh"
 
 namespace ism {
 namespace tc {
 namespace {
 
-constexpr int kStages = 4;
+constexpr int kMaxStages = 8;
 constexpr int kHeadsPad = 16;  // N of S^T = K Q^T
 constexpr int kMaxTiles = kDecTcMaxKeys / 128;
-constexpr uint32_t kQHalf = kHeadsPad * 128;  // one 64-column half of the Q tile: 16 rows x 128 B
-constexpr uint32_t kQBytes = 2 * kQHalf;
-constexpr uint32_t OFF_RING = 0, OFF_P = kStages * kTileBytes, OFF_Q = OFF_P + 2 * kTileBytes,
-                   OFF_BAR = OFF_Q + 2 * kQBytes;
-constexpr uint32_t kSmemBytes = OFF_BAR + 1024 + 1024;  // barrier block + 1024-byte alignment slack
 constexpr int kThreads = 192;
 constexpr int kLoadWarp = 4, kMmaWarp = 5;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t TM_O = 0, TM_S = 128;
 static_assert(TM_S + kHeadsPad * kMaxTiles <= kTmemCols, "S tiles fit in tensor memory");
-static_assert(kSmemBytes <= 232448, "shared memory per CTA");
+
+// Shared-memory plan: ring of K / V tiles, two P operands, two Q tiles, barriers.
+template <bool kE4M3>
+struct DecCfg {
+  static constexpr int kStages = kE4M3 ? 8 : 4;
+  static constexpr uint32_t kTile = kE4M3 ? kHalfBytes : kTileBytes;  // 128 keys x 128 dims
+  static constexpr uint32_t kQHalf = kHeadsPad * 128;                  // 16 rows x 128 bytes
+  static constexpr uint32_t kQBytes = kE4M3 ? kQHalf : 2 * kQHalf;
+  static constexpr uint32_t OFF_RING = 0, OFF_P = kStages * kTile, OFF_Q = OFF_P + 2 * kTile,
+                            OFF_BAR = OFF_Q + 2 * kQBytes;
+  static constexpr uint32_t kSmemBytes = OFF_BAR + 1024 + 1024;  // barrier block + 1024-byte alignment slack
+  static_assert(kStages <= kMaxStages, "ring");
+  static_assert(kSmemBytes <= 232448, "shared memory per CTA");
+};
 
 struct Bars {
-  uint64_t full[kStages], empty[kStages];
+  uint64_t full[kMaxStages], empty[kMaxStages];
   uint64_t q_full[2], q_empty[2];
   uint64_t s_full, s_free, p_ready[2], p_free[2], o_full, o_free, final_mma;
   uint64_t red_m_full, red_l_full;  // the four softmax warps' partial maxima / sums are written
@@ -78,9 +89,24 @@ __device__ __forceinline__ DecItem dec_item(const DecodeArgs& a, int64_t item) {
   return x;
 }
 
+// Element (row h, key k) of the P operand (rows = heads, 128 keys), in the
+// layout a 128-byte swizzled TMA box produces: bf16 two 64-key halves, e4m3 one.
+template <bool kE4M3>
+__device__ __forceinline__ uint32_t p_offset(uint32_t h, uint32_t k) {
+  if constexpr (kE4M3)
+    return h * 128u + (((k >> 4) ^ (h & 7u)) << 4) + (k & 15u);
+  else
+    return swz_offset(h, k);
+}
+
+template <bool kE4M3>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                      const __grid_constant__ CUtensorMap tmV, const DecodeArgs a, int64_t n_items) {
+  using Cfg = DecCfg<kE4M3>;
+  constexpr int kStages = Cfg::kStages;
+  constexpr uint32_t kTile = Cfg::kTile, kQHalf = Cfg::kQHalf, kQBytes = Cfg::kQBytes;
+  constexpr uint32_t OFF_RING = Cfg::OFF_RING, OFF_P = Cfg::OFF_P, OFF_Q = Cfg::OFF_Q, OFF_BAR = Cfg::OFF_BAR;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   Bars* bar = reinterpret_cast<Bars*>(smem + OFF_BAR);
@@ -125,7 +151,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kLoadWarp) {
     // ------------------------------------------------ TMA loads (the warp waits converged, lane 0 issues)
     uint32_t nl = 0, nu = 0;  // ring tiles issued; non-empty items
-    uint32_t nf[kStages] = {0, 0, 0, 0}, nq[2] = {0, 0};
+    uint32_t nf[kStages] = {}, nq[2] = {0, 0};
     bool ok = true;
     const uint64_t pol = ptx::l2_policy_evict_first();  // the cache is streamed once per step
     if (lane == 0) {
@@ -148,7 +174,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint8_t* dq = smem + OFF_Q + qb * kQBytes;
         ptx::mbar_expect_tx(&bar->q_full[qb], kQBytes);
         ptx::tma_load_2d(dq, &tmQ, &bar->q_full[qb], 0, qy);
-        ptx::tma_load_2d(dq + kQHalf, &tmQ, &bar->q_full[qb], 64, qy);
+        if (!kE4M3) ptx::tma_load_2d(dq + kQHalf, &tmQ, &bar->q_full[qb], 64, qy);
       }
       __syncwarp();
       ++nq[qb];
@@ -166,10 +192,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             // a tile starts at a multiple of 128 keys and lies in one page
             const int64_t p = (int64_t)x.k0 + (int64_t)t * 128;
             const int32_t y = a.pages.table ? (int32_t)paged_row(a.pages, x.b, p) : (int32_t)((int64_t)x.b * a.cap + p);
-            uint8_t* dst = smem + OFF_RING + s * kTileBytes;
-            ptx::mbar_expect_tx(&bar->full[s], kTileBytes);
+            uint8_t* dst = smem + OFF_RING + s * kTile;
+            ptx::mbar_expect_tx(&bar->full[s], kTile);
             ptx::tma_load_2d_hint(dst, map, &bar->full[s], x.g * kD, y, pol);
-            ptx::tma_load_2d_hint(dst + kHalfBytes, map, &bar->full[s], x.g * kD + 64, y, pol);
+            if (!kE4M3) ptx::tma_load_2d_hint(dst + kHalfBytes, map, &bar->full[s], x.g * kD + 64, y, pol);
           }
           __syncwarp();
           ++nf[s];
@@ -188,8 +214,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == kMmaWarp) {
     // ------------------------------------------------ MMA issue (the whole warp runs the loop,
     // one elected lane issues each instruction)
-    constexpr uint32_t idesc_s = ptx::idesc_bf16_f32(128, kHeadsPad, 0, 0);
-    constexpr uint32_t idesc_pv = ptx::idesc_bf16_f32(128, 128, 0, 1);
+    constexpr uint32_t idesc_s =
+        kE4M3 ? ptx::idesc_e4m3_f32(128, kHeadsPad, 0, 0) : ptx::idesc_bf16_f32(128, kHeadsPad, 0, 0);
+    constexpr uint32_t idesc_pv = kE4M3 ? ptx::idesc_e4m3_f32(128, 128, 0, 1) : ptx::idesc_bf16_f32(128, 128, 0, 1);
     uint32_t nl = 0, nu = 0, T = 0;  // ring tiles consumed; non-empty items; P tiles
     bool ok = true;
     for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
@@ -212,9 +239,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         ptx::tc_fence_after();
-        const uint32_t sK = ptx::smem_u32(smem + OFF_RING + s * kTileBytes);
-        ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128Rows16>(
-            tmem + TM_S + kHeadsPad * (uint32_t)t, desc_kmajor(sK, 0), desc_kmajor(sQ, 0), idesc_s, 0u);
+        const uint32_t sK = ptx::smem_u32(smem + OFF_RING + s * kTile);
+        const uint32_t tS = tmem + TM_S + kHeadsPad * (uint32_t)t;
+        if constexpr (kE4M3)  // 128-byte rows: four k-steps of 32 bytes in one box
+          ptx::mma4_e4m3_ss_warp<2, 2>(tS, desc_kmajor(sK, 0), desc_kmajor(sQ, 0), idesc_s, 0u);
+        else
+          ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128Rows16>(tS, desc_kmajor(sK, 0), desc_kmajor(sQ, 0),
+                                                                          idesc_s, 0u);
         ptx::mma_commit_warp(&bar->empty[s]);
       }
       if (!ok) break;
@@ -235,10 +266,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         }
         ptx::tc_fence_after();
-        const uint32_t sP = ptx::smem_u32(smem + OFF_P + pb * kTileBytes);
-        const uint32_t sV = ptx::smem_u32(smem + OFF_RING + s * kTileBytes);
-        ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::MnMajorSw128>(tmem + TM_O, desc_kmajor(sP, 0),
-                                                                   desc_mnmajor(sV, 0), idesc_pv, t > 0 ? 1u : 0u);
+        const uint32_t sP = ptx::smem_u32(smem + OFF_P + pb * kTile);
+        const uint32_t sV = ptx::smem_u32(smem + OFF_RING + s * kTile);
+        if constexpr (kE4M3)  // V MN-major: 32 keys of 128 bytes a k-step
+          ptx::mma4_e4m3_ss_warp<2, 256>(tmem + TM_O, desc_kmajor(sP, 0), desc_kmajor(sV, 0), idesc_pv,
+                                         t > 0 ? 1u : 0u);
+        else
+          ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::MnMajorSw128>(tmem + TM_O, desc_kmajor(sP, 0),
+                                                                     desc_mnmajor(sV, 0), idesc_pv, t > 0 ? 1u : 0u);
         ptx::mma_commit_warp(&bar->empty[s]);
         ptx::mma_commit_warp(&bar->p_free[pb]);
       }
@@ -255,7 +290,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------ softmax and epilogue: thread r = key r of a tile
     const int r = threadIdx.x;
     const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
-    const float c2 = a.scale * kLog2e;
+    const float c2 = a.scale * kLog2e * (kE4M3 ? a.qk_descale : 1.f);
+    const float o_scale = kE4M3 ? a.v_descale : 1.f;
     const int group = a.group;
     uint32_t nu = 0, T = 0;
     bool ok = true;
@@ -322,13 +358,28 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           break;
         }
-        uint8_t* P = smem + OFF_P + pb * kTileBytes;
+        uint8_t* P = smem + OFF_P + pb * kTile;
+        if constexpr (kE4M3) {
 #pragma unroll
-        for (int h = 0; h < kHeadsPad; ++h) {
-          const float p = (valid && h < group) ? ex2(__uint_as_float(v[h]) * c2 - m2[h]) : 0.f;
-          const __nv_bfloat16 pr = __float2bfloat16_rn(p);
-          l[h] += __bfloat162float(pr);  // the sum of the P that enters P V
-          *reinterpret_cast<__nv_bfloat16*>(P + swz_offset((uint32_t)h, (uint32_t)r)) = pr;
+          for (int h = 0; h < kHeadsPad; h += 4) {
+            float p4[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              p4[e] = (valid && h + e < group) ? ex2(__uint_as_float(v[h + e]) * c2 - m2[h + e]) : 0.f;
+              l[h + e] += p4[e];
+            }
+            const uint32_t b4 = pack_e4m3x4(p4[0], p4[1], p4[2], p4[3]);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) P[p_offset<true>((uint32_t)(h + e), (uint32_t)r)] = (uint8_t)(b4 >> (8 * e));
+          }
+        } else {
+#pragma unroll
+          for (int h = 0; h < kHeadsPad; ++h) {
+            const float p = (valid && h < group) ? ex2(__uint_as_float(v[h]) * c2 - m2[h]) : 0.f;
+            const __nv_bfloat16 pr = __float2bfloat16_rn(p);
+            l[h] += __bfloat162float(pr);  // the sum of the P that enters P V
+            *reinterpret_cast<__nv_bfloat16*>(P + p_offset<false>((uint32_t)h, (uint32_t)r)) = pr;
+          }
         }
         ptx::fence_proxy_async_smem();
         ptx::mbar_arrive(&bar->p_ready[pb]);
@@ -369,8 +420,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int i = 0; i < 8; ++i)
               reinterpret_cast<float4*>(dst + 32 * q4)[i] =
-                  make_float4(__uint_as_float(o[4 * i]), __uint_as_float(o[4 * i + 1]), __uint_as_float(o[4 * i + 2]),
-                              __uint_as_float(o[4 * i + 3]));
+                  make_float4(__uint_as_float(o[4 * i]) * o_scale, __uint_as_float(o[4 * i + 1]) * o_scale,
+                              __uint_as_float(o[4 * i + 2]) * o_scale, __uint_as_float(o[4 * i + 3]) * o_scale);
           }
         }
         if (mine) {
@@ -398,18 +449,22 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-}  // namespace
-
-cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t st) {
-  if (a.d != kD || a.dtype != ISM_BF16 || a.group > kHeadsPad || a.chunk % 128 != 0 || a.chunk > kDecTcMaxKeys)
-    return cudaErrorInvalidValue;
+template <bool kE4M3>
+cudaError_t launch_decode_tc_t(const DecodeArgs& a, cudaStream_t st) {
+  using Cfg = DecCfg<kE4M3>;
   CUtensorMap tq, tk, tv;
   cudaError_t e;
-  if ((e = make_tmap_bf16_box(&tq, a.q, (uint64_t)kD, (uint64_t)a.batch * a.hq, kHeadsPad)) != cudaSuccess) return e;
-  if ((e = make_tmap_bf16(&tk, a.k_cache, (uint64_t)a.hkv * kD, (uint64_t)a.kv_rows)) != cudaSuccess) return e;
-  if ((e = make_tmap_bf16(&tv, a.v_cache, (uint64_t)a.hkv * kD, (uint64_t)a.kv_rows)) != cudaSuccess) return e;
-  if ((e = cudaFuncSetAttribute(decode_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
-      cudaSuccess)
+  if constexpr (kE4M3) {
+    if ((e = make_tmap_e4m3_box(&tq, a.q, (uint64_t)kD, (uint64_t)a.batch * a.hq, kHeadsPad)) != cudaSuccess) return e;
+    if ((e = make_tmap_e4m3_box(&tk, a.k_cache, (uint64_t)a.hkv * kD, (uint64_t)a.kv_rows, 128)) != cudaSuccess) return e;
+    if ((e = make_tmap_e4m3_box(&tv, a.v_cache, (uint64_t)a.hkv * kD, (uint64_t)a.kv_rows, 128)) != cudaSuccess) return e;
+  } else {
+    if ((e = make_tmap_bf16_box(&tq, a.q, (uint64_t)kD, (uint64_t)a.batch * a.hq, kHeadsPad)) != cudaSuccess) return e;
+    if ((e = make_tmap_bf16(&tk, a.k_cache, (uint64_t)a.hkv * kD, (uint64_t)a.kv_rows)) != cudaSuccess) return e;
+    if ((e = make_tmap_bf16(&tv, a.v_cache, (uint64_t)a.hkv * kD, (uint64_t)a.kv_rows)) != cudaSuccess) return e;
+  }
+  if ((e = cudaFuncSetAttribute(decode_tc_kernel<kE4M3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)Cfg::kSmemBytes)) != cudaSuccess)
     return e;
   int dev = 0, sms = 0;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
@@ -420,14 +475,23 @@ cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.dynamicSmemBytes = Cfg::kSmemBytes;
   cfg.stream = st;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, decode_tc_kernel, tq, tk, tv, a, n_items);
+  return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kE4M3>, tq, tk, tv, a, n_items);
+}
+
+}  // namespace
+
+cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t st) {
+  if (a.d != kD || (a.dtype != ISM_BF16 && a.dtype != ISM_E4M3) || a.group > kHeadsPad || a.chunk % 128 != 0 ||
+      a.chunk > kDecTcMaxKeys)
+    return cudaErrorInvalidValue;
+  return a.dtype == ISM_E4M3 ? launch_decode_tc_t<true>(a, st) : launch_decode_tc_t<false>(a, st);
 }
 
 }  // namespace tc

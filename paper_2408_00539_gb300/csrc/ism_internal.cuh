@@ -166,7 +166,7 @@ struct DecodeArgs {
   float* part_o;         // [B, Hq, splits, D]
   float* part_ml;        // [B, Hq, splits, 2]
   int32_t tma;           // stream the cache with TMA (head_dim 128, sm_103)
-  int32_t tc;            // tensor-core kernel (bf16, head_dim 128, group <= 16; chunk a multiple of 128)
+  int32_t tc;            // tensor-core kernel (bf16 or e4m3, head_dim 128, group <= 16; chunk a multiple of 128)
   uint32_t* status;      // device status word (bounded waits)
   int32_t* cache_len;    // nullable: the combine kernel advances it by one (single-token steps)
 };

@@ -147,6 +147,8 @@ __device__ __forceinline__ uint64_t desc_ilv_mnmajor(uint32_t tile_saddr, int kk
 cudaError_t make_tmap_bf16(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows);
 // Host: the same with a 64-column x box_rows box (box_rows <= 256).
 cudaError_t make_tmap_bf16_box(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows);
+// Host: 2D e4m3 tensor map with a 128-column (128-byte) x box_rows box, 128B swizzle.
+cudaError_t make_tmap_e4m3_box(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows);
 // Host: 2D bf16 tensor map with a 64-column x box_rows box, no swizzle.
 cudaError_t make_tmap_bf16_plain(CUtensorMap* m, const void* base, uint64_t cols, uint64_t rows, uint32_t box_rows);
 // 1-byte elements, box of 128 columns x box_rows, no swizzle

@@ -588,12 +588,19 @@ def test_e4m3_rejects_other_entry_points(ism):
     ism.check_status()
 
 
+@pytest.mark.parametrize("path", ["tensor_cores", "cuda_cores"])
 @pytest.mark.parametrize("l_new,segs,hq,hkv", [(200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2),
                                                 (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 3, 3),
-                                                (1, ([1], [1]), 8, 2), (1, ([1], [1]), 6, 2)])
-def test_prefill_append_e4m3(ism, l_new, segs, hq, hkv):
+                                                (1, ([1], [1]), 8, 2), (1, ([1], [1]), 6, 2),
+                                                (1, ([1], [1]), 16, 1), (1, ([1], [1]), 4, 4)])
+def test_prefill_append_e4m3(ism, l_new, segs, hq, hkv, path, monkeypatch):
     """e4m3 queries and caches (cache factors shared by the new keys / values)
-    against the oracle on the dequantised values."""
+    against the oracle on the dequantised values; single-token steps on the
+    tensor-core decode or the CUDA-core one."""
+    if path == "cuda_cores":
+        if l_new != 1:
+            pytest.skip("the decode path choice applies to single-token steps")
+        monkeypatch.setenv("ISM_DECODE_NO_TC", "1")
     B, d = 3, 128
     c_lens = np.array([0, 77, 300], dtype=np.int32)
     cap = 300 + l_new + 5
