@@ -897,6 +897,34 @@ def measure_session(dev):
                     "ism.AppendStep (one C call a step); the first turn's calls include warm-up"}
 
 
+def profile_decode(dtype: str, steps: int):
+    """Only the single-token steps of the 8 x 16K cache workload (the decode of
+    ``measure_append``), ``steps`` of them, printing nothing: for ncu.  bf16
+    caches, or e4m3 ones with per-tensor factors."""
+    import torch
+    from paper_2408_00539_gb300 import ism
+    dev = "cuda:0"
+    a = wl.append_16k()
+    B, cap, hq, hkv, d = a.batch, a.capacity, a.num_heads_q, a.num_heads_kv, a.head_dim
+    g = torch.Generator(device=dev).manual_seed(a.seed)
+
+    def rnd(shape):
+        x = torch.randn(shape, generator=g, device=dev).mul_(a.value_std)
+        return x.to(torch.float8_e4m3fn) if dtype == "e4m3" else x.bfloat16()
+    kc, vc = rnd((B, cap, hkv, d)), rnd((B, cap, hkv, d))
+    qd, kd, vd = rnd((B, 1, hq, d)), rnd((B, 1, hkv, d)), rnd((B, 1, hkv, d))
+    c_host = a.cache_len.copy() + a.l_new
+    cl = torch.from_numpy(c_host.copy()).to(dev)
+    for _ in range(steps):
+        if dtype == "e4m3":
+            ism.prefill_append_e4m3(qd, kd, vd, kc, vc, cl, c_host, [1], [1], 1.0, 1.0, 1.0, a.softmax_scale)
+        else:
+            ism.prefill_append(qd, kd, vd, kc, vc, cl, c_host, [1], [1], a.softmax_scale)
+        c_host = c_host + 1
+    torch.cuda.synchronize()
+    ism.check_status(dev)
+
+
 WORKLOADS = {"gqa_8k": wl.gqa_8k, "mha_4k": wl.mha_4k, "packed_32k": wl.packed_32k,
              # one 4K dialogue of the same recipe: small enough for full ncu captures
              "gqa_4k_b1": lambda: wl.gqa_8k(batch=1, seqlen=4096)}
@@ -913,8 +941,13 @@ def main():
     ap.add_argument("--no-append", action="store_true", help="skip the append-prefill / decode measurement")
     ap.add_argument("--profile-step", action="store_true",
                     help="run the warm-up steps and one more step, print nothing (for ncu)")
+    ap.add_argument("--profile-decode", choices=["bf16", "e4m3"],
+                    help="run only warm-up + steps single-token steps on the 8 x 16K cache, print nothing (for ncu)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    if args.profile_decode:
+        profile_decode(args.profile_decode, args.warmup + args.steps)
+        return
     w = WORKLOADS[args.workload]()
     if args.impl == "reference":
         run_reference(args, w)

@@ -424,15 +424,35 @@ __global__ void decode_combine_kernel(DecodeArgs a) {
   const int bh = blockIdx.x;
   const int d = threadIdx.x;
   const float* pml = a.part_ml + (int64_t)bh * a.splits * 2;
+  // splits in chunks of eight with every load of a chunk issued before any
+  // use (a split count below eight is one chunk); a split without keys (max
+  // -inf) has weight 0 and its partial O, never written, is replaced by 0
+  const float* po = a.part_o + (int64_t)bh * a.splits * D + d;
   float M = -INFINITY;
-  for (int s = 0; s < a.splits; ++s) M = fmaxf(M, pml[2 * s]);
+  for (int s0 = 0; s0 < a.splits; s0 += 8) {
+    float ms[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) ms[u] = s0 + u < a.splits ? pml[2 * (s0 + u)] : -INFINITY;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) M = fmaxf(M, ms[u]);
+  }
   float acc = 0.f, L = 0.f;
-  for (int s = 0; s < a.splits; ++s) {
-    const float ms = pml[2 * s];
-    if (ms == -INFINITY) continue;  // a split without keys (its partial O is not written)
-    const float f = exp2f(ms - M);
-    acc = fmaf(a.part_o[((int64_t)bh * a.splits + s) * D + d], f, acc);
-    L = fmaf(pml[2 * s + 1], f, L);
+  for (int s0 = 0; s0 < a.splits; s0 += 8) {
+    float ms[8], ls[8], v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const bool in = s0 + u < a.splits;
+      ms[u] = in ? pml[2 * (s0 + u)] : -INFINITY;
+      ls[u] = in ? pml[2 * (s0 + u) + 1] : 0.f;
+      v[u] = in ? po[(int64_t)(s0 + u) * D] : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const bool live = ms[u] != -INFINITY;
+      const float f = live ? exp2f(ms[u] - M) : 0.f;
+      acc = fmaf(live ? v[u] : 0.f, f, acc);
+      L = fmaf(live ? ls[u] : 0.f, f, L);
+    }
   }
   ((__nv_bfloat16*)a.out)[(int64_t)bh * D + d] = __float2bfloat16_rn(acc / L);
   const int b = bh / a.hq, h = bh % a.hq;
