@@ -91,6 +91,15 @@ def test_malformed_segments_rejected(lib, segs, msg):
     assert msg in lib.ism_last_error().decode()
 
 
+def test_too_many_sequences(lib):
+    keep = _Keep()
+    n = 8193                                                       # one past the most one call takes
+    s = _segs(list(range(n + 1)), list(range(n + 1)), [1] * n, [0] * n, keep)
+    nt, nq, nk = C.c_int64(), C.c_int64(), C.c_int64()
+    assert lib.ism_tile_map_size(C.byref(s), 128, 128, C.byref(nt), C.byref(nq), C.byref(nk)) == 2
+    assert "num_seqs 8193" in lib.ism_last_error().decode()
+
+
 def test_shape_errors(lib):
     keep = _Keep()
     s = _segs([0, 10], [0, 2], [4, 10], [0, 1], keep)
@@ -141,6 +150,10 @@ def test_append_errors(lib):
     assert call(seg_type=np.array([0, 2], np.uint8)) == 1
     assert call(nseg=0) == 1
     assert call(cache_host=np.array([-1, 0], np.int32)) == 1
+    many_end = np.arange(1, 258, dtype=np.int32)                  # 257 segments: one past the limit
+    many_type = np.zeros(257, np.uint8)
+    assert call(l_new=257, cap=300, seg_end=many_end, seg_type=many_type, nseg=257) == 1
+    assert "1..256 segments" in lib.ism_last_error().decode()
 
 
 def test_paged_append_errors(lib):

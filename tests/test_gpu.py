@@ -868,3 +868,77 @@ def test_paged_and_e4m3_appends_ignore_garbage(ism):
                                     segs[0], segs[1], qd_, kd_, vd_, scale)
     ism.check_status()
     _cmp_e4m3("e4m3 o_new", o8, o8_ref, float(torch.cat([vc, vn], 1).float().abs().max()))
+
+
+# ---------------------------------------------------------------- limits
+
+def test_max_sequences_fwd_bwd_sampled(ism):
+    """8192 sequences (the most one call takes) of 1-40 tokens with random
+    segments (empty and same-type neighbours included) in one fwd + bwd
+    call; the oracle checks every 517th sequence and the last."""
+    rng = np.random.Generator(np.random.PCG64(81))
+    segs = wl.random_dialogue_set(rng, 8192, 40)
+    w = wl.Workload("many_short", segs, 4, 2, 128, "bf16", 128 ** -0.5, 0.5, 82)
+    (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w)
+    for b in list(range(0, 8192, 517)) + [8191]:
+        t0, L, se, st = segs.seq(b)
+        sub = wl.pack([(se, st)])
+        sl = slice(t0, t0 + L)
+        o_ref, lse_ref = orc.attn_fwd(q[sl], k[sl], v[sl], sub, w.softmax_scale)
+        dq_ref, dk_ref, dv_ref = orc.attn_bwd(q[sl], k[sl], v[sl], do[sl], sub, w.softmax_scale)
+        _cmp(f"o of sequence {b}", o[sl], o_ref, "bf16")
+        _cmp_lse(f"lse of sequence {b}", lse[:, sl], lse_ref, "bf16")
+        _cmp(f"dq of sequence {b}", dq[sl], dq_ref, "bf16")
+        _cmp(f"dk of sequence {b}", dk[sl], dk_ref, "bf16")
+        _cmp(f"dv of sequence {b}", dv[sl], dv_ref, "bf16")
+
+
+def test_append_max_segments(ism):
+    """A chunk of 256 segments (the most one append takes): alternating query
+    and answer runs of 0-3 tokens."""
+    rng = np.random.Generator(np.random.PCG64(83))
+    lens = rng.integers(0, 4, size=256)
+    lens[-1] = max(int(lens[-1]), 1)
+    ends = np.cumsum(lens).astype(np.int32)
+    types = np.array([i % 2 for i in range(256)], dtype=np.uint8)
+    l_new = int(ends[-1])
+    B, hq, hkv, d = 2, 8, 2, 128
+    c_lens = np.array([0, 333], dtype=np.int32)
+    cap = 333 + l_new + 4
+    kc, vc, qn, kn, vn = _append_inputs(B, cap, c_lens, l_new, hq, hkv, d, seed=84)
+    cl = torch.from_numpy(c_lens.copy()).to(DEV)
+    o, lse = ism.prefill_append(qn.to(DEV), kn.to(DEV), vn.to(DEV), kc.to(DEV), vc.to(DEV), cl, c_lens, ends, types,
+                                d ** -0.5)
+    ism.check_status()
+    o_ref, lse_ref = orc.prefill_append(qn, kn, vn, kc, vc, c_lens, ends, types, d ** -0.5)
+    _cmp("o_new", o, o_ref, "bf16")
+    _cmp_lse("lse_new", lse, np.transpose(lse_ref, (1, 0, 2)), "bf16")
+
+
+@pytest.mark.parametrize("keys", [150000, 200000])
+def test_decode_long_cache(ism, keys):
+    """Single-token steps over one cache of 150 000 keys (the tensor-core
+    decode with close to its 64 splits of at most 3072 keys) and of 200 000
+    (past 64 x 3072 keys: the CUDA-core decode takes it); the oracle checks
+    one KV head's group."""
+    B, hq, hkv, d, steps = 1, 8, 2, 128, 2
+    cap = keys + steps
+    kc, vc, qn, kn, vn = _append_inputs(B, cap, None, steps, hq, hkv, d, seed=85)
+    kcd, vcd = kc.clone().to(DEV), vc.clone().to(DEV)
+    c_host = np.array([keys], dtype=np.int32)
+    cl = torch.from_numpy(c_host.copy()).to(DEV)
+    g, grp = 1, hq // hkv
+    hs = list(range(g * grp, (g + 1) * grp))
+    for t in range(steps):
+        o, lse = ism.prefill_append(qn[:, t:t + 1].contiguous().to(DEV), kn[:, t:t + 1].contiguous().to(DEV),
+                                    vn[:, t:t + 1].contiguous().to(DEV), kcd, vcd, cl, c_host, [1], [1], d ** -0.5)
+        kref = kc[:, :, g:g + 1].clone()
+        vref = vc[:, :, g:g + 1].clone()
+        kref[0, keys:keys + t] = kn[0, :t, g:g + 1]
+        vref[0, keys:keys + t] = vn[0, :t, g:g + 1]
+        o_ref, lse_ref = orc.prefill_append(qn[:, t:t + 1, hs], kn[:, t:t + 1, g:g + 1], vn[:, t:t + 1, g:g + 1],
+                                            kref, vref, c_host, [1], [1], d ** -0.5)
+        _cmp(f"decode o step {t}", o[:, :, hs], o_ref, "bf16")
+        _cmp_lse(f"decode lse step {t}", lse[hs], np.transpose(lse_ref, (1, 0, 2)), "bf16")
+        c_host = c_host + 1
+    ism.check_status()
