@@ -51,7 +51,9 @@ __device__ __forceinline__ void set_abort(int32_t* f) { *reinterpret_cast<volati
 // kE4M3: Q, K, V in e4m3 (kind::f8f6f4 MMAs, K = 32 a step); the scores are
 // scaled by qk_descale, P is rounded to e4m3 for O += P V and O is scaled by
 // v_descale (per-tensor dequantisation factors of the inputs).
-template <bool kTilePairs, bool kE4M3>
+// kSplit: the launch runs items past a.split_whole as two key-range halves
+// (head pairs only); the instantiation without it is the plain kernel.
+template <bool kTilePairs, bool kE4M3, bool kSplit = false>
 __global__ void __launch_bounds__(kThreads, 1)
     fwd_pair_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                     const __grid_constant__ CUtensorMap tmV, const AttnArgs a) {
@@ -63,13 +65,26 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   Tile w0, w1;
   int h0, h1, nkb0, nkb1;
+  int jb = 0, half = -1;  // first key tile; half of a split item (-1: the whole item)
+  int64_t split_k = 0;    // index of a split item among the split ones
   if constexpr (!kTilePairs) {
     const int npairs = a.hq >> 1;
-    const int hp = blockIdx.x % npairs;
-    w0 = w1 = a.qtiles[a.q_order[blockIdx.x / npairs]];
+    int64_t item = blockIdx.x;
+    if (kSplit && item >= a.split_whole) {
+      split_k = (item - a.split_whole) >> 1;
+      half = (int)((item - a.split_whole) & 1);
+      item = a.split_whole + split_k;
+    }
+    const int hp = (int)(item % npairs);
+    w0 = w1 = a.qtiles[a.q_order[item / npairs]];
     h0 = 2 * hp;
     h1 = h0 + 1;
     nkb0 = nkb1 = w0.a1;
+    if (half >= 0) {  // key tiles [0, mid) or [mid, a1)
+      const int mid = w0.a1 / 2;
+      jb = half ? mid : 0;
+      nkb0 = nkb1 = half ? w0.a1 - mid : mid;
+    }
   } else {
     h0 = h1 = blockIdx.x % a.hq;
     const int gq = a.pair_order[blockIdx.x / a.hq];
@@ -84,6 +99,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     nkb1 = second ? w1.a1 : 0;
   }
   const Tile& w = w0;  // K/V rows (k_base) are those of the shared sequence
+  const int k_first = jb * kRows;  // first key of this CTA's key range
   const int g = h0 / (a.hq / a.hkv);
   const int nkb = nkb0 > nkb1 ? nkb0 : nkb1;
 
@@ -135,8 +151,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int s = j & 1;
         const uint32_t n = (uint32_t)(j >> 1);
         if (__any_sync(0xffffffffu, aborted(&bar->abort))) break;
-        const int32_t ky = a.pages.table ? (int32_t)paged_row(a.pages, w.k_base, (int64_t)j * kRows)
-                                         : w.k_base + j * kRows;
+        const int32_t ky = a.pages.table ? (int32_t)paged_row(a.pages, w.k_base, (int64_t)k_first + j * kRows)
+                                         : w.k_base + k_first + j * kRows;
         if (j >= 2 && !wait_warp(&bar->k_empty[s], (n - 1) & 1, a.status)) {
           if (lane == 0) set_abort(&bar->abort);
           break;
@@ -251,12 +267,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = threadIdx.x & 127;
     const int h = x ? h1 : h0;
     const Tile wm = x ? w1 : w0;
-    const int nkbm = x ? nkb1 : nkb0, kfull = wm.a0;
+    const int nkbm = x ? nkb1 : nkb0, kfull = wm.a0 - jb;  // key tiles counted from this CTA's first
     const uint32_t lane_addr = (uint32_t)((warp & 3) * 32) << 16;
     const uint32_t tS = tmem + lane_addr + (x ? 256u : 0u), tO = tmem + lane_addr + (x ? 384u : 128u);
     const int row = wm.tile * kRows + r;
     const bool valid = row < wm.q_len;
-    const int ke = a.kv_end[wm.kv_base + (valid ? row : wm.q_len - 1)];
+    const int ke = a.kv_end[wm.kv_base + (valid ? row : wm.q_len - 1)] - k_first;
     const float sl2 = a.scale * kLog2e * (kE4M3 ? a.qk_descale : 1.f);
     float m_use = -INFINITY, l = 0.f;
     bool ok = nkbm > 0;
@@ -359,7 +375,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::mbar_arrive(&bar->p_full[x]);
     }
     if (ok) ok = wait(&bar->pv_done[x], (uint32_t)(nkbm - 1) & 1, a.status);
-    if (!ok) {
+    if (kSplit && half >= 0) {
+      // half of a split item: unnormalised O and (max, sum) for the merge; a
+      // half without key tiles leaves max -inf (weight 0, its O is not read)
+      if (!ok && nkbm > 0) set_abort(&bar->abort);
+      const int64_t pu = ((split_k * 2 + half) * 2 + x) * kRows + r;
+      a.part_ml[pu * 2] = ok ? m_use : -INFINITY;
+      a.part_ml[pu * 2 + 1] = ok ? l : 0.f;
+      if (ok) {
+        ptx::tc_fence_after();
+        const float f = kE4M3 ? a.v_descale : 1.f;
+        float4* dst = reinterpret_cast<float4*>(a.part_o + pu * kD);
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          uint32_t o[32];
+          ptx::tmem_ld32(tO + c * 32, o);
+          ptx::tmem_ld_wait();
+          ptx::reg_fence(o);
+#pragma unroll
+          for (int i = 0; i < 8; ++i)
+            dst[c * 8 + i] = make_float4(__uint_as_float(o[4 * i]) * f, __uint_as_float(o[4 * i + 1]) * f,
+                                         __uint_as_float(o[4 * i + 2]) * f, __uint_as_float(o[4 * i + 3]) * f);
+        }
+      }
+    } else if (!ok) {
       if (nkbm > 0) set_abort(&bar->abort);  // a unit without key blocks has nothing to write
     } else {
       ptx::tc_fence_after();
@@ -395,18 +434,52 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// Merge of the two halves of each split item: block (split item k, head x,
+// row r) of 128 threads (dimensions).  m in the base-2 scaled units of the
+// forward, so O = (w0 O0 + w1 O1) / (w0 l0 + w1 l1) with w = 2^(m - M), and
+// LSE = (M + log2 L) ln 2, as the whole-item epilogue writes them.
+__global__ void __launch_bounds__(128) fwd_split_merge_kernel(const AttnArgs a) {
+  const int64_t b = blockIdx.x;
+  const int r = (int)(b % kRows), x = (int)((b / kRows) & 1);
+  const int64_t k = b / (2 * kRows);
+  const int npairs = a.hq >> 1;
+  const int64_t item = a.split_whole + k;
+  const Tile w = a.qtiles[a.q_order[item / npairs]];
+  const int h = 2 * (int)(item % npairs) + x;
+  const int row = w.tile * kRows + r;
+  if (row >= w.q_len) return;
+  const int d = threadIdx.x;
+  const int64_t p0 = ((k * 2 + 0) * 2 + x) * kRows + r, p1 = ((k * 2 + 1) * 2 + x) * kRows + r;
+  const float m0 = a.part_ml[p0 * 2], l0 = a.part_ml[p0 * 2 + 1];
+  const float m1 = a.part_ml[p1 * 2], l1 = a.part_ml[p1 * 2 + 1];
+  const float M = fmaxf(m0, m1);
+  const float f0 = m0 == -INFINITY ? 0.f : exp2f(m0 - M), f1 = m1 == -INFINITY ? 0.f : exp2f(m1 - M);
+  const float o0 = f0 != 0.f ? a.part_o[p0 * kD + d] : 0.f, o1 = f1 != 0.f ? a.part_o[p1 * kD + d] : 0.f;
+  const float L = (f0 != 0.f ? f0 * l0 : 0.f) + (f1 != 0.f ? f1 * l1 : 0.f);
+  const int64_t orow = (int64_t)w.q_base + row;
+  reinterpret_cast<__nv_bfloat16*>(a.out)[(orow * a.hq + h) * kD + d] = __float2bfloat16_rn((f0 * o0 + f1 * o1) / L);
+  if (d == 0 && a.lse) a.lse[(int64_t)h * a.q_rows + orow] = (M + log2f(L)) * kLn2;
+}
+
 template <bool kE4M3>
 cudaError_t launch_fwd_pair_t(const AttnArgs& a, const CUtensorMap& tq, const CUtensorMap& tk, const CUtensorMap& tv,
                               cudaStream_t st) {
   cudaError_t e;
   const bool tile_pairs = a.pair_order != nullptr;
-  auto kern = tile_pairs ? fwd_pair_kernel<true, kE4M3> : fwd_pair_kernel<false, kE4M3>;
+  const bool split_launch = !tile_pairs && a.split_items > 0;
+  auto kern = tile_pairs ? fwd_pair_kernel<true, kE4M3>
+                         : (split_launch ? fwd_pair_kernel<false, kE4M3, true> : fwd_pair_kernel<false, kE4M3>);
   constexpr uint32_t smem = PairLayout<kE4M3>::SMEM;
   if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
     return e;
-  const int64_t grid = tile_pairs ? a.npairs * a.hq : a.nq * (a.hq / 2);
-  if (grid == 0) return cudaSuccess;
+  const int64_t items = tile_pairs ? a.npairs * a.hq : a.nq * (a.hq / 2);
+  if (items == 0) return cudaSuccess;
+  const bool split = !tile_pairs && a.split_items > 0;
+  if (split && (a.split_whole + a.split_items != items || !a.part_o || !a.part_ml)) return cudaErrorInvalidValue;
+  const int64_t grid = split ? a.split_whole + 2 * a.split_items : items;
   kern<<<(unsigned)grid, kThreads, smem, st>>>(tq, tk, tv, a);
+  if ((e = cudaGetLastError()) != cudaSuccess || !split) return e;
+  fwd_split_merge_kernel<<<(unsigned)(a.split_items * 2 * kRows), 128, 0, st>>>(a);
   return cudaGetLastError();
 }
 

@@ -138,6 +138,14 @@ struct AttnArgs {
   // e4m3 forward: per-tensor dequantisation factors (scores scaled by
   // q_descale * k_descale, the output by v_descale).
   float qk_descale, v_descale;
+  // Key-range split of the paired forward (head pairs only): launch items
+  // [0, split_whole) run whole; each later item runs as two CTAs over the
+  // first and the second half of its key tiles, writing unnormalised O and
+  // (max, sum) to part_o / part_ml, merged by a second kernel.  Off when
+  // split_items == 0.
+  int64_t split_whole, split_items;
+  float* part_o;    // [split_items][2 halves][2 heads][128 rows][128] fp32
+  float* part_ml;   // [split_items][2 halves][2 heads][128 rows][2] fp32
   // Bit 0: before an MMA that overwrites tensor memory an earlier MMA reads
   // as its A operand, wait for that earlier MMA to complete.  Clear: rely on
   // MMAs issued by one thread executing in issue order.

@@ -942,3 +942,42 @@ def test_decode_long_cache(ism, keys):
         _cmp_lse(f"decode lse step {t}", lse[hs], np.transpose(lse_ref, (1, 0, 2)), "bf16")
         c_host = c_host + 1
     ism.check_status()
+
+
+# ---------------------------------------------------------------- key-range split of the prefill
+
+@pytest.mark.parametrize("dtype", ["bf16", "e4m3"])
+@pytest.mark.parametrize("n_split", ["0", "2", "1000"])
+def test_prefill_key_split(ism, dtype, n_split, monkeypatch):
+    """Prefill items that run as two halves of their key range (the last ones,
+    or all of them with 1000: some halves then have no key tile at all) give
+    the oracle's result; ISM_PREFILL_SPLIT forces the count."""
+    monkeypatch.setenv("ISM_PREFILL_SPLIT", n_split)
+    B, d, hq, hkv, l_new = 3, 128, 8, 2, 200
+    segs = ([40, 41, 120, 200], [0, 1, 0, 1])
+    c_lens = np.array([0, 77, 300], dtype=np.int32)
+    cap = 300 + l_new + 5
+    kc, vc, qn, kn, vn = _append_inputs(B, cap, c_lens, l_new, hq, hkv, d, seed=91)
+    cl = torch.from_numpy(c_lens.copy()).to(DEV)
+    scale = d ** -0.5
+    if dtype == "bf16":
+        o, lse = ism.prefill_append(qn.to(DEV), kn.to(DEV), vn.to(DEV), kc.to(DEV), vc.to(DEV), cl, c_lens, segs[0],
+                                    segs[1], scale)
+        ism.check_status()
+        o_ref, lse_ref = orc.prefill_append(qn, kn, vn, kc, vc, c_lens, segs[0], segs[1], scale)
+        _cmp("o_new", o, o_ref, "bf16")
+    else:
+        _, ks = wl.quantize_e4m3(torch.cat([kc.reshape(-1), kn.reshape(-1)]))
+        _, vs = wl.quantize_e4m3(torch.cat([vc.reshape(-1), vn.reshape(-1)]))
+        q8, qs = wl.quantize_e4m3(qn)
+        k8c, k8n = ((t.float() / ks).to(torch.float8_e4m3fn) for t in (kc, kn))
+        v8c, v8n = ((t.float() / vs).to(torch.float8_e4m3fn) for t in (vc, vn))
+        o, lse = ism.prefill_append_e4m3(q8.to(DEV), k8n.to(DEV), v8n.to(DEV), k8c.to(DEV), v8c.to(DEV), cl, c_lens,
+                                         segs[0], segs[1], qs, ks, vs, scale)
+        ism.check_status()
+        deq = lambda t, s: t.double() * s  # noqa: E731
+        o_ref, lse_ref = orc.prefill_append(deq(q8, qs), deq(k8n, ks), deq(v8n, vs), deq(k8c, ks), deq(v8c, vs),
+                                            c_lens, segs[0], segs[1], scale)
+        vmax = max(float(deq(v8c, vs).abs().max()), float(deq(v8n, vs).abs().max()))
+        _cmp_e4m3("o_new", o, o_ref, vmax)
+    _cmp_lse("lse_new", lse, np.transpose(lse_ref, (1, 0, 2)), "bf16")
