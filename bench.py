@@ -893,7 +893,8 @@ def measure_session(dev):
             "ttft_ism_over_causal": float(np.mean(ttft_i) / np.mean(ttft_c)),
             "ttft_ms_first_last_turn": [float(ttft_i[0]), float(ttft_i[-1])],
             "tpot_us": float(np.mean(tpot)), "tpot_us_first_last_turn": [tpot[0], tpot[-1]],
-            "note": "one attention layer per call (append plan, cache write, attention) through a prepared "
+            "note": "one attention layer per call (query chunk: append plan, cache write, forward; answer token: cache "
+                    "write, tensor-core decode, combine) through a prepared "
                     "ism.AppendStep (one C call a step); the first turn's calls include warm-up"}
 
 
