@@ -471,13 +471,16 @@ def _to_pages(kc, vc, page_size, rng, spare=3):
     return kp, vp, table
 
 
+@pytest.mark.parametrize("split", ["0", "1000"])
 @pytest.mark.parametrize("l_new,segs,hq,hkv,d", [(200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2, 128),
                                                   (128, ([128], [0]), 8, 2, 128), (1, ([1], [1]), 8, 2, 128),
                                                   (1, ([1], [1]), 8, 1, 128), (37, ([37], [0]), 3, 3, 128),
                                                   (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2, 64)])
-def test_prefill_append_paged_matches_contiguous(ism, l_new, segs, hq, hkv, d):
+def test_prefill_append_paged_matches_contiguous(ism, l_new, segs, hq, hkv, d, split, monkeypatch):
     """The paged cache gives bit for bit the contiguous result (same kernels,
-    rows through the block table) and the oracle's result on the gathered cache."""
+    rows through the block table) and the oracle's result on the gathered
+    cache, with every prefill item split into key-range halves or none."""
+    monkeypatch.setenv("ISM_PREFILL_SPLIT", split)
     B, ps = 3, 128
     c_lens = np.array([0, 77, 300], dtype=np.int32)
     cap = int(c_lens.max()) + l_new
