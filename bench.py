@@ -127,6 +127,13 @@ class ClockSampler:
         for line in self.proc.stdout:
             self.lines.append((time.time(), line.strip()))
 
+    def wait_first(self, timeout: float = 2.0):
+        """Wait (at most ``timeout`` s) until nvidia-smi has printed a sample,
+        so that a short timed window that follows gets one."""
+        t_end = time.time() + timeout
+        while self.proc is not None and not self.lines and time.time() < t_end:
+            time.sleep(0.01)
+
     def mark_start(self):
         self.t0 = time.time()
 
@@ -505,6 +512,13 @@ def run_cuda(args, w):
         "gpu_launches": int(launches),
         "clocks": clocks.summary(),
     }
+    if not args.no_extra:
+        line["sustained"] = measure_sustained(dev, step, flops, peaks)
+        del ins, outs, ob, lb
+        torch.cuda.empty_cache()
+        line["bwd_min_workspace"] = measure_training_config(dev, w, peaks, steps=args.steps, minimal_workspace=True)
+        line["configs"] = {wname: measure_training_config(dev, WORKLOADS[wname](), peaks, steps=args.steps)
+                           for wname in ("mha_4k", "packed_32k") if WORKLOADS[wname]().name != w.name}
     if not args.no_append:
         line["append"] = measure_append(dev, read_peaks()[0])
         line["session"] = measure_session(dev)
@@ -554,8 +568,12 @@ def measure_append(dev, peaks):
     n_vis_pre = int(B * hq * ln * (int(c0[0]) + ln))  # every new row sees the cache and the whole new query
     pre = float(np.median(pre_ms))
     # decode steps after the prefill
-    c_host = c0 + ln
+    # decode steps after the prefill, through a prepared call (one C call a
+    # step, as a generation loop makes them); the decode kernels are timed by
+    # the library's timer hook inside each call
+    c_host = (c0 + ln).astype(np.int32)
     cl.copy_(torch.from_numpy(c_host))
+    step = ism.AppendStep(qd, kd, vd, kc, vc, cl, c_host, [1], [1], a.softmax_scale)
     dec_us, dec_kernel_us, dec_bytes = [], [], []
     for t in range(a.decode_steps):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -564,18 +582,30 @@ def measure_append(dev, peaks):
             e.record(stream)
         ism.set_kernel_timer(ism.KERNEL_DECODE, k0, k1)
         e0.record(stream)
-        ism.prefill_append(qd, kd, vd, kc, vc, cl, c_host, [1], [1], a.softmax_scale)
+        step()
         e1.record(stream)
         e1.synchronize()
         ism.set_kernel_timer(ism.KERNEL_DECODE)
         dec_us.append(e0.elapsed_time(e1) * 1e3)
         dec_kernel_us.append(k0.elapsed_time(k1) * 1e3)
         dec_bytes.append(2 * B * (int(c_host[0]) + 1) * hkv * d * 2)
-        c_host = c_host + 1
+        c_host += 1
     ism.check_status(dev)
     us = float(np.median(dec_us[3:]))
     kus = float(np.median(dec_kernel_us[3:]))
     gbs = float(np.median(np.array(dec_bytes[3:]) / (np.array(dec_kernel_us[3:]) * 1e-6) / 1e9))
+    # the same step through the plain binding (argument conversion, workspace
+    # and output allocation on every call)
+    plain_us = []
+    for t in range(16):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        ism.prefill_append(qd, kd, vd, kc, vc, cl, c_host, [1], [1], a.softmax_scale)
+        e1.record(stream)
+        e1.synchronize()
+        plain_us.append(e0.elapsed_time(e1) * 1e3)
+        c_host += 1
+    ism.check_status(dev)
     paged = measure_append_paged(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush)
     e4m3 = measure_append_e4m3(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, peaks)
     rope = measure_append_rope(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush)
@@ -583,14 +613,16 @@ def measure_append(dev, peaks):
             "prefill_ms": pre, "prefill_tflops": 4 * d * n_vis_pre / (pre * 1e-3) / 1e12,
             "prefill_frac_of_bf16_peak": 4 * d * n_vis_pre / (pre * 1e-3) / 1e12 / peaks["bf16_tflops"],
             "decode_us_per_call": us, "decode_kernel_us": kus,
+            "decode_us_per_call_plain_binding": float(np.median(plain_us[3:])),
             "decode_hbm_gbs": gbs, "decode_frac_of_hbm": gbs / peaks["hbm_gbs"],
             "decode_steps": a.decode_steps,
             "paged": paged,
             "e4m3": e4m3,
             "rope": rope,
             "note": "decode bytes = K and V cache read once: 2*B*(c+1)*Hkv*D*2 per step; GB/s over the "
-                    "split-KV + merge kernels (decode_kernel_us); decode_us_per_call adds the plan and "
-                    "cache-write kernels and host launch overhead"}
+                    "split-KV + merge kernels (decode_kernel_us); decode_us_per_call: CUDA events around one "
+                    "prepared call (ism.AppendStep), which adds the cache-write kernel and the host time of the "
+                    "call; decode_us_per_call_plain_binding: the same through ism.prefill_append"}
 
 
 def measure_append_paged(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, page_size=256, decode_steps=64):
@@ -699,6 +731,117 @@ def measure_append_rope(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, decode_st
     return out
 
 
+def measure_training_config(dev, w, peaks, steps=20, minimal_workspace=False):
+    """fwd+bwd steps of one workload timed as the headline is: inputs resident,
+    L2 flushed between steps (outside the events), CUDA events around each
+    step, per-kernel times from separate steps through the library's timer
+    hooks, clocks sampled over the timed steps.  minimal_workspace runs the
+    backward with ism_attn_bwd_workspace_size_min bytes (the recompute
+    schedule: no stored dS)."""
+    import torch
+    from paper_2408_00539_gb300 import ism
+    q, k, v, do = (t.to(dev) for t in wl.attention_tensors(w))
+    segs = ism.Segments.from_workload(w.segs, dev)
+    n_vis = n_visible(w.segs) * w.num_heads_q
+    D = w.head_dim
+    flops = 14 * D * n_vis
+    ws_bytes = ism.bwd_workspace_size(segs, q, k, w.softmax_scale, minimal=minimal_workspace)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    o, lse = ism.fwd(segs, q, k, v, w.softmax_scale)
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        ism.fwd(segs, q, k, v, w.softmax_scale, out=o, lse=lse)
+        ism.bwd(segs, q, k, v, o, lse, do, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws)
+
+    with ClockSampler(dev.index) as clocks:
+        for _ in range(3):
+            step()
+        torch.cuda.synchronize()
+        clocks.wait_first()
+        ms = []
+        clocks.mark_start()
+        for _ in range(steps):
+            flush.fill_(1)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            step()
+            e1.record(stream)
+            e1.synchronize()
+            ms.append(e0.elapsed_time(e1))
+        clocks.mark_end()
+        for _ in range(3):
+            step()
+        torch.cuda.synchronize()
+    ism.check_status(dev)
+    kinds = {"fwd": ism.KERNEL_FWD, "bwd_dkdv": ism.KERNEL_BWD_DKDV, "bwd_dq": ism.KERNEL_BWD_DQ,
+             "bwd_pre": ism.KERNEL_BWD_PRE, "meta": ism.KERNEL_META}
+    kt = {n: [] for n in kinds}
+    for _ in range(5):
+        flush.fill_(1)
+        ev = {n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for n in kinds}
+        for n, kid in kinds.items():
+            for e in ev[n]:
+                e.record(stream)
+            ism.set_kernel_timer(kid, *ev[n])
+        step()
+        torch.cuda.synchronize()
+        for n in kinds:
+            kt[n].append(ev[n][0].elapsed_time(ev[n][1]))
+    for kid in kinds.values():
+        ism.set_kernel_timer(kid)
+    ism.check_status(dev)
+    ms_step = float(np.sum(ms)) / steps
+    tflops = flops / (ms_step * 1e-3) / 1e12
+    mean_k = {n: float(np.mean(t)) for n, t in kt.items()}
+    peak = peaks["bf16_tflops"]
+    fracs = {"fwd": 4 * D * n_vis / (mean_k["fwd"] * 1e-3) / 1e12 / peak,
+             "bwd_dkdv": 8 * D * n_vis / (mean_k["bwd_dkdv"] * 1e-3) / 1e12 / peak}
+    out = {"workload": w.name, "tokens": w.total_tokens, "n_vis_pairs": n_vis, "flops_per_step": flops,
+           "ms_per_step": ms_step, "steps": steps, "tflops": tflops, "pct_of_bf16_peak": tflops / peak * 100,
+           "bwd_schedule": "recompute dQ" if minimal_workspace else "stored dS",
+           "bwd_workspace_bytes": ws_bytes, "kernel_ms": mean_k, "kernel_frac_of_bf16_peak": fracs,
+           "clocks": clocks.summary()}
+    del q, k, v, do, o, lse, dq, dk, dv, ws, flush
+    torch.cuda.empty_cache()
+    return out
+
+
+def measure_sustained(dev, step, flops, peaks, seconds=3.0):
+    """The headline step run back to back, as a training loop runs it (no L2
+    flush), for at least ``seconds``: the rate once the clocks have settled
+    under the power limit, against the sustained bf16 peak."""
+    import torch
+    probe = []
+    stream = torch.cuda.current_stream(dev)
+    for _ in range(5):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        step()
+        e1.record(stream)
+        e1.synchronize()
+        probe.append(e0.elapsed_time(e1))
+    n = int(np.ceil(seconds * 1e3 / float(np.median(probe))))
+    with ClockSampler(dev.index) as clocks:
+        torch.cuda.synchronize()
+        clocks.mark_start()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(n):
+            step()
+        e1.record(stream)
+        e1.synchronize()
+        clocks.mark_end()
+    total = e0.elapsed_time(e1)
+    tflops = flops * n / (total * 1e-3) / 1e12
+    return {"steps": n, "seconds": total * 1e-3, "ms_per_step": total / n, "tflops": tflops,
+            "frac_of_bf16_sustained_peak": tflops / peaks["bf16_tflops_sustained"],
+            "bf16_sustained_peak_tflops": peaks["bf16_tflops_sustained"], "clocks": clocks.summary(),
+            "note": "steps back to back without an L2 flush (inputs 335 MB exceed L2), one event pair around all"}
+
+
 def measure_training_cost(dev, w, reps=3):
     """What one ISM pass saves in training against a prefix-LM, which needs
     one sample per answer turn (history and query as a bidirectional prefix,
@@ -770,8 +913,10 @@ def measure_fwd_e4m3(dev, w, peaks, reps=10):
     peak8 = 2 * peaks["bf16_tflops"]  # e4m3 dense rate = 2x bf16 (nominal 4.5 vs 2.25 PFLOP/s)
     return {"workload": w.name, "ms": ms8, "tflops": flops / (ms8 * 1e-3) / 1e12,
             "frac_of_e4m3_peak": flops / (ms8 * 1e-3) / 1e12 / peak8, "e4m3_peak_tflops": peak8,
+            "e4m3_peak_kind": "derived, not measured: measured bf16 burst peak x 2, the nominal dense "
+                              "fp8/bf16 ratio (4.5 / 2.25 PFLOP/s)",
             "bf16_fwd_ms": ms16, "speedup_over_bf16": ms16 / ms8,
-            "note": "fwd call incl. metadata pass; peak = measured bf16 x 2 (nominal fp8/bf16 ratio)"}
+            "note": "fwd call incl. metadata pass"}
 
 
 def measure_append_e4m3(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, peaks, decode_steps=64):
@@ -940,6 +1085,8 @@ def main():
     ap.add_argument("--workload", default="gqa_8k", choices=sorted(WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-append", action="store_true", help="skip the append-prefill / decode measurement")
+    ap.add_argument("--no-extra", action="store_true",
+                    help="skip the sustained run, the minimum-workspace backward and the other training configs")
     ap.add_argument("--profile-step", action="store_true",
                     help="run the warm-up steps and one more step, print nothing (for ncu)")
     ap.add_argument("--profile-decode", choices=["bf16", "e4m3"],

@@ -155,10 +155,11 @@ ism_status_t ism_attn_fwd_e4m3(const ism_segments_t* segs, const ism_attn_shape_
 
 /* Forward without a caller-provided workspace (the paper has no counterpart;
  * this is a deployment convenience).  Some callers cannot allocate device
- * memory at the point where they run attention: code recorded into a CUDA
- * graph (allocation during capture is not allowed), servers that reserve all
- * device memory once at start-up and never grow it, or plain C hosts with no
- * device allocator of their own.  This variant takes the forward's scratch
+ * memory at the point where they run attention: inference servers that carve
+ * all device memory into their own pools once at start-up and may not grow
+ * them afterwards (a late cudaMalloc can fail there, and it synchronises the
+ * device), and hosts that drive the GPU only through this C interface, with
+ * no device allocator of their own.  This variant takes the forward's scratch
  * from a fixed array of ism_attn_fwd_noalloc_max_workspace() bytes (4 MiB)
  * that the library keeps in device memory on every GPU that loads it, until
  * the process exits.  It calls no allocator.
@@ -369,6 +370,13 @@ enum {
 };
 ism_status_t ism_set_kernel_timer(int32_t kernel_id, void* start_event, void* stop_event);
 uint64_t ism_kernel_launches(void);
+
+/* Debug and tuning switches (no counterpart in the paper).  The library reads
+ * its ISM_* environment variables once, when it is loaded, so that no call
+ * spends host time on them.  ism_debug_reload_env reads them again (for tests
+ * that change a switch in a running process); it must not run concurrently
+ * with other calls of the library. */
+void ism_debug_reload_env(void);
 
 /* Diagnostic of the tensor-core building blocks (no counterpart in the
  * paper): one 128x128x128 bf16 tile product on tcgen05 with fp32 result.

@@ -230,15 +230,9 @@ PassLayout pass_layout(void* ws, const ism_segments_t* s, const Counts& c, int64
   return L;
 }
 
-bool force_cuda_cores() {
-  const char* e = getenv("ISM_FORCE_CUDA_CORES");
-  return e && e[0] == '1';
-}
+bool force_cuda_cores() { return knobs().force_cuda_cores; }
 
-uint32_t tc_flags() {
-  const char* e = getenv("ISM_DRAIN_TMEM_REUSE");
-  return (e && e[0] == '1') ? kFlagDrainTmemReuse : 0u;
-}
+uint32_t tc_flags() { return knobs().drain_tmem_reuse ? kFlagDrainTmemReuse : 0u; }
 
 bool use_tc(const ism_attn_shape_t* sh) {
   return sh->dtype == ISM_BF16 && sh->head_dim == 128 && tc_available() && !force_cuda_cores();
@@ -252,8 +246,7 @@ bool fwd_tile_pairs(const ism_attn_shape_t* sh) {
   if ((sh->num_heads_q / sh->num_heads_kv) % 2 == 0) return false;
   if (sh->dtype == ISM_E4M3) return true;  // the e4m3 forward runs only the paired kernel
   if (!use_tc(sh)) return false;
-  const char* e = getenv("ISM_FWD_ONE_HEAD");
-  return !(e && e[0] == '1');
+  return !knobs().fwd_one_head;
 }
 
 // dS tile slots of the stored-dS backward (pairs x query heads), or 0 where
@@ -261,8 +254,7 @@ bool fwd_tile_pairs(const ism_attn_shape_t* sh) {
 // more pairs than the 32-bit pair offsets hold.
 int64_t stored_ds_slots(const ism_segments_t* s, const ism_attn_shape_t* sh) {
   if (!use_tc_bwd(sh)) return 0;
-  const char* e = getenv("ISM_BWD_RECOMPUTE_DQ");
-  if (e && e[0] == '1') return 0;
+  if (knobs().bwd_recompute_dq) return 0;
   const int64_t pairs = count_pairs(s);
   if (pairs >= (int64_t(1) << 31)) return 0;
   return pairs * sh->num_heads_q;
@@ -299,6 +291,52 @@ void timer_end(int id, cudaStream_t st) {
 void count_launch(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
 void set_error(const char* msg) { g_last_error = msg; }
 
+namespace {
+bool env_on(const char* name) {
+  const char* e = getenv(name);
+  return e && e[0] == '1';
+}
+int64_t env_int(const char* name, int64_t unset) {
+  const char* e = getenv(name);
+  return (e && e[0]) ? atoll(e) : unset;
+}
+Knobs read_knobs() {
+  Knobs k;
+  k.force_cuda_cores = env_on("ISM_FORCE_CUDA_CORES");
+  k.drain_tmem_reuse = env_on("ISM_DRAIN_TMEM_REUSE");
+  k.fwd_one_head = env_on("ISM_FWD_ONE_HEAD");
+  k.bwd_recompute_dq = env_on("ISM_BWD_RECOMPUTE_DQ");
+  k.decode_no_tma = env_on("ISM_DECODE_NO_TMA");
+  k.decode_no_tc = env_on("ISM_DECODE_NO_TC");
+  const int64_t split = env_int("ISM_PREFILL_SPLIT", -1);
+  k.prefill_split = split < 0 ? -1 : split;
+  const int64_t g1 = env_int("ISM_DKDV_GRID", 0), g2 = env_int("ISM_DQ_GRID", 0);
+  k.dkdv_grid = g1 > 0 && g1 < (1 << 20) ? (int32_t)g1 : 0;
+  k.dq_grid = g2 > 0 && g2 < (1 << 20) ? (int32_t)g2 : 0;
+  return k;
+}
+Knobs g_knobs = read_knobs();  // read when the library is loaded
+
+std::mutex g_sm_mu;
+std::vector<int> g_sm_count;
+}  // namespace
+
+const Knobs& knobs() { return g_knobs; }
+void reload_knobs() { g_knobs = read_knobs(); }
+
+int sm_count() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 152;
+  std::lock_guard<std::mutex> lk(g_sm_mu);
+  if ((int)g_sm_count.size() <= dev) g_sm_count.resize(dev + 1, 0);
+  if (!g_sm_count[dev]) {
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) return 152;
+    g_sm_count[dev] = sms;
+  }
+  return g_sm_count[dev];
+}
+
 }  // namespace ism
 
 using namespace ism;
@@ -331,6 +369,8 @@ ism_status_t ism_set_kernel_timer(int32_t kernel_id, void* start_event, void* st
 }
 
 uint64_t ism_kernel_launches(void) { return g_launches.load(); }
+
+void ism_debug_reload_env(void) { reload_knobs(); }
 
 ism_status_t ism_tile_map_size(const ism_segments_t* segs, int32_t bm, int32_t bn, int64_t* n_tiles,
                                int64_t* n_qtiles, int64_t* n_ktiles) {
@@ -704,13 +744,9 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
     // kernel (four waves, so each CTA's ring runs several tiles)
     int64_t kv_max = (int64_t)max_c + 1;
     int64_t pairs = (int64_t)batch * hkv;
-    int dev = 0, sms = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-      sms = 152;
-    const char* no_tma = getenv("ISM_DECODE_NO_TMA");
-    const char* no_tc = getenv("ISM_DECODE_NO_TC");
-    a.tma = (d == 128 && tc_available() && !(no_tma && no_tma[0] == '1')) ? 1 : 0;
-    a.tc = (a.tma && !(no_tc && no_tc[0] == '1') &&
+    const int sms = sm_count();
+    a.tma = (d == 128 && tc_available() && !knobs().decode_no_tma) ? 1 : 0;
+    a.tc = (a.tma && !knobs().decode_no_tc &&
             kv_max <= (int64_t)kMaxSplits * kDecTcMaxKeys)
                ? 1
                : 0;
@@ -779,14 +815,10 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
       L.split_cap > 0) {
     const int64_t items = a.nq * (hq / 2);
     int64_t n_split = 0;
-    const char* force = getenv("ISM_PREFILL_SPLIT");
-    if (force && force[0]) {
-      n_split = atoll(force);
+    if (knobs().prefill_split >= 0) {
+      n_split = knobs().prefill_split;
     } else {
-      int dev = 0, sms = 0;
-      if (cudaGetDevice(&dev) != cudaSuccess ||
-          cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-        sms = 152;
+      const int sms = sm_count();
       const int64_t key_tiles = ((int64_t)max_c + l_new + kTile - 1) / kTile;
       if (items > sms && shape->dtype == ISM_BF16 && key_tiles >= 64) n_split = items % sms;
     }

@@ -930,12 +930,7 @@ cudaError_t launch_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) {
                                   (int)dkv::kSmemBytes)) != cudaSuccess)
       return e;
     // persistent: one CTA per SM takes (k-tile, KV head) items from the work counter
-    int dev = 0, sms = 0;
-    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-    int64_t grid = sms;
-    const char* ov = getenv("ISM_DKDV_GRID");  // persistent grid size (default: one CTA per SM)
-    if (ov && atoi(ov) > 0) grid = atoi(ov);
+    int64_t grid = knobs().dkdv_grid > 0 ? knobs().dkdv_grid : sm_count();
     if (grid > a.nk * a.hkv) grid = a.nk * a.hkv;
     if (!a.work_counter) return cudaErrorInvalidValue;
     timer_begin(ISM_KERNEL_BWD_DKDV, st);

@@ -214,13 +214,8 @@ cudaError_t launch_dq_gemm(const AttnArgs& a, const CUtensorMap& tk, cudaStream_
   if ((e = cudaFuncSetAttribute(dq_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
       cudaSuccess)
     return e;
-  int dev = 0, sms = 0;
-  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
   const int64_t n_items = a.nq * a.hq;
-  int grid = sms;
-  const char* ov = getenv("ISM_DQ_GRID");  // persistent grid size (default: one CTA per SM)
-  if (ov && atoi(ov) > 0) grid = atoi(ov);
+  int grid = knobs().dq_grid > 0 ? knobs().dq_grid : sm_count();
   if (grid > n_items) grid = (int)n_items;
   if (grid <= 0) return cudaSuccess;
   dq_gemm_kernel<<<(unsigned)grid, kThreads, kSmemBytes, st>>>(tk, a, n_items);

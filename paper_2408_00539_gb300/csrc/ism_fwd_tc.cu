@@ -564,8 +564,7 @@ cudaError_t launch_fwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) {
   if ((e = make_tmap_bf16(&tq, a.q, (uint64_t)a.hq * kD, (uint64_t)a.q_rows)) != cudaSuccess) return e;
   if ((e = make_tmap_bf16(&tk, a.k, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;
   if ((e = make_tmap_bf16(&tv, a.v, (uint64_t)a.hkv * kD, (uint64_t)k_rows)) != cudaSuccess) return e;
-  const char* single = getenv("ISM_FWD_ONE_HEAD");
-  if (((a.hq / a.hkv) % 2 == 0 || a.pair_order) && !(single && single[0] == '1'))
+  if (((a.hq / a.hkv) % 2 == 0 || a.pair_order) && !knobs().fwd_one_head)
     return launch_fwd_pair(a, tq, tk, tv, st);
   if ((e = cudaFuncSetAttribute(fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
       cudaSuccess)

@@ -195,6 +195,25 @@ cudaError_t launch_tc_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st);
 
 cudaError_t launch_timeout_probe(uint32_t spin_limit, uint32_t* status, cudaStream_t st);
 
+// Debug and tuning switches from the environment (ISM_*), read once when the
+// library is loaded and again by ism_debug_reload_env(), so that no call reads
+// the environment.
+struct Knobs {
+  bool force_cuda_cores;   // ISM_FORCE_CUDA_CORES=1: CUDA-core kernels for bf16 too
+  bool drain_tmem_reuse;   // ISM_DRAIN_TMEM_REUSE=1: wait for A-operand readers before overwriting TMEM
+  bool fwd_one_head;       // ISM_FWD_ONE_HEAD=1: one-head forward kernel
+  bool bwd_recompute_dq;   // ISM_BWD_RECOMPUTE_DQ=1: recompute backward even with a stored-dS workspace
+  bool decode_no_tma;      // ISM_DECODE_NO_TMA=1: register-load CUDA-core decode
+  bool decode_no_tc;       // ISM_DECODE_NO_TC=1: CUDA-core decode kernels
+  int64_t prefill_split;   // ISM_PREFILL_SPLIT=n: n key-range split items in a prefill (-1: chosen by the library)
+  int32_t dkdv_grid;       // ISM_DKDV_GRID=n: CTAs of the persistent dK/dV kernel (0: one per SM)
+  int32_t dq_grid;         // ISM_DQ_GRID=n: CTAs of the persistent dQ kernel (0: one per SM)
+};
+const Knobs& knobs();
+void reload_knobs();
+// Multiprocessor count of the current device (looked up once per device).
+int sm_count();
+
 // Measurement hooks (ism_api.cu): events recorded around launches of one
 // kernel kind on the calling host thread, and a count of every launch.
 void timer_begin(int kernel_id, cudaStream_t st);

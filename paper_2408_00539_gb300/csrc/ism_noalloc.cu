@@ -1,8 +1,8 @@
 // Forward entry point that allocates nothing, for callers that cannot call
-// cudaMalloc themselves (for example code running while a CUDA graph is
-// being captured, inference servers whose device memory is carved out once
-// at start-up and may not grow, or hosts that drive the GPU through a plain C
-// interface with no device allocator).  The forward's scratch (per-token key
+// cudaMalloc where they run attention (inference servers whose device memory
+// is carved into their own pools once at start-up and may not grow, or hosts
+// that drive the GPU only through the plain C interface, with no device
+// allocator of their own).  The forward's scratch (per-token key
 // bounds, tile descriptors and the work order) lives in a fixed-size array in
 // device memory that this library owns for the lifetime of the process.
 #include <cstdio>
@@ -68,7 +68,11 @@ ism_status_t ism_attn_fwd_noalloc(const ism_segments_t* segs, const ism_attn_sha
   void* scratch = nullptr;
   r = scratch_address(&scratch);
   if (r != ISM_OK) return r;
-  // The forward rewrites every scratch byte it reads, so nothing needs clearing.
+  // Nothing in the scratch has to start at zero: the forward's layout holds
+  // only the per-token key bounds, tile descriptors and work lists, and its
+  // metadata pass writes every entry the attention kernel then reads.  (The
+  // backward's layout also carries work counters; a forward that ever gains
+  // such state must clear it here before the launch.)
   return ism_attn_fwd(segs, shape, q, k, v, o, lse, scratch, kNoAllocScratchBytes, stream);
 }
 

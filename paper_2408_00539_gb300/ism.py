@@ -83,6 +83,7 @@ EXPORTS = {
     "ism_has_tensor_cores": (C.c_int32, []),
     "ism_set_kernel_timer": (C.c_int, [C.c_int32, C.c_void_p, C.c_void_p]),
     "ism_kernel_launches": (C.c_uint64, []),
+    "ism_debug_reload_env": (None, []),
     "ism_debug_mma_tile": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p]),
     "ism_debug_mma_tile_e4m3": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p]),
     "ism_attn_fwd_noalloc_max_workspace": (C.c_size_t, []),

@@ -112,9 +112,9 @@ def _small_bf16(d, hq=8, hkv=2, seed=9):
 
 @pytest.mark.parametrize("d", [128, 64])
 @pytest.mark.parametrize("path", ["default", "recompute_dq", "cuda_cores"])
-def test_small_bf16_fwd_bwd(ism, d, path, monkeypatch):
+def test_small_bf16_fwd_bwd(ism, d, path, knobs):
     if path == "cuda_cores":
-        monkeypatch.setenv("ISM_FORCE_CUDA_CORES", "1")
+        knobs("ISM_FORCE_CUDA_CORES", "1")
     w = _small_bf16(d)
     _check_small(ism, w, path)
 
@@ -189,16 +189,12 @@ def _largest_seq(segs):
     return int(np.argmax(lens))
 
 
-@pytest.mark.parametrize("make", [wl.mha_4k, wl.gqa_8k, wl.packed_32k], ids=["mha_4k", "gqa_8k", "packed_32k"])
-def test_full_size_parity_sampled_group(ism, make):
-    """Full-size launch (all sequences, all heads, as benchmarked); the oracle
-    recomputes one complete GQA group of one sequence (the longest)."""
-    w = make()
-    (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w)
-    b = _largest_seq(w.segs)
+def _check_group(w, b, g, inputs, outputs):
+    """One sequence b and KV head g of a full-size launch against the oracle:
+    O and LSE of the group's query heads, dQ of those heads, dK and dV of g."""
+    (q, k, v, do), (o, lse, dq, dk, dv) = inputs, outputs
     t0, L, se, st = w.segs.seq(b)
     grp = w.num_heads_q // w.num_heads_kv
-    g = 1 if w.num_heads_kv > 1 else 0
     hs = slice(g * grp, (g + 1) * grp)
     sub = wl.pack([(se, st)])
     sl = slice(t0, t0 + L)
@@ -206,11 +202,57 @@ def test_full_size_parity_sampled_group(ism, make):
     ks, vs = k[sl][:, g:g + 1].contiguous(), v[sl][:, g:g + 1].contiguous()
     o_ref, lse_ref = orc.attn_fwd(qs, ks, vs, sub, w.softmax_scale)
     dq_ref, dk_ref, dv_ref = orc.attn_bwd(qs, ks, vs, dos, sub, w.softmax_scale)
-    _cmp("o", o[sl][:, hs], o_ref, "bf16")
-    _cmp_lse("lse", lse[hs][:, sl], lse_ref, "bf16")
-    _cmp("dq", dq[sl][:, hs], dq_ref, "bf16")
-    _cmp("dk", dk[sl][:, g:g + 1], dk_ref, "bf16")
-    _cmp("dv", dv[sl][:, g:g + 1], dv_ref, "bf16")
+    tag = f"seq {b} (rows {t0}..{t0 + L}) kv head {g}"
+    _cmp(f"o {tag}", o[sl][:, hs], o_ref, "bf16")
+    _cmp_lse(f"lse {tag}", lse[hs][:, sl], lse_ref, "bf16")
+    _cmp(f"dq {tag}", dq[sl][:, hs], dq_ref, "bf16")
+    _cmp(f"dk {tag}", dk[sl][:, g:g + 1], dk_ref, "bf16")
+    _cmp(f"dv {tag}", dv[sl][:, g:g + 1], dv_ref, "bf16")
+
+
+@pytest.mark.parametrize("make", [wl.mha_4k, wl.gqa_8k, wl.packed_32k], ids=["mha_4k", "gqa_8k", "packed_32k"])
+def test_full_size_parity_sampled_groups(ism, make):
+    """Full-size launch (all sequences, all heads, as benchmarked); the oracle
+    recomputes complete GQA groups: the first and the last KV head of the
+    longest sequence, and for the packed buffer also the last dialogue, which
+    starts at an offset that is not a multiple of the 128-row tile.  Every
+    output element of the launch must be finite."""
+    w = make()
+    inputs, outputs = _run_pass(ism, w)
+    for name, t in zip(("o", "lse", "dq", "dk", "dv"), outputs):
+        assert bool(torch.isfinite(t).all()), f"{name}: non-finite values"
+    b = _largest_seq(w.segs)
+    checks = [(b, 0), (b, w.num_heads_kv - 1)]
+    if w.segs.num_seqs > 1 and w.name.startswith("packed"):
+        last = w.segs.num_seqs - 1
+        assert int(w.segs.cu_seqlens[last]) % 128 != 0, "the last dialogue should start off a tile boundary"
+        checks.append((last, w.num_heads_kv // 2))
+    for bb, g in dict.fromkeys(checks):
+        _check_group(w, bb, g, inputs, outputs)
+
+
+@pytest.mark.parametrize("schedule", ["stored_ds", "recompute_dq"])
+def test_mid_size_every_head_gqa32_8(ism, schedule):
+    """The headline head layout (32 query heads over 8 KV heads, head_dim
+    128, bf16) on two dialogues of 1536 and 700 tokens packed back to back,
+    every head of O, LSE, dQ, dK and dV against the oracle, under both
+    backward schedules."""
+    rng = np.random.Generator(np.random.PCG64(2024))
+    segs = wl.pack([wl.draw_dialogue(rng, 1536, 4, 16), wl.draw_dialogue(rng, 700, 2, 8)])
+    w = wl.Workload("mid_gqa32_8", segs, 32, 8, 128, "bf16", 128 ** -0.5, 0.5, 77)
+    (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w, minimal_workspace=schedule == "recompute_dq")
+    if schedule == "stored_ds":
+        assert ism.bwd_workspace_size(ism.Segments.from_workload(segs, DEV), q, k, w.softmax_scale) > \
+            ism.bwd_workspace_size(ism.Segments.from_workload(segs, DEV), q, k, w.softmax_scale, minimal=True)
+    o_ref, lse_ref = orc.attn_fwd(q, k, v, w.segs, w.softmax_scale)
+    dq_ref, dk_ref, dv_ref = orc.attn_bwd(q, k, v, do, w.segs, w.softmax_scale)
+    for h in range(w.num_heads_q):
+        _cmp(f"o head {h}", o[:, h], o_ref[:, h], "bf16")
+        _cmp_lse(f"lse head {h}", lse[h], lse_ref[h], "bf16")
+        _cmp(f"dq head {h}", dq[:, h], dq_ref[:, h], "bf16")
+    for g in range(w.num_heads_kv):
+        _cmp(f"dk kv head {g}", dk[:, g], dk_ref[:, g], "bf16")
+        _cmp(f"dv kv head {g}", dv[:, g], dv_ref[:, g], "bf16")
 
 
 # ---------------------------------------------------------------- KV cache
@@ -273,11 +315,11 @@ def test_prefill_append_matches_one_pass_rows(ism):
 
 @pytest.mark.parametrize("path", ["tensor_cores", "cuda_cores"])
 @pytest.mark.parametrize("hq,hkv", [(8, 2), (4, 4), (8, 1), (4, 2), (6, 2), (10, 2), (7, 1), (16, 1), (40, 2)])
-def test_decode_steps_small(ism, hq, hkv, path, monkeypatch):
+def test_decode_steps_small(ism, hq, hkv, path, knobs):
     """Group sizes 1-16 run the decode kernels (the tensor-core kernel, or the
     CUDA-core ones padded to a power of two), 20 the forward kernels."""
     if path == "cuda_cores":
-        monkeypatch.setenv("ISM_DECODE_NO_TC", "1")
+        knobs("ISM_DECODE_NO_TC", "1")
     B, d, c0, steps = 2, 128, 700, 6
     cap = c0 + steps
     kc, vc, qn, kn, vn = _append_inputs(B, cap, None, steps, hq, hkv, d, seed=31)
@@ -358,7 +400,7 @@ def test_append_16k_prefill_and_decode(ism):
     assert cl.cpu().numpy().tolist() == c_host.tolist()
 
 
-def test_in_order_tmem_reuse_matches_drained_bit_exact(ism, monkeypatch):
+def test_in_order_tmem_reuse_matches_drained_bit_exact(ism, knobs):
     """The tensor-core kernels issue an MMA that overwrites tensor memory
     right after the MMA that reads it, relying on MMAs of one thread
     executing in issue order.  The drained variant (each such MMA waits for
@@ -374,9 +416,9 @@ def test_in_order_tmem_reuse_matches_drained_bit_exact(ism, monkeypatch):
         ism.check_status()
         return o, lse, dq, dk, dv
 
-    monkeypatch.setenv("ISM_DRAIN_TMEM_REUSE", "1")
+    knobs("ISM_DRAIN_TMEM_REUSE", "1")
     ref = run()
-    monkeypatch.setenv("ISM_DRAIN_TMEM_REUSE", "0")
+    knobs("ISM_DRAIN_TMEM_REUSE", "0")
     for _ in range(8):
         got = run()
         for name, a_, b_ in zip(("o", "lse", "dq", "dk", "dv"), got, ref):
@@ -476,11 +518,11 @@ def _to_pages(kc, vc, page_size, rng, spare=3):
                                                   (128, ([128], [0]), 8, 2, 128), (1, ([1], [1]), 8, 2, 128),
                                                   (1, ([1], [1]), 8, 1, 128), (37, ([37], [0]), 3, 3, 128),
                                                   (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2, 64)])
-def test_prefill_append_paged_matches_contiguous(ism, l_new, segs, hq, hkv, d, split, monkeypatch):
+def test_prefill_append_paged_matches_contiguous(ism, l_new, segs, hq, hkv, d, split, knobs):
     """The paged cache gives bit for bit the contiguous result (same kernels,
     rows through the block table) and the oracle's result on the gathered
     cache, with every prefill item split into key-range halves or none."""
-    monkeypatch.setenv("ISM_PREFILL_SPLIT", split)
+    knobs("ISM_PREFILL_SPLIT", split)
     B, ps = 3, 128
     c_lens = np.array([0, 77, 300], dtype=np.int32)
     cap = int(c_lens.max()) + l_new
@@ -596,14 +638,14 @@ def test_e4m3_rejects_other_entry_points(ism):
                                                 (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 3, 3),
                                                 (1, ([1], [1]), 8, 2), (1, ([1], [1]), 6, 2),
                                                 (1, ([1], [1]), 16, 1), (1, ([1], [1]), 4, 4)])
-def test_prefill_append_e4m3(ism, l_new, segs, hq, hkv, path, monkeypatch):
+def test_prefill_append_e4m3(ism, l_new, segs, hq, hkv, path, knobs):
     """e4m3 queries and caches (cache factors shared by the new keys / values)
     against the oracle on the dequantised values; single-token steps on the
     tensor-core decode or the CUDA-core one."""
     if path == "cuda_cores":
         if l_new != 1:
             pytest.skip("the decode path choice applies to single-token steps")
-        monkeypatch.setenv("ISM_DECODE_NO_TC", "1")
+        knobs("ISM_DECODE_NO_TC", "1")
     B, d = 3, 128
     c_lens = np.array([0, 77, 300], dtype=np.int32)
     cap = 300 + l_new + 5
@@ -951,11 +993,11 @@ def test_decode_long_cache(ism, keys):
 
 @pytest.mark.parametrize("dtype", ["bf16", "e4m3"])
 @pytest.mark.parametrize("n_split", ["0", "2", "1000"])
-def test_prefill_key_split(ism, dtype, n_split, monkeypatch):
+def test_prefill_key_split(ism, dtype, n_split, knobs):
     """Prefill items that run as two halves of their key range (the last ones,
     or all of them with 1000: some halves then have no key tile at all) give
     the oracle's result; ISM_PREFILL_SPLIT forces the count."""
-    monkeypatch.setenv("ISM_PREFILL_SPLIT", n_split)
+    knobs("ISM_PREFILL_SPLIT", n_split)
     B, d, hq, hkv, l_new = 3, 128, 8, 2, 200
     segs = ([40, 41, 120, 200], [0, 1, 0, 1])
     c_lens = np.array([0, 77, 300], dtype=np.int32)
