@@ -137,6 +137,17 @@ class ClockSampler:
     def mark_start(self):
         self.t0 = time.time()
 
+    def hold(self, step, sync, limit: float = 1.0):
+        """Keep running ``step`` (the timed work, outside the window) until a
+        sample taken after the window's start has arrived, at most ``limit``
+        seconds, so that short windows still get a clock record."""
+        t_end = time.time() + limit
+        while self.proc is not None and time.time() < t_end:
+            if any(t >= (self.t0 or 0) for t, _ in list(self.lines)):
+                break
+            step()
+            sync()
+
     def mark_end(self):
         self.t1 = time.time()
 
@@ -333,9 +344,7 @@ def run_cuda(args, w):
     launches = ism.kernel_launches() - launches0
     # keep the GPU busy with the same steps a little longer, so that a timed
     # region shorter than the sampling interval still gets a sample
-    for _ in range(3):
-        step()
-    torch.cuda.synchronize()
+    clocks.hold(step, torch.cuda.synchronize)
     clocks.__exit__(None, None, None)
     ism.check_status(dev)
 
@@ -517,6 +526,7 @@ def run_cuda(args, w):
         del ins, outs, ob, lb
         torch.cuda.empty_cache()
         line["bwd_min_workspace"] = measure_training_config(dev, w, peaks, steps=args.steps, minimal_workspace=True)
+        line["rope"] = measure_training_config(dev, w, peaks, steps=args.steps, rope=True)
         line["configs"] = {wname: measure_training_config(dev, WORKLOADS[wname](), peaks, steps=args.steps)
                            for wname in ("mha_4k", "packed_32k") if WORKLOADS[wname]().name != w.name}
     if not args.no_append:
@@ -595,7 +605,9 @@ def measure_append(dev, peaks):
     kus = float(np.median(dec_kernel_us[3:]))
     gbs = float(np.median(np.array(dec_bytes[3:]) / (np.array(dec_kernel_us[3:]) * 1e-6) / 1e9))
     # the same step through the plain binding (argument conversion, workspace
-    # and output allocation on every call)
+    # and output allocation on every call), over the last 16 positions again
+    c_host -= 16
+    cl.copy_(torch.from_numpy(c_host))
     plain_us = []
     for t in range(16):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -731,13 +743,14 @@ def measure_append_rope(dev, a, kc, vc, qn, kn, vn, qd, kd, vd, flush, decode_st
     return out
 
 
-def measure_training_config(dev, w, peaks, steps=20, minimal_workspace=False):
+def measure_training_config(dev, w, peaks, steps=20, minimal_workspace=False, rope=False):
     """fwd+bwd steps of one workload timed as the headline is: inputs resident,
     L2 flushed between steps (outside the events), CUDA events around each
     step, per-kernel times from separate steps through the library's timer
     hooks, clocks sampled over the timed steps.  minimal_workspace runs the
     backward with ism_attn_bwd_workspace_size_min bytes (the recompute
-    schedule: no stored dS)."""
+    schedule: no stored dS); rope runs the rotary forward and backward
+    (queries and keys rotated at their positions, the usual schedule)."""
     import torch
     from paper_2408_00539_gb300 import ism
     q, k, v, do = (t.to(dev) for t in wl.attention_tensors(w))
@@ -756,6 +769,16 @@ def measure_training_config(dev, w, peaks, steps=20, minimal_workspace=False):
         ism.fwd(segs, q, k, v, w.softmax_scale, out=o, lse=lse)
         ism.bwd(segs, q, k, v, o, lse, do, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws)
 
+    if rope:
+        cos_np, sin_np = wl.rope_tables(int(np.diff(w.segs.cu_seqlens).max()), D)
+        cos_t, sin_t = torch.from_numpy(cos_np).to(dev), torch.from_numpy(sin_np).to(dev)
+        q_rot, k_rot = torch.empty_like(q), torch.empty_like(k)
+
+        def step():  # noqa: F811
+            ism.fwd_rope(segs, q, k, v, cos_t, sin_t, w.softmax_scale, q_rot=q_rot, k_rot=k_rot, out=o, lse=lse)
+            ism.bwd_rope(segs, q_rot, k_rot, v, o, lse, do, cos_t, sin_t, w.softmax_scale, dq=dq, dk=dk, dv=dv,
+                         workspace=ws)
+
     with ClockSampler(dev.index) as clocks:
         for _ in range(3):
             step()
@@ -772,12 +795,12 @@ def measure_training_config(dev, w, peaks, steps=20, minimal_workspace=False):
             e1.synchronize()
             ms.append(e0.elapsed_time(e1))
         clocks.mark_end()
-        for _ in range(3):
-            step()
-        torch.cuda.synchronize()
+        clocks.hold(step, torch.cuda.synchronize)
     ism.check_status(dev)
     kinds = {"fwd": ism.KERNEL_FWD, "bwd_dkdv": ism.KERNEL_BWD_DKDV, "bwd_dq": ism.KERNEL_BWD_DQ,
              "bwd_pre": ism.KERNEL_BWD_PRE, "meta": ism.KERNEL_META}
+    if rope:
+        kinds["rope"] = ism.KERNEL_ROPE
     kt = {n: [] for n in kinds}
     for _ in range(5):
         flush.fill_(1)
@@ -801,7 +824,7 @@ def measure_training_config(dev, w, peaks, steps=20, minimal_workspace=False):
              "bwd_dkdv": 8 * D * n_vis / (mean_k["bwd_dkdv"] * 1e-3) / 1e12 / peak}
     out = {"workload": w.name, "tokens": w.total_tokens, "n_vis_pairs": n_vis, "flops_per_step": flops,
            "ms_per_step": ms_step, "steps": steps, "tflops": tflops, "pct_of_bf16_peak": tflops / peak * 100,
-           "bwd_schedule": "recompute dQ" if minimal_workspace else "stored dS",
+           "bwd_schedule": "recompute dQ" if minimal_workspace else "stored dS", "rope": rope,
            "bwd_workspace_bytes": ws_bytes, "kernel_ms": mean_k, "kernel_frac_of_bf16_peak": fracs,
            "clocks": clocks.summary()}
     del q, k, v, do, o, lse, dq, dk, dv, ws, flush

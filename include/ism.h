@@ -92,6 +92,22 @@ typedef struct {
   float softmax_scale;
 } ism_attn_shape_t;
 
+/* Rotary position encoding tables (positional encoding is outside the
+ * operation of Section 2.1, which leaves it out; models that take up ISM,
+ * Section 2.3, rotate queries and keys by their positions before attention).
+ * For a head row x at position p and k < D/2, the pair (x_k, x_{k+D/2}) is
+ * turned by the angle whose cosine and sine are cos[p * D/2 + k] and
+ * sin[p * D/2 + k]:
+ *     y_k = x_k cos - x_{k+D/2} sin,     y_{k+D/2} = x_{k+D/2} cos + x_k sin
+ * (the rotary encoding of RoFormer in its rotate-half form), in fp32 with one
+ * rounding to the element type.  cos / sin: fp32 device tables [rows, D/2],
+ * 16-byte aligned, read only.  Any angles are accepted. */
+typedef struct {
+  const float* cos;
+  const float* sin;
+  int32_t rows;
+} ism_rope_t;
+
 /* ---------------------------------------------------------------------------
  * Tile map.  Classifies each (q-tile, k-tile) rectangle of each sequence:
  * rows [t*bm, t*bm+bm) and keys [c*bn, c*bn+bn) relative to the sequence.
@@ -206,6 +222,39 @@ ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
                           void* workspace, size_t workspace_bytes, ism_stream_t stream);
 
 /* ---------------------------------------------------------------------------
+ * One-pass forward and backward with rotary encoding (see ism_rope_t).  The
+ * positions of a packed batch restart at every sequence: token t of sequence
+ * b sits at position t - cu_seqlens[b]; rope->rows must be at least the
+ * longest sequence.  bf16 or fp32 inputs, head_dim 64 or 128.
+ *
+ * ism_attn_fwd_rope rotates q [T, Hq, D] and k [T, Hkv, D] (unrotated) into
+ * q_rot / k_rot (same shapes and dtype, written; they may be q / k themselves
+ * for a rotation in place) in one pass over both, then runs ism_attn_fwd on
+ * q_rot, k_rot and v.  A training step keeps q_rot and k_rot for the
+ * backward, which takes them instead of q and k.
+ *
+ * ism_attn_bwd_rope is ism_attn_bwd on q_rot, k_rot (as written by the
+ * forward), v, o, lse, dout, except that dq and dk are the gradients with
+ * respect to the UNROTATED q and k: the gradients of the rotated rows go back
+ * through the transposed rotation (the rotation by the opposite angle).  On
+ * the tensor cores (bf16, head_dim 128) that happens in the dQ and dK
+ * epilogues; otherwise one more pass rotates dq and dk in place.
+ * Workspaces: ism_attn_fwd_workspace_size / ism_attn_bwd_workspace_size (or
+ * _min) of the same segments and shape.  Errors as ism_attn_fwd /
+ * ism_attn_bwd, plus ISM_ERR_INVALID_ARG for a missing or misaligned table,
+ * tables too short for the longest sequence, or e4m3 inputs.
+ * ------------------------------------------------------------------------- */
+ism_status_t ism_attn_fwd_rope(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                               const void* q, const void* k, const void* v, const ism_rope_t* rope,
+                               void* q_rot, void* k_rot, void* o, float* lse,
+                               void* workspace, size_t workspace_bytes, ism_stream_t stream);
+ism_status_t ism_attn_bwd_rope(const ism_segments_t* segs, const ism_attn_shape_t* shape,
+                               const void* q_rot, const void* k_rot, const void* v, const void* o,
+                               const float* lse, const void* dout, const ism_rope_t* rope,
+                               void* dq, void* dk, void* dv,
+                               void* workspace, size_t workspace_bytes, ism_stream_t stream);
+
+/* ---------------------------------------------------------------------------
  * Append-prefill of a new turn against a reused KV cache (Section 2.3: the
  * history's keys/values C_h are reused, the new chunk's C_q are computed and
  * [C_h; C_q] concatenated).  Valid because no token sees past the end of its
@@ -298,14 +347,8 @@ ism_status_t ism_attn_prefill_append_paged(const ism_attn_shape_t* shape, int32_
 
 /* ---------------------------------------------------------------------------
  * Append-prefill and decode with rotary position encoding applied on the way
- * into the cache.  Positional encoding is outside the operation of Section 2.1
- * (which leaves it out); models that take up ISM (Section 2.3) rotate queries
- * and keys by their absolute positions before attention.  Token j of
- * sequence b sits at position p = cache_len[b] + j; for k < D/2 the pair
- * (x_k, x_{k+D/2}) of its query and of its key is turned by the angle whose
- * cosine and sine are rope->cos[p * D/2 + k] and rope->sin[p * D/2 + k]:
- *     y_k = x_k cos - x_{k+D/2} sin,     y_{k+D/2} = x_{k+D/2} cos + x_k sin
- * (the rotary encoding of RoFormer in its rotate-half form), in fp32 and
+ * into the cache (see ism_rope_t).  Token j of sequence b sits at position
+ * p = cache_len[b] + j; its query and its key are rotated there, in fp32, and
  * rounded once to bf16.  The rotated keys are what the cache stores, values
  * are stored unchanged, and the new rows attend exactly as in
  * ism_attn_prefill_append, with the rotated queries.  The rotation runs inside
@@ -321,11 +364,6 @@ ism_status_t ism_attn_prefill_append_paged(const ism_attn_shape_t* shape, int32_
  * Errors: ISM_ERR_INVALID_ARG for a missing or misaligned table, rows too few
  * for the positions written, or a dtype other than ISM_BF16.
  * ------------------------------------------------------------------------- */
-typedef struct {
-  const float* cos;
-  const float* sin;
-  int32_t rows;
-} ism_rope_t;
 ism_status_t ism_attn_prefill_append_rope_workspace_size(const ism_attn_shape_t* shape, int32_t batch,
                                                          int32_t l_new, size_t* bytes);
 ism_status_t ism_attn_prefill_append_rope(const ism_attn_shape_t* shape, int32_t batch,
@@ -336,6 +374,51 @@ ism_status_t ism_attn_prefill_append_rope(const ism_attn_shape_t* shape, int32_t
                                           int32_t* cache_len, const int32_t* cache_len_host,
                                           const ism_rope_t* rope, void* o_new, float* lse_new,
                                           void* workspace, size_t workspace_bytes, ism_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * The rotary append on the other cache layouts: the operation of
+ * ism_attn_prefill_append_rope (Section 2.3 with rotary encoding, see
+ * ism_rope_t; token j of sequence b at position cache_len[b] + j) against a
+ * paged bf16 cache (the layout and arguments of ism_attn_prefill_append_paged)
+ * or an e4m3 cache (those of ism_attn_prefill_append_e4m3).
+ *
+ * ism_attn_prefill_append_paged_rope: shape->dtype ISM_BF16; results equal
+ * those of ism_attn_prefill_append_rope on the gathered cache.
+ *
+ * ism_attn_prefill_append_e4m3_rope: shape->dtype ISM_E4M3 (the caches and the
+ * attention), head_dim 128, but q_new, k_new and v_new are bf16 and
+ * UNROTATED: the pass that writes the cache rotates queries and keys in fp32
+ * and then quantises, so that the stored keys are rounded once.  Rotated keys
+ * are stored as round(k_rot / k_descale), values as round(v / v_descale)
+ * (e4m3, round to nearest, saturating at +-448), and the rotated queries
+ * round(q_rot / q_descale) go to the workspace; the attention is that of
+ * ism_attn_prefill_append_e4m3 with these factors.  A rotation can raise a
+ * coordinate up to sqrt(2) times the largest input coordinate; choose the
+ * factors with that headroom.
+ *
+ * Workspace (both): ism_attn_prefill_append_rope_workspace_size with the same
+ * shape.  Errors as the append they extend, plus ISM_ERR_INVALID_ARG for a
+ * NULL rope, a missing or misaligned table, or tables shorter than the
+ * positions written.
+ * ------------------------------------------------------------------------- */
+ism_status_t ism_attn_prefill_append_paged_rope(const ism_attn_shape_t* shape, int32_t batch,
+                                                const void* q_new, const void* k_new, const void* v_new,
+                                                int32_t l_new, const int32_t* new_seg_end_host,
+                                                const uint8_t* new_seg_type_host, int32_t n_new_segs,
+                                                void* k_pool, void* v_pool, int32_t num_pages, int32_t page_size,
+                                                const int32_t* block_table, const int32_t* block_table_host,
+                                                int32_t max_pages, int32_t* cache_len, const int32_t* cache_len_host,
+                                                const ism_rope_t* rope, void* o_new, float* lse_new,
+                                                void* workspace, size_t workspace_bytes, ism_stream_t stream);
+ism_status_t ism_attn_prefill_append_e4m3_rope(const ism_attn_shape_t* shape, int32_t batch,
+                                               const void* q_new, const void* k_new, const void* v_new,
+                                               int32_t l_new, const int32_t* new_seg_end_host,
+                                               const uint8_t* new_seg_type_host, int32_t n_new_segs,
+                                               void* k_cache, void* v_cache, int64_t cache_capacity,
+                                               int32_t* cache_len, const int32_t* cache_len_host,
+                                               float q_descale, float k_descale, float v_descale,
+                                               const ism_rope_t* rope, void* o_new, float* lse_new,
+                                               void* workspace, size_t workspace_bytes, ism_stream_t stream);
 
 /* ---------------------------------------------------------------------------
  * Status and diagnostics.
@@ -366,7 +449,8 @@ enum {
   ISM_KERNEL_BWD_DQ = 3,     /* backward dQ */
   ISM_KERNEL_BWD_PRE = 4,    /* backward preprocessing (Delta) */
   ISM_KERNEL_DECODE = 5,     /* single-token append (split-KV + merge) */
-  ISM_KERNEL_META = 6        /* tile map / work lists */
+  ISM_KERNEL_META = 6,       /* tile map / work lists */
+  ISM_KERNEL_ROPE = 7        /* rotary encoding pass of the one-pass forward (and CUDA-core backward) */
 };
 ism_status_t ism_set_kernel_timer(int32_t kernel_id, void* start_event, void* stop_event);
 uint64_t ism_kernel_launches(void);

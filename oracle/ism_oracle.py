@@ -422,3 +422,50 @@ def prefill_append_rope(q_new, k_new, v_new, k_cache, v_cache, cache_len, new_se
     k_used = k_rot if key_round is None else _f64(key_round(k_rot))
     o, lse = prefill_append(q_rot, k_used, v_new, k_cache, v_cache, cache_len, new_seg_end, new_seg_type, scale)
     return o, lse, k_rot
+
+
+# --------------------------------------------------------------------------
+# Rotary position encoding on the one-pass training path.  The positions of a
+# packed batch restart at every sequence: token t of sequence b (rows
+# cu_seqlens[b] <= t < cu_seqlens[b+1]) sits at position t - cu_seqlens[b].
+# The attention of Eq. (e_ISM) then runs on the rotated queries and keys.
+# --------------------------------------------------------------------------
+
+def seq_positions(segs) -> np.ndarray:
+    """Position of every token of a varlen batch: its index inside its own
+    packed sequence."""
+    pos = []
+    for b in range(int(segs.cu_seqlens.shape[0]) - 1):
+        _, L, _, _ = segs.seq(b)
+        pos.extend(range(L))
+    return np.asarray(pos, dtype=np.int64)
+
+
+def attn_fwd_rope(q, k, v, segs, scale: float, cos_table, sin_table, round_fn=None):
+    """Forward with rotary encoding: q and k are rotated at their positions in
+    their sequences (``rope_rotate``), ``round_fn`` (when given) maps the
+    rotated values to those the attention is computed on (e.g. the element
+    type they are stored in), then ``attn_fwd``.  Returns (O, LSE, q_rot,
+    k_rot), the last two before rounding."""
+    pos = seq_positions(segs)
+    q_rot = rope_rotate(q, pos, cos_table, sin_table)
+    k_rot = rope_rotate(k, pos, cos_table, sin_table)
+    qa, ka = (q_rot, k_rot) if round_fn is None else (_f64(round_fn(q_rot)), _f64(round_fn(k_rot)))
+    o, lse = attn_fwd(qa, ka, v, segs, scale)
+    return o, lse, q_rot, k_rot
+
+
+def attn_bwd_rope(q, k, v, dout, segs, scale: float, cos_table, sin_table, round_fn=None):
+    """Gradients of the rotary forward with respect to the unrotated q, k and
+    to v.  The chain rule through y = R x is dx = R^T dy, and the transpose of
+    a rotation is the rotation by the opposite angle: the gradients of the
+    rotated queries and keys (``attn_bwd`` on the rotated, optionally rounded,
+    values) are rotated back with the sines negated."""
+    pos = seq_positions(segs)
+    q_rot = rope_rotate(q, pos, cos_table, sin_table)
+    k_rot = rope_rotate(k, pos, cos_table, sin_table)
+    if round_fn is not None:
+        q_rot, k_rot = _f64(round_fn(q_rot)), _f64(round_fn(k_rot))
+    dq_rot, dk_rot, dv = attn_bwd(q_rot, k_rot, v, dout, segs, scale)
+    neg_sin = -_f64(sin_table)
+    return rope_rotate(dq_rot, pos, cos_table, neg_sin), rope_rotate(dk_rot, pos, cos_table, neg_sin), dv

@@ -447,19 +447,40 @@ namespace {
 
 // The one-pass forward for bf16 / fp32 (ism_attn_fwd) and e4m3 inputs
 // (ism_attn_fwd_e4m3; qk_descale = q_descale * k_descale).
+// Checks the rotary tables of a one-pass call: present, aligned, covering
+// every position of the batch (the longest sequence), for bf16 / fp32 inputs.
+ism_status_t check_rope_pass(const ism_rope_t* rope, const ism_attn_shape_t* shape, const SegInfo& info) {
+  if (!rope) return fail(ISM_ERR_INVALID_ARG, "rope is NULL");
+  if (shape->dtype != ISM_BF16 && shape->dtype != ISM_FP32)
+    return fail(ISM_ERR_INVALID_ARG, "rotary encoding on the one-pass path needs bf16 or fp32 inputs");
+  if (!rope->cos || !rope->sin || !aligned16(rope->cos) || !aligned16(rope->sin))
+    return fail(ISM_ERR_INVALID_ARG, "rope tables must be non-NULL and 16-byte aligned");
+  if (info.max_len > rope->rows)
+    return fail(ISM_ERR_INVALID_ARG, "rope tables cover %d positions, the longest sequence has %lld tokens", rope->rows,
+                (long long)info.max_len);
+  return ISM_OK;
+}
+
+// The one-pass forward for bf16 / fp32 (ism_attn_fwd) and e4m3 inputs
+// (ism_attn_fwd_e4m3; qk_descale = q_descale * k_descale); with rope set,
+// q and k are first rotated into q_rot / k_rot and the attention reads those.
 ism_status_t fwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q, const void* k,
                       const void* v, void* o, float* lse, void* workspace, size_t workspace_bytes, ism_stream_t stream,
-                      float qk_descale, float v_descale) {
+                      float qk_descale, float v_descale, const ism_rope_t* rope = nullptr, void* q_rot = nullptr,
+                      void* k_rot = nullptr) {
   SegInfo info;
   ism_status_t r = check_segments(segs, &info);
   if (r != ISM_OK) return r;
   const bool e4m3 = shape && shape->dtype == ISM_E4M3;
   if ((r = check_shape(shape, e4m3)) != ISM_OK) return r;
   if (e4m3 && !tc_available()) return fail(ISM_ERR_UNSUPPORTED, "e4m3 forward needs the sm_103 tensor cores");
+  if (rope && (r = check_rope_pass(rope, shape, info)) != ISM_OK) return r;
   if (info.total_tokens == 0) return ISM_OK;
   if (!q || !k || !v || !o) return fail(ISM_ERR_INVALID_ARG, "q, k, v, o must be non-NULL");
   if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || (lse && !aligned16(lse)))
     return fail(ISM_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
+  if (rope && (!q_rot || !k_rot || !aligned16(q_rot) || !aligned16(k_rot)))
+    return fail(ISM_ERR_INVALID_ARG, "q_rot and k_rot must be non-NULL and 16-byte aligned");
   Counts c = count_tiles(segs, kTile, kTile);
   PassLayout L =
       pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, false, 0, fwd_tile_pairs(shape));
@@ -467,6 +488,17 @@ ism_status_t fwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape,
   uint32_t* status;
   if ((r = status_ptr(&status)) != ISM_OK) return r;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (rope) {
+    timer_begin(ISM_KERNEL_ROPE, st);
+    ISM_TRY_CUDA(launch_rope_rows(segs->cu_seqlens, segs->num_seqs, info.total_tokens, shape->num_heads_q,
+                                  shape->num_heads_kv, shape->head_dim, shape->dtype, q, k, q_rot, k_rot, rope->cos,
+                                  rope->sin, 1.f, st),
+                 "rope launch");
+    timer_end(ISM_KERNEL_ROPE, st);
+    count_launch(1);
+    q = q_rot;
+    k = k_rot;
+  }
   if ((r = build_pass_meta(segs, c, L, false, st)) != ISM_OK) return r;
 
   AttnArgs a{};
@@ -518,14 +550,27 @@ ism_status_t ism_attn_fwd_e4m3(const ism_segments_t* segs, const ism_attn_shape_
   return fwd_impl(segs, shape, q, k, v, o, lse, workspace, workspace_bytes, stream, q_descale * k_descale, v_descale);
 }
 
-ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q,
-                          const void* k, const void* v, const void* o, const float* lse, const void* dout,
-                          void* dq, void* dk, void* dv, void* workspace, size_t workspace_bytes,
-                          ism_stream_t stream) {
+ism_status_t ism_attn_fwd_rope(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q,
+                               const void* k, const void* v, const ism_rope_t* rope, void* q_rot, void* k_rot,
+                               void* o, float* lse, void* workspace, size_t workspace_bytes, ism_stream_t stream) {
+  if (shape && shape->dtype == ISM_E4M3)
+    return fail(ISM_ERR_INVALID_ARG, "rotary encoding on the one-pass path needs bf16 or fp32 inputs");
+  if (!rope) return fail(ISM_ERR_INVALID_ARG, "rope is NULL");
+  return fwd_impl(segs, shape, q, k, v, o, lse, workspace, workspace_bytes, stream, 1.f, 1.f, rope, q_rot, k_rot);
+}
+
+}  // extern "C"
+
+namespace {
+
+ism_status_t bwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q, const void* k,
+                      const void* v, const void* o, const float* lse, const void* dout, void* dq, void* dk, void* dv,
+                      void* workspace, size_t workspace_bytes, ism_stream_t stream, const ism_rope_t* rope) {
   SegInfo info;
   ism_status_t r = check_segments(segs, &info);
   if (r != ISM_OK) return r;
   if ((r = check_shape(shape)) != ISM_OK) return r;
+  if (rope && (r = check_rope_pass(rope, shape, info)) != ISM_OK) return r;
   if (info.total_tokens == 0) return ISM_OK;
   if (!q || !k || !v || !o || !lse || !dout || !dq || !dk || !dv)
     return fail(ISM_ERR_INVALID_ARG, "q, k, v, o, lse, dout, dq, dk, dv must be non-NULL");
@@ -556,11 +601,43 @@ ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* sh
   a.status = status;
   a.flags = tc_flags();
   if (use_tc_bwd(shape)) {
+    if (rope) {  // the dQ and dK epilogues rotate the gradients back
+      a.rope_cos = rope->cos;
+      a.rope_sin = rope->sin;
+    }
     ISM_TRY_CUDA(launch_tc_bwd(a, info.total_tokens, st), "tensor-core backward launch");
   } else {
     ISM_TRY_CUDA(launch_simt_bwd(a, st), "backward launch");
+    if (rope) {  // gradients of the rotated rows, rotated back in place
+      timer_begin(ISM_KERNEL_ROPE, st);
+      ISM_TRY_CUDA(launch_rope_rows(segs->cu_seqlens, segs->num_seqs, info.total_tokens, shape->num_heads_q,
+                                    shape->num_heads_kv, shape->head_dim, shape->dtype, dq, dk, dq, dk, rope->cos,
+                                    rope->sin, -1.f, st),
+                   "rope launch");
+      timer_end(ISM_KERNEL_ROPE, st);
+      count_launch(1);
+    }
   }
   return ISM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+ism_status_t ism_attn_bwd(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q,
+                          const void* k, const void* v, const void* o, const float* lse, const void* dout,
+                          void* dq, void* dk, void* dv, void* workspace, size_t workspace_bytes,
+                          ism_stream_t stream) {
+  return bwd_impl(segs, shape, q, k, v, o, lse, dout, dq, dk, dv, workspace, workspace_bytes, stream, nullptr);
+}
+
+ism_status_t ism_attn_bwd_rope(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q_rot,
+                               const void* k_rot, const void* v, const void* o, const float* lse, const void* dout,
+                               const ism_rope_t* rope, void* dq, void* dk, void* dv, void* workspace,
+                               size_t workspace_bytes, ism_stream_t stream) {
+  if (!rope) return fail(ISM_ERR_INVALID_ARG, "rope is NULL");
+  return bwd_impl(segs, shape, q_rot, k_rot, v, o, lse, dout, dq, dk, dv, workspace, workspace_bytes, stream, rope);
 }
 
 // ---------------------------------------------------------------- append
@@ -632,7 +709,7 @@ ism_status_t ism_attn_prefill_append_workspace_size(const ism_attn_shape_t* shap
 
 ism_status_t ism_attn_prefill_append_rope_workspace_size(const ism_attn_shape_t* shape, int32_t batch,
                                                          int32_t l_new, size_t* bytes) {
-  ism_status_t r = check_shape(shape);
+  ism_status_t r = check_shape(shape, true);
   if (r != ISM_OK) return r;
   if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
   if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
@@ -659,7 +736,9 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
                          const uint8_t* new_seg_type_host, int32_t n_new_segs, void* k_cache, void* v_cache,
                          const CacheGeom& cg, int32_t* cache_len, const int32_t* cache_len_host, void* o_new,
                          float* lse_new, void* workspace, size_t workspace_bytes, cudaStream_t st,
-                         float qk_descale = 1.f, float v_descale = 1.f, const ism_rope_t* rope = nullptr) {
+                         float q_descale = 1.f, float k_descale = 1.f, float v_descale = 1.f,
+                         const ism_rope_t* rope = nullptr) {
+  const float qk_descale = q_descale * k_descale;
   ism_status_t r;
   if (!q_new || !k_new || !v_new || !k_cache || !v_cache || !cache_len || !cache_len_host || !o_new)
     return fail(ISM_ERR_INVALID_ARG, "q_new, k_new, v_new, caches, cache_len (device+host), o_new must be non-NULL");
@@ -718,8 +797,9 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
   const int32_t* c_src = decode ? cache_len : L.c_snap;
   int32_t* snap_out = decode ? L.c_snap : nullptr;
   if (rope) {
-    ISM_TRY_CUDA(launch_rope_cache_write(batch, l_new, hq, hkv, d, cg.cap, cg.pages, c_src, q_new, k_new, v_new,
-                                         rope->cos, rope->sin, L.q_rot, k_cache, v_cache, st, snap_out),
+    ISM_TRY_CUDA(launch_rope_cache_write(shape->dtype, batch, l_new, hq, hkv, d, cg.cap, cg.pages, c_src, q_new,
+                                         k_new, v_new, rope->cos, rope->sin, q_descale, k_descale, v_descale,
+                                         L.q_rot, k_cache, v_cache, st, snap_out),
                  "rope cache write launch");
     q_new = L.q_rot;  // the attention below reads the rotated queries
   } else {
@@ -892,7 +972,7 @@ ism_status_t ism_attn_prefill_append_e4m3(const ism_attn_shape_t* shape, int32_t
   cg.pages = KvPages{nullptr, 0, 0};
   return append_impl(shape, batch, q_new, k_new, v_new, l_new, new_seg_end_host, new_seg_type_host, n_new_segs,
                      k_cache, v_cache, cg, cache_len, cache_len_host, o_new, lse_new, workspace, workspace_bytes,
-                     reinterpret_cast<cudaStream_t>(stream), q_descale * k_descale, v_descale);
+                     reinterpret_cast<cudaStream_t>(stream), q_descale, k_descale, v_descale);
 }
 
 ism_status_t ism_attn_prefill_append_rope(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,
@@ -917,8 +997,75 @@ ism_status_t ism_attn_prefill_append_rope(const ism_attn_shape_t* shape, int32_t
   cg.pages = KvPages{nullptr, 0, 0};
   return append_impl(shape, batch, q_new, k_new, v_new, l_new, new_seg_end_host, new_seg_type_host, n_new_segs,
                      k_cache, v_cache, cg, cache_len, cache_len_host, o_new, lse_new, workspace, workspace_bytes,
-                     reinterpret_cast<cudaStream_t>(stream), 1.f, 1.f, rope);
+                     reinterpret_cast<cudaStream_t>(stream), 1.f, 1.f, 1.f, rope);
 }
+
+ism_status_t ism_attn_prefill_append_e4m3_rope(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,
+                                               const void* k_new, const void* v_new, int32_t l_new,
+                                               const int32_t* new_seg_end_host, const uint8_t* new_seg_type_host,
+                                               int32_t n_new_segs, void* k_cache, void* v_cache,
+                                               int64_t cache_capacity, int32_t* cache_len,
+                                               const int32_t* cache_len_host, float q_descale, float k_descale,
+                                               float v_descale, const ism_rope_t* rope, void* o_new, float* lse_new,
+                                               void* workspace, size_t workspace_bytes, ism_stream_t stream) {
+  ism_status_t r = check_shape(shape, true);
+  if (r != ISM_OK) return r;
+  if (shape->dtype != ISM_E4M3) return fail(ISM_ERR_INVALID_ARG, "ism_attn_prefill_append_e4m3_rope needs ISM_E4M3");
+  if (!valid_descales(q_descale, k_descale, v_descale))
+    return fail(ISM_ERR_INVALID_ARG, "descales must be positive finite numbers");
+  if (!rope) return fail(ISM_ERR_INVALID_ARG, "rope is NULL");
+  if (!tc_available()) return fail(ISM_ERR_UNSUPPORTED, "e4m3 attention needs the sm_103 tensor cores");
+  if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
+  if (batch == 0 || l_new == 0) return ISM_OK;
+  if (cache_capacity <= 0 || (int64_t)batch * cache_capacity >= (int64_t(1) << 31))
+    return fail(ISM_ERR_INVALID_ARG, "batch * cache_capacity must be in (0, 2^31)");
+  CacheGeom cg;
+  cg.cap = cache_capacity;
+  cg.kv_rows = (int64_t)batch * cache_capacity;
+  cg.max_keys = cache_capacity;
+  cg.pages = KvPages{nullptr, 0, 0};
+  return append_impl(shape, batch, q_new, k_new, v_new, l_new, new_seg_end_host, new_seg_type_host, n_new_segs,
+                     k_cache, v_cache, cg, cache_len, cache_len_host, o_new, lse_new, workspace, workspace_bytes,
+                     reinterpret_cast<cudaStream_t>(stream), q_descale, k_descale, v_descale, rope);
+}
+
+}  // extern "C"
+
+namespace {
+
+// Validates a paged cache and describes it: every page a sequence reads or
+// writes in this call lies in the pool.
+ism_status_t paged_geom(int32_t batch, int32_t l_new, int32_t num_pages, int32_t page_size,
+                        const int32_t* block_table, const int32_t* block_table_host, int32_t max_pages,
+                        const int32_t* cache_len_host, CacheGeom* cg) {
+  if (page_size <= 0 || page_size % kTile != 0)
+    return fail(ISM_ERR_INVALID_ARG, "page_size %d must be a positive multiple of %d", page_size, kTile);
+  if (num_pages <= 0 || (int64_t)num_pages * page_size >= (int64_t(1) << 31))
+    return fail(ISM_ERR_INVALID_ARG, "num_pages * page_size must be in (0, 2^31)");
+  if (max_pages <= 0 || !block_table || !block_table_host || !cache_len_host)
+    return fail(ISM_ERR_INVALID_ARG, "block_table (device+host), cache_len_host and max_pages > 0 are required");
+  for (int b = 0; b < batch; ++b) {
+    const int64_t keys = (int64_t)cache_len_host[b] + l_new;
+    if (cache_len_host[b] < 0 || keys > (int64_t)max_pages * page_size)
+      return fail(ISM_ERR_INVALID_ARG, "sequence %d: cache_len %d + l_new %d exceeds its %d pages", b, cache_len_host[b],
+                  l_new, max_pages);
+    for (int64_t i = 0; i < (keys + page_size - 1) / page_size; ++i) {
+      const int32_t pg = block_table_host[(int64_t)b * max_pages + i];
+      if (pg < 0 || pg >= num_pages)
+        return fail(ISM_ERR_INVALID_ARG, "sequence %d: page %lld of the block table is %d, outside [0, %d)", b,
+                    (long long)i, pg, num_pages);
+    }
+  }
+  cg->cap = 0;
+  cg->kv_rows = (int64_t)num_pages * page_size;
+  cg->max_keys = (int64_t)max_pages * page_size;
+  cg->pages = KvPages{block_table, page_size, max_pages};
+  return ISM_OK;
+}
+
+}  // namespace
+
+extern "C" {
 
 ism_status_t ism_attn_prefill_append_paged(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,
                                            const void* k_new, const void* v_new, int32_t l_new,
@@ -932,33 +1079,38 @@ ism_status_t ism_attn_prefill_append_paged(const ism_attn_shape_t* shape, int32_
   if (r != ISM_OK) return r;
   if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
   if (batch == 0 || l_new == 0) return ISM_OK;
-  if (page_size <= 0 || page_size % kTile != 0)
-    return fail(ISM_ERR_INVALID_ARG, "page_size %d must be a positive multiple of %d", page_size, kTile);
-  if (num_pages <= 0 || (int64_t)num_pages * page_size >= (int64_t(1) << 31))
-    return fail(ISM_ERR_INVALID_ARG, "num_pages * page_size must be in (0, 2^31)");
-  if (max_pages <= 0 || !block_table || !block_table_host || !cache_len_host)
-    return fail(ISM_ERR_INVALID_ARG, "block_table (device+host), cache_len_host and max_pages > 0 are required");
-  // every page a sequence reads or writes in this call lies in the pool
-  for (int b = 0; b < batch; ++b) {
-    const int64_t keys = (int64_t)cache_len_host[b] + l_new;
-    if (cache_len_host[b] < 0 || keys > (int64_t)max_pages * page_size)
-      return fail(ISM_ERR_INVALID_ARG, "sequence %d: cache_len %d + l_new %d exceeds its %d pages", b, cache_len_host[b],
-                  l_new, max_pages);
-    for (int64_t i = 0; i < (keys + page_size - 1) / page_size; ++i) {
-      const int32_t pg = block_table_host[(int64_t)b * max_pages + i];
-      if (pg < 0 || pg >= num_pages)
-        return fail(ISM_ERR_INVALID_ARG, "sequence %d: page %lld of the block table is %d, outside [0, %d)", b,
-                    (long long)i, pg, num_pages);
-    }
-  }
   CacheGeom cg;
-  cg.cap = 0;
-  cg.kv_rows = (int64_t)num_pages * page_size;
-  cg.max_keys = (int64_t)max_pages * page_size;
-  cg.pages = KvPages{block_table, page_size, max_pages};
+  if ((r = paged_geom(batch, l_new, num_pages, page_size, block_table, block_table_host, max_pages, cache_len_host,
+                      &cg)) != ISM_OK)
+    return r;
   return append_impl(shape, batch, q_new, k_new, v_new, l_new, new_seg_end_host, new_seg_type_host, n_new_segs,
                      k_pool, v_pool, cg, cache_len, cache_len_host, o_new, lse_new, workspace, workspace_bytes,
                      reinterpret_cast<cudaStream_t>(stream));
+}
+
+ism_status_t ism_attn_prefill_append_paged_rope(const ism_attn_shape_t* shape, int32_t batch, const void* q_new,
+                                                const void* k_new, const void* v_new, int32_t l_new,
+                                                const int32_t* new_seg_end_host, const uint8_t* new_seg_type_host,
+                                                int32_t n_new_segs, void* k_pool, void* v_pool, int32_t num_pages,
+                                                int32_t page_size, const int32_t* block_table,
+                                                const int32_t* block_table_host, int32_t max_pages,
+                                                int32_t* cache_len, const int32_t* cache_len_host,
+                                                const ism_rope_t* rope, void* o_new, float* lse_new, void* workspace,
+                                                size_t workspace_bytes, ism_stream_t stream) {
+  ism_status_t r = check_shape(shape);
+  if (r != ISM_OK) return r;
+  if (shape->dtype != ISM_BF16)
+    return fail(ISM_ERR_INVALID_ARG, "ism_attn_prefill_append_paged_rope needs ISM_BF16");
+  if (!rope) return fail(ISM_ERR_INVALID_ARG, "rope is NULL");
+  if (batch < 0 || l_new < 0) return fail(ISM_ERR_INVALID_ARG, "batch and l_new must be >= 0");
+  if (batch == 0 || l_new == 0) return ISM_OK;
+  CacheGeom cg;
+  if ((r = paged_geom(batch, l_new, num_pages, page_size, block_table, block_table_host, max_pages, cache_len_host,
+                      &cg)) != ISM_OK)
+    return r;
+  return append_impl(shape, batch, q_new, k_new, v_new, l_new, new_seg_end_host, new_seg_type_host, n_new_segs,
+                     k_pool, v_pool, cg, cache_len, cache_len_host, o_new, lse_new, workspace, workspace_bytes,
+                     reinterpret_cast<cudaStream_t>(stream), 1.f, 1.f, 1.f, rope);
 }
 
 // ---------------------------------------------------------------- status

@@ -322,11 +322,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
       ptx::tc_fence_after();
       uint32_t q0[32], q1[32];
-      ld64(tmem + lane_addr + TM_DQ + wg * 64, q0, q1);
+      if (a.rope_cos) {
+        // rotary encoding: warpgroup wg takes columns wg*32.. and 64 + wg*32.., which pair up
+        ptx::tmem_ld32(tmem + lane_addr + TM_DQ + wg * 32, q0);
+        ptx::tmem_ld32(tmem + lane_addr + TM_DQ + 64 + wg * 32, q1);
+      } else {
+        ld64(tmem + lane_addr + TM_DQ + wg * 64, q0, q1);
+      }
       ptx::tmem_ld_wait();
       ptx::reg_fence(q0);
       ptx::reg_fence(q1);
-      if (valid) {
+      if (valid && a.rope_cos) {
+        const int64_t pos = (int64_t)w.tile * kRows + r;
+        uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) + grow * a.hq * kD + h * kD);
+        rope_back_store32(q0, q1, a.scale, a.rope_cos + pos * 64 + wg * 32, a.rope_sin + pos * 64 + wg * 32,
+                          dst + 4 * wg, dst + 8 + 4 * wg);
+      } else if (valid) {
         uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) + grow * a.hq * kD + h * kD +
                                               wg * 64);
 #pragma unroll
@@ -862,6 +873,24 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
       __nv_bfloat16* outp = reinterpret_cast<__nv_bfloat16*>(wg == 0 ? a.dv : a.dk) + krow * a.hkv * kD + x.g * kD;
       const float f = wg == 0 ? 1.f : a.scale;
       const uint32_t col = wg == 0 ? TM_DV : TM_DK;
+      if (wg == 1 && a.rope_cos) {
+        // rotary encoding: dK of the unrotated keys, columns k and k + 64 pair up
+#pragma unroll 1
+        for (int q2 = 0; q2 < 2; ++q2) {
+          uint32_t lo[32], hi[32];
+          ptx::tmem_ld32(tmem + lane_addr + col + q2 * 32, lo);
+          ptx::tmem_ld32(tmem + lane_addr + col + 64 + q2 * 32, hi);
+          ptx::tmem_ld_wait();
+          ptx::reg_fence(lo);
+          ptx::reg_fence(hi);
+          if (kvalid)
+            rope_back_store32(lo, hi, f, a.rope_cos + (int64_t)key * 64 + 32 * q2,
+                              a.rope_sin + (int64_t)key * 64 + 32 * q2, reinterpret_cast<uint4*>(outp + q2 * 32),
+                              reinterpret_cast<uint4*>(outp + 64 + q2 * 32));
+        }
+        ptx::tc_fence_before();
+        continue;
+      }
 #pragma unroll 1
       for (int q4 = 0; q4 < 4; ++q4) {
         uint32_t v[32];

@@ -171,6 +171,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tc_fence_after();
       uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) +
                                             ((int64_t)x.w.q_base + row) * a.hq * kD + x.h * kD);
+      if (a.rope_cos) {
+        // rotary encoding: columns k and k + 64 of the row pair up
+#pragma unroll 1
+        for (int q2 = 0; q2 < 2; ++q2) {
+          uint32_t lo[32], hi[32];
+          if (x.nkb > 0) {
+            ptx::tmem_ld32(acc + 32 * q2, lo);
+            ptx::tmem_ld32(acc + 64 + 32 * q2, hi);
+            ptx::tmem_ld_wait();
+            ptx::reg_fence(lo);
+            ptx::reg_fence(hi);
+          } else {
+#pragma unroll
+            for (int k = 0; k < 32; ++k) lo[k] = hi[k] = 0u;
+          }
+          if (valid)
+            rope_back_store32(lo, hi, a.scale, a.rope_cos + (int64_t)row * 64 + 32 * q2,
+                              a.rope_sin + (int64_t)row * 64 + 32 * q2, dst + 4 * q2, dst + 8 + 4 * q2);
+        }
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(&bar->acc_empty[b]);
+        continue;
+      }
 #pragma unroll 1
       for (int q4 = 0; q4 < 4; ++q4) {
         uint32_t v[32];

@@ -96,14 +96,24 @@ cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t kbase_
 cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, int64_t cap, const KvPages& pages,
                                const int32_t* c_snap, const void* k_new, const void* v_new,
                                void* k_cache, void* v_cache, cudaStream_t st, int32_t* snap_out = nullptr);
-// Cache write with the rotary encoding of the new queries and keys (bf16,
-// head_dim a multiple of 16): rotated keys and plain values into the cache,
-// rotated queries into q_rot [batch * l_new, hq, d].
-cudaError_t launch_rope_cache_write(int batch, int l_new, int hq, int hkv, int d, int64_t cap,
+// Cache write with the rotary encoding of the new queries and keys (bf16
+// inputs, head_dim a multiple of 16): rotated keys and plain values into the
+// cache, rotated queries into q_rot [batch * l_new, hq, d], all in the cache's
+// type: bf16, or e4m3 (dtype ISM_E4M3) after division by the descales.
+cudaError_t launch_rope_cache_write(int dtype, int batch, int l_new, int hq, int hkv, int d, int64_t cap,
                                    const KvPages& pages, const int32_t* c_snap, const void* q_new,
                                    const void* k_new, const void* v_new, const float* cos_t, const float* sin_t,
-                                   void* q_rot, void* k_cache, void* v_cache, cudaStream_t st,
-                                   int32_t* snap_out = nullptr);
+                                   float q_descale, float k_descale, float v_descale, void* q_rot, void* k_cache,
+                                   void* v_cache, cudaStream_t st, int32_t* snap_out = nullptr);
+
+// Rotary encoding of the one-pass path (ism_rope.cu): rotates every query and
+// key head row of a packed batch by its position inside its sequence (pairs
+// k, k + d/2; tables [rows, d/2] fp32), from q_src / k_src into q_dst / k_dst
+// (in place allowed).  sin_sign = -1 applies the transposed rotation.  bf16
+// or fp32 rows, d a multiple of 16.
+cudaError_t launch_rope_rows(const int32_t* cu_seqlens, int num_seqs, int64_t T, int hq, int hkv, int d, int dtype,
+                             const void* q_src, const void* k_src, void* q_dst, void* k_dst, const float* cos_t,
+                             const float* sin_t, float sin_sign, cudaStream_t st);
 
 // CUDA-core attention (ism_simt.cu), fp32 or bf16 storage, fp32 math.
 struct AttnArgs {
@@ -146,6 +156,12 @@ struct AttnArgs {
   int64_t split_whole, split_items;
   float* part_o;    // [split_items][2 halves][2 heads][128 rows][128] fp32
   float* part_ml;   // [split_items][2 halves][2 heads][128 rows][2] fp32
+  // Rotary encoding (tensor-core backward only): when rope_cos is set, the dQ
+  // and dK epilogues store the gradients of the unrotated queries and keys,
+  // applying the transposed rotation of the row's position in its sequence
+  // (tables [rows, 64] fp32, the angle of pair k of position p at p * 64 + k).
+  const float* rope_cos;
+  const float* rope_sin;
   // Bit 0: before an MMA that overwrites tensor memory an earlier MMA reads
   // as its A operand, wait for that earlier MMA to complete.  Clear: rely on
   // MMAs issued by one thread executing in issue order.

@@ -390,28 +390,50 @@ __global__ void cache_write_kernel(int batch, int l_new, int row_bytes, int64_t 
 // consecutive coordinates k0..k0+7 of the first half of one head row and
 // their partners k0+D/2.. (a query head, a key head, or a value head, which
 // is copied as is).  Position of new token j of sequence b: c_snap[b] + j.
-__device__ __forceinline__ void rotate8(const uint4& lo, const uint4& hi, const float* c, const float* s,
-                                        uint4& out_lo, uint4& out_hi) {
-  const __nv_bfloat162* l2 = reinterpret_cast<const __nv_bfloat162*>(&lo);
-  const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&hi);
-  __nv_bfloat162* ol = reinterpret_cast<__nv_bfloat162*>(&out_lo);
-  __nv_bfloat162* oh = reinterpret_cast<__nv_bfloat162*>(&out_hi);
+// The rotation is in fp32; the results are rounded once to the cache's type:
+// bf16, or e4m3 after division by the tensor's dequantisation factor
+// (q_descale for the rotated queries, k_descale / v_descale for the cache).
+__device__ __forceinline__ void load8(const __nv_bfloat16* p, float (&x)[8]) {
+  const uint4 u = *reinterpret_cast<const uint4*>(p);
+  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
 #pragma unroll
   for (int e = 0; e < 4; ++e) {
-    const float2 x = __bfloat1622float2(l2[e]);
-    const float2 y = __bfloat1622float2(h2[e]);
-    const float c0 = c[2 * e], c1 = c[2 * e + 1], s0 = s[2 * e], s1 = s[2 * e + 1];
-    ol[e] = __floats2bfloat162_rn(x.x * c0 - y.x * s0, x.y * c1 - y.y * s1);
-    oh[e] = __floats2bfloat162_rn(y.x * c0 + x.x * s0, y.y * c1 + x.y * s1);
+    const float2 f = __bfloat1622float2(h[e]);
+    x[2 * e] = f.x;
+    x[2 * e + 1] = f.y;
+  }
+}
+__device__ __forceinline__ uint32_t e4m3x2(float lo, float hi) {
+  uint16_t r;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+// Eight values stored in the element type of the output: bf16 (descale
+// ignored) or e4m3 (x / descale, round to nearest, saturating).
+template <bool kE4M3>
+__device__ __forceinline__ void store8(void* base, int64_t elem, const float (&x)[8], float descale) {
+  if constexpr (kE4M3) {
+    uint2 u;
+    u.x = e4m3x2(x[0] / descale, x[1] / descale) | (e4m3x2(x[2] / descale, x[3] / descale) << 16);
+    u.y = e4m3x2(x[4] / descale, x[5] / descale) | (e4m3x2(x[6] / descale, x[7] / descale) << 16);
+    *reinterpret_cast<uint2*>(static_cast<uint8_t*>(base) + elem) = u;
+  } else {
+    uint4 u;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) h[e] = __floats2bfloat162_rn(x[2 * e], x[2 * e + 1]);
+    *reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(base) + elem) = u;
   }
 }
 
+template <bool kE4M3>
 __global__ void rope_cache_write_kernel(int batch, int l_new, int hq, int hkv, int d, int64_t cap, KvPages pages,
                                         const int32_t* __restrict__ c_snap, const __nv_bfloat16* __restrict__ q_new,
                                         const __nv_bfloat16* __restrict__ k_new,
                                         const __nv_bfloat16* __restrict__ v_new, const float* __restrict__ cos_t,
-                                        const float* __restrict__ sin_t, __nv_bfloat16* q_rot,
-                                        __nv_bfloat16* k_cache, __nv_bfloat16* v_cache, int32_t* snap_out) {
+                                        const float* __restrict__ sin_t, float q_descale, float k_descale,
+                                        float v_descale, void* q_rot, void* k_cache, void* v_cache,
+                                        int32_t* snap_out) {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   copy_snapshot(batch, c_snap, snap_out);
   const int half = d / 2;
@@ -428,34 +450,47 @@ __global__ void rope_cache_write_kernel(int batch, int l_new, int hq, int hkv, i
     const int64_t p = (int64_t)c_snap[b] + row % l_new;
     const int64_t dst_row = pages.table ? paged_row(pages, b, p) : (int64_t)b * cap + p;
     const __nv_bfloat16* src;
-    __nv_bfloat16* dst;
+    void* dst;
+    int64_t off;  // element offset of the head row in dst
+    float descale;
     if (head < hq) {
       src = q_new + (row * hq + head) * d;
-      dst = q_rot + (row * hq + head) * d;
+      dst = q_rot;
+      off = (row * hq + head) * d;
+      descale = q_descale;
     } else if (head < hq + hkv) {
       src = k_new + (row * hkv + (head - hq)) * d;
-      dst = k_cache + (dst_row * hkv + (head - hq)) * d;
+      dst = k_cache;
+      off = (dst_row * hkv + (head - hq)) * d;
+      descale = k_descale;
     } else {
       src = v_new + (row * hkv + (head - hq - hkv)) * d;
-      dst = v_cache + (dst_row * hkv + (head - hq - hkv)) * d;
-      *reinterpret_cast<uint4*>(dst + k0) = *reinterpret_cast<const uint4*>(src + k0);
-      *reinterpret_cast<uint4*>(dst + half + k0) = *reinterpret_cast<const uint4*>(src + half + k0);
+      off = (dst_row * hkv + (head - hq - hkv)) * d;
+      float lo[8], hi[8];
+      load8(src + k0, lo);
+      load8(src + half + k0, hi);
+      store8<kE4M3>(v_cache, off + k0, lo, v_descale);
+      store8<kE4M3>(v_cache, off + half + k0, hi, v_descale);
       continue;
     }
-    const uint4 lo = *reinterpret_cast<const uint4*>(src + k0);
-    const uint4 hi = *reinterpret_cast<const uint4*>(src + half + k0);
-    float c[8], s[8];
+    float lo[8], hi[8], c[8], s[8];
+    load8(src + k0, lo);
+    load8(src + half + k0, hi);
     const float4* cp = reinterpret_cast<const float4*>(cos_t + p * half + k0);
     const float4* sp = reinterpret_cast<const float4*>(sin_t + p * half + k0);
     const float4 c0 = __ldg(cp), c1 = __ldg(cp + 1), s0 = __ldg(sp), s1 = __ldg(sp + 1);
     c[0] = c0.x; c[1] = c0.y; c[2] = c0.z; c[3] = c0.w; c[4] = c1.x; c[5] = c1.y; c[6] = c1.z; c[7] = c1.w;
     s[0] = s0.x; s[1] = s0.y; s[2] = s0.z; s[3] = s0.w; s[4] = s1.x; s[5] = s1.y; s[6] = s1.z; s[7] = s1.w;
-    uint4 out_lo, out_hi;
-    rotate8(lo, hi, c, s, out_lo, out_hi);
-    *reinterpret_cast<uint4*>(dst + k0) = out_lo;
-    *reinterpret_cast<uint4*>(dst + half + k0) = out_hi;
+    float ol[8], oh[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      ol[e] = lo[e] * c[e] - hi[e] * s[e];
+      oh[e] = hi[e] * c[e] + lo[e] * s[e];
+    }
+    store8<kE4M3>(dst, off + k0, ol, descale);
+    store8<kE4M3>(dst, off + half + k0, oh, descale);
   }
-  zero_value_tail(batch, l_new, hkv * d / 8, cap, pages, c_snap, reinterpret_cast<uint4*>(v_cache));
+  zero_value_tail(batch, l_new, hkv * d * (kE4M3 ? 1 : 2) / 16, cap, pages, c_snap, reinterpret_cast<uint4*>(v_cache));
 }
 
 }  // namespace
@@ -541,21 +576,22 @@ cudaError_t launch_cache_write(int dtype, int batch, int l_new, int hkv, int d, 
   return cudaGetLastError();
 }
 
-cudaError_t launch_rope_cache_write(int batch, int l_new, int hq, int hkv, int d, int64_t cap,
+cudaError_t launch_rope_cache_write(int dtype, int batch, int l_new, int hq, int hkv, int d, int64_t cap,
                                    const KvPages& pages, const int32_t* c_snap, const void* q_new,
                                    const void* k_new, const void* v_new, const float* cos_t, const float* sin_t,
-                                   void* q_rot, void* k_cache, void* v_cache, cudaStream_t st,
-                                   int32_t* snap_out) {
+                                   float q_descale, float k_descale, float v_descale, void* q_rot, void* k_cache,
+                                   void* v_cache, cudaStream_t st, int32_t* snap_out) {
   int64_t total = (int64_t)batch * l_new * (hq + 2 * hkv) * (d / 16);
   if (total == 0) return cudaSuccess;
-  const int64_t tail = (int64_t)batch * 128 * (hkv * d / 8);  // value rows zeroed past the new end
+  const bool e4m3 = dtype == ISM_E4M3;
+  const int64_t tail = (int64_t)batch * 128 * (hkv * d * (e4m3 ? 1 : 2) / 16);  // value rows zeroed past the new end
   if (tail > total) total = tail;
   int grid = (int)((total + 255) / 256);
   if (grid > 152 * 16) grid = 152 * 16;
-  rope_cache_write_kernel<<<grid, 256, 0, st>>>(
-      batch, l_new, hq, hkv, d, cap, pages, c_snap, (const __nv_bfloat16*)q_new, (const __nv_bfloat16*)k_new,
-      (const __nv_bfloat16*)v_new, cos_t, sin_t, (__nv_bfloat16*)q_rot, (__nv_bfloat16*)k_cache,
-      (__nv_bfloat16*)v_cache, snap_out);
+  auto kern = e4m3 ? rope_cache_write_kernel<true> : rope_cache_write_kernel<false>;
+  kern<<<grid, 256, 0, st>>>(batch, l_new, hq, hkv, d, cap, pages, c_snap, (const __nv_bfloat16*)q_new,
+                             (const __nv_bfloat16*)k_new, (const __nv_bfloat16*)v_new, cos_t, sin_t, q_descale,
+                             k_descale, v_descale, q_rot, k_cache, v_cache, snap_out);
   return cudaGetLastError();
 }
 

@@ -108,6 +108,39 @@ __device__ __forceinline__ uint32_t pack_e4m3x4(float x0, float x1, float x2, fl
   return r;
 }
 
+// Gradient store of a rotary-encoded head row (the rotation of the one-pass
+// path pairs column k with k + 64): lo holds columns k0..k0+31 and hi columns
+// k0+64..k0+95 of the gradient of the ROTATED row (fp32 bit patterns); after
+// scaling by f, each pair (g_k, g_{k+64}) goes back through the transposed
+// rotation, x_k = g_k c + g_{k+64} s and x_{k+64} = g_{k+64} c - g_k s, with
+// c, s the cosines and sines of pairs k0.. of the row's position (cs, sn),
+// and the bf16 results are stored at dst_lo (columns k0..) and dst_hi
+// (columns k0+64..).
+__device__ __forceinline__ void rope_back_store32(const uint32_t (&lo)[32], const uint32_t (&hi)[32], float f,
+                                                  const float* __restrict__ cs, const float* __restrict__ sn,
+                                                  uint4* dst_lo, uint4* dst_hi) {
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float4 c0 = __ldg(reinterpret_cast<const float4*>(cs + 8 * i));
+    const float4 c1 = __ldg(reinterpret_cast<const float4*>(cs + 8 * i + 4));
+    const float4 s0 = __ldg(reinterpret_cast<const float4*>(sn + 8 * i));
+    const float4 s1 = __ldg(reinterpret_cast<const float4*>(sn + 8 * i + 4));
+    const float c[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
+    const float s[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
+    float xl[8], xh[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const float gl = __uint_as_float(lo[8 * i + e]) * f, gh = __uint_as_float(hi[8 * i + e]) * f;
+      xl[e] = gl * c[e] + gh * s[e];
+      xh[e] = gh * c[e] - gl * s[e];
+    }
+    dst_lo[i] = make_uint4(pack_bf16(xl[0], xl[1]), pack_bf16(xl[2], xl[3]), pack_bf16(xl[4], xl[5]),
+                           pack_bf16(xl[6], xl[7]));
+    dst_hi[i] = make_uint4(pack_bf16(xh[0], xh[1]), pack_bf16(xh[2], xh[3]), pack_bf16(xh[4], xh[5]),
+                           pack_bf16(xh[6], xh[7]));
+  }
+}
+
 // Byte offset of element (r, c) of a [128 x 128] bf16 tile in the layout a
 // 128B-swizzled TMA box of 64 columns x 128 rows produces (two such boxes,
 // one per 64-column half): 16-byte chunk index XOR (row mod 8).

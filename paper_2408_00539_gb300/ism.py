@@ -57,6 +57,8 @@ EXPORTS = {
     "ism_attn_bwd_workspace_size": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "ism_attn_bwd_workspace_size_min": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
     "ism_attn_bwd": (C.c_int, [C.c_void_p] * 12 + [C.c_size_t, C.c_void_p]),
+    "ism_attn_fwd_rope": (C.c_int, [C.c_void_p] * 11 + [C.c_size_t, C.c_void_p]),
+    "ism_attn_bwd_rope": (C.c_int, [C.c_void_p] * 13 + [C.c_size_t, C.c_void_p]),
     "ism_attn_prefill_append_workspace_size": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_void_p]),
     "ism_attn_prefill_append": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
                                           C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_int64,
@@ -76,6 +78,16 @@ EXPORTS = {
                                                C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_int64,
                                                C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                                C.c_void_p, C.c_size_t, C.c_void_p]),
+    "ism_attn_prefill_append_paged_rope": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
+                                                     C.c_int32, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p,
+                                                     C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p,
+                                                     C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                                     C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p]),
+    "ism_attn_prefill_append_e4m3_rope": (C.c_int, [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
+                                                    C.c_int32, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p,
+                                                    C.c_void_p, C.c_int64, C.c_void_p, C.c_void_p, C.c_float,
+                                                    C.c_float, C.c_float, C.c_void_p, C.c_void_p, C.c_void_p,
+                                                    C.c_void_p, C.c_size_t, C.c_void_p]),
     "ism_check_status": (C.c_int, [C.c_void_p]),
     "ism_debug_timeout_probe": (C.c_int, [C.c_uint32, C.c_void_p]),
     "ism_status_string": (C.c_char_p, [C.c_int]),
@@ -90,7 +102,7 @@ EXPORTS = {
     "ism_attn_fwd_noalloc": (C.c_int, [C.c_void_p] * 8),
 }
 
-KERNEL_FWD, KERNEL_BWD_DKDV, KERNEL_BWD_DQ, KERNEL_BWD_PRE, KERNEL_DECODE, KERNEL_META = 1, 2, 3, 4, 5, 6
+KERNEL_FWD, KERNEL_BWD_DKDV, KERNEL_BWD_DQ, KERNEL_BWD_PRE, KERNEL_DECODE, KERNEL_META, KERNEL_ROPE = 1, 2, 3, 4, 5, 6, 7
 
 _lib = None
 
@@ -262,6 +274,55 @@ def fwd_e4m3(segs: Segments, q, k, v, q_descale: float, k_descale: float, v_desc
                                  _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(), _stream(q.device)),
            "ism_attn_fwd_e4m3")
     return out, lse
+
+
+def fwd_rope(segs: Segments, q, k, v, rope_cos, rope_sin, softmax_scale: float, q_rot=None, k_rot=None, out=None,
+             lse=None, workspace=None):
+    """Forward with rotary encoding: q [T,Hq,D] and k [T,Hkv,D] (unrotated)
+    are rotated at their positions inside their sequences (tables rope_cos /
+    rope_sin float32 [rows, D/2]) into q_rot / k_rot, then attended.
+    Returns (o, lse, q_rot, k_rot); the backward takes q_rot and k_rot."""
+    lib = load()
+    _contig(q, k, v)
+    T, hq, D = q.shape
+    s, sh = segs.struct(), _shape(q, k, softmax_scale)
+    rope = _rope_struct(rope_cos, rope_sin)
+    nbytes = C.c_size_t()
+    _check(lib.ism_attn_fwd_workspace_size(C.byref(s), C.byref(sh), C.byref(nbytes)), "ism_attn_fwd_workspace_size")
+    q_rot = torch.empty_like(q) if q_rot is None else q_rot
+    k_rot = torch.empty_like(k) if k_rot is None else k_rot
+    out = torch.empty_like(q) if out is None else out
+    lse = torch.empty((hq, T), dtype=torch.float32, device=q.device) if lse is None else lse
+    if workspace is None or workspace.numel() < nbytes.value:
+        workspace = _workspace(nbytes.value, q.device)
+    _check(lib.ism_attn_fwd_rope(C.byref(s), C.byref(sh), _ptr(q), _ptr(k), _ptr(v), C.byref(rope), _ptr(q_rot),
+                                 _ptr(k_rot), _ptr(out), _ptr(lse), _ptr(workspace), workspace.numel(),
+                                 _stream(q.device)), "ism_attn_fwd_rope")
+    return out, lse, q_rot, k_rot
+
+
+def bwd_rope(segs: Segments, q_rot, k_rot, v, o, lse, dout, rope_cos, rope_sin, softmax_scale: float, dq=None,
+             dk=None, dv=None, workspace=None, minimal_workspace: bool = False):
+    """Backward of ``fwd_rope``: takes the rotated q_rot / k_rot the forward
+    wrote and returns (dq, dk, dv) with dq, dk the gradients of the UNROTATED
+    queries and keys.  Workspace as for ``bwd``."""
+    lib = load()
+    _contig(q_rot, k_rot, v, o, lse, dout)
+    s, sh = segs.struct(), _shape(q_rot, k_rot, softmax_scale)
+    rope = _rope_struct(rope_cos, rope_sin)
+    full, low = C.c_size_t(), C.c_size_t()
+    _check(lib.ism_attn_bwd_workspace_size(C.byref(s), C.byref(sh), C.byref(full)), "ism_attn_bwd_workspace_size")
+    _check(lib.ism_attn_bwd_workspace_size_min(C.byref(s), C.byref(sh), C.byref(low)),
+           "ism_attn_bwd_workspace_size_min")
+    dq = torch.empty_like(q_rot) if dq is None else dq
+    dk = torch.empty_like(k_rot) if dk is None else dk
+    dv = torch.empty_like(v) if dv is None else dv
+    if workspace is None or workspace.numel() < low.value:
+        workspace = _workspace(low.value if minimal_workspace else full.value, q_rot.device)
+    _check(lib.ism_attn_bwd_rope(C.byref(s), C.byref(sh), _ptr(q_rot), _ptr(k_rot), _ptr(v), _ptr(o), _ptr(lse),
+                                 _ptr(dout), C.byref(rope), _ptr(dq), _ptr(dk), _ptr(dv), _ptr(workspace),
+                                 workspace.numel(), _stream(q_rot.device)), "ism_attn_bwd_rope")
+    return dq, dk, dv
 
 
 def bwd_workspace_size(segs: Segments, q, k, softmax_scale: float, minimal: bool = False) -> int:
@@ -492,6 +553,72 @@ def prefill_append_paged(q_new, k_new, v_new, k_pool, v_pool, page_size: int, bl
                                              _ptr(cache_len), C.c_void_p(ch.ctypes.data), _ptr(out), _ptr(lse),
                                              _ptr(workspace), workspace.numel(), _stream(q_new.device)),
            "ism_attn_prefill_append_paged")
+    return out, lse
+
+
+def prefill_append_paged_rope(q_new, k_new, v_new, k_pool, v_pool, page_size: int, block_table, block_table_host,
+                              cache_len, cache_len_host, new_seg_end, new_seg_type, rope_cos, rope_sin,
+                              softmax_scale: float, out=None, lse=None, workspace=None):
+    """``prefill_append_paged`` with rotary encoding of the new queries and
+    keys at positions cache_len[b] + j (as ``prefill_append_rope``)."""
+    lib = load()
+    _contig(q_new, k_new, v_new, k_pool, v_pool, cache_len, block_table)
+    B, Ln, hq, D = q_new.shape
+    rows = k_pool.shape[0]
+    if rows % page_size:
+        raise ValueError("pool rows must be a whole number of pages")
+    sh = _shape(q_new, k_new, softmax_scale)
+    se = np.ascontiguousarray(new_seg_end, dtype=np.int32)
+    st = np.ascontiguousarray(new_seg_type, dtype=np.uint8)
+    ch = np.ascontiguousarray(cache_len_host, dtype=np.int32)
+    bt = np.ascontiguousarray(block_table_host, dtype=np.int32)
+    rope = _rope_struct(rope_cos, rope_sin)
+    out = torch.empty_like(q_new) if out is None else out
+    lse = torch.empty((hq, B, Ln), dtype=torch.float32, device=q_new.device) if lse is None else lse
+    if workspace is None:
+        workspace = _workspace(append_workspace_size(q_new, k_new, softmax_scale, rope=True), q_new.device)
+    _check(lib.ism_attn_prefill_append_paged_rope(C.byref(sh), B, _ptr(q_new), _ptr(k_new), _ptr(v_new), Ln,
+                                                  C.c_void_p(se.ctypes.data), C.c_void_p(st.ctypes.data),
+                                                  se.shape[0], _ptr(k_pool), _ptr(v_pool), rows // page_size,
+                                                  page_size, _ptr(block_table), C.c_void_p(bt.ctypes.data),
+                                                  block_table.shape[1], _ptr(cache_len), C.c_void_p(ch.ctypes.data),
+                                                  C.byref(rope), _ptr(out), _ptr(lse), _ptr(workspace),
+                                                  workspace.numel(), _stream(q_new.device)),
+           "ism_attn_prefill_append_paged_rope")
+    return out, lse
+
+
+def prefill_append_e4m3_rope(q_new, k_new, v_new, k_cache, v_cache, cache_len, cache_len_host, new_seg_end,
+                             new_seg_type, q_descale: float, k_descale: float, v_descale: float, rope_cos, rope_sin,
+                             softmax_scale: float, out=None, lse=None, workspace=None):
+    """Rotary append against e4m3 caches: q_new, k_new, v_new are bf16 and
+    unrotated; queries and keys are rotated at positions cache_len[b] + j,
+    then quantised with the factors (keys and values into the caches).
+    Returns (o bf16, lse [Hq,B,Ln])."""
+    lib = load()
+    _contig(q_new, k_new, v_new, k_cache, v_cache, cache_len)
+    B, Ln, hq, D = q_new.shape
+    sh = _Shape()
+    sh.num_heads_q, sh.num_heads_kv, sh.head_dim = hq, k_new.shape[2], D
+    sh.dtype, sh.softmax_scale = ISM_E4M3, float(softmax_scale)
+    se = np.ascontiguousarray(new_seg_end, dtype=np.int32)
+    st = np.ascontiguousarray(new_seg_type, dtype=np.uint8)
+    ch = np.ascontiguousarray(cache_len_host, dtype=np.int32)
+    rope = _rope_struct(rope_cos, rope_sin)
+    out = torch.empty(q_new.shape, dtype=torch.bfloat16, device=q_new.device) if out is None else out
+    lse = torch.empty((hq, B, Ln), dtype=torch.float32, device=q_new.device) if lse is None else lse
+    if workspace is None:
+        nbytes = C.c_size_t()
+        _check(lib.ism_attn_prefill_append_rope_workspace_size(C.byref(sh), B, Ln, C.byref(nbytes)),
+               "ism_attn_prefill_append_rope_workspace_size")
+        workspace = _workspace(nbytes.value, q_new.device)
+    _check(lib.ism_attn_prefill_append_e4m3_rope(C.byref(sh), B, _ptr(q_new), _ptr(k_new), _ptr(v_new), Ln,
+                                                 C.c_void_p(se.ctypes.data), C.c_void_p(st.ctypes.data), se.shape[0],
+                                                 _ptr(k_cache), _ptr(v_cache), k_cache.shape[1], _ptr(cache_len),
+                                                 C.c_void_p(ch.ctypes.data), q_descale, k_descale, v_descale,
+                                                 C.byref(rope), _ptr(out), _ptr(lse), _ptr(workspace),
+                                                 workspace.numel(), _stream(q_new.device)),
+           "ism_attn_prefill_append_e4m3_rope")
     return out, lse
 
 

@@ -482,3 +482,113 @@ def test_workload_generator_shapes():
     assert t.segs.seg_end.tolist() == [40, 70, 100, 160, 210, 256]
     assert wl.gqa_8k().segs.cu_seqlens.tolist() == [0, 8192, 16384]
     assert wl.packed_32k().total_tokens == 32768
+
+
+# ---------------------------------------------------------------- rotary encoding, one pass
+
+def _mask_sdpa_torch(q, k, v, segs, scale):
+    """Masked attention of a packed batch in plain torch fp64 ([T, H, D]
+    tensors; the masks from the prose construction), for autograd."""
+    outs = []
+    grp = q.shape[1] // k.shape[1]
+    for b in range(segs.num_seqs):
+        t0, L, se, st = segs.seq(b)
+        sl = slice(t0, t0 + L)
+        o = torch.nn.functional.scaled_dot_product_attention(
+            q[sl].permute(1, 0, 2), k[sl].permute(1, 0, 2).repeat_interleave(grp, 0),
+            v[sl].permute(1, 0, 2).repeat_interleave(grp, 0),
+            attn_mask=torch.from_numpy(orc.mask_from_prose(se, st)), scale=scale)
+        outs.append(o.permute(1, 0, 2))
+    return torch.cat(outs, 0)
+
+
+def _torch_complex_rotate(x, ang):
+    half = x.shape[-1] // 2
+    z = torch.complex(x[..., :half], x[..., half:]) * torch.polar(torch.ones_like(ang), ang)
+    return torch.cat([z.real, z.imag], -1)
+
+
+def test_seq_positions_restart_per_sequence():
+    segs = wl.pack([([3, 5], [0, 1]), ([1], [1]), ([4], [0])])
+    assert orc.seq_positions(segs).tolist() == [0, 1, 2, 3, 4, 0, 0, 1, 2, 3]
+
+
+def test_rope_fwd_bwd_vs_library_autograd_through_complex_rotation():
+    # independent construction: rotation as complex multiplication in torch,
+    # masked SDPA, autograd for the gradients of the unrotated inputs
+    rng = np.random.Generator(np.random.PCG64(54))
+    segs = wl.random_dialogue_set(rng, 3, 60, min_len=3)
+    T, hq, hkv, D = segs.total_tokens, 4, 2, 8
+    q, k, v, do = _rand(rng, T, hq, D), _rand(rng, T, hkv, D), _rand(rng, T, hkv, D), _rand(rng, T, hq, D)
+    ang = rng.uniform(-6.0, 6.0, size=(70, D // 2))
+    scale = 0.45
+    o, lse, q_rot, k_rot = orc.attn_fwd_rope(q, k, v, segs, scale, np.cos(ang), np.sin(ang))
+    dq, dk, dv = orc.attn_bwd_rope(q, k, v, do, segs, scale, np.cos(ang), np.sin(ang))
+    pos = np.concatenate([np.arange(segs.seq(b)[1]) for b in range(segs.num_seqs)])
+    a = torch.from_numpy(ang[pos])[:, None, :]
+    qt, kt, vt = (torch.from_numpy(x).requires_grad_() for x in (q, k, v))
+    ot = _mask_sdpa_torch(_torch_complex_rotate(qt, a), _torch_complex_rotate(kt, a), vt, segs, scale)
+    ot.backward(torch.from_numpy(do))
+    np.testing.assert_allclose(o, ot.detach().numpy(), rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(q_rot, _complex_rotate(q, ang[pos][:, None, :]), rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(dq, qt.grad.numpy(), rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(dk, kt.grad.numpy(), rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(dv, vt.grad.numpy(), rtol=1e-10, atol=1e-12)
+
+
+def test_rope_bwd_vs_finite_differences():
+    rng = np.random.Generator(np.random.PCG64(55))
+    segs = wl.pack([([3, 6, 9], [0, 1, 0]), ([2, 7], [1, 0])])
+    T = segs.total_tokens
+    q, k, v, do = _rand(rng, T, 2, 4), _rand(rng, T, 1, 4), _rand(rng, T, 1, 4), _rand(rng, T, 2, 4)
+    ang = rng.uniform(-4.0, 4.0, size=(12, 2))
+    c, s = np.cos(ang), np.sin(ang)
+    scale = 0.8
+    dq, dk, dv = orc.attn_bwd_rope(q, k, v, do, segs, scale, c, s)
+
+    def loss(q_, k_, v_):
+        return float((orc.attn_fwd_rope(q_, k_, v_, segs, scale, c, s)[0] * do).sum())
+
+    eps = 1e-6
+    for i, (x, g) in enumerate(((q, dq), (k, dk), (v, dv))):
+        num = np.zeros_like(x)
+        for idx in np.ndindex(*x.shape):
+            args_p, args_m = [q, k, v], [q, k, v]
+            xp, xm = x.copy(), x.copy()
+            xp[idx] += eps
+            xm[idx] -= eps
+            args_p[i], args_m[i] = xp, xm
+            num[idx] = (loss(*args_p) - loss(*args_m)) / (2 * eps)
+        np.testing.assert_allclose(g, num, rtol=1e-6, atol=1e-8)
+
+
+def test_rope_with_zero_angles_is_plain_attention():
+    rng = np.random.Generator(np.random.PCG64(56))
+    segs = wl.pack([([5, 9, 14], [0, 1, 0]), ([6], [1])])
+    T = segs.total_tokens
+    q, k, v, do = _rand(rng, T, 4, 6), _rand(rng, T, 2, 6), _rand(rng, T, 2, 6), _rand(rng, T, 4, 6)
+    c, s = np.ones((20, 3)), np.zeros((20, 3))
+    o, lse, _, _ = orc.attn_fwd_rope(q, k, v, segs, 0.3, c, s)
+    o0, lse0 = orc.attn_fwd(q, k, v, segs, 0.3)
+    np.testing.assert_array_equal(o, o0)
+    np.testing.assert_array_equal(lse, lse0)
+    for g, g0 in zip(orc.attn_bwd_rope(q, k, v, do, segs, 0.3, c, s), orc.attn_bwd(q, k, v, do, segs, 0.3)):
+        np.testing.assert_array_equal(g, g0)
+
+
+def test_rope_output_invariant_to_a_common_position_shift():
+    # scores depend only on relative positions, so shifting every position of
+    # a sequence by the same amount leaves O and LSE unchanged (tables of the
+    # usual schedule, fp64 angles)
+    rng = np.random.Generator(np.random.PCG64(57))
+    segs = wl.pack([([4, 10, 13, 20], [0, 1, 0, 1])])
+    T, D = segs.total_tokens, 8
+    q, k, v = _rand(rng, T, 2, D), _rand(rng, T, 1, D), _rand(rng, T, 1, D)
+    inv = 10000.0 ** (-2.0 * np.arange(D // 2) / D)
+    for shift in (0, 37, 500):
+        ang = (np.arange(T + shift, dtype=np.float64)[:, None] * inv[None, :])[shift:]
+        o, lse, _, _ = orc.attn_fwd_rope(q, k, v, segs, 0.5, np.cos(ang), np.sin(ang))
+        if shift == 0:
+            o_ref, lse_ref = o, lse
+        np.testing.assert_allclose(o, o_ref, rtol=1e-9, atol=1e-11)
+        np.testing.assert_allclose(lse, lse_ref, rtol=1e-9, atol=1e-11)
