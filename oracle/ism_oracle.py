@@ -19,7 +19,11 @@ Everything here is the plain definition, written out slowly:
 * the standard softmax-attention gradients;
 * the KV-cache append of Section 2.3: cached keys/values of the history are
   reused, the new turn is computed and the two are concatenated;
-* the tile map (empty / full / partial) by brute force over the mask.
+* the tile map (empty / full / partial) by brute force over the mask;
+* rotary position encoding (outside the paper's operation, which leaves
+  positional encoding out): the rotation itself, the rotary append, and the
+  one-pass forward / backward with queries and keys rotated at their
+  positions inside their sequences.
 
 All arithmetic is float64 on the exact input values (bf16/fp32 inputs are
 upcast exactly).  Every function is pinned by ``tests/test_oracle.py``.
