@@ -308,6 +308,17 @@ def run_cuda(args, w):
         ism.fwd(segs, qd, kd, vd, w.softmax_scale, out=o, lse=lse)
         ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws_b)
 
+    if args.profile_step and args.rope:
+        # the rotary step (usual schedule) for a profiler: same tensors, rotated copies
+        cos_np, sin_np = wl.rope_tables(int(np.diff(w.segs.cu_seqlens).max()), D)
+        cos_t, sin_t = torch.from_numpy(cos_np).to(dev), torch.from_numpy(sin_np).to(dev)
+        q_rot, k_rot = torch.empty_like(qd), torch.empty_like(kd)
+
+        def step():  # noqa: F811
+            ism.fwd_rope(segs, qd, kd, vd, cos_t, sin_t, w.softmax_scale, q_rot=q_rot, k_rot=k_rot, out=o, lse=lse)
+            ism.bwd_rope(segs, q_rot, k_rot, vd, o, lse, dod, cos_t, sin_t, w.softmax_scale, dq=dq, dk=dk, dv=dv,
+                         workspace=ws_b)
+
     # clocks are sampled from the warm-up on (nvidia-smi needs a moment to start)
     clocks = ClockSampler(dev.index) if not args.profile_step else None
     if clocks is not None:
@@ -1095,8 +1106,9 @@ def profile_decode(dtype: str, steps: int):
 
 
 WORKLOADS = {"gqa_8k": wl.gqa_8k, "mha_4k": wl.mha_4k, "packed_32k": wl.packed_32k,
-             # one 4K dialogue of the same recipe: small enough for full ncu captures
-             "gqa_4k_b1": lambda: wl.gqa_8k(batch=1, seqlen=4096)}
+             # one 4K dialogue of the same recipes: small enough for full ncu captures
+             "gqa_4k_b1": lambda: wl.gqa_8k(batch=1, seqlen=4096),
+             "mha_4k_b1": lambda: wl.mha_4k(batch=1)}
 
 
 def main():
@@ -1112,6 +1124,7 @@ def main():
                     help="skip the sustained run, the minimum-workspace backward and the other training configs")
     ap.add_argument("--profile-step", action="store_true",
                     help="run the warm-up steps and one more step, print nothing (for ncu)")
+    ap.add_argument("--rope", action="store_true", help="with --profile-step: the rotary forward and backward")
     ap.add_argument("--profile-decode", choices=["bf16", "e4m3"],
                     help="run only warm-up + steps single-token steps on the 8 x 16K cache, print nothing (for ncu)")
     args = ap.parse_args()

@@ -96,8 +96,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = align1024(smem_raw);
   Bars* bar = reinterpret_cast<Bars*>(smem + OFF_BAR);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int h = blockIdx.x % a.hq;
-  const Tile w = a.qtiles[a.q_order[blockIdx.x / a.hq]];
+  int64_t tpos;
+  int h;
+  bucket_item(blockIdx.x, a.nq, a.hq, tpos, h, a.hq == a.hkv);  // blocks start roughly in index order
+  const Tile w = a.qtiles[a.q_order[tpos]];
   const int g = h / (a.hq / a.hkv);
   const int nkb = w.a1, kfull = w.a0;
 
@@ -335,8 +337,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (valid && a.rope_cos) {
         const int64_t pos = (int64_t)w.tile * kRows + r;
         uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) + grow * a.hq * kD + h * kD);
-        rope_back_store32(q0, q1, a.scale, a.rope_cos + pos * 64 + wg * 32, a.rope_sin + pos * 64 + wg * 32,
-                          dst + 4 * wg, dst + 8 + 4 * wg);
+        float rc[32], rs[32];
+        rope_row32(a.rope_cos + pos * 64 + wg * 32, a.rope_sin + pos * 64 + wg * 32, rc, rs);
+        rope_back_store32(q0, q1, a.scale, rc, rs, dst + 4 * wg, dst + 8 + 4 * wg);
       } else if (valid) {
         uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) + grow * a.hq * kD + h * kD +
                                               wg * 64);
@@ -456,8 +459,9 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
     Tile w;
   };
   auto decode = [&](int item, Item& x) {
-    x.g = item % a.hkv;
-    x.gk = a.k_order[item / a.hkv];
+    int64_t kpos;
+    bucket_item(item, a.nk, a.hkv, kpos, x.g);
+    x.gk = a.k_order[kpos];
     x.w = a.ktiles[x.gk];
     x.c = x.w.tile;
     x.qt0 = x.w.a0;
@@ -883,10 +887,12 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
           ptx::tmem_ld_wait();
           ptx::reg_fence(lo);
           ptx::reg_fence(hi);
-          if (kvalid)
-            rope_back_store32(lo, hi, f, a.rope_cos + (int64_t)key * 64 + 32 * q2,
-                              a.rope_sin + (int64_t)key * 64 + 32 * q2, reinterpret_cast<uint4*>(outp + q2 * 32),
+          if (kvalid) {
+            float rc[32], rs[32];
+            rope_row32(a.rope_cos + (int64_t)key * 64 + 32 * q2, a.rope_sin + (int64_t)key * 64 + 32 * q2, rc, rs);
+            rope_back_store32(lo, hi, f, rc, rs, reinterpret_cast<uint4*>(outp + q2 * 32),
                               reinterpret_cast<uint4*>(outp + 64 + q2 * 32));
+          }
         }
         ptx::tc_fence_before();
         continue;

@@ -74,14 +74,17 @@ __device__ __forceinline__ void set_abort(int32_t* f) { *reinterpret_cast<volati
 struct DecItem {
   int b, g, split, k0, k1, nt;
 };
-// item = (split * hkv + g) * batch + b: consecutive CTAs take the same split
-// of different sequences
+// item = (split * batch + b) * hkv + g: consecutive CTAs take the KV heads of
+// one (sequence, split), whose rows lie side by side in the cache
+// ([B, cap, Hkv, D]): CTAs that start together read neighbouring pieces of
+// the same cache rows, which keeps DRAM pages open across their requests
+// (an e4m3 head row is only 128 bytes of a 1 KB cache row)
 __device__ __forceinline__ DecItem dec_item(const DecodeArgs& a, int64_t item) {
   DecItem x;
-  x.b = (int)(item % a.batch);
-  const int64_t rest = item / a.batch;
-  x.g = (int)(rest % a.hkv);
-  x.split = (int)(rest / a.hkv);
+  x.g = (int)(item % a.hkv);
+  const int64_t rest = item / a.hkv;
+  x.b = (int)(rest % a.batch);
+  x.split = (int)(rest / a.batch);
   const int kv_len = a.c_snap[x.b] + 1;
   x.k0 = x.split * a.chunk;
   x.k1 = min(kv_len, x.k0 + a.chunk);

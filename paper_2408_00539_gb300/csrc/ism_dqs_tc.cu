@@ -47,8 +47,9 @@ struct Item {
 };
 __device__ __forceinline__ Item decode(const AttnArgs& a, int64_t item) {
   Item it;
-  it.h = (int)(item % a.hq);
-  const int gq = a.q_order[item / a.hq];
+  int64_t tpos;
+  bucket_item(item, a.nq, a.hq, tpos, it.h, a.hq == a.hkv);  // bucketed only when no two heads share K
+  const int gq = a.q_order[tpos];
   it.w = a.qtiles[gq];
   it.g = it.h / (a.hq / a.hkv);
   it.nkb = it.w.a1;
@@ -164,6 +165,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t b = local & 1, acc = tmem + lane_addr + 128u * b;
       const int row = x.t * kRows + r;
       const bool valid = row < x.w.q_len;
+      // rotary encoding: the cosines and sines of the row's first 32 pairs,
+      // loaded while the accumulator is still being computed
+      float rc[32], rs[32];
+      if (a.rope_cos && valid) rope_row32(a.rope_cos + (int64_t)row * 64, a.rope_sin + (int64_t)row * 64, rc, rs);
       if (!wait(&bar->acc_full[b], (local >> 1) & 1, a.status) || aborted(&bar->abort)) {
         set_abort(&bar->abort);
         break;
@@ -186,9 +191,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int k = 0; k < 32; ++k) lo[k] = hi[k] = 0u;
           }
-          if (valid)
-            rope_back_store32(lo, hi, a.scale, a.rope_cos + (int64_t)row * 64 + 32 * q2,
-                              a.rope_sin + (int64_t)row * 64 + 32 * q2, dst + 4 * q2, dst + 8 + 4 * q2);
+          if (valid) {
+            if (q2 == 1) rope_row32(a.rope_cos + (int64_t)row * 64 + 32, a.rope_sin + (int64_t)row * 64 + 32, rc, rs);
+            rope_back_store32(lo, hi, a.scale, rc, rs, dst + 4 * q2, dst + 8 + 4 * q2);
+          }
         }
         ptx::tc_fence_before();
         ptx::mbar_arrive(&bar->acc_empty[b]);

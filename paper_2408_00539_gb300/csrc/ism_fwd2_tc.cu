@@ -72,8 +72,10 @@ __device__ __forceinline__ Unit decode_unit(const AttnArgs& a, int64_t u) {
       x.half = (int)((item - a.split_whole) & 1);
       item = a.split_whole + x.split_k;
     }
-    const int hp = (int)(item % npairs);
-    x.w0 = x.w1 = a.qtiles[a.q_order[item / npairs]];
+    int64_t tpos;
+    int hp;
+    bucket_item(item, a.nq, npairs, tpos, hp, false);  // head pairs of a tile share K / V
+    x.w0 = x.w1 = a.qtiles[a.q_order[tpos]];
     x.h0 = 2 * hp;
     x.h1 = x.h0 + 1;
     x.nkb0 = x.nkb1 = x.w0.a1;
@@ -83,8 +85,10 @@ __device__ __forceinline__ Unit decode_unit(const AttnArgs& a, int64_t u) {
       x.nkb0 = x.nkb1 = x.half ? x.w0.a1 - mid : mid;
     }
   } else {
-    x.h0 = x.h1 = (int)(u % a.hq);
-    const int gq = a.pair_order[u / a.hq];
+    int64_t ppos;
+    bucket_item(u, a.npairs, a.hq, ppos, x.h0, a.hq == a.hkv);  // one query head per KV head: bucketed
+    x.h1 = x.h0;
+    const int gq = a.pair_order[ppos];
     x.w0 = a.qtiles[gq];
     bool second = false;
     if (gq + 1 < a.nq) {
@@ -527,8 +531,11 @@ __global__ void __launch_bounds__(128) fwd_split_merge_kernel(const AttnArgs a) 
   const int64_t k = b / (2 * kRows);
   const int npairs = a.hq >> 1;
   const int64_t item = a.split_whole + k;
-  const Tile w = a.qtiles[a.q_order[item / npairs]];
-  const int h = 2 * (int)(item % npairs) + x;
+  int64_t tpos;
+  int hp;
+  bucket_item(item, a.nq, npairs, tpos, hp, false);  // as fwd_pair_kernel decodes its items
+  const Tile w = a.qtiles[a.q_order[tpos]];
+  const int h = 2 * hp + x;
   const int row = w.tile * kRows + r;
   if (row >= w.q_len) return;
   const int d = threadIdx.x;

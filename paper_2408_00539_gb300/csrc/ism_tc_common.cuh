@@ -109,36 +109,71 @@ __device__ __forceinline__ uint32_t pack_e4m3x4(float x0, float x1, float x2, fl
 }
 
 // Gradient store of a rotary-encoded head row (the rotation of the one-pass
-// path pairs column k with k + 64): lo holds columns k0..k0+31 and hi columns
-// k0+64..k0+95 of the gradient of the ROTATED row (fp32 bit patterns); after
-// scaling by f, each pair (g_k, g_{k+64}) goes back through the transposed
-// rotation, x_k = g_k c + g_{k+64} s and x_{k+64} = g_{k+64} c - g_k s, with
-// c, s the cosines and sines of pairs k0.. of the row's position (cs, sn),
-// and the bf16 results are stored at dst_lo (columns k0..) and dst_hi
-// (columns k0+64..).
+// path pairs column k with k + 64).  rope_row32 loads the cosines and sines
+// of 32 pairs of a row's position (all loads issued before any use, so their
+// latency is paid once).  rope_back_store32: lo holds columns k0..k0+31 and
+// hi columns k0+64..k0+95 of the gradient of the ROTATED row (fp32 bit
+// patterns); after scaling by f, each pair (g_k, g_{k+64}) goes back through
+// the transposed rotation, x_k = g_k c + g_{k+64} s and
+// x_{k+64} = g_{k+64} c - g_k s, and the bf16 results are stored at dst_lo
+// (columns k0..) and dst_hi (columns k0+64..).
+__device__ __forceinline__ void rope_row32(const float* __restrict__ cs, const float* __restrict__ sn,
+                                           float (&c)[32], float (&s)[32]) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float4 cv = __ldg(reinterpret_cast<const float4*>(cs) + i);
+    const float4 sv = __ldg(reinterpret_cast<const float4*>(sn) + i);
+    c[4 * i] = cv.x; c[4 * i + 1] = cv.y; c[4 * i + 2] = cv.z; c[4 * i + 3] = cv.w;
+    s[4 * i] = sv.x; s[4 * i + 1] = sv.y; s[4 * i + 2] = sv.z; s[4 * i + 3] = sv.w;
+  }
+}
 __device__ __forceinline__ void rope_back_store32(const uint32_t (&lo)[32], const uint32_t (&hi)[32], float f,
-                                                  const float* __restrict__ cs, const float* __restrict__ sn,
-                                                  uint4* dst_lo, uint4* dst_hi) {
+                                                  const float (&c)[32], const float (&s)[32], uint4* dst_lo,
+                                                  uint4* dst_hi) {
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const float4 c0 = __ldg(reinterpret_cast<const float4*>(cs + 8 * i));
-    const float4 c1 = __ldg(reinterpret_cast<const float4*>(cs + 8 * i + 4));
-    const float4 s0 = __ldg(reinterpret_cast<const float4*>(sn + 8 * i));
-    const float4 s1 = __ldg(reinterpret_cast<const float4*>(sn + 8 * i + 4));
-    const float c[8] = {c0.x, c0.y, c0.z, c0.w, c1.x, c1.y, c1.z, c1.w};
-    const float s[8] = {s0.x, s0.y, s0.z, s0.w, s1.x, s1.y, s1.z, s1.w};
     float xl[8], xh[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-      const float gl = __uint_as_float(lo[8 * i + e]) * f, gh = __uint_as_float(hi[8 * i + e]) * f;
-      xl[e] = gl * c[e] + gh * s[e];
-      xh[e] = gh * c[e] - gl * s[e];
+      const int k = 8 * i + e;
+      const float gl = __uint_as_float(lo[k]) * f, gh = __uint_as_float(hi[k]) * f;
+      xl[e] = gl * c[k] + gh * s[k];
+      xh[e] = gh * c[k] - gl * s[k];
     }
     dst_lo[i] = make_uint4(pack_bf16(xl[0], xl[1]), pack_bf16(xl[2], xl[3]), pack_bf16(xl[4], xl[5]),
                            pack_bf16(xl[6], xl[7]));
     dst_hi[i] = make_uint4(pack_bf16(xh[0], xh[1]), pack_bf16(xh[2], xh[3]), pack_bf16(xh[4], xh[5]),
                            pack_bf16(xh[6], xh[7]));
   }
+}
+
+// Work item i of a list of n_tiles x n_heads items whose tiles come in cost
+// order (most expensive first).  The tiles are taken in four buckets of a
+// quarter of the list each, and inside a bucket head by head: the CTAs that
+// run at the same time then work on one head of neighbouring tiles, which
+// stream the same operand tiles (K / V in the forward, Q / dO in dK/dV) in
+// the same order, so those reads mostly hit L2.  Taking the heads of a tile
+// one after the other instead spreads the CTAs over all heads, which with
+// one query head per KV head leaves almost no operand tile shared.
+// With bucketed == false the order is the plain one (the heads of a tile
+// one after the other), which keeps the cost order exact: the statically
+// scheduled kernels take it whenever the heads of a tile already share
+// operands (two or more query heads per KV head).
+__device__ __forceinline__ void bucket_item(int64_t i, int64_t n_tiles, int n_heads, int64_t& tile_pos, int& head,
+                                            bool bucketed = true) {
+  if (!bucketed) {
+    tile_pos = i / n_heads;
+    head = (int)(i % n_heads);
+    return;
+  }
+  const int64_t bt = (n_tiles + 3) / 4;
+  const int64_t per_bucket = bt * n_heads;
+  const int64_t b = i / per_bucket;
+  const int64_t w = i - b * per_bucket;
+  const int64_t t0 = b * bt;
+  const int64_t nb = n_tiles - t0 < bt ? n_tiles - t0 : bt;
+  head = (int)(w / nb);
+  tile_pos = t0 + w % nb;
 }
 
 // Byte offset of element (r, c) of a [128 x 128] bf16 tile in the layout a
