@@ -80,9 +80,11 @@ typedef struct {
 } ism_segments_t;
 
 /* Heads and element type.  Supported: head_dim 64 or 128; Hq % Hkv == 0;
- * ISM_BF16 (fp32 accumulation, tensor cores) or ISM_FP32 (fp32 CUDA-core
- * path); ISM_E4M3 (fp8 inputs, head_dim 128) only for ism_attn_fwd_e4m3 and
- * its workspace query.  softmax_scale multiplies q.k before the softmax (the paper omits
+ * ISM_BF16 (fp32 accumulation) or ISM_FP32 (fp32 CUDA-core path); ISM_E4M3
+ * (fp8 inputs, head_dim 128) only for the e4m3 entry points and their
+ * workspace queries.  The tensor-core kernels serve bf16 and e4m3 at
+ * head_dim 128; bf16 at head_dim 64 runs the CUDA-core kernels (correct, but
+ * far from the tensor-core rate), as does fp32.  softmax_scale multiplies q.k before the softmax (the paper omits
  * the factor, Section 2.1; 1/sqrt(head_dim) is the usual choice). */
 typedef struct {
   int32_t num_heads_q;

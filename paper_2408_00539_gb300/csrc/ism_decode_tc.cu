@@ -23,8 +23,13 @@
 // warp 4: TMA loads (Q of the item, then its K tiles, then its V tiles,
 // through one ring); warp 5: MMA issue.
 // e4m3 caches (kE4M3): Q, K, V, P in e4m3 (kind::f8f6f4 MMAs, K = 32 a step,
-// 128-byte rows: one swizzled box a tile), scores scaled by qk_descale, O by
-// v_descale; tiles are half the size, so the ring has twice the stages.
+// 128-byte rows: one swizzled box per 128 keys), scores scaled by qk_descale,
+// O by v_descale.  A ring tile holds 256 keys (two 128-key boxes, 32 KB, the
+// size of a bf16 tile): each hand-off between the loads, the MMAs and the
+// softmax warps then covers as many bytes as in bf16.  With 128-key e4m3
+// tiles the per-tile chain, not DRAM, set the pace (0.77 of the copy
+// bandwidth, the same with a deeper ring).  The last tile of an item may hold
+// one 128-key half only; the other half is neither loaded nor multiplied.
 #include "ism_tc_common.cuh"
 
 namespace ism {
@@ -43,8 +48,10 @@ static_assert(TM_S + kHeadsPad * kMaxTiles <= kTmemCols, "S tiles fit in tensor 
 // Shared-memory plan: ring of K / V tiles, two P operands, two Q tiles, barriers.
 template <bool kE4M3>
 struct DecCfg {
-  static constexpr int kStages = kE4M3 ? 8 : 4;
-  static constexpr uint32_t kTile = kE4M3 ? kHalfBytes : kTileBytes;  // 128 keys x 128 dims
+  static constexpr int kStages = 4;
+  static constexpr int kSub = kE4M3 ? 2 : 1;          // 128-key sub-tiles of a ring tile
+  static constexpr uint32_t kTile = kTileBytes;       // bf16: 128 keys x 128 dims; e4m3: 256 keys x 128 dims
+  static constexpr uint32_t kSubBytes = kTile / kSub;  // one 128-key sub-tile
   static constexpr uint32_t kQHalf = kHeadsPad * 128;                  // 16 rows x 128 bytes
   static constexpr uint32_t kQBytes = kE4M3 ? kQHalf : 2 * kQHalf;
   static constexpr uint32_t OFF_RING = 0, OFF_P = kStages * kTile, OFF_Q = OFF_P + 2 * kTile,
@@ -72,13 +79,16 @@ __device__ __forceinline__ bool aborted(const int32_t* f) { return *reinterpret_
 __device__ __forceinline__ void set_abort(int32_t* f) { *reinterpret_cast<volatile int32_t*>(f) = 1; }
 
 struct DecItem {
-  int b, g, split, k0, k1, nt;
+  int b, g, split, k0, k1;
+  int nt;    // ring tiles (kSub sub-tiles of 128 keys each, the last possibly short)
+  int nsub;  // 128-key sub-tiles
 };
 // item = (split * batch + b) * hkv + g: consecutive CTAs take the KV heads of
 // one (sequence, split), whose rows lie side by side in the cache
 // ([B, cap, Hkv, D]): CTAs that start together read neighbouring pieces of
 // the same cache rows, which keeps DRAM pages open across their requests
 // (an e4m3 head row is only 128 bytes of a 1 KB cache row)
+template <int kSub>
 __device__ __forceinline__ DecItem dec_item(const DecodeArgs& a, int64_t item) {
   DecItem x;
   x.g = (int)(item % a.hkv);
@@ -88,7 +98,8 @@ __device__ __forceinline__ DecItem dec_item(const DecodeArgs& a, int64_t item) {
   const int kv_len = a.c_snap[x.b] + 1;
   x.k0 = x.split * a.chunk;
   x.k1 = min(kv_len, x.k0 + a.chunk);
-  x.nt = x.k1 > x.k0 ? (x.k1 - x.k0 + 127) / 128 : 0;
+  x.nsub = x.k1 > x.k0 ? (x.k1 - x.k0 + 127) / 128 : 0;
+  x.nt = (x.nsub + kSub - 1) / kSub;
   return x;
 }
 
@@ -107,8 +118,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                      const __grid_constant__ CUtensorMap tmV, const DecodeArgs a, int64_t n_items) {
   using Cfg = DecCfg<kE4M3>;
-  constexpr int kStages = Cfg::kStages;
-  constexpr uint32_t kTile = Cfg::kTile, kQHalf = Cfg::kQHalf, kQBytes = Cfg::kQBytes;
+  constexpr int kStages = Cfg::kStages, kSub = Cfg::kSub;
+  constexpr uint32_t kTile = Cfg::kTile, kSubBytes = Cfg::kSubBytes, kQHalf = Cfg::kQHalf, kQBytes = Cfg::kQBytes;
   constexpr uint32_t OFF_RING = Cfg::OFF_RING, OFF_P = Cfg::OFF_P, OFF_Q = Cfg::OFF_Q, OFF_BAR = Cfg::OFF_BAR;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
@@ -162,7 +173,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tma_prefetch_desc(&tmV);
     }
     for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
-      const DecItem x = dec_item(a, item);
+      const DecItem x = dec_item<Cfg::kSub>(a, item);
       if (x.nt == 0) continue;
       const uint32_t qb = nu & 1;
       if (__any_sync(0xffffffffu, aborted(&bar->abort)) ||
@@ -192,13 +203,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           }
           if (lane == 0) {
-            // a tile starts at a multiple of 128 keys and lies in one page
-            const int64_t p = (int64_t)x.k0 + (int64_t)t * 128;
-            const int32_t y = a.pages.table ? (int32_t)paged_row(a.pages, x.b, p) : (int32_t)((int64_t)x.b * a.cap + p);
+            // a 128-key sub-tile starts at a multiple of 128 keys and lies in one page
+            const int nh = min(kSub, x.nsub - t * kSub);
             uint8_t* dst = smem + OFF_RING + s * kTile;
-            ptx::mbar_expect_tx(&bar->full[s], kTile);
-            ptx::tma_load_2d_hint(dst, map, &bar->full[s], x.g * kD, y, pol);
-            if (!kE4M3) ptx::tma_load_2d_hint(dst + kHalfBytes, map, &bar->full[s], x.g * kD + 64, y, pol);
+            ptx::mbar_expect_tx(&bar->full[s], (uint32_t)nh * kSubBytes);
+            for (int hh = 0; hh < nh; ++hh) {
+              const int64_t p = (int64_t)x.k0 + (int64_t)(t * kSub + hh) * 128;
+              const int32_t y =
+                  a.pages.table ? (int32_t)paged_row(a.pages, x.b, p) : (int32_t)((int64_t)x.b * a.cap + p);
+              ptx::tma_load_2d_hint(dst + hh * kSubBytes, map, &bar->full[s], x.g * kD, y, pol);
+              if (!kE4M3) ptx::tma_load_2d_hint(dst + kHalfBytes, map, &bar->full[s], x.g * kD + 64, y, pol);
+            }
           }
           __syncwarp();
           ++nf[s];
@@ -223,7 +238,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t nl = 0, nu = 0, T = 0;  // ring tiles consumed; non-empty items; P tiles
     bool ok = true;
     for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
-      const DecItem x = dec_item(a, item);
+      const DecItem x = dec_item<Cfg::kSub>(a, item);
       if (x.nt == 0) continue;
       const uint32_t qb = nu & 1;
       // Q landed; the softmax warps have read the previous item's S
@@ -243,12 +258,15 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         ptx::tc_fence_after();
         const uint32_t sK = ptx::smem_u32(smem + OFF_RING + s * kTile);
-        const uint32_t tS = tmem + TM_S + kHeadsPad * (uint32_t)t;
-        if constexpr (kE4M3)  // 128-byte rows: four k-steps of 32 bytes in one box
-          ptx::mma4_e4m3_ss_warp<2, 2>(tS, desc_kmajor(sK, 0), desc_kmajor(sQ, 0), idesc_s, 0u);
-        else
-          ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128Rows16>(tS, desc_kmajor(sK, 0), desc_kmajor(sQ, 0),
-                                                                          idesc_s, 0u);
+        if constexpr (kE4M3) {  // 128-byte rows: four k-steps of 32 bytes in one box, per 128-key sub-tile
+          const int nh = min(kSub, x.nsub - t * kSub);
+          for (int hh = 0; hh < nh; ++hh)
+            ptx::mma4_e4m3_ss_warp<2, 2>(tmem + TM_S + kHeadsPad * (uint32_t)(t * kSub + hh),
+                                         desc_kmajor(sK + hh * kSubBytes, 0), desc_kmajor(sQ, 0), idesc_s, 0u);
+        } else {
+          ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::KMajorSw128Rows16>(
+              tmem + TM_S + kHeadsPad * (uint32_t)t, desc_kmajor(sK, 0), desc_kmajor(sQ, 0), idesc_s, 0u);
+        }
         ptx::mma_commit_warp(&bar->empty[s]);
       }
       if (!ok) break;
@@ -271,10 +289,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         ptx::tc_fence_after();
         const uint32_t sP = ptx::smem_u32(smem + OFF_P + pb * kTile);
         const uint32_t sV = ptx::smem_u32(smem + OFF_RING + s * kTile);
-        if constexpr (kE4M3)  // V MN-major: 32 keys of 128 bytes a k-step
-          ptx::mma4_e4m3_ss_warp<2, 256>(tmem + TM_O, desc_kmajor(sP, 0), desc_kmajor(sV, 0), idesc_pv,
-                                         t > 0 ? 1u : 0u);
-        else
+        if constexpr (kE4M3) {  // V MN-major: 32 keys of 128 bytes a k-step, per 128-key sub-tile
+          const int nh = min(kSub, x.nsub - t * kSub);
+          for (int hh = 0; hh < nh; ++hh)
+            ptx::mma4_e4m3_ss_warp<2, 256>(tmem + TM_O, desc_kmajor(sP + hh * kSubBytes, 0),
+                                           desc_kmajor(sV + hh * kSubBytes, 0), idesc_pv,
+                                           (t > 0 || hh > 0) ? 1u : 0u);
+        } else
           ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::MnMajorSw128>(tmem + TM_O, desc_kmajor(sP, 0),
                                                                      desc_mnmajor(sV, 0), idesc_pv, t > 0 ? 1u : 0u);
         ptx::mma_commit_warp(&bar->empty[s]);
@@ -299,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t nu = 0, T = 0;
     bool ok = true;
     for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
-      const DecItem x = dec_item(a, item);
+      const DecItem x = dec_item<Cfg::kSub>(a, item);
       const int64_t pbase = ((int64_t)x.b * a.hq + (int64_t)x.g * group) * a.splits + x.split;
       if (x.nt == 0) {
         // a split past the sequence's keys: a partial the combine skips
@@ -318,12 +339,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       float mx[kHeadsPad];
 #pragma unroll
       for (int h = 0; h < kHeadsPad; ++h) mx[h] = -INFINITY;
-      for (int t = 0; t < x.nt; ++t) {
+      for (int j = 0; j < x.nsub; ++j) {
         uint32_t v[kHeadsPad];
-        ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)t, v);
+        ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)j, v);
         ptx::tmem_ld_wait();
         ptx::reg_fence(v);
-        if (x.k0 + t * 128 + r < x.k1) {
+        if (x.k0 + j * 128 + r < x.k1) {
 #pragma unroll
           for (int h = 0; h < kHeadsPad; ++h) mx[h] = fmaxf(mx[h], __uint_as_float(v[h]));
         }
@@ -351,11 +372,6 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
       for (int h = 0; h < kHeadsPad; ++h) l[h] = 0.f;
       for (int t = 0; t < x.nt; ++t, ++T) {
-        uint32_t v[kHeadsPad];
-        ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)t, v);
-        ptx::tmem_ld_wait();
-        ptx::reg_fence(v);
-        const bool valid = x.k0 + t * 128 + r < x.k1;
         const uint32_t pb = T & 1;
         if (T >= 2 && !wait(&bar->p_free[pb], ((T >> 1) - 1) & 1, a.status)) {
           ok = false;
@@ -363,19 +379,35 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         uint8_t* P = smem + OFF_P + pb * kTile;
         if constexpr (kE4M3) {
+          const int nh = min(kSub, x.nsub - t * kSub);
+          for (int hh = 0; hh < nh; ++hh) {
+            const int j = t * kSub + hh;
+            uint32_t v[kHeadsPad];
+            ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)j, v);
+            ptx::tmem_ld_wait();
+            ptx::reg_fence(v);
+            const bool valid = x.k0 + j * 128 + r < x.k1;
+            uint8_t* Ph = P + hh * kSubBytes;
 #pragma unroll
-          for (int h = 0; h < kHeadsPad; h += 4) {
-            float p4[4];
+            for (int h = 0; h < kHeadsPad; h += 4) {
+              float p4[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              p4[e] = (valid && h + e < group) ? ex2(__uint_as_float(v[h + e]) * c2 - m2[h + e]) : 0.f;
-              l[h + e] += p4[e];
+              for (int e = 0; e < 4; ++e) {
+                p4[e] = (valid && h + e < group) ? ex2(__uint_as_float(v[h + e]) * c2 - m2[h + e]) : 0.f;
+                l[h + e] += p4[e];
+              }
+              const uint32_t b4 = pack_e4m3x4(p4[0], p4[1], p4[2], p4[3]);
+#pragma unroll
+              for (int e = 0; e < 4; ++e)
+                Ph[p_offset<true>((uint32_t)(h + e), (uint32_t)r)] = (uint8_t)(b4 >> (8 * e));
             }
-            const uint32_t b4 = pack_e4m3x4(p4[0], p4[1], p4[2], p4[3]);
-#pragma unroll
-            for (int e = 0; e < 4; ++e) P[p_offset<true>((uint32_t)(h + e), (uint32_t)r)] = (uint8_t)(b4 >> (8 * e));
           }
         } else {
+          uint32_t v[kHeadsPad];
+          ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)t, v);
+          ptx::tmem_ld_wait();
+          ptx::reg_fence(v);
+          const bool valid = x.k0 + t * 128 + r < x.k1;
 #pragma unroll
           for (int h = 0; h < kHeadsPad; ++h) {
             const float p = (valid && h < group) ? ex2(__uint_as_float(v[h]) * c2 - m2[h]) : 0.f;
