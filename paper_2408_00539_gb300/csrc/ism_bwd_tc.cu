@@ -33,29 +33,47 @@ __device__ __forceinline__ void ld64(uint32_t taddr, uint32_t (&a)[32], uint32_t
 }
 
 // ------------------------------------------------------------------ delta
-// One 16-lane group per (row, head): 8 bf16 per lane, D = 128.
+// One 16-lane group per (row, head): 8 bf16 per lane, D = 128.  A group takes
+// four (row, head) pairs per round with all eight loads issued before any
+// use (more bytes in flight per thread: the kernel only streams O and dO).
+// The reductions shuffle within the group's own 16 lanes, so the two groups
+// of a warp may run different numbers of rounds.
 __global__ void delta_kernel(const __nv_bfloat16* __restrict__ O, const __nv_bfloat16* __restrict__ dO,
                              float* __restrict__ delta, int64_t rows, int hq) {
+  constexpr int kUnroll = 4;
   const int64_t n = rows * hq;
   const int sub = threadIdx.x & 15;
-  for (int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 4; i < n;
-       i += ((int64_t)gridDim.x * blockDim.x) >> 4) {
-    const uint4 a = reinterpret_cast<const uint4*>(O + i * kD)[sub];
-    const uint4 b = reinterpret_cast<const uint4*>(dO + i * kD)[sub];
-    const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&a);
-    const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&b);
-    float acc = 0.f;
+  const uint32_t group_mask = 0xFFFFu << (threadIdx.x & 16);
+  const int64_t groups = ((int64_t)gridDim.x * blockDim.x) >> 4;
+  for (int64_t i0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 4; i0 < n; i0 += groups * kUnroll) {
+    uint4 a[kUnroll], b[kUnroll];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const float2 x = __bfloat1622float2(pa[k]), y = __bfloat1622float2(pb[k]);
-      acc = fmaf(x.x, y.x, fmaf(x.y, y.y, acc));
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t i = i0 + u * groups;
+      if (i < n) {
+        a[u] = reinterpret_cast<const uint4*>(O + i * kD)[sub];
+        b[u] = reinterpret_cast<const uint4*>(dO + i * kD)[sub];
+      }
     }
 #pragma unroll
-    for (int o = 8; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (sub == 0) {
-      const int64_t row = i / hq;
-      const int h = (int)(i % hq);
-      delta[(int64_t)h * rows + row] = acc;
+    for (int u = 0; u < kUnroll; ++u) {
+      const int64_t i = i0 + u * groups;
+      if (i >= n) break;
+      const __nv_bfloat162* pa = reinterpret_cast<const __nv_bfloat162*>(&a[u]);
+      const __nv_bfloat162* pb = reinterpret_cast<const __nv_bfloat162*>(&b[u]);
+      float acc = 0.f;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float2 x = __bfloat1622float2(pa[k]), y = __bfloat1622float2(pb[k]);
+        acc = fmaf(x.x, y.x, fmaf(x.y, y.y, acc));
+      }
+#pragma unroll
+      for (int o = 8; o > 0; o >>= 1) acc += __shfl_xor_sync(group_mask, acc, o);
+      if (sub == 0) {
+        const int64_t row = i / hq;
+        const int h = (int)(i % hq);
+        delta[(int64_t)h * rows + row] = acc;
+      }
     }
   }
 }

@@ -125,6 +125,17 @@ def test_small_bf16_group_sizes(ism, hq, hkv):
     _check_small(ism, _small_bf16(128, hq=hq, hkv=hkv, seed=hq * 10 + hkv), "default")
 
 
+def test_small_bf16_odd_heads_odd_tokens(ism):
+    """Three query heads on one KV head and an odd number of tokens: the
+    backward's Delta pass pairs (row, head) items with 16-lane groups, two to
+    a warp, and here the two groups of a warp run different numbers of
+    rounds."""
+    segs = wl.pack([([70, 150, 170, 301], [0, 1, 0, 1]), ([33, 90, 200, 517], [0, 1, 0, 1]), ([1], [1])])
+    assert segs.total_tokens % 2 == 1
+    w = wl.Workload("odd_heads", segs, 3, 1, 128, "bf16", 128 ** -0.5, 0.5, 23)
+    _check_small(ism, w, "default")
+
+
 def _check_small(ism, w, path):
     (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w, minimal_workspace=path == "recompute_dq")
     o_ref, lse_ref = orc.attn_fwd(q, k, v, w.segs, w.softmax_scale)
