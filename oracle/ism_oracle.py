@@ -308,6 +308,34 @@ def attn_bwd(q, k, v, dout, segs, scale: float):
     return dq, dk, dv
 
 
+def attn_bwd_dq_rows(q, k, v, dout, segs, scale: float, rows):
+    """dQ of ISM attention for a subset of query rows (sorted global token
+    indices), every query head.  Row j of dQ needs only row j of P and of dP:
+    dQ_j = scale * sum_i dS_ji k_i with dS_j = P_j * (dP_j - Delta_j),
+    dP_j = dO_j V^T and Delta_j = dO_j . O_j (O_j from the same row's
+    forward).  Returns float64 dq [T, Hq, D] with NaN outside ``rows``."""
+    q, k, v, dout = _f64(q), _f64(k), _f64(v), _f64(dout)
+    T, hq, D = q.shape
+    hkv = k.shape[1]
+    rows = np.asarray(rows)
+    dq = np.full((T, hq, D), np.nan)
+    for b in range(int(segs.cu_seqlens.shape[0]) - 1):
+        t0, L, se, st = segs.seq(b)
+        want = rows[(rows >= t0) & (rows < t0 + L)] - t0
+        if L == 0 or want.shape[0] == 0:
+            continue
+        mask = mask_eq_fj(se, st, rows=want)
+        for h in range(hq):
+            g = _group(hq, hkv, h)
+            kk, vv = k[t0:t0 + L, g], v[t0:t0 + L, g]
+            qq, do = q[t0 + want, h], dout[t0 + want, h]
+            o, _, p = attn_rows(qq, kk, vv, mask, scale)
+            dp = do @ vv.T
+            delta = (do * o).sum(axis=1, keepdims=True)
+            dq[t0 + want, h] = scale * ((p * (dp - delta)) @ kk)
+    return dq
+
+
 # --------------------------------------------------------------------------
 # KV-cache reuse, Section 2.3
 # --------------------------------------------------------------------------

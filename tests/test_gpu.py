@@ -226,7 +226,8 @@ def test_full_size_parity_sampled_groups(ism, make):
     """Full-size launch (all sequences, all heads, as benchmarked); the oracle
     recomputes complete GQA groups: the first and the last KV head of the
     longest sequence, and for the packed buffer also the last dialogue, which
-    starts at an offset that is not a multiple of the 128-row tile.  Every
+    starts at an offset that is not a multiple of the 128-row tile; and O,
+    LSE and dQ of every query head on sampled rows of every sequence.  Every
     output element of the launch must be finite."""
     w = make()
     inputs, outputs = _run_pass(ism, w)
@@ -240,6 +241,35 @@ def test_full_size_parity_sampled_groups(ism, make):
         checks.append((last, w.num_heads_kv // 2))
     for bb, g in dict.fromkeys(checks):
         _check_group(w, bb, g, inputs, outputs)
+    _check_all_heads_sampled_rows(w, inputs, outputs)
+
+
+def _sample_rows(segs, rng, n_random=24):
+    """Global rows to check at full size: each sequence's first and last rows,
+    the first and last row of every segment, and random rows."""
+    rows = set()
+    for b in range(segs.num_seqs):
+        t0, L, se, st = segs.seq(b)
+        start = 0
+        for e in se.tolist():
+            if e > start:
+                rows.update((t0 + start, t0 + e - 1))
+            start = e
+        rows.update(int(t0 + x) for x in rng.integers(0, L, size=n_random))
+    return np.array(sorted(rows), dtype=np.int64)
+
+
+def _check_all_heads_sampled_rows(w, inputs, outputs):
+    """Every query head of the full-size launch on sampled rows: O and LSE of
+    a row need only that row's forward, and dQ of a row only that row's P and
+    dP, so the oracle computes them row by row for all 32 heads."""
+    (q, k, v, do), (o, lse, dq, dk, dv) = inputs, outputs
+    rows = _sample_rows(w.segs, np.random.Generator(np.random.PCG64(w.seed + 99)))
+    o_ref, lse_ref = orc.attn_fwd(q, k, v, w.segs, w.softmax_scale, rows=rows)
+    dq_ref = orc.attn_bwd_dq_rows(q, k, v, do, w.segs, w.softmax_scale, rows)
+    _cmp(f"o, all heads, {rows.size} rows", o[rows], o_ref[rows], "bf16")
+    _cmp_lse(f"lse, all heads, {rows.size} rows", lse[:, rows], lse_ref[:, rows], "bf16")
+    _cmp(f"dq, all heads, {rows.size} rows", dq[rows], dq_ref[rows], "bf16")
 
 
 @pytest.mark.parametrize("schedule", ["stored_ds", "recompute_dq"])

@@ -334,6 +334,24 @@ def test_bwd_vs_library_autograd():
         np.testing.assert_allclose(dv[sl], vt.grad.permute(1, 0, 2).numpy(), rtol=1e-10, atol=1e-12)
 
 
+def test_dq_rows_vs_library_autograd():
+    # independent construction: masked SDPA in torch fp64 and autograd; the
+    # row-subset dQ must equal the gradient rows it selects
+    rng = np.random.Generator(np.random.PCG64(33))
+    segs = wl.random_dialogue_set(rng, 3, 70, min_len=3)
+    T = segs.total_tokens
+    q, k, v, do = _rand(rng, T, 4, 8), _rand(rng, T, 2, 8), _rand(rng, T, 2, 8), _rand(rng, T, 4, 8)
+    scale = 0.4
+    rows = np.sort(rng.choice(T, size=T // 3, replace=False))
+    dq = orc.attn_bwd_dq_rows(q, k, v, do, segs, scale, rows)
+    qt = torch.from_numpy(q).requires_grad_()
+    ot = _mask_sdpa_torch(qt, torch.from_numpy(k), torch.from_numpy(v), segs, scale)
+    ot.backward(torch.from_numpy(do))
+    np.testing.assert_allclose(dq[rows], qt.grad.numpy()[rows], rtol=1e-10, atol=1e-12)
+    others = np.setdiff1d(np.arange(T), rows)
+    assert np.isnan(dq[others]).all()
+
+
 # ---------------------------------------------------------------- KV cache
 
 def test_prefill_append_equals_rows_of_full_forward():
