@@ -332,3 +332,21 @@ def test_e4m3_rope_append(ism, l_new, segs, hq, hkv):
     assert err.max() <= (2 ** -4 + 2 ** -9) * vmax, f"o_new: max abs err {err.max():.3e} (max|V| {vmax:.3f})"
     assert err.mean() <= 4e-3, f"o_new: mean abs err {err.mean():.3e}"
     _cmp_lse("lse_new", lse, np.transpose(lse_ref, (1, 0, 2)), "bf16")
+
+
+def test_rope_zero_length_sequences_and_empty_batch(ism):
+    """Zero-length sequences share their offset with the next sequence: the
+    rotation pass must still find each token's own sequence (positions
+    restart after every boundary).  An empty batch launches nothing."""
+    segs = wl.pack([([0], [0]), ([40, 100], [0, 1]), ([0], [1]), ([0], [0]), ([1], [1]), ([130, 131], [0, 1])])
+    w = wl.Workload("rope_zero_len", segs, 4, 2, 128, "bf16", 128 ** -0.5, 0.5, 84)
+    cos_t, sin_t = _tables(131, 128, "random", seed=7)
+    inputs, outputs = _run(ism, w, cos_t, sin_t)
+    _check_all(w, cos_t, sin_t, inputs, outputs)
+    empty = ism.Segments.from_numpy([0, 0], [0, 0], [], [], DEV)
+    q = torch.zeros((0, 4, 128), dtype=torch.bfloat16, device=DEV)
+    k = torch.zeros((0, 2, 128), dtype=torch.bfloat16, device=DEV)
+    launches = ism.kernel_launches()
+    o, lse, qr, kr = ism.fwd_rope(empty, q, k, k, cos_t.to(DEV), sin_t.to(DEV), 0.1)
+    assert o.shape == (0, 4, 128) and ism.kernel_launches() == launches
+    ism.check_status()
