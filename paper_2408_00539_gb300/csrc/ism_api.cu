@@ -885,12 +885,12 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
   a.status = status;
   a.flags = tc_flags();
   // The items of the paired forward (query tile, head pair) all cost about the
-  // same in a prefill; those that would form a last, partial wave of CTAs run
+  // same in a prefill; those that would leave a last round with idle SMs run
   // as two halves of their key range instead, when the items are long enough
-  // (at least 64 key tiles) for the halves to outweigh the merge; measured on
-  // the 8 x 16K prefill: 0.781 -> 0.751 ms in bf16, but slower in e4m3 and for
-  // 40-token chunks over 4000 keys, which stay whole.  ISM_PREFILL_SPLIT=n
-  // forces n split items.
+  // (at least 64 key tiles) for the halves to outweigh the merge.  Measured
+  // on the 8 x 16K prefill with the persistent forward: bf16 0.795 -> 0.719
+  // ms, e4m3 0.668 -> 0.595 ms; 40-token chunks over 4000 keys stay whole.
+  // ISM_PREFILL_SPLIT=n forces n split items.
   if ((use_tc(shape) || shape->dtype == ISM_E4M3) && d == 128 && (hq / hkv) % 2 == 0 && !a.pair_order &&
       L.split_cap > 0) {
     const int64_t items = a.nq * (hq / 2);
@@ -900,7 +900,7 @@ ism_status_t append_impl(const ism_attn_shape_t* shape, int32_t batch, const voi
     } else {
       const int sms = sm_count();
       const int64_t key_tiles = ((int64_t)max_c + l_new + kTile - 1) / kTile;
-      if (items > sms && shape->dtype == ISM_BF16 && key_tiles >= 64) n_split = items % sms;
+      if (items > sms && key_tiles >= 64) n_split = items % sms;
     }
     if (n_split > L.split_cap) n_split = L.split_cap;
     if (n_split > 0) {
