@@ -519,6 +519,17 @@ def run_cuda(args, w):
                    else "cuda cores", "bwd_schedule": "stored dS" if stored_ds else "recompute dQ",
                    "bwd_workspace_bytes": ws_bytes, "parallelism": f"replicas x{world}"},
         "kernel_ms": mean_k,
+        "phases": {
+            "fwd": {"ms": mean_k["meta"] + mean_k["fwd"], "flops": 4 * D * n_vis,
+                    "tflops": 4 * D * n_vis / ((mean_k["meta"] + mean_k["fwd"]) * 1e-3) / 1e12,
+                    "kernels": "metadata pass + forward"},
+            "bwd": {"ms": mean_k["meta"] + mean_k["bwd_pre"] + mean_k["bwd_dkdv"] + mean_k["bwd_dq"],
+                    "flops": 10 * D * n_vis,
+                    "tflops": 10 * D * n_vis / ((mean_k["meta"] + mean_k["bwd_pre"] + mean_k["bwd_dkdv"] +
+                                                 mean_k["bwd_dq"]) * 1e-3) / 1e12,
+                    "kernels": "metadata pass + Delta + dK/dV + dQ"},
+            "note": "per-call kernel times from the timer hooks (each call runs its own metadata pass); the "
+                    "headline counts fwd 4*D*N_vis and bwd 10*D*N_vis"},
         "roofline": roofline,
         "kernel_rooflines": rooflines,
         "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
