@@ -445,8 +445,6 @@ ism_status_t ism_attn_bwd_workspace_size_min(const ism_segments_t* segs, const i
 
 namespace {
 
-// The one-pass forward for bf16 / fp32 (ism_attn_fwd) and e4m3 inputs
-// (ism_attn_fwd_e4m3; qk_descale = q_descale * k_descale).
 // Checks the rotary tables of a one-pass call: present, aligned, covering
 // every position of the batch (the longest sequence), for bf16 / fp32 inputs.
 ism_status_t check_rope_pass(const ism_rope_t* rope, const ism_attn_shape_t* shape, const SegInfo& info) {
