@@ -501,9 +501,7 @@ cudaError_t launch_decode_tc_t(const DecodeArgs& a, cudaStream_t st) {
   if ((e = cudaFuncSetAttribute(decode_tc_kernel<kE4M3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)Cfg::kSmemBytes)) != cudaSuccess)
     return e;
-  int dev = 0, sms = 0;
-  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  const int64_t sms = sm_count();
   const int64_t n_items = (int64_t)a.batch * a.hkv * a.splits;
   int64_t grid = sms < n_items ? sms : n_items;
   if (grid <= 0) return cudaSuccess;
