@@ -336,6 +336,47 @@ def attn_bwd_dq_rows(q, k, v, dout, segs, scale: float, rows):
     return dq
 
 
+def attn_bwd_dkdv_keys(q, k, v, dout, segs, scale: float, keys):
+    """dK and dV of ISM attention for a subset of key rows (sorted global token
+    indices), every KV head.  Key i receives contributions only from the query
+    rows j that see it (i < kv_end[j], Eq. fj); each of those rows needs its
+    whole softmax row (P_j over all of its visible keys, O_j, and with it
+    Delta_j = dO_j . O_j), so the rows are computed in full and the
+    gradients summed over them for the selected keys only:
+    dV_i = sum_j P_ji dO_j, dK_i = scale * sum_j dS_ji q_j with
+    dS_j = P_j * (dO_j V^T - Delta_j), summed over the query heads of the
+    KV head.  Returns float64 (dk, dv) [T, Hkv, D] with NaN outside ``keys``."""
+    q, k, v, dout = _f64(q), _f64(k), _f64(v), _f64(dout)
+    T, hq, D = q.shape
+    hkv = k.shape[1]
+    keys = np.asarray(keys)
+    dk = np.full((T, hkv, D), np.nan)
+    dv = np.full((T, hkv, D), np.nan)
+    for b in range(int(segs.cu_seqlens.shape[0]) - 1):
+        t0, L, se, st = segs.seq(b)
+        sel = keys[(keys >= t0) & (keys < t0 + L)] - t0
+        if L == 0 or sel.shape[0] == 0:
+            continue
+        f = f_vector(se, st)                       # row j (0-based) sees keys [0, f[j])
+        rows = np.nonzero(f > sel.min())[0]        # the rows that see at least one selected key
+        mask = mask_eq_fj(se, st, rows=rows)
+        dk[t0 + sel] = 0.0
+        dv[t0 + sel] = 0.0
+        for h in range(hq):
+            g = _group(hq, hkv, h)
+            kk, vv = k[t0:t0 + L, g], v[t0:t0 + L, g]
+            for r0 in range(0, rows.shape[0], ROW_BLOCK):
+                idx = rows[r0:r0 + ROW_BLOCK]
+                qq, do = q[t0 + idx, h], dout[t0 + idx, h]
+                o, _, p = attn_rows(qq, kk, vv, mask[r0:r0 + ROW_BLOCK], scale)
+                delta = (do * o).sum(axis=1, keepdims=True)
+                ps = p[:, sel]
+                ds = ps * (do @ vv[sel].T - delta)
+                dv[t0 + sel, g] += ps.T @ do
+                dk[t0 + sel, g] += scale * (ds.T @ qq)
+    return dk, dv
+
+
 # --------------------------------------------------------------------------
 # KV-cache reuse, Section 2.3
 # --------------------------------------------------------------------------

@@ -1067,3 +1067,38 @@ def test_prefill_key_split(ism, dtype, n_split, knobs):
         vmax = max(float(deq(v8c, vs).abs().max()), float(deq(v8n, vs).abs().max()))
         _cmp_e4m3("o_new", o, o_ref, vmax)
     _cmp_lse("lse_new", lse, np.transpose(lse_ref, (1, 0, 2)), "bf16")
+
+
+# ---------------------------------------------------------------- maximum size: one long dialogue
+
+def test_long_context_128k_minimum_workspace(ism):
+    """One 131072-token dialogue of a few hundred turns (8 query / 2 KV
+    heads, head_dim 128, bf16) through the forward and the minimum-workspace
+    backward (the stored-dS workspace would need about 137 GB here; long
+    contexts run the recompute schedule).  The oracle checks O, LSE and dQ of
+    every head on sampled rows, and dK / dV of two whole key tiles near the
+    end of the dialogue (the last one and the one 640 keys before the end)
+    for both KV heads, from the full softmax rows of every query that sees
+    those keys."""
+    L = 131072
+    rng = np.random.Generator(np.random.PCG64(128))
+    segs_np = wl.pack([wl.draw_dialogue(rng, L, 300, 400)])
+    w = wl.Workload("long_128k", segs_np, 8, 2, 128, "bf16", 128 ** -0.5, 0.5, 128)
+    (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w, minimal_workspace=True)
+    for name, t in zip(("o", "lse", "dq", "dk", "dv"), (o, lse, dq, dk, dv)):
+        assert bool(torch.isfinite(t).all()), f"{name}: non-finite values"
+    # O, LSE, dQ: every head, 32 segment boundaries and 16 random rows
+    ends = segs_np.seg_end
+    bounds = np.unique(np.concatenate([ends[ends < L], np.maximum(ends - 1, 0)]))
+    rows = np.unique(np.concatenate([rng.choice(bounds, size=32, replace=False), rng.integers(0, L, size=16),
+                                     [0, L - 1]])).astype(np.int64)
+    o_ref, lse_ref = orc.attn_fwd(q, k, v, segs_np, w.softmax_scale, rows=rows)
+    dq_ref = orc.attn_bwd_dq_rows(q, k, v, do, segs_np, w.softmax_scale, rows)
+    _cmp(f"o, all heads, {rows.size} rows", o[rows], o_ref[rows], "bf16")
+    _cmp_lse(f"lse, all heads, {rows.size} rows", lse[:, rows], lse_ref[:, rows], "bf16")
+    _cmp(f"dq, all heads, {rows.size} rows", dq[rows], dq_ref[rows], "bf16")
+    # dK, dV: two key tiles near the end, both KV heads
+    keys = np.concatenate([np.arange(L - 640, L - 512), np.arange(L - 128, L)])
+    dk_ref, dv_ref = orc.attn_bwd_dkdv_keys(q, k, v, do, segs_np, w.softmax_scale, keys)
+    _cmp(f"dk, {keys.size} keys", dk[keys], dk_ref[keys], "bf16")
+    _cmp(f"dv, {keys.size} keys", dv[keys], dv_ref[keys], "bf16")

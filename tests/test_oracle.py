@@ -352,6 +352,25 @@ def test_dq_rows_vs_library_autograd():
     assert np.isnan(dq[others]).all()
 
 
+def test_dkdv_keys_vs_library_autograd():
+    # independent construction: masked SDPA in torch fp64 and autograd; the
+    # key-subset dK / dV must equal the gradient rows it selects, GQA summed
+    rng = np.random.Generator(np.random.PCG64(34))
+    segs = wl.random_dialogue_set(rng, 3, 70, min_len=3)
+    T = segs.total_tokens
+    q, k, v, do = _rand(rng, T, 4, 8), _rand(rng, T, 2, 8), _rand(rng, T, 2, 8), _rand(rng, T, 4, 8)
+    scale = 0.4
+    keys = np.sort(rng.choice(T, size=T // 3, replace=False))
+    dk, dv = orc.attn_bwd_dkdv_keys(q, k, v, do, segs, scale, keys)
+    kt, vt = torch.from_numpy(k).requires_grad_(), torch.from_numpy(v).requires_grad_()
+    ot = _mask_sdpa_torch(torch.from_numpy(q), kt, vt, segs, scale)
+    ot.backward(torch.from_numpy(do))
+    np.testing.assert_allclose(dk[keys], kt.grad.numpy()[keys], rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(dv[keys], vt.grad.numpy()[keys], rtol=1e-10, atol=1e-12)
+    others = np.setdiff1d(np.arange(T), keys)
+    assert np.isnan(dk[others]).all() and np.isnan(dv[others]).all()
+
+
 # ---------------------------------------------------------------- KV cache
 
 def test_prefill_append_equals_rows_of_full_forward():
