@@ -551,6 +551,7 @@ def run_cuda(args, w):
         line["rope"] = measure_training_config(dev, w, peaks, steps=args.steps, rope=True)
         line["configs"] = {wname: measure_training_config(dev, WORKLOADS[wname](), peaks, steps=args.steps)
                            for wname in ("mha_4k", "packed_32k") if WORKLOADS[wname]().name != w.name}
+        line["long_context"] = measure_long_context(dev, peaks)
     if not args.no_append:
         line["append"] = measure_append(dev, read_peaks()[0])
         line["session"] = measure_session(dev)
@@ -850,6 +851,68 @@ def measure_training_config(dev, w, peaks, steps=20, minimal_workspace=False, ro
            "bwd_workspace_bytes": ws_bytes, "kernel_ms": mean_k, "kernel_frac_of_bf16_peak": fracs,
            "clocks": clocks.summary()}
     del q, k, v, do, o, lse, dq, dk, dv, ws, flush
+    torch.cuda.empty_cache()
+    return out
+
+
+def measure_long_context(dev, peaks, length=131072, steps=3):
+    """One dialogue of ``length`` tokens (a few hundred turns of the config-2
+    recipe, 32 query / 8 KV heads, head_dim 128, bf16) through the forward and
+    the minimum-workspace backward: the stored-dS workspace would need
+    pairs x 32 heads x 32 KiB (about 0.5 TB at 128K), so long contexts run
+    the recompute schedule.  Inputs drawn on the device (seeded); CUDA events
+    around each step; the step is far larger than L2."""
+    import torch
+    from paper_2408_00539_gb300 import ism
+    rng = np.random.Generator(np.random.PCG64(131))
+    segs_np = wl.pack([wl.draw_dialogue(rng, length, 300, 400)])
+    hq, hkv, D = 32, 8, 128
+    scale = D ** -0.5
+    g = torch.Generator(device=dev).manual_seed(131)
+    q = torch.randn((length, hq, D), generator=g, device=dev).mul_(0.5).bfloat16()
+    k = torch.randn((length, hkv, D), generator=g, device=dev).mul_(0.5).bfloat16()
+    v = torch.randn((length, hkv, D), generator=g, device=dev).mul_(0.5).bfloat16()
+    do = torch.randn((length, hq, D), generator=g, device=dev).bfloat16()
+    segs = ism.Segments.from_workload(segs_np, dev)
+    ws = torch.empty(ism.bwd_workspace_size(segs, q, k, scale, minimal=True), dtype=torch.uint8, device=dev)
+    o, lse = ism.fwd(segs, q, k, v, scale)
+    dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    stream = torch.cuda.current_stream(dev)
+    n_vis = n_visible(segs_np) * hq
+    flops = 14 * D * n_vis
+    kinds = {"fwd": ism.KERNEL_FWD, "bwd_dkdv": ism.KERNEL_BWD_DKDV, "bwd_dq": ism.KERNEL_BWD_DQ}
+    ms, kt = [], {n: [] for n in kinds}
+    for it in range(steps + 1):
+        ev = {n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for n in kinds}
+        for n, kid in kinds.items():
+            for e in ev[n]:
+                e.record(stream)
+            ism.set_kernel_timer(kid, *ev[n])
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        ism.fwd(segs, q, k, v, scale, out=o, lse=lse)
+        ism.bwd(segs, q, k, v, o, lse, do, scale, dq=dq, dk=dk, dv=dv, workspace=ws)
+        e1.record(stream)
+        e1.synchronize()
+        if it:
+            ms.append(e0.elapsed_time(e1))
+            for n in kinds:
+                kt[n].append(ev[n][0].elapsed_time(ev[n][1]))
+    for kid in kinds.values():
+        ism.set_kernel_timer(kid)
+    ism.check_status(dev)
+    step_ms = float(np.median(ms))
+    tflops = flops / (step_ms * 1e-3) / 1e12
+    mean_k = {n: float(np.mean(t)) for n, t in kt.items()}
+    fr = {"fwd": 4 * D * n_vis / (mean_k["fwd"] * 1e-3) / 1e12 / peaks["bf16_tflops"],
+          "bwd_dkdv": 8 * D * n_vis / (mean_k["bwd_dkdv"] * 1e-3) / 1e12 / peaks["bf16_tflops"],
+          "bwd_dq": 6 * D * n_vis / (mean_k["bwd_dq"] * 1e-3) / 1e12 / peaks["bf16_tflops"]}
+    out = {"workload": f"long_t{length}_hq32_hkv8_d128", "segments": int(segs_np.seg_end.shape[0]),
+           "n_vis_pairs": n_vis, "ms_per_step": step_ms, "steps": steps, "tflops": tflops,
+           "pct_of_bf16_peak": tflops / peaks["bf16_tflops"] * 100, "bwd_schedule": "recompute dQ",
+           "bwd_workspace_bytes": int(ws.numel()), "kernel_ms": mean_k, "kernel_frac_of_bf16_peak": fr,
+           "note": "dQ kernel recomputes S and dP: 6*D*N_vis; dK/dV 8*D*N_vis; forward 4*D*N_vis"}
+    del q, k, v, do, o, lse, dq, dk, dv, ws
     torch.cuda.empty_cache()
     return out
 
