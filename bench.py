@@ -298,7 +298,8 @@ def run_cuda(args, w):
     flops = 14 * D * n_vis
     o, lse = ism.fwd(segs, qd, kd, vd, w.softmax_scale)
     # backward workspace sized for the stored-dS schedule where it applies
-    ws_bytes = ism.bwd_workspace_size(segs, qd, kd, w.softmax_scale)
+    # (the minimum with --min-workspace: the recompute schedule)
+    ws_bytes = ism.bwd_workspace_size(segs, qd, kd, w.softmax_scale, minimal=args.min_workspace)
     stored_ds = ws_bytes > ism.bwd_workspace_size(segs, qd, kd, w.softmax_scale, minimal=True)
     ws_b = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
     dq, dk, dv = ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, workspace=ws_b)
@@ -1182,7 +1183,9 @@ def profile_decode(dtype: str, steps: int):
 WORKLOADS = {"gqa_8k": wl.gqa_8k, "mha_4k": wl.mha_4k, "packed_32k": wl.packed_32k,
              # one 4K dialogue of the same recipes: small enough for full ncu captures
              "gqa_4k_b1": lambda: wl.gqa_8k(batch=1, seqlen=4096),
-             "mha_4k_b1": lambda: wl.mha_4k(batch=1)}
+             "mha_4k_b1": lambda: wl.mha_4k(batch=1),
+             # one long dialogue (few hundred turns): with --min-workspace, the recompute schedule
+             "long_32k": lambda: wl.long_dialogue(32768)}
 
 
 def main():
@@ -1199,6 +1202,8 @@ def main():
     ap.add_argument("--profile-step", action="store_true",
                     help="run the warm-up steps and one more step, print nothing (for ncu)")
     ap.add_argument("--rope", action="store_true", help="with --profile-step: the rotary forward and backward")
+    ap.add_argument("--min-workspace", action="store_true",
+                    help="backward with the minimum workspace (recompute schedule) in the headline step")
     ap.add_argument("--profile-decode", choices=["bf16", "e4m3"],
                     help="run only warm-up + steps single-token steps on the 8 x 16K cache, print nothing (for ncu)")
     args = ap.parse_args()

@@ -177,6 +177,14 @@ def packed_32k(seed: int = 4, total: int = 32768, min_len: int = 512) -> Workloa
                     1.0 / np.sqrt(128.0), 0.5, seed)
 
 
+def long_dialogue(length: int, seed: int = 131, turns=(300, 400)) -> Workload:
+    """One dialogue of ``length`` tokens with a few hundred turns of the
+    config-2 length recipe, 32 query / 8 KV heads, head_dim 128, bf16."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    dia = [draw_dialogue(rng, length, turns[0], turns[1])]
+    return Workload(f"long_t{length}_hq32_hkv8_d128", pack(dia), 32, 8, 128, "bf16", 1.0 / np.sqrt(128.0), 0.5, seed)
+
+
 @dataclass
 class AppendWorkload:
     name: str
