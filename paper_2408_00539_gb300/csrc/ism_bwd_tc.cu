@@ -336,6 +336,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tc_fence_before();
       ptx::mbar_arrive(&bar->p_full[R]);
     }
+    // rotary encoding: this warpgroup's 32 pairs of the row's tables, loaded
+    // while the last dQ MMAs run
+    float rc[32], rs[32];
+    if (valid && a.rope_cos) {
+      const int64_t pos = (int64_t)w.tile * kRows + r;
+      rope_row<32>(a.rope_cos + pos * 64 + wg * 32, a.rope_sin + pos * 64 + wg * 32, rc, rs);
+    }
     if (ok) ok = wait(&bar->final_mma, 0, a.status);
     if (!ok) {
       set_abort(&bar->abort);
@@ -353,11 +360,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::reg_fence(q0);
       ptx::reg_fence(q1);
       if (valid && a.rope_cos) {
-        const int64_t pos = (int64_t)w.tile * kRows + r;
         uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) + grow * a.hq * kD + h * kD);
-        float rc[32], rs[32];
-        rope_row32(a.rope_cos + pos * 64 + wg * 32, a.rope_sin + pos * 64 + wg * 32, rc, rs);
-        rope_back_store32(q0, q1, a.scale, rc, rs, dst + 4 * wg, dst + 8 + 4 * wg);
+        rope_back_store<32>(q0, q1, a.scale, rc, rs, dst + 4 * wg, dst + 8 + 4 * wg);
       } else if (valid) {
         uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) + grow * a.hq * kD + h * kD +
                                               wg * 64);
@@ -885,44 +889,22 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
       }
       if (!ok) break;
       // epilogue of the item: dV, dK from tensor memory
+      const int key = x.c * kRows + r;
+      const bool kvalid = key < x.w.k_len;
       if (!wait(&bar->acc_full, nacc & 1, a.status)) { ok = false; break; }
       ++nacc;
       ptx::tc_fence_after();
-      const int key = x.c * kRows + r;
-      const bool kvalid = key < x.w.k_len;
       const int64_t krow = (int64_t)x.w.k_base + key;
-      // warpgroup 0 writes dV, warpgroup 1 writes dK (scaled)
-      __nv_bfloat16* outp = reinterpret_cast<__nv_bfloat16*>(wg == 0 ? a.dv : a.dk) + krow * a.hkv * kD + x.g * kD;
-      const float f = wg == 0 ? 1.f : a.scale;
-      const uint32_t col = wg == 0 ? TM_DV : TM_DK;
-      if (wg == 1 && a.rope_cos) {
-        // rotary encoding: dK of the unrotated keys, columns k and k + 64 pair up
-#pragma unroll 1
-        for (int q2 = 0; q2 < 2; ++q2) {
-          uint32_t lo[32], hi[32];
-          ptx::tmem_ld32(tmem + lane_addr + col + q2 * 32, lo);
-          ptx::tmem_ld32(tmem + lane_addr + col + 64 + q2 * 32, hi);
-          ptx::tmem_ld_wait();
-          ptx::reg_fence(lo);
-          ptx::reg_fence(hi);
-          if (kvalid) {
-            float rc[32], rs[32];
-            rope_row32(a.rope_cos + (int64_t)key * 64 + 32 * q2, a.rope_sin + (int64_t)key * 64 + 32 * q2, rc, rs);
-            rope_back_store32(lo, hi, f, rc, rs, reinterpret_cast<uint4*>(outp + q2 * 32),
-                              reinterpret_cast<uint4*>(outp + 64 + q2 * 32));
-          }
-        }
-        ptx::tc_fence_before();
-        continue;
-      }
-#pragma unroll 1
-      for (int q4 = 0; q4 < 4; ++q4) {
+      __nv_bfloat16* const dvp = reinterpret_cast<__nv_bfloat16*>(a.dv) + krow * a.hkv * kD + x.g * kD;
+      __nv_bfloat16* const dkp = reinterpret_cast<__nv_bfloat16*>(a.dk) + krow * a.hkv * kD + x.g * kD;
+      // 32 columns of an accumulator, scaled by f, to bf16 at dst
+      auto store32 = [&](uint32_t tcol, float f, __nv_bfloat16* dst) {
         uint32_t v[32];
-        ptx::tmem_ld32(tmem + lane_addr + col + q4 * 32, v);
+        ptx::tmem_ld32(tmem + lane_addr + tcol, v);
         ptx::tmem_ld_wait();
         ptx::reg_fence(v);
         if (kvalid) {
-          uint4* dst = reinterpret_cast<uint4*>(outp + q4 * 32);
+          uint4* d4 = reinterpret_cast<uint4*>(dst);
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             uint4 o;
@@ -930,9 +912,36 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
             o.y = pack_bf16(__uint_as_float(v[8 * k + 2]) * f, __uint_as_float(v[8 * k + 3]) * f);
             o.z = pack_bf16(__uint_as_float(v[8 * k + 4]) * f, __uint_as_float(v[8 * k + 5]) * f);
             o.w = pack_bf16(__uint_as_float(v[8 * k + 6]) * f, __uint_as_float(v[8 * k + 7]) * f);
-            dst[k] = o;
+            d4[k] = o;
           }
         }
+      };
+      if (wg == 1 && a.rope_cos) {
+#pragma unroll 1
+        for (int q2 = 0; q2 < 2; ++q2) {
+          uint32_t lo[32], hi[32];
+          ptx::tmem_ld32(tmem + lane_addr + TM_DK + q2 * 32, lo);
+          ptx::tmem_ld32(tmem + lane_addr + TM_DK + 64 + q2 * 32, hi);
+          ptx::tmem_ld_wait();
+          ptx::reg_fence(lo);
+          ptx::reg_fence(hi);
+          if (kvalid) {
+            float rc[32], rs[32];
+            rope_row<32>(a.rope_cos + (int64_t)key * 64 + 32 * q2, a.rope_sin + (int64_t)key * 64 + 32 * q2, rc, rs);
+            rope_back_store<32>(lo, hi, a.scale, rc, rs, reinterpret_cast<uint4*>(dkp + q2 * 32),
+                                reinterpret_cast<uint4*>(dkp + 64 + q2 * 32));
+          }
+        }
+        ptx::tc_fence_before();
+        continue;
+      }
+      // warpgroup 0 writes dV, warpgroup 1 writes dK (scaled)
+#pragma unroll 1
+      for (int q4 = 0; q4 < 4; ++q4) {
+        if (wg == 0)
+          store32(TM_DV + 32 * q4, 1.f, dvp + 32 * q4);
+        else
+          store32(TM_DK + 32 * q4, a.scale, dkp + 32 * q4);
       }
       ptx::tc_fence_before();
     }

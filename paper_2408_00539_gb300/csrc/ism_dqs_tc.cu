@@ -160,15 +160,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = threadIdx.x;
     const uint32_t lane_addr = (uint32_t)(warp * 32) << 16;
     uint32_t local = 0;
+    // rotary encoding: the cosines and sines of the row's 64 pairs are loaded
+    // one item ahead (at the end of the previous epilogue).  A table load
+    // waited for inside the epilogue costs microseconds while the dS stream
+    // keeps the memory system saturated, and the epilogues of the short
+    // items at the end of the walk set the pace.
+    float nc[64], ns[64];
+    auto first_tables = [&](int64_t item) {
+      if (item >= n_items) return;
+      const Item y = decode(a, item);
+      const int row = y.t * kRows + r;
+      if (row < y.w.q_len) rope_row<64>(a.rope_cos + (int64_t)row * 64, a.rope_sin + (int64_t)row * 64, nc, ns);
+    };
+    if (a.rope_cos) first_tables(blockIdx.x);
     for (int64_t item = blockIdx.x; item < n_items; item += gridDim.x, ++local) {
       const Item x = decode(a, item);
       const uint32_t b = local & 1, acc = tmem + lane_addr + 128u * b;
       const int row = x.t * kRows + r;
       const bool valid = row < x.w.q_len;
-      // rotary encoding: the cosines and sines of the row's first 32 pairs,
-      // loaded while the accumulator is still being computed
-      float rc[32], rs[32];
-      if (a.rope_cos && valid) rope_row32(a.rope_cos + (int64_t)row * 64, a.rope_sin + (int64_t)row * 64, rc, rs);
       if (!wait(&bar->acc_full[b], (local >> 1) & 1, a.status) || aborted(&bar->abort)) {
         set_abort(&bar->abort);
         break;
@@ -178,7 +187,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                             ((int64_t)x.w.q_base + row) * a.hq * kD + x.h * kD);
       if (a.rope_cos) {
         // rotary encoding: columns k and k + 64 of the row pair up
-#pragma unroll 1
+#pragma unroll
         for (int q2 = 0; q2 < 2; ++q2) {
           uint32_t lo[32], hi[32];
           if (x.nkb > 0) {
@@ -191,13 +200,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int k = 0; k < 32; ++k) lo[k] = hi[k] = 0u;
           }
-          if (valid) {
-            if (q2 == 1) rope_row32(a.rope_cos + (int64_t)row * 64 + 32, a.rope_sin + (int64_t)row * 64 + 32, rc, rs);
-            rope_back_store32(lo, hi, a.scale, rc, rs, dst + 4 * q2, dst + 8 + 4 * q2);
-          }
+          if (valid) rope_back_store<32>(lo, hi, a.scale, nc + 32 * q2, ns + 32 * q2, dst + 4 * q2, dst + 8 + 4 * q2);
         }
         ptx::tc_fence_before();
         ptx::mbar_arrive(&bar->acc_empty[b]);
+        first_tables(item + gridDim.x);
         continue;
       }
 #pragma unroll 1

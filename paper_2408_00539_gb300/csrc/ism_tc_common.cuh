@@ -109,29 +109,34 @@ __device__ __forceinline__ uint32_t pack_e4m3x4(float x0, float x1, float x2, fl
 }
 
 // Gradient store of a rotary-encoded head row (the rotation of the one-pass
-// path pairs column k with k + 64).  rope_row32 loads the cosines and sines
-// of 32 pairs of a row's position (all loads issued before any use, so their
-// latency is paid once).  rope_back_store32: lo holds columns k0..k0+31 and
-// hi columns k0+64..k0+95 of the gradient of the ROTATED row (fp32 bit
-// patterns); after scaling by f, each pair (g_k, g_{k+64}) goes back through
-// the transposed rotation, x_k = g_k c + g_{k+64} s and
+// path pairs column k with k + 64).  rope_row<N> loads the cosines and sines
+// of N pairs of a row's position (all loads issued before any use, so their
+// latency is paid once; callers issue them well before the values are
+// needed).  rope_back_store<N>: lo holds columns k0..k0+N-1 and hi columns
+// k0+64..k0+63+N of the gradient of the ROTATED row (fp32 bit patterns);
+// after scaling by f, each pair (g_k, g_{k+64}) goes back through the
+// transposed rotation, x_k = g_k c + g_{k+64} s and
 // x_{k+64} = g_{k+64} c - g_k s, and the bf16 results are stored at dst_lo
-// (columns k0..) and dst_hi (columns k0+64..).
-__device__ __forceinline__ void rope_row32(const float* __restrict__ cs, const float* __restrict__ sn,
-                                           float (&c)[32], float (&s)[32]) {
+// (columns k0..) and dst_hi (columns k0+64..).  c and s point into register
+// arrays at offsets fixed at compile time (the loops are unrolled).
+template <int N>
+__device__ __forceinline__ void rope_row(const float* __restrict__ cs, const float* __restrict__ sn, float* c,
+                                         float* s) {
+  static_assert(N % 4 == 0, "whole float4 loads");
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
+  for (int i = 0; i < N / 4; ++i) {
     const float4 cv = __ldg(reinterpret_cast<const float4*>(cs) + i);
     const float4 sv = __ldg(reinterpret_cast<const float4*>(sn) + i);
     c[4 * i] = cv.x; c[4 * i + 1] = cv.y; c[4 * i + 2] = cv.z; c[4 * i + 3] = cv.w;
     s[4 * i] = sv.x; s[4 * i + 1] = sv.y; s[4 * i + 2] = sv.z; s[4 * i + 3] = sv.w;
   }
 }
-__device__ __forceinline__ void rope_back_store32(const uint32_t (&lo)[32], const uint32_t (&hi)[32], float f,
-                                                  const float (&c)[32], const float (&s)[32], uint4* dst_lo,
-                                                  uint4* dst_hi) {
+template <int N>
+__device__ __forceinline__ void rope_back_store(const uint32_t* lo, const uint32_t* hi, float f, const float* c,
+                                                const float* s, uint4* dst_lo, uint4* dst_hi) {
+  static_assert(N % 8 == 0, "whole 16-byte stores");
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
+  for (int i = 0; i < N / 8; ++i) {
     float xl[8], xh[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
