@@ -10,7 +10,9 @@
 // tiles of 128 keys.  A persistent CTA per SM walks the items; per item
 //   pass 1: S^T_t = K_t Q^T for every tile t (M = 128 keys, N = 16 query
 //           heads of the group, zero or foreign rows past the group), all
-//           tiles kept in tensor memory (16 columns each);
+//           tiles kept in tensor memory (16 columns each); the softmax
+//           warps fold each ring tile's scores into a running maximum as
+//           soon as its MMAs complete, while the next K tiles stream in;
 //   the exact maximum per head over the item's keys;
 //   pass 2: P_t = exp2(S_t * scale * log2 e - m) as bf16 into a 128-byte
 //           swizzled K-major operand in shared memory (rows = heads), then
@@ -64,7 +66,10 @@ struct DecCfg {
 struct Bars {
   uint64_t full[kMaxStages], empty[kMaxStages];
   uint64_t q_full[2], q_empty[2];
-  uint64_t s_full, s_free, p_ready[2], p_free[2], o_full, o_free, final_mma;
+  // S of ring tile n complete (s_tile[n % 4]) / read by the softmax warps (s_seen[n % 4]); the
+  // MMA warp runs at most four ring tiles ahead, so a phase parity is never ambiguous
+  uint64_t s_tile[4], s_seen[4];
+  uint64_t s_free, p_ready[2], p_free[2], o_full, o_free, final_mma;
   uint64_t red_m_full, red_l_full;  // the four softmax warps' partial maxima / sums are written
   uint32_t tmem_base;
   int32_t abort;
@@ -137,7 +142,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::mbar_init(&bar->p_ready[i], 128);
       ptx::mbar_init(&bar->p_free[i], 1);
     }
-    ptx::mbar_init(&bar->s_full, 1);
+    for (int i = 0; i < 4; ++i) {
+      ptx::mbar_init(&bar->s_tile[i], 1);
+      ptx::mbar_init(&bar->s_seen[i], 128);
+    }
     ptx::mbar_init(&bar->s_free, 128);
     ptx::mbar_init(&bar->o_full, 1);
     ptx::mbar_init(&bar->o_free, 32);
@@ -235,7 +243,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr uint32_t idesc_s =
         kE4M3 ? ptx::idesc_e4m3_f32(128, kHeadsPad, 0, 0) : ptx::idesc_bf16_f32(128, kHeadsPad, 0, 0);
     constexpr uint32_t idesc_pv = kE4M3 ? ptx::idesc_e4m3_f32(128, 128, 0, 1) : ptx::idesc_bf16_f32(128, 128, 0, 1);
-    uint32_t nl = 0, nu = 0, T = 0;  // ring tiles consumed; non-empty items; P tiles
+    uint32_t nl = 0, nu = 0, T = 0, TS = 0;  // ring tiles consumed; non-empty items; P tiles; S tiles
     bool ok = true;
     for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
       const DecItem x = dec_item<Cfg::kSub>(a, item);
@@ -256,6 +264,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = false;
           break;
         }
+        // the softmax warps have read S of the ring tile four back (its barrier is reused)
+        if (TS >= 4 && !wait_warp(&bar->s_seen[TS & 3], ((TS >> 2) - 1) & 1, a.status)) {
+          ok = false;
+          break;
+        }
         ptx::tc_fence_after();
         const uint32_t sK = ptx::smem_u32(smem + OFF_RING + s * kTile);
         if constexpr (kE4M3) {  // 128-byte rows: four k-steps of 32 bytes in one box, per 128-key sub-tile
@@ -268,9 +281,10 @@ __global__ void __launch_bounds__(kThreads, 1)
               tmem + TM_S + kHeadsPad * (uint32_t)t, desc_kmajor(sK, 0), desc_kmajor(sQ, 0), idesc_s, 0u);
         }
         ptx::mma_commit_warp(&bar->empty[s]);
+        ptx::mma_commit_warp(&bar->s_tile[TS & 3]);
+        ++TS;
       }
       if (!ok) break;
-      ptx::mma_commit_warp(&bar->s_full);
       ptx::mma_commit_warp(&bar->q_empty[qb]);
       // the epilogue has read the previous item's O
       if (nu >= 1 && !wait_warp(&bar->o_free, (nu - 1) & 1, a.status)) {
@@ -317,7 +331,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const float c2 = a.scale * kLog2e * (kE4M3 ? a.qk_descale : 1.f);
     const float o_scale = kE4M3 ? a.v_descale : 1.f;
     const int group = a.group;
-    uint32_t nu = 0, T = 0;
+    uint32_t nu = 0, T = 0, TS = 0;
     bool ok = true;
     for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
       const DecItem x = dec_item<Cfg::kSub>(a, item);
@@ -330,25 +344,33 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         continue;
       }
-      if (!wait(&bar->s_full, nu & 1, a.status)) {
-        ok = false;
-        break;
-      }
-      ptx::tc_fence_after();
-      // pass 1: maximum of the scaled scores per head over the item's keys
+      // pass 1: maximum of the scaled scores per head over the item's keys,
+      // ring tile by ring tile as the score MMAs complete
       float mx[kHeadsPad];
 #pragma unroll
       for (int h = 0; h < kHeadsPad; ++h) mx[h] = -INFINITY;
-      for (int j = 0; j < x.nsub; ++j) {
-        uint32_t v[kHeadsPad];
-        ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)j, v);
-        ptx::tmem_ld_wait();
-        ptx::reg_fence(v);
-        if (x.k0 + j * 128 + r < x.k1) {
-#pragma unroll
-          for (int h = 0; h < kHeadsPad; ++h) mx[h] = fmaxf(mx[h], __uint_as_float(v[h]));
+      for (int t = 0; t < x.nt; ++t, ++TS) {
+        if (!wait(&bar->s_tile[TS & 3], (TS >> 2) & 1, a.status)) {
+          ok = false;
+          break;
         }
+        ptx::tc_fence_after();
+        const int nh = min(kSub, x.nsub - t * kSub);
+        for (int hh = 0; hh < nh; ++hh) {
+          const int j = t * kSub + hh;
+          uint32_t v[kHeadsPad];
+          ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)j, v);
+          ptx::tmem_ld_wait();
+          ptx::reg_fence(v);
+          if (x.k0 + j * 128 + r < x.k1) {
+#pragma unroll
+            for (int h = 0; h < kHeadsPad; ++h) mx[h] = fmaxf(mx[h], __uint_as_float(v[h]));
+          }
+        }
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(&bar->s_seen[TS & 3]);
       }
+      if (!ok) break;
 #pragma unroll
       for (int h = 0; h < kHeadsPad; ++h) {
 #pragma unroll
