@@ -58,7 +58,7 @@ struct DecCfg {
   static constexpr uint32_t kQBytes = kE4M3 ? kQHalf : 2 * kQHalf;
   static constexpr uint32_t OFF_RING = 0, OFF_P = kStages * kTile, OFF_Q = OFF_P + 2 * kTile,
                             OFF_BAR = OFF_Q + 2 * kQBytes;
-  static constexpr uint32_t kSmemBytes = OFF_BAR + 1024 + 1024;  // barrier block + 1024-byte alignment slack
+  static constexpr uint32_t kSmemBytes = OFF_BAR + 2048 + 1024;  // barrier block + 1024-byte alignment slack
   static_assert(kStages <= kMaxStages, "ring");
   static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 };
@@ -73,9 +73,11 @@ struct Bars {
   uint64_t red_m_full, red_l_full;  // the four softmax warps' partial maxima / sums are written
   uint32_t tmem_base;
   int32_t abort;
-  float red_m[4][kHeadsPad], red_l[4][kHeadsPad];
+  // per item parity: warp 0's epilogue of item u reads them while the other
+  // warps may already fold the scores of item u + 1
+  float red_m[2][4][kHeadsPad], red_l[2][4][kHeadsPad];
 };
-static_assert(sizeof(Bars) <= 1024, "barrier block");
+static_assert(sizeof(Bars) <= 2048, "barrier block");
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
@@ -378,7 +380,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (lane == 0) {
 #pragma unroll
-        for (int h = 0; h < kHeadsPad; ++h) bar->red_m[warp][h] = mx[h];
+        for (int h = 0; h < kHeadsPad; ++h) bar->red_m[nu & 1][warp][h] = mx[h];
       }
       ptx::mbar_arrive(&bar->red_m_full);
       if (!wait(&bar->red_m_full, nu & 1, a.status)) {
@@ -388,7 +390,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       float m2[kHeadsPad];  // max of scale * log2(e) * S per head (finite: every item has a key)
 #pragma unroll
       for (int h = 0; h < kHeadsPad; ++h)
-        m2[h] = fmaxf(fmaxf(bar->red_m[0][h], bar->red_m[1][h]), fmaxf(bar->red_m[2][h], bar->red_m[3][h])) * c2;
+        m2[h] = fmaxf(fmaxf(bar->red_m[nu & 1][0][h], bar->red_m[nu & 1][1][h]),
+                      fmaxf(bar->red_m[nu & 1][2][h], bar->red_m[nu & 1][3][h])) *
+                c2;
       // pass 2: P as bf16 into the A operand of O += P V (rows = heads, columns = keys)
       float l[kHeadsPad];
 #pragma unroll
@@ -451,7 +455,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (lane == 0) {
 #pragma unroll
-        for (int h = 0; h < kHeadsPad; ++h) bar->red_l[warp][h] = l[h];
+        for (int h = 0; h < kHeadsPad; ++h) bar->red_l[nu & 1][warp][h] = l[h];
       }
       ptx::mbar_arrive(&bar->red_l_full);
       if (!wait(&bar->red_l_full, nu & 1, a.status)) {
@@ -485,8 +489,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           float mh = -INFINITY, lh = 0.f;
 #pragma unroll
           for (int w = 0; w < 4; ++w) {
-            mh = fmaxf(mh, bar->red_m[w][lane]);
-            lh += bar->red_l[w][lane];
+            mh = fmaxf(mh, bar->red_m[nu & 1][w][lane]);
+            lh += bar->red_l[nu & 1][w][lane];
           }
           a.part_ml[(pbase + (int64_t)lane * a.splits) * 2] = mh * c2;
           a.part_ml[(pbase + (int64_t)lane * a.splits) * 2 + 1] = lh;
