@@ -545,19 +545,22 @@ def run_cuda(args, w):
         "clocks": clocks.summary(),
     }
     if not args.no_extra:
-        line["sustained"] = measure_sustained(dev, step, flops, peaks)
-        del ins, outs, ob, lb
-        torch.cuda.empty_cache()
         line["bwd_min_workspace"] = measure_training_config(dev, w, peaks, steps=args.steps, minimal_workspace=True)
         line["rope"] = measure_training_config(dev, w, peaks, steps=args.steps, rope=True)
         line["configs"] = {wname: measure_training_config(dev, WORKLOADS[wname](), peaks, steps=args.steps)
                            for wname in ("mha_4k", "packed_32k") if WORKLOADS[wname]().name != w.name}
-        line["long_context"] = measure_long_context(dev, peaks)
     if not args.no_append:
         line["append"] = measure_append(dev, read_peaks()[0])
         line["session"] = measure_session(dev)
         line["training_cost"] = measure_training_cost(dev, w)
         line["fwd_e4m3"] = measure_fwd_e4m3(dev, w, read_peaks()[0])
+    if not args.no_extra:
+        # the seconds-long runs come last: the power-capped clocks they leave
+        # behind would slow the short measurements taken right after them
+        line["sustained"] = measure_sustained(dev, step, flops, peaks)
+        del ins, outs, ob, lb
+        torch.cuda.empty_cache()
+        line["long_context"] = measure_long_context(dev, peaks)
     if world == 1 and not args.no_cpu_baseline:
         val, dt, sample = oracle_sample(w, q, k, v, do, heads_per_sample=4)
         line["cpu_baseline"] = {"value": val, "unit": "TFLOP/s", "cores": cpu_cores(), "kind": "oracle",
