@@ -15,9 +15,11 @@
 //           soon as its MMAs complete, while the next K tiles stream in;
 //   the exact maximum per head over the item's keys;
 //   pass 2: P_t = exp2(S_t * scale * log2 e - m) as bf16 into a 128-byte
-//           swizzled K-major operand in shared memory (rows = heads), then
-//           O += P_t V_t (M = 128 with the group in rows 0-15, N = 128
-//           dimensions, K = 128 keys; V MN-major as it arrives).
+//           swizzled MN-major operand in shared memory (rows = keys, the
+//           heads contiguous: a thread stores its key's 16 heads as whole
+//           16-byte chunks), then O += P_t V_t (M = 128 with the group in
+//           rows 0-15, N = 128 dimensions, K = 128 keys; V MN-major as it
+//           arrives).
 // With the exact maximum known before any P, no rescaling of O is needed.
 // The item's (max, sum, unnormalised O) per head go to the split partials,
 // which decode_combine_kernel merges as for the CUDA-core kernels.
@@ -110,15 +112,12 @@ __device__ __forceinline__ DecItem dec_item(const DecodeArgs& a, int64_t item) {
   return x;
 }
 
-// Element (row h, key k) of the P operand (rows = heads, 128 keys), in the
-// layout a 128-byte swizzled TMA box produces: bf16 two 64-key halves, e4m3 one.
-template <bool kE4M3>
-__device__ __forceinline__ uint32_t p_offset(uint32_t h, uint32_t k) {
-  if constexpr (kE4M3)
-    return h * 128u + (((k >> 4) ^ (h & 7u)) << 4) + (k & 15u);
-  else
-    return swz_offset(h, k);
-}
+// The P operand is stored MN-major (128-byte swizzled rows = keys, the heads
+// contiguous along a row, as the V tile stores dimensions): the thread of key
+// k writes its 16 heads as whole 16-byte chunks (bf16: chunks 0 and 1 of the
+// row, e4m3: chunk 0), swizzled by k & 7.  Heads past 16 (M up to 128) are
+// never written; they only feed output rows that are not read.
+__device__ __forceinline__ uint32_t p_chunk(uint32_t k, uint32_t c) { return k * 128u + ((c ^ (k & 7u)) << 4); }
 
 template <bool kE4M3>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -244,7 +243,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // one elected lane issues each instruction)
     constexpr uint32_t idesc_s =
         kE4M3 ? ptx::idesc_e4m3_f32(128, kHeadsPad, 0, 0) : ptx::idesc_bf16_f32(128, kHeadsPad, 0, 0);
-    constexpr uint32_t idesc_pv = kE4M3 ? ptx::idesc_e4m3_f32(128, 128, 0, 1) : ptx::idesc_bf16_f32(128, 128, 0, 1);
+    constexpr uint32_t idesc_pv = kE4M3 ? ptx::idesc_e4m3_f32(128, 128, 1, 1) : ptx::idesc_bf16_f32(128, 128, 1, 1);
     uint32_t nl = 0, nu = 0, T = 0, TS = 0;  // ring tiles consumed; non-empty items; P tiles; S tiles
     bool ok = true;
     for (int64_t item = blockIdx.x; ok && item < n_items; item += gridDim.x) {
@@ -308,12 +307,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         if constexpr (kE4M3) {  // V MN-major: 32 keys of 128 bytes a k-step, per 128-key sub-tile
           const int nh = min(kSub, x.nsub - t * kSub);
           for (int hh = 0; hh < nh; ++hh)
-            ptx::mma4_e4m3_ss_warp<2, 256>(tmem + TM_O, desc_kmajor(sP + hh * kSubBytes, 0),
+            ptx::mma4_e4m3_ss_warp<256, 256>(tmem + TM_O, desc_kmajor(sP + hh * kSubBytes, 0),
                                            desc_kmajor(sV + hh * kSubBytes, 0), idesc_pv,
                                            (t > 0 || hh > 0) ? 1u : 0u);
         } else
-          ptx::mma8_bf16_ss_warp<ptx::KMajorSw128, ptx::MnMajorSw128>(tmem + TM_O, desc_kmajor(sP, 0),
-                                                                     desc_mnmajor(sV, 0), idesc_pv, t > 0 ? 1u : 0u);
+          ptx::mma8_bf16_ss_warp<ptx::MnMajorSw128, ptx::MnMajorSw128>(tmem + TM_O, desc_mnmajor(sP, 0),
+                                                                      desc_mnmajor(sV, 0), idesc_pv, t > 0 ? 1u : 0u);
         ptx::mma_commit_warp(&bar->empty[s]);
         ptx::mma_commit_warp(&bar->p_free[pb]);
       }
@@ -413,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ptx::tmem_ld_wait();
             ptx::reg_fence(v);
             const bool valid = x.k0 + j * 128 + r < x.k1;
-            uint8_t* Ph = P + hh * kSubBytes;
+            uint32_t b4[4];
 #pragma unroll
             for (int h = 0; h < kHeadsPad; h += 4) {
               float p4[4];
@@ -422,11 +421,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 p4[e] = (valid && h + e < group) ? ex2(__uint_as_float(v[h + e]) * c2 - m2[h + e]) : 0.f;
                 l[h + e] += p4[e];
               }
-              const uint32_t b4 = pack_e4m3x4(p4[0], p4[1], p4[2], p4[3]);
-#pragma unroll
-              for (int e = 0; e < 4; ++e)
-                Ph[p_offset<true>((uint32_t)(h + e), (uint32_t)r)] = (uint8_t)(b4 >> (8 * e));
+              b4[h >> 2] = pack_e4m3x4(p4[0], p4[1], p4[2], p4[3]);
             }
+            *reinterpret_cast<uint4*>(P + hh * kSubBytes + p_chunk((uint32_t)r, 0u)) =
+                make_uint4(b4[0], b4[1], b4[2], b4[3]);
           }
         } else {
           uint32_t v[kHeadsPad];
@@ -434,13 +432,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           ptx::tmem_ld_wait();
           ptx::reg_fence(v);
           const bool valid = x.k0 + t * 128 + r < x.k1;
+          uint32_t pk[kHeadsPad / 2];
 #pragma unroll
-          for (int h = 0; h < kHeadsPad; ++h) {
-            const float p = (valid && h < group) ? ex2(__uint_as_float(v[h]) * c2 - m2[h]) : 0.f;
-            const __nv_bfloat16 pr = __float2bfloat16_rn(p);
-            l[h] += __bfloat162float(pr);  // the sum of the P that enters P V
-            *reinterpret_cast<__nv_bfloat16*>(P + p_offset<false>((uint32_t)h, (uint32_t)r)) = pr;
+          for (int h = 0; h < kHeadsPad; h += 2) {
+            const float p0 = (valid && h < group) ? ex2(__uint_as_float(v[h]) * c2 - m2[h]) : 0.f;
+            const float p1 = (valid && h + 1 < group) ? ex2(__uint_as_float(v[h + 1]) * c2 - m2[h + 1]) : 0.f;
+            pk[h >> 1] = pack_bf16(p0, p1);
+            l[h] += __uint_as_float(pk[h >> 1] << 16);  // the sum of the P that enters P V
+            l[h + 1] += __uint_as_float(pk[h >> 1] & 0xFFFF0000u);
           }
+          *reinterpret_cast<uint4*>(P + p_chunk((uint32_t)r, 0u)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          *reinterpret_cast<uint4*>(P + p_chunk((uint32_t)r, 1u)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
         }
         ptx::fence_proxy_async_smem();
         ptx::mbar_arrive(&bar->p_ready[pb]);
