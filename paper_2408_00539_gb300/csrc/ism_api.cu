@@ -207,6 +207,7 @@ struct PassLayout {
   int32_t* kpair_off;
   void* ds;
   int32_t* pair_order;
+  int32_t* kp_order;  // k-tile pairs in cost order (backward only)
   int32_t* counters;  // work counters of the persistent backward kernels (backward only)
   size_t bytes;
 };
@@ -225,6 +226,7 @@ PassLayout pass_layout(void* ws, const ism_segments_t* s, const Counts& c, int64
   L.kpair_off = ds_slots > 0 ? cv.take<int32_t>(c.nk) : nullptr;
   L.ds = ds_slots > 0 ? static_cast<void*>(cv.take<uint16_t>(ds_slots * kTile * kTile)) : nullptr;
   L.pair_order = tile_pairs ? cv.take<int32_t>(c.npairs) : nullptr;
+  L.kp_order = bwd ? cv.take<int32_t>(c.npairs) : nullptr;  // k-tile pairs number as q-tile pairs here
   L.counters = bwd ? cv.take<int32_t>(kPassCounters) : nullptr;
   L.bytes = ((cv.off + 255) & ~size_t(255)) + 256;
   return L;
@@ -273,7 +275,7 @@ ism_status_t build_pass_meta(const ism_segments_t* s, const Counts& c, const Pas
   timer_begin(ISM_KERNEL_META, st);
   ISM_TRY_CUDA(launch_pass_meta(d, L.kv_end, kTile, kTile, c.nq, bwd ? c.nk : 0, L.qtiles, bwd ? L.ktiles : nullptr,
                                 c.max_cost, L.q_order, bwd ? L.k_order : nullptr, L.pair_order, L.kpair_off,
-                                L.counters, L.counters ? kPassCounters : 0, st),
+                                L.counters, L.counters ? kPassCounters : 0, st, L.kp_order),
                "metadata launch");
   timer_end(ISM_KERNEL_META, st);
   count_launch(1);
@@ -313,6 +315,7 @@ Knobs read_knobs() {
   const int64_t g1 = env_int("ISM_DKDV_GRID", 0), g2 = env_int("ISM_DQ_GRID", 0);
   k.dkdv_grid = g1 > 0 && g1 < (1 << 20) ? (int32_t)g1 : 0;
   k.dq_grid = g2 > 0 && g2 < (1 << 20) ? (int32_t)g2 : 0;
+  k.dkdv_pair = env_on("ISM_DKDV_PAIR");
   return k;
 }
 Knobs g_knobs = read_knobs();  // read when the library is loaded
@@ -596,6 +599,7 @@ ism_status_t bwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape,
   a.ktiles = L.ktiles; a.k_order = L.k_order; a.nk = c.nk;
   a.ds = L.ds; a.kpair_off = L.kpair_off; a.ds_slots = L.ds ? slots : 0;
   a.work_counter = L.counters;
+  a.kp_order = L.kp_order; a.nkp = L.kp_order ? c.npairs : 0;
   a.status = status;
   a.flags = tc_flags();
   if (use_tc_bwd(shape)) {

@@ -957,6 +957,8 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
 
 }  // namespace
 
+cudaError_t launch_dkdv_pair(const AttnArgs& a, const CUtensorMap& tk, const CUtensorMap& tv, cudaStream_t st);
+
 cudaError_t launch_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) {
   cudaError_t e;
   if (a.q_rows > 0) {
@@ -987,7 +989,13 @@ cudaError_t launch_bwd(const AttnArgs& a, int64_t k_rows, cudaStream_t st) {
     count_launch();
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
-  if (a.nk) {
+  if (a.nk && knobs().dkdv_pair && a.kp_order) {
+    // the CTA-pair kernel (ism_dkdv2_tc.cu)
+    timer_begin(ISM_KERNEL_BWD_DKDV, st);
+    if ((e = launch_dkdv_pair(a, tk, tv, st)) != cudaSuccess) return e;
+    timer_end(ISM_KERNEL_BWD_DKDV, st);
+    count_launch();
+  } else if (a.nk) {
     if ((e = cudaFuncSetAttribute(dkdv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   (int)dkv::kSmemBytes)) != cudaSuccess)
       return e;

@@ -82,11 +82,12 @@ cudaError_t launch_tiles(const SegsDev& s, int bm, int bn, const int32_t* kv_end
 cudaError_t launch_order(const Tile* qtiles, int64_t nq, const Tile* ktiles, int64_t nk, int max_cost,
                          int32_t* q_order, int32_t* k_order, cudaStream_t st, int32_t* pair_order = nullptr);
 cudaError_t launch_pair_offsets(const Tile* ktiles, int64_t nk, int32_t* kpair_off, cudaStream_t st);
-// kv_end, tiles, work lists (and pair offsets when kpair_off is set) in one launch.
+// kv_end, tiles, work lists (and pair offsets when kpair_off is set, the
+// k-tile pair list when kp_order is set) in one launch.
 cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, int64_t nq, int64_t nk,
                              Tile* qtiles, Tile* ktiles, int max_cost, int32_t* q_order, int32_t* k_order,
                              int32_t* pair_order, int32_t* kpair_off, int32_t* counters, int n_counters,
-                             cudaStream_t st);
+                             cudaStream_t st, int32_t* kp_order = nullptr);
 // k_base of sequence b's tiles = b * kbase_stride (the cache capacity, or 1 for a paged cache)
 cudaError_t launch_append_plan(const AppendSegs& segs, int batch, int64_t kbase_stride, int bm, int bn,
                                int32_t* cache_len, int32_t* c_snap, int32_t* kv_end, Tile* qtiles,
@@ -142,6 +143,10 @@ struct AttnArgs {
   int64_t npairs;
   // Work counter of the persistent dK/dV kernel (zeroed by the metadata pass).
   int32_t* work_counter;
+  // dK/dV on CTA pairs: kp_order lists the even-indexed k-tiles (each with the
+  // next k-tile of its sequence, when there is one) in cost order; nkp of them.
+  const int32_t* kp_order;
+  int64_t nkp;
   // Paged K/V (forward over an appended chunk only): Tile::k_base holds the
   // sequence index and key p's row is paged_row(pages, k_base, p).
   KvPages pages;
@@ -224,6 +229,7 @@ struct Knobs {
   int64_t prefill_split;   // ISM_PREFILL_SPLIT=n: n key-range split items in a prefill (-1: chosen by the library)
   int32_t dkdv_grid;       // ISM_DKDV_GRID=n: CTAs of the persistent dK/dV kernel (0: one per SM)
   int32_t dq_grid;         // ISM_DQ_GRID=n: CTAs of the persistent dQ kernel (0: one per SM)
+  bool dkdv_pair;          // ISM_DKDV_PAIR=1: dK/dV on CTA pairs (cta_group::2)
 };
 const Knobs& knobs();
 void reload_knobs();

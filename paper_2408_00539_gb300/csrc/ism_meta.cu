@@ -144,7 +144,10 @@ __global__ void __launch_bounds__(256) tiles_kernel(SegsDev s, int bm, int bn, c
 // a q-tile = its non-empty k-tiles; of a k-tile = its non-empty q-tiles.  The
 // optional third list holds the q-tiles with an even index in their sequence
 // (the first of each pair of neighbouring q-tiles), costed by the pair's
-// larger count (the second tile's, kv_end being non-decreasing).
+// larger count (the second tile's, kv_end being non-decreasing); the optional
+// fourth the k-tiles with an even index (pairs of neighbouring k-tiles),
+// costed by the first tile's count, which covers the second's (its first
+// non-empty q-tile comes no earlier).
 // Items of equal cost come in arbitrary order; results do not depend on it.
 __device__ __forceinline__ bool pair_head(const Tile* qtiles, int64_t nq, int64_t i, int* cost) {
   const Tile w = qtiles[i];
@@ -159,11 +162,12 @@ __device__ __forceinline__ bool pair_head(const Tile* qtiles, int64_t nq, int64_
 }
 
 __device__ void order_body(const Tile* __restrict__ qtiles, int64_t nq, const Tile* __restrict__ ktiles, int64_t nk,
-                           int max_cost, int32_t* q_order, int32_t* k_order, int32_t* pair_order, int32_t* hist) {
-  for (int pass = 0; pass < 3; ++pass) {
-    const Tile* items = pass == 1 ? ktiles : qtiles;
-    int64_t n = pass == 1 ? nk : nq;
-    int32_t* order = pass == 0 ? q_order : pass == 1 ? k_order : pair_order;
+                           int max_cost, int32_t* q_order, int32_t* k_order, int32_t* pair_order, int32_t* hist,
+                           int32_t* kp_order = nullptr) {
+  for (int pass = 0; pass < 4; ++pass) {
+    const Tile* items = pass == 1 || pass == 3 ? ktiles : qtiles;
+    int64_t n = pass == 1 || pass == 3 ? nk : nq;
+    int32_t* order = pass == 0 ? q_order : pass == 1 ? k_order : pass == 2 ? pair_order : kp_order;
     if (items == nullptr || order == nullptr || n == 0) continue;
     for (int i = threadIdx.x; i <= max_cost; i += blockDim.x) hist[i] = 0;
     __syncthreads();
@@ -173,6 +177,7 @@ __device__ void order_body(const Tile* __restrict__ qtiles, int64_t nq, const Ti
         if (!pair_head(items, n, i, &cost)) continue;
       } else {
         const Tile w = items[i];
+        if (pass == 3 && (w.tile & 1)) continue;  // k-tile pairs: the even tile, costed by its query tiles
         cost = pass == 0 ? w.a1 : w.a1 - w.a0;
       }
       cost = min(max(cost, 0), max_cost);
@@ -190,6 +195,7 @@ __device__ void order_body(const Tile* __restrict__ qtiles, int64_t nq, const Ti
         if (!pair_head(items, n, i, &cost)) continue;
       } else {
         const Tile w = items[i];
+        if (pass == 3 && (w.tile & 1)) continue;  // k-tile pairs: the even tile, costed by its query tiles
         cost = pass == 0 ? w.a1 : w.a1 - w.a0;
       }
       cost = min(max(cost, 0), max_cost);
@@ -246,7 +252,7 @@ __global__ void pair_offsets_kernel(const Tile* __restrict__ ktiles, int64_t nk,
 __global__ void __launch_bounds__(1024)
     pass_meta_kernel(SegsDev s, int32_t* kv_end, int bm, int bn, int64_t nq, int64_t nk, Tile* qtiles,
                      Tile* ktiles, int max_cost, int32_t* q_order, int32_t* k_order, int32_t* pair_order,
-                     int32_t* kpair_off, int32_t* counters, int n_counters) {
+                     int32_t* kpair_off, int32_t* counters, int n_counters, int32_t* kp_order) {
   extern __shared__ __align__(16) unsigned char dyn[];
   if ((int)threadIdx.x < n_counters) counters[threadIdx.x] = 0;  // work counters of the kernels that follow
   // kv_end: one warp per segment, lanes over its tokens
@@ -262,7 +268,8 @@ __global__ void __launch_bounds__(1024)
   __syncthreads();
   tiles_body(s, bm, bn, kv_end, nq, nk, qtiles, ktiles, nullptr, nullptr, nullptr, nullptr, dyn);
   __syncthreads();
-  order_body(qtiles, nq, ktiles, nk, max_cost, q_order, k_order, pair_order, reinterpret_cast<int32_t*>(dyn));
+  order_body(qtiles, nq, ktiles, nk, max_cost, q_order, k_order, pair_order, reinterpret_cast<int32_t*>(dyn),
+             kp_order);
   if (kpair_off) pair_offsets_body(ktiles, nk, kpair_off);
 }
 
@@ -533,7 +540,7 @@ cudaError_t launch_order(const Tile* qtiles, int64_t nq, const Tile* ktiles, int
 cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, int64_t nq, int64_t nk,
                              Tile* qtiles, Tile* ktiles, int max_cost, int32_t* q_order, int32_t* k_order,
                              int32_t* pair_order, int32_t* kpair_off, int32_t* counters, int n_counters,
-                             cudaStream_t st) {
+                             cudaStream_t st, int32_t* kp_order) {
   size_t a = (size_t)(s.num_seqs + 1) * (sizeof(int64_t) + 2 * sizeof(int32_t));
   size_t b = sizeof(int32_t) * (size_t)(max_cost + 1);
   size_t smem = a > b ? a : b;
@@ -542,7 +549,7 @@ cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, 
     if (e != cudaSuccess) return e;
   }
   pass_meta_kernel<<<1, 1024, smem, st>>>(s, kv_end, bm, bn, nq, nk, qtiles, ktiles, max_cost, q_order, k_order,
-                                          pair_order, kpair_off, counters, n_counters);
+                                          pair_order, kpair_off, counters, n_counters, kp_order);
   return cudaGetLastError();
 }
 

@@ -440,5 +440,130 @@ __device__ __forceinline__ void mma4_e4m3_ts_warp(uint32_t d_tmem, uint32_t a_tm
       : "memory");
 }
 
+// ---------------------------------------------------------------- CTA pairs (cluster of two)
+// The pair's MMAs (cta_group::2) are issued by the even CTA; each CTA holds
+// its half of A (rows) and of B (columns of N) at the same shared-memory
+// offsets, and its own rows of D in its own tensor memory.
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Every thread of both CTAs: arrive (release) and wait (acquire) at the cluster barrier.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Shared-memory address of `p` (a shared::cta object) in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t cluster_addr(const void* p, uint32_t rank) {
+  uint32_t a;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(p)), "r"(rank));
+  return a;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar) : "memory");
+}
+// Arrival without release semantics: for hand-offs whose data the sender has
+// already completed by other means (tensor-memory stores waited for with
+// tcgen05.wait::st), so that the arrival does not wait for the sender's
+// unrelated global stores to become visible across the cluster.
+__device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint32_t cluster_bar) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_bar) : "memory");
+}
+__device__ __forceinline__ void st_cluster_u32(uint32_t cluster_addr_, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(cluster_addr_), "r"(v) : "memory");
+}
+// Phase test with cluster-scope acquire (for barriers that CTAs of the pair arrive on).
+__device__ __forceinline__ bool mbar_test_cluster(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.test_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool mbar_test_cluster_warp(uint64_t* bar, uint32_t parity) {
+  return __all_sync(0xffffffffu, mbar_test_cluster(bar, parity));
+}
+// Tensor memory for the pair: one warp of each CTA, the same column count.
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t* dst, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(dst)), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish_pair() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+// Completion of the pair's MMAs issued so far, signalled on the barrier at
+// the same offset in both CTAs.
+__device__ __forceinline__ void mma_commit_pair_warp(uint64_t* bar) {
+  asm volatile(
+      "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
+      " @e tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n}" ::"r"(
+          smem_u32(bar)),
+      "h"((uint16_t)3)
+      : "memory");
+}
+// Eight k-steps of a pair MMA (M = 256), issued like mma8_bf16_ss_warp / _ts_warp.
+template <class LA, class LB, uint32_t kAStep = LA::step, uint32_t kAHalf = LA::half, uint32_t kBStep = LB::step,
+          uint32_t kBHalf = LB::half>
+__device__ __forceinline__ void mma8_bf16_ss_pair_warp(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
+                                                       uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred e, p, t;\n .reg .b64 a1, a2, a3, a4, a5, a6, a7, b1, b2, b3, b4, b5, b6, b7;\n"
+      " elect.sync _|e, 0xffffffff;\n @!e bra MMA8_SSP_DONE;\n"
+      " setp.ne.b32 p, %4, 0;\n setp.eq.u32 t, 0, 0;\n"
+      " add.s64 a1, %1, %5; add.s64 a2, %1, %6; add.s64 a3, %1, %7; add.s64 a4, %1, %8;\n"
+      " add.s64 a5, %1, %9; add.s64 a6, %1, %10; add.s64 a7, %1, %11;\n"
+      " add.s64 b1, %2, %12; add.s64 b2, %2, %13; add.s64 b3, %2, %14; add.s64 b4, %2, %15;\n"
+      " add.s64 b5, %2, %16; add.s64 b6, %2, %17; add.s64 b7, %2, %18;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], a1, b1, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], a2, b2, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], a3, b3, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], a4, b4, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], a5, b5, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], a6, b6, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], a7, b7, %3, t;\n"
+      " MMA8_SSP_DONE:\n}" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(acc), "n"(kAStep), "n"(2 * kAStep), "n"(3 * kAStep), "n"(kAHalf),
+      "n"(kAHalf + kAStep), "n"(kAHalf + 2 * kAStep), "n"(kAHalf + 3 * kAStep), "n"(kBStep), "n"(2 * kBStep),
+      "n"(3 * kBStep), "n"(kBHalf), "n"(kBHalf + kBStep), "n"(kBHalf + 2 * kBStep), "n"(kBHalf + 3 * kBStep)
+      : "memory");
+}
+template <class LA, class LB, uint32_t kAStep = LA::step, uint32_t kAHalf = LA::half, uint32_t kBStep = LB::step,
+          uint32_t kBHalf = LB::half>
+__device__ __forceinline__ void mma8_bf16_ts_pair_warp(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc,
+                                                       uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred e, p, t;\n .reg .b32 a1, a2, a3, a4, a5, a6, a7;\n"
+      " .reg .b64 b1, b2, b3, b4, b5, b6, b7;\n"
+      " elect.sync _|e, 0xffffffff;\n @!e bra MMA8_TSP_DONE;\n"
+      " setp.ne.b32 p, %4, 0;\n setp.eq.u32 t, 0, 0;\n"
+      " add.u32 a1, %1, %5; add.u32 a2, %1, %6; add.u32 a3, %1, %7; add.u32 a4, %1, %8;\n"
+      " add.u32 a5, %1, %9; add.u32 a6, %1, %10; add.u32 a7, %1, %11;\n"
+      " add.s64 b1, %2, %12; add.s64 b2, %2, %13; add.s64 b3, %2, %14; add.s64 b4, %2, %15;\n"
+      " add.s64 b5, %2, %16; add.s64 b6, %2, %17; add.s64 b7, %2, %18;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], [%1], %2, %3, p;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], [a1], b1, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], [a2], b2, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], [a3], b3, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], [a4], b4, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], [a5], b5, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], [a6], b6, %3, t;\n"
+      " tcgen05.mma.cta_group::2.kind::f16 [%0], [a7], b7, %3, t;\n"
+      " MMA8_TSP_DONE:\n}" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(acc), "n"(kAStep), "n"(2 * kAStep), "n"(3 * kAStep), "n"(kAHalf),
+      "n"(kAHalf + kAStep), "n"(kAHalf + 2 * kAStep), "n"(kAHalf + 3 * kAStep), "n"(kBStep), "n"(2 * kBStep),
+      "n"(3 * kBStep), "n"(kBHalf), "n"(kBHalf + kBStep), "n"(kBHalf + 2 * kBStep), "n"(kBHalf + 3 * kBStep)
+      : "memory");
+}
+// K-major, 128-byte swizzled, 64-row operand whose two 64-column halves are 8 KB apart
+struct KMajorSw128Half8K { static constexpr uint32_t step = 2, half = 512; };
+
 }  // namespace ptx
 }  // namespace ism

@@ -496,6 +496,34 @@ def test_bwd_schedules_agree(ism):
 
 
 
+def test_dkdv_pair_matches_single_cta_bit_exact(ism, knobs):
+    """dK/dV on CTA pairs (ISM_DKDV_PAIR=1: one M = 256 MMA over two
+    neighbouring key tiles, B split across the pair) runs the arithmetic of
+    the single-CTA kernel row by row in the same order; the odd CTA of a pair
+    also visits the query tiles the even tile sees before its own, where its
+    P and dS are exact zeros.  So dQ, dK and dV agree bit for bit, for both
+    backward schedules, with sequences of an odd number of key tiles (the
+    last pair has one tile) and query heads 3 per KV head."""
+    if not ism.has_tensor_cores():
+        pytest.skip("tensor-core backward only")
+    cases = [wl.gqa_8k(),
+             wl.Workload("pairs", wl.pack([([70, 150, 170, 300], [0, 1, 0, 1]), ([33, 90, 200, 517], [0, 1, 0, 1]),
+                                           ([129], [0]), ([1, 256, 257], [1, 0, 1])]),
+                         6, 2, 128, "bf16", 128 ** -0.5, 0.5, 77)]
+    for w in cases:
+        q, k, v, do = (t.to(DEV) for t in wl.attention_tensors(w))
+        segs = ism.Segments.from_workload(w.segs, DEV)
+        o, lse = ism.fwd(segs, q, k, v, w.softmax_scale)
+        for minimal in (False, True):
+            knobs("ISM_DKDV_PAIR", "0")
+            single = ism.bwd(segs, q, k, v, o, lse, do, w.softmax_scale, minimal_workspace=minimal)
+            knobs("ISM_DKDV_PAIR", "1")
+            pair = ism.bwd(segs, q, k, v, o, lse, do, w.softmax_scale, minimal_workspace=minimal)
+            ism.check_status()
+            for name, a_, b_ in zip(("dq", "dk", "dv"), pair, single):
+                assert torch.equal(a_, b_), (w.name, minimal, name)
+
+
 def test_session_turn_by_turn_matches_one_pass(ism):
     """A dialogue served turn by turn (each query appended in one call, each
     answer token decoded alone against the growing cache) gives the rows of
