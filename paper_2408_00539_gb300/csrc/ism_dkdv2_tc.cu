@@ -34,7 +34,11 @@ constexpr uint32_t kTmemCols = 512;
 
 __device__ __forceinline__ bool aborted(const int32_t* f) { return *reinterpret_cast<const volatile int32_t*>(f) != 0; }
 
-// Bounded waits with cluster-scope acquire, for barriers the other CTA arrives on.
+// Bounded waits with cluster-scope acquire: the item ring (the even CTA writes
+// the entries into this CTA's shared memory before arriving) and the final
+// completion.  The hand-off barriers carry no data the waiter reads itself
+// (the MMAs read tensor and shared memory through the async proxy), and use
+// the CTA-scope waits of the single-CTA kernel.
 __device__ __forceinline__ bool wait_c(uint64_t* bar, uint32_t parity, uint32_t* status) {
   if (ptx::mbar_test_cluster(bar, parity)) return true;
   const uint64_t t0 = globaltimer();
