@@ -275,7 +275,8 @@ ism_status_t build_pass_meta(const ism_segments_t* s, const Counts& c, const Pas
   timer_begin(ISM_KERNEL_META, st);
   ISM_TRY_CUDA(launch_pass_meta(d, L.kv_end, kTile, kTile, c.nq, bwd ? c.nk : 0, L.qtiles, bwd ? L.ktiles : nullptr,
                                 c.max_cost, L.q_order, bwd ? L.k_order : nullptr, L.pair_order, L.kpair_off,
-                                L.counters, L.counters ? kPassCounters : 0, st, L.kp_order),
+                                L.counters, L.counters ? kPassCounters : 0, st,
+                                knobs().dkdv_pair ? L.kp_order : nullptr),
                "metadata launch");
   timer_end(ISM_KERNEL_META, st);
   count_launch(1);
@@ -599,7 +600,9 @@ ism_status_t bwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape,
   a.ktiles = L.ktiles; a.k_order = L.k_order; a.nk = c.nk;
   a.ds = L.ds; a.kpair_off = L.kpair_off; a.ds_slots = L.ds ? slots : 0;
   a.work_counter = L.counters;
-  a.kp_order = L.kp_order; a.nkp = L.kp_order ? c.npairs : 0;
+  // the k-tile pair list exists only when the CTA-pair dK/dV kernel will run
+  a.kp_order = knobs().dkdv_pair ? L.kp_order : nullptr;
+  a.nkp = a.kp_order ? c.npairs : 0;
   a.status = status;
   a.flags = tc_flags();
   if (use_tc_bwd(shape)) {
