@@ -119,7 +119,20 @@ __device__ __forceinline__ DecItem dec_item(const DecodeArgs& a, int64_t item) {
 // never written; they only feed output rows that are not read.
 __device__ __forceinline__ uint32_t p_chunk(uint32_t k, uint32_t c) { return k * 128u + ((c ^ (k & 7u)) << 4); }
 
-template <bool kE4M3>
+// The scores of the first G heads of a 128-key sub-tile (thread = key).
+template <int G>
+__device__ __forceinline__ void ld_scores(uint32_t taddr, uint32_t (&v)[G]) {
+  if constexpr (G == 4)
+    ptx::tmem_ld4(taddr, v);
+  else if constexpr (G == 8)
+    ptx::tmem_ld8(taddr, v);
+  else
+    ptx::tmem_ld16(taddr, v);
+}
+
+// kG: the heads the softmax warps process (4, 8 or 16, at least the group);
+// the score MMAs always compute 16 (N = 16), the columns past kG are not read.
+template <bool kE4M3, int kG>
 __global__ void __launch_bounds__(kThreads, 1)
     decode_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
                      const __grid_constant__ CUtensorMap tmV, const DecodeArgs a, int64_t n_items) {
@@ -347,9 +360,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // pass 1: maximum of the scaled scores per head over the item's keys,
       // ring tile by ring tile as the score MMAs complete
-      float mx[kHeadsPad];
+      static_assert(kG == 4 || kG == 8 || kG == kHeadsPad, "heads per softmax pass");
+      float mx[kG];
 #pragma unroll
-      for (int h = 0; h < kHeadsPad; ++h) mx[h] = -INFINITY;
+      for (int h = 0; h < kG; ++h) mx[h] = -INFINITY;
       for (int t = 0; t < x.nt; ++t, ++TS) {
         if (!wait(&bar->s_tile[TS & 3], (TS >> 2) & 1, a.status)) {
           ok = false;
@@ -359,13 +373,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int nh = min(kSub, x.nsub - t * kSub);
         for (int hh = 0; hh < nh; ++hh) {
           const int j = t * kSub + hh;
-          uint32_t v[kHeadsPad];
-          ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)j, v);
+          uint32_t v[kG];
+          ld_scores<kG>(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)j, v);
           ptx::tmem_ld_wait();
           ptx::reg_fence(v);
           if (x.k0 + j * 128 + r < x.k1) {
 #pragma unroll
-            for (int h = 0; h < kHeadsPad; ++h) mx[h] = fmaxf(mx[h], __uint_as_float(v[h]));
+            for (int h = 0; h < kG; ++h) mx[h] = fmaxf(mx[h], __uint_as_float(v[h]));
           }
         }
         ptx::tc_fence_before();
@@ -373,29 +387,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!ok) break;
 #pragma unroll
-      for (int h = 0; h < kHeadsPad; ++h) {
+      for (int h = 0; h < kG; ++h) {
 #pragma unroll
         for (int o = 16; o >= 1; o >>= 1) mx[h] = fmaxf(mx[h], __shfl_xor_sync(0xffffffffu, mx[h], o));
       }
       if (lane == 0) {
 #pragma unroll
-        for (int h = 0; h < kHeadsPad; ++h) bar->red_m[nu & 1][warp][h] = mx[h];
+        for (int h = 0; h < kG; ++h) bar->red_m[nu & 1][warp][h] = mx[h];
       }
       ptx::mbar_arrive(&bar->red_m_full);
       if (!wait(&bar->red_m_full, nu & 1, a.status)) {
         ok = false;
         break;
       }
-      float m2[kHeadsPad];  // max of scale * log2(e) * S per head (finite: every item has a key)
+      float m2[kG];  // max of scale * log2(e) * S per head (finite: every item has a key)
 #pragma unroll
-      for (int h = 0; h < kHeadsPad; ++h)
+      for (int h = 0; h < kG; ++h)
         m2[h] = fmaxf(fmaxf(bar->red_m[nu & 1][0][h], bar->red_m[nu & 1][1][h]),
                       fmaxf(bar->red_m[nu & 1][2][h], bar->red_m[nu & 1][3][h])) *
                 c2;
       // pass 2: P as bf16 into the A operand of O += P V (rows = heads, columns = keys)
-      float l[kHeadsPad];
+      float l[kG];
 #pragma unroll
-      for (int h = 0; h < kHeadsPad; ++h) l[h] = 0.f;
+      for (int h = 0; h < kG; ++h) l[h] = 0.f;
       for (int t = 0; t < x.nt; ++t, ++T) {
         const uint32_t pb = T & 1;
         if (T >= 2 && !wait(&bar->p_free[pb], ((T >> 1) - 1) & 1, a.status)) {
@@ -407,14 +421,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int nh = min(kSub, x.nsub - t * kSub);
           for (int hh = 0; hh < nh; ++hh) {
             const int j = t * kSub + hh;
-            uint32_t v[kHeadsPad];
-            ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)j, v);
+            uint32_t v[kG];
+            ld_scores<kG>(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)j, v);
             ptx::tmem_ld_wait();
             ptx::reg_fence(v);
             const bool valid = x.k0 + j * 128 + r < x.k1;
-            uint32_t b4[4];
+            uint32_t b4[4] = {0u, 0u, 0u, 0u};  // heads past kG: zero
 #pragma unroll
-            for (int h = 0; h < kHeadsPad; h += 4) {
+            for (int h = 0; h < kG; h += 4) {
               float p4[4];
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
@@ -427,14 +441,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 make_uint4(b4[0], b4[1], b4[2], b4[3]);
           }
         } else {
-          uint32_t v[kHeadsPad];
-          ptx::tmem_ld16(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)t, v);
+          uint32_t v[kG];
+          ld_scores<kG>(tmem + lane_addr + TM_S + kHeadsPad * (uint32_t)t, v);
           ptx::tmem_ld_wait();
           ptx::reg_fence(v);
           const bool valid = x.k0 + t * 128 + r < x.k1;
-          uint32_t pk[kHeadsPad / 2];
+          uint32_t pk[kHeadsPad / 2] = {};  // heads past kG: zero
 #pragma unroll
-          for (int h = 0; h < kHeadsPad; h += 2) {
+          for (int h = 0; h < kG; h += 2) {
             const float p0 = (valid && h < group) ? ex2(__uint_as_float(v[h]) * c2 - m2[h]) : 0.f;
             const float p1 = (valid && h + 1 < group) ? ex2(__uint_as_float(v[h + 1]) * c2 - m2[h + 1]) : 0.f;
             pk[h >> 1] = pack_bf16(p0, p1);
@@ -442,7 +456,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             l[h + 1] += __uint_as_float(pk[h >> 1] & 0xFFFF0000u);
           }
           *reinterpret_cast<uint4*>(P + p_chunk((uint32_t)r, 0u)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-          *reinterpret_cast<uint4*>(P + p_chunk((uint32_t)r, 1u)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+          // heads 8-15 feed only output rows that are not read when kG is 8 or less
+          if constexpr (kG > 8)
+            *reinterpret_cast<uint4*>(P + p_chunk((uint32_t)r, 1u)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
         }
         ptx::fence_proxy_async_smem();
         ptx::mbar_arrive(&bar->p_ready[pb]);
@@ -451,13 +467,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tc_fence_before();
       ptx::mbar_arrive(&bar->s_free);
 #pragma unroll
-      for (int h = 0; h < kHeadsPad; ++h) {
+      for (int h = 0; h < kG; ++h) {
 #pragma unroll
         for (int o = 16; o >= 1; o >>= 1) l[h] += __shfl_xor_sync(0xffffffffu, l[h], o);
       }
       if (lane == 0) {
 #pragma unroll
-        for (int h = 0; h < kHeadsPad; ++h) bar->red_l[nu & 1][warp][h] = l[h];
+        for (int h = 0; h < kG; ++h) bar->red_l[nu & 1][warp][h] = l[h];
       }
       ptx::mbar_arrive(&bar->red_l_full);
       if (!wait(&bar->red_l_full, nu & 1, a.status)) {
@@ -512,7 +528,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <bool kE4M3>
+template <bool kE4M3, int kG>
 cudaError_t launch_decode_tc_t(const DecodeArgs& a, cudaStream_t st) {
   using Cfg = DecCfg<kE4M3>;
   CUtensorMap tq, tk, tv;
@@ -526,7 +542,7 @@ cudaError_t launch_decode_tc_t(const DecodeArgs& a, cudaStream_t st) {
     if ((e = make_tmap_bf16(&tk, a.k_cache, (uint64_t)a.hkv * kD, (uint64_t)a.kv_rows)) != cudaSuccess) return e;
     if ((e = make_tmap_bf16(&tv, a.v_cache, (uint64_t)a.hkv * kD, (uint64_t)a.kv_rows)) != cudaSuccess) return e;
   }
-  if ((e = cudaFuncSetAttribute(decode_tc_kernel<kE4M3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if ((e = cudaFuncSetAttribute(decode_tc_kernel<kE4M3, kG>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)Cfg::kSmemBytes)) != cudaSuccess)
     return e;
   const int64_t sms = sm_count();
@@ -543,7 +559,7 @@ cudaError_t launch_decode_tc_t(const DecodeArgs& a, cudaStream_t st) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kE4M3>, tq, tk, tv, a, n_items);
+  return cudaLaunchKernelEx(&cfg, decode_tc_kernel<kE4M3, kG>, tq, tk, tv, a, n_items);
 }
 
 }  // namespace
@@ -552,7 +568,14 @@ cudaError_t launch_decode_tc(const DecodeArgs& a, cudaStream_t st) {
   if (a.d != kD || (a.dtype != ISM_BF16 && a.dtype != ISM_E4M3) || a.group > kHeadsPad || a.chunk % 128 != 0 ||
       a.chunk > kDecTcMaxKeys)
     return cudaErrorInvalidValue;
-  return a.dtype == ISM_E4M3 ? launch_decode_tc_t<true>(a, st) : launch_decode_tc_t<false>(a, st);
+  // the softmax warps process the group's heads rounded up to 4, 8 or 16
+  if (a.dtype == ISM_E4M3)
+    return a.group <= 4 ? launch_decode_tc_t<true, 4>(a, st)
+           : a.group <= 8 ? launch_decode_tc_t<true, 8>(a, st)
+                          : launch_decode_tc_t<true, kHeadsPad>(a, st);
+  return a.group <= 4 ? launch_decode_tc_t<false, 4>(a, st)
+         : a.group <= 8 ? launch_decode_tc_t<false, 8>(a, st)
+                        : launch_decode_tc_t<false, kHeadsPad>(a, st);
 }
 
 }  // namespace tc

@@ -706,7 +706,8 @@ def test_e4m3_rejects_other_entry_points(ism):
 @pytest.mark.parametrize("l_new,segs,hq,hkv", [(200, ([40, 41, 120, 200], [0, 1, 0, 1]), 8, 2),
                                                 (200, ([40, 41, 120, 200], [0, 1, 0, 1]), 3, 3),
                                                 (1, ([1], [1]), 8, 2), (1, ([1], [1]), 6, 2),
-                                                (1, ([1], [1]), 16, 1), (1, ([1], [1]), 4, 4)])
+                                                (1, ([1], [1]), 16, 1), (1, ([1], [1]), 4, 4),
+                                                (1, ([1], [1]), 10, 2), (1, ([1], [1]), 8, 1)])
 def test_prefill_append_e4m3(ism, l_new, segs, hq, hkv, path, knobs):
     """e4m3 queries and caches (cache factors shared by the new keys / values)
     against the oracle on the dequantised values; single-token steps on the
