@@ -359,26 +359,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       ptx::tmem_ld_wait();
       ptx::reg_fence(q0);
       ptx::reg_fence(q1);
-      if (valid && a.rope_cos) {
-        uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) + grow * a.hq * kD + h * kD);
-        rope_back_store<32>(q0, q1, a.scale, rc, rs, dst + 4 * wg, dst + 8 + 4 * wg);
-      } else if (valid) {
-        uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) + grow * a.hq * kD + h * kD +
-                                              wg * 64);
+      // rows are stored by groups of four lanes (store_slice32)
+      const int64_t rstride = (int64_t)a.hq * kD;
+      __nv_bfloat16* const g0 = reinterpret_cast<__nv_bfloat16*>(a.dq) + (grow - (lane & 3)) * rstride + h * kD;
+      const int g_rows = w.q_len - (row - (lane & 3));
+      uint32_t w0[16], w1[16];
+      if (a.rope_cos) {
+        if (!valid) {
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          uint4 v;
-          v.x = pack_bf16(__uint_as_float(q0[8 * i + 0]) * a.scale, __uint_as_float(q0[8 * i + 1]) * a.scale);
-          v.y = pack_bf16(__uint_as_float(q0[8 * i + 2]) * a.scale, __uint_as_float(q0[8 * i + 3]) * a.scale);
-          v.z = pack_bf16(__uint_as_float(q0[8 * i + 4]) * a.scale, __uint_as_float(q0[8 * i + 5]) * a.scale);
-          v.w = pack_bf16(__uint_as_float(q0[8 * i + 6]) * a.scale, __uint_as_float(q0[8 * i + 7]) * a.scale);
-          dst[i] = v;
-          v.x = pack_bf16(__uint_as_float(q1[8 * i + 0]) * a.scale, __uint_as_float(q1[8 * i + 1]) * a.scale);
-          v.y = pack_bf16(__uint_as_float(q1[8 * i + 2]) * a.scale, __uint_as_float(q1[8 * i + 3]) * a.scale);
-          v.z = pack_bf16(__uint_as_float(q1[8 * i + 4]) * a.scale, __uint_as_float(q1[8 * i + 5]) * a.scale);
-          v.w = pack_bf16(__uint_as_float(q1[8 * i + 6]) * a.scale, __uint_as_float(q1[8 * i + 7]) * a.scale);
-          dst[4 + i] = v;
+          for (int k = 0; k < 32; ++k) rc[k] = rs[k] = 0.f;
         }
+        rope_back_pack(q0, q1, a.scale, rc, rs, w0, w1);
+        store_slice32(w0, g0 + 32 * wg, rstride, g_rows);
+        store_slice32(w1, g0 + 64 + 32 * wg, rstride, g_rows);
+      } else {
+        pack_scaled32(q0, a.scale, w0);
+        pack_scaled32(q1, a.scale, w1);
+        store_slice32(w0, g0 + 64 * wg, rstride, g_rows);
+        store_slice32(w1, g0 + 64 * wg + 32, rstride, g_rows);
       }
     }
   }
@@ -891,31 +889,17 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
       // epilogue of the item: dV, dK from tensor memory
       const int key = x.c * kRows + r;
       const bool kvalid = key < x.w.k_len;
-      if (!wait(&bar->acc_full, nacc & 1, a.status)) { ok = false; break; }
+      // one decision for the whole warp: the epilogue's loads and shuffles are warp-wide
+      if (!__all_sync(0xffffffffu, wait(&bar->acc_full, nacc & 1, a.status))) { ok = false; break; }
       ++nacc;
       ptx::tc_fence_after();
-      const int64_t krow = (int64_t)x.w.k_base + key;
-      __nv_bfloat16* const dvp = reinterpret_cast<__nv_bfloat16*>(a.dv) + krow * a.hkv * kD + x.g * kD;
-      __nv_bfloat16* const dkp = reinterpret_cast<__nv_bfloat16*>(a.dk) + krow * a.hkv * kD + x.g * kD;
-      // 32 columns of an accumulator, scaled by f, to bf16 at dst
-      auto store32 = [&](uint32_t tcol, float f, __nv_bfloat16* dst) {
-        uint32_t v[32];
-        ptx::tmem_ld32(tmem + lane_addr + tcol, v);
-        ptx::tmem_ld_wait();
-        ptx::reg_fence(v);
-        if (kvalid) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst);
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            uint4 o;
-            o.x = pack_bf16(__uint_as_float(v[8 * k + 0]) * f, __uint_as_float(v[8 * k + 1]) * f);
-            o.y = pack_bf16(__uint_as_float(v[8 * k + 2]) * f, __uint_as_float(v[8 * k + 3]) * f);
-            o.z = pack_bf16(__uint_as_float(v[8 * k + 4]) * f, __uint_as_float(v[8 * k + 5]) * f);
-            o.w = pack_bf16(__uint_as_float(v[8 * k + 6]) * f, __uint_as_float(v[8 * k + 7]) * f);
-            d4[k] = o;
-          }
-        }
-      };
+      // rows are stored by groups of four lanes (store_slice32): the group of
+      // this lane starts at key - (lane & 3)
+      const int64_t rstride = (int64_t)a.hkv * kD;
+      const int64_t grow = (int64_t)x.w.k_base + key - (lane & 3);
+      const int g_rows = x.w.k_len - (key - (lane & 3));
+      __nv_bfloat16* const dvg = reinterpret_cast<__nv_bfloat16*>(a.dv) + grow * rstride + x.g * kD;
+      __nv_bfloat16* const dkg = reinterpret_cast<__nv_bfloat16*>(a.dk) + grow * rstride + x.g * kD;
       if (wg == 1 && a.rope_cos) {
 #pragma unroll 1
         for (int q2 = 0; q2 < 2; ++q2) {
@@ -925,12 +909,17 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
           ptx::tmem_ld_wait();
           ptx::reg_fence(lo);
           ptx::reg_fence(hi);
+          float rc[32], rs[32];
           if (kvalid) {
-            float rc[32], rs[32];
             rope_row<32>(a.rope_cos + (int64_t)key * 64 + 32 * q2, a.rope_sin + (int64_t)key * 64 + 32 * q2, rc, rs);
-            rope_back_store<32>(lo, hi, a.scale, rc, rs, reinterpret_cast<uint4*>(dkp + q2 * 32),
-                                reinterpret_cast<uint4*>(dkp + 64 + q2 * 32));
+          } else {
+#pragma unroll
+            for (int k = 0; k < 32; ++k) rc[k] = rs[k] = 0.f;
           }
+          uint32_t wl[16], wh[16];
+          rope_back_pack(lo, hi, a.scale, rc, rs, wl, wh);
+          store_slice32(wl, dkg + q2 * 32, rstride, g_rows);
+          store_slice32(wh, dkg + 64 + q2 * 32, rstride, g_rows);
         }
         ptx::tc_fence_before();
         continue;
@@ -938,10 +927,12 @@ __global__ void __launch_bounds__(dkv::kThreads, 1)
       // warpgroup 0 writes dV, warpgroup 1 writes dK (scaled)
 #pragma unroll 1
       for (int q4 = 0; q4 < 4; ++q4) {
-        if (wg == 0)
-          store32(TM_DV + 32 * q4, 1.f, dvp + 32 * q4);
-        else
-          store32(TM_DK + 32 * q4, a.scale, dkp + 32 * q4);
+        uint32_t v[32], w[16];
+        ptx::tmem_ld32(tmem + lane_addr + (wg == 0 ? TM_DV : TM_DK) + 32 * q4, v);
+        ptx::tmem_ld_wait();
+        ptx::reg_fence(v);
+        pack_scaled32(v, wg == 0 ? 1.f : a.scale, w);
+        store_slice32(w, (wg == 0 ? dvg : dkg) + 32 * q4, rstride, g_rows);
       }
       ptx::tc_fence_before();
     }

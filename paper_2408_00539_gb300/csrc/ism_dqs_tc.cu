@@ -177,14 +177,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       const Item x = decode(a, item);
       const uint32_t b = local & 1, acc = tmem + lane_addr + 128u * b;
       const int row = x.t * kRows + r;
-      const bool valid = row < x.w.q_len;
-      if (!wait(&bar->acc_full[b], (local >> 1) & 1, a.status) || aborted(&bar->abort)) {
+      // one decision for the whole warp: the epilogue's loads and shuffles are warp-wide
+      if (__any_sync(0xffffffffu, !wait(&bar->acc_full[b], (local >> 1) & 1, a.status) || aborted(&bar->abort))) {
         set_abort(&bar->abort);
         break;
       }
       ptx::tc_fence_after();
-      uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.dq) +
-                                            ((int64_t)x.w.q_base + row) * a.hq * kD + x.h * kD);
+      // rows are stored by groups of four lanes (store_slice32)
+      const int64_t rstride = (int64_t)a.hq * kD;
+      __nv_bfloat16* const g0 =
+          reinterpret_cast<__nv_bfloat16*>(a.dq) + ((int64_t)x.w.q_base + row - (lane & 3)) * rstride + x.h * kD;
+      const int g_rows = x.w.q_len - (row - (lane & 3));
       if (a.rope_cos) {
         // rotary encoding: columns k and k + 64 of the row pair up
 #pragma unroll
@@ -200,7 +203,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
             for (int k = 0; k < 32; ++k) lo[k] = hi[k] = 0u;
           }
-          if (valid) rope_back_store<32>(lo, hi, a.scale, nc + 32 * q2, ns + 32 * q2, dst + 4 * q2, dst + 8 + 4 * q2);
+          // (rows past the tile's end compute on stale tables and are not stored)
+          uint32_t wl[16], wh[16];
+          rope_back_pack(lo, hi, a.scale, nc + 32 * q2, ns + 32 * q2, wl, wh);
+          store_slice32(wl, g0 + 32 * q2, rstride, g_rows);
+          store_slice32(wh, g0 + 64 + 32 * q2, rstride, g_rows);
         }
         ptx::tc_fence_before();
         ptx::mbar_arrive(&bar->acc_empty[b]);
@@ -209,7 +216,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
 #pragma unroll 1
       for (int q4 = 0; q4 < 4; ++q4) {
-        uint32_t v[32];
+        uint32_t v[32], w[16];
         if (x.nkb > 0) {
           ptx::tmem_ld32(acc + 32 * q4, v);
           ptx::tmem_ld_wait();
@@ -218,17 +225,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int k = 0; k < 32; ++k) v[k] = 0u;
         }
-        if (valid) {
-#pragma unroll
-          for (int i = 0; i < 4; ++i) {
-            uint4 o;
-            o.x = pack_bf16(__uint_as_float(v[8 * i + 0]) * a.scale, __uint_as_float(v[8 * i + 1]) * a.scale);
-            o.y = pack_bf16(__uint_as_float(v[8 * i + 2]) * a.scale, __uint_as_float(v[8 * i + 3]) * a.scale);
-            o.z = pack_bf16(__uint_as_float(v[8 * i + 4]) * a.scale, __uint_as_float(v[8 * i + 5]) * a.scale);
-            o.w = pack_bf16(__uint_as_float(v[8 * i + 6]) * a.scale, __uint_as_float(v[8 * i + 7]) * a.scale);
-            dst[4 * q4 + i] = o;
-          }
-        }
+        pack_scaled32(v, a.scale, w);
+        store_slice32(w, g0 + 32 * q4, rstride, g_rows);
       }
       ptx::tc_fence_before();
       ptx::mbar_arrive(&bar->acc_empty[b]);

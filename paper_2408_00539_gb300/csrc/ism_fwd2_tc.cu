@@ -462,7 +462,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!ok) break;
       if (nkbm > 0) {
         nb += (uint32_t)nkbm;
-        if (!wait(&bar->pv_done[xh], (nb - 1) & 1, a.status)) { ok = false; break; }
+        // one decision for the whole warp: the epilogue's loads and shuffles are warp-wide
+        if (!__all_sync(0xffffffffu, wait(&bar->pv_done[xh], (nb - 1) & 1, a.status))) { ok = false; break; }
         ptx::tc_fence_after();
       }
       if (kSplit && x.half >= 0) {
@@ -489,24 +490,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       } else if (nkbm > 0) {
         const float inv = (kE4M3 ? a.v_descale : 1.f) / l;
         const int64_t orow = (int64_t)wm.q_base + row;
-        uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(a.out) + orow * a.hq * kD + h * kD);
+        // rows are stored by groups of four lanes (store_slice32)
+        const int li = r & 3;
+        const int64_t rstride = (int64_t)a.hq * kD;
+        __nv_bfloat16* const g0 = reinterpret_cast<__nv_bfloat16*>(a.out) + (orow - li) * rstride + h * kD;
 #pragma unroll 1
         for (int c = 0; c < 4; ++c) {
-          uint32_t o[32];
+          uint32_t o[32], w[16];
           ptx::tmem_ld32(tO + c * 32, o);
           ptx::tmem_ld_wait();
           ptx::reg_fence(o);
-          if (valid) {
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              uint4 v4;
-              v4.x = pack_bf16(__uint_as_float(o[8 * i + 0]) * inv, __uint_as_float(o[8 * i + 1]) * inv);
-              v4.y = pack_bf16(__uint_as_float(o[8 * i + 2]) * inv, __uint_as_float(o[8 * i + 3]) * inv);
-              v4.z = pack_bf16(__uint_as_float(o[8 * i + 4]) * inv, __uint_as_float(o[8 * i + 5]) * inv);
-              v4.w = pack_bf16(__uint_as_float(o[8 * i + 6]) * inv, __uint_as_float(o[8 * i + 7]) * inv);
-              dst[c * 4 + i] = v4;
-            }
-          }
+          pack_scaled32(o, inv, w);
+          store_slice32(w, g0 + 32 * c, rstride, wm.q_len - (row - li));
         }
         if (valid && a.lse) a.lse[(int64_t)h * a.q_rows + orow] = (m_use + log2f(l)) * kLn2;
       }

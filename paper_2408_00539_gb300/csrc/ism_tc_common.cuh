@@ -108,17 +108,63 @@ __device__ __forceinline__ uint32_t pack_e4m3x4(float x0, float x1, float x2, fl
   return r;
 }
 
-// Gradient store of a rotary-encoded head row (the rotation of the one-pass
-// path pairs column k with k + 64).  rope_row<N> loads the cosines and sines
-// of N pairs of a row's position (all loads issued before any use, so their
+// Store of a 32-column slice of 32 consecutive rows held one row per lane
+// (thread = TMEM lane): w holds this lane's 32 bf16 values as 16 packed
+// pairs.  Stored as they are, each 16-byte store instruction of the warp
+// would write 32 different rows; instead the lanes of each group of four
+// (rows 4m .. 4m + 3) exchange their 16-byte pieces, a 4 x 4 transpose in two
+// xor-shuffle rounds, after which lane 4m + i holds piece i of the group's
+// four rows, and each store instruction writes 8 rows of 64 contiguous
+// bytes.  Every lane of the warp must call it (full-warp shuffles).
+// group_row: the slice's first column in row 4m, the first row of this
+// lane's group; rs: the row stride in elements; n_rows: how many of the
+// group's rows exist (rows 4m + j with j >= n_rows are not stored).
+__device__ __forceinline__ void store_slice32(uint32_t (&w)[16], __nv_bfloat16* group_row, int64_t rs, int n_rows) {
+  const int lane = (int)(threadIdx.x & 31), li = lane & 3;
+#pragma unroll
+  for (int d = 2; d >= 1; d >>= 1) {
+    const bool upper = (lane & d) != 0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      if (k & d) continue;
+      // pieces k and k + d: the lower lane of the pair keeps k and receives
+      // the upper lane's k (into k + d); the upper keeps k + d and receives
+      // the lower lane's k + d (into k)
+#pragma unroll
+      for (int c = 0; c < 4; ++c) {
+        const uint32_t out = upper ? w[4 * k + c] : w[4 * (k | d) + c];
+        const uint32_t in = __shfl_xor_sync(0xffffffffu, out, d);
+        if (upper)
+          w[4 * k + c] = in;
+        else
+          w[4 * (k | d) + c] = in;
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+    if (j < n_rows)
+      *reinterpret_cast<uint4*>(group_row + j * rs + 8 * li) =
+          make_uint4(w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+}
+
+// 32 fp32 accumulator columns (bit patterns) scaled by f, as 16 bf16 pairs.
+__device__ __forceinline__ void pack_scaled32(const uint32_t (&v)[32], float f, uint32_t (&w)[16]) {
+#pragma unroll
+  for (int k = 0; k < 16; ++k) w[k] = pack_bf16(__uint_as_float(v[2 * k]) * f, __uint_as_float(v[2 * k + 1]) * f);
+}
+
+// Gradient of a rotary-encoded head row (the rotation of the one-pass path
+// pairs column k with k + 64).  rope_row<N> loads the cosines and sines of N
+// pairs of a row's position (all loads issued before any use, so their
 // latency is paid once; callers issue them well before the values are
-// needed).  rope_back_store<N>: lo holds columns k0..k0+N-1 and hi columns
-// k0+64..k0+63+N of the gradient of the ROTATED row (fp32 bit patterns);
+// needed).  rope_back_pack: lo holds columns k0..k0+31 and hi columns
+// k0+64..k0+95 of the gradient of the ROTATED row (fp32 bit patterns);
 // after scaling by f, each pair (g_k, g_{k+64}) goes back through the
 // transposed rotation, x_k = g_k c + g_{k+64} s and
-// x_{k+64} = g_{k+64} c - g_k s, and the bf16 results are stored at dst_lo
-// (columns k0..) and dst_hi (columns k0+64..).  c and s point into register
-// arrays at offsets fixed at compile time (the loops are unrolled).
+// x_{k+64} = g_{k+64} c - g_k s, packed as bf16 pairs into wl (columns
+// k0..) and wh (columns k0+64..) for store_slice32.  c and s point into
+// register arrays at offsets fixed at compile time (the loops are unrolled).
 template <int N>
 __device__ __forceinline__ void rope_row(const float* __restrict__ cs, const float* __restrict__ sn, float* c,
                                          float* s) {
@@ -131,24 +177,21 @@ __device__ __forceinline__ void rope_row(const float* __restrict__ cs, const flo
     s[4 * i] = sv.x; s[4 * i + 1] = sv.y; s[4 * i + 2] = sv.z; s[4 * i + 3] = sv.w;
   }
 }
-template <int N>
-__device__ __forceinline__ void rope_back_store(const uint32_t* lo, const uint32_t* hi, float f, const float* c,
-                                                const float* s, uint4* dst_lo, uint4* dst_hi) {
-  static_assert(N % 8 == 0, "whole 16-byte stores");
+__device__ __forceinline__ void rope_back_pack(const uint32_t (&lo)[32], const uint32_t (&hi)[32], float f,
+                                               const float* c, const float* s, uint32_t (&wl)[16],
+                                               uint32_t (&wh)[16]) {
 #pragma unroll
-  for (int i = 0; i < N / 8; ++i) {
-    float xl[8], xh[8];
+  for (int k = 0; k < 16; ++k) {
+    float xl[2], xh[2];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      const int k = 8 * i + e;
-      const float gl = __uint_as_float(lo[k]) * f, gh = __uint_as_float(hi[k]) * f;
-      xl[e] = gl * c[k] + gh * s[k];
-      xh[e] = gh * c[k] - gl * s[k];
+    for (int e = 0; e < 2; ++e) {
+      const int j = 2 * k + e;
+      const float gl = __uint_as_float(lo[j]) * f, gh = __uint_as_float(hi[j]) * f;
+      xl[e] = gl * c[j] + gh * s[j];
+      xh[e] = gh * c[j] - gl * s[j];
     }
-    dst_lo[i] = make_uint4(pack_bf16(xl[0], xl[1]), pack_bf16(xl[2], xl[3]), pack_bf16(xl[4], xl[5]),
-                           pack_bf16(xl[6], xl[7]));
-    dst_hi[i] = make_uint4(pack_bf16(xh[0], xh[1]), pack_bf16(xh[2], xh[3]), pack_bf16(xh[4], xh[5]),
-                           pack_bf16(xh[6], xh[7]));
+    wl[k] = pack_bf16(xl[0], xl[1]);
+    wh[k] = pack_bf16(xh[0], xh[1]);
   }
 }
 
