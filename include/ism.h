@@ -185,8 +185,7 @@ ism_status_t ism_attn_fwd_e4m3(const ism_segments_t* segs, const ism_attn_shape_
  *  - Batches whose forward workspace (ism_attn_fwd_workspace_size) exceeds
  *    the array return ISM_ERR_WORKSPACE before anything is launched.
  *  - The first call on a device looks the array's device address up
- *    (cudaGetSymbolAddress) with that device current; make that first call
- *    before any stream capture.
+ *    (cudaGetSymbolAddress, a host-side query) with that device current.
  *  - All calls share the one array: calls whose kernels may overlap on the
  *    GPU (different streams without ordering) race on it. */
 size_t ism_attn_fwd_noalloc_max_workspace(void);
