@@ -320,6 +320,13 @@ def run_cuda(args, w):
             ism.bwd_rope(segs, q_rot, k_rot, vd, o, lse, dod, cos_t, sin_t, w.softmax_scale, dq=dq, dk=dk, dv=dv,
                          workspace=ws_b)
 
+    if args.profile_step and args.e4m3:
+        # the e4m3 forward alone for a profiler: e4m3 copies of the same Q, K, V
+        q8, k8, v8 = (wl.quantize_e4m3(t) for t in (qd, kd, vd))
+
+        def step():  # noqa: F811
+            ism.fwd_e4m3(segs, q8[0], k8[0], v8[0], q8[1], k8[1], v8[1], w.softmax_scale)
+
     # clocks are sampled from the warm-up on (nvidia-smi needs a moment to start)
     clocks = ClockSampler(dev.index) if not args.profile_step else None
     if clocks is not None:
@@ -1256,6 +1263,7 @@ def main():
     ap.add_argument("--profile-step", action="store_true",
                     help="run the warm-up steps and one more step, print nothing (for ncu)")
     ap.add_argument("--rope", action="store_true", help="with --profile-step: the rotary forward and backward")
+    ap.add_argument("--e4m3", action="store_true", help="with --profile-step: the e4m3 forward alone")
     ap.add_argument("--min-workspace", action="store_true",
                     help="backward with the minimum workspace (recompute schedule) in the headline step")
     ap.add_argument("--profile-decode", choices=["bf16", "e4m3"],
