@@ -16,43 +16,67 @@ __device__ __forceinline__ int upper_bound_i32(const int32_t* a, int n, int32_t 
   return lo;
 }
 
+// Inclusive prefix sum of one value per thread over the block (blockDim.x a
+// multiple of 32, at most 1024): shuffle scans within each warp, then warp 0
+// scans the warp totals.  *total receives the block's sum.  Every thread of
+// the block calls it (it holds __syncthreads).
+template <typename T>
+__device__ T block_inclusive_scan(T v, T* total) {
+  __shared__ T wsum[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const T t = __shfl_up_sync(0xffffffffu, v, o);
+    if (lane >= o) v += t;
+  }
+  if (lane == 31) wsum[warp] = v;
+  __syncthreads();
+  if (warp == 0) {
+    T w = lane < nw ? wsum[lane] : T(0);
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const T t = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += t;
+    }
+    wsum[lane] = w;  // inclusive over the warps
+  }
+  __syncthreads();
+  const T add = warp > 0 ? wsum[warp - 1] : T(0);
+  *total = wsum[nw - 1];
+  __syncthreads();  // wsum is free for the next call
+  return v + add;
+}
+
 // Per-sequence tile offsets computed by every block into shared memory:
 // qoff/koff [B+1] (q-tiles / k-tiles before sequence b) and toff [B+1]
 // (tile_class bytes before sequence b).  Block-wide scans over chunks of
-// blockDim.x (at most 1024) sequences with a running carry.
+// blockDim.x sequences with a running carry.
 __device__ void seq_offsets_smem(const SegsDev& s, int bm, int bn, int32_t* qoff, int32_t* koff, int64_t* toff) {
-  __shared__ int32_t sq[1024], sk[1024];
-  __shared__ int64_t stl[1024];
-  __shared__ int32_t cq, ck;
-  __shared__ int64_t ct;
-  if (threadIdx.x == 0) { cq = 0; ck = 0; ct = 0; qoff[0] = 0; koff[0] = 0; toff[0] = 0; }
-  __syncthreads();
+  if (threadIdx.x == 0) { qoff[0] = 0; koff[0] = 0; toff[0] = 0; }
+  int32_t cq = 0, ck = 0;  // carries, the same in every thread
+  int64_t ct = 0;
   for (int base = 0; base < s.num_seqs; base += blockDim.x) {
-    int b = base + threadIdx.x;
+    const int b = base + threadIdx.x;
     int32_t nq = 0, nk = 0;
     if (b < s.num_seqs) {
-      int32_t L = s.cu_seqlens[b + 1] - s.cu_seqlens[b];
+      const int32_t L = s.cu_seqlens[b + 1] - s.cu_seqlens[b];
       nq = (L + bm - 1) / bm;
       nk = (L + bn - 1) / bn;
     }
-    sq[threadIdx.x] = nq; sk[threadIdx.x] = nk; stl[threadIdx.x] = (int64_t)nq * nk;
-    __syncthreads();
-    for (int off = 1; off < blockDim.x; off <<= 1) {  // Hillis-Steele inclusive scan
-      int32_t a = 0, c = 0; int64_t t = 0;
-      if (threadIdx.x >= off) { a = sq[threadIdx.x - off]; c = sk[threadIdx.x - off]; t = stl[threadIdx.x - off]; }
-      __syncthreads();
-      sq[threadIdx.x] += a; sk[threadIdx.x] += c; stl[threadIdx.x] += t;
-      __syncthreads();
-    }
+    int32_t tq, tk;
+    int64_t tt;
+    const int32_t iq = block_inclusive_scan<int32_t>(nq, &tq), ik = block_inclusive_scan<int32_t>(nk, &tk);
+    const int64_t it = block_inclusive_scan<int64_t>((int64_t)nq * nk, &tt);
     if (b < s.num_seqs) {
-      qoff[b + 1] = cq + sq[threadIdx.x];
-      koff[b + 1] = ck + sk[threadIdx.x];
-      toff[b + 1] = ct + stl[threadIdx.x];
+      qoff[b + 1] = cq + iq;
+      koff[b + 1] = ck + ik;
+      toff[b + 1] = ct + it;
     }
-    __syncthreads();
-    if (threadIdx.x == blockDim.x - 1) { cq += sq[threadIdx.x]; ck += sk[threadIdx.x]; ct += stl[threadIdx.x]; }
-    __syncthreads();
+    cq += tq;
+    ck += tk;
+    ct += tt;
   }
+  __syncthreads();
 }
 
 // kv_end of every token (Eq. fj): a token of a query segment is bounded by
@@ -184,9 +208,16 @@ __device__ void order_body(const Tile* __restrict__ qtiles, int64_t nq, const Ti
       atomicAdd(&hist[cost], 1);
     }
     __syncthreads();
-    if (threadIdx.x == 0) {  // exclusive scan from the highest cost down
-      int32_t run = 0;
-      for (int c = max_cost; c >= 0; --c) { int32_t h = hist[c]; hist[c] = run; run += h; }
+    // exclusive scan from the highest cost down (each thread rewrites the
+    // entries it read, so no barrier is needed between the read and the write)
+    int32_t run = 0;
+    for (int base = 0; base <= max_cost; base += blockDim.x) {
+      const int c = max_cost - (base + (int)threadIdx.x);
+      const int32_t h = c >= 0 ? hist[c] : 0;
+      int32_t tot;
+      const int32_t incl = block_inclusive_scan<int32_t>(h, &tot);
+      if (c >= 0) hist[c] = run + incl - h;
+      run += tot;
     }
     __syncthreads();
     for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
@@ -215,10 +246,7 @@ __global__ void order_kernel(const Tile* __restrict__ qtiles, int64_t nq, const 
 // the first (k-tile, q-tile) pair slot of each k-tile.  One block, chunks of
 // blockDim.x with a running carry.
 __device__ void pair_offsets_body(const Tile* __restrict__ ktiles, int64_t nk, int32_t* kpair_off) {
-  __shared__ int32_t buf[1024];
-  __shared__ int32_t carry;
-  if (threadIdx.x == 0) carry = 0;
-  __syncthreads();
+  int32_t carry = 0;  // the same in every thread
   for (int64_t base = 0; base < nk; base += blockDim.x) {
     const int64_t i = base + threadIdx.x;
     int32_t v = 0;
@@ -226,18 +254,10 @@ __device__ void pair_offsets_body(const Tile* __restrict__ ktiles, int64_t nk, i
       const Tile w = ktiles[i];
       v = w.a1 - w.a0 > 0 ? w.a1 - w.a0 : 0;
     }
-    buf[threadIdx.x] = v;
-    __syncthreads();
-    for (int off = 1; off < blockDim.x; off <<= 1) {
-      const int32_t add = threadIdx.x >= off ? buf[threadIdx.x - off] : 0;
-      __syncthreads();
-      buf[threadIdx.x] += add;
-      __syncthreads();
-    }
-    if (i < nk) kpair_off[i] = carry + buf[threadIdx.x] - v;
-    __syncthreads();
-    if (threadIdx.x == blockDim.x - 1) carry += buf[threadIdx.x];
-    __syncthreads();
+    int32_t tot;
+    const int32_t incl = block_inclusive_scan<int32_t>(v, &tot);
+    if (i < nk) kpair_off[i] = carry + incl - v;
+    carry += tot;
   }
 }
 
