@@ -304,10 +304,14 @@ def run_cuda(args, w):
     ws_b = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
     dq, dk, dv = ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, workspace=ws_b)
     flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
+    # a step builds the batch's plan (one metadata pass) and runs the forward
+    # and the backward on it, as a training step over the same segments does
+    plan = ism.Plan(segs, w.num_heads_q, w.num_heads_kv, w.head_dim, qd.dtype, dev)
 
     def step():
-        ism.fwd(segs, qd, kd, vd, w.softmax_scale, out=o, lse=lse)
-        ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws_b)
+        plan.build()
+        ism.fwd(segs, qd, kd, vd, w.softmax_scale, out=o, lse=lse, plan=plan)
+        ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws_b, plan=plan)
 
     if args.profile_step and args.rope:
         # the rotary step (usual schedule) for a profiler: same tensors, rotated copies
@@ -436,9 +440,10 @@ def run_cuda(args, w):
         copy_stream.wait_stream(stream)
         with torch.cuda.stream(copy_stream):
             dod.copy_(doh, non_blocking=True)
-        ism.fwd(segs, qd, kd, vd, w.softmax_scale, out=o, lse=lse)
+        plan.build()
+        ism.fwd(segs, qd, kd, vd, w.softmax_scale, out=o, lse=lse, plan=plan)
         stream.wait_stream(copy_stream)
-        ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws_b)
+        ism.bwd(segs, qd, kd, vd, o, lse, dod, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws_b, plan=plan)
         dqh.copy_(dq, non_blocking=True)
         dkh.copy_(dk, non_blocking=True)
         dvh.copy_(dv, non_blocking=True)
@@ -494,9 +499,10 @@ def run_cuda(args, w):
                 stream.wait_event(ev_out[i - 2])  # its gradients were read back
             qb, kb, vb, dob = ins[bsel]
             dqb, dkb, dvb = outs[bsel]
-            ism.fwd(segs, qb, kb, vb, w.softmax_scale, out=ob[bsel], lse=lb[bsel])
+            plan.build()
+            ism.fwd(segs, qb, kb, vb, w.softmax_scale, out=ob[bsel], lse=lb[bsel], plan=plan)
             ism.bwd(segs, qb, kb, vb, ob[bsel], lb[bsel], dob, w.softmax_scale, dq=dqb, dk=dkb, dv=dvb,
-                    workspace=ws_b)
+                    workspace=ws_b, plan=plan)
             ev_done[i].record(stream)
             down.wait_event(ev_done[i])
             with torch.cuda.stream(down):
@@ -531,30 +537,33 @@ def run_cuda(args, w):
                    "strict_tflops_12D": value * 12 / 14, "l2": "flushed between timed steps (258 MB write)",
                    "pct_of_peak": value / peak_tc * 100, "path": "tensor cores" if ism.has_tensor_cores()
                    else "cuda cores", "bwd_schedule": "stored dS" if stored_ds else "recompute dQ",
-                   "bwd_workspace_bytes": ws_bytes, "parallelism": f"replicas x{world}"},
+                   "bwd_workspace_bytes": ws_bytes,
+                   "metadata": "one pass a step (ism_attn_plan_build), shared by the forward and the backward",
+                   "parallelism": f"replicas x{world}"},
         "kernel_ms": mean_k,
         "phases": {
             "fwd": {"ms": mean_k["meta"] + mean_k["fwd"], "flops": 4 * D * n_vis,
                     "tflops": 4 * D * n_vis / ((mean_k["meta"] + mean_k["fwd"]) * 1e-3) / 1e12,
-                    "kernels": "metadata pass + forward"},
-            "bwd": {"ms": mean_k["meta"] + mean_k["bwd_pre"] + mean_k["bwd_dkdv"] + mean_k["bwd_dq"],
+                    "kernels": "metadata pass (the plan) + forward"},
+            "bwd": {"ms": mean_k["bwd_pre"] + mean_k["bwd_dkdv"] + mean_k["bwd_dq"],
                     "flops": 10 * D * n_vis,
-                    "tflops": 10 * D * n_vis / ((mean_k["meta"] + mean_k["bwd_pre"] + mean_k["bwd_dkdv"] +
+                    "tflops": 10 * D * n_vis / ((mean_k["bwd_pre"] + mean_k["bwd_dkdv"] +
                                                  mean_k["bwd_dq"]) * 1e-3) / 1e12,
-                    "kernels": "metadata pass + Delta + dK/dV + dQ"},
-            "note": "per-call kernel times from the timer hooks (each call runs its own metadata pass); the "
-                    "headline counts fwd 4*D*N_vis and bwd 10*D*N_vis"},
+                    "kernels": "Delta + dK/dV + dQ on the plan"},
+            "note": "per-kernel times from the timer hooks; a step builds the plan (one metadata pass) and "
+                    "runs the forward and the backward on it; the headline counts fwd 4*D*N_vis and bwd "
+                    "10*D*N_vis"},
         "roofline": roofline,
         "kernel_rooflines": rooflines,
         "e2e": {"value": e2e_value, "unit": "TFLOP/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_total / args.steps,
                 "ms_per_step_runs": [t / args.steps for t in e2e_runs],
-                "how": "median of three runs of K steps back to back through ism.fwd/ism.bwd; step i+1's Q, K, V, dO uploads (pinned host, "
+                "how": "median of three runs of K steps back to back through ism.Plan.build/ism.fwd/ism.bwd; step i+1's Q, K, V, dO uploads (pinned host, "
                        "copy stream) and step i's dQ, dK, dV read-backs (second copy stream) overlap the kernels; "
                        "double-buffered device tensors; inputs (335 MB) exceed L2, no flush",
                 "serial": {"value": job_throughput(flops, world, args.steps, serial_total) / 1e12,
                            "ms_per_step": serial_total / args.steps,
-                           "how": "each step alone: upload, fwd+bwd, read-back, L2 flushed between steps"}},
+                           "how": "each step alone: upload, plan + fwd + bwd, read-back, L2 flushed between steps"}},
         "gpu_launches": int(launches),
         "clocks": clocks.summary(),
     }
@@ -805,10 +814,12 @@ def measure_training_config(dev, w, peaks, steps=20, minimal_workspace=False, ro
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
     flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream(dev)
+    plan = ism.Plan(segs, w.num_heads_q, w.num_heads_kv, w.head_dim, q.dtype, dev)
 
-    def step():
-        ism.fwd(segs, q, k, v, w.softmax_scale, out=o, lse=lse)
-        ism.bwd(segs, q, k, v, o, lse, do, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws)
+    def step():  # the plan (one metadata pass), the forward and the backward on it
+        plan.build()
+        ism.fwd(segs, q, k, v, w.softmax_scale, out=o, lse=lse, plan=plan)
+        ism.bwd(segs, q, k, v, o, lse, do, w.softmax_scale, dq=dq, dk=dk, dv=dv, workspace=ws, plan=plan)
 
     if rope:
         cos_np, sin_np = wl.rope_tables(int(np.diff(w.segs.cu_seqlens).max()), D)
@@ -896,6 +907,7 @@ def measure_long_context(dev, peaks, length=131072, steps=3):
     o, lse = ism.fwd(segs, q, k, v, scale)
     dq, dk, dv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
     stream = torch.cuda.current_stream(dev)
+    plan = ism.Plan(segs, hq, hkv, D, q.dtype, dev)
     n_vis = n_visible(segs_np) * hq
     flops = 14 * D * n_vis
     kinds = {"fwd": ism.KERNEL_FWD, "bwd_dkdv": ism.KERNEL_BWD_DKDV, "bwd_dq": ism.KERNEL_BWD_DQ}
@@ -908,8 +920,9 @@ def measure_long_context(dev, peaks, length=131072, steps=3):
             ism.set_kernel_timer(kid, *ev[n])
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        ism.fwd(segs, q, k, v, scale, out=o, lse=lse)
-        ism.bwd(segs, q, k, v, o, lse, do, scale, dq=dq, dk=dk, dv=dv, workspace=ws)
+        plan.build()
+        ism.fwd(segs, q, k, v, scale, out=o, lse=lse, plan=plan)
+        ism.bwd(segs, q, k, v, o, lse, do, scale, dq=dq, dk=dk, dv=dv, workspace=ws, plan=plan)
         e1.record(stream)
         e1.synchronize()
         if it:

@@ -256,6 +256,50 @@ ism_status_t ism_attn_bwd_rope(const ism_segments_t* segs, const ism_attn_shape_
                                void* workspace, size_t workspace_bytes, ism_stream_t stream);
 
 /* ---------------------------------------------------------------------------
+ * Plans: the metadata of one batch of segments, built once and shared by the
+ * forward and the backward of every attention layer over those segments
+ * with the same head counts.  The metadata is what ism_attn_fwd and
+ * ism_attn_bwd otherwise rebuild at the start of every call: the per-token
+ * key bounds (Eq. fj), the (query tile, key tile) descriptors and the work
+ * lists in cost order.  A training step then runs one metadata pass for all
+ * of its layers instead of two per layer.
+ *
+ * ism_attn_plan_size: device bytes of the plan for these segments and shape
+ *   (head counts; dtype ISM_BF16 or ISM_FP32; head_dim as for ism_attn_fwd).
+ * ism_attn_plan_build: runs the metadata pass into `plan` (device memory of
+ *   at least that size, 256-byte aligned, owned by the caller) on `stream`
+ *   and fills *plan_info on the host: a fingerprint of the segments' host
+ *   arrays and the head counts, and the plan's size.
+ * ism_attn_fwd_planned / ism_attn_bwd_planned: ism_attn_fwd / ism_attn_bwd
+ *   on the plan's metadata, with identical results.  The segments and shape
+ *   must be those of the build (same host arrays and head counts; the
+ *   softmax scale may differ): a mismatch of the fingerprint returns
+ *   ISM_ERR_INVALID_ARG before any launch.  The forward needs no workspace;
+ *   the backward takes a workspace as ism_attn_bwd does
+ *   (ism_attn_bwd_workspace_size for the stored-dS schedule, _min for the
+ *   recompute schedule: both cover what the planned call uses).
+ * The plan must stay unchanged while a call that uses it may run, and calls
+ * that share a plan run in stream order (the backward resets a work counter
+ * held in the plan).  No counterpart in the paper.
+ * ------------------------------------------------------------------------- */
+typedef struct {
+  uint64_t fingerprint;
+  size_t bytes;
+} ism_attn_plan_info_t;
+
+ism_status_t ism_attn_plan_size(const ism_segments_t* segs, const ism_attn_shape_t* shape, size_t* bytes);
+ism_status_t ism_attn_plan_build(const ism_segments_t* segs, const ism_attn_shape_t* shape, void* plan,
+                                 size_t plan_bytes, ism_attn_plan_info_t* plan_info, ism_stream_t stream);
+ism_status_t ism_attn_fwd_planned(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* plan,
+                                  const ism_attn_plan_info_t* plan_info, const void* q, const void* k,
+                                  const void* v, void* o, float* lse, ism_stream_t stream);
+ism_status_t ism_attn_bwd_planned(const ism_segments_t* segs, const ism_attn_shape_t* shape, void* plan,
+                                  const ism_attn_plan_info_t* plan_info, const void* q, const void* k,
+                                  const void* v, const void* o, const float* lse, const void* dout, void* dq,
+                                  void* dk, void* dv, void* workspace, size_t workspace_bytes,
+                                  ism_stream_t stream);
+
+/* ---------------------------------------------------------------------------
  * Append-prefill of a new turn against a reused KV cache (Section 2.3: the
  * history's keys/values C_h are reused, the new chunk's C_q are computed and
  * [C_h; C_q] concatenated).  Valid because no token sees past the end of its

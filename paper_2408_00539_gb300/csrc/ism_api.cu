@@ -232,6 +232,46 @@ PassLayout pass_layout(void* ws, const ism_segments_t* s, const Counts& c, int64
   return L;
 }
 
+// Device layout of a plan (ism_attn_plan_build): the metadata of both
+// passes for one batch of segments and head counts, without the backward's
+// Delta and dS tiles, which stay in the backward's workspace.
+bool fwd_tile_pairs(const ism_attn_shape_t* sh);
+PassLayout plan_layout(void* plan, const Counts& c, int64_t T, bool tile_pairs) {
+  Carve cv(plan);
+  PassLayout L{};
+  L.kv_end = cv.take<int32_t>(T);
+  L.qtiles = cv.take<Tile>(c.nq);
+  L.q_order = cv.take<int32_t>(c.nq);
+  L.ktiles = cv.take<Tile>(c.nk);
+  L.k_order = cv.take<int32_t>(c.nk);
+  L.kpair_off = cv.take<int32_t>(c.nk);
+  L.pair_order = tile_pairs ? cv.take<int32_t>(c.npairs) : nullptr;
+  L.counters = cv.take<int32_t>(kPassCounters);
+  L.bytes = ((cv.off + 255) & ~size_t(255)) + 256;
+  return L;
+}
+
+// What a plan was built for: FNV-1a over the segments' host arrays, the head
+// counts and whether the forward pairs query tiles (the work lists differ).
+uint64_t plan_fingerprint(const ism_segments_t* s, const ism_attn_shape_t* sh, bool tile_pairs) {
+  uint64_t h = 1469598103934665603ull;
+  auto mix = [&](const void* p, size_t n) {
+    const unsigned char* b = static_cast<const unsigned char*>(p);
+    for (size_t i = 0; i < n; ++i) h = (h ^ b[i]) * 1099511628211ull;
+  };
+  const int32_t head[4] = {s->num_seqs, s->num_segs, sh->num_heads_q, sh->num_heads_kv};
+  mix(head, sizeof(head));
+  const uint8_t tp = tile_pairs ? 1 : 0;
+  mix(&tp, 1);
+  mix(s->cu_seqlens_host, sizeof(int32_t) * (size_t)(s->num_seqs + 1));
+  mix(s->cu_segs_host, sizeof(int32_t) * (size_t)(s->num_seqs + 1));
+  if (s->num_segs > 0) {
+    mix(s->seg_end_host, sizeof(int32_t) * (size_t)s->num_segs);
+    mix(s->seg_type_host, (size_t)s->num_segs);
+  }
+  return h;
+}
+
 bool force_cuda_cores() { return knobs().force_cuda_cores; }
 
 uint32_t tc_flags() { return knobs().drain_tmem_reuse ? kFlagDrainTmemReuse : 0u; }
@@ -469,7 +509,7 @@ ism_status_t check_rope_pass(const ism_rope_t* rope, const ism_attn_shape_t* sha
 ism_status_t fwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q, const void* k,
                       const void* v, void* o, float* lse, void* workspace, size_t workspace_bytes, ism_stream_t stream,
                       float qk_descale, float v_descale, const ism_rope_t* rope = nullptr, void* q_rot = nullptr,
-                      void* k_rot = nullptr) {
+                      void* k_rot = nullptr, const PassLayout* pre = nullptr) {
   SegInfo info;
   ism_status_t r = check_segments(segs, &info);
   if (r != ISM_OK) return r;
@@ -484,9 +524,11 @@ ism_status_t fwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape,
   if (rope && (!q_rot || !k_rot || !aligned16(q_rot) || !aligned16(k_rot)))
     return fail(ISM_ERR_INVALID_ARG, "q_rot and k_rot must be non-NULL and 16-byte aligned");
   Counts c = count_tiles(segs, kTile, kTile);
-  PassLayout L =
-      pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, false, 0, fwd_tile_pairs(shape));
-  if ((r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
+  // pre: the metadata of a plan (ism_attn_plan_build), already on the device
+  PassLayout L = pre ? *pre
+                     : pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, false, 0,
+                                   fwd_tile_pairs(shape));
+  if (!pre && (r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
   uint32_t* status;
   if ((r = status_ptr(&status)) != ISM_OK) return r;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -501,7 +543,7 @@ ism_status_t fwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape,
     q = q_rot;
     k = k_rot;
   }
-  if ((r = build_pass_meta(segs, c, L, false, st)) != ISM_OK) return r;
+  if (!pre && (r = build_pass_meta(segs, c, L, false, st)) != ISM_OK) return r;
 
   AttnArgs a{};
   a.q = q; a.k = k; a.v = v; a.out = o; a.lse = lse;
@@ -567,7 +609,8 @@ namespace {
 
 ism_status_t bwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* q, const void* k,
                       const void* v, const void* o, const float* lse, const void* dout, void* dq, void* dk, void* dv,
-                      void* workspace, size_t workspace_bytes, ism_stream_t stream, const ism_rope_t* rope) {
+                      void* workspace, size_t workspace_bytes, ism_stream_t stream, const ism_rope_t* rope,
+                      const PassLayout* pre = nullptr) {
   SegInfo info;
   ism_status_t r = check_segments(segs, &info);
   if (r != ISM_OK) return r;
@@ -581,15 +624,36 @@ ism_status_t bwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape,
     if (!aligned16(p)) return fail(ISM_ERR_INVALID_ARG, "tensors must be 16-byte aligned");
   Counts c = count_tiles(segs, kTile, kTile);
   // the stored-dS path when the workspace holds its tiles, else recompute
-  const int64_t slots = stored_ds_slots(segs, shape);
-  PassLayout L = pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, true, slots);
-  if (slots > 0 && workspace_bytes < L.bytes)
-    L = pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, true);
+  int64_t slots = stored_ds_slots(segs, shape);
+  PassLayout L;
+  if (pre) {
+    // metadata from a plan; Delta and the dS tiles from the workspace
+    L = *pre;
+    Carve cv(workspace);
+    L.delta = cv.take<float>((int64_t)shape->num_heads_q * info.total_tokens);
+    const size_t need_min = ((cv.off + 255) & ~size_t(255)) + 256;
+    void* ds = slots > 0 ? static_cast<void*>(cv.take<uint16_t>(slots * kTile * kTile)) : nullptr;
+    const size_t need_full = ((cv.off + 255) & ~size_t(255)) + 256;
+    L.ds = ds && workspace_bytes >= need_full ? ds : nullptr;
+    if (!L.ds) slots = 0;
+    L.bytes = L.ds ? need_full : need_min;
+  } else {
+    L = pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, true, slots);
+    if (slots > 0 && workspace_bytes < L.bytes) {
+      L = pass_layout(workspace, segs, c, info.total_tokens, shape->num_heads_q, true);
+      slots = 0;
+    }
+  }
   if ((r = check_ws(workspace, workspace_bytes, L.bytes)) != ISM_OK) return r;
   uint32_t* status;
   if ((r = status_ptr(&status)) != ISM_OK) return r;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  if ((r = build_pass_meta(segs, c, L, true, st)) != ISM_OK) return r;
+  if (pre) {
+    // the plan's work counters start at zero for this call
+    ISM_TRY_CUDA(cudaMemsetAsync(L.counters, 0, kPassCounters * sizeof(int32_t), st), "work counter reset");
+  } else if ((r = build_pass_meta(segs, c, L, true, st)) != ISM_OK) {
+    return r;
+  }
 
   AttnArgs a{};
   a.q = q; a.k = k; a.v = v; a.o = o; a.dout = dout; a.lse_in = lse;
@@ -601,7 +665,8 @@ ism_status_t bwd_impl(const ism_segments_t* segs, const ism_attn_shape_t* shape,
   a.ds = L.ds; a.kpair_off = L.kpair_off; a.ds_slots = L.ds ? slots : 0;
   a.work_counter = L.counters;
   // the k-tile pair list exists only when the CTA-pair dK/dV kernel will run
-  a.kp_order = knobs().dkdv_pair ? L.kp_order : nullptr;
+  // (and a plan holds none)
+  a.kp_order = knobs().dkdv_pair && !pre ? L.kp_order : nullptr;
   a.nkp = a.kp_order ? c.npairs : 0;
   a.status = status;
   a.flags = tc_flags();
@@ -643,6 +708,86 @@ ism_status_t ism_attn_bwd_rope(const ism_segments_t* segs, const ism_attn_shape_
                                size_t workspace_bytes, ism_stream_t stream) {
   if (!rope) return fail(ISM_ERR_INVALID_ARG, "rope is NULL");
   return bwd_impl(segs, shape, q_rot, k_rot, v, o, lse, dout, dq, dk, dv, workspace, workspace_bytes, stream, rope);
+}
+
+// ---------------------------------------------------------------- plans
+
+ism_status_t ism_attn_plan_size(const ism_segments_t* segs, const ism_attn_shape_t* shape, size_t* bytes) {
+  SegInfo info;
+  ism_status_t r = check_segments(segs, &info);
+  if (r != ISM_OK) return r;
+  if ((r = check_shape(shape)) != ISM_OK) return r;
+  if (!bytes) return fail(ISM_ERR_INVALID_ARG, "bytes is NULL");
+  Counts c = count_tiles(segs, kTile, kTile);
+  *bytes = plan_layout(nullptr, c, info.total_tokens, fwd_tile_pairs(shape)).bytes;
+  return ISM_OK;
+}
+
+ism_status_t ism_attn_plan_build(const ism_segments_t* segs, const ism_attn_shape_t* shape, void* plan,
+                                 size_t plan_bytes, ism_attn_plan_info_t* plan_info, ism_stream_t stream) {
+  SegInfo info;
+  ism_status_t r = check_segments(segs, &info);
+  if (r != ISM_OK) return r;
+  if ((r = check_shape(shape)) != ISM_OK) return r;
+  if (!plan_info) return fail(ISM_ERR_INVALID_ARG, "plan_info is NULL");
+  Counts c = count_tiles(segs, kTile, kTile);
+  const bool tile_pairs = fwd_tile_pairs(shape);
+  PassLayout L = plan_layout(plan, c, info.total_tokens, tile_pairs);
+  if ((r = check_ws(plan, plan_bytes, L.bytes)) != ISM_OK) return r;
+  if (info.total_tokens > 0) {
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if ((r = build_pass_meta(segs, c, L, true, st)) != ISM_OK) return r;
+  }
+  plan_info->fingerprint = plan_fingerprint(segs, shape, tile_pairs);
+  plan_info->bytes = L.bytes;
+  return ISM_OK;
+}
+
+}  // extern "C"
+
+namespace {
+
+// The layout of a plan for these segments and shape, after checking that the
+// plan was built for them.
+ism_status_t planned_layout(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* plan,
+                            const ism_attn_plan_info_t* plan_info, PassLayout* L) {
+  SegInfo info;
+  ism_status_t r = check_segments(segs, &info);
+  if (r != ISM_OK) return r;
+  if ((r = check_shape(shape)) != ISM_OK) return r;
+  if (!plan || !plan_info) return fail(ISM_ERR_INVALID_ARG, "plan and plan_info must be non-NULL");
+  if (reinterpret_cast<uintptr_t>(plan) & 255u) return fail(ISM_ERR_INVALID_ARG, "plan must be 256-byte aligned");
+  const bool tile_pairs = fwd_tile_pairs(shape);
+  if (plan_fingerprint(segs, shape, tile_pairs) != plan_info->fingerprint)
+    return fail(ISM_ERR_INVALID_ARG, "the plan was built for other segments or head counts");
+  Counts c = count_tiles(segs, kTile, kTile);
+  *L = plan_layout(const_cast<void*>(plan), c, info.total_tokens, tile_pairs);
+  if (plan_info->bytes < L->bytes) return fail(ISM_ERR_INVALID_ARG, "plan_info does not describe this plan");
+  return ISM_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+ism_status_t ism_attn_fwd_planned(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* plan,
+                                  const ism_attn_plan_info_t* plan_info, const void* q, const void* k,
+                                  const void* v, void* o, float* lse, ism_stream_t stream) {
+  PassLayout L;
+  ism_status_t r = planned_layout(segs, shape, plan, plan_info, &L);
+  if (r != ISM_OK) return r;
+  return fwd_impl(segs, shape, q, k, v, o, lse, nullptr, 0, stream, 1.f, 1.f, nullptr, nullptr, nullptr, &L);
+}
+
+ism_status_t ism_attn_bwd_planned(const ism_segments_t* segs, const ism_attn_shape_t* shape, void* plan,
+                                  const ism_attn_plan_info_t* plan_info, const void* q, const void* k,
+                                  const void* v, const void* o, const float* lse, const void* dout, void* dq,
+                                  void* dk, void* dv, void* workspace, size_t workspace_bytes,
+                                  ism_stream_t stream) {
+  PassLayout L;
+  ism_status_t r = planned_layout(segs, shape, plan, plan_info, &L);
+  if (r != ISM_OK) return r;
+  return bwd_impl(segs, shape, q, k, v, o, lse, dout, dq, dk, dv, workspace, workspace_bytes, stream, nullptr, &L);
 }
 
 // ---------------------------------------------------------------- append

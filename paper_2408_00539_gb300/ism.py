@@ -48,6 +48,10 @@ class _Shape(C.Structure):
                 ("dtype", C.c_int32), ("softmax_scale", C.c_float)]
 
 
+class _PlanInfo(C.Structure):
+    _fields_ = [("fingerprint", C.c_uint64), ("bytes", C.c_size_t)]
+
+
 EXPORTS = {
     "ism_tile_map_size": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p]),
     "ism_build_tile_map": (C.c_int, [C.c_void_p, C.c_int32, C.c_int32] + [C.c_void_p] * 6),
@@ -100,6 +104,10 @@ EXPORTS = {
     "ism_debug_mma_tile_e4m3": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32, C.c_void_p]),
     "ism_attn_fwd_noalloc_max_workspace": (C.c_size_t, []),
     "ism_attn_fwd_noalloc": (C.c_int, [C.c_void_p] * 8),
+    "ism_attn_plan_size": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p]),
+    "ism_attn_plan_build": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
+    "ism_attn_fwd_planned": (C.c_int, [C.c_void_p] * 10),
+    "ism_attn_bwd_planned": (C.c_int, [C.c_void_p] * 14 + [C.c_size_t, C.c_void_p]),
 }
 
 KERNEL_FWD, KERNEL_BWD_DKDV, KERNEL_BWD_DQ, KERNEL_BWD_PRE, KERNEL_DECODE, KERNEL_META, KERNEL_ROPE = 1, 2, 3, 4, 5, 6, 7
@@ -234,12 +242,49 @@ def tile_map(segs: Segments, bm: int = 128, bn: int = 128):
     return out
 
 
-def fwd(segs: Segments, q, k, v, softmax_scale: float, out=None, lse=None, workspace=None):
-    """Forward over packed dialogues.  q [T,Hq,D], k/v [T,Hkv,D] -> (o, lse [Hq,T])."""
+class Plan:
+    """The metadata of one batch of segments (ism_attn_plan_build) for the
+    forward and backward of every layer over those segments and head counts:
+    built once, passed to fwd / bwd as plan=.  Holds its device buffer."""
+
+    def __init__(self, segs: Segments, num_heads_q: int, num_heads_kv: int, head_dim: int = 128,
+                 dtype: torch.dtype = torch.bfloat16, device="cuda"):
+        lib = load()
+        self.segs = segs
+        probe = torch.empty((0, num_heads_q, head_dim), dtype=dtype)
+        self._shape = _shape(probe, torch.empty((0, num_heads_kv, head_dim), dtype=dtype), 1.0)
+        n = C.c_size_t()
+        _check(lib.ism_attn_plan_size(C.byref(segs.struct()), C.byref(self._shape), C.byref(n)), "ism_attn_plan_size")
+        self.buffer = _workspace(n.value, device)
+        self.info = _PlanInfo()
+        self.build()
+
+    def build(self):
+        """Run the metadata pass into the plan (on the current stream)."""
+        lib = load()
+        _check(lib.ism_attn_plan_build(C.byref(self.segs.struct()), C.byref(self._shape), _ptr(self.buffer),
+                                       self.buffer.numel(), C.byref(self.info), _stream(self.buffer.device)),
+               "ism_attn_plan_build")
+        return self
+
+
+def fwd(segs: Segments, q, k, v, softmax_scale: float, out=None, lse=None, workspace=None, plan: Plan = None):
+    """Forward over packed dialogues.  q [T,Hq,D], k/v [T,Hkv,D] -> (o, lse [Hq,T]).
+    With a plan of these segments the metadata pass is not run again (and no
+    workspace is needed)."""
     lib = load()
     _contig(q, k, v)
     T, hq, D = q.shape
     s, sh = segs.struct(), _shape(q, k, softmax_scale)
+    if plan is not None:
+        if out is None:
+            out = torch.empty_like(q)
+        if lse is None:
+            lse = torch.empty((hq, T), dtype=torch.float32, device=q.device)
+        _check(lib.ism_attn_fwd_planned(C.byref(s), C.byref(sh), _ptr(plan.buffer), C.byref(plan.info), _ptr(q),
+                                        _ptr(k), _ptr(v), _ptr(out), _ptr(lse), _stream(q.device)),
+               "ism_attn_fwd_planned")
+        return out, lse
     nbytes = C.c_size_t()
     _check(lib.ism_attn_fwd_workspace_size(C.byref(s), C.byref(sh), C.byref(nbytes)), "ism_attn_fwd_workspace_size")
     if out is None:
@@ -337,7 +382,7 @@ def bwd_workspace_size(segs: Segments, q, k, softmax_scale: float, minimal: bool
 
 
 def bwd(segs: Segments, q, k, v, o, lse, dout, softmax_scale: float, dq=None, dk=None, dv=None, workspace=None,
-        minimal_workspace: bool = False):
+        minimal_workspace: bool = False, plan: Plan = None):
     """Backward: (dq, dk, dv) of sum(O * dout).  The library takes the
     stored-dS schedule when the workspace is large enough for it, else the
     recompute schedule.  A given workspace is used as it is (it must hold at
@@ -362,6 +407,12 @@ def bwd(segs: Segments, q, k, v, o, lse, dout, softmax_scale: float, dq=None, dk
                 workspace = _workspace(full.value, q.device)
             except torch.cuda.OutOfMemoryError:
                 workspace = _workspace(low.value, q.device)
+    if plan is not None:  # the plan's metadata instead of a metadata pass
+        _check(lib.ism_attn_bwd_planned(C.byref(s), C.byref(sh), _ptr(plan.buffer), C.byref(plan.info), _ptr(q),
+                                        _ptr(k), _ptr(v), _ptr(o), _ptr(lse), _ptr(dout), _ptr(dq), _ptr(dk),
+                                        _ptr(dv), _ptr(workspace), workspace.numel(), _stream(q.device)),
+               "ism_attn_bwd_planned")
+        return dq, dk, dv
     _check(lib.ism_attn_bwd(C.byref(s), C.byref(sh), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), _ptr(dout),
                             _ptr(dq), _ptr(dk), _ptr(dv), _ptr(workspace), workspace.numel(), _stream(q.device)),
            "ism_attn_bwd")

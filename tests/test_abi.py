@@ -243,3 +243,36 @@ def test_e4m3_entry_errors(lib):
     need = C.c_size_t()
     assert lib.ism_attn_fwd_workspace_size(C.byref(s), C.byref(_shape(dtype=2)), C.byref(need)) == 0
     assert lib.ism_attn_fwd_workspace_size(C.byref(s), C.byref(_shape(dtype=2, d=64)), C.byref(need)) == 2
+
+
+def test_plan_size_host_only(lib):
+    """The plan's size is a host computation: the per-token key bounds, the
+    tile descriptors and work lists of both passes, growing with the tokens;
+    the same for any softmax scale."""
+    keep = _Keep()
+    sizes = []
+    for L in (100, 1000, 10000):
+        s = _segs([0, L], [0, 2], [L // 2, L], [0, 1], keep)
+        n = C.c_size_t()
+        assert lib.ism_attn_plan_size(C.byref(s), C.byref(_shape()), C.byref(n)) == 0
+        n2 = C.c_size_t()
+        assert lib.ism_attn_plan_size(C.byref(s), C.byref(_shape(scale=0.7)), C.byref(n2)) == 0
+        assert n.value == n2.value
+        sizes.append(n.value)
+    assert sizes[0] < sizes[1] < sizes[2]
+    assert sizes[2] >= 4 * 10000                                   # a key bound per token at least
+
+
+@host_only
+def test_planned_calls_need_a_plan(lib):
+    """Planned calls without a plan or its host record are refused on the
+    host before anything else."""
+    keep = _Keep()
+    s = _segs([0, 10], [0, 2], [4, 10], [0, 1], keep)
+    info = ism._PlanInfo()
+    r = lib.ism_attn_fwd_planned(C.byref(s), C.byref(_shape()), None, C.byref(info), FAKE, FAKE, FAKE, FAKE, FAKE,
+                                 None)
+    assert r == 1 and "plan" in lib.ism_last_error().decode()
+    r = lib.ism_attn_bwd_planned(C.byref(s), C.byref(_shape()), FAKE, None, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE,
+                                 FAKE, FAKE, FAKE, FAKE, 1 << 30, None)
+    assert r == 1 and "plan" in lib.ism_last_error().decode()
