@@ -564,7 +564,10 @@ cudaError_t launch_pass_meta(const SegsDev& s, int32_t* kv_end, int bm, int bn, 
   size_t a = (size_t)(s.num_seqs + 1) * (sizeof(int64_t) + 2 * sizeof(int32_t));
   size_t b = sizeof(int32_t) * (size_t)(max_cost + 1);
   size_t smem = a > b ? a : b;
-  if (smem > 48 * 1024) {
+  // opted in well below 48 KB: the kernel's static shared memory (the block
+  // scans' warp totals) and the dynamic part together must fit what a launch
+  // gets without opting in
+  if (smem > 16 * 1024) {
     cudaError_t e = cudaFuncSetAttribute(pass_meta_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
   }

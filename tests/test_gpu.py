@@ -987,15 +987,17 @@ def test_paged_and_e4m3_appends_ignore_garbage(ism):
 
 # ---------------------------------------------------------------- limits
 
-def test_max_sequences_fwd_bwd_sampled(ism):
-    """8192 sequences (the most one call takes) of 1-40 tokens with random
-    segments (empty and same-type neighbours included) in one fwd + bwd
-    call; the oracle checks every 517th sequence and the last."""
+@pytest.mark.parametrize("n_seqs", [2500, 8192])
+def test_max_sequences_fwd_bwd_sampled(ism, n_seqs):
+    """8192 sequences (the most one call takes; and 2500, whose per-sequence
+    offsets fill 40 KB of the metadata pass's shared memory) of 1-40 tokens
+    with random segments (empty and same-type neighbours included) in one
+    fwd + bwd call; the oracle checks every 517th sequence and the last."""
     rng = np.random.Generator(np.random.PCG64(81))
-    segs = wl.random_dialogue_set(rng, 8192, 40)
+    segs = wl.random_dialogue_set(rng, n_seqs, 40)
     w = wl.Workload("many_short", segs, 4, 2, 128, "bf16", 128 ** -0.5, 0.5, 82)
     (q, k, v, do), (o, lse, dq, dk, dv) = _run_pass(ism, w)
-    for b in list(range(0, 8192, 517)) + [8191]:
+    for b in list(range(0, n_seqs, 517)) + [n_seqs - 1]:
         t0, L, se, st = segs.seq(b)
         sub = wl.pack([(se, st)])
         sl = slice(t0, t0 + L)
