@@ -827,9 +827,11 @@ def measure_training_config(dev, w, peaks, steps=20, minimal_workspace=False, ro
         q_rot, k_rot = torch.empty_like(q), torch.empty_like(k)
 
         def step():  # noqa: F811
-            ism.fwd_rope(segs, q, k, v, cos_t, sin_t, w.softmax_scale, q_rot=q_rot, k_rot=k_rot, out=o, lse=lse)
+            plan.build()
+            ism.fwd_rope(segs, q, k, v, cos_t, sin_t, w.softmax_scale, q_rot=q_rot, k_rot=k_rot, out=o, lse=lse,
+                         plan=plan)
             ism.bwd_rope(segs, q_rot, k_rot, v, o, lse, do, cos_t, sin_t, w.softmax_scale, dq=dq, dk=dk, dv=dv,
-                         workspace=ws)
+                         workspace=ws, plan=plan)
 
     with ClockSampler(dev.index) as clocks:
         for _ in range(3):

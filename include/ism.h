@@ -278,6 +278,8 @@ ism_status_t ism_attn_bwd_rope(const ism_segments_t* segs, const ism_attn_shape_
  *   the backward takes a workspace as ism_attn_bwd does
  *   (ism_attn_bwd_workspace_size for the stored-dS schedule, _min for the
  *   recompute schedule: both cover what the planned call uses).
+ * ism_attn_fwd_rope_planned / ism_attn_bwd_rope_planned: the same for
+ *   ism_attn_fwd_rope / ism_attn_bwd_rope (arguments as there).
  * The plan must stay unchanged while a call that uses it may run, and calls
  * that share a plan run in stream order (the backward resets a work counter
  * held in the plan).  No counterpart in the paper.
@@ -298,6 +300,15 @@ ism_status_t ism_attn_bwd_planned(const ism_segments_t* segs, const ism_attn_sha
                                   const void* v, const void* o, const float* lse, const void* dout, void* dq,
                                   void* dk, void* dv, void* workspace, size_t workspace_bytes,
                                   ism_stream_t stream);
+ism_status_t ism_attn_fwd_rope_planned(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* plan,
+                                       const ism_attn_plan_info_t* plan_info, const void* q, const void* k,
+                                       const void* v, const ism_rope_t* rope, void* q_rot, void* k_rot, void* o,
+                                       float* lse, ism_stream_t stream);
+ism_status_t ism_attn_bwd_rope_planned(const ism_segments_t* segs, const ism_attn_shape_t* shape, void* plan,
+                                       const ism_attn_plan_info_t* plan_info, const void* q_rot, const void* k_rot,
+                                       const void* v, const void* o, const float* lse, const void* dout,
+                                       const ism_rope_t* rope, void* dq, void* dk, void* dv, void* workspace,
+                                       size_t workspace_bytes, ism_stream_t stream);
 
 /* ---------------------------------------------------------------------------
  * Append-prefill of a new turn against a reused KV cache (Section 2.3: the

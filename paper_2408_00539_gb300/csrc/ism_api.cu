@@ -790,6 +790,30 @@ ism_status_t ism_attn_bwd_planned(const ism_segments_t* segs, const ism_attn_sha
   return bwd_impl(segs, shape, q, k, v, o, lse, dout, dq, dk, dv, workspace, workspace_bytes, stream, nullptr, &L);
 }
 
+ism_status_t ism_attn_fwd_rope_planned(const ism_segments_t* segs, const ism_attn_shape_t* shape, const void* plan,
+                                       const ism_attn_plan_info_t* plan_info, const void* q, const void* k,
+                                       const void* v, const ism_rope_t* rope, void* q_rot, void* k_rot, void* o,
+                                       float* lse, ism_stream_t stream) {
+  if (!rope) return fail(ISM_ERR_INVALID_ARG, "rope is NULL");
+  PassLayout L;
+  ism_status_t r = planned_layout(segs, shape, plan, plan_info, &L);
+  if (r != ISM_OK) return r;
+  return fwd_impl(segs, shape, q, k, v, o, lse, nullptr, 0, stream, 1.f, 1.f, rope, q_rot, k_rot, &L);
+}
+
+ism_status_t ism_attn_bwd_rope_planned(const ism_segments_t* segs, const ism_attn_shape_t* shape, void* plan,
+                                       const ism_attn_plan_info_t* plan_info, const void* q_rot, const void* k_rot,
+                                       const void* v, const void* o, const float* lse, const void* dout,
+                                       const ism_rope_t* rope, void* dq, void* dk, void* dv, void* workspace,
+                                       size_t workspace_bytes, ism_stream_t stream) {
+  if (!rope) return fail(ISM_ERR_INVALID_ARG, "rope is NULL");
+  PassLayout L;
+  ism_status_t r = planned_layout(segs, shape, plan, plan_info, &L);
+  if (r != ISM_OK) return r;
+  return bwd_impl(segs, shape, q_rot, k_rot, v, o, lse, dout, dq, dk, dv, workspace, workspace_bytes, stream, rope,
+                  &L);
+}
+
 // ---------------------------------------------------------------- append
 
 namespace {

@@ -108,6 +108,8 @@ EXPORTS = {
     "ism_attn_plan_build": (C.c_int, [C.c_void_p, C.c_void_p, C.c_void_p, C.c_size_t, C.c_void_p, C.c_void_p]),
     "ism_attn_fwd_planned": (C.c_int, [C.c_void_p] * 10),
     "ism_attn_bwd_planned": (C.c_int, [C.c_void_p] * 14 + [C.c_size_t, C.c_void_p]),
+    "ism_attn_fwd_rope_planned": (C.c_int, [C.c_void_p] * 13),
+    "ism_attn_bwd_rope_planned": (C.c_int, [C.c_void_p] * 15 + [C.c_size_t, C.c_void_p]),
 }
 
 KERNEL_FWD, KERNEL_BWD_DKDV, KERNEL_BWD_DQ, KERNEL_BWD_PRE, KERNEL_DECODE, KERNEL_META, KERNEL_ROPE = 1, 2, 3, 4, 5, 6, 7
@@ -322,7 +324,7 @@ def fwd_e4m3(segs: Segments, q, k, v, q_descale: float, k_descale: float, v_desc
 
 
 def fwd_rope(segs: Segments, q, k, v, rope_cos, rope_sin, softmax_scale: float, q_rot=None, k_rot=None, out=None,
-             lse=None, workspace=None):
+             lse=None, workspace=None, plan: "Plan" = None):
     """Forward with rotary encoding: q [T,Hq,D] and k [T,Hkv,D] (unrotated)
     are rotated at their positions inside their sequences (tables rope_cos /
     rope_sin float32 [rows, D/2]) into q_rot / k_rot, then attended.
@@ -338,6 +340,11 @@ def fwd_rope(segs: Segments, q, k, v, rope_cos, rope_sin, softmax_scale: float, 
     k_rot = torch.empty_like(k) if k_rot is None else k_rot
     out = torch.empty_like(q) if out is None else out
     lse = torch.empty((hq, T), dtype=torch.float32, device=q.device) if lse is None else lse
+    if plan is not None:  # the plan's metadata instead of a metadata pass
+        _check(lib.ism_attn_fwd_rope_planned(C.byref(s), C.byref(sh), _ptr(plan.buffer), C.byref(plan.info),
+                                             _ptr(q), _ptr(k), _ptr(v), C.byref(rope), _ptr(q_rot), _ptr(k_rot),
+                                             _ptr(out), _ptr(lse), _stream(q.device)), "ism_attn_fwd_rope_planned")
+        return out, lse, q_rot, k_rot
     if workspace is None or workspace.numel() < nbytes.value:
         workspace = _workspace(nbytes.value, q.device)
     _check(lib.ism_attn_fwd_rope(C.byref(s), C.byref(sh), _ptr(q), _ptr(k), _ptr(v), C.byref(rope), _ptr(q_rot),
@@ -347,7 +354,7 @@ def fwd_rope(segs: Segments, q, k, v, rope_cos, rope_sin, softmax_scale: float, 
 
 
 def bwd_rope(segs: Segments, q_rot, k_rot, v, o, lse, dout, rope_cos, rope_sin, softmax_scale: float, dq=None,
-             dk=None, dv=None, workspace=None, minimal_workspace: bool = False):
+             dk=None, dv=None, workspace=None, minimal_workspace: bool = False, plan: "Plan" = None):
     """Backward of ``fwd_rope``: takes the rotated q_rot / k_rot the forward
     wrote and returns (dq, dk, dv) with dq, dk the gradients of the UNROTATED
     queries and keys.  Workspace as for ``bwd``."""
@@ -364,6 +371,12 @@ def bwd_rope(segs: Segments, q_rot, k_rot, v, o, lse, dout, rope_cos, rope_sin, 
     dv = torch.empty_like(v) if dv is None else dv
     if workspace is None or workspace.numel() < low.value:
         workspace = _workspace(low.value if minimal_workspace else full.value, q_rot.device)
+    if plan is not None:  # the plan's metadata instead of a metadata pass
+        _check(lib.ism_attn_bwd_rope_planned(C.byref(s), C.byref(sh), _ptr(plan.buffer), C.byref(plan.info),
+                                             _ptr(q_rot), _ptr(k_rot), _ptr(v), _ptr(o), _ptr(lse), _ptr(dout),
+                                             C.byref(rope), _ptr(dq), _ptr(dk), _ptr(dv), _ptr(workspace),
+                                             workspace.numel(), _stream(q_rot.device)), "ism_attn_bwd_rope_planned")
+        return dq, dk, dv
     _check(lib.ism_attn_bwd_rope(C.byref(s), C.byref(sh), _ptr(q_rot), _ptr(k_rot), _ptr(v), _ptr(o), _ptr(lse),
                                  _ptr(dout), C.byref(rope), _ptr(dq), _ptr(dk), _ptr(dv), _ptr(workspace),
                                  workspace.numel(), _stream(q_rot.device)), "ism_attn_bwd_rope")

@@ -106,3 +106,23 @@ def test_plan_for_other_segments_or_heads_rejected(ism):
     assert e.value.code == 1
     assert ism.kernel_launches() == launches
     ism.check_status()
+
+
+@pytest.mark.parametrize("hq,hkv", [(8, 2), (4, 4)])
+def test_planned_rope_calls_equal_one_pass_calls(ism, hq, hkv):
+    """The rotary forward and backward on a plan: rotated rows, O, LSE, dQ,
+    dK, dV identical to the one-pass rotary calls."""
+    w = wl.Workload("plan_rope", _segs(), hq, hkv, 128, "bf16", 128 ** -0.5, 0.5, 91 + hq)
+    q, k, v, do = (t.to(DEV) for t in wl.attention_tensors(w))
+    segs = ism.Segments.from_workload(w.segs, DEV)
+    cos_np, sin_np = wl.rope_tables(int(np.diff(w.segs.cu_seqlens).max()), 128)
+    cos_t, sin_t = torch.from_numpy(cos_np).to(DEV), torch.from_numpy(sin_np).to(DEV)
+    plan = _plan(ism, segs, w, q)
+    o, lse, qr, kr = ism.fwd_rope(segs, q, k, v, cos_t, sin_t, w.softmax_scale)
+    ref = (o, lse, qr, kr) + ism.bwd_rope(segs, qr, kr, v, o, lse, do, cos_t, sin_t, w.softmax_scale)
+    o2, lse2, qr2, kr2 = ism.fwd_rope(segs, q, k, v, cos_t, sin_t, w.softmax_scale, plan=plan)
+    got = (o2, lse2, qr2, kr2) + ism.bwd_rope(segs, qr2, kr2, v, o2, lse2, do, cos_t, sin_t, w.softmax_scale,
+                                              plan=plan)
+    ism.check_status()
+    for name, a, b in zip(("o", "lse", "q_rot", "k_rot", "dq", "dk", "dv"), ref, got):
+        assert torch.equal(a, b), name
